@@ -1,0 +1,290 @@
+"""Plain CPU oracle of the Lodestar routing hot path -- test infrastructure.
+
+Only the test suite, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
+``bench.py`` may import this package.  The CUDA library never does, and this
+package imports nothing from it.
+
+The arithmetic lives in ``lodestar_oracle.c`` (scalar loops, fp64
+accumulation); this module compiles it with gcc on first use and wraps each
+function for numpy arrays.  Paper sections each function follows are cited in
+the C source.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "lodestar_oracle.c")
+_OUT = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_OUT, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+F64, F32, BF16 = 0, 1, 2
+SGD, ADAM = 0, 1
+BLOCK = 16
+MODES = {"f64": F64, "f32": F32, "bf16": BF16}
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle (gcc, no FMA contraction, no fast-math)."""
+    os.makedirs(_OUT, exist_ok=True)
+    if (not force and os.path.exists(_LIB_PATH)
+            and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
+        return _LIB_PATH
+    tmp = _LIB_PATH + f".tmp{os.getpid()}"
+    cmd = ["gcc", "-std=c11", "-O2", "-fPIC", "-shared", "-ffp-contract=off",
+           "-fno-fast-math", "-o", tmp, _SRC, "-lm"]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def lib():
+    global _lib
+    with _lock:
+        if _lib is None:
+            L = C.CDLL(build())
+            P = C.c_void_p
+            i64, i32, dbl = C.c_int64, C.c_int32, C.c_double
+            L.or_mix64.restype = C.c_uint64
+            L.or_mix64.argtypes = [C.c_uint64]
+            L.or_block_content.restype = C.c_uint64
+            L.or_block_content.argtypes = [P]
+            L.or_hash_blocks.argtypes = [i64, P, P, P, P]
+            L.or_prefix_hits.argtypes = [i64, P, P, i32, P, P, P]
+            L.or_prefix_hits_by_marking.argtypes = [i64, P, P, i32, P, P, P]
+            L.or_raw_features_row.argtypes = [i64, i32, P, C.c_int, P, C.c_int, P]
+            L.or_raw_features_row.restype = None
+            L.or_features.argtypes = [i64, i32, P, P, P, C.c_int, P, C.c_int, P, P, P]
+            L.or_bf16.restype = C.c_float
+            L.or_bf16.argtypes = [C.c_float]
+            L.or_param_count.restype = i64
+            L.or_param_count.argtypes = [C.c_int, P]
+            L.or_mlp_forward.argtypes = [C.c_int, C.c_int, P, P, i64, P, P]
+            L.or_argmin.argtypes = [i64, i32, P, P, P]
+            L.or_ring_append.argtypes = [i64, C.c_int, P, P, i64, i64, P, P]
+            L.or_train_step.argtypes = [C.c_int, C.c_int, P, P, P, P, i64, C.c_int, dbl,
+                                        C.c_int, P, P, P, P, P, P, P]
+            L.or_loss.argtypes = [C.c_int, C.c_int, P, P, C.c_int, P, P, P, P, P, P]
+            _lib = L
+    return _lib
+
+
+def _p(a: np.ndarray):
+    return a.ctypes.data_as(C.c_void_p)
+
+
+def _c(a, dtype):
+    return np.ascontiguousarray(a, dtype=dtype)
+
+
+def _check(rc, what):
+    if rc != 0:
+        raise RuntimeError(f"oracle {what} failed ({rc})")
+
+
+# --------------------------------------------------------------------------
+# hashing and prefix hits
+# --------------------------------------------------------------------------
+
+def mix64(z: int) -> int:
+    return int(lib().or_mix64(C.c_uint64(z & (2**64 - 1))))
+
+
+def block_content(tokens16) -> int:
+    t = _c(tokens16, np.int32)
+    assert t.size == BLOCK
+    return int(lib().or_block_content(_p(t)))
+
+
+def key_offsets(tok_off) -> np.ndarray:
+    """CSR offsets of block keys: floor(L/16) keys per sequence."""
+    L = np.diff(np.asarray(tok_off, np.int64))
+    off = np.zeros(len(L) + 1, np.int64)
+    off[1:] = np.cumsum(L // BLOCK)
+    return off
+
+
+def hash_blocks(tok, tok_off):
+    """Returns (keys uint64 [sum floor(L/16)], key_off int64 [n+1])."""
+    tok = _c(tok, np.int32)
+    tok_off = _c(tok_off, np.int64)
+    koff = key_offsets(tok_off)
+    keys = np.zeros(max(int(koff[-1]), 1), np.uint64)
+    _check(lib().or_hash_blocks(len(tok_off) - 1, _p(tok), _p(tok_off), _p(keys), _p(koff)), "hash")
+    return keys[: koff[-1]], koff
+
+
+def prefix_hits(req_keys, req_key_off, inst_keys, inst_key_off, by_marking: bool = False):
+    rk = _c(req_keys, np.uint64) if len(req_keys) else np.zeros(1, np.uint64)
+    rko = _c(req_key_off, np.int64)
+    ik = _c(inst_keys, np.uint64) if len(inst_keys) else np.zeros(1, np.uint64)
+    iko = _c(inst_key_off, np.int64)
+    R, N = len(rko) - 1, len(iko) - 1
+    hits = np.zeros((R, N), np.int32)
+    fn = lib().or_prefix_hits_by_marking if by_marking else lib().or_prefix_hits
+    _check(fn(R, _p(rk), _p(rko), N, _p(ik), _p(iko), _p(hits)), "prefix_hits")
+    return hits
+
+
+def instance_keys(wl, seq_keys=None, seq_key_off=None):
+    """Key multiset of every instance of a workload: the oracle's own hash of
+    the cached chains (first k blocks of a cached sequence) plus the
+    workload's random stand-in keys.  Returns (keys, off) CSR."""
+    if seq_keys is None:
+        seq_keys, seq_key_off = hash_blocks(wl.seq_tok, wl.seq_off)
+    parts, off = [], [0]
+    N = len(wl.inst_chain_off) - 1
+    for i in range(N):
+        ks = []
+        for c in range(int(wl.inst_chain_off[i]), int(wl.inst_chain_off[i + 1])):
+            s, k = int(wl.chain_seq[c]), int(wl.chain_blocks[c])
+            ks.append(seq_keys[seq_key_off[s]: seq_key_off[s] + k])
+        ks.append(wl.rand_keys[wl.inst_rand_off[i]: wl.inst_rand_off[i + 1]])
+        kk = np.concatenate(ks) if ks else np.zeros(0, np.uint64)
+        parts.append(kk)
+        off.append(off[-1] + len(kk))
+    return (np.concatenate(parts).astype(np.uint64) if parts else np.zeros(0, np.uint64),
+            np.asarray(off, np.int64))
+
+
+# --------------------------------------------------------------------------
+# features, predictor, selection
+# --------------------------------------------------------------------------
+
+def raw_features_row(L: int, h: int, inst, req) -> np.ndarray:
+    """Raw (un-normalised) feature row of one (request, instance) pair."""
+    inst = _c(inst, np.float32).ravel()
+    req = _c(req, np.float32).ravel()
+    x = np.zeros(6 + inst.size + req.size, np.float32)
+    one = np.zeros(1, np.float32)
+    lib().or_raw_features_row(int(L), int(h), _p(inst if inst.size else one), inst.size,
+                              _p(req if req.size else one), req.size, _p(x))
+    return x
+
+
+def features(L, hits, inst_state, req_feats, mean, std):
+    """Normalised features [R*N, d] (row r*N + i)."""
+    L = _c(L, np.int64)
+    hits = _c(hits, np.int32)
+    inst = _c(inst_state, np.float32)
+    req = _c(req_feats, np.float32)
+    R, N = hits.shape
+    d_inst, d_req = inst.shape[1], (req.shape[1] if req.ndim == 2 else 0)
+    d = 6 + d_inst + d_req
+    out = np.zeros((R * N, d), np.float32)
+    reqp = req if req.size else np.zeros(1, np.float32)
+    _check(lib().or_features(R, N, _p(L), _p(hits), _p(inst), d_inst, _p(reqp), d_req,
+                             _p(_c(mean, np.float32)), _p(_c(std, np.float32)), _p(out)),
+           "features")
+    return out
+
+
+def bf16(x) -> np.ndarray:
+    f = np.vectorize(lambda v: lib().or_bf16(float(v)), otypes=[np.float32])
+    return f(np.asarray(x, np.float32))
+
+
+def param_count(widths) -> int:
+    w = _c(widths, np.int32)
+    return int(lib().or_param_count(len(w) - 1, _p(w)))
+
+
+def mlp_forward(mode, widths, params, x) -> np.ndarray:
+    mode = MODES.get(mode, mode)
+    w = _c(widths, np.int32)
+    p = _c(params, np.float64)
+    x = _c(x, np.float64).reshape(-1, w[0])
+    y = np.zeros(x.shape[0], np.float64)
+    _check(lib().or_mlp_forward(mode, len(w) - 1, _p(w), _p(p), x.shape[0], _p(x), _p(y)), "mlp")
+    return y
+
+
+def argmin(scores):
+    s = _c(scores, np.float32)
+    R, N = s.shape
+    choice = np.zeros(R, np.int32)
+    best = np.zeros(R, np.float32)
+    _check(lib().or_argmin(R, N, _p(s), _p(choice), _p(best)), "argmin")
+    return choice, best
+
+
+def route(wl, hits=None, inst_keys=None, params=None, mode=None, req_idx=None):
+    """Full oracle route of (a subset of) a workload's requests.
+    Returns dict(hits, scores, choice, best)."""
+    cfg = wl.cfg
+    mode = mode or cfg.dtype
+    R_all = len(wl.tok_off) - 1
+    idx = np.arange(R_all) if req_idx is None else np.asarray(req_idx)
+    if hits is None:
+        tok_off = wl.tok_off
+        seqs = [wl.tok[tok_off[r]: tok_off[r + 1]] for r in idx]
+        sub_off = np.zeros(len(idx) + 1, np.int64)
+        sub_off[1:] = np.cumsum([len(s) for s in seqs])
+        sub_tok = np.concatenate(seqs) if seqs else np.zeros(0, np.int32)
+        rk, rko = hash_blocks(sub_tok, sub_off)
+        if inst_keys is None:
+            inst_keys = instance_keys(wl)
+        ik, iko = inst_keys
+        hits = prefix_hits(rk, rko, ik, iko, by_marking=len(idx) * 64 < len(ik))
+    L = np.diff(wl.tok_off)[idx]
+    x = features(L, hits, wl.inst_state, wl.req_feats[idx], wl.mean, wl.std)
+    y = mlp_forward(mode, cfg.widths, wl.params if params is None else params, x)
+    scores = y.astype(np.float32).reshape(len(idx), -1)
+    choice, best = argmin(scores)
+    return dict(hits=hits, scores=scores, choice=choice, best=best)
+
+
+# --------------------------------------------------------------------------
+# sample ring and training
+# --------------------------------------------------------------------------
+
+def ring_append(ring_x, ring_y, count, x, y):
+    C_, d = ring_x.shape
+    x = _c(x, np.float32)
+    y = _c(y, np.float32)
+    _check(lib().or_ring_append(C_, d, _p(ring_x), _p(ring_y), int(count), len(y), _p(x), _p(y)), "ring")
+    return count + len(y)
+
+
+class Trainer:
+    """Oracle optimiser state: fp32-valued params, Adam moments, step count."""
+
+    def __init__(self, widths, params, mode="f32"):
+        self.w = _c(widths, np.int32)
+        self.mode = MODES.get(mode, mode)
+        self.params = _c(params, np.float64).copy()
+        self.m = np.zeros_like(self.params)
+        self.v = np.zeros_like(self.params)
+        self.t = 0
+
+    def step(self, ring_x, ring_y, idx, mean, std, opt="adam", lr=3e-4, want_grad=False):
+        self.t += 1
+        loss = np.zeros(1, np.float64)
+        g = np.zeros_like(self.params) if want_grad else None
+        idx = _c(idx, np.int32)
+        rc = lib().or_train_step(self.mode, len(self.w) - 1, _p(self.w), _p(self.params),
+                                 _p(self.m), _p(self.v), self.t, ADAM if opt == "adam" else SGD,
+                                 float(lr), len(idx), _p(_c(ring_x, np.float32)),
+                                 _p(_c(ring_y, np.float32)), _p(idx), _p(_c(mean, np.float32)),
+                                 _p(_c(std, np.float32)), _p(loss),
+                                 _p(g) if g is not None else None)
+        _check(rc, "train_step")
+        return (float(loss[0]), g) if want_grad else float(loss[0])
+
+
+def loss(mode, widths, params, ring_x, ring_y, idx, mean, std) -> float:
+    w = _c(widths, np.int32)
+    out = np.zeros(1, np.float64)
+    idx = _c(idx, np.int32)
+    _check(lib().or_loss(MODES.get(mode, mode), len(w) - 1, _p(w), _p(_c(params, np.float64)),
+                         len(idx), _p(_c(ring_x, np.float32)), _p(_c(ring_y, np.float32)),
+                         _p(idx), _p(_c(mean, np.float32)), _p(_c(std, np.float32)), _p(out)),
+           "loss")
+    return float(out[0])

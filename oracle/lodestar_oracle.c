@@ -1,0 +1,479 @@
+/*
+ * Lodestar routing hot path -- plain CPU oracle (test infrastructure only).
+ *
+ * This file is the checker for the CUDA path, not part of it.  Only the test
+ * suite, the smoke check and the CPU-baseline leg of the benchmark load it.
+ * It shares no code, header or table with the CUDA library.
+ *
+ * Everything here is written for obviousness, not speed: scalar loops, fp64
+ * accumulation, qsort + bsearch for set membership, no blocking or fusion.
+ *
+ * Paper: "Lodestar" (online-learned LLM inference router).
+ *   Sec. 2 (LLM inference serving): prefix reuse is strictly sequential -- a
+ *          cached block helps only if all preceding blocks are cached.
+ *   Sec. 2 (Gateway infrastructure): the gateway keeps a prefix index (radix
+ *          tree or hash tables) and computes each instance's prefix-match ratio.
+ *   Sec. 4.1 (Request-instance reward model): one shared f_theta scores each
+ *          instance from [x_i || r]; route to argmax reward = argmin TTFT.
+ *   Sec. 4.1 (Model architecture): MLP, ReLU, scalar output.
+ *   Sec. 4.1 (Features): input length, expected KV-hit ratio, running / queued
+ *          requests, inflight prefill / decode tokens, KV utilisation, GPU model.
+ *   Algorithm 4: per-feature z-score normalisation, batched forward, argmax.
+ *   Sec. 4.3.2 (Online learning): periodic retraining on logged
+ *          (features, TTFT) records; FIFO buffer of recent samples.
+ *
+ * Readings where the paper is silent (each also listed in the design notes):
+ *   - block hash: SplitMix64 finaliser based content hash, prefix state chained
+ *     by a linear recurrence mod 2^64 (definition below);
+ *   - hit length: stop at the first missing block, no cap at L-1;
+ *   - kappa = 16h/L with kappa = 0 when L = 0; std < 1e-12 replaced by 1;
+ *   - loss: mean squared error on TTFT in seconds; SGD or Adam (PyTorch
+ *     defaults beta1 = 0.9, beta2 = 0.999, eps = 1e-8);
+ *   - bf16 mode: weights, layer-1 input and hidden activations rounded to
+ *     bf16 (round to nearest even); biases and accumulation stay wide;
+ *   - argmin ties -> lowest index, -0 == +0, NaN after every number.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define OR_BLOCK 16
+#define OR_G 0x9E3779B97F4A7C15ull /* floor(2^64 / golden ratio) */
+
+enum { OR_F64 = 0, OR_F32 = 1, OR_BF16 = 2 };
+enum { OR_SGD = 0, OR_ADAM = 1 };
+
+/* ------------------------------------------------------------------------ */
+/* block hash                                                               */
+/* ------------------------------------------------------------------------ */
+
+/* SplitMix64 output finaliser (Steele, Lea & Flood, OOPSLA 2014; Stafford's
+ * "variant 13" mixer): xor-shift 30, multiply, xor-shift 27, multiply,
+ * xor-shift 31. */
+uint64_t or_mix64(uint64_t z) {
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+}
+
+/* Content hash of one 16-token block: the 16 int32 tokens form 8 little-endian
+ * 64-bit words w_j (token 2j in the low half), each word is mixed with its own
+ * offset (j+1)*G, the 8 results are xor-ed and mixed once more. */
+uint64_t or_block_content(const int32_t *t) {
+    uint64_t acc = 0;
+    for (int j = 0; j < 8; ++j) {
+        uint64_t lo = (uint64_t)(uint32_t)t[2 * j];
+        uint64_t hi = (uint64_t)(uint32_t)t[2 * j + 1];
+        uint64_t w = lo | (hi << 32);
+        acc ^= or_mix64(w + (uint64_t)(j + 1) * OR_G);
+    }
+    return or_mix64(acc);
+}
+
+/* Keys of the full blocks of each sequence.  Prefix state s_{-1} = G,
+ * s_b = s_{b-1} * G + c_b (mod 2^64), key_b = mix64(s_b), with 0 mapped to 1
+ * (0 marks an empty table slot).  key_b therefore depends on all tokens of
+ * blocks 0..b, in order.  A trailing partial block gets no key.
+ * keys for sequence s go to keys[key_off[s] .. key_off[s] + floor(L_s/16)). */
+int or_hash_blocks(int64_t n_seq, const int32_t *tok, const int64_t *tok_off,
+                   uint64_t *keys, const int64_t *key_off) {
+    for (int64_t s = 0; s < n_seq; ++s) {
+        int64_t L = tok_off[s + 1] - tok_off[s];
+        if (L < 0) return -1;
+        int64_t nb = L / OR_BLOCK;
+        const int32_t *t = tok + tok_off[s];
+        uint64_t state = OR_G;
+        for (int64_t b = 0; b < nb; ++b) {
+            state = state * OR_G + or_block_content(t + b * OR_BLOCK);
+            uint64_t k = or_mix64(state);
+            keys[key_off[s] + b] = k ? k : 1ull;
+        }
+    }
+    return 0;
+}
+
+/* ------------------------------------------------------------------------ */
+/* prefix hit length                                                        */
+/* ------------------------------------------------------------------------ */
+
+static int cmp_u64(const void *a, const void *b) {
+    uint64_t x = *(const uint64_t *)a, y = *(const uint64_t *)b;
+    return (x > y) - (x < y);
+}
+
+static int contains(const uint64_t *sorted, int64_t n, uint64_t k) {
+    return bsearch(&k, sorted, (size_t)n, sizeof(uint64_t), cmp_u64) != NULL;
+}
+
+/* h[r, i] = largest k <= n_r such that keys of blocks 0..k-1 of request r are
+ * all in instance i's key set (scan stops at the first missing block).
+ * Instance key sets are CSR lists (duplicates allowed). */
+int or_prefix_hits(int64_t n_req, const uint64_t *req_keys, const int64_t *req_key_off,
+                   int32_t n_inst, const uint64_t *inst_keys, const int64_t *inst_key_off,
+                   int32_t *hits) {
+    for (int32_t i = 0; i < n_inst; ++i) {
+        int64_t n = inst_key_off[i + 1] - inst_key_off[i];
+        uint64_t *set = (uint64_t *)malloc((size_t)(n > 0 ? n : 1) * sizeof(uint64_t));
+        if (!set) return -1;
+        memcpy(set, inst_keys + inst_key_off[i], (size_t)n * sizeof(uint64_t));
+        qsort(set, (size_t)n, sizeof(uint64_t), cmp_u64);
+        for (int64_t r = 0; r < n_req; ++r) {
+            int64_t nb = req_key_off[r + 1] - req_key_off[r];
+            int64_t b = 0;
+            while (b < nb && contains(set, n, req_keys[req_key_off[r] + b])) ++b;
+            hits[r * n_inst + i] = (int32_t)b;
+        }
+        free(set);
+    }
+    return 0;
+}
+
+/* Same result, organised for few requests against huge instance sets: the
+ * request keys are sorted once and every instance key is looked up among
+ * them, marking (request block, instance) pairs that are cached. */
+typedef struct { uint64_t key; int64_t pos; } or_kp;
+static int cmp_kp(const void *a, const void *b) {
+    uint64_t x = ((const or_kp *)a)->key, y = ((const or_kp *)b)->key;
+    return (x > y) - (x < y);
+}
+
+int or_prefix_hits_by_marking(int64_t n_req, const uint64_t *req_keys, const int64_t *req_key_off,
+                              int32_t n_inst, const uint64_t *inst_keys, const int64_t *inst_key_off,
+                              int32_t *hits) {
+    int64_t nk = req_key_off[n_req];
+    or_kp *kp = (or_kp *)malloc((size_t)(nk > 0 ? nk : 1) * sizeof(or_kp));
+    unsigned char *mark = (unsigned char *)malloc((size_t)(nk > 0 ? nk : 1));
+    if (!kp || !mark) { free(kp); free(mark); return -1; }
+    for (int64_t p = 0; p < nk; ++p) { kp[p].key = req_keys[p]; kp[p].pos = p; }
+    qsort(kp, (size_t)nk, sizeof(or_kp), cmp_kp);
+    for (int32_t i = 0; i < n_inst; ++i) {
+        memset(mark, 0, (size_t)(nk > 0 ? nk : 1));
+        for (int64_t q = inst_key_off[i]; q < inst_key_off[i + 1]; ++q) {
+            /* binary search for the first entry with key >= inst key */
+            uint64_t k = inst_keys[q];
+            int64_t lo = 0, hi = nk;
+            while (lo < hi) {
+                int64_t mid = lo + (hi - lo) / 2;
+                if (kp[mid].key < k) lo = mid + 1; else hi = mid;
+            }
+            for (int64_t p = lo; p < nk && kp[p].key == k; ++p) mark[kp[p].pos] = 1;
+        }
+        for (int64_t r = 0; r < n_req; ++r) {
+            int64_t nb = req_key_off[r + 1] - req_key_off[r];
+            int64_t b = 0;
+            while (b < nb && mark[req_key_off[r] + b]) ++b;
+            hits[r * n_inst + i] = (int32_t)b;
+        }
+    }
+    free(kp);
+    free(mark);
+    return 0;
+}
+
+/* ------------------------------------------------------------------------ */
+/* features (Sec. 4.1 "Features"; Algorithm 4 Normalize)                    */
+/* ------------------------------------------------------------------------ */
+
+/* Raw feature row of pair (r, i): [pair(6) || instance state || request extras].
+ * Pair block, all in fp32:
+ *   f0 = L, f1 = h, f2 = 16h (hit tokens), f3 = kappa = 16h / L (hit ratio),
+ *   f4 = L - 16h (tokens to prefill), f5 = ceil(L/16) - h (blocks to allocate). */
+void or_raw_features_row(int64_t L, int32_t h, const float *inst, int d_inst,
+                         const float *req, int d_req, float *x) {
+    float hit_tok = (float)((int64_t)OR_BLOCK * h);
+    x[0] = (float)L;
+    x[1] = (float)h;
+    x[2] = hit_tok;
+    x[3] = L > 0 ? hit_tok / (float)L : 0.0f;
+    x[4] = (float)(L - (int64_t)OR_BLOCK * h);
+    x[5] = (float)((L + OR_BLOCK - 1) / OR_BLOCK - h);
+    for (int k = 0; k < d_inst; ++k) x[6 + k] = inst[k];
+    for (int k = 0; k < d_req; ++k) x[6 + d_inst + k] = req[k];
+}
+
+/* Per-feature z-score in fp32: (x - mean) / std, std < 1e-12 replaced by 1. */
+void or_zscore(int d, const float *x, const float *mean, const float *std, float *out) {
+    for (int k = 0; k < d; ++k) {
+        float s = std[k] < 1e-12f ? 1.0f : std[k];
+        float c = x[k] - mean[k];
+        out[k] = c / s;
+    }
+}
+
+/* Normalised features of all (r, i) pairs, row r*n_inst + i. */
+int or_features(int64_t n_req, int32_t n_inst, const int64_t *L, const int32_t *hits,
+                const float *inst, int d_inst, const float *req, int d_req,
+                const float *mean, const float *std, float *out) {
+    int d = 6 + d_inst + d_req;
+    float *x = (float *)malloc((size_t)d * sizeof(float));
+    if (!x) return -1;
+    for (int64_t r = 0; r < n_req; ++r)
+        for (int32_t i = 0; i < n_inst; ++i) {
+            or_raw_features_row(L[r], hits[r * n_inst + i], inst + (int64_t)i * d_inst, d_inst,
+                                req + r * d_req, d_req, x);
+            or_zscore(d, x, mean, std, out + (r * n_inst + i) * d);
+        }
+    free(x);
+    return 0;
+}
+
+/* ------------------------------------------------------------------------ */
+/* predictor (Sec. 4.1 "Model architecture")                                */
+/* ------------------------------------------------------------------------ */
+
+/* bf16 round-to-nearest-even of an fp32 value (NaN kept as a quiet NaN). */
+float or_bf16(float f) {
+    uint32_t u;
+    memcpy(&u, &f, 4);
+    if ((u & 0x7F800000u) == 0x7F800000u && (u & 0x007FFFFFu)) {
+        u = (u | 0x00400000u) & 0xFFFF0000u;
+    } else {
+        u += 0x7FFFu + ((u >> 16) & 1u);
+        u &= 0xFFFF0000u;
+    }
+    float r;
+    memcpy(&r, &u, 4);
+    return r;
+}
+
+/* value as stored at a rounding point of the given mode */
+static double rnd(int mode, double v) {
+    if (mode == OR_F64) return v;
+    return (double)(float)v;
+}
+static double rnd_op(int mode, double v) { /* operand of a product */
+    if (mode == OR_BF16) return (double)or_bf16((float)v);
+    return rnd(mode, v);
+}
+
+/* parameter offsets: W_l [w[l+1], w[l]] row-major then b_l [w[l+1]] */
+static int64_t param_offset(int n_layers, const int *w, int l, int bias) {
+    int64_t off = 0;
+    (void)n_layers;
+    for (int k = 0; k < l; ++k) off += (int64_t)w[k + 1] * w[k] + w[k + 1];
+    return bias ? off + (int64_t)w[l + 1] * w[l] : off;
+}
+
+int64_t or_param_count(int n_layers, const int *w) {
+    return param_offset(n_layers, w, n_layers, 0);
+}
+
+/* Forward pass of one row.  z_l = W_l a_{l-1} + b_l summed in fp64; a_l = relu(z_l)
+ * for hidden layers; the last layer is linear.  Rounding per mode:
+ *   F64 : none;  F32 : each z_l rounded to fp32;
+ *   BF16: additionally W_l, a_0 = x and every hidden a_l rounded to bf16.
+ * If z_save / a_save are given, z_l and a_l of every layer are stored at
+ * offsets act_off[l] (the input a_0 at a_save + 0). */
+static double forward_row(int mode, int n_layers, const int *w, const double *params,
+                          const double *x, double *z_save, double *a_save, const int64_t *act_off,
+                          double *buf_a, double *buf_b) {
+    double *a = buf_a, *z = buf_b;
+    for (int k = 0; k < w[0]; ++k) a[k] = rnd_op(mode, x[k]);
+    if (a_save) for (int k = 0; k < w[0]; ++k) a_save[k] = a[k];
+    for (int l = 0; l < n_layers; ++l) {
+        const double *W = params + param_offset(n_layers, w, l, 0);
+        const double *b = params + param_offset(n_layers, w, l, 1);
+        for (int o = 0; o < w[l + 1]; ++o) {
+            double s = 0.0;
+            for (int k = 0; k < w[l]; ++k) s += rnd_op(mode, W[(int64_t)o * w[l] + k]) * a[k];
+            z[o] = rnd(mode, s + rnd(mode, b[o]));
+        }
+        if (z_save) for (int o = 0; o < w[l + 1]; ++o) z_save[act_off[l + 1] + o] = z[o];
+        if (l + 1 < n_layers) {
+            for (int o = 0; o < w[l + 1]; ++o) {
+                double r = z[o] > 0.0 ? z[o] : 0.0;
+                z[o] = rnd_op(mode, r);
+            }
+            if (a_save) for (int o = 0; o < w[l + 1]; ++o) a_save[act_off[l + 1] + o] = z[o];
+        }
+        double *t = a; a = z; z = t;
+    }
+    return a[0];
+}
+
+static int max_width(int n_layers, const int *w) {
+    int m = 1;
+    for (int l = 0; l <= n_layers; ++l) m = w[l] > m ? w[l] : m;
+    return m;
+}
+
+int or_mlp_forward(int mode, int n_layers, const int *w, const double *params,
+                   int64_t rows, const double *x, double *y) {
+    int m = max_width(n_layers, w);
+    double *ba = (double *)malloc((size_t)m * sizeof(double));
+    double *bb = (double *)malloc((size_t)m * sizeof(double));
+    if (!ba || !bb) { free(ba); free(bb); return -1; }
+    for (int64_t r = 0; r < rows; ++r)
+        y[r] = forward_row(mode, n_layers, w, params, x + r * w[0], NULL, NULL, NULL, ba, bb);
+    free(ba);
+    free(bb);
+    return 0;
+}
+
+/* ------------------------------------------------------------------------ */
+/* greedy selection (Sec. 4.1; Algorithm 4 argmax of reward = -TTFT)        */
+/* ------------------------------------------------------------------------ */
+
+/* (a, i) precedes (b, j) in the lexicographic order (score, index), where NaN
+ * comes after every number and -0 equals +0. */
+static int precedes(float a, int32_t i, float b, int32_t j) {
+    int an = isnan(a), bn = isnan(b);
+    if (an != bn) return bn;          /* the number precedes the NaN */
+    if (!an && a != b) return a < b;  /* -0 == +0 compares equal here */
+    return i < j;
+}
+
+int or_argmin(int64_t n_req, int32_t n_inst, const float *scores, int32_t *choice, float *best) {
+    for (int64_t r = 0; r < n_req; ++r) {
+        int32_t c = 0;
+        for (int32_t i = 1; i < n_inst; ++i)
+            if (precedes(scores[r * n_inst + i], i, scores[r * n_inst + c], c)) c = i;
+        choice[r] = n_inst > 0 ? c : -1;
+        best[r] = n_inst > 0 ? scores[r * n_inst + c] : NAN;
+    }
+    return 0;
+}
+
+/* ------------------------------------------------------------------------ */
+/* sample ring (Sec. 4.3.2: recent records, oldest evicted on overflow)     */
+/* ------------------------------------------------------------------------ */
+
+/* Record j of the batch goes to slot (count + j) mod capacity. */
+int or_ring_append(int64_t capacity, int d, float *ring_x, float *ring_y, int64_t count,
+                   int64_t n, const float *x, const float *y) {
+    for (int64_t j = 0; j < n; ++j) {
+        int64_t slot = (count + j) % capacity;
+        memcpy(ring_x + slot * d, x + j * d, (size_t)d * sizeof(float));
+        ring_y[slot] = y[j];
+    }
+    return 0;
+}
+
+/* ------------------------------------------------------------------------ */
+/* online training step (Sec. 4.3.2; loss and optimiser are readings)       */
+/* ------------------------------------------------------------------------ */
+
+/* One minibatch step.  Rows idx[j] of the ring are z-scored (fp32), run forward
+ * (activations kept), the loss L = mean_j (yhat_j - y_j)^2 is formed and
+ * back-propagated:
+ *   dZ_L = 2 (yhat - y) / B
+ *   for l = L..1:  G = dZ_l (rounded to bf16 in BF16 mode)
+ *                  dW_l = G^T A_{l-1},  db_l = column sums of dZ_l (unrounded)
+ *                  dA_{l-1} = G W_l (W_l rounded to bf16 in BF16 mode)
+ *                  dZ_{l-1} = dA_{l-1} * [z_{l-1} > 0]
+ * (every quantity rounded to fp32 when formed, except in F64 mode), then
+ *   SGD : theta -= lr g
+ *   Adam: m = b1 m + (1-b1) g; v = b2 v + (1-b2) g^2;
+ *         theta -= lr (m / (1-b1^t)) / (sqrt(v / (1-b2^t)) + eps)
+ * with t the 1-based step number.  params / m / v are updated in place; the
+ * gradient is written to grad_out if given, the loss to *loss_out. */
+int or_train_step(int mode, int n_layers, const int *w, double *params, double *adam_m,
+                  double *adam_v, int64_t t, int opt, double lr, int batch,
+                  const float *ring_x, const float *ring_y, const int32_t *idx,
+                  const float *mean, const float *std, double *loss_out, double *grad_out) {
+    const double b1 = 0.9, b2 = 0.999, eps = 1e-8;
+    int d = w[0];
+    int64_t P = or_param_count(n_layers, w);
+    int64_t act_off[17];
+    act_off[0] = 0;
+    for (int l = 0; l < n_layers; ++l) act_off[l + 1] = act_off[l] + w[l];
+    int64_t act_row = act_off[n_layers] + 1;  /* a_0..a_{L-1} plus the output */
+    int m = max_width(n_layers, w);
+    double *Z = (double *)calloc((size_t)batch * act_row, sizeof(double));
+    double *A = (double *)calloc((size_t)batch * act_row, sizeof(double));
+    double *g = (double *)calloc((size_t)P, sizeof(double));
+    double *dz = (double *)calloc((size_t)batch * m, sizeof(double));
+    double *dz_prev = (double *)calloc((size_t)batch * m, sizeof(double));
+    double *ba = (double *)malloc((size_t)m * sizeof(double));
+    double *bb = (double *)malloc((size_t)m * sizeof(double));
+    double *xr = (double *)malloc((size_t)d * sizeof(double));
+    float *xf = (float *)malloc((size_t)d * sizeof(float));
+    double *yhat = (double *)malloc((size_t)(batch > 0 ? batch : 1) * sizeof(double));
+    if (!Z || !A || !g || !dz || !dz_prev || !ba || !bb || !xr || !xf || !yhat) return -1;
+
+    /* forward */
+    double loss = 0.0;
+    for (int j = 0; j < batch; ++j) {
+        or_zscore(d, ring_x + (int64_t)idx[j] * d, mean, std, xf);
+        for (int k = 0; k < d; ++k) xr[k] = (double)xf[k];
+        yhat[j] = forward_row(mode, n_layers, w, params, xr, Z + (int64_t)j * act_row,
+                              A + (int64_t)j * act_row, act_off, ba, bb);
+        double e = yhat[j] - (double)ring_y[idx[j]];
+        loss += e * e;
+    }
+    loss /= (double)batch;
+    if (loss_out) *loss_out = loss;
+
+    /* backward (the output layer has width 1) */
+    for (int j = 0; j < batch; ++j)
+        dz[(int64_t)j * m] = rnd(mode, 2.0 * (yhat[j] - (double)ring_y[idx[j]]) / (double)batch);
+    for (int l = n_layers - 1; l >= 0; --l) {
+        int fi = w[l], fo = w[l + 1];
+        double *gW = g + param_offset(n_layers, w, l, 0);
+        double *gb = g + param_offset(n_layers, w, l, 1);
+        const double *W = params + param_offset(n_layers, w, l, 0);
+        for (int o = 0; o < fo; ++o) {
+            double sb = 0.0;
+            for (int j = 0; j < batch; ++j) sb += dz[(int64_t)j * m + o];
+            gb[o] = rnd(mode, sb);
+            for (int k = 0; k < fi; ++k) {
+                double s = 0.0;
+                for (int j = 0; j < batch; ++j)
+                    s += rnd_op(mode, dz[(int64_t)j * m + o]) * A[(int64_t)j * act_row + act_off[l] + k];
+                gW[(int64_t)o * fi + k] = rnd(mode, s);
+            }
+        }
+        if (l > 0) {
+            for (int j = 0; j < batch; ++j)
+                for (int k = 0; k < fi; ++k) {
+                    double s = 0.0;
+                    for (int o = 0; o < fo; ++o)
+                        s += rnd_op(mode, dz[(int64_t)j * m + o]) * rnd_op(mode, W[(int64_t)o * fi + k]);
+                    double zprev = Z[(int64_t)j * act_row + act_off[l] + k];
+                    dz_prev[(int64_t)j * m + k] = zprev > 0.0 ? rnd(mode, s) : 0.0;
+                }
+            double *tmp = dz; dz = dz_prev; dz_prev = tmp;
+        }
+    }
+    if (grad_out) memcpy(grad_out, g, (size_t)P * sizeof(double));
+
+    /* update */
+    if (opt == OR_SGD) {
+        for (int64_t p = 0; p < P; ++p) params[p] = rnd(mode, params[p] - lr * g[p]);
+    } else {
+        double bc1 = 1.0 - pow(b1, (double)t), bc2 = 1.0 - pow(b2, (double)t);
+        for (int64_t p = 0; p < P; ++p) {
+            adam_m[p] = rnd(mode, b1 * adam_m[p] + (1.0 - b1) * g[p]);
+            adam_v[p] = rnd(mode, b2 * adam_v[p] + (1.0 - b2) * g[p] * g[p]);
+            double mh = adam_m[p] / bc1, vh = adam_v[p] / bc2;
+            params[p] = rnd(mode, params[p] - lr * mh / (sqrt(vh) + eps));
+        }
+    }
+    free(Z); free(A); free(g); free(dz); free(dz_prev);
+    free(ba); free(bb); free(xr); free(xf); free(yhat);
+    return 0;
+}
+
+/* Loss only (forward over the minibatch), for finite-difference checks. */
+int or_loss(int mode, int n_layers, const int *w, const double *params, int batch,
+            const float *ring_x, const float *ring_y, const int32_t *idx,
+            const float *mean, const float *std, double *loss_out) {
+    int d = w[0], m = max_width(n_layers, w);
+    double *ba = (double *)malloc((size_t)m * sizeof(double));
+    double *bb = (double *)malloc((size_t)m * sizeof(double));
+    double *xr = (double *)malloc((size_t)d * sizeof(double));
+    float *xf = (float *)malloc((size_t)d * sizeof(float));
+    if (!ba || !bb || !xr || !xf) return -1;
+    double loss = 0.0;
+    for (int j = 0; j < batch; ++j) {
+        or_zscore(d, ring_x + (int64_t)idx[j] * d, mean, std, xf);
+        for (int k = 0; k < d; ++k) xr[k] = (double)xf[k];
+        double e = forward_row(mode, n_layers, w, params, xr, NULL, NULL, NULL, ba, bb)
+                   - (double)ring_y[idx[j]];
+        loss += e * e;
+    }
+    *loss_out = loss / (double)batch;
+    free(ba); free(bb); free(xr); free(xf);
+    return 0;
+}
