@@ -1,0 +1,434 @@
+"""Benchmark of the Lodestar routing hot path on GB300.
+
+One step = one pass of the whole path over one batch of the homogeneous
+workload (32 instances x 4096 pending requests, prompts 64-4096 tokens with
+Zipf-shared prefixes, 64-dim features, bf16 MLP 64->256->256->1):
+  ls_snapshot_update (instance state rows)  -> ls_route_batch (hash, probe,
+  features, MLP, argmin for 131,072 pairs) -> ls_log_samples (4096 records)
+  -> ls_train_step (Adam, batch 4096) -> ls_publish.
+Metric: routing decisions per second (requests routed per second of whole
+steps).  Inputs resident in HBM; L2 flushed (512 MB write) between timed
+steps; CUDA events on the launching stream; W untimed warm-up steps.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Under torchrun each rank routes its own batch on its own GPU (replicas, weak
+scaling, no collective on the data path); rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+WORKLOAD = "homogeneous"
+METRIC = "routing decisions/sec (requests routed per second of whole route+log+train+publish steps)"
+UNIT = "decisions/s"
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-seconds", type=float, default=12.0, help="target oracle work for cpu_baseline")
+    return p.parse_args()
+
+
+def dist_setup(n_gpus):
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        dist.init_process_group(backend)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(world, value, device=None):
+    if world == 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ----------------------------------------------------------------------------
+# algorithmic cost of each kernel (per launch), for the roofline object
+# ----------------------------------------------------------------------------
+
+def mlp_flops_per_score(widths):
+    """Layer-1 factorised: only the 6 pair columns are per-(request, instance)
+    work; instance and request columns are done once per instance / request."""
+    f = 2 * 6 * widths[1]
+    for l in range(1, len(widths) - 1):
+        f += 2 * widths[l] * widths[l + 1]
+    return f
+
+
+def route_costs(cfg, R, N, hits, lens, keys, key_off):
+    """flops of the scorer and bytes of the prefix matcher for one batch."""
+    w = cfg.widths
+    flops = (mlp_flops_per_score(w) * R * N + 2 * N * cfg.d_inst * w[1] + 2 * R * cfg.d_req * w[1])
+    nb = lens // 16
+    need_blocks = np.minimum(nb, hits.max(axis=1) + 1)                 # blocks that must be hashed
+    tok_bytes = 4 * int(np.sum(np.minimum(lens, 16 * need_blocks)))
+    # distinct (instance, probed key): blocks 0..h (the miss included when h < n_r)
+    pr = []
+    for i in range(N):
+        upto = np.minimum(hits[:, i] + 1, nb).astype(np.int64)
+        tot = int(upto.sum())
+        base = np.repeat(key_off[:-1], upto)
+        within = np.arange(tot) - np.repeat(np.cumsum(upto) - upto, upto)
+        pr.append(np.unique(keys[base + within]).size if tot else 0)
+    probe_bytes = 8 * int(np.sum(pr))
+    out_bytes = 4 * R * N + 8 * R
+    return dict(score_flops=float(flops), prefix_bytes=float(tok_bytes + probe_bytes + out_bytes),
+                tok_bytes=tok_bytes, probe_bytes=probe_bytes)
+
+
+def train_flops(widths, B):
+    fwd = sum(2 * B * widths[l] * widths[l + 1] for l in range(len(widths) - 1))
+    bwd = sum(2 * B * widths[l] * widths[l + 1] for l in range(len(widths) - 1))        # dW
+    bwd += sum(2 * B * widths[l] * widths[l + 1] for l in range(1, len(widths) - 1))    # dX (l >= 1)
+    return fwd + bwd
+
+
+# ----------------------------------------------------------------------------
+# clocks during the timed region
+# ----------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("uuid,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid):
+        self.uuid = (uuid or "").lower()
+        self.p = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.f = open(self.path, "w")
+            self.p = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                       "-lms", "200"], stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.p = None
+
+    def stop(self):
+        if not self.p:
+            return None
+        self.p.terminate()
+        try:
+            self.p.wait(timeout=5)
+        except Exception:
+            self.p.kill()
+        self.f.close()
+        rows = []
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 8:
+                continue
+            if self.uuid and self.uuid not in parts[0].lower():
+                continue
+            rows.append(parts)
+        if not rows:
+            return None
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return float("nan")
+        sm = np.array([num(r[1]) for r in rows])
+        reasons = []
+        for k, name in zip(range(4, 8), ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
+                                         "sw_power_cap")):
+            if any(r[k].lower() == "active" for r in rows):
+                reasons.append(name)
+        return {"sm_mhz": float(np.nanmedian(sm)), "sm_max_mhz": float(np.nanmax([num(r[2]) for r in rows])),
+                "reasons": reasons, "samples": len(rows),
+                "power_w_max": float(np.nanmax([num(r[3]) for r in rows]))}
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+# ----------------------------------------------------------------------------
+# CPU oracle (cpu_baseline and --impl reference)
+# ----------------------------------------------------------------------------
+
+def oracle_work(wl, inst_keys, n_req, rng):
+    """Oracle pass over a sample: route n_req requests (hash, hits, features,
+    bf16 MLP, argmin) and one training step on n_req logged records."""
+    import oracle
+    idx = np.sort(rng.choice(len(wl.tok_off) - 1, size=n_req, replace=False))
+    t0 = time.perf_counter()
+    oracle.route(wl, inst_keys=inst_keys, req_idx=idx)
+    tr = oracle.Trainer(wl.cfg.widths, wl.params, wl.cfg.dtype)
+    bidx = rng.integers(0, len(wl.samples_y), size=n_req).astype(np.int32)
+    tr.step(wl.samples_x, wl.samples_y, bidx, wl.mean, wl.std, "adam", 3e-4)
+    return time.perf_counter() - t0
+
+
+def cpu_baseline(wl, inst_keys, target_s):
+    rng = np.random.default_rng(0)
+    t_cal = oracle_work(wl, inst_keys, 16, rng)
+    n = int(np.clip(16 * target_s / max(t_cal, 1e-3), 16, len(wl.tok_off) - 1))
+    t = oracle_work(wl, inst_keys, n, rng)
+    return {"value": n / t, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{n} of {len(wl.tok_off) - 1} requests of the {WORKLOAD} batch routed by the "
+                      f"single-thread C oracle (hash, hits, features, fp64-accumulated bf16 MLP, argmin) "
+                      f"plus one Adam step on {n} logged records; {t:.1f} s"}
+
+
+def run_reference(args, world, rank):
+    from paper_2606_00946_gb300 import workload as W
+    import oracle
+    if rank != 0:
+        return 0
+    wl = W.generate(WORKLOAD)
+    inst_keys = oracle.instance_keys(wl)
+    rng = np.random.default_rng(1)
+    n = 48
+    for _ in range(args.warmup):
+        oracle_work(wl, inst_keys, n, rng)
+    times = [oracle_work(wl, inst_keys, n, rng) for _ in range(args.steps)]
+    ms = 1e3 * float(np.mean(times))
+    value = n / (ms / 1e3)
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded generator shaped like the paper's prefix-sharing workloads)",
+            "config": {"workload": f"{WORKLOAD}: 32 instances x 4096 requests, bf16 MLP 64-256-256-1",
+                       "sample_requests_per_step": n},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                             "sample": f"{n} requests + one Adam step on {n} records per step"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
+# ----------------------------------------------------------------------------
+# GPU arm
+# ----------------------------------------------------------------------------
+
+def main():
+    args = parse()
+    world, rank, local = dist_setup(args.gpus)
+    if args.impl == "reference":
+        return run_reference(args, world, rank)
+
+    import torch
+    from paper_2606_00946_gb300 import build as B
+    from paper_2606_00946_gb300 import harness as H
+    from paper_2606_00946_gb300 import lodestar as L
+    from paper_2606_00946_gb300 import workload as W
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    B.build()
+    wl = W.generate(WORKLOAD)
+    cfg = wl.cfg
+    R, N, Bt = cfg.n_req, cfg.n_inst, cfg.train_batch
+    ring = max(cfg.n_samples, 4 * Bt)
+    r = H.Router.for_config(cfg, ring_capacity=ring)
+    dw = H.DeviceWorkload(wl, device=dev)
+    dw.load(r)
+    sx = torch.from_numpy(wl.samples_x).to(dev)
+    sy = torch.from_numpy(wl.samples_y).to(dev)
+    r.log(sx, sy)                                   # fill the ring once
+    states = [dw.inst_state, torch.from_numpy(W.instance_state(np.random.default_rng(99), cfg)).to(dev)]
+    out = {"choice": torch.empty(R, dtype=torch.int32, device=dev),
+           "best": torch.empty(R, dtype=torch.float32, device=dev), "scores": None, "hits": None}
+    loss = torch.zeros(1, device=dev)
+    flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step(k):
+        r.snapshot(N, states[k & 1])
+        r.route(dw.tok, dw.tok_off, dw.req_feats, N, out=out)
+        a = (k * Bt) % len(wl.samples_y)
+        r.log(sx[a:a + Bt], sy[a:a + Bt])
+        r.train(Bt, None, opt="adam", lr=cfg.train_lr, loss_out=loss)
+        r.publish()
+
+    for k in range(args.warmup):
+        step(k)
+    torch.cuda.synchronize()
+    # per-pair hits of this batch (for the algorithmic byte count; not timed)
+    chk = r.route(dw.tok, dw.tok_off, dw.req_feats, N)
+    hits = chk["hits"].cpu().numpy()
+    keys, ko = r.hash_blocks(dw.tok, dw.tok_off)
+    costs = route_costs(cfg, R, N, hits, np.diff(wl.tok_off), keys.cpu().numpy(), ko.cpu().numpy())
+
+    uuid = None
+    try:
+        uuid = str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:
+        pass
+    clocks = ClockSampler(uuid)
+    L.ls_trace_enable(r.h, True)
+    L.ls_trace_read(r.h)
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks.start()
+    times = []
+    for k in range(args.steps):
+        flush.fill_(k & 0xFF)                       # evict L2 between timed steps
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        step(args.warmup + k)
+        e1.record(stream)
+        e1.synchronize()
+        times.append(e0.elapsed_time(e1))
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    rc, trace = L.ls_trace_read(r.h)
+    L.ls_trace_enable(r.h, False)
+    barrier(world)
+    ms = max_over_ranks(world, float(np.mean(times)), dev if world > 1 and torch.distributed.get_backend() == "nccl" else None)
+    value = world * R / (ms / 1e3)
+
+    # roofline of the dominant kernel (largest device time in the timed region)
+    peaks, peak_src = measured_peaks()
+    per = {k: v[1] / max(v[0], 1) for k, v in trace.items()}
+    dom = max(trace, key=lambda k: trace[k][1])
+    launches = int(sum(v[0] for v in trace.values()))
+    if dom == "prefix_match":
+        alg, peak, unit, bound = costs["prefix_bytes"] / 1e9, peaks["hbm_gbs"], "GB/s", "hbm"
+    elif dom in ("score_simt", "score_tc"):
+        alg, peak, unit, bound = costs["score_flops"] / 1e12, peaks["bf16_tflops"], "TFLOP/s", "tensor"
+    else:
+        alg, peak, unit, bound = train_flops(cfg.widths, Bt) / 1e12 / 5, peaks["bf16_tflops"], "TFLOP/s", "tensor"
+    achieved = alg / (per[dom] / 1e3)
+    roofline = {"kernel": dom, "bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
+                "frac": achieved / peak, "traffic": None, "peak_source": f"{peak_src} (burst)",
+                "avg_launch_ms": per[dom]}
+
+    # end to end through the C ABI with host buffers
+    e2e = None
+    if not args.no_e2e:
+        h_tok = torch.from_numpy(wl.tok).pin_memory()
+        h_off = torch.from_numpy(wl.tok_off).pin_memory()
+        h_req = torch.from_numpy(wl.req_feats).pin_memory()
+        h_st = [s.cpu().pin_memory() for s in states]
+        h_x = torch.from_numpy(wl.samples_x).pin_memory()
+        h_y = torch.from_numpy(wl.samples_y).pin_memory()
+        d_tok = torch.empty_like(dw.tok)
+        d_off = torch.empty_like(dw.tok_off)
+        d_req = torch.empty_like(dw.req_feats)
+        d_st = torch.empty_like(states[0])
+        d_x = torch.empty(Bt, cfg.d, device=dev)
+        d_y = torch.empty(Bt, device=dev)
+        h_choice = torch.empty(R, dtype=torch.int32).pin_memory()
+        h_best = torch.empty(R, dtype=torch.float32).pin_memory()
+        h_loss = torch.empty(1).pin_memory()
+        h2d = d_tok.numel() * 4 + d_off.numel() * 8 + d_req.numel() * 4 + d_st.numel() * 4 + \
+            d_x.numel() * 4 + d_y.numel() * 4
+        d2h = R * 4 + R * 4 + 4
+
+        def e2e_step(k):
+            a = (k * Bt) % len(wl.samples_y)
+            d_tok.copy_(h_tok, non_blocking=True)
+            d_off.copy_(h_off, non_blocking=True)
+            d_req.copy_(h_req, non_blocking=True)
+            d_st.copy_(h_st[k & 1], non_blocking=True)
+            d_x.copy_(h_x[a:a + Bt], non_blocking=True)
+            d_y.copy_(h_y[a:a + Bt], non_blocking=True)
+            r.snapshot(N, d_st)
+            r.route(d_tok, d_off, d_req, N, out=out)
+            r.log(d_x, d_y)
+            r.train(Bt, None, opt="adam", lr=cfg.train_lr, loss_out=loss)
+            r.publish()
+            h_choice.copy_(out["choice"], non_blocking=True)
+            h_best.copy_(out["best"], non_blocking=True)
+            h_loss.copy_(loss, non_blocking=True)
+
+        for k in range(args.warmup):
+            e2e_step(k)
+        torch.cuda.synchronize()
+        et = []
+        for k in range(args.steps):
+            flush.fill_(k & 0xFF)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            e2e_step(k)
+            e1.record(stream)
+            e1.synchronize()
+            et.append(e0.elapsed_time(e1))
+        ems = max_over_ranks(world, float(np.mean(et)), None)
+        e2e = {"value": world * R / (ems / 1e3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+               "d2h_bytes_per_step": int(d2h), "ms_per_step": ems}
+
+    status = r.sync()
+    if status != L.LS_OK:
+        print(json.dumps({"error": f"device status {status}"}), file=sys.stderr)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        cpu = cpu_baseline(wl, oracle.instance_keys(wl), args.cpu_seconds)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded generator shaped like the paper's prefix-sharing workloads)",
+            "config": {"workload": f"{WORKLOAD}: 32 instances x 4096 requests/step, prompts 64-4096 "
+                                   "tokens with Zipf(1.1) prefixes over 256 templates, 16384 cached "
+                                   "blocks/instance, bf16 MLP 64-256-256-1, Adam batch 4096",
+                       "pairs_per_step": R * N, "train_samples_per_step": Bt,
+                       "l2": "flushed between timed steps (512 MB write)", "parallelism": "replicas"},
+            "train_samples_per_s": world * Bt / (ms / 1e3),
+            "scores_per_s": world * R * N / (ms / 1e3),
+            "roofline": roofline,
+            "kernels_ms_per_step": {k: v[1] / args.steps for k, v in sorted(trace.items(), key=lambda kv: -kv[1][1])},
+            "cpu_baseline": cpu,
+            "e2e": e2e,
+            "gpu_launches": launches,
+            "gpu_launches_per_step": launches / args.steps,
+            "clocks": clk,
+            "algorithmic": costs,
+        }
+        print(json.dumps(line))
+    r.close()
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

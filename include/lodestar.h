@@ -1,0 +1,213 @@
+/*
+ * lodestar.h -- C ABI of the GB300 routing hot path of Lodestar, an
+ * online-learned LLM inference router.
+ *
+ * Per routing batch the library computes, for every (request, instance) pair,
+ * the prefix-cache hit length of the request's prompt on the instance, the
+ * pair's feature vector, the predicted TTFT of the shared reward model, and
+ * per request the instance with the lowest prediction.  It also logs
+ * (features, observed TTFT) records and runs minibatch training steps of the
+ * predictor, publishing new weights atomically to the routing side.
+ *
+ * Conventions (all entry points):
+ *  - Every array argument is a DEVICE pointer owned by the caller unless the
+ *    comment says otherwise; it is read or written only by work enqueued on
+ *    the given stream, so it must stay valid until that work completes.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *    Calls are asynchronous with respect to the host.
+ *  - Return value: LS_OK (0) or a negative ls_status.  Argument errors are
+ *    detected on the host before anything is enqueued.  Errors found on the
+ *    device (table overflow, an out-of-range ring slot) are latched in the
+ *    context and reported by ls_sync_status().  ls_last_error() gives a
+ *    message for the last failing call on the calling thread.
+ *  - No call aborts, traps or throws across the ABI.
+ *  - A context is used from one host thread at a time, except that
+ *    ls_route_batch (on one stream) may run concurrently with
+ *    ls_log_samples / ls_train_step / ls_publish (on another stream).
+ *  - Block size is 16 tokens; prompts are int32 token ids.
+ */
+#ifndef LODESTAR_H
+#define LODESTAR_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define LS_MAX_LAYERS 8
+#define LS_BLOCK_TOKENS 16
+#define LS_PAIR_FEATURES 6
+
+typedef struct ls_ctx ls_ctx;
+
+typedef enum {
+    LS_OK = 0,
+    LS_ERR_ARG = -1,        /* invalid argument (null pointer, bad size, ...) */
+    LS_ERR_CUDA = -2,       /* a CUDA runtime call failed */
+    LS_ERR_OOM = -3,        /* device allocation failed */
+    LS_ERR_TABLE_FULL = -4, /* an instance holds more keys than configured */
+    LS_ERR_TIMEOUT = -5,    /* a bounded device-side wait gave up */
+    LS_ERR_STATE = -6       /* call not valid in the current state */
+} ls_status;
+
+enum { LS_F32 = 0, LS_BF16 = 1 };      /* predictor arithmetic */
+enum { LS_REPLACE = 0, LS_INSERT = 1 };/* ls_snapshot_update key modes */
+enum { LS_SGD = 0, LS_ADAM = 1 };      /* ls_train_step optimisers */
+
+/* Predictor and capacity configuration, fixed at ls_create.
+ * widths[0] = d = 6 + d_inst + d_req (pair features, instance state, request
+ * extras), widths[1..n_layers-1] = hidden widths, widths[n_layers] = 1. */
+typedef struct {
+    int32_t n_layers;                    /* Linear layers, 1..LS_MAX_LAYERS */
+    int32_t widths[LS_MAX_LAYERS + 1];
+    int32_t d_inst;                      /* instance-state features per instance */
+    int32_t d_req;                       /* request extras per request */
+    int32_t dtype;                       /* LS_F32 or LS_BF16 */
+    int32_t max_instances;
+    int32_t max_requests;                /* per ls_route_batch call */
+    int64_t max_keys_per_instance;       /* cached blocks tracked per instance */
+    float max_load;                      /* hash-table load bound in (0, 1) */
+    int64_t ring_capacity;               /* logged samples kept (oldest evicted) */
+    int32_t max_train_batch;
+} ls_config;
+
+typedef struct {
+    int32_t n_inst;              /* instances in the current snapshot */
+    int32_t d;                   /* feature width */
+    int64_t n_params;            /* predictor parameter count */
+    int64_t table_slots;         /* slots per instance table */
+    int64_t ring_count;          /* samples ever logged */
+    int64_t train_steps;         /* training steps taken */
+    uint64_t weight_version;     /* version of the last published weights, 0 = none */
+} ls_info;
+
+/* Number of predictor parameters: sum over layers of out*in + out. */
+int64_t ls_param_count(const ls_config *cfg);
+
+/* Create a context on the current CUDA device.  Allocates all device memory
+ * the context will ever use (tables, weights, optimiser state, sample ring,
+ * scratch).  *out receives the context.  LS_ERR_ARG on an invalid config,
+ * LS_ERR_OOM if an allocation fails. */
+int ls_create(const ls_config *cfg, ls_ctx **out);
+
+/* Release the context and its device memory (synchronises the device). */
+void ls_destroy(ls_ctx *ctx);
+
+/* Message for the last failing call on this thread ("" if none). */
+const char *ls_last_error(void);
+
+/* Blocks until all work of the device has completed, then returns and clears
+ * the first error latched by device code (LS_OK if none). */
+int ls_sync_status(ls_ctx *ctx);
+
+int ls_get_info(ls_ctx *ctx, ls_info *out /* host */);
+
+/* Set the fp32 master parameters (device, ls_param_count floats: W1 [w1,w0]
+ * row-major, b1 [w1], W2, b2, ...), reset optimiser state and step count.
+ * Routing keeps using the previously published weights until ls_publish. */
+int ls_set_params(ls_ctx *ctx, const float *params, void *stream);
+int ls_get_params(ls_ctx *ctx, float *params_out, void *stream);
+
+/* Optimiser state for checkpointing: Adam first and second moments (device,
+ * n_params floats each) and the step count (host). */
+int ls_get_opt_state(ls_ctx *ctx, float *m_out, float *v_out, int64_t *step_out, void *stream);
+int ls_set_opt_state(ls_ctx *ctx, const float *m, const float *v, int64_t step, void *stream);
+
+/* Per-feature normalisation statistics (Algorithm 4, Normalize): mean[d],
+ * std[d] (device floats).  Features are z-scored as (x - mean) / std, with a
+ * std below 1e-12 replaced by 1. */
+int ls_set_normalizer(ls_ctx *ctx, const float *mean, const float *std, void *stream);
+
+/* Cluster snapshot (Sec. 4.2 cluster snapshot manager, prefix KV-cache tracker).
+ * n_inst instances; inst_state [n_inst, d_inst] row-major floats (queued and
+ * running requests, inflight prefill / decode tokens, KV utilisation, ...).
+ * keys: cached-block keys of each instance as CSR, keys[key_off[i] ..
+ * key_off[i+1]) for instance i, key_off [n_inst+1] int64 on the device,
+ * n_keys = key_off[n_inst] given on the host.  keys == NULL updates the state
+ * rows only.  mode LS_REPLACE empties the tables of instances 0..n_inst-1
+ * first; LS_INSERT adds to them.  A key value 0 is stored as 1 (0 marks an
+ * empty slot).  More than max_keys_per_instance distinct keys in one table
+ * latches LS_ERR_TABLE_FULL. */
+int ls_snapshot_update(ls_ctx *ctx, int32_t n_inst, const float *inst_state,
+                       const uint64_t *keys, const int64_t *key_off, int64_t n_keys,
+                       int32_t mode, void *stream);
+
+/* Block keys of token sequences (the keys the prefix tracker stores).
+ * Sequence s is tok[tok_off[s] .. tok_off[s+1]) (tok_off int64 [n_seq+1]);
+ * its floor(L_s/16) full blocks get keys keys_out[key_off[s] + b].
+ * Definition (this library's reading; the paper says only that the prefix
+ * index may be a hash table, Sec. 2):
+ *   mix64 = SplitMix64 output finaliser, G = 0x9E3779B97F4A7C15;
+ *   c_b = mix64( XOR_{j<8} mix64(w_{b,j} + (j+1) G) ), w_{b,j} the 64-bit word
+ *         of tokens 16b+2j (low half) and 16b+2j+1 (high half);
+ *   s_{-1} = G, s_b = s_{b-1} G + c_b (mod 2^64); key_b = mix64(s_b), 0 -> 1.
+ * key_b depends on every token of blocks 0..b (prefix reuse is strictly
+ * sequential, Sec. 2). */
+int ls_hash_blocks(ls_ctx *ctx, int32_t n_seq, const int32_t *tok, const int64_t *tok_off,
+                   uint64_t *keys_out, const int64_t *key_off, void *stream);
+
+/* Normalised feature rows of all (request, instance) pairs for given hit
+ * lengths (hits [n_req, n_inst] int32): row r*n_inst + i of x_out [n_req*n_inst, d]
+ * is the z-scored [L, h, 16h, 16h/L, L-16h, ceil(L/16)-h || inst_state[i] ||
+ * req_feats[r]] (Sec. 4.1 Features; Algorithm 4 Normalize), L = prompt length
+ * from tok_off.  Parity hook; ls_route_batch computes the same rows on chip. */
+int ls_assemble_features(ls_ctx *ctx, int32_t n_req, const int64_t *tok_off, const int32_t *hits,
+                         const float *req_feats, float *x_out, void *stream);
+
+/* Route a batch (Sec. 4.1 reward model, Algorithm 4): for each request r
+ * (prompt tok[tok_off[r] .. tok_off[r+1]), request extras req_feats [n_req,
+ * d_req]) and each snapshot instance i: hit length h[r,i] (leading full blocks
+ * whose keys are all in instance i's table, stopping at the first miss),
+ * features, predicted TTFT yhat[r,i] from the last published weights, and
+ * choice[r] = argmin_i yhat[r,i] (ties -> lowest index, NaN last),
+ * best[r] = yhat[r, choice[r]].  Optional outputs (NULL to skip):
+ * scores_opt [n_req, n_inst] floats, hits_opt [n_req, n_inst] int32.
+ * *weight_version_out (HOST pointer, nullable) receives the version used.
+ * All requests of a batch see the same snapshot.  LS_ERR_STATE if no
+ * weights were published or the snapshot is empty. */
+int ls_route_batch(ls_ctx *ctx, int32_t n_req, const int32_t *tok, const int64_t *tok_off,
+                   const float *req_feats, int32_t *choice, float *best, float *scores_opt,
+                   int32_t *hits_opt, uint64_t *weight_version_out, void *stream);
+
+/* Append n logged records (raw feature rows feats [n, d], observed TTFT in
+ * seconds ttft [n]) to the sample ring: record j goes to slot
+ * (count + j) mod ring_capacity, evicting the oldest (Sec. 4.3.2). */
+int ls_log_samples(ls_ctx *ctx, int32_t n, const float *feats, const float *ttft, void *stream);
+
+/* One minibatch step of the predictor on ring slots idx [batch] (int32 on the
+ * device; NULL = slots (k*batch + j) mod min(count, capacity) at step k).
+ * Loss = mean squared error of the predicted TTFT (seconds).  opt LS_SGD:
+ * theta -= lr g; LS_ADAM: beta1 0.9, beta2 0.999, eps 1e-8, bias-corrected.
+ * Updates the master weights only; routing sees them after ls_publish.
+ * loss_out: device float (nullable) receives the minibatch loss before the
+ * update.  An idx entry outside the filled part of the ring latches
+ * LS_ERR_ARG and is read as slot 0. */
+int ls_train_step(ls_ctx *ctx, int32_t batch, const int32_t *idx, int32_t opt, float lr,
+                  float *loss_out, void *stream);
+
+/* Atomically publish the master weights to routing (Sec. 4.3.1 P2: swap of the
+ * model pointer).  Route calls enqueued after this call (in host order) use
+ * the new version once this stream reaches the publish point; earlier routes
+ * keep the version they started with. */
+int ls_publish(ls_ctx *ctx, void *stream);
+
+/* Kernel tracing.  While enabled, each kernel launch of this context is
+ * bracketed by CUDA events on its launching stream (a few microseconds of host
+ * time per launch).  ls_trace_read synchronises the device, writes up to
+ * max_entries per-kernel totals (name, launches, summed device time in ms)
+ * to the HOST array out, sets *n_out, and resets the totals. */
+typedef struct {
+    char name[32];
+    int64_t launches;
+    double total_ms;
+} ls_trace_entry;
+
+int ls_trace_enable(ls_ctx *ctx, int32_t on);
+int ls_trace_read(ls_ctx *ctx, ls_trace_entry *out, int32_t max_entries, int32_t *n_out);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LODESTAR_H */

@@ -1,0 +1,471 @@
+// C ABI entry points (include/lodestar.h): argument checks, the context's
+// device memory, stream ordering of publish / route, and error reporting.
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <string>
+
+#include "common.cuh"
+
+using namespace ls;
+
+namespace ls {
+const char* const kTraceNames[TR_COUNT] = {
+    "hash_blocks", "table_insert", "prefix_match", "score_simt", "argmin", "assemble_features",
+    "ring_append", "publish", "train_gather", "gemm_fwd", "loss_grad", "gemm_dw", "reduce_dw",
+    "colsum_db", "gemm_dx", "optimizer", "memset"};
+}
+
+struct ls_ctx {
+  Ctx c;
+};
+
+namespace {
+
+thread_local std::string g_err;
+
+int fail(int code, const std::string& msg) {
+  g_err = msg;
+  return code;
+}
+
+int cuda_fail(cudaError_t e, const char* where) {
+  g_err = std::string(where) + ": " + cudaGetErrorString(e);
+  return e == cudaErrorMemoryAllocation ? LS_ERR_OOM : LS_ERR_CUDA;
+}
+
+#define LS_CK(call)                                   \
+  do {                                                \
+    cudaError_t e_ = (call);                          \
+    if (e_ != cudaSuccess) return cuda_fail(e_, #call); \
+  } while (0)
+
+inline cudaStream_t S(void* p) { return reinterpret_cast<cudaStream_t>(p); }
+
+int64_t count_params(const ls_config& c) {
+  int64_t n = 0;
+  for (int l = 0; l < c.n_layers; ++l) n += (int64_t)c.widths[l + 1] * c.widths[l] + c.widths[l + 1];
+  return n;
+}
+
+bool check_config(const ls_config* c, std::string& why) {
+  if (!c) { why = "config is NULL"; return false; }
+  if (c->n_layers < 1 || c->n_layers > LS_MAX_LAYERS) { why = "n_layers must be 1..8"; return false; }
+  if (c->d_inst < 0 || c->d_req < 0) { why = "d_inst and d_req must be >= 0"; return false; }
+  if (c->widths[0] != LS_PAIR_FEATURES + c->d_inst + c->d_req) {
+    why = "widths[0] must equal 6 + d_inst + d_req";
+    return false;
+  }
+  for (int l = 0; l <= c->n_layers; ++l)
+    if (c->widths[l] < 1 || c->widths[l] > 1024) { why = "widths must be 1..1024"; return false; }
+  if (c->widths[c->n_layers] != 1) { why = "the output width must be 1"; return false; }
+  if (c->dtype != LS_F32 && c->dtype != LS_BF16) { why = "dtype must be LS_F32 or LS_BF16"; return false; }
+  if (c->max_instances < 1 || c->max_instances > 8192) { why = "max_instances must be 1..8192"; return false; }
+  if (c->max_requests < 1) { why = "max_requests must be >= 1"; return false; }
+  if (c->max_keys_per_instance < 1) { why = "max_keys_per_instance must be >= 1"; return false; }
+  if (!(c->max_load > 0.0f && c->max_load < 1.0f)) { why = "max_load must be in (0, 1)"; return false; }
+  if (c->ring_capacity < 1) { why = "ring_capacity must be >= 1"; return false; }
+  if (c->max_train_batch < 1) { why = "max_train_batch must be >= 1"; return false; }
+  const double need = std::ceil((double)c->max_keys_per_instance / (double)c->max_load);
+  if (need > (double)(1ull << 31)) { why = "table would exceed 2^31 slots"; return false; }
+  return true;
+}
+
+int64_t table_slots(const ls_config& c) {
+  const double need = std::ceil((double)c.max_keys_per_instance / (double)c.max_load);
+  int64_t s = 16;
+  while ((double)s < need) s <<= 1;
+  return s;
+}
+
+template <class T>
+cudaError_t dalloc(T** p, int64_t n) {
+  *p = nullptr;
+  if (n <= 0) n = 1;
+  return cudaMalloc(reinterpret_cast<void**>(p), (size_t)n * sizeof(T));
+}
+
+void free_all(Ctx& c) {
+  void* ptrs[] = {c.tables, c.table_count, c.inst_state, c.mean, c.stdv, c.master, c.adam_m,
+                  c.adam_v, c.pub[0].params, c.pub[0].wt, c.pub[1].params, c.pub[1].wt,
+                  c.ring_x, c.ring_y, c.hits, c.scores, c.tx, c.tz, c.ty, c.dz0, c.dz1, c.grad,
+                  c.gpart, c.loss_tmp, c.d_err};
+  for (void* p : ptrs)
+    if (p) cudaFree(p);
+  for (int b = 0; b < 2; ++b) {
+    if (c.pub_ready[b]) cudaEventDestroy(c.pub_ready[b]);
+    if (c.route_done[b]) cudaEventDestroy(c.route_done[b]);
+  }
+  if (c.tracer.ready)
+    for (int i = 0; i < Tracer::kPool; ++i) cudaEventDestroy(c.tracer.ev[i]);
+}
+
+}  // namespace
+
+extern "C" {
+
+int64_t ls_param_count(const ls_config* cfg) {
+  std::string why;
+  if (!check_config(cfg, why)) return fail(LS_ERR_ARG, why);
+  return count_params(*cfg);
+}
+
+const char* ls_last_error(void) { return g_err.c_str(); }
+
+int ls_create(const ls_config* cfg, ls_ctx** out) {
+  std::string why;
+  if (!out) return fail(LS_ERR_ARG, "out is NULL");
+  *out = nullptr;
+  if (!check_config(cfg, why)) return fail(LS_ERR_ARG, why);
+  ls_ctx* h = new ls_ctx();
+  Ctx& c = h->c;
+  c.cfg = *cfg;
+  MlpDesc& m = c.mlp;
+  m.n_layers = cfg->n_layers;
+  m.bf16 = cfg->dtype == LS_BF16;
+  int64_t off = 0, wt = 0;
+  m.max_width = 1;
+  for (int l = 0; l <= cfg->n_layers; ++l) {
+    m.w[l] = cfg->widths[l];
+    m.max_width = std::max(m.max_width, cfg->widths[l]);
+  }
+  for (int l = 0; l < cfg->n_layers; ++l) {
+    m.woff[l] = off;
+    off += (int64_t)m.w[l + 1] * m.w[l];
+    m.boff[l] = off;
+    off += m.w[l + 1];
+    m.wtoff[l] = wt;
+    wt += (int64_t)m.w[l + 1] * m.w[l];
+  }
+  c.d = m.w[0];
+  c.n_params = off;
+  c.wt_total = wt;
+  {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&c.sms, cudaDevAttrMultiProcessorCount, dev);
+  }
+  c.slots = table_slots(*cfg);
+  c.mask = (uint32_t)(c.slots - 1);
+
+  const int64_t NI = cfg->max_instances, R = cfg->max_requests, B = cfg->max_train_batch;
+  int64_t sum_in = 0, sum_out = 0, max_wl = 1;
+  for (int l = 0; l < cfg->n_layers; ++l) {
+    sum_in += m.w[l];
+    sum_out += m.w[l + 1];
+    max_wl = std::max<int64_t>(max_wl, (int64_t)m.w[l] * m.w[l + 1]);
+  }
+  cudaError_t e = cudaSuccess;
+  auto A = [&](cudaError_t r) { if (e == cudaSuccess) e = r; };
+  A(dalloc(&c.tables, NI * c.slots));
+  A(dalloc(&c.table_count, NI));
+  A(dalloc(&c.inst_state, NI * std::max(1, cfg->d_inst)));
+  A(dalloc(&c.mean, c.d));
+  A(dalloc(&c.stdv, c.d));
+  A(dalloc(&c.master, c.n_params));
+  A(dalloc(&c.adam_m, c.n_params));
+  A(dalloc(&c.adam_v, c.n_params));
+  for (int b = 0; b < 2; ++b) {
+    A(dalloc(&c.pub[b].params, c.n_params));
+    A(dalloc(&c.pub[b].wt, c.wt_total));
+  }
+  A(dalloc(&c.ring_x, cfg->ring_capacity * c.d));
+  A(dalloc(&c.ring_y, cfg->ring_capacity));
+  A(dalloc(&c.hits, R * NI));
+  A(dalloc(&c.scores, R * NI));
+  A(dalloc(&c.tx, B * sum_in));
+  A(dalloc(&c.tz, B * sum_out));
+  A(dalloc(&c.ty, B));
+  A(dalloc(&c.dz0, B * m.max_width));
+  A(dalloc(&c.dz1, B * m.max_width));
+  A(dalloc(&c.grad, c.n_params));
+  c.gpart_floats = 64 * max_wl;
+  A(dalloc(&c.gpart, c.gpart_floats));
+  A(dalloc(&c.loss_tmp, 1));
+  A(dalloc(&c.d_err, 1));
+  for (int b = 0; b < 2 && e == cudaSuccess; ++b) {
+    A(cudaEventCreateWithFlags(&c.pub_ready[b], cudaEventDisableTiming));
+    A(cudaEventCreateWithFlags(&c.route_done[b], cudaEventDisableTiming));
+  }
+  if (e == cudaSuccess) {
+    A(cudaMemset(c.tables, 0, (size_t)NI * c.slots * sizeof(uint64_t)));
+    A(cudaMemset(c.table_count, 0, (size_t)NI * sizeof(int32_t)));
+    A(cudaMemset(c.adam_m, 0, (size_t)c.n_params * sizeof(float)));
+    A(cudaMemset(c.adam_v, 0, (size_t)c.n_params * sizeof(float)));
+    A(cudaMemset(c.d_err, 0, sizeof(int)));
+    A(cudaDeviceSynchronize());
+  }
+  if (e != cudaSuccess) {
+    int rc = cuda_fail(e, "ls_create");
+    free_all(c);
+    delete h;
+    return rc;
+  }
+  *out = h;
+  return LS_OK;
+}
+
+void ls_destroy(ls_ctx* h) {
+  if (!h) return;
+  cudaDeviceSynchronize();
+  free_all(h->c);
+  delete h;
+}
+
+int ls_sync_status(ls_ctx* h) {
+  if (!h) return fail(LS_ERR_ARG, "ctx is NULL");
+  LS_CK(cudaDeviceSynchronize());
+  int code = 0;
+  LS_CK(cudaMemcpy(&code, h->c.d_err, sizeof(int), cudaMemcpyDeviceToHost));
+  LS_CK(cudaMemset(h->c.d_err, 0, sizeof(int)));
+  LS_CK(cudaDeviceSynchronize());
+  if (code) return fail(code, "error latched by device code");
+  return LS_OK;
+}
+
+int ls_get_info(ls_ctx* h, ls_info* out) {
+  if (!h || !out) return fail(LS_ERR_ARG, "NULL argument");
+  Ctx& c = h->c;
+  std::lock_guard<std::mutex> g(c.mu);
+  out->n_inst = c.n_inst;
+  out->d = c.d;
+  out->n_params = c.n_params;
+  out->table_slots = c.slots;
+  out->ring_count = c.ring_count;
+  out->train_steps = c.step;
+  out->weight_version = c.version;
+  return LS_OK;
+}
+
+int ls_set_params(ls_ctx* h, const float* params, void* stream) {
+  if (!h || !params) return fail(LS_ERR_ARG, "NULL argument");
+  Ctx& c = h->c;
+  const size_t n = (size_t)c.n_params * sizeof(float);
+  LS_CK(cudaMemcpyAsync(c.master, params, n, cudaMemcpyDeviceToDevice, S(stream)));
+  LS_CK(cudaMemsetAsync(c.adam_m, 0, n, S(stream)));
+  LS_CK(cudaMemsetAsync(c.adam_v, 0, n, S(stream)));
+  c.step = 0;
+  c.have_params = true;
+  return LS_OK;
+}
+
+int ls_get_params(ls_ctx* h, float* params_out, void* stream) {
+  if (!h || !params_out) return fail(LS_ERR_ARG, "NULL argument");
+  Ctx& c = h->c;
+  LS_CK(cudaMemcpyAsync(params_out, c.master, (size_t)c.n_params * sizeof(float),
+                        cudaMemcpyDeviceToDevice, S(stream)));
+  return LS_OK;
+}
+
+int ls_get_opt_state(ls_ctx* h, float* m_out, float* v_out, int64_t* step_out, void* stream) {
+  if (!h || !m_out || !v_out || !step_out) return fail(LS_ERR_ARG, "NULL argument");
+  Ctx& c = h->c;
+  const size_t n = (size_t)c.n_params * sizeof(float);
+  LS_CK(cudaMemcpyAsync(m_out, c.adam_m, n, cudaMemcpyDeviceToDevice, S(stream)));
+  LS_CK(cudaMemcpyAsync(v_out, c.adam_v, n, cudaMemcpyDeviceToDevice, S(stream)));
+  *step_out = c.step;
+  return LS_OK;
+}
+
+int ls_set_opt_state(ls_ctx* h, const float* m, const float* v, int64_t step, void* stream) {
+  if (!h || !m || !v || step < 0) return fail(LS_ERR_ARG, "bad argument");
+  Ctx& c = h->c;
+  const size_t n = (size_t)c.n_params * sizeof(float);
+  LS_CK(cudaMemcpyAsync(c.adam_m, m, n, cudaMemcpyDeviceToDevice, S(stream)));
+  LS_CK(cudaMemcpyAsync(c.adam_v, v, n, cudaMemcpyDeviceToDevice, S(stream)));
+  c.step = step;
+  return LS_OK;
+}
+
+int ls_set_normalizer(ls_ctx* h, const float* mean, const float* stdv, void* stream) {
+  if (!h || !mean || !stdv) return fail(LS_ERR_ARG, "NULL argument");
+  Ctx& c = h->c;
+  LS_CK(cudaMemcpyAsync(c.mean, mean, (size_t)c.d * sizeof(float), cudaMemcpyDeviceToDevice, S(stream)));
+  LS_CK(cudaMemcpyAsync(c.stdv, stdv, (size_t)c.d * sizeof(float), cudaMemcpyDeviceToDevice, S(stream)));
+  c.have_norm = true;
+  return LS_OK;
+}
+
+int ls_snapshot_update(ls_ctx* h, int32_t n_inst, const float* inst_state, const uint64_t* keys,
+                       const int64_t* key_off, int64_t n_keys, int32_t mode, void* stream) {
+  if (!h) return fail(LS_ERR_ARG, "ctx is NULL");
+  Ctx& c = h->c;
+  if (n_inst < 1 || n_inst > c.cfg.max_instances) return fail(LS_ERR_ARG, "n_inst out of range");
+  if (c.cfg.d_inst > 0 && !inst_state) return fail(LS_ERR_ARG, "inst_state is NULL");
+  if (mode != LS_REPLACE && mode != LS_INSERT) return fail(LS_ERR_ARG, "bad mode");
+  if (keys && (!key_off || n_keys < 0)) return fail(LS_ERR_ARG, "keys need key_off and n_keys >= 0");
+  if (!keys && n_keys != 0) return fail(LS_ERR_ARG, "n_keys given without keys");
+  if (c.cfg.d_inst > 0)
+    LS_CK(cudaMemcpyAsync(c.inst_state, inst_state, (size_t)n_inst * c.cfg.d_inst * sizeof(float),
+                          cudaMemcpyDeviceToDevice, S(stream)));
+  if (keys) {
+    if (mode == LS_REPLACE) {
+      LS_CK(cudaMemsetAsync(c.tables, 0, (size_t)n_inst * c.slots * sizeof(uint64_t), S(stream)));
+      LS_CK(cudaMemsetAsync(c.table_count, 0, (size_t)n_inst * sizeof(int32_t), S(stream)));
+    }
+    LS_CK(traced(c, TR_INSERT, 1, S(stream), [&] {
+      return launch_table_insert(keys, key_off, n_inst, n_keys, c.tables, c.mask, c.slots,
+                                 c.table_count, c.cfg.max_keys_per_instance, c.d_err, S(stream));
+    }));
+  }
+  c.n_inst = n_inst;
+  return LS_OK;
+}
+
+int ls_hash_blocks(ls_ctx* h, int32_t n_seq, const int32_t* tok, const int64_t* tok_off,
+                   uint64_t* keys_out, const int64_t* key_off, void* stream) {
+  if (!h) return fail(LS_ERR_ARG, "ctx is NULL");
+  if (n_seq < 0) return fail(LS_ERR_ARG, "n_seq < 0");
+  if (n_seq == 0) return LS_OK;
+  if (!tok || !tok_off || !keys_out || !key_off) return fail(LS_ERR_ARG, "NULL argument");
+  LS_CK(traced(h->c, TR_HASH, 1, S(stream), [&] {
+    return launch_hash_blocks(n_seq, tok, tok_off, keys_out, key_off, S(stream));
+  }));
+  return LS_OK;
+}
+
+int ls_assemble_features(ls_ctx* h, int32_t n_req, const int64_t* tok_off, const int32_t* hits,
+                         const float* req_feats, float* x_out, void* stream) {
+  if (!h) return fail(LS_ERR_ARG, "ctx is NULL");
+  Ctx& c = h->c;
+  if (n_req < 0) return fail(LS_ERR_ARG, "n_req < 0");
+  if (n_req == 0) return LS_OK;
+  if (!tok_off || !hits || !x_out || (c.cfg.d_req > 0 && !req_feats))
+    return fail(LS_ERR_ARG, "NULL argument");
+  if (c.n_inst < 1) return fail(LS_ERR_STATE, "no snapshot");
+  if (!c.have_norm) return fail(LS_ERR_STATE, "normaliser not set");
+  LS_CK(traced(c, TR_ASSEMBLE, 1, S(stream), [&] {
+    return launch_assemble_features(n_req, c.n_inst, tok_off, hits, c.inst_state, c.cfg.d_inst,
+                                    req_feats, c.cfg.d_req, c.mean, c.stdv, x_out, S(stream));
+  }));
+  return LS_OK;
+}
+
+int ls_route_batch(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* tok_off,
+                   const float* req_feats, int32_t* choice, float* best, float* scores_opt,
+                   int32_t* hits_opt, uint64_t* weight_version_out, void* stream) {
+  if (!h) return fail(LS_ERR_ARG, "ctx is NULL");
+  Ctx& c = h->c;
+  if (n_req < 0 || n_req > c.cfg.max_requests) return fail(LS_ERR_ARG, "n_req out of range");
+  if (n_req > 0 && (!tok || !tok_off || !choice || !best || (c.cfg.d_req > 0 && !req_feats)))
+    return fail(LS_ERR_ARG, "NULL argument");
+  if (c.n_inst < 1) return fail(LS_ERR_STATE, "no snapshot");
+  if (!c.have_norm) return fail(LS_ERR_STATE, "normaliser not set");
+  cudaStream_t s = S(stream);
+  int b;
+  uint64_t v;
+  {
+    std::lock_guard<std::mutex> g(c.mu);
+    if (c.cur < 0) return fail(LS_ERR_STATE, "no weights published");
+    b = c.cur;
+    v = c.pub[b].version;
+    LS_CK(cudaStreamWaitEvent(s, c.pub_ready[b], 0));
+  }
+  if (weight_version_out) *weight_version_out = v;
+  if (n_req == 0) return LS_OK;
+  int32_t* hits = hits_opt ? hits_opt : c.hits;
+  float* scores = scores_opt ? scores_opt : c.scores;
+  LS_CK(traced(c, TR_PREFIX, 1, s, [&] {
+    return launch_prefix_match(n_req, tok, tok_off, c.tables, c.mask, c.slots, c.n_inst, hits, s);
+  }));
+  LS_CK(traced(c, TR_SCORE, 1, s, [&] {
+    return launch_score_simt(c.mlp, c.pub[b], n_req, c.n_inst, tok_off, hits, c.inst_state,
+                             c.cfg.d_inst, req_feats, c.cfg.d_req, c.mean, c.stdv, scores, s);
+  }));
+  LS_CK(traced(c, TR_ARGMIN, 1, s, [&] { return launch_argmin(n_req, c.n_inst, scores, choice, best, s); }));
+  {
+    std::lock_guard<std::mutex> g(c.mu);
+    LS_CK(cudaEventRecord(c.route_done[b], s));
+  }
+  return LS_OK;
+}
+
+int ls_log_samples(ls_ctx* h, int32_t n, const float* feats, const float* ttft, void* stream) {
+  if (!h) return fail(LS_ERR_ARG, "ctx is NULL");
+  Ctx& c = h->c;
+  if (n < 0) return fail(LS_ERR_ARG, "n < 0");
+  if (n == 0) return LS_OK;
+  if (!feats || !ttft) return fail(LS_ERR_ARG, "NULL argument");
+  LS_CK(traced(c, TR_RING, 1, S(stream), [&] {
+    return launch_ring_append(n, c.d, feats, ttft, c.ring_x, c.ring_y, c.ring_count,
+                              c.cfg.ring_capacity, S(stream));
+  }));
+  std::lock_guard<std::mutex> g(c.mu);
+  c.ring_count += n;
+  return LS_OK;
+}
+
+int ls_train_step(ls_ctx* h, int32_t batch, const int32_t* idx, int32_t opt, float lr, float* loss_out,
+                  void* stream) {
+  if (!h) return fail(LS_ERR_ARG, "ctx is NULL");
+  Ctx& c = h->c;
+  if (batch < 1 || batch > c.cfg.max_train_batch) return fail(LS_ERR_ARG, "batch out of range");
+  if (opt != LS_SGD && opt != LS_ADAM) return fail(LS_ERR_ARG, "bad optimiser");
+  if (!std::isfinite(lr)) return fail(LS_ERR_ARG, "lr is not finite");
+  if (!c.have_params) return fail(LS_ERR_STATE, "parameters not set");
+  if (!c.have_norm) return fail(LS_ERR_STATE, "normaliser not set");
+  if (c.ring_count < 1) return fail(LS_ERR_STATE, "sample ring is empty");
+  LS_CK(run_train_step(c, batch, idx, opt, lr, loss_out, S(stream)));
+  c.step += 1;
+  return LS_OK;
+}
+
+int ls_publish(ls_ctx* h, void* stream) {
+  if (!h) return fail(LS_ERR_ARG, "ctx is NULL");
+  Ctx& c = h->c;
+  if (!c.have_params) return fail(LS_ERR_STATE, "parameters not set");
+  cudaStream_t s = S(stream);
+  std::lock_guard<std::mutex> g(c.mu);
+  const int target = c.cur < 0 ? 0 : 1 - c.cur;
+  LS_CK(cudaStreamWaitEvent(s, c.route_done[target], 0));
+  LS_CK(traced(c, TR_PUBLISH, c.mlp.n_layers, s, [&] { return launch_publish(c.mlp, c.master, c.pub[target], s); }));
+  LS_CK(cudaEventRecord(c.pub_ready[target], s));
+  c.version += 1;
+  c.pub[target].version = c.version;
+  c.cur = target;
+  return LS_OK;
+}
+
+int ls_trace_enable(ls_ctx* h, int32_t on) {
+  if (!h) return fail(LS_ERR_ARG, "ctx is NULL");
+  Tracer& t = h->c.tracer;
+  std::lock_guard<std::mutex> g(t.mu);
+  if (on && !t.ready) {
+    for (int i = 0; i < Tracer::kPool; ++i) LS_CK(cudaEventCreate(&t.ev[i]));
+    t.ready = true;
+  }
+  t.on = on != 0;
+  return LS_OK;
+}
+
+int ls_trace_read(ls_ctx* h, ls_trace_entry* out, int32_t max_entries, int32_t* n_out) {
+  if (!h || (!out && max_entries > 0) || max_entries < 0 || !n_out) return fail(LS_ERR_ARG, "bad argument");
+  Tracer& t = h->c.tracer;
+  LS_CK(cudaDeviceSynchronize());
+  std::lock_guard<std::mutex> g(t.mu);
+  for (const auto& p : t.pend) {
+    float ms = 0.0f;
+    LS_CK(cudaEventElapsedTime(&ms, t.ev[p.a], t.ev[p.a + 1]));
+    t.ms[p.id] += ms;
+  }
+  t.pend.clear();
+  t.used = 0;
+  int n = 0;
+  for (int id = 0; id < TR_COUNT; ++id) {
+    if (t.launches[id] == 0) continue;
+    if (n < max_entries) {
+      std::memset(out[n].name, 0, sizeof(out[n].name));
+      std::strncpy(out[n].name, kTraceNames[id], sizeof(out[n].name) - 1);
+      out[n].launches = t.launches[id];
+      out[n].total_ms = t.ms[id];
+    }
+    ++n;
+    t.launches[id] = 0;
+    t.ms[id] = 0.0;
+  }
+  *n_out = n < max_entries ? n : max_entries;
+  t.dropped = 0;
+  return LS_OK;
+}
+
+}  // extern "C"

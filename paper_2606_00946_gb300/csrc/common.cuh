@@ -1,0 +1,212 @@
+// Internal declarations of the Lodestar GB300 library: context layout, device
+// helpers shared by the kernels, and the launchers each .cu file provides.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <cstdint>
+#include <mutex>
+#include <vector>
+
+#include "lodestar.h"
+
+namespace ls {
+
+constexpr uint64_t kG = 0x9E3779B97F4A7C15ull;  // floor(2^64 / golden ratio)
+constexpr int kBlockTok = LS_BLOCK_TOKENS;
+constexpr int kPair = LS_PAIR_FEATURES;
+
+// ---------------------------------------------------------------------------
+// predictor layout
+// ---------------------------------------------------------------------------
+struct MlpDesc {
+  int n_layers;
+  int w[LS_MAX_LAYERS + 1];
+  int64_t woff[LS_MAX_LAYERS];   // W_l offset in the flat parameter vector
+  int64_t boff[LS_MAX_LAYERS];   // b_l offset
+  int64_t wtoff[LS_MAX_LAYERS];  // offset of the transposed copy W_l^T [in, out]
+  int bf16;                      // 1: bf16 operands (weights, layer input, hidden activations)
+  int max_width;
+};
+
+// One published weight version (Sec. 4.3.1 P2: the routing side reads a
+// version that training never writes).
+struct Published {
+  float* params = nullptr;  // flat, same layout as the master; weights rounded in bf16 mode
+  float* wt = nullptr;      // per-layer transposed weights [in, out]
+  uint64_t version = 0;
+};
+
+// Kernel-level tracing: when enabled, every launch is bracketed by CUDA events
+// recorded on the launching stream; ls_trace_read() sums the elapsed times.
+enum TraceId {
+  TR_HASH, TR_INSERT, TR_PREFIX, TR_SCORE, TR_ARGMIN, TR_ASSEMBLE, TR_RING, TR_PUBLISH,
+  TR_GATHER, TR_GEMM_FWD, TR_LOSS, TR_GEMM_DW, TR_REDUCE, TR_COLSUM, TR_GEMM_DX, TR_OPT,
+  TR_MEMSET, TR_COUNT
+};
+extern const char* const kTraceNames[TR_COUNT];
+
+struct Tracer {
+  static constexpr int kPool = 8192;
+  bool on = false;
+  bool ready = false;
+  cudaEvent_t ev[kPool];
+  int used = 0;
+  struct Pending { int id, a, launches; };
+  std::vector<Pending> pend;
+  int64_t launches[TR_COUNT] = {};
+  double ms[TR_COUNT] = {};
+  int64_t dropped = 0;
+  std::mutex mu;
+
+  int begin(cudaStream_t s) {
+    if (!on) return -1;
+    std::lock_guard<std::mutex> g(mu);
+    if (used + 2 > kPool) return -2;
+    const int t = used;
+    used += 2;
+    cudaEventRecord(ev[t], s);
+    return t;
+  }
+  void end(int t, int id, int n, cudaStream_t s) {
+    if (t == -1) return;
+    std::lock_guard<std::mutex> g(mu);
+    launches[id] += n;
+    if (t < 0) { ++dropped; return; }
+    cudaEventRecord(ev[t + 1], s);
+    pend.push_back({id, t, n});
+  }
+};
+
+struct Ctx {
+  ls_config cfg{};
+  MlpDesc mlp{};
+  int d = 0;
+  int64_t n_params = 0;
+  int64_t wt_total = 0;
+
+  // snapshot (Sec. 4.2): instance state rows and per-instance key tables
+  int n_inst = 0;
+  int64_t slots = 0;       // per-instance table slots (power of two)
+  uint32_t mask = 0;
+  uint64_t* tables = nullptr;
+  int32_t* table_count = nullptr;
+  float* inst_state = nullptr;
+  float* mean = nullptr;
+  float* stdv = nullptr;
+  bool have_norm = false;
+
+  // parameters and optimiser state
+  float* master = nullptr;
+  float* adam_m = nullptr;
+  float* adam_v = nullptr;
+  int64_t step = 0;
+  bool have_params = false;
+
+  // publish / swap
+  Published pub[2];
+  int cur = -1;
+  uint64_t version = 0;
+  cudaEvent_t pub_ready[2] = {nullptr, nullptr};
+  cudaEvent_t route_done[2] = {nullptr, nullptr};
+
+  // sample ring (Sec. 4.3.2)
+  float* ring_x = nullptr;
+  float* ring_y = nullptr;
+  int64_t ring_count = 0;
+
+  // route scratch
+  int32_t* hits = nullptr;    // [max_requests, max_instances]
+  float* scores = nullptr;    // [max_requests, max_instances]
+
+  // train scratch
+  float* tx = nullptr;        // activations a_0..a_{L-1}, [B, sum w[0..L-1]]
+  float* tz = nullptr;        // pre-activations z_1..z_L, [B, sum w[1..L]]
+  float* ty = nullptr;        // targets [B]
+  float* dz0 = nullptr;       // [B, max_width]
+  float* dz1 = nullptr;
+  float* grad = nullptr;      // [n_params]
+  float* gpart = nullptr;     // split-K partials
+  int64_t gpart_floats = 0;
+  float* loss_tmp = nullptr;  // [1]
+
+  int* d_err = nullptr;       // first device-side error (0 = none)
+  int sms = 148;              // SM count of the context's device
+  std::mutex mu;
+  Tracer tracer;
+};
+
+template <class F>
+cudaError_t traced(Ctx& c, int id, int n_launch, cudaStream_t s, F&& f) {
+  const int t = c.tracer.begin(s);
+  const cudaError_t e = f();
+  c.tracer.end(t, id, n_launch, s);
+  return e;
+}
+
+// ---------------------------------------------------------------------------
+// device helpers
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float round_bf16(float x) {
+  return __bfloat162float(__float2bfloat16_rn(x));
+}
+
+__device__ __forceinline__ void latch_error(int* err, int code) {
+  atomicCAS(err, 0, code);
+}
+
+// Raw feature k of pair (request with prompt length L and hit length h,
+// instance row inst, request extras req):  [L, h, 16h, 16h/L, L-16h,
+// ceil(L/16)-h || inst[0..d_inst) || req[0..d_req)]  (Sec. 4.1 Features).
+__device__ __forceinline__ float raw_feature(int k, int64_t L, int h, const float* inst,
+                                            int d_inst, const float* req) {
+  switch (k) {
+    case 0: return (float)L;
+    case 1: return (float)h;
+    case 2: return (float)((int64_t)kBlockTok * h);
+    case 3: return L > 0 ? (float)((int64_t)kBlockTok * h) / (float)L : 0.0f;
+    case 4: return (float)(L - (int64_t)kBlockTok * h);
+    case 5: return (float)((L + kBlockTok - 1) / kBlockTok - h);
+    default: break;
+  }
+  k -= kPair;
+  return k < d_inst ? inst[k] : req[k - d_inst];
+}
+
+// Per-feature z-score (Algorithm 4, Normalize); std below 1e-12 -> 1.
+__device__ __forceinline__ float zscore(float x, float mu, float sd) {
+  float s = sd < 1e-12f ? 1.0f : sd;
+  return (x - mu) / s;
+}
+
+// ---------------------------------------------------------------------------
+// launchers (each returns the launch status)
+// ---------------------------------------------------------------------------
+cudaError_t launch_hash_blocks(int n_seq, const int32_t* tok, const int64_t* tok_off,
+                               uint64_t* keys_out, const int64_t* key_off, cudaStream_t s);
+cudaError_t launch_table_insert(const uint64_t* keys, const int64_t* key_off, int n_inst,
+                                int64_t n_keys, uint64_t* tables, uint32_t mask, int64_t slots,
+                                int32_t* counts, int64_t max_keys, int* err, cudaStream_t s);
+cudaError_t launch_prefix_match(int n_req, const int32_t* tok, const int64_t* tok_off,
+                                const uint64_t* tables, uint32_t mask, int64_t slots, int n_inst,
+                                int32_t* hits, cudaStream_t s);
+
+cudaError_t launch_assemble_features(int n_req, int n_inst, const int64_t* tok_off,
+                                     const int32_t* hits, const float* inst_state, int d_inst,
+                                     const float* req_feats, int d_req, const float* mean,
+                                     const float* stdv, float* x_out, cudaStream_t s);
+cudaError_t launch_score_simt(const MlpDesc& mlp, const Published& pub, int n_req, int n_inst,
+                              const int64_t* tok_off, const int32_t* hits, const float* inst_state,
+                              int d_inst, const float* req_feats, int d_req, const float* mean,
+                              const float* stdv, float* scores, cudaStream_t s);
+cudaError_t launch_argmin(int n_req, int n_inst, const float* scores, int32_t* choice,
+                          float* best, cudaStream_t s);
+
+cudaError_t launch_publish(const MlpDesc& mlp, const float* master, Published& pub,
+                           cudaStream_t s);
+cudaError_t launch_ring_append(int n, int d, const float* x, const float* y, float* ring_x,
+                               float* ring_y, int64_t count, int64_t capacity, cudaStream_t s);
+cudaError_t run_train_step(Ctx& c, int batch, const int32_t* idx, int opt, float lr,
+                           float* loss_out, cudaStream_t s);
+
+}  // namespace ls

@@ -1,0 +1,298 @@
+// Prefix tracker kernels: block hashing, table inserts, and the fused
+// hash + probe that yields the prefix hit length of every (request, instance)
+// pair (Sec. 2: prefix reuse is strictly sequential; Sec. 4.1 Features (2)).
+//
+// Block key definition (this library's reading; the paper only says that
+// gateways index cached prefixes with radix trees or hash tables, Sec. 2):
+//   mix64  = SplitMix64 output finaliser;  G = 0x9E3779B97F4A7C15
+//   c_b    = mix64( XOR_{j<8} mix64(w_{b,j} + (j+1) G) )       (content)
+//   s_{-1} = G,  s_b = s_{b-1} * G + c_b  (mod 2^64)            (prefix state)
+//   key_b  = mix64(s_b), 0 mapped to 1                           (table key)
+// The prefix state is a linear recurrence, so a CTA computes the keys of 256
+// consecutive blocks with one parallel scan instead of a serial chain.
+#include "common.cuh"
+
+namespace ls {
+namespace {
+
+constexpr int kThreads = 256;           // threads per CTA = blocks per chunk
+constexpr int kWarps = kThreads / 32;
+constexpr unsigned kFull = 0xffffffffu;
+
+__host__ __device__ constexpr uint64_t gpow(uint64_t e) {
+  uint64_t r = 1, b = kG;
+  while (e) {
+    if (e & 1) r *= b;
+    b *= b;
+    e >>= 1;
+  }
+  return r;
+}
+
+__device__ __forceinline__ uint64_t mix64(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+__device__ __forceinline__ uint64_t word_mix(uint32_t lo, uint32_t hi, int j) {
+  uint64_t w = (uint64_t)lo | ((uint64_t)hi << 32);
+  return mix64(w + (uint64_t)(j + 1) * kG);
+}
+
+// Content hash of the 16 tokens at p.  `aligned`: p is 16-byte aligned.
+__device__ __forceinline__ uint64_t block_content(const int32_t* p, bool aligned) {
+  uint64_t acc = 0;
+  if (aligned) {
+    const int4* q = reinterpret_cast<const int4*>(p);
+#pragma unroll
+    for (int v = 0; v < 4; ++v) {
+      int4 t = __ldg(q + v);
+      acc ^= word_mix((uint32_t)t.x, (uint32_t)t.y, 2 * v);
+      acc ^= word_mix((uint32_t)t.z, (uint32_t)t.w, 2 * v + 1);
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      acc ^= word_mix((uint32_t)__ldg(p + 2 * j), (uint32_t)__ldg(p + 2 * j + 1), j);
+  }
+  return mix64(acc);
+}
+
+// Prefix state after this thread's block, for a chunk whose first block
+// follows state s_in.  Thread t holds content c (0 for threads past the last
+// block: they come after every real block, so they change nothing).
+// Inclusive scan of B_t = sum_{j<=t} G^(t-j) c_j, state_t = G^(t+1) s_in + B_t.
+__device__ __forceinline__ uint64_t chain_scan(uint64_t c, uint64_t s_in, uint64_t* wtot,
+                                               uint64_t* wpre) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  uint64_t B = c;
+#pragma unroll
+  for (int k = 0; k < 5; ++k) {
+    const int off = 1 << k;
+    uint64_t o = __shfl_up_sync(kFull, B, off);
+    if (lane >= off) B = gpow(off) * o + B;  // left span times G^(right span)
+  }
+  if (lane == 31) wtot[warp] = B;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    uint64_t e = s_in;
+    for (int w = 0; w < kWarps; ++w) {
+      wpre[w] = e;
+      e = gpow(32) * e + wtot[w];
+    }
+  }
+  __syncthreads();
+  uint64_t gl = 1, base = kG;  // G^(lane+1)
+  for (unsigned e = (unsigned)lane + 1; e; e >>= 1) {
+    if (e & 1) gl *= base;
+    base *= base;
+  }
+  return gl * wpre[warp] + B;
+}
+
+__device__ __forceinline__ uint64_t key_of(uint64_t state) {
+  uint64_t k = mix64(state);
+  return k ? k : 1ull;
+}
+
+// Open-addressing membership: linear probing from key & mask, 0 = empty slot.
+__device__ __forceinline__ bool table_contains(const uint64_t* __restrict__ tab, uint32_t mask,
+                                               uint64_t key) {
+  uint32_t s = (uint32_t)key & mask;
+  for (uint32_t n = 0; n <= mask; ++n) {
+    uint64_t v = __ldg(reinterpret_cast<const unsigned long long*>(tab) + s);
+    if (v == key) return true;
+    if (v == 0) return false;
+    s = (s + 1) & mask;
+  }
+  return false;
+}
+
+// One CTA per sequence: keys of every full block.
+__global__ void __launch_bounds__(kThreads) k_hash_blocks(int n_seq, const int32_t* __restrict__ tok,
+                                                          const int64_t* __restrict__ tok_off,
+                                                          uint64_t* __restrict__ keys_out,
+                                                          const int64_t* __restrict__ key_off) {
+  __shared__ uint64_t wtot[kWarps], wpre[kWarps], carry;
+  for (int s = blockIdx.x; s < n_seq; s += gridDim.x) {
+    const int64_t t0 = tok_off[s];
+    const int64_t nb = (tok_off[s + 1] - t0) / kBlockTok;
+    const int32_t* base = tok + t0;
+    const bool aligned = ((reinterpret_cast<uintptr_t>(base) & 15) == 0);
+    uint64_t* out = keys_out + key_off[s];
+    if (threadIdx.x == 0) carry = kG;
+    __syncthreads();
+    for (int64_t c0 = 0; c0 < nb; c0 += kThreads) {
+      const int n = (int)(nb - c0 < kThreads ? nb - c0 : kThreads);
+      const int t = threadIdx.x;
+      const uint64_t s_in = carry;
+      uint64_t c = t < n ? block_content(base + (c0 + t) * kBlockTok, aligned) : 0ull;
+      uint64_t st = chain_scan(c, s_in, wtot, wpre);
+      if (t < n) out[c0 + t] = key_of(st);
+      if (t == n - 1) carry = st;
+      __syncthreads();
+    }
+    __syncthreads();
+  }
+}
+
+// Insert keys into per-instance tables.  Thread per key; the owning instance
+// is found by binary search in key_off.  A table holding more than max_keys
+// distinct keys, or a probe sequence that visits every slot, latches
+// LS_ERR_TABLE_FULL (the loop is bounded by the table size).
+__global__ void k_table_insert(const uint64_t* __restrict__ keys, const int64_t* __restrict__ key_off,
+                               int n_inst, int64_t n_keys, uint64_t* tables, uint32_t mask,
+                               int64_t slots, int32_t* counts, int64_t max_keys, int* err) {
+  for (int64_t k = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; k < n_keys;
+       k += (int64_t)gridDim.x * blockDim.x) {
+    int lo = 0, hi = n_inst - 1;
+    while (lo < hi) {
+      int mid = (lo + hi + 1) >> 1;
+      if (key_off[mid] <= k) lo = mid; else hi = mid - 1;
+    }
+    uint64_t key = keys[k];
+    if (key == 0) key = 1;
+    unsigned long long* tab = reinterpret_cast<unsigned long long*>(tables + (int64_t)lo * slots);
+    uint32_t s = (uint32_t)key & mask;
+    bool done = false;
+    for (uint32_t n = 0; n <= mask; ++n) {
+      unsigned long long prev = atomicCAS(tab + s, 0ull, (unsigned long long)key);
+      if (prev == 0ull) {
+        int cnt = atomicAdd(counts + lo, 1);
+        if (cnt >= max_keys) latch_error(err, LS_ERR_TABLE_FULL);
+        done = true;
+        break;
+      }
+      if (prev == key) { done = true; break; }
+      s = (s + 1) & mask;
+    }
+    if (!done) latch_error(err, LS_ERR_TABLE_FULL);
+  }
+}
+
+// Fused hash + probe.  One CTA per request (grid-stride).  The request's
+// blocks are hashed 256 at a time into shared memory; every instance still
+// matching probes them, and hashing stops as soon as no instance matches.
+//  - block 0 is screened with one thread per instance (most pairs end there);
+//  - an instance still matching is then walked by one warp, 32 blocks per
+//    round (32 independent table lookups in flight), ballot -> first miss.
+__global__ void __launch_bounds__(kThreads) k_prefix_match(int n_req, const int32_t* __restrict__ tok,
+                                                           const int64_t* __restrict__ tok_off,
+                                                           const uint64_t* __restrict__ tables,
+                                                           uint32_t mask, int64_t slots, int n_inst,
+                                                           int32_t* __restrict__ hits) {
+  __shared__ uint64_t keys[kThreads];
+  __shared__ uint64_t wtot[kWarps], wpre[kWarps], carry;
+  __shared__ int n_alive;
+  extern __shared__ int32_t dyn[];
+  int32_t* hv = dyn;                 // [n_inst] hit length so far
+  int32_t* dead = dyn + n_inst;      // [n_inst] 1 once the first miss is found
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+
+  for (int r = blockIdx.x; r < n_req; r += gridDim.x) {
+    const int64_t t0 = tok_off[r];
+    const int64_t nb = (tok_off[r + 1] - t0) / kBlockTok;
+    const int32_t* base = tok + t0;
+    const bool aligned = ((reinterpret_cast<uintptr_t>(base) & 15) == 0);
+    for (int i = threadIdx.x; i < n_inst; i += kThreads) { hv[i] = 0; dead[i] = 0; }
+    if (threadIdx.x == 0) { carry = kG; n_alive = n_inst; }
+    __syncthreads();
+
+    for (int64_t c0 = 0; c0 < nb; c0 += kThreads) {
+      if (n_alive == 0) break;  // uniform: read after a barrier
+      const int n = (int)(nb - c0 < kThreads ? nb - c0 : kThreads);
+      const int t = threadIdx.x;
+      const uint64_t s_in = carry;
+      uint64_t c = t < n ? block_content(base + (c0 + t) * kBlockTok, aligned) : 0ull;
+      uint64_t st = chain_scan(c, s_in, wtot, wpre);
+      if (t < n) keys[t] = key_of(st);
+      if (t == n - 1) carry = st;
+      __syncthreads();
+
+      int start = 0;
+      if (c0 == 0) {
+        for (int i = threadIdx.x; i < n_inst; i += kThreads) {
+          const bool hit = table_contains(tables + (int64_t)i * slots, mask, keys[0]);
+          hv[i] = hit ? 1 : 0;
+          dead[i] = hit ? 0 : 1;
+        }
+        __syncthreads();
+        start = 1;
+      }
+      for (int i = warp; i < n_inst; i += kWarps) {
+        if (dead[i]) continue;
+        const uint64_t* tab = tables + (int64_t)i * slots;
+        bool found = false;
+        for (int p = start; p < n; p += 32) {
+          const int b = p + lane;
+          const bool miss = b < n && !table_contains(tab, mask, keys[b]);
+          const unsigned bal = __ballot_sync(kFull, miss);
+          if (bal) {
+            if (lane == 0) { hv[i] = (int32_t)(c0 + p + __ffs(bal) - 1); dead[i] = 1; }
+            found = true;
+            break;
+          }
+        }
+        if (!found && lane == 0) hv[i] = (int32_t)(c0 + n);
+      }
+      if (threadIdx.x == 0) n_alive = 0;
+      __syncthreads();
+      int alive = 0;
+      for (int i = threadIdx.x; i < n_inst; i += kThreads) alive += dead[i] ? 0 : 1;
+      if (alive) atomicAdd(&n_alive, alive);
+      __syncthreads();
+    }
+    for (int i = threadIdx.x; i < n_inst; i += kThreads) hits[(int64_t)r * n_inst + i] = hv[i];
+    __syncthreads();
+  }
+}
+
+int grid_for(int64_t n) {
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  int64_t g = n;
+  const int64_t cap = (int64_t)sms * 16;
+  return (int)(g < 1 ? 1 : (g > cap ? cap : g));
+}
+
+}  // namespace
+
+cudaError_t launch_hash_blocks(int n_seq, const int32_t* tok, const int64_t* tok_off,
+                               uint64_t* keys_out, const int64_t* key_off, cudaStream_t s) {
+  if (n_seq <= 0) return cudaSuccess;
+  k_hash_blocks<<<grid_for(n_seq), kThreads, 0, s>>>(n_seq, tok, tok_off, keys_out, key_off);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_table_insert(const uint64_t* keys, const int64_t* key_off, int n_inst,
+                                int64_t n_keys, uint64_t* tables, uint32_t mask, int64_t slots,
+                                int32_t* counts, int64_t max_keys, int* err, cudaStream_t s) {
+  if (n_keys <= 0 || n_inst <= 0) return cudaSuccess;
+  int64_t blocks = (n_keys + 255) / 256;
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (blocks > (int64_t)sms * 32) blocks = (int64_t)sms * 32;
+  k_table_insert<<<(int)blocks, 256, 0, s>>>(keys, key_off, n_inst, n_keys, tables, mask, slots,
+                                             counts, max_keys, err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_prefix_match(int n_req, const int32_t* tok, const int64_t* tok_off,
+                                const uint64_t* tables, uint32_t mask, int64_t slots, int n_inst,
+                                int32_t* hits, cudaStream_t s) {
+  if (n_req <= 0) return cudaSuccess;
+  const size_t smem = (size_t)n_inst * 2 * sizeof(int32_t);
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(k_prefix_match, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+  }
+  k_prefix_match<<<grid_for(n_req), kThreads, smem, s>>>(n_req, tok, tok_off, tables, mask, slots,
+                                                         n_inst, hits);
+  return cudaGetLastError();
+}
+
+}  // namespace ls

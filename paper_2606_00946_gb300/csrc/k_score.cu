@@ -1,0 +1,253 @@
+// Scoring kernels on CUDA cores: feature assembly (Sec. 4.1 Features,
+// Algorithm 4 Normalize), the reward-model forward pass for small or fp32
+// predictors (Sec. 4.1 Model architecture), the greedy argmin selector
+// (Algorithm 4, argmax reward = argmin predicted TTFT), weight publishing and
+// the sample ring.
+#include "common.cuh"
+
+namespace ls {
+namespace {
+
+constexpr unsigned kFull = 0xffffffffu;
+
+// (a, i) precedes (b, j) in the order (score, index): NaN after every number,
+// -0 == +0, ties to the lower index.
+__device__ __forceinline__ bool precedes(float a, int i, float b, int j) {
+  const bool an = isnan(a), bn = isnan(b);
+  if (an != bn) return bn;
+  if (!an && a != b) return a < b;
+  return i < j;
+}
+
+__device__ __forceinline__ float norm_feature(int k, int64_t L, int h, const float* inst,
+                                             int d_inst, const float* req, const float* mean,
+                                             const float* stdv) {
+  return zscore(raw_feature(k, L, h, inst, d_inst, req), mean[k], stdv[k]);
+}
+
+__global__ void k_assemble(int n_req, int n_inst, const int64_t* __restrict__ tok_off,
+                           const int32_t* __restrict__ hits, const float* __restrict__ inst_state,
+                           int d_inst, const float* __restrict__ req_feats, int d_req,
+                           const float* __restrict__ mean, const float* __restrict__ stdv,
+                           float* __restrict__ x_out) {
+  const int d = kPair + d_inst + d_req;
+  const int64_t total = (int64_t)n_req * n_inst * d;
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t row = e / d;
+    const int k = (int)(e - row * d);
+    const int r = (int)(row / n_inst), i = (int)(row - (int64_t)r * n_inst);
+    const int64_t L = tok_off[r + 1] - tok_off[r];
+    x_out[e] = norm_feature(k, L, hits[row], inst_state + (int64_t)i * d_inst, d_inst,
+                            req_feats + (int64_t)r * d_req, mean, stdv);
+  }
+}
+
+// Forward pass of a tile of TR pair rows (row = r * n_inst + i) held in shared
+// memory.  Hidden layer: thread o computes output column o for all TR rows
+// from the transposed weights W^T [in, out] (coalesced across threads);
+// output layer (width 1): one warp per row, lanes split the dot product.
+template <int TR>
+__global__ void __launch_bounds__(256) k_score_simt(MlpDesc mlp, const float* __restrict__ pp,
+                                                    const float* __restrict__ wt, int n_req,
+                                                    int n_inst, const int64_t* __restrict__ tok_off,
+                                                    const int32_t* __restrict__ hits,
+                                                    const float* __restrict__ inst_state, int d_inst,
+                                                    const float* __restrict__ req_feats, int d_req,
+                                                    const float* __restrict__ mean,
+                                                    const float* __restrict__ stdv,
+                                                    float* __restrict__ scores) {
+  extern __shared__ float smem[];
+  const int H = mlp.max_width;
+  float* a = smem;
+  float* b = smem + TR * H;
+  const int d = mlp.w[0];
+  const int64_t rows = (int64_t)n_req * n_inst;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+
+  for (int64_t row0 = (int64_t)blockIdx.x * TR; row0 < rows; row0 += (int64_t)gridDim.x * TR) {
+    for (int e = threadIdx.x; e < TR * d; e += blockDim.x) {
+      const int rr = e / d, k = e - rr * d;
+      const int64_t g = row0 + rr;
+      float v = 0.0f;
+      if (g < rows) {
+        const int r = (int)(g / n_inst), i = (int)(g - (int64_t)r * n_inst);
+        const int64_t L = tok_off[r + 1] - tok_off[r];
+        v = norm_feature(k, L, hits[g], inst_state + (int64_t)i * d_inst, d_inst,
+                         req_feats + (int64_t)r * d_req, mean, stdv);
+        if (mlp.bf16) v = round_bf16(v);
+      }
+      a[rr * d + k] = v;
+    }
+    __syncthreads();
+    for (int l = 0; l < mlp.n_layers; ++l) {
+      const int in = mlp.w[l], out = mlp.w[l + 1];
+      const float* W = wt + mlp.wtoff[l];
+      const float* bias = pp + mlp.boff[l];
+      if (l == mlp.n_layers - 1) {  // output layer, width 1
+        for (int rr = warp; rr < TR; rr += blockDim.x / 32) {
+          float s = 0.0f;
+          for (int k = lane; k < in; k += 32) s = fmaf(a[rr * in + k], W[k], s);
+#pragma unroll
+          for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(kFull, s, o);
+          const int64_t g = row0 + rr;
+          if (lane == 0 && g < rows) scores[g] = s + bias[0];
+        }
+      } else {
+        for (int o = threadIdx.x; o < out; o += blockDim.x) {
+          float acc[TR];
+#pragma unroll
+          for (int rr = 0; rr < TR; ++rr) acc[rr] = 0.0f;
+          for (int k = 0; k < in; ++k) {
+            const float wv = W[(int64_t)k * out + o];
+#pragma unroll
+            for (int rr = 0; rr < TR; ++rr) acc[rr] = fmaf(a[rr * in + k], wv, acc[rr]);
+          }
+          const float bo = bias[o];
+#pragma unroll
+          for (int rr = 0; rr < TR; ++rr) {
+            float z = acc[rr] + bo;
+            z = z > 0.0f ? z : 0.0f;
+            b[rr * out + o] = mlp.bf16 ? round_bf16(z) : z;
+          }
+        }
+      }
+      __syncthreads();
+      float* t = a; a = b; b = t;
+    }
+  }
+}
+
+// One warp per request: lexicographic (score, index) minimum over instances.
+__global__ void k_argmin(int n_req, int n_inst, const float* __restrict__ scores,
+                         int32_t* __restrict__ choice, float* __restrict__ best) {
+  const int lane = threadIdx.x & 31;
+  const int64_t r = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  if (r >= n_req) return;
+  const float* s = scores + r * n_inst;
+  float bv = 0.0f;
+  int bi = -1;
+  for (int i = lane; i < n_inst; i += 32) {
+    const float v = s[i];
+    if (bi < 0 || precedes(v, i, bv, bi)) { bv = v; bi = i; }
+  }
+#pragma unroll
+  for (int o = 16; o; o >>= 1) {
+    const float ov = __shfl_xor_sync(kFull, bv, o);
+    const int oi = __shfl_xor_sync(kFull, bi, o);
+    if (oi >= 0 && (bi < 0 || precedes(ov, oi, bv, bi))) { bv = ov; bi = oi; }
+  }
+  if (lane == 0) { choice[r] = bi; best[r] = bv; }
+}
+
+// Publish layer l: rounded weights (bf16 mode), biases, and the transposed copy.
+__global__ void k_publish_layer(const float* __restrict__ W, const float* __restrict__ bsrc,
+                                int out, int in, int bf16, float* __restrict__ Wdst,
+                                float* __restrict__ bdst, float* __restrict__ Wt) {
+  const int64_t n = (int64_t)out * in;
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n + out;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    if (e < n) {
+      const int o = (int)(e / in), k = (int)(e - (int64_t)o * in);
+      const float v = bf16 ? round_bf16(W[e]) : W[e];
+      Wdst[e] = v;
+      Wt[(int64_t)k * out + o] = v;
+    } else {
+      bdst[e - n] = bsrc[e - n];
+    }
+  }
+}
+
+// Record j of the batch -> slot (count + j) mod capacity.  When a batch is
+// longer than the ring only its last `capacity` records are kept.
+__global__ void k_ring_append(int n, int d, const float* __restrict__ x, const float* __restrict__ y,
+                              float* __restrict__ ring_x, float* __restrict__ ring_y, int64_t count,
+                              int64_t capacity) {
+  const int64_t first = n > capacity ? n - capacity : 0;
+  const int64_t total = (int64_t)(n - first) * (d + 1);
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t j = first + e / (d + 1);
+    const int k = (int)(e % (d + 1));
+    const int64_t slot = (count + j) % capacity;
+    if (k < d) ring_x[slot * d + k] = x[j * d + k];
+    else ring_y[slot] = y[j];
+  }
+}
+
+int sm_count() {
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  return sms;
+}
+
+int grid_1d(int64_t n, int threads, int per_sm = 8) {
+  int64_t g = (n + threads - 1) / threads;
+  const int64_t cap = (int64_t)sm_count() * per_sm;
+  return (int)(g < 1 ? 1 : (g > cap ? cap : g));
+}
+
+}  // namespace
+
+cudaError_t launch_assemble_features(int n_req, int n_inst, const int64_t* tok_off,
+                                     const int32_t* hits, const float* inst_state, int d_inst,
+                                     const float* req_feats, int d_req, const float* mean,
+                                     const float* stdv, float* x_out, cudaStream_t s) {
+  const int64_t total = (int64_t)n_req * n_inst * (kPair + d_inst + d_req);
+  if (total <= 0) return cudaSuccess;
+  k_assemble<<<grid_1d(total, 256), 256, 0, s>>>(n_req, n_inst, tok_off, hits, inst_state, d_inst,
+                                                req_feats, d_req, mean, stdv, x_out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_score_simt(const MlpDesc& mlp, const Published& pub, int n_req, int n_inst,
+                              const int64_t* tok_off, const int32_t* hits, const float* inst_state,
+                              int d_inst, const float* req_feats, int d_req, const float* mean,
+                              const float* stdv, float* scores, cudaStream_t s) {
+  constexpr int TR = 16;
+  const int64_t rows = (int64_t)n_req * n_inst;
+  if (rows <= 0) return cudaSuccess;
+  const size_t smem = (size_t)2 * TR * mlp.max_width * sizeof(float);
+  cudaError_t e = cudaFuncSetAttribute(k_score_simt<TR>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem);
+  if (e != cudaSuccess) return e;
+  int64_t tiles = (rows + TR - 1) / TR;
+  const int64_t cap = (int64_t)sm_count() * 8;
+  const int grid = (int)(tiles > cap ? cap : tiles);
+  k_score_simt<TR><<<grid, 256, smem, s>>>(mlp, pub.params, pub.wt, n_req, n_inst, tok_off, hits,
+                                           inst_state, d_inst, req_feats, d_req, mean, stdv, scores);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_argmin(int n_req, int n_inst, const float* scores, int32_t* choice, float* best,
+                          cudaStream_t s) {
+  if (n_req <= 0) return cudaSuccess;
+  const int64_t threads = (int64_t)n_req * 32;
+  k_argmin<<<(int)((threads + 255) / 256), 256, 0, s>>>(n_req, n_inst, scores, choice, best);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_publish(const MlpDesc& mlp, const float* master, Published& pub, cudaStream_t s) {
+  for (int l = 0; l < mlp.n_layers; ++l) {
+    const int out = mlp.w[l + 1], in = mlp.w[l];
+    const int64_t n = (int64_t)out * in + out;
+    k_publish_layer<<<grid_1d(n, 256), 256, 0, s>>>(master + mlp.woff[l], master + mlp.boff[l], out, in,
+                                                   mlp.bf16, pub.params + mlp.woff[l],
+                                                   pub.params + mlp.boff[l], pub.wt + mlp.wtoff[l]);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+cudaError_t launch_ring_append(int n, int d, const float* x, const float* y, float* ring_x,
+                               float* ring_y, int64_t count, int64_t capacity, cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  const int64_t keep = n > capacity ? capacity : n;
+  const int64_t total = keep * (d + 1);
+  k_ring_append<<<grid_1d(total, 256), 256, 0, s>>>(n, d, x, y, ring_x, ring_y, count, capacity);
+  return cudaGetLastError();
+}
+
+}  // namespace ls

@@ -1,0 +1,243 @@
+"""Thin ctypes binding of the C ABI in include/lodestar.h.
+
+The functions below have the ABI's names and only marshal arguments: torch
+tensors become device pointers, streams become cudaStream_t handles, and the
+integer status is returned unchanged.  All computation happens in the CUDA
+library (_build/liblodestar.so); if it is missing the import of `lib()` fails
+loudly -- there is no other implementation to fall back on.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+from . import build as _build
+
+LS_MAX_LAYERS = 8
+LS_OK, LS_ERR_ARG, LS_ERR_CUDA, LS_ERR_OOM = 0, -1, -2, -3
+LS_ERR_TABLE_FULL, LS_ERR_TIMEOUT, LS_ERR_STATE = -4, -5, -6
+LS_F32, LS_BF16 = 0, 1
+LS_REPLACE, LS_INSERT = 0, 1
+LS_SGD, LS_ADAM = 0, 1
+
+
+class ls_config(C.Structure):
+    _fields_ = [("n_layers", C.c_int32), ("widths", C.c_int32 * (LS_MAX_LAYERS + 1)),
+                ("d_inst", C.c_int32), ("d_req", C.c_int32), ("dtype", C.c_int32),
+                ("max_instances", C.c_int32), ("max_requests", C.c_int32),
+                ("max_keys_per_instance", C.c_int64), ("max_load", C.c_float),
+                ("ring_capacity", C.c_int64), ("max_train_batch", C.c_int32)]
+
+
+class ls_info(C.Structure):
+    _fields_ = [("n_inst", C.c_int32), ("d", C.c_int32), ("n_params", C.c_int64),
+                ("table_slots", C.c_int64), ("ring_count", C.c_int64),
+                ("train_steps", C.c_int64), ("weight_version", C.c_uint64)]
+
+
+class ls_trace_entry(C.Structure):
+    _fields_ = [("name", C.c_char * 32), ("launches", C.c_int64), ("total_ms", C.c_double)]
+
+
+_P, _i32, _i64 = C.c_void_p, C.c_int32, C.c_int64
+_SIGS = {
+    "ls_param_count": (_i64, [C.POINTER(ls_config)]),
+    "ls_create": (C.c_int, [C.POINTER(ls_config), C.POINTER(_P)]),
+    "ls_destroy": (None, [_P]),
+    "ls_last_error": (C.c_char_p, []),
+    "ls_sync_status": (C.c_int, [_P]),
+    "ls_get_info": (C.c_int, [_P, C.POINTER(ls_info)]),
+    "ls_set_params": (C.c_int, [_P, _P, _P]),
+    "ls_get_params": (C.c_int, [_P, _P, _P]),
+    "ls_get_opt_state": (C.c_int, [_P, _P, _P, C.POINTER(_i64), _P]),
+    "ls_set_opt_state": (C.c_int, [_P, _P, _P, _i64, _P]),
+    "ls_set_normalizer": (C.c_int, [_P, _P, _P, _P]),
+    "ls_snapshot_update": (C.c_int, [_P, _i32, _P, _P, _P, _i64, _i32, _P]),
+    "ls_hash_blocks": (C.c_int, [_P, _i32, _P, _P, _P, _P, _P]),
+    "ls_assemble_features": (C.c_int, [_P, _i32, _P, _P, _P, _P, _P]),
+    "ls_route_batch": (C.c_int, [_P, _i32, _P, _P, _P, _P, _P, _P, _P, C.POINTER(C.c_uint64), _P]),
+    "ls_log_samples": (C.c_int, [_P, _i32, _P, _P, _P]),
+    "ls_train_step": (C.c_int, [_P, _i32, _P, _i32, C.c_float, _P, _P]),
+    "ls_publish": (C.c_int, [_P, _P]),
+    "ls_trace_enable": (C.c_int, [_P, _i32]),
+    "ls_trace_read": (C.c_int, [_P, C.POINTER(ls_trace_entry), _i32, C.POINTER(_i32)]),
+}
+
+_lib = None
+
+
+def lib_path() -> str:
+    return _build.LIB
+
+
+def lib():
+    """Load the CUDA library (build it first with build.build())."""
+    global _lib
+    if _lib is None:
+        path = lib_path()
+        if not os.path.exists(path):
+            raise RuntimeError(f"{path} is missing: build the CUDA library first "
+                               "(__graft_entry__.build() or paper_2606_00946_gb300.build.build())")
+        L = C.CDLL(path)
+        for name, (res, args) in _SIGS.items():
+            f = getattr(L, name)
+            f.restype = res
+            f.argtypes = args
+        _lib = L
+    return _lib
+
+
+def ptr(t):
+    """Device pointer of a tensor (None -> NULL)."""
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    return t.data_ptr()
+
+
+def stream_handle(s=None):
+    if s is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(s, int):
+        return s
+    return s.cuda_stream
+
+
+class LodestarError(RuntimeError):
+    def __init__(self, code, msg):
+        super().__init__(f"lodestar status {code}: {msg}")
+        self.code = code
+
+
+def last_error() -> str:
+    m = lib().ls_last_error()
+    return m.decode() if m else ""
+
+
+def check(rc: int) -> int:
+    if rc != LS_OK:
+        raise LodestarError(rc, last_error())
+    return rc
+
+
+def make_config(widths, d_inst, d_req, dtype="bf16", max_instances=64, max_requests=4096,
+                max_keys_per_instance=16384, max_load=0.5, ring_capacity=65536,
+                max_train_batch=4096) -> ls_config:
+    c = ls_config()
+    c.n_layers = len(widths) - 1
+    for i, w in enumerate(widths):
+        c.widths[i] = int(w)
+    c.d_inst, c.d_req = int(d_inst), int(d_req)
+    c.dtype = LS_BF16 if dtype in ("bf16", LS_BF16) else LS_F32
+    c.max_instances, c.max_requests = int(max_instances), int(max_requests)
+    c.max_keys_per_instance, c.max_load = int(max_keys_per_instance), float(max_load)
+    c.ring_capacity, c.max_train_batch = int(ring_capacity), int(max_train_batch)
+    return c
+
+
+# ---------------------------------------------------------------------------
+# ABI functions, same names, status returned as is
+# ---------------------------------------------------------------------------
+
+def ls_param_count(cfg: ls_config) -> int:
+    return lib().ls_param_count(C.byref(cfg))
+
+
+def ls_create(cfg: ls_config):
+    """Returns (status, handle)."""
+    h = _P()
+    rc = lib().ls_create(C.byref(cfg), C.byref(h))
+    return rc, h
+
+
+def ls_destroy(ctx):
+    lib().ls_destroy(ctx)
+
+
+def ls_last_error() -> str:
+    return last_error()
+
+
+def ls_sync_status(ctx) -> int:
+    return lib().ls_sync_status(ctx)
+
+
+def ls_get_info(ctx):
+    info = ls_info()
+    rc = lib().ls_get_info(ctx, C.byref(info))
+    return rc, info
+
+
+def ls_set_params(ctx, params, stream=None) -> int:
+    return lib().ls_set_params(ctx, ptr(params), stream_handle(stream))
+
+
+def ls_get_params(ctx, out, stream=None) -> int:
+    return lib().ls_get_params(ctx, ptr(out), stream_handle(stream))
+
+
+def ls_get_opt_state(ctx, m_out, v_out, stream=None):
+    step = _i64()
+    rc = lib().ls_get_opt_state(ctx, ptr(m_out), ptr(v_out), C.byref(step), stream_handle(stream))
+    return rc, step.value
+
+
+def ls_set_opt_state(ctx, m, v, step, stream=None) -> int:
+    return lib().ls_set_opt_state(ctx, ptr(m), ptr(v), int(step), stream_handle(stream))
+
+
+def ls_set_normalizer(ctx, mean, std, stream=None) -> int:
+    return lib().ls_set_normalizer(ctx, ptr(mean), ptr(std), stream_handle(stream))
+
+
+def ls_snapshot_update(ctx, n_inst, inst_state, keys, key_off, n_keys, mode=LS_REPLACE,
+                       stream=None) -> int:
+    return lib().ls_snapshot_update(ctx, int(n_inst), ptr(inst_state), ptr(keys), ptr(key_off),
+                                    int(n_keys), int(mode), stream_handle(stream))
+
+
+def ls_hash_blocks(ctx, n_seq, tok, tok_off, keys_out, key_off, stream=None) -> int:
+    return lib().ls_hash_blocks(ctx, int(n_seq), ptr(tok), ptr(tok_off), ptr(keys_out),
+                                ptr(key_off), stream_handle(stream))
+
+
+def ls_assemble_features(ctx, n_req, tok_off, hits, req_feats, x_out, stream=None) -> int:
+    return lib().ls_assemble_features(ctx, int(n_req), ptr(tok_off), ptr(hits), ptr(req_feats),
+                                      ptr(x_out), stream_handle(stream))
+
+
+def ls_route_batch(ctx, n_req, tok, tok_off, req_feats, choice, best, scores_opt=None,
+                   hits_opt=None, stream=None):
+    """Returns (status, weight_version)."""
+    v = C.c_uint64(0)
+    rc = lib().ls_route_batch(ctx, int(n_req), ptr(tok), ptr(tok_off), ptr(req_feats), ptr(choice),
+                              ptr(best), ptr(scores_opt), ptr(hits_opt), C.byref(v),
+                              stream_handle(stream))
+    return rc, v.value
+
+
+def ls_log_samples(ctx, n, feats, ttft, stream=None) -> int:
+    return lib().ls_log_samples(ctx, int(n), ptr(feats), ptr(ttft), stream_handle(stream))
+
+
+def ls_train_step(ctx, batch, idx, opt, lr, loss_out=None, stream=None) -> int:
+    return lib().ls_train_step(ctx, int(batch), ptr(idx), int(opt), float(lr), ptr(loss_out),
+                               stream_handle(stream))
+
+
+def ls_publish(ctx, stream=None) -> int:
+    return lib().ls_publish(ctx, stream_handle(stream))
+
+
+def ls_trace_enable(ctx, on=True) -> int:
+    return lib().ls_trace_enable(ctx, 1 if on else 0)
+
+
+def ls_trace_read(ctx, max_entries=64):
+    """Returns (status, {name: (launches, total_ms)})."""
+    arr = (ls_trace_entry * max_entries)()
+    n = _i32(0)
+    rc = lib().ls_trace_read(ctx, arr, max_entries, C.byref(n))
+    return rc, {arr[i].name.decode(): (arr[i].launches, arr[i].total_ms) for i in range(n.value)}

@@ -1,0 +1,73 @@
+"""The C-ABI library builds for sm_103a, loads, and exports every entry point
+that include/lodestar.h declares; host-side argument checks answer without a
+GPU (no compute call is made here)."""
+import ctypes as C
+import os
+import re
+
+import pytest
+
+from paper_2606_00946_gb300 import build as B
+from paper_2606_00946_gb300 import lodestar as L
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "lodestar.h")
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?[A-Za-z_][\w\s\*]*?\b(ls_\w+)\s*\(", src, flags=re.M)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    B.build()
+    return L.lib()
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for must in ("ls_create", "ls_destroy", "ls_snapshot_update", "ls_route_batch", "ls_train_step",
+                 "ls_publish", "ls_log_samples", "ls_hash_blocks"):
+        assert must in names
+    assert set(names) == set(L._SIGS), "binding and header disagree"
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def _cfg(**kw):
+    base = dict(widths=[16, 64, 64, 1], d_inst=10, d_req=0, dtype="f32")
+    base.update(kw)
+    return L.make_config(**base)
+
+
+def test_param_count_and_config_validation(lib):
+    assert L.ls_param_count(_cfg()) == 16 * 64 + 64 + 64 * 64 + 64 + 64 + 1
+    bad = [
+        _cfg(widths=[17, 64, 1]),                   # widths[0] != 6 + d_inst + d_req
+        _cfg(widths=[16, 64, 2]),                   # output width must be 1
+        _cfg(max_load=1.0),
+        _cfg(max_load=0.0),
+        _cfg(max_instances=0),
+        _cfg(ring_capacity=0),
+    ]
+    for c in bad:
+        assert L.ls_param_count(c) == L.LS_ERR_ARG
+        rc, h = L.ls_create(c)
+        assert rc == L.LS_ERR_ARG and not h.value
+        assert L.last_error()
+    c = _cfg()
+    c.n_layers = 0
+    assert L.ls_param_count(c) == L.LS_ERR_ARG
+
+
+def test_null_arguments_rejected_on_host(lib):
+    assert lib.ls_create(None, None) == L.LS_ERR_ARG
+    assert lib.ls_route_batch(None, 1, None, None, None, None, None, None, None, None, None) == L.LS_ERR_ARG
+    assert lib.ls_train_step(None, 1, None, 0, C.c_float(1e-3), None, None) == L.LS_ERR_ARG
+    assert lib.ls_publish(None, None) == L.LS_ERR_ARG
+    assert lib.ls_sync_status(None) == L.LS_ERR_ARG
+    lib.ls_destroy(None)

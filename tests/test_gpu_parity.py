@@ -1,0 +1,420 @@
+"""CUDA path vs the CPU oracle on the same seeded inputs, through the C ABI.
+
+Bars: bit-exact block keys, hit lengths and selected instances (the selector
+is checked on the GPU's own scores; against the oracle's scores wherever the
+oracle's top-2 gap exceeds twice the tolerance); predictions within 1e-5
+(fp32) / 2e-2 (bf16) of the prediction scale max(|o|, rms(o)).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2606_00946_gb300 import build as B
+from paper_2606_00946_gb300 import harness as H
+from paper_2606_00946_gb300 import lodestar as L
+from paper_2606_00946_gb300 import workload as W
+
+pytestmark = pytest.mark.gpu
+
+TOL = {"f32": 1e-5, "bf16": 2e-2}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    B.build()
+
+
+_cache = {}
+
+
+def staged(name):
+    if name not in _cache:
+        wl = W.generate(name)
+        r = H.Router.for_config(wl.cfg)
+        dw = H.DeviceWorkload(wl)
+        dw.load(r)
+        _cache[name] = (wl, dw, r)
+    return _cache[name]
+
+
+_okeys = {}
+
+
+def oracle_inst_keys(name, wl):
+    if name not in _okeys:
+        _okeys[name] = oracle.instance_keys(wl)
+    return _okeys[name]
+
+
+def u64(t):
+    return t.cpu().numpy().view(np.uint64)
+
+
+def assert_scores_close(g, o, tol):
+    g = np.asarray(g, np.float64)
+    o = np.asarray(o, np.float64)
+    scale = np.maximum(np.abs(o), np.sqrt(np.mean(o ** 2)))
+    bad = np.abs(g - o) > tol * scale
+    assert not bad.any(), f"{bad.sum()} of {bad.size} predictions off; worst {np.max(np.abs(g-o)/scale):.3g}"
+
+
+def assert_choices(choice, scores_gpu, oracle_scores, tol):
+    # (i) the selector is exact on the GPU's own scores
+    c_own, _ = oracle.argmin(scores_gpu)
+    assert np.array_equal(choice, c_own)
+    # (ii) equal to the oracle's choice wherever the oracle's top-2 gap is clear
+    c_or, b_or = oracle.argmin(oracle_scores)
+    s = np.sort(oracle_scores.astype(np.float64), axis=1)
+    gap = s[:, 1] - s[:, 0] if s.shape[1] > 1 else np.full(len(s), np.inf)
+    scale = np.maximum(np.abs(b_or), np.sqrt(np.mean(oracle_scores.astype(np.float64) ** 2)))
+    clear = gap > 2 * tol * scale
+    assert np.array_equal(choice[clear], c_or[clear])
+    # (iii) near ties: the GPU's pick is within tolerance of the oracle's best
+    near = ~clear
+    if near.any():
+        picked = oracle_scores[np.arange(len(choice)), choice][near]
+        assert np.all(picked - b_or[near] <= 2 * tol * scale[near])
+    return clear.mean()
+
+
+# ----------------------------------------------------------------------------
+# hashing
+# ----------------------------------------------------------------------------
+
+def test_hash_golden_vectors():
+    from test_golden import load_golden
+    wl, dw, r = staged("tiny")
+    for name, t, k in load_golden():
+        tok = torch.from_numpy(t).cuda()
+        off = torch.tensor([0, len(t)], dtype=torch.int64, device="cuda")
+        keys, _ = r.hash_blocks(tok, off)
+        assert np.array_equal(u64(keys), k), name
+
+
+@pytest.mark.parametrize("name", ["tiny", "homogeneous", "heterogeneous"])
+def test_hash_parity(name):
+    wl, dw, r = staged(name)
+    keys, ko = r.hash_blocks(dw.tok, dw.tok_off)
+    want, wko = oracle.hash_blocks(wl.tok, wl.tok_off)
+    assert np.array_equal(ko.cpu().numpy(), wko)
+    assert np.array_equal(u64(keys), want)
+
+
+def test_hash_unaligned_ragged_and_empty():
+    wl, dw, r = staged("tiny")
+    rng = np.random.default_rng(11)
+    lens = [0, 1, 15, 16, 17, 31, 32, 33, 255, 256, 257, 4095, 4096, 4097, 16 * 300 + 3]
+    seqs = [rng.integers(-2**31, 2**31 - 1, size=n, dtype=np.int64).astype(np.int32) for n in lens]
+    tok = np.concatenate([np.array([7], np.int32)] + seqs)           # shift: odd starting offsets
+    off = np.concatenate([[1], 1 + np.cumsum([len(s) for s in seqs])]).astype(np.int64)
+    keys, ko = r.hash_blocks(torch.from_numpy(tok).cuda(), torch.from_numpy(off).cuda())
+    want, _ = oracle.hash_blocks(tok, off)
+    assert np.array_equal(u64(keys), want)
+
+
+# ----------------------------------------------------------------------------
+# prefix hits
+# ----------------------------------------------------------------------------
+
+@pytest.mark.parametrize("name", ["tiny", "homogeneous", "heterogeneous"])
+def test_hits_parity(name):
+    wl, dw, r = staged(name)
+    out = r.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)
+    rk, rko = oracle.hash_blocks(wl.tok, wl.tok_off)
+    ik, iko = oracle_inst_keys(name, wl)
+    want = oracle.prefix_hits(rk, rko, ik, iko)
+    got = out["hits"].cpu().numpy()
+    assert np.array_equal(got, want)
+    assert want.max() > 0 and (want == 0).any()
+
+
+def test_hits_parity_large_sampled():
+    wl, dw, r = staged("large")
+    out = r.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)
+    got = out["hits"].cpu().numpy()
+    idx = np.random.default_rng(5).choice(wl.cfg.n_req, size=48, replace=False)
+    ref = oracle.route(wl, inst_keys=oracle_inst_keys("large", wl), req_idx=idx)
+    assert np.array_equal(got[idx], ref["hits"])
+    assert_scores_close(out["scores"].cpu().numpy()[idx], ref["scores"], TOL["bf16"])
+    assert_choices(out["choice"].cpu().numpy()[idx], out["scores"].cpu().numpy()[idx], ref["scores"],
+                   TOL["bf16"])
+
+
+# ----------------------------------------------------------------------------
+# features, predictions, selection
+# ----------------------------------------------------------------------------
+
+@pytest.mark.parametrize("name", ["tiny", "homogeneous"])
+def test_features_parity(name):
+    wl, dw, r = staged(name)
+    out = r.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)
+    x = r.features(dw.tok_off, out["hits"], dw.req_feats).cpu().numpy()
+    want = oracle.features(np.diff(wl.tok_off), out["hits"].cpu().numpy(), wl.inst_state, wl.req_feats,
+                           wl.mean, wl.std)
+    ulp = np.abs(x.view(np.int32).astype(np.int64) - want.view(np.int32).astype(np.int64))
+    assert ulp.max() <= 1
+
+
+def test_route_parity_tiny_fp32():
+    wl, dw, r = staged("tiny")
+    out = r.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)
+    ref = oracle.route(wl, inst_keys=oracle_inst_keys("tiny", wl))
+    assert np.array_equal(out["hits"].cpu().numpy(), ref["hits"])
+    sg = out["scores"].cpu().numpy()
+    assert_scores_close(sg, ref["scores"], TOL["f32"])
+    frac = assert_choices(out["choice"].cpu().numpy(), sg, ref["scores"], TOL["f32"])
+    assert frac > 0.95
+    assert np.array_equal(out["best"].cpu().numpy(), sg[np.arange(len(sg)), out["choice"].cpu().numpy()])
+
+
+@pytest.mark.parametrize("name,n_sample", [("homogeneous", 512), ("heterogeneous", 96)])
+def test_route_parity_bf16(name, n_sample):
+    wl, dw, r = staged(name)
+    out = r.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)
+    idx = np.sort(np.random.default_rng(3).choice(wl.cfg.n_req, size=n_sample, replace=False))
+    ref = oracle.route(wl, inst_keys=oracle_inst_keys(name, wl), req_idx=idx)
+    sg = out["scores"].cpu().numpy()
+    assert np.array_equal(out["hits"].cpu().numpy()[idx], ref["hits"])
+    assert_scores_close(sg[idx], ref["scores"], TOL["bf16"])
+    assert_choices(out["choice"].cpu().numpy()[idx], sg[idx], ref["scores"], TOL["bf16"])
+    # the selector on every request of the batch
+    c_own, b_own = oracle.argmin(sg)
+    assert np.array_equal(out["choice"].cpu().numpy(), c_own)
+
+
+def test_optional_outputs_do_not_change_the_result():
+    wl, dw, r = staged("homogeneous")
+    full = r.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)
+    bare = r.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst, want_scores=False, want_hits=False)
+    assert torch.equal(full["choice"], bare["choice"]) and torch.equal(full["best"], bare["best"])
+
+
+def test_instance_permutation_and_count_independence():
+    # Sec. 4.1: one shared model, instance identity is never an input.
+    wl, dw, r = staged("tiny")
+    base = r.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)
+    N = wl.cfg.n_inst
+    perm = np.random.default_rng(4).permutation(N)
+    ko = dw.inst_key_off.cpu().numpy()
+    keys = [dw.inst_keys[ko[i]:ko[i + 1]] for i in range(N)]
+    pk = torch.cat([keys[i] for i in perm])
+    pko = torch.tensor(np.concatenate([[0], np.cumsum([len(keys[i]) for i in perm])]), device="cuda")
+    r2 = H.Router.for_config(wl.cfg)
+    r2.set_normalizer(dw.mean, dw.std)
+    r2.snapshot(N, dw.inst_state[torch.from_numpy(perm).cuda()].contiguous(), pk, pko)
+    r2.set_params(dw.params)
+    r2.publish()
+    out = r2.route(dw.tok, dw.tok_off, dw.req_feats, N)
+    assert torch.equal(out["scores"], base["scores"][:, torch.from_numpy(perm).cuda()])
+    assert torch.equal(out["hits"], base["hits"][:, torch.from_numpy(perm).cuda()])
+    # fewer instances: the remaining instances' scores are unchanged
+    keep = 3
+    r2.snapshot(keep, dw.inst_state[:keep].contiguous(), torch.cat(keys[:keep]),
+                torch.tensor(np.concatenate([[0], np.cumsum([len(k) for k in keys[:keep]])]), device="cuda"))
+    out3 = r2.route(dw.tok, dw.tok_off, dw.req_feats, keep)
+    assert torch.equal(out3["scores"], base["scores"][:, :keep])
+    r2.close()
+
+
+def test_edge_cases_empty_short_single_and_nan():
+    wl, dw, r = staged("tiny")
+    # empty batch
+    out = r.route(dw.tok, dw.tok_off[:1], dw.req_feats[:0], wl.cfg.n_inst)
+    assert out["choice"].numel() == 0
+    # empty prompt, prompt shorter than a block, one request
+    tok = torch.tensor([5, 6, 7], dtype=torch.int32, device="cuda")
+    off = torch.tensor([0, 0, 3], dtype=torch.int64, device="cuda")
+    out = r.route(tok, off, dw.req_feats[:2], wl.cfg.n_inst)
+    assert (out["hits"] == 0).all()
+    ref = oracle.features(np.array([0, 3]), np.zeros((2, wl.cfg.n_inst), np.int32), wl.inst_state,
+                          wl.req_feats[:2], wl.mean, wl.std)
+    y = oracle.mlp_forward("f32", wl.cfg.widths, wl.params, ref).reshape(2, -1)
+    assert_scores_close(out["scores"].cpu().numpy(), y, TOL["f32"])
+    # NaN predictions: every score NaN -> choice 0, best NaN
+    p = dw.params.clone()
+    p[-1] = float("nan")
+    r.set_params(p)
+    r.publish()
+    out = r.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)
+    assert (out["choice"] == 0).all() and torch.isnan(out["best"]).all()
+    r.set_params(dw.params)
+    r.publish()
+
+
+def test_publish_versions_and_isolation():
+    wl = W.generate("tiny")
+    r = H.Router.for_config(wl.cfg)
+    dw = H.DeviceWorkload(wl)
+    dw.load(r, publish=False)
+    rc, _ = L.ls_route_batch(r.h, 1, dw.tok, dw.tok_off, dw.req_feats,
+                             torch.empty(1, dtype=torch.int32, device="cuda"),
+                             torch.empty(1, device="cuda"))
+    assert rc == L.LS_ERR_STATE
+    r.publish()
+    a = r.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)
+    assert a["version"] == 1
+    # new master weights are invisible until published
+    p2 = dw.params * 0.5
+    r.set_params(p2)
+    b = r.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)
+    assert b["version"] == 1 and torch.equal(a["scores"], b["scores"])
+    r.publish()
+    c = r.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)
+    assert c["version"] == 2
+    ref = oracle.route(wl, hits=c["hits"].cpu().numpy(), params=p2.cpu().numpy())
+    assert_scores_close(c["scores"].cpu().numpy(), ref["scores"], TOL["f32"])
+    assert r.info().weight_version == 2
+    r.close()
+
+
+# ----------------------------------------------------------------------------
+# training
+# ----------------------------------------------------------------------------
+
+def _weights_close(g, o, before, tol):
+    """Post-step weights, and the step itself (w' - w) in norm."""
+    g, o, before = (np.asarray(a, np.float64) for a in (g, o, before))
+    assert np.all(np.abs(g - o) <= 1e-5 * np.maximum(np.abs(o), 1e-3) + np.abs(o - before) * tol * 4)
+    dg, do = g - before, o - before
+    assert np.linalg.norm(dg - do) <= tol * np.linalg.norm(do)
+
+
+def test_train_sgd_tiny_fp32():
+    wl, dw, r = staged("tiny")
+    r.set_params(dw.params)
+    x = torch.from_numpy(wl.samples_x).cuda()
+    y = torch.from_numpy(wl.samples_y).cuda()
+    r.log(x, y)
+    loss = torch.zeros(1, device="cuda")
+    n = wl.cfg.n_samples
+    idx = torch.arange(n, dtype=torch.int32, device="cuda")
+    r.train(n, idx, opt="sgd", lr=1e-3, loss_out=loss)
+    got = r.get_params().cpu().numpy()
+    tr = oracle.Trainer(wl.cfg.widths, wl.params, "f32")
+    oloss = tr.step(wl.samples_x, wl.samples_y, np.arange(n, dtype=np.int32), wl.mean, wl.std, "sgd", 1e-3)
+    assert abs(loss.item() - oloss) <= 1e-5 * oloss
+    _weights_close(got, tr.params, wl.params, 1e-3)
+    assert r.sync() == L.LS_OK
+    r.set_params(dw.params)
+    r.publish()
+
+
+def _train_router(cfg, ring):
+    return H.Router(cfg.widths, cfg.d_inst, cfg.d_req, cfg.dtype, max_instances=4, max_requests=16,
+                    max_keys_per_instance=64, ring_capacity=ring, max_train_batch=4096)
+
+
+@pytest.mark.parametrize("steps,batch", [(1, 4096), (10, 300)])
+def test_train_adam_bf16(steps, batch):
+    # Every step is compared from the GPU's own starting state (weights, Adam
+    # moments, step count), so bf16 drift between the trajectories cannot hide
+    # or fake a difference in the step itself.
+    cfg = W.CONFIGS["training"]
+    rng = np.random.default_rng(12)
+    n = 20000
+    x, y = W.records(rng, cfg, n)
+    mean, std = W.normaliser(np.random.default_rng(13), cfg)
+    params = W.xavier_params(cfg.widths, 0)
+    r = _train_router(cfg, n)
+    r.set_normalizer(torch.from_numpy(mean).cuda(), torch.from_numpy(std).cuda())
+    r.set_params(torch.from_numpy(params).cuda())
+    r.log(torch.from_numpy(x).cuda(), torch.from_numpy(y).cuda())
+    loss = torch.zeros(1, device="cuda")
+    lr = 3e-4
+    for k in range(steps):
+        idx = W.minibatch_indices(4, k, n, batch)
+        before = r.get_params().cpu().numpy()
+        m0, v0, t0 = r.get_opt_state()
+        r.train(batch, torch.from_numpy(idx).cuda(), opt="adam", lr=lr, loss_out=loss)
+        after = r.get_params().cpu().numpy()
+        m1, v1, t1 = r.get_opt_state()
+        assert t1 == t0 + 1 == k + 1
+        tr = oracle.Trainer(cfg.widths, before, "bf16")
+        tr.m, tr.v, tr.t = m0.cpu().numpy().astype(np.float64), v0.cpu().numpy().astype(np.float64), t0
+        g = oracle.Trainer(cfg.widths, before, "bf16").step(x, y, idx, mean, std, "sgd", 0.0,
+                                                           want_grad=True)[1]
+        ol = tr.step(x, y, idx, mean, std, "adam", lr)
+        assert abs(loss.item() - ol) <= 2e-2 * ol
+        dg, do = after - before.astype(np.float64), tr.params - before.astype(np.float64)
+        clear = np.abs(g) > 0.05 * np.sqrt(np.mean(g ** 2))
+        assert clear.mean() > 0.5
+        assert np.all(np.abs(dg - do)[clear] <= 0.1 * np.abs(do)[clear] + 1e-9)
+        assert np.mean(np.sign(dg) == np.sign(do)) > 0.99
+        np.testing.assert_allclose(m1.cpu().numpy()[clear], tr.m[clear], rtol=5e-2, atol=1e-9)
+        assert np.abs(after - tr.params).max() <= 2.5 * lr
+    assert r.sync() == L.LS_OK
+    r.close()
+
+
+def test_train_gradient_bf16_via_sgd():
+    # SGD with lr 0.1 exposes the bf16 gradient as (w - w') / 0.1.
+    cfg = W.CONFIGS["training"]
+    rng = np.random.default_rng(14)
+    n = 4096
+    x, y = W.records(rng, cfg, n)
+    mean, std = W.normaliser(np.random.default_rng(15), cfg)
+    params = W.xavier_params(cfg.widths, 0)
+    r = _train_router(cfg, n)
+    r.set_normalizer(torch.from_numpy(mean).cuda(), torch.from_numpy(std).cuda())
+    r.set_params(torch.from_numpy(params).cuda())
+    r.log(torch.from_numpy(x).cuda(), torch.from_numpy(y).cuda())
+    idx = W.minibatch_indices(4, 0, n, 4096)
+    r.train(4096, torch.from_numpy(idx).cuda(), opt="sgd", lr=0.1)
+    g_gpu = (params.astype(np.float64) - r.get_params().cpu().numpy()) / 0.1
+    _, g_or = oracle.Trainer(cfg.widths, params, "bf16").step(x, y, idx, mean, std, "sgd", 0.0,
+                                                              want_grad=True)
+    assert np.linalg.norm(g_gpu - g_or) <= 2e-2 * np.linalg.norm(g_or)
+    r.close()
+
+
+def test_ring_wraparound_then_train():
+    cfg = W.CONFIGS["tiny"]
+    rng = np.random.default_rng(16)
+    x, y = W.records(rng, cfg, 700)
+    r = _train_router(cfg, 256)
+    mean, std = W.normaliser(np.random.default_rng(17), cfg)
+    params = W.xavier_params(cfg.widths, 0)
+    r.set_normalizer(torch.from_numpy(mean).cuda(), torch.from_numpy(std).cuda())
+    r.set_params(torch.from_numpy(params).cuda())
+    ox, oy, count = np.zeros((256, cfg.d), np.float32), np.zeros(256, np.float32), 0
+    for a, b in ((0, 100), (100, 350), (350, 700)):   # the last batch is longer than the ring
+        r.log(torch.from_numpy(x[a:b]).cuda(), torch.from_numpy(y[a:b]).cuda())
+        count = oracle.ring_append(ox, oy, count, x[a:b], y[a:b])
+    assert r.info().ring_count == 700
+    idx = np.arange(256, dtype=np.int32)
+    loss = torch.zeros(1, device="cuda")
+    r.train(256, torch.from_numpy(idx).cuda(), opt="sgd", lr=1e-3, loss_out=loss)
+    tr = oracle.Trainer(cfg.widths, params, "f32")
+    ol = tr.step(ox, oy, idx, mean, std, "sgd", 1e-3)
+    assert abs(loss.item() - ol) <= 1e-5 * ol
+    # sequential minibatch (idx = NULL): slots (k*B + j) mod count
+    r.train(100, None, opt="sgd", lr=1e-3, loss_out=loss)
+    ol2 = tr.step(ox, oy, (1 * 100 + np.arange(100)) % 256, mean, std, "sgd", 1e-3)
+    assert abs(loss.item() - ol2) <= 1e-5 * ol2
+    r.close()
+
+
+# ----------------------------------------------------------------------------
+# device-latched errors (no GPU fault involved)
+# ----------------------------------------------------------------------------
+
+def test_table_full_and_bad_slot_are_latched():
+    cfg = W.CONFIGS["tiny"]
+    r = H.Router(cfg.widths, cfg.d_inst, cfg.d_req, "f32", max_instances=2, max_requests=4,
+                 max_keys_per_instance=100, ring_capacity=16, max_train_batch=16)
+    keys = torch.arange(1, 151, dtype=torch.int64, device="cuda")
+    off = torch.tensor([0, 150, 150], dtype=torch.int64, device="cuda")
+    state = torch.zeros(2, cfg.d_inst, device="cuda")
+    r.snapshot(2, state, keys, off)
+    assert r.sync() == L.LS_ERR_TABLE_FULL
+    assert r.sync() == L.LS_OK                       # cleared after reporting
+    r.snapshot(2, state, keys[:100], torch.tensor([0, 100, 100], dtype=torch.int64, device="cuda"))
+    assert r.sync() == L.LS_OK
+    mean = torch.zeros(cfg.d, device="cuda")
+    r.set_normalizer(mean, torch.ones(cfg.d, device="cuda"))
+    r.set_params(torch.from_numpy(W.xavier_params(cfg.widths, 0)).cuda())
+    r.log(torch.zeros(4, cfg.d, device="cuda"), torch.ones(4, device="cuda"))
+    r.train(2, torch.tensor([1, 9], dtype=torch.int32, device="cuda"), opt="sgd", lr=0.0)
+    assert r.sync() == L.LS_ERR_ARG
+    r.close()
