@@ -54,6 +54,7 @@ typedef enum {
 enum { LS_F32 = 0, LS_BF16 = 1 };      /* predictor arithmetic */
 enum { LS_REPLACE = 0, LS_INSERT = 1 };/* ls_snapshot_update key modes */
 enum { LS_SGD = 0, LS_ADAM = 1 };      /* ls_train_step optimisers */
+enum { LS_SCORER_AUTO = 0, LS_SCORER_CUDA_CORES = 1, LS_SCORER_TENSOR_CORES = 2 };
 
 /* Predictor and capacity configuration, fixed at ls_create.
  * widths[0] = d = 6 + d_inst + d_req (pair features, instance state, request
@@ -70,6 +71,10 @@ typedef struct {
     float max_load;                      /* hash-table load bound in (0, 1) */
     int64_t ring_capacity;               /* logged samples kept (oldest evicted) */
     int32_t max_train_batch;
+    int32_t scorer;                      /* LS_SCORER_*: AUTO picks the tensor-core scorer
+                                            for bf16 predictors whose hidden widths are
+                                            multiples of 64 (<= 512), CUDA cores otherwise;
+                                            TENSOR_CORES on an unsupported shape -> LS_ERR_ARG */
 } ls_config;
 
 typedef struct {
@@ -80,6 +85,7 @@ typedef struct {
     int64_t ring_count;          /* samples ever logged */
     int64_t train_steps;         /* training steps taken */
     uint64_t weight_version;     /* version of the last published weights, 0 = none */
+    int32_t scorer;              /* LS_SCORER_CUDA_CORES or LS_SCORER_TENSOR_CORES in use */
 } ls_info;
 
 /* Number of predictor parameters: sum over layers of out*in + out. */

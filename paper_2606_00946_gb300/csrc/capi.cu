@@ -13,7 +13,7 @@ namespace ls {
 const char* const kTraceNames[TR_COUNT] = {
     "hash_blocks", "table_insert", "prefix_match", "score_simt", "argmin", "assemble_features",
     "ring_append", "publish", "train_gather", "gemm_fwd", "loss_grad", "gemm_dw", "reduce_dw",
-    "colsum_db", "gemm_dx", "optimizer", "memset"};
+    "colsum_db", "gemm_dx", "optimizer", "memset", "score_tc", "norm_rows", "publish_tc"};
 }
 
 struct ls_ctx {
@@ -66,6 +66,7 @@ bool check_config(const ls_config* c, std::string& why) {
   if (!(c->max_load > 0.0f && c->max_load < 1.0f)) { why = "max_load must be in (0, 1)"; return false; }
   if (c->ring_capacity < 1) { why = "ring_capacity must be >= 1"; return false; }
   if (c->max_train_batch < 1) { why = "max_train_batch must be >= 1"; return false; }
+  if (c->scorer < LS_SCORER_AUTO || c->scorer > LS_SCORER_TENSOR_CORES) { why = "bad scorer"; return false; }
   const double need = std::ceil((double)c->max_keys_per_instance / (double)c->max_load);
   if (need > (double)(1ull << 31)) { why = "table would exceed 2^31 slots"; return false; }
   return true;
@@ -89,7 +90,7 @@ void free_all(Ctx& c) {
   void* ptrs[] = {c.tables, c.table_count, c.inst_state, c.mean, c.stdv, c.master, c.adam_m,
                   c.adam_v, c.pub[0].params, c.pub[0].wt, c.pub[1].params, c.pub[1].wt,
                   c.ring_x, c.ring_y, c.hits, c.scores, c.tx, c.tz, c.ty, c.dz0, c.dz1, c.grad,
-                  c.gpart, c.loss_tmp, c.d_err};
+                  c.gpart, c.loss_tmp, c.d_err, c.pub[0].img, c.pub[1].img, c.xin, c.xrq};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   for (int b = 0; b < 2; ++b) {
@@ -139,6 +140,15 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
   }
   c.d = m.w[0];
   c.n_params = off;
+  {
+    const bool can_tc = plan_tc(m, c.tc);
+    if (cfg->scorer == LS_SCORER_TENSOR_CORES && !can_tc) {
+      delete h;
+      return fail(LS_ERR_ARG, "tensor-core scorer needs a bf16 predictor with hidden widths that are "
+                              "multiples of 64 and at most 512");
+    }
+    c.use_tc = can_tc && cfg->scorer != LS_SCORER_CUDA_CORES;
+  }
   c.wt_total = wt;
   {
     int dev = 0;
@@ -168,7 +178,10 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
   for (int b = 0; b < 2; ++b) {
     A(dalloc(&c.pub[b].params, c.n_params));
     A(dalloc(&c.pub[b].wt, c.wt_total));
+    if (c.use_tc) A(dalloc(&c.pub[b].img, c.tc.img_bytes));
   }
+  A(dalloc(&c.xin, NI * std::max(1, cfg->d_inst)));
+  A(dalloc(&c.xrq, R * std::max(1, cfg->d_req)));
   A(dalloc(&c.ring_x, cfg->ring_capacity * c.d));
   A(dalloc(&c.ring_y, cfg->ring_capacity));
   A(dalloc(&c.hits, R * NI));
@@ -234,6 +247,7 @@ int ls_get_info(ls_ctx* h, ls_info* out) {
   out->ring_count = c.ring_count;
   out->train_steps = c.step;
   out->weight_version = c.version;
+  out->scorer = c.use_tc ? LS_SCORER_TENSOR_CORES : LS_SCORER_CUDA_CORES;
   return LS_OK;
 }
 
@@ -368,10 +382,22 @@ int ls_route_batch(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* 
   LS_CK(traced(c, TR_PREFIX, 1, s, [&] {
     return launch_prefix_match(n_req, tok, tok_off, c.tables, c.mask, c.slots, c.n_inst, hits, s);
   }));
-  LS_CK(traced(c, TR_SCORE, 1, s, [&] {
-    return launch_score_simt(c.mlp, c.pub[b], n_req, c.n_inst, tok_off, hits, c.inst_state,
-                             c.cfg.d_inst, req_feats, c.cfg.d_req, c.mean, c.stdv, scores, s);
-  }));
+  if (c.use_tc) {
+    LS_CK(traced(c, TR_NORM_ROWS, 1, s, [&] {
+      return launch_norm_rows(c.n_inst, c.cfg.d_inst, c.inst_state, n_req, c.cfg.d_req, req_feats, c.mean,
+                              c.stdv, c.xin, c.xrq, c.sms, s);
+    }));
+    LS_CK(traced(c, TR_SCORE_TC, 1, s, [&] {
+      return launch_score_tc(c.mlp, c.tc, c.pub[b].img, c.pub[b].params, n_req, c.n_inst, tok_off, hits,
+                             c.xin, c.xrq, c.cfg.d_inst, c.cfg.d_req, c.mean, c.stdv, scores, c.d_err, c.sms,
+                             s);
+    }));
+  } else {
+    LS_CK(traced(c, TR_SCORE, 1, s, [&] {
+      return launch_score_simt(c.mlp, c.pub[b], n_req, c.n_inst, tok_off, hits, c.inst_state,
+                               c.cfg.d_inst, req_feats, c.cfg.d_req, c.mean, c.stdv, scores, s);
+    }));
+  }
   LS_CK(traced(c, TR_ARGMIN, 1, s, [&] { return launch_argmin(n_req, c.n_inst, scores, choice, best, s); }));
   {
     std::lock_guard<std::mutex> g(c.mu);
@@ -419,6 +445,9 @@ int ls_publish(ls_ctx* h, void* stream) {
   const int target = c.cur < 0 ? 0 : 1 - c.cur;
   LS_CK(cudaStreamWaitEvent(s, c.route_done[target], 0));
   LS_CK(traced(c, TR_PUBLISH, c.mlp.n_layers, s, [&] { return launch_publish(c.mlp, c.master, c.pub[target], s); }));
+  if (c.use_tc)
+    LS_CK(traced(c, TR_PUBLISH_TC, c.tc.n_tc, s,
+                 [&] { return launch_publish_tc(c.mlp, c.tc, c.master, c.pub[target].img, s); }));
   LS_CK(cudaEventRecord(c.pub_ready[target], s));
   c.version += 1;
   c.pub[target].version = c.version;

@@ -4,6 +4,7 @@
 
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
+#include <algorithm>
 #include <cstdint>
 #include <mutex>
 #include <vector>
@@ -29,11 +30,34 @@ struct MlpDesc {
   int max_width;
 };
 
+// Layout of the tensor-core scorer (k_score_tc.cu), planned once per context.
+struct TcPlan {
+  int n_tc = 0;                    // tensor-core layers (all but the width-1 output layer)
+  int in_pad[LS_MAX_LAYERS] = {};  // K of layer l rounded up to 64
+  int out[LS_MAX_LAYERS] = {};     // N of layer l
+  int nc[LS_MAX_LAYERS] = {};      // N columns per MMA chunk (<= 256)
+  int64_t img_off[LS_MAX_LAYERS] = {};
+  int64_t chunk_off[64] = {};      // byte offset of weight chunk q (per-tile order)
+  int32_t chunk_len[64] = {};
+  int chunks = 0;
+  int64_t img_bytes = 0;
+  int chunk_bytes = 0;
+  int a_bytes = 0;
+  int stages = 0;
+  int resident = 0;
+  int smem = 0;
+  uint32_t tmem_cols = 0;
+  int d_pad = 0;
+  int64_t w_last_off = 0;
+  int64_t b_last_off = 0;
+};
+
 // One published weight version (Sec. 4.3.1 P2: the routing side reads a
 // version that training never writes).
 struct Published {
   float* params = nullptr;  // flat, same layout as the master; weights rounded in bf16 mode
   float* wt = nullptr;      // per-layer transposed weights [in, out]
+  uint8_t* img = nullptr;   // pre-swizzled bf16 hidden-layer weights (tensor-core scorer)
   uint64_t version = 0;
 };
 
@@ -42,7 +66,7 @@ struct Published {
 enum TraceId {
   TR_HASH, TR_INSERT, TR_PREFIX, TR_SCORE, TR_ARGMIN, TR_ASSEMBLE, TR_RING, TR_PUBLISH,
   TR_GATHER, TR_GEMM_FWD, TR_LOSS, TR_GEMM_DW, TR_REDUCE, TR_COLSUM, TR_GEMM_DX, TR_OPT,
-  TR_MEMSET, TR_COUNT
+  TR_MEMSET, TR_SCORE_TC, TR_NORM_ROWS, TR_PUBLISH_TC, TR_COUNT
 };
 extern const char* const kTraceNames[TR_COUNT];
 
@@ -118,6 +142,10 @@ struct Ctx {
   // route scratch
   int32_t* hits = nullptr;    // [max_requests, max_instances]
   float* scores = nullptr;    // [max_requests, max_instances]
+  uint16_t* xin = nullptr;    // normalised bf16 instance rows [max_instances, d_inst]
+  uint16_t* xrq = nullptr;    // normalised bf16 request rows [max_requests, d_req]
+  bool use_tc = false;
+  TcPlan tc;
 
   // train scratch
   float* tx = nullptr;        // activations a_0..a_{L-1}, [B, sum w[0..L-1]]
@@ -204,6 +232,17 @@ cudaError_t launch_argmin(int n_req, int n_inst, const float* scores, int32_t* c
 
 cudaError_t launch_publish(const MlpDesc& mlp, const float* master, Published& pub,
                            cudaStream_t s);
+bool plan_tc(const MlpDesc& m, TcPlan& p);
+cudaError_t launch_publish_tc(const MlpDesc& m, const TcPlan& p, const float* master, uint8_t* img,
+                              cudaStream_t s);
+cudaError_t launch_norm_rows(int n_inst, int d_inst, const float* inst, int n_req, int d_req,
+                             const float* req, const float* mean, const float* stdv, uint16_t* xin,
+                             uint16_t* xrq, int sms, cudaStream_t s);
+cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const uint8_t* img, const float* params,
+                            int n_req, int n_inst, const int64_t* tok_off, const int32_t* hits,
+                            const uint16_t* xin, const uint16_t* xrq, int d_inst, int d_req,
+                            const float* mean, const float* stdv, float* scores, int* err, int sms,
+                            cudaStream_t s);
 cudaError_t launch_ring_append(int n, int d, const float* x, const float* y, float* ring_x,
                                float* ring_y, int64_t count, int64_t capacity, cudaStream_t s);
 cudaError_t run_train_step(Ctx& c, int batch, const int32_t* idx, int opt, float lr,

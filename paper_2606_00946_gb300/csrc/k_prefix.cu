@@ -10,6 +10,8 @@
 //   key_b  = mix64(s_b), 0 mapped to 1                           (table key)
 // The prefix state is a linear recurrence, so a CTA computes the keys of 256
 // consecutive blocks with one parallel scan instead of a serial chain.
+#include <climits>
+
 #include "common.cuh"
 
 namespace ls {
@@ -174,9 +176,11 @@ __global__ void k_table_insert(const uint64_t* __restrict__ keys, const int64_t*
 // Fused hash + probe.  One CTA per request (grid-stride).  The request's
 // blocks are hashed 256 at a time into shared memory; every instance still
 // matching probes them, and hashing stops as soon as no instance matches.
-//  - block 0 is screened with one thread per instance (most pairs end there);
-//  - an instance still matching is then walked by one warp, 32 blocks per
-//    round (32 independent table lookups in flight), ballot -> first miss.
+//  - block 0 is screened with one probe per instance (most pairs end there);
+//  - then, round by round, the instances still matching share the CTA's 256
+//    threads: each gets a window of W = 256 / n_matching consecutive blocks
+//    (power of two), all windows are probed at once, and the first miss of
+//    each window is found with a shared-memory atomicMin.
 __global__ void __launch_bounds__(kThreads) k_prefix_match(int n_req, const int32_t* __restrict__ tok,
                                                            const int64_t* __restrict__ tok_off,
                                                            const uint64_t* __restrict__ tables,
@@ -184,66 +188,96 @@ __global__ void __launch_bounds__(kThreads) k_prefix_match(int n_req, const int3
                                                            int32_t* __restrict__ hits) {
   __shared__ uint64_t keys[kThreads];
   __shared__ uint64_t wtot[kWarps], wpre[kWarps], carry;
-  __shared__ int n_alive;
+  __shared__ int n_alive, n_list;
   extern __shared__ int32_t dyn[];
-  int32_t* hv = dyn;                 // [n_inst] hit length so far
-  int32_t* dead = dyn + n_inst;      // [n_inst] 1 once the first miss is found
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int32_t* hv = dyn;                  // [n_inst] hit length so far
+  int32_t* dead = dyn + n_inst;       // [n_inst] 1 once the first miss is found
+  int32_t* lst = dyn + 2 * n_inst;    // [n_inst] instances with work in this chunk
+  int32_t* fm = dyn + 3 * n_inst;     // [n_inst] first miss of list entry k in this round
+  const int t = threadIdx.x;
 
   for (int r = blockIdx.x; r < n_req; r += gridDim.x) {
     const int64_t t0 = tok_off[r];
     const int64_t nb = (tok_off[r + 1] - t0) / kBlockTok;
     const int32_t* base = tok + t0;
     const bool aligned = ((reinterpret_cast<uintptr_t>(base) & 15) == 0);
-    for (int i = threadIdx.x; i < n_inst; i += kThreads) { hv[i] = 0; dead[i] = 0; }
-    if (threadIdx.x == 0) { carry = kG; n_alive = n_inst; }
+    for (int i = t; i < n_inst; i += kThreads) { hv[i] = 0; dead[i] = 0; }
+    if (t == 0) { carry = kG; n_alive = n_inst; }
     __syncthreads();
 
     for (int64_t c0 = 0; c0 < nb; c0 += kThreads) {
       if (n_alive == 0) break;  // uniform: read after a barrier
       const int n = (int)(nb - c0 < kThreads ? nb - c0 : kThreads);
-      const int t = threadIdx.x;
       const uint64_t s_in = carry;
       uint64_t c = t < n ? block_content(base + (c0 + t) * kBlockTok, aligned) : 0ull;
       uint64_t st = chain_scan(c, s_in, wtot, wpre);
       if (t < n) keys[t] = key_of(st);
       if (t == n - 1) carry = st;
+      if (t == 0) n_list = 0;
       __syncthreads();
 
-      int start = 0;
       if (c0 == 0) {
-        for (int i = threadIdx.x; i < n_inst; i += kThreads) {
+        for (int i = t; i < n_inst; i += kThreads) {
           const bool hit = table_contains(tables + (int64_t)i * slots, mask, keys[0]);
           hv[i] = hit ? 1 : 0;
           dead[i] = hit ? 0 : 1;
         }
         __syncthreads();
-        start = 1;
       }
-      for (int i = warp; i < n_inst; i += kWarps) {
-        if (dead[i]) continue;
-        const uint64_t* tab = tables + (int64_t)i * slots;
-        bool found = false;
-        for (int p = start; p < n; p += 32) {
-          const int b = p + lane;
-          const bool miss = b < n && !table_contains(tab, mask, keys[b]);
-          const unsigned bal = __ballot_sync(kFull, miss);
-          if (bal) {
-            if (lane == 0) { hv[i] = (int32_t)(c0 + p + __ffs(bal) - 1); dead[i] = 1; }
-            found = true;
-            break;
+      // list of instances still matching with blocks left in this chunk
+      for (int i = t; i < n_inst; i += kThreads)
+        if (!dead[i] && hv[i] < c0 + n) {
+          const int k = atomicAdd(&n_list, 1);
+          lst[k] = i;
+          fm[k] = INT_MAX;
+        }
+      __syncthreads();
+      while (n_list > 0) {
+        const int nl = n_list;
+        int logw = 0;
+        while (logw < 8 && (nl << (logw + 1)) <= kThreads) ++logw;
+        const int W = 1 << logw;
+        for (int e = t; e < nl * W; e += kThreads) {
+          const int k = e >> logw;
+          const int i = lst[k];
+          const int b = (int)(hv[i] - c0) + (e & (W - 1));
+          if (b < n && !table_contains(tables + (int64_t)i * slots, mask, keys[b])) atomicMin(&fm[k], b);
+        }
+        __syncthreads();
+        if (t == 0) n_list = 0;
+        __syncthreads();
+        for (int k = t; k < nl; k += kThreads) {
+          const int i = lst[k];
+          if (fm[k] != INT_MAX) {
+            hv[i] = (int32_t)(c0 + fm[k]);
+            dead[i] = 1;
+          } else {
+            const int64_t nv = (int64_t)hv[i] + W;
+            hv[i] = (int32_t)(nv < c0 + n ? nv : c0 + n);
           }
         }
-        if (!found && lane == 0) hv[i] = (int32_t)(c0 + n);
+        __syncthreads();
+        // next list: staged in fm (its values are consumed), then moved to lst
+        for (int k = t; k < nl; k += kThreads) {
+          const int i = lst[k];
+          if (!dead[i] && hv[i] < c0 + n) fm[atomicAdd(&n_list, 1)] = i;
+        }
+        __syncthreads();
+        const int nn = n_list;
+        for (int k = t; k < nn; k += kThreads) {
+          lst[k] = fm[k];
+          fm[k] = INT_MAX;
+        }
+        __syncthreads();
       }
-      if (threadIdx.x == 0) n_alive = 0;
+      if (t == 0) n_alive = 0;
       __syncthreads();
       int alive = 0;
-      for (int i = threadIdx.x; i < n_inst; i += kThreads) alive += dead[i] ? 0 : 1;
+      for (int i = t; i < n_inst; i += kThreads) alive += dead[i] ? 0 : 1;
       if (alive) atomicAdd(&n_alive, alive);
       __syncthreads();
     }
-    for (int i = threadIdx.x; i < n_inst; i += kThreads) hits[(int64_t)r * n_inst + i] = hv[i];
+    for (int i = t; i < n_inst; i += kThreads) hits[(int64_t)r * n_inst + i] = hv[i];
     __syncthreads();
   }
 }
@@ -284,7 +318,7 @@ cudaError_t launch_prefix_match(int n_req, const int32_t* tok, const int64_t* to
                                 const uint64_t* tables, uint32_t mask, int64_t slots, int n_inst,
                                 int32_t* hits, cudaStream_t s) {
   if (n_req <= 0) return cudaSuccess;
-  const size_t smem = (size_t)n_inst * 2 * sizeof(int32_t);
+  const size_t smem = (size_t)n_inst * 4 * sizeof(int32_t);
   if (smem > 48 * 1024) {
     cudaError_t e = cudaFuncSetAttribute(k_prefix_match, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);

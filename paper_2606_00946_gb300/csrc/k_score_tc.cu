@@ -1,0 +1,423 @@
+// Tensor-core scorer for bf16 predictors (Sec. 4.1 reward model; Algorithm 4
+// batched forward): every hidden Linear layer is a tcgen05 MMA with the fp32
+// accumulator in tensor memory; feature tiles and hidden activations are
+// built in shared memory in the 128-byte-swizzled K-major layout the MMA
+// reads; weights arrive by bulk copy (TMA engine) from a pre-swizzled bf16
+// image written at publish time; the width-1 output layer is a dot product in
+// the last epilogue.
+//
+// One persistent CTA per SM (256 threads) walks 128-row tiles (row = r*N + i).
+// Per tile: build the feature tile -> for each hidden layer: one thread issues
+// the MMAs (K = 16 per instruction, N-chunks of <= 256 columns), all warps then
+// read the accumulator (warp w: TMEM lanes 32*(w%4).., column half w/4), add
+// the bias, apply ReLU, round to bf16 and write the next layer's operand tile.
+// When every weight chunk fits in shared memory the weights are loaded once per
+// CTA; otherwise they stream through a ring of stages, the next chunk's copy
+// overlapping the current MMAs.
+#include "common.cuh"
+#include "sm100.cuh"
+
+namespace ls {
+using namespace sm100;
+
+namespace {
+
+constexpr int kTileM = 128;
+constexpr int kThreadsTc = 256;
+constexpr int kMaxChunks = 64;
+constexpr int kMaxSmem = 232448;  // 227 KB opt-in per CTA
+
+struct TcArgs {
+  TcPlan p;
+  const uint8_t* img;
+  const float* params;
+  int64_t boff[LS_MAX_LAYERS];
+  int64_t w_last_off;
+  int n_req, n_inst, d, d_inst, d_req;
+  const int64_t* tok_off;
+  const int32_t* hits;
+  const uint16_t* xin;
+  const uint16_t* xrq;
+  const float* mean;
+  const float* stdv;
+  float* scores;
+  int* err;
+  int64_t rows;
+  int n_tiles;
+};
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+__device__ __forceinline__ uint16_t bf16_bits(float x) {
+  __nv_bfloat16 v = __float2bfloat16_rn(x);
+  return *reinterpret_cast<uint16_t*>(&v);
+}
+
+__device__ __forceinline__ void st_shared_v4(uint8_t* p, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+  asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(smem_u32(p)), "r"(a), "r"(b), "r"(c), "r"(d)
+               : "memory");
+}
+
+// Feature tile of rows row0..row0+127: [pair(6) || inst || req || 0-pad] as bf16.
+__device__ void build_features(const TcArgs& a, uint8_t* A, int64_t row0) {
+  const int cpr = a.p.d_pad / 8;  // 16-byte chunks per row
+  for (int e = threadIdx.x; e < kTileM * cpr; e += kThreadsTc) {
+    const int m = e / cpr, c = e - m * cpr;
+    const int64_t g = row0 + m;
+    uint16_t v[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) v[j] = 0;
+    if (g < a.rows) {
+      const int r = (int)(g / a.n_inst), i = (int)(g - (int64_t)r * a.n_inst);
+      int64_t L = 0;
+      int h = 0;
+      if (c == 0) {
+        L = a.tok_off[r + 1] - a.tok_off[r];
+        h = a.hits[g];
+      }
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int k = c * 8 + j;
+        if (k < kPair) {
+          v[j] = bf16_bits(zscore(raw_feature(k, L, h, nullptr, 0, nullptr), a.mean[k], a.stdv[k]));
+        } else if (k < kPair + a.d_inst) {
+          v[j] = a.xin[(int64_t)i * a.d_inst + (k - kPair)];
+        } else if (k < a.d) {
+          v[j] = a.xrq[(int64_t)r * a.d_req + (k - kPair - a.d_inst)];
+        }
+      }
+    }
+    st_shared_v4(A + sw128_offset(m, c * 8, kTileM), v[0] | ((uint32_t)v[1] << 16),
+                 v[2] | ((uint32_t)v[3] << 16), v[4] | ((uint32_t)v[5] << 16), v[6] | ((uint32_t)v[7] << 16));
+  }
+}
+
+__global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc(const __grid_constant__ TcArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const TcPlan& p = a.p;
+  uint8_t* A = smem;
+  uint8_t* ring = smem + p.a_bytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(ring + (size_t)p.stages * p.chunk_bytes);
+  uint64_t* empty = full + p.stages;
+  uint64_t* done = empty + p.stages;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(done + 1);
+  int* abort_flag = reinterpret_cast<int*>(tmem_holder + 1);
+  float* part = reinterpret_cast<float*>(tmem_holder + 4);  // [2][128]
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  if (tid == 0) {
+    for (int s = 0; s < p.stages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(done, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0) {
+    tmem_alloc(tmem_holder, p.tmem_cols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_holder;
+
+  const int my_tiles = blockIdx.x < a.n_tiles ? (a.n_tiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
+  const int64_t total = (int64_t)my_tiles * p.chunks;
+  int64_t g_load = 0;  // thread 0: next chunk (in consumption order) to copy
+
+  auto issue_load = [&](int64_t gq) {  // thread 0, streaming mode
+    const int s = (int)(gq % p.stages);
+    const int64_t u = gq / p.stages;
+    if (u >= 1 && !mbar_wait(&empty[s], (uint32_t)((u - 1) & 1))) return false;
+    const int q = (int)(gq % p.chunks);
+    mbar_arrive_expect_tx(&full[s], (uint32_t)p.chunk_len[q]);
+    bulk_g2s(ring + (size_t)s * p.chunk_bytes, a.img + p.chunk_off[q], (uint32_t)p.chunk_len[q], &full[s]);
+    return true;
+  };
+
+  if (tid == 0 && my_tiles > 0) {
+    if (p.resident) {
+      for (int q = 0; q < p.chunks; ++q) {
+        mbar_arrive_expect_tx(&full[q], (uint32_t)p.chunk_len[q]);
+        bulk_g2s(ring + (size_t)q * p.chunk_bytes, a.img + p.chunk_off[q], (uint32_t)p.chunk_len[q], &full[q]);
+      }
+    } else {
+      while (g_load < total && g_load < p.stages - 1) {
+        if (!issue_load(g_load)) { *abort_flag = 1; break; }
+        ++g_load;
+      }
+    }
+  }
+  uint32_t done_phase = 0;
+  const int q4 = warp & 3, hh = warp >> 2;
+  const int row = 32 * q4 + lane;
+
+  for (int it = 0; it < my_tiles; ++it) {
+    const int64_t row0 = (int64_t)(blockIdx.x + (int64_t)it * gridDim.x) * kTileM;
+    build_features(a, A, row0);
+    fence_async_smem();
+    __syncthreads();
+    if (*abort_flag) break;
+    int q = 0;
+    for (int l = 0; l < p.n_tc; ++l) {
+      if (tid == 0) {
+        tc_fence_after();
+        bool ok = true;
+        const int nk = p.in_pad[l] / 64, nn = p.out[l] / p.nc[l];
+        const uint32_t idesc = idesc_bf16_f32(kTileM, p.nc[l]);
+        for (int nci = 0; nci < nn && ok; ++nci) {
+          for (int kb = 0; kb < nk && ok; ++kb, ++q) {
+            const int64_t gq = (int64_t)it * p.chunks + q;
+            int s;
+            uint32_t par;
+            if (p.resident) { s = q; par = 0; }
+            else { s = (int)(gq % p.stages); par = (uint32_t)((gq / p.stages) & 1); }
+            if (!mbar_wait(&full[s], par)) { ok = false; break; }
+            tc_fence_after();
+            const uint32_t a_base = smem_u32(A) + (uint32_t)kb * kTileM * 128u;
+            const uint32_t b_base = smem_u32(ring + (size_t)s * p.chunk_bytes);
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+              umma_bf16(tmem + (uint32_t)(nci * p.nc[l]), sdesc_sw128(a_base + 32u * j),
+                        sdesc_sw128(b_base + 32u * j), idesc, (kb | j) ? 1u : 0u);
+            if (!p.resident) {
+              umma_commit(&empty[s]);
+              while (ok && g_load < total && g_load < gq + p.stages) {
+                ok = issue_load(g_load);
+                ++g_load;
+              }
+            }
+          }
+        }
+        umma_commit(done);
+        if (!ok) {
+          *abort_flag = 1;
+          latch_error(a.err, LS_ERR_TIMEOUT);
+        }
+      }
+      __syncwarp();
+      if (!mbar_wait(done, done_phase)) {
+        *abort_flag = 1;
+        latch_error(a.err, LS_ERR_TIMEOUT);
+      }
+      done_phase ^= 1u;
+      tc_fence_after();
+      const int H = p.out[l];
+      const int half = H / 2;
+      const float* bias = a.params + a.boff[l];
+      if (l + 1 < p.n_tc) {
+        // hidden epilogue: bias, ReLU, bf16 -> next layer's operand tile
+        for (int c0 = hh * half; c0 < (hh + 1) * half; c0 += 32) {
+          uint32_t v[32];
+          tmem_ld32(tmem + ((uint32_t)(32 * q4) << 16) + (uint32_t)c0, v);
+          tmem_wait_ld();
+          uint32_t pk[16];
+#pragma unroll
+          for (int j = 0; j < 32; j += 2) {
+            const float f0 = fmaxf(__uint_as_float(v[j]) + __ldg(bias + c0 + j), 0.0f);
+            const float f1 = fmaxf(__uint_as_float(v[j + 1]) + __ldg(bias + c0 + j + 1), 0.0f);
+            pk[j / 2] = pack_bf16(f0, f1);
+          }
+#pragma unroll
+          for (int cc = 0; cc < 4; ++cc)
+            st_shared_v4(A + sw128_offset(row, c0 + 8 * cc, kTileM), pk[4 * cc], pk[4 * cc + 1], pk[4 * cc + 2],
+                         pk[4 * cc + 3]);
+        }
+        tc_fence_before();
+        fence_async_smem();
+        __syncthreads();
+      } else {
+        // last hidden layer: bias, ReLU, bf16 rounding, then the width-1 output layer
+        const float* wl = a.params + a.w_last_off;
+        float s = 0.0f;
+        for (int c0 = hh * half; c0 < (hh + 1) * half; c0 += 32) {
+          uint32_t v[32];
+          tmem_ld32(tmem + ((uint32_t)(32 * q4) << 16) + (uint32_t)c0, v);
+          tmem_wait_ld();
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            const float f = fmaxf(__uint_as_float(v[j]) + __ldg(bias + c0 + j), 0.0f);
+            s = fmaf(round_bf16(f), __ldg(wl + c0 + j), s);
+          }
+        }
+        part[hh * kTileM + row] = s;
+        tc_fence_before();
+        __syncthreads();
+        if (tid < kTileM) {
+          const int64_t g = row0 + tid;
+          if (g < a.rows) a.scores[g] = (part[tid] + part[kTileM + tid]) + __ldg(a.params + a.p.b_last_off);
+        }
+      }
+      if (*abort_flag) break;
+    }
+    if (*abort_flag) break;
+  }
+  __syncthreads();
+  // streaming copies still in flight (only after an abort): wait for them, bounded
+  if (tid == 0 && !p.resident) {
+    for (int64_t gq = g_load - 1; gq >= 0 && gq >= g_load - p.stages; --gq)
+      mbar_wait(&full[gq % p.stages], (uint32_t)((gq / p.stages) & 1));
+  }
+  if (tid == 0 && p.resident && my_tiles == 0) {
+    // nothing was issued
+  }
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tmem, p.tmem_cols);
+}
+
+// Normalised bf16 instance rows and request rows (the inst and req blocks of the
+// feature vector), computed once per batch.
+__global__ void k_norm_rows(int n_inst, int d_inst, const float* __restrict__ inst, int n_req, int d_req,
+                            const float* __restrict__ req, const float* __restrict__ mean,
+                            const float* __restrict__ stdv, uint16_t* __restrict__ xin,
+                            uint16_t* __restrict__ xrq) {
+  const int64_t ni = (int64_t)n_inst * d_inst, nr = (int64_t)n_req * d_req;
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < ni + nr;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    if (e < ni) {
+      const int k = (int)(e % d_inst);
+      xin[e] = bf16_bits(zscore(inst[e], mean[kPair + k], stdv[kPair + k]));
+    } else {
+      const int64_t f = e - ni;
+      const int k = (int)(f % d_req);
+      xrq[f] = bf16_bits(zscore(req[f], mean[kPair + d_inst + k], stdv[kPair + d_inst + k]));
+    }
+  }
+}
+
+// Pre-swizzled bf16 image of hidden layer l: N-chunks of nc rows, each split into
+// K-blocks of 64 columns laid out exactly as the MMA reads them from shared memory.
+__global__ void k_publish_tc(const float* __restrict__ W, int out, int in, int in_pad, int nc,
+                             uint8_t* __restrict__ img) {
+  const int64_t n = (int64_t)out * in_pad;
+  const int nk = in_pad / 64;
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n; e += (int64_t)gridDim.x * blockDim.x) {
+    const int o = (int)(e / in_pad), k = (int)(e - (int64_t)o * in_pad);
+    const float v = k < in ? W[(int64_t)o * in + k] : 0.0f;
+    const int nci = o / nc, orow = o - nci * nc;
+    const int64_t off = (int64_t)nci * nk * nc * 128 + sw128_offset(orow, k, nc);
+    *reinterpret_cast<uint16_t*>(img + off) = bf16_bits(v);
+  }
+}
+
+}  // namespace
+
+bool plan_tc(const MlpDesc& m, TcPlan& p) {
+  p = TcPlan{};
+  if (!m.bf16 || m.n_layers < 2) return false;
+  p.n_tc = m.n_layers - 1;
+  int amax = 0, cb = 0, outmax = 0;
+  int64_t off = 0;
+  int q = 0;
+  p.d_pad = ((m.w[0] + 63) / 64) * 64;
+  for (int l = 0; l < p.n_tc; ++l) {
+    const int in = m.w[l], out = m.w[l + 1];
+    if (out % 64 != 0 || out > 512) return false;
+    if (in > 512) return false;
+    p.in_pad[l] = ((in + 63) / 64) * 64;
+    p.out[l] = out;
+    p.nc[l] = out <= 256 ? out : 256;
+    if (out % p.nc[l] != 0) return false;
+    p.img_off[l] = off;
+    const int nk = p.in_pad[l] / 64, nn = out / p.nc[l];
+    for (int nci = 0; nci < nn; ++nci)
+      for (int kb = 0; kb < nk; ++kb) {
+        if (q >= kMaxChunks) return false;
+        p.chunk_off[q] = off + ((int64_t)nci * nk + kb) * p.nc[l] * 128;
+        p.chunk_len[q] = p.nc[l] * 128;
+        ++q;
+      }
+    off += (int64_t)out * p.in_pad[l] * 2;
+    amax = std::max(amax, p.in_pad[l]);
+    cb = std::max(cb, p.nc[l] * 128);
+    outmax = std::max(outmax, out);
+  }
+  // the operand tile must also hold every hidden output written by an epilogue
+  for (int l = 0; l + 1 < p.n_tc; ++l) amax = std::max(amax, p.out[l]);
+  p.chunks = q;
+  p.img_bytes = off;
+  p.chunk_bytes = cb;
+  p.a_bytes = kTileM * amax * 2;
+  const int fixed = 1024 + 1024 + 64;
+  const int avail = kMaxSmem - fixed - p.a_bytes;
+  const int smax = avail / (cb + 16);
+  if (p.chunks <= smax) {
+    p.resident = 1;
+    p.stages = p.chunks;
+  } else {
+    p.resident = 0;
+    p.stages = std::min(smax, 8);
+    if (p.stages < 2) return false;
+  }
+  p.smem = p.a_bytes + p.stages * cb + (2 * p.stages + 1) * 8 + 16 + 1024 + 1024;
+  p.tmem_cols = 32;
+  while ((int)p.tmem_cols < outmax) p.tmem_cols <<= 1;
+  p.w_last_off = m.woff[m.n_layers - 1];
+  p.b_last_off = m.boff[m.n_layers - 1];
+  return true;
+}
+
+cudaError_t launch_publish_tc(const MlpDesc& m, const TcPlan& p, const float* master, uint8_t* img,
+                              cudaStream_t s) {
+  for (int l = 0; l < p.n_tc; ++l) {
+    const int64_t n = (int64_t)p.out[l] * p.in_pad[l];
+    const int grid = (int)std::min<int64_t>((n + 255) / 256, 1024);
+    k_publish_tc<<<grid, 256, 0, s>>>(master + m.woff[l], p.out[l], m.w[l], p.in_pad[l], p.nc[l],
+                                      img + p.img_off[l]);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+cudaError_t launch_norm_rows(int n_inst, int d_inst, const float* inst, int n_req, int d_req, const float* req,
+                             const float* mean, const float* stdv, uint16_t* xin, uint16_t* xrq, int sms,
+                             cudaStream_t s) {
+  const int64_t n = (int64_t)n_inst * d_inst + (int64_t)n_req * d_req;
+  if (n <= 0) return cudaSuccess;
+  const int grid = (int)std::min<int64_t>((n + 255) / 256, (int64_t)sms * 8);
+  k_norm_rows<<<grid, 256, 0, s>>>(n_inst, d_inst, inst, n_req, d_req, req, mean, stdv, xin, xrq);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const uint8_t* img, const float* params,
+                            int n_req, int n_inst, const int64_t* tok_off, const int32_t* hits,
+                            const uint16_t* xin, const uint16_t* xrq, int d_inst, int d_req, const float* mean,
+                            const float* stdv, float* scores, int* err, int sms, cudaStream_t s) {
+  const int64_t rows = (int64_t)n_req * n_inst;
+  if (rows <= 0) return cudaSuccess;
+  TcArgs a{};
+  a.p = p;
+  a.img = img;
+  a.params = params;
+  for (int l = 0; l < m.n_layers; ++l) a.boff[l] = m.boff[l];
+  a.w_last_off = p.w_last_off;
+  a.n_req = n_req;
+  a.n_inst = n_inst;
+  a.d = m.w[0];
+  a.d_inst = d_inst;
+  a.d_req = d_req;
+  a.tok_off = tok_off;
+  a.hits = hits;
+  a.xin = xin;
+  a.xrq = xrq;
+  a.mean = mean;
+  a.stdv = stdv;
+  a.scores = scores;
+  a.err = err;
+  a.rows = rows;
+  a.n_tiles = (int)((rows + kTileM - 1) / kTileM);
+  cudaError_t e = cudaFuncSetAttribute(k_score_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, p.smem);
+  if (e != cudaSuccess) return e;
+  const int grid = std::min(a.n_tiles, sms);
+  k_score_tc<<<grid, kThreadsTc, p.smem, s>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace ls

@@ -152,13 +152,23 @@ __global__ void __launch_bounds__(1024) k_loss_grad(int B, const float* __restri
   }
 }
 
-// db[o] = sum_j dz[j, o] (unrounded dZ).
-__global__ void k_colsum(int B, int out, const float* __restrict__ dz, float* __restrict__ db) {
-  const int o = blockIdx.x * blockDim.x + threadIdx.x;
-  if (o >= out) return;
+// db[o] = sum_j dz[j, o] (unrounded dZ).  32 columns per CTA; the 32 rows of
+// threads stride over the batch, then the column partials are summed in order.
+__global__ void __launch_bounds__(1024) k_colsum(int B, int out, const float* __restrict__ dz,
+                                                 float* __restrict__ db) {
+  __shared__ float part[32][33];
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+  const int o = blockIdx.x * 32 + tx;
   float s = 0.0f;
-  for (int j = 0; j < B; ++j) s += dz[(int64_t)j * out + o];
-  db[o] = s;
+  if (o < out)
+    for (int j = ty; j < B; j += 32) s += dz[(int64_t)j * out + o];
+  part[ty][tx] = s;
+  __syncthreads();
+  if (ty == 0 && o < out) {
+    float t = 0.0f;
+    for (int k = 0; k < 32; ++k) t += part[k][tx];
+    db[o] = t;
+  }
 }
 
 __global__ void k_reduce_partials(int S, int64_t n, const float* __restrict__ part,
@@ -279,7 +289,7 @@ cudaError_t run_train_step(Ctx& c, int B, const int32_t* idx, int opt, float lr,
     });
     if (e != cudaSuccess) return e;
     e = traced(c, TR_COLSUM, 1, s, [&] {
-      k_colsum<<<(out + 127) / 128, 128, 0, s>>>(B, out, dz, c.grad + m.boff[l]);
+      k_colsum<<<(out + 31) / 32, 1024, 0, s>>>(B, out, dz, c.grad + m.boff[l]);
       return cudaGetLastError();
     });
     if (e != cudaSuccess) return e;

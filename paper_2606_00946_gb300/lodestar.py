@@ -19,6 +19,8 @@ LS_ERR_TABLE_FULL, LS_ERR_TIMEOUT, LS_ERR_STATE = -4, -5, -6
 LS_F32, LS_BF16 = 0, 1
 LS_REPLACE, LS_INSERT = 0, 1
 LS_SGD, LS_ADAM = 0, 1
+LS_SCORER_AUTO, LS_SCORER_CUDA_CORES, LS_SCORER_TENSOR_CORES = 0, 1, 2
+SCORERS = {"auto": 0, "cuda_cores": 1, "tensor_cores": 2}
 
 
 class ls_config(C.Structure):
@@ -26,13 +28,14 @@ class ls_config(C.Structure):
                 ("d_inst", C.c_int32), ("d_req", C.c_int32), ("dtype", C.c_int32),
                 ("max_instances", C.c_int32), ("max_requests", C.c_int32),
                 ("max_keys_per_instance", C.c_int64), ("max_load", C.c_float),
-                ("ring_capacity", C.c_int64), ("max_train_batch", C.c_int32)]
+                ("ring_capacity", C.c_int64), ("max_train_batch", C.c_int32),
+                ("scorer", C.c_int32)]
 
 
 class ls_info(C.Structure):
     _fields_ = [("n_inst", C.c_int32), ("d", C.c_int32), ("n_params", C.c_int64),
                 ("table_slots", C.c_int64), ("ring_count", C.c_int64),
-                ("train_steps", C.c_int64), ("weight_version", C.c_uint64)]
+                ("train_steps", C.c_int64), ("weight_version", C.c_uint64), ("scorer", C.c_int32)]
 
 
 class ls_trace_entry(C.Structure):
@@ -124,7 +127,7 @@ def check(rc: int) -> int:
 
 def make_config(widths, d_inst, d_req, dtype="bf16", max_instances=64, max_requests=4096,
                 max_keys_per_instance=16384, max_load=0.5, ring_capacity=65536,
-                max_train_batch=4096) -> ls_config:
+                max_train_batch=4096, scorer="auto") -> ls_config:
     c = ls_config()
     c.n_layers = len(widths) - 1
     for i, w in enumerate(widths):
@@ -134,6 +137,7 @@ def make_config(widths, d_inst, d_req, dtype="bf16", max_instances=64, max_reque
     c.max_instances, c.max_requests = int(max_instances), int(max_requests)
     c.max_keys_per_instance, c.max_load = int(max_keys_per_instance), float(max_load)
     c.ring_capacity, c.max_train_batch = int(ring_capacity), int(max_train_batch)
+    c.scorer = SCORERS.get(scorer, scorer)
     return c
 
 

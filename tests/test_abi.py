@@ -71,3 +71,15 @@ def test_null_arguments_rejected_on_host(lib):
     assert lib.ls_publish(None, None) == L.LS_ERR_ARG
     assert lib.ls_sync_status(None) == L.LS_ERR_ARG
     lib.ls_destroy(None)
+
+
+def test_tensor_core_scorer_rejected_for_unsupported_predictors(lib):
+    # fp32 predictor, and a bf16 predictor whose hidden width is not a multiple of 64
+    for c in (_cfg(scorer="tensor_cores"),
+              L.make_config([16, 48, 1], 10, 0, "bf16", scorer="tensor_cores")):
+        rc, h = L.ls_create(c)
+        assert rc == L.LS_ERR_ARG and not h.value
+        assert "tensor-core" in L.last_error()
+    bad = _cfg()
+    bad.scorer = 7
+    assert L.ls_param_count(bad) == L.LS_ERR_ARG

@@ -183,6 +183,22 @@ def test_route_parity_bf16(name, n_sample):
     assert np.array_equal(out["choice"].cpu().numpy(), c_own)
 
 
+@pytest.mark.parametrize("name", ["homogeneous", "heterogeneous", "large"])
+def test_tensor_core_scorer_matches_cuda_core_scorer(name):
+    wl, dw, r = staged(name)
+    assert r.info().scorer == L.LS_SCORER_TENSOR_CORES
+    out = r.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)
+    r2 = H.Router.for_config(wl.cfg, scorer="cuda_cores")
+    assert r2.info().scorer == L.LS_SCORER_CUDA_CORES
+    dw.load(r2)
+    out2 = r2.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)
+    assert torch.equal(out["hits"], out2["hits"])
+    s1, s2 = out["scores"].cpu().numpy(), out2["scores"].cpu().numpy()
+    assert_scores_close(s1, s2, TOL["bf16"])
+    assert_choices(out["choice"].cpu().numpy(), s1, s2, TOL["bf16"])
+    r2.close()
+
+
 def test_optional_outputs_do_not_change_the_result():
     wl, dw, r = staged("homogeneous")
     full = r.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)
@@ -337,9 +353,12 @@ def test_train_adam_bf16(steps, batch):
         ol = tr.step(x, y, idx, mean, std, "adam", lr)
         assert abs(loss.item() - ol) <= 2e-2 * ol
         dg, do = after - before.astype(np.float64), tr.params - before.astype(np.float64)
-        clear = np.abs(g) > 0.05 * np.sqrt(np.mean(g ** 2))
+        # coordinates whose gradient is clear of bf16 noise and whose first
+        # moment does not cancel (|m| at least a tenth of its new term)
+        clear = (np.abs(g) > 0.05 * np.sqrt(np.mean(g ** 2))) & (np.abs(tr.m) > 0.01 * np.abs(g))
         assert clear.mean() > 0.5
-        assert np.all(np.abs(dg - do)[clear] <= 0.1 * np.abs(do)[clear] + 1e-9)
+        assert np.all(np.abs(dg - do)[clear] <= 0.1 * np.abs(do)[clear] + 0.05 * lr)
+        assert np.mean(np.abs(dg - do)[clear] <= 0.02 * np.abs(do)[clear] + 0.01 * lr) > 0.99
         assert np.mean(np.sign(dg) == np.sign(do)) > 0.99
         np.testing.assert_allclose(m1.cpu().numpy()[clear], tr.m[clear], rtol=5e-2, atol=1e-9)
         assert np.abs(after - tr.params).max() <= 2.5 * lr
