@@ -121,57 +121,62 @@ def train_flops(widths, B):
 # ----------------------------------------------------------------------------
 
 class ClockSampler:
-    FIELDS = ("uuid,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
-              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
-              "clocks_event_reasons.sw_power_cap")
+    """Polls nvidia-smi (one query per poll) from a thread while the timed
+    region runs; reports the median SM clock, the max clock and every
+    throttle reason seen active."""
+    FIELDS = ("uuid,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    NAMES = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
 
     def __init__(self, uuid):
-        self.uuid = (uuid or "").lower()
-        self.p = None
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_{os.getpid()}.csv")
+        self.uuid = (uuid or "").lower().replace("gpu-", "")
+        self.rows = []
+        self.error = None
+        self._stop = None
+        self._t = None
+
+    def _poll(self):
+        while not self._stop.is_set():
+            try:
+                out = subprocess.run(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits"],
+                                     capture_output=True, text=True, timeout=10)
+                if out.returncode != 0:
+                    self.error = (out.stderr or out.stdout).strip()[:200]
+                    return
+                lines = [[x.strip() for x in ln.split(",")] for ln in out.stdout.splitlines()]
+                lines = [p for p in lines if len(p) >= 9]
+                mine = [p for p in lines if self.uuid and self.uuid in p[0].lower()]
+                self.rows.extend(mine if mine else (lines if len(lines) == 1 else []))
+            except Exception as e:  # no nvidia-smi: report it
+                self.error = str(e)[:200]
+                return
+            self._stop.wait(0.02)
 
     def start(self):
-        try:
-            os.makedirs(os.path.dirname(self.path), exist_ok=True)
-            self.f = open(self.path, "w")
-            self.p = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
-                                       "-lms", "200"], stdout=self.f, stderr=subprocess.DEVNULL)
-        except Exception:
-            self.p = None
+        import threading
+        self._stop = threading.Event()
+        self._t = threading.Thread(target=self._poll, daemon=True)
+        self._t.start()
 
     def stop(self):
-        if not self.p:
+        if self._t is None:
             return None
-        self.p.terminate()
-        try:
-            self.p.wait(timeout=5)
-        except Exception:
-            self.p.kill()
-        self.f.close()
-        rows = []
-        for line in open(self.path):
-            parts = [x.strip() for x in line.split(",")]
-            if len(parts) < 8:
-                continue
-            if self.uuid and self.uuid not in parts[0].lower():
-                continue
-            rows.append(parts)
-        if not rows:
-            return None
+        self._stop.set()
+        self._t.join(timeout=15)
+        if not self.rows:
+            return {"error": self.error or "no samples"}
+
         def num(x):
             try:
                 return float(x)
             except ValueError:
                 return float("nan")
-        sm = np.array([num(r[1]) for r in rows])
-        reasons = []
-        for k, name in zip(range(4, 8), ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
-                                         "sw_power_cap")):
-            if any(r[k].lower() == "active" for r in rows):
-                reasons.append(name)
-        return {"sm_mhz": float(np.nanmedian(sm)), "sm_max_mhz": float(np.nanmax([num(r[2]) for r in rows])),
-                "reasons": reasons, "samples": len(rows),
-                "power_w_max": float(np.nanmax([num(r[3]) for r in rows]))}
+        sm = np.array([num(r[1]) for r in self.rows])
+        reasons = [n for k, n in zip(range(5, 9), self.NAMES) if any(r[k].lower() == "active" for r in self.rows)]
+        return {"sm_mhz": float(np.nanmedian(sm)), "sm_max_mhz": float(np.nanmax([num(r[2]) for r in self.rows])),
+                "reasons": reasons, "samples": len(self.rows),
+                "power_w_max": float(np.nanmax([num(r[3]) for r in self.rows]))}
 
 
 def measured_peaks():

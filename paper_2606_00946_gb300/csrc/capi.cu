@@ -13,7 +13,8 @@ namespace ls {
 const char* const kTraceNames[TR_COUNT] = {
     "hash_blocks", "table_insert", "prefix_match", "score_simt", "argmin", "assemble_features",
     "ring_append", "publish", "train_gather", "gemm_fwd", "loss_grad", "gemm_dw", "reduce_dw",
-    "colsum_db", "gemm_dx", "optimizer", "memset", "score_tc", "norm_rows", "publish_tc"};
+    "colsum_db", "gemm_dx", "optimizer", "memset", "score_tc", "norm_rows", "publish_tc",
+    "hash_batch", "probe_screen", "probe_walk"};
 }
 
 struct ls_ctx {
@@ -67,6 +68,8 @@ bool check_config(const ls_config* c, std::string& why) {
   if (c->ring_capacity < 1) { why = "ring_capacity must be >= 1"; return false; }
   if (c->max_train_batch < 1) { why = "max_train_batch must be >= 1"; return false; }
   if (c->scorer < LS_SCORER_AUTO || c->scorer > LS_SCORER_TENSOR_CORES) { why = "bad scorer"; return false; }
+  if (c->prefix_mode < LS_PREFIX_AUTO || c->prefix_mode > LS_PREFIX_FUSED) { why = "bad prefix_mode"; return false; }
+  if (c->max_batch_tokens < 1) { why = "max_batch_tokens must be >= 1"; return false; }
   const double need = std::ceil((double)c->max_keys_per_instance / (double)c->max_load);
   if (need > (double)(1ull << 31)) { why = "table would exceed 2^31 slots"; return false; }
   return true;
@@ -90,7 +93,8 @@ void free_all(Ctx& c) {
   void* ptrs[] = {c.tables, c.table_count, c.inst_state, c.mean, c.stdv, c.master, c.adam_m,
                   c.adam_v, c.pub[0].params, c.pub[0].wt, c.pub[1].params, c.pub[1].wt,
                   c.ring_x, c.ring_y, c.hits, c.scores, c.tx, c.tz, c.ty, c.dz0, c.dz1, c.grad,
-                  c.gpart, c.loss_tmp, c.d_err, c.pub[0].img, c.pub[1].img, c.xin, c.xrq};
+                  c.gpart, c.loss_tmp, c.d_err, c.pub[0].img, c.pub[1].img, c.xin, c.xrq,
+                  c.bkeys, c.work, c.work_n};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   for (int b = 0; b < 2; ++b) {
@@ -180,8 +184,14 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
     A(dalloc(&c.pub[b].wt, c.wt_total));
     if (c.use_tc) A(dalloc(&c.pub[b].img, c.tc.img_bytes));
   }
-  A(dalloc(&c.xin, NI * std::max(1, cfg->d_inst)));
-  A(dalloc(&c.xrq, R * std::max(1, cfg->d_req)));
+  c.bkeys_cap = cfg->max_batch_tokens / kBlockTok + 1;
+  if (cfg->prefix_mode != LS_PREFIX_FUSED) {
+    A(dalloc(&c.bkeys, c.bkeys_cap));
+    A(dalloc(&c.work, R * NI));
+  }
+  A(dalloc(&c.work_n, 1));
+  A(dalloc(&c.xin, NI * std::max(1, c.tc.d_pad)));
+  A(dalloc(&c.xrq, R * std::max(1, c.tc.d_pad)));
   A(dalloc(&c.ring_x, cfg->ring_capacity * c.d));
   A(dalloc(&c.ring_y, cfg->ring_capacity));
   A(dalloc(&c.hits, R * NI));
@@ -333,7 +343,7 @@ int ls_hash_blocks(ls_ctx* h, int32_t n_seq, const int32_t* tok, const int64_t* 
   if (n_seq == 0) return LS_OK;
   if (!tok || !tok_off || !keys_out || !key_off) return fail(LS_ERR_ARG, "NULL argument");
   LS_CK(traced(h->c, TR_HASH, 1, S(stream), [&] {
-    return launch_hash_blocks(n_seq, tok, tok_off, keys_out, key_off, S(stream));
+    return launch_hash_blocks(n_seq, tok, tok_off, keys_out, key_off, 0, h->c.d_err, S(stream));
   }));
   return LS_OK;
 }
@@ -379,13 +389,28 @@ int ls_route_batch(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* 
   if (n_req == 0) return LS_OK;
   int32_t* hits = hits_opt ? hits_opt : c.hits;
   float* scores = scores_opt ? scores_opt : c.scores;
-  LS_CK(traced(c, TR_PREFIX, 1, s, [&] {
-    return launch_prefix_match(n_req, tok, tok_off, c.tables, c.mask, c.slots, c.n_inst, hits, s);
-  }));
+  if (c.cfg.prefix_mode == LS_PREFIX_FUSED) {
+    LS_CK(traced(c, TR_PREFIX, 1, s, [&] {
+      return launch_prefix_match(n_req, tok, tok_off, c.tables, c.mask, c.slots, c.n_inst, hits, s);
+    }));
+  } else {
+    LS_CK(traced(c, TR_HASH_BATCH, 1, s, [&] {
+      return launch_hash_blocks(n_req, tok, tok_off, c.bkeys, nullptr, c.bkeys_cap, c.d_err, s);
+    }));
+    LS_CK(traced(c, TR_MEMSET, 1, s, [&] { return cudaMemsetAsync(c.work_n, 0, sizeof(int), s); }));
+    LS_CK(traced(c, TR_SCREEN, 1, s, [&] {
+      return launch_probe_screen(n_req, c.n_inst, tok_off, c.bkeys, c.bkeys_cap, c.tables, c.mask, c.slots,
+                                 hits, c.work, c.work_n, c.sms, s);
+    }));
+    LS_CK(traced(c, TR_WALK, 1, s, [&] {
+      return launch_probe_walk(c.n_inst, tok_off, c.bkeys, c.bkeys_cap, c.tables, c.mask, c.slots, hits,
+                               c.work, c.work_n, c.sms, s);
+    }));
+  }
   if (c.use_tc) {
     LS_CK(traced(c, TR_NORM_ROWS, 1, s, [&] {
       return launch_norm_rows(c.n_inst, c.cfg.d_inst, c.inst_state, n_req, c.cfg.d_req, req_feats, c.mean,
-                              c.stdv, c.xin, c.xrq, c.sms, s);
+                              c.stdv, c.tc.d_pad, c.xin, c.xrq, c.sms, s);
     }));
     LS_CK(traced(c, TR_SCORE_TC, 1, s, [&] {
       return launch_score_tc(c.mlp, c.tc, c.pub[b].img, c.pub[b].params, n_req, c.n_inst, tok_off, hits,

@@ -66,7 +66,7 @@ struct Published {
 enum TraceId {
   TR_HASH, TR_INSERT, TR_PREFIX, TR_SCORE, TR_ARGMIN, TR_ASSEMBLE, TR_RING, TR_PUBLISH,
   TR_GATHER, TR_GEMM_FWD, TR_LOSS, TR_GEMM_DW, TR_REDUCE, TR_COLSUM, TR_GEMM_DX, TR_OPT,
-  TR_MEMSET, TR_SCORE_TC, TR_NORM_ROWS, TR_PUBLISH_TC, TR_COUNT
+  TR_MEMSET, TR_SCORE_TC, TR_NORM_ROWS, TR_PUBLISH_TC, TR_HASH_BATCH, TR_SCREEN, TR_WALK, TR_COUNT
 };
 extern const char* const kTraceNames[TR_COUNT];
 
@@ -142,8 +142,12 @@ struct Ctx {
   // route scratch
   int32_t* hits = nullptr;    // [max_requests, max_instances]
   float* scores = nullptr;    // [max_requests, max_instances]
-  uint16_t* xin = nullptr;    // normalised bf16 instance rows [max_instances, d_inst]
-  uint16_t* xrq = nullptr;    // normalised bf16 request rows [max_requests, d_req]
+  uint64_t* bkeys = nullptr;  // block keys of the batch, slot tok_off[r]/16 + b
+  int64_t bkeys_cap = 0;
+  uint32_t* work = nullptr;   // (request, instance) pairs that hit block 0
+  int* work_n = nullptr;
+  uint16_t* xin = nullptr;    // bf16 instance template rows [max_instances, d_pad]
+  uint16_t* xrq = nullptr;    // bf16 request template rows [max_requests, d_pad]
   bool use_tc = false;
   TcPlan tc;
 
@@ -211,7 +215,14 @@ __device__ __forceinline__ float zscore(float x, float mu, float sd) {
 // launchers (each returns the launch status)
 // ---------------------------------------------------------------------------
 cudaError_t launch_hash_blocks(int n_seq, const int32_t* tok, const int64_t* tok_off,
-                               uint64_t* keys_out, const int64_t* key_off, cudaStream_t s);
+                               uint64_t* keys_out, const int64_t* key_off, int64_t cap, int* err,
+                               cudaStream_t s);
+cudaError_t launch_probe_screen(int n_req, int n_inst, const int64_t* tok_off, const uint64_t* keys,
+                                int64_t cap, const uint64_t* tables, uint32_t mask, int64_t slots,
+                                int32_t* hits, uint32_t* work, int* work_n, int sms, cudaStream_t s);
+cudaError_t launch_probe_walk(int n_inst, const int64_t* tok_off, const uint64_t* keys, int64_t cap,
+                              const uint64_t* tables, uint32_t mask, int64_t slots, int32_t* hits,
+                              const uint32_t* work, const int* work_n, int sms, cudaStream_t s);
 cudaError_t launch_table_insert(const uint64_t* keys, const int64_t* key_off, int n_inst,
                                 int64_t n_keys, uint64_t* tables, uint32_t mask, int64_t slots,
                                 int32_t* counts, int64_t max_keys, int* err, cudaStream_t s);
@@ -236,8 +247,8 @@ bool plan_tc(const MlpDesc& m, TcPlan& p);
 cudaError_t launch_publish_tc(const MlpDesc& m, const TcPlan& p, const float* master, uint8_t* img,
                               cudaStream_t s);
 cudaError_t launch_norm_rows(int n_inst, int d_inst, const float* inst, int n_req, int d_req,
-                             const float* req, const float* mean, const float* stdv, uint16_t* xin,
-                             uint16_t* xrq, int sms, cudaStream_t s);
+                             const float* req, const float* mean, const float* stdv, int d_pad,
+                             uint16_t* xin, uint16_t* xrq, int sms, cudaStream_t s);
 cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const uint8_t* img, const float* params,
                             int n_req, int n_inst, const int64_t* tok_off, const int32_t* hits,
                             const uint16_t* xin, const uint16_t* xrq, int d_inst, int d_req,

@@ -10,6 +10,7 @@
 //   key_b  = mix64(s_b), 0 mapped to 1                           (table key)
 // The prefix state is a linear recurrence, so a CTA computes the keys of 256
 // consecutive blocks with one parallel scan instead of a serial chain.
+#include <algorithm>
 #include <climits>
 
 #include "common.cuh"
@@ -111,18 +112,25 @@ __device__ __forceinline__ bool table_contains(const uint64_t* __restrict__ tab,
   return false;
 }
 
-// One CTA per sequence: keys of every full block.
+// One CTA per sequence: keys of every full block.  Keys of sequence s go to
+// keys_out[key_off[s] + b], or, with key_off == nullptr, to the slot
+// floor(tok_off[s] / 16) + b (distinct for every (s, b) because the blocks of
+// a sequence lie inside its own token range); slots at or beyond `cap` are not
+// written and latch LS_ERR_ARG.
 __global__ void __launch_bounds__(kThreads) k_hash_blocks(int n_seq, const int32_t* __restrict__ tok,
                                                           const int64_t* __restrict__ tok_off,
                                                           uint64_t* __restrict__ keys_out,
-                                                          const int64_t* __restrict__ key_off) {
+                                                          const int64_t* __restrict__ key_off, int64_t cap,
+                                                          int* err) {
   __shared__ uint64_t wtot[kWarps], wpre[kWarps], carry;
   for (int s = blockIdx.x; s < n_seq; s += gridDim.x) {
     const int64_t t0 = tok_off[s];
     const int64_t nb = (tok_off[s + 1] - t0) / kBlockTok;
     const int32_t* base = tok + t0;
     const bool aligned = ((reinterpret_cast<uintptr_t>(base) & 15) == 0);
-    uint64_t* out = keys_out + key_off[s];
+    const int64_t k0 = key_off ? key_off[s] : t0 / kBlockTok;
+    uint64_t* out = keys_out + k0;
+    if (!key_off && threadIdx.x == 0 && k0 + nb > cap) latch_error(err, LS_ERR_ARG);
     if (threadIdx.x == 0) carry = kG;
     __syncthreads();
     for (int64_t c0 = 0; c0 < nb; c0 += kThreads) {
@@ -131,11 +139,72 @@ __global__ void __launch_bounds__(kThreads) k_hash_blocks(int n_seq, const int32
       const uint64_t s_in = carry;
       uint64_t c = t < n ? block_content(base + (c0 + t) * kBlockTok, aligned) : 0ull;
       uint64_t st = chain_scan(c, s_in, wtot, wpre);
-      if (t < n) out[c0 + t] = key_of(st);
+      if (t < n && (key_off || k0 + c0 + t < cap)) out[c0 + t] = key_of(st);
       if (t == n - 1) carry = st;
       __syncthreads();
     }
     __syncthreads();
+  }
+}
+
+// Block 0 of every (request, instance) pair, one thread per pair (consecutive
+// threads: consecutive instances of one request).  h = 0 on a miss; on a hit
+// h = 1 and, if the prompt has more blocks, the pair joins the work list.
+__global__ void k_probe_screen(int n_req, int n_inst, const int64_t* __restrict__ tok_off,
+                               const uint64_t* __restrict__ keys, int64_t cap,
+                               const uint64_t* __restrict__ tables, uint32_t mask, int64_t slots,
+                               int32_t* __restrict__ hits, uint32_t* __restrict__ work, int* work_n) {
+  const int64_t pairs = (int64_t)n_req * n_inst;
+  const int lane = threadIdx.x & 31;
+  for (int64_t base = blockIdx.x * (int64_t)blockDim.x; base < pairs; base += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t g = base + threadIdx.x;
+    bool more = false;
+    if (g < pairs) {
+      const int r = (int)(g / n_inst), i = (int)(g - (int64_t)r * n_inst);
+      const int64_t t0 = tok_off[r];
+      const int64_t nb = (tok_off[r + 1] - t0) / kBlockTok;
+      const int64_t k0 = t0 / kBlockTok;
+      bool hit = false;
+      if (nb > 0 && k0 < cap) hit = table_contains(tables + (int64_t)i * slots, mask, keys[k0]);
+      hits[g] = hit ? 1 : 0;
+      more = hit && nb > 1;
+    }
+    const unsigned bal = __ballot_sync(kFull, more);
+    int slot = 0;
+    if (lane == 0 && bal) slot = atomicAdd(work_n, __popc(bal));
+    slot = __shfl_sync(kFull, slot, 0);
+    if (more) work[slot + __popc(bal & ((1u << lane) - 1u))] = (uint32_t)g;
+  }
+}
+
+// Pairs that hit block 0: one warp per pair walks blocks 1, 2, ... 32 at a
+// time (32 independent lookups in flight); the first miss ends the walk.
+__global__ void k_probe_walk(int n_inst, const int64_t* __restrict__ tok_off,
+                             const uint64_t* __restrict__ keys, int64_t cap,
+                             const uint64_t* __restrict__ tables, uint32_t mask, int64_t slots,
+                             int32_t* __restrict__ hits, const uint32_t* __restrict__ work,
+                             const int* __restrict__ work_n) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  const int n = *work_n;
+  for (int64_t e = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; e < n; e += warps) {
+    const uint32_t g = work[e];
+    const int r = (int)(g / (uint32_t)n_inst), i = (int)(g - (uint32_t)r * (uint32_t)n_inst);
+    const int64_t t0 = tok_off[r];
+    const int64_t nb = (tok_off[r + 1] - t0) / kBlockTok;
+    const int64_t k0 = t0 / kBlockTok;
+    const uint64_t* tab = tables + (int64_t)i * slots;
+    int64_t h = nb;
+    for (int64_t p = 1; p < nb; p += 32) {
+      const int64_t b = p + lane;
+      const bool miss = b < nb && (k0 + b >= cap || !table_contains(tab, mask, keys[k0 + b]));
+      const unsigned bal = __ballot_sync(kFull, miss);
+      if (bal) {
+        h = p + __ffs(bal) - 1;
+        break;
+      }
+    }
+    if (lane == 0) hits[g] = (int32_t)h;
   }
 }
 
@@ -294,9 +363,28 @@ int grid_for(int64_t n) {
 }  // namespace
 
 cudaError_t launch_hash_blocks(int n_seq, const int32_t* tok, const int64_t* tok_off,
-                               uint64_t* keys_out, const int64_t* key_off, cudaStream_t s) {
+                               uint64_t* keys_out, const int64_t* key_off, int64_t cap, int* err,
+                               cudaStream_t s) {
   if (n_seq <= 0) return cudaSuccess;
-  k_hash_blocks<<<grid_for(n_seq), kThreads, 0, s>>>(n_seq, tok, tok_off, keys_out, key_off);
+  k_hash_blocks<<<grid_for(n_seq), kThreads, 0, s>>>(n_seq, tok, tok_off, keys_out, key_off, cap, err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_probe_screen(int n_req, int n_inst, const int64_t* tok_off, const uint64_t* keys,
+                                int64_t cap, const uint64_t* tables, uint32_t mask, int64_t slots,
+                                int32_t* hits, uint32_t* work, int* work_n, int sms, cudaStream_t s) {
+  const int64_t pairs = (int64_t)n_req * n_inst;
+  if (pairs <= 0) return cudaSuccess;
+  const int grid = (int)std::min<int64_t>((pairs + 255) / 256, (int64_t)sms * 8);
+  k_probe_screen<<<grid, 256, 0, s>>>(n_req, n_inst, tok_off, keys, cap, tables, mask, slots, hits, work,
+                                      work_n);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_probe_walk(int n_inst, const int64_t* tok_off, const uint64_t* keys, int64_t cap,
+                              const uint64_t* tables, uint32_t mask, int64_t slots, int32_t* hits,
+                              const uint32_t* work, const int* work_n, int sms, cudaStream_t s) {
+  k_probe_walk<<<sms * 8, 256, 0, s>>>(n_inst, tok_off, keys, cap, tables, mask, slots, hits, work, work_n);
   return cudaGetLastError();
 }
 

@@ -6,10 +6,10 @@
 // image written at publish time; the width-1 output layer is a dot product in
 // the last epilogue.
 //
-// One persistent CTA per SM (256 threads) walks 128-row tiles (row = r*N + i).
+// One persistent CTA per SM (512 threads) walks 128-row tiles (row = r*N + i).
 // Per tile: build the feature tile -> for each hidden layer: one thread issues
 // the MMAs (K = 16 per instruction, N-chunks of <= 256 columns), all warps then
-// read the accumulator (warp w: TMEM lanes 32*(w%4).., column half w/4), add
+// read the accumulator (warp w: TMEM lanes 32*(w%4).., column quarter w/4), add
 // the bias, apply ReLU, round to bf16 and write the next layer's operand tile.
 // When every weight chunk fits in shared memory the weights are loaded once per
 // CTA; otherwise they stream through a ring of stages, the next chunk's copy
@@ -23,7 +23,7 @@ using namespace sm100;
 namespace {
 
 constexpr int kTileM = 128;
-constexpr int kThreadsTc = 256;
+constexpr int kThreadsTc = 512;  // 16 warps: 4 per TMEM lane quadrant
 constexpr int kMaxChunks = 64;
 constexpr int kMaxSmem = 232448;  // 227 KB opt-in per CTA
 
@@ -36,8 +36,8 @@ struct TcArgs {
   int n_req, n_inst, d, d_inst, d_req;
   const int64_t* tok_off;
   const int32_t* hits;
-  const uint16_t* xin;
-  const uint16_t* xrq;
+  const uint16_t* xin;   // [n_inst, d_pad] bf16 instance template rows (zero outside inst columns)
+  const uint16_t* xrq;   // [n_req, d_pad]  bf16 request template rows (zero outside req columns)
   const float* mean;
   const float* stdv;
   float* scores;
@@ -62,38 +62,57 @@ __device__ __forceinline__ void st_shared_v4(uint8_t* p, uint32_t a, uint32_t b,
 }
 
 // Feature tile of rows row0..row0+127: [pair(6) || inst || req || 0-pad] as bf16.
-__device__ void build_features(const TcArgs& a, uint8_t* A, int64_t row0) {
+// The instance and request blocks come from template rows that hold the
+// normalised values at their feature positions and zeros elsewhere, so a
+// 16-byte chunk of a feature row is the OR of the two templates' chunks (the
+// pair features, computed here, only occupy chunk 0).
+__device__ __forceinline__ void build_features(const TcArgs& a, uint8_t* A, int64_t row0) {
   const int cpr = a.p.d_pad / 8;  // 16-byte chunks per row
+  const int64_t r0 = row0 / a.n_inst;
+  const int i0 = (int)(row0 - r0 * a.n_inst);
   for (int e = threadIdx.x; e < kTileM * cpr; e += kThreadsTc) {
     const int m = e / cpr, c = e - m * cpr;
     const int64_t g = row0 + m;
-    uint16_t v[8];
-#pragma unroll
-    for (int j = 0; j < 8; ++j) v[j] = 0;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
     if (g < a.rows) {
-      const int r = (int)(g / a.n_inst), i = (int)(g - (int64_t)r * a.n_inst);
-      int64_t L = 0;
-      int h = 0;
-      if (c == 0) {
-        L = a.tok_off[r + 1] - a.tok_off[r];
-        h = a.hits[g];
+      int i = i0 + m;
+      int64_t r = r0;
+      if (a.n_inst >= 16) {
+        while (i >= a.n_inst) { i -= a.n_inst; ++r; }
+      } else {
+        r += i / a.n_inst;
+        i -= (i / a.n_inst) * a.n_inst;
       }
+      const uint4 ti = __ldg(reinterpret_cast<const uint4*>(a.xin + (int64_t)i * a.p.d_pad) + c);
+      const uint4 tr = __ldg(reinterpret_cast<const uint4*>(a.xrq + r * a.p.d_pad) + c);
+      v = make_uint4(ti.x | tr.x, ti.y | tr.y, ti.z | tr.z, ti.w | tr.w);
+      if (c == 0) {
+        const int64_t L = a.tok_off[r + 1] - a.tok_off[r];
+        const int h = a.hits[g];
+        uint16_t f[kPair];
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const int k = c * 8 + j;
-        if (k < kPair) {
-          v[j] = bf16_bits(zscore(raw_feature(k, L, h, nullptr, 0, nullptr), a.mean[k], a.stdv[k]));
-        } else if (k < kPair + a.d_inst) {
-          v[j] = a.xin[(int64_t)i * a.d_inst + (k - kPair)];
-        } else if (k < a.d) {
-          v[j] = a.xrq[(int64_t)r * a.d_req + (k - kPair - a.d_inst)];
-        }
+        for (int k = 0; k < kPair; ++k)
+          f[k] = bf16_bits(zscore(raw_feature(k, L, h, nullptr, 0, nullptr), a.mean[k], a.stdv[k]));
+        v.x = f[0] | ((uint32_t)f[1] << 16);
+        v.y = f[2] | ((uint32_t)f[3] << 16);
+        v.z = f[4] | ((uint32_t)f[5] << 16);
       }
     }
-    st_shared_v4(A + sw128_offset(m, c * 8, kTileM), v[0] | ((uint32_t)v[1] << 16),
-                 v[2] | ((uint32_t)v[3] << 16), v[4] | ((uint32_t)v[5] << 16), v[6] | ((uint32_t)v[7] << 16));
+    st_shared_v4(A + sw128_offset(m, c * 8, kTileM), v.x, v.y, v.z, v.w);
   }
 }
+
+// 16 consecutive fp32 columns of the warp's 32 TMEM lanes.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+
+__device__ __forceinline__ float4 ldg4(const float* p) { return __ldg(reinterpret_cast<const float4*>(p)); }
 
 __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc(const __grid_constant__ TcArgs a) {
   extern __shared__ uint8_t smem_raw[];
@@ -106,7 +125,9 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc(const __grid_constan
   uint64_t* done = empty + p.stages;
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(done + 1);
   int* abort_flag = reinterpret_cast<int*>(tmem_holder + 1);
-  float* part = reinterpret_cast<float*>(tmem_holder + 4);  // [2][128]
+  // partial dot products of the output layer [4][128]; they reuse the operand
+  // tile, whose last reader (the final layer's MMA) has completed by then
+  float* part = reinterpret_cast<float*>(A);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (tid == 0) {
@@ -155,8 +176,10 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc(const __grid_constan
     }
   }
   uint32_t done_phase = 0;
-  const int q4 = warp & 3, hh = warp >> 2;
+  const int q4 = warp & 3;   // TMEM lane quadrant: rows 32*q4 .. 32*q4+31
+  const int cq = warp >> 2;  // column quarter handled by this warp
   const int row = 32 * q4 + lane;
+  const uint32_t lane_addr = (uint32_t)(32 * q4) << 16;
 
   for (int it = 0; it < my_tiles; ++it) {
     const int64_t row0 = (int64_t)(blockIdx.x + (int64_t)it * gridDim.x) * kTileM;
@@ -208,26 +231,26 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc(const __grid_constan
       }
       done_phase ^= 1u;
       tc_fence_after();
-      const int H = p.out[l];
-      const int half = H / 2;
+      const int qw = p.out[l] / 4;  // columns per warp
+      const int cbeg = cq * qw;
       const float* bias = a.params + a.boff[l];
       if (l + 1 < p.n_tc) {
         // hidden epilogue: bias, ReLU, bf16 -> next layer's operand tile
-        for (int c0 = hh * half; c0 < (hh + 1) * half; c0 += 32) {
-          uint32_t v[32];
-          tmem_ld32(tmem + ((uint32_t)(32 * q4) << 16) + (uint32_t)c0, v);
+        for (int c0 = cbeg; c0 < cbeg + qw; c0 += 16) {
+          uint32_t v[16];
+          tmem_ld16(tmem + lane_addr + (uint32_t)c0, v);
           tmem_wait_ld();
-          uint32_t pk[16];
+          uint32_t pk[8];
 #pragma unroll
-          for (int j = 0; j < 32; j += 2) {
-            const float f0 = fmaxf(__uint_as_float(v[j]) + __ldg(bias + c0 + j), 0.0f);
-            const float f1 = fmaxf(__uint_as_float(v[j + 1]) + __ldg(bias + c0 + j + 1), 0.0f);
-            pk[j / 2] = pack_bf16(f0, f1);
+          for (int j4 = 0; j4 < 4; ++j4) {
+            const float4 b = ldg4(bias + c0 + 4 * j4);
+            pk[2 * j4] = pack_bf16(fmaxf(__uint_as_float(v[4 * j4]) + b.x, 0.0f),
+                                   fmaxf(__uint_as_float(v[4 * j4 + 1]) + b.y, 0.0f));
+            pk[2 * j4 + 1] = pack_bf16(fmaxf(__uint_as_float(v[4 * j4 + 2]) + b.z, 0.0f),
+                                       fmaxf(__uint_as_float(v[4 * j4 + 3]) + b.w, 0.0f));
           }
-#pragma unroll
-          for (int cc = 0; cc < 4; ++cc)
-            st_shared_v4(A + sw128_offset(row, c0 + 8 * cc, kTileM), pk[4 * cc], pk[4 * cc + 1], pk[4 * cc + 2],
-                         pk[4 * cc + 3]);
+          st_shared_v4(A + sw128_offset(row, c0, kTileM), pk[0], pk[1], pk[2], pk[3]);
+          st_shared_v4(A + sw128_offset(row, c0 + 8, kTileM), pk[4], pk[5], pk[6], pk[7]);
         }
         tc_fence_before();
         fence_async_smem();
@@ -235,24 +258,35 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc(const __grid_constan
       } else {
         // last hidden layer: bias, ReLU, bf16 rounding, then the width-1 output layer
         const float* wl = a.params + a.w_last_off;
-        float s = 0.0f;
-        for (int c0 = hh * half; c0 < (hh + 1) * half; c0 += 32) {
-          uint32_t v[32];
-          tmem_ld32(tmem + ((uint32_t)(32 * q4) << 16) + (uint32_t)c0, v);
+        float sacc = 0.0f;
+        for (int c0 = cbeg; c0 < cbeg + qw; c0 += 16) {
+          uint32_t v[16];
+          tmem_ld16(tmem + lane_addr + (uint32_t)c0, v);
           tmem_wait_ld();
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            const float f = fmaxf(__uint_as_float(v[j]) + __ldg(bias + c0 + j), 0.0f);
-            s = fmaf(round_bf16(f), __ldg(wl + c0 + j), s);
+          for (int j4 = 0; j4 < 4; ++j4) {
+            const float4 b = ldg4(bias + c0 + 4 * j4);
+            const float4 w = ldg4(wl + c0 + 4 * j4);
+            const __nv_bfloat162 lo = __floats2bfloat162_rn(fmaxf(__uint_as_float(v[4 * j4]) + b.x, 0.0f),
+                                                            fmaxf(__uint_as_float(v[4 * j4 + 1]) + b.y, 0.0f));
+            const __nv_bfloat162 hi = __floats2bfloat162_rn(fmaxf(__uint_as_float(v[4 * j4 + 2]) + b.z, 0.0f),
+                                                            fmaxf(__uint_as_float(v[4 * j4 + 3]) + b.w, 0.0f));
+            sacc = fmaf(__low2float(lo), w.x, sacc);
+            sacc = fmaf(__high2float(lo), w.y, sacc);
+            sacc = fmaf(__low2float(hi), w.z, sacc);
+            sacc = fmaf(__high2float(hi), w.w, sacc);
           }
         }
-        part[hh * kTileM + row] = s;
+        part[cq * kTileM + row] = sacc;
         tc_fence_before();
         __syncthreads();
         if (tid < kTileM) {
           const int64_t g = row0 + tid;
-          if (g < a.rows) a.scores[g] = (part[tid] + part[kTileM + tid]) + __ldg(a.params + a.p.b_last_off);
+          if (g < a.rows)
+            a.scores[g] = ((part[tid] + part[kTileM + tid]) + (part[2 * kTileM + tid] + part[3 * kTileM + tid])) +
+                          __ldg(a.params + a.p.b_last_off);
         }
+        __syncthreads();
       }
       if (*abort_flag) break;
     }
@@ -264,29 +298,32 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc(const __grid_constan
     for (int64_t gq = g_load - 1; gq >= 0 && gq >= g_load - p.stages; --gq)
       mbar_wait(&full[gq % p.stages], (uint32_t)((gq / p.stages) & 1));
   }
-  if (tid == 0 && p.resident && my_tiles == 0) {
-    // nothing was issued
-  }
   __syncthreads();
   if (warp == 0) tmem_dealloc(tmem, p.tmem_cols);
 }
 
-// Normalised bf16 instance rows and request rows (the inst and req blocks of the
-// feature vector), computed once per batch.
+// Normalised bf16 template rows, computed once per batch: instance row i holds
+// the z-scored instance features at their feature positions (6 .. 6+d_inst)
+// and zeros elsewhere; request row r likewise for the request block.
 __global__ void k_norm_rows(int n_inst, int d_inst, const float* __restrict__ inst, int n_req, int d_req,
                             const float* __restrict__ req, const float* __restrict__ mean,
-                            const float* __restrict__ stdv, uint16_t* __restrict__ xin,
+                            const float* __restrict__ stdv, int d_pad, uint16_t* __restrict__ xin,
                             uint16_t* __restrict__ xrq) {
-  const int64_t ni = (int64_t)n_inst * d_inst, nr = (int64_t)n_req * d_req;
+  const int64_t ni = (int64_t)n_inst * d_pad, nr = (int64_t)n_req * d_pad;
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < ni + nr;
        e += (int64_t)gridDim.x * blockDim.x) {
     if (e < ni) {
-      const int k = (int)(e % d_inst);
-      xin[e] = bf16_bits(zscore(inst[e], mean[kPair + k], stdv[kPair + k]));
+      const int64_t i = e / d_pad;
+      const int k = (int)(e - i * d_pad) - kPair;
+      xin[e] = (k >= 0 && k < d_inst) ? bf16_bits(zscore(inst[i * d_inst + k], mean[kPair + k], stdv[kPair + k]))
+                                      : (uint16_t)0;
     } else {
       const int64_t f = e - ni;
-      const int k = (int)(f % d_req);
-      xrq[f] = bf16_bits(zscore(req[f], mean[kPair + d_inst + k], stdv[kPair + d_inst + k]));
+      const int64_t r = f / d_pad;
+      const int k = (int)(f - r * d_pad) - kPair - d_inst;
+      xrq[f] = (k >= 0 && k < d_req)
+                   ? bf16_bits(zscore(req[r * d_req + k], mean[kPair + d_inst + k], stdv[kPair + d_inst + k]))
+                   : (uint16_t)0;
     }
   }
 }
@@ -344,7 +381,7 @@ bool plan_tc(const MlpDesc& m, TcPlan& p) {
   p.img_bytes = off;
   p.chunk_bytes = cb;
   p.a_bytes = kTileM * amax * 2;
-  const int fixed = 1024 + 1024 + 64;
+  const int fixed = 1024 + 64;
   const int avail = kMaxSmem - fixed - p.a_bytes;
   const int smax = avail / (cb + 16);
   if (p.chunks <= smax) {
@@ -355,7 +392,7 @@ bool plan_tc(const MlpDesc& m, TcPlan& p) {
     p.stages = std::min(smax, 8);
     if (p.stages < 2) return false;
   }
-  p.smem = p.a_bytes + p.stages * cb + (2 * p.stages + 1) * 8 + 16 + 1024 + 1024;
+  p.smem = p.a_bytes + p.stages * cb + (2 * p.stages + 1) * 8 + 16 + 1024;
   p.tmem_cols = 32;
   while ((int)p.tmem_cols < outmax) p.tmem_cols <<= 1;
   p.w_last_off = m.woff[m.n_layers - 1];
@@ -377,12 +414,12 @@ cudaError_t launch_publish_tc(const MlpDesc& m, const TcPlan& p, const float* ma
 }
 
 cudaError_t launch_norm_rows(int n_inst, int d_inst, const float* inst, int n_req, int d_req, const float* req,
-                             const float* mean, const float* stdv, uint16_t* xin, uint16_t* xrq, int sms,
-                             cudaStream_t s) {
-  const int64_t n = (int64_t)n_inst * d_inst + (int64_t)n_req * d_req;
+                             const float* mean, const float* stdv, int d_pad, uint16_t* xin, uint16_t* xrq,
+                             int sms, cudaStream_t s) {
+  const int64_t n = (int64_t)(n_inst + n_req) * d_pad;
   if (n <= 0) return cudaSuccess;
   const int grid = (int)std::min<int64_t>((n + 255) / 256, (int64_t)sms * 8);
-  k_norm_rows<<<grid, 256, 0, s>>>(n_inst, d_inst, inst, n_req, d_req, req, mean, stdv, xin, xrq);
+  k_norm_rows<<<grid, 256, 0, s>>>(n_inst, d_inst, inst, n_req, d_req, req, mean, stdv, d_pad, xin, xrq);
   return cudaGetLastError();
 }
 

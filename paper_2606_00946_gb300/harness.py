@@ -38,7 +38,8 @@ class Router:
     def for_config(cls, cfg, **caps):
         base = dict(max_instances=cfg.n_inst, max_requests=cfg.n_req,
                     max_keys_per_instance=cfg.cache_blocks, max_load=0.5,
-                    ring_capacity=max(cfg.n_samples, 1024), max_train_batch=cfg.train_batch)
+                    ring_capacity=max(cfg.n_samples, 1024), max_train_batch=cfg.train_batch,
+                    max_batch_tokens=cfg.n_req * cfg.max_len)
         base.update(caps)
         return cls(cfg.widths, cfg.d_inst, cfg.d_req, cfg.dtype, **base)
 

@@ -21,6 +21,8 @@ LS_REPLACE, LS_INSERT = 0, 1
 LS_SGD, LS_ADAM = 0, 1
 LS_SCORER_AUTO, LS_SCORER_CUDA_CORES, LS_SCORER_TENSOR_CORES = 0, 1, 2
 SCORERS = {"auto": 0, "cuda_cores": 1, "tensor_cores": 2}
+LS_PREFIX_AUTO, LS_PREFIX_TWO_PHASE, LS_PREFIX_FUSED = 0, 1, 2
+PREFIX_MODES = {"auto": 0, "two_phase": 1, "fused": 2}
 
 
 class ls_config(C.Structure):
@@ -29,7 +31,7 @@ class ls_config(C.Structure):
                 ("max_instances", C.c_int32), ("max_requests", C.c_int32),
                 ("max_keys_per_instance", C.c_int64), ("max_load", C.c_float),
                 ("ring_capacity", C.c_int64), ("max_train_batch", C.c_int32),
-                ("scorer", C.c_int32)]
+                ("max_batch_tokens", C.c_int64), ("prefix_mode", C.c_int32), ("scorer", C.c_int32)]
 
 
 class ls_info(C.Structure):
@@ -127,7 +129,8 @@ def check(rc: int) -> int:
 
 def make_config(widths, d_inst, d_req, dtype="bf16", max_instances=64, max_requests=4096,
                 max_keys_per_instance=16384, max_load=0.5, ring_capacity=65536,
-                max_train_batch=4096, scorer="auto") -> ls_config:
+                max_train_batch=4096, scorer="auto", max_batch_tokens=1 << 24,
+                prefix_mode="auto") -> ls_config:
     c = ls_config()
     c.n_layers = len(widths) - 1
     for i, w in enumerate(widths):
@@ -138,6 +141,8 @@ def make_config(widths, d_inst, d_req, dtype="bf16", max_instances=64, max_reque
     c.max_keys_per_instance, c.max_load = int(max_keys_per_instance), float(max_load)
     c.ring_capacity, c.max_train_batch = int(ring_capacity), int(max_train_batch)
     c.scorer = SCORERS.get(scorer, scorer)
+    c.max_batch_tokens = int(max_batch_tokens)
+    c.prefix_mode = PREFIX_MODES.get(prefix_mode, prefix_mode)
     return c
 
 

@@ -129,6 +129,32 @@ def test_hits_parity(name):
     assert want.max() > 0 and (want == 0).any()
 
 
+@pytest.mark.parametrize("name", ["homogeneous", "heterogeneous"])
+def test_fused_prefix_mode_matches_two_phase(name):
+    wl, dw, r = staged(name)
+    out = r.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)
+    r2 = H.Router.for_config(wl.cfg, prefix_mode="fused")
+    dw.load(r2)
+    out2 = r2.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)
+    assert torch.equal(out["hits"], out2["hits"])
+    assert torch.equal(out["choice"], out2["choice"]) and torch.equal(out["scores"], out2["scores"])
+    r2.close()
+
+
+def test_batch_over_token_capacity_is_latched_not_faulted():
+    wl, dw, r = staged("tiny")
+    small = H.Router.for_config(wl.cfg, max_batch_tokens=1000)
+    dw.load(small)
+    small.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)   # ~20k tokens > 1000
+    assert small.sync() == L.LS_ERR_ARG
+    n = 3                                                           # a batch that fits
+    ok = small.route(dw.tok, dw.tok_off[:n + 1], dw.req_feats[:n], wl.cfg.n_inst)
+    assert small.sync() == L.LS_OK
+    ref = r.route(dw.tok, dw.tok_off[:n + 1], dw.req_feats[:n], wl.cfg.n_inst)
+    assert torch.equal(ok["hits"], ref["hits"])
+    small.close()
+
+
 def test_hits_parity_large_sampled():
     wl, dw, r = staged("large")
     out = r.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)
