@@ -14,7 +14,7 @@ const char* const kTraceNames[TR_COUNT] = {
     "hash_blocks", "table_insert", "prefix_match", "score_simt", "argmin", "assemble_features",
     "ring_append", "publish", "train_gather", "gemm_fwd", "loss_grad", "gemm_dw", "reduce_dw",
     "colsum_db", "gemm_dx", "optimizer", "memset", "score_tc", "norm_rows", "publish_tc",
-    "hash_batch", "probe_screen", "probe_walk"};
+    "hash_screen", "probe_screen", "probe_walk", "gemm_tc_fwd", "gemm_tc_dw", "gemm_tc_dx"};
 }
 
 struct ls_ctx {
@@ -202,7 +202,7 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
   A(dalloc(&c.dz0, B * m.max_width));
   A(dalloc(&c.dz1, B * m.max_width));
   A(dalloc(&c.grad, c.n_params));
-  c.gpart_floats = 64 * max_wl;
+  c.gpart_floats = 64 * max_wl + 64 * (int64_t)m.max_width;  // dW partials, then column-sum partials
   A(dalloc(&c.gpart, c.gpart_floats));
   A(dalloc(&c.loss_tmp, 1));
   A(dalloc(&c.d_err, 1));
@@ -394,13 +394,10 @@ int ls_route_batch(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* 
       return launch_prefix_match(n_req, tok, tok_off, c.tables, c.mask, c.slots, c.n_inst, hits, s);
     }));
   } else {
-    LS_CK(traced(c, TR_HASH_BATCH, 1, s, [&] {
-      return launch_hash_blocks(n_req, tok, tok_off, c.bkeys, nullptr, c.bkeys_cap, c.d_err, s);
-    }));
     LS_CK(traced(c, TR_MEMSET, 1, s, [&] { return cudaMemsetAsync(c.work_n, 0, sizeof(int), s); }));
-    LS_CK(traced(c, TR_SCREEN, 1, s, [&] {
-      return launch_probe_screen(n_req, c.n_inst, tok_off, c.bkeys, c.bkeys_cap, c.tables, c.mask, c.slots,
-                                 hits, c.work, c.work_n, c.sms, s);
+    LS_CK(traced(c, TR_HASH_BATCH, 1, s, [&] {
+      return launch_hash_screen(n_req, tok, tok_off, c.bkeys, c.bkeys_cap, c.d_err, c.tables, c.mask, c.slots,
+                                c.n_inst, hits, c.work, c.work_n, c.sms, s);
     }));
     LS_CK(traced(c, TR_WALK, 1, s, [&] {
       return launch_probe_walk(c.n_inst, tok_off, c.bkeys, c.bkeys_cap, c.tables, c.mask, c.slots, hits,

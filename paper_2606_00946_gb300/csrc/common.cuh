@@ -66,7 +66,8 @@ struct Published {
 enum TraceId {
   TR_HASH, TR_INSERT, TR_PREFIX, TR_SCORE, TR_ARGMIN, TR_ASSEMBLE, TR_RING, TR_PUBLISH,
   TR_GATHER, TR_GEMM_FWD, TR_LOSS, TR_GEMM_DW, TR_REDUCE, TR_COLSUM, TR_GEMM_DX, TR_OPT,
-  TR_MEMSET, TR_SCORE_TC, TR_NORM_ROWS, TR_PUBLISH_TC, TR_HASH_BATCH, TR_SCREEN, TR_WALK, TR_COUNT
+  TR_MEMSET, TR_SCORE_TC, TR_NORM_ROWS, TR_PUBLISH_TC, TR_HASH_BATCH, TR_SCREEN, TR_WALK,
+  TR_GEMM_TC_FWD, TR_GEMM_TC_DW, TR_GEMM_TC_DX, TR_COUNT
 };
 extern const char* const kTraceNames[TR_COUNT];
 
@@ -158,7 +159,7 @@ struct Ctx {
   float* dz0 = nullptr;       // [B, max_width]
   float* dz1 = nullptr;
   float* grad = nullptr;      // [n_params]
-  float* gpart = nullptr;     // split-K partials
+  float* gpart = nullptr;     // split-K partials (also column-sum partials)
   int64_t gpart_floats = 0;
   float* loss_tmp = nullptr;  // [1]
 
@@ -217,9 +218,10 @@ __device__ __forceinline__ float zscore(float x, float mu, float sd) {
 cudaError_t launch_hash_blocks(int n_seq, const int32_t* tok, const int64_t* tok_off,
                                uint64_t* keys_out, const int64_t* key_off, int64_t cap, int* err,
                                cudaStream_t s);
-cudaError_t launch_probe_screen(int n_req, int n_inst, const int64_t* tok_off, const uint64_t* keys,
-                                int64_t cap, const uint64_t* tables, uint32_t mask, int64_t slots,
-                                int32_t* hits, uint32_t* work, int* work_n, int sms, cudaStream_t s);
+cudaError_t launch_hash_screen(int n_req, const int32_t* tok, const int64_t* tok_off, uint64_t* keys,
+                               int64_t cap, int* err, const uint64_t* tables, uint32_t mask, int64_t slots,
+                               int n_inst, int32_t* hits, uint32_t* work, int* work_n, int sms,
+                               cudaStream_t s);
 cudaError_t launch_probe_walk(int n_inst, const int64_t* tok_off, const uint64_t* keys, int64_t cap,
                               const uint64_t* tables, uint32_t mask, int64_t slots, int32_t* hits,
                               const uint32_t* work, const int* work_n, int sms, cudaStream_t s);
@@ -258,5 +260,10 @@ cudaError_t launch_ring_append(int n, int d, const float* x, const float* y, flo
                                float* ring_y, int64_t count, int64_t capacity, cudaStream_t s);
 cudaError_t run_train_step(Ctx& c, int batch, const int32_t* idx, int opt, float lr,
                            float* loss_out, cudaStream_t s);
+cudaError_t launch_gemm_tc(int M, int N, int K, const float* A, int64_t sam, int64_t sak, const float* B,
+                           int64_t sbn, int64_t sbk, int splits, int epi, float* C, int64_t ldc,
+                           int64_t split_stride, const float* bias, float* act, int64_t ld_act, int hidden,
+                           const float* zprev, int64_t ld_zprev, int* err, int sms, cudaStream_t s);
+int gemm_tc_splits_used(int K, int splits);
 
 }  // namespace ls

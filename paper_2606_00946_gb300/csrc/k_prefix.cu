@@ -66,6 +66,7 @@ __device__ __forceinline__ uint64_t block_content(const int32_t* p, bool aligned
 // follows state s_in.  Thread t holds content c (0 for threads past the last
 // block: they come after every real block, so they change nothing).
 // Inclusive scan of B_t = sum_{j<=t} G^(t-j) c_j, state_t = G^(t+1) s_in + B_t.
+template <int NT = kThreads>
 __device__ __forceinline__ uint64_t chain_scan(uint64_t c, uint64_t s_in, uint64_t* wtot,
                                                uint64_t* wpre) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -80,7 +81,7 @@ __device__ __forceinline__ uint64_t chain_scan(uint64_t c, uint64_t s_in, uint64
   __syncthreads();
   if (threadIdx.x == 0) {
     uint64_t e = s_in;
-    for (int w = 0; w < kWarps; ++w) {
+    for (int w = 0; w < NT / 32; ++w) {
       wpre[w] = e;
       e = gpow(32) * e + wtot[w];
     }
@@ -99,81 +100,92 @@ __device__ __forceinline__ uint64_t key_of(uint64_t state) {
   return k ? k : 1ull;
 }
 
-// Open-addressing membership: linear probing from key & mask, 0 = empty slot.
-__device__ __forceinline__ bool table_contains(const uint64_t* __restrict__ tab, uint32_t mask,
-                                               uint64_t key) {
+// Open-addressing membership (linear probing from key & mask, 0 = empty slot),
+// read one aligned 32-byte bucket (4 slots, two 16-byte loads) per step: the
+// probe sequence from slot s is s, s+1, ... so only slots at or after s count
+// in the first bucket, which is visited again in full if the walk wraps
+// around.  Tables have >= 16 slots.
+__device__ __forceinline__ bool table_contains_v(const uint64_t* __restrict__ tab, uint32_t mask,
+                                                 uint64_t key) {
   uint32_t s = (uint32_t)key & mask;
-  for (uint32_t n = 0; n <= mask; ++n) {
-    uint64_t v = __ldg(reinterpret_cast<const unsigned long long*>(tab) + s);
-    if (v == key) return true;
-    if (v == 0) return false;
-    s = (s + 1) & mask;
+  uint32_t first = s & 3u;
+  uint32_t b = s & ~3u;
+  for (uint32_t n = 0; n <= (mask >> 2) + 1; ++n) {
+    const ulonglong2* q = reinterpret_cast<const ulonglong2*>(tab + b);
+    const ulonglong2 v01 = __ldg(q), v23 = __ldg(q + 1);
+    const uint64_t v[4] = {v01.x, v01.y, v23.x, v23.y};
+#pragma unroll
+    for (uint32_t j = 0; j < 4; ++j) {
+      if (j < first) continue;
+      if (v[j] == key) return true;
+      if (v[j] == 0) return false;
+    }
+    first = 0;
+    b = (b + 4) & mask;
   }
   return false;
 }
 
 // One CTA per sequence: keys of every full block.  Keys of sequence s go to
 // keys_out[key_off[s] + b], or, with key_off == nullptr, to the slot
-// floor(tok_off[s] / 16) + b (distinct for every (s, b) because the blocks of
-// a sequence lie inside its own token range); slots at or beyond `cap` are not
-// written and latch LS_ERR_ARG.
-__global__ void __launch_bounds__(kThreads) k_hash_blocks(int n_seq, const int32_t* __restrict__ tok,
-                                                          const int64_t* __restrict__ tok_off,
-                                                          uint64_t* __restrict__ keys_out,
-                                                          const int64_t* __restrict__ key_off, int64_t cap,
-                                                          int* err) {
-  __shared__ uint64_t wtot[kWarps], wpre[kWarps], carry;
+// floor((tok_off[s] - tok_off[0]) / 16) + b (distinct for every (s, b)
+// because the blocks of a sequence lie inside its own token range); slots at
+// or beyond `cap` are not written and latch LS_ERR_ARG.
+// With tables != nullptr the CTA then screens block 0 of its request against
+// every instance: h = 0 on a miss, h = 1 on a hit, and hits with more blocks
+// join the work list of k_probe_walk.
+template <int NT>
+__global__ void __launch_bounds__(NT) k_hash_blocks(int n_seq, const int32_t* __restrict__ tok,
+                                                    const int64_t* __restrict__ tok_off,
+                                                    uint64_t* __restrict__ keys_out,
+                                                    const int64_t* __restrict__ key_off, int64_t cap, int* err,
+                                                    const uint64_t* __restrict__ tables, uint32_t mask,
+                                                    int64_t slots, int n_inst, int32_t* __restrict__ hits,
+                                                    uint32_t* __restrict__ work, int* work_n) {
+  constexpr int W = NT / 32;
+  __shared__ uint64_t wtot[W], wpre[W], carry, key0;
+  const int64_t tbase = tok_off[0];
+  const int lane = threadIdx.x & 31;
   for (int s = blockIdx.x; s < n_seq; s += gridDim.x) {
     const int64_t t0 = tok_off[s];
     const int64_t nb = (tok_off[s + 1] - t0) / kBlockTok;
     const int32_t* base = tok + t0;
     const bool aligned = ((reinterpret_cast<uintptr_t>(base) & 15) == 0);
-    const int64_t k0 = key_off ? key_off[s] : t0 / kBlockTok;
+    const int64_t k0 = key_off ? key_off[s] : (t0 - tbase) / kBlockTok;
     uint64_t* out = keys_out + k0;
     if (!key_off && threadIdx.x == 0 && k0 + nb > cap) latch_error(err, LS_ERR_ARG);
     if (threadIdx.x == 0) carry = kG;
     __syncthreads();
-    for (int64_t c0 = 0; c0 < nb; c0 += kThreads) {
-      const int n = (int)(nb - c0 < kThreads ? nb - c0 : kThreads);
+    for (int64_t c0 = 0; c0 < nb; c0 += NT) {
+      const int n = (int)(nb - c0 < NT ? nb - c0 : NT);
       const int t = threadIdx.x;
       const uint64_t s_in = carry;
       uint64_t c = t < n ? block_content(base + (c0 + t) * kBlockTok, aligned) : 0ull;
-      uint64_t st = chain_scan(c, s_in, wtot, wpre);
-      if (t < n && (key_off || k0 + c0 + t < cap)) out[c0 + t] = key_of(st);
+      uint64_t st = chain_scan<NT>(c, s_in, wtot, wpre);
+      const uint64_t key = key_of(st);
+      if (t < n && (key_off || k0 + c0 + t < cap)) out[c0 + t] = key;
+      if (c0 == 0 && t == 0) key0 = key;
       if (t == n - 1) carry = st;
       __syncthreads();
     }
-    __syncthreads();
-  }
-}
-
-// Block 0 of every (request, instance) pair, one thread per pair (consecutive
-// threads: consecutive instances of one request).  h = 0 on a miss; on a hit
-// h = 1 and, if the prompt has more blocks, the pair joins the work list.
-__global__ void k_probe_screen(int n_req, int n_inst, const int64_t* __restrict__ tok_off,
-                               const uint64_t* __restrict__ keys, int64_t cap,
-                               const uint64_t* __restrict__ tables, uint32_t mask, int64_t slots,
-                               int32_t* __restrict__ hits, uint32_t* __restrict__ work, int* work_n) {
-  const int64_t pairs = (int64_t)n_req * n_inst;
-  const int lane = threadIdx.x & 31;
-  for (int64_t base = blockIdx.x * (int64_t)blockDim.x; base < pairs; base += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t g = base + threadIdx.x;
-    bool more = false;
-    if (g < pairs) {
-      const int r = (int)(g / n_inst), i = (int)(g - (int64_t)r * n_inst);
-      const int64_t t0 = tok_off[r];
-      const int64_t nb = (tok_off[r + 1] - t0) / kBlockTok;
-      const int64_t k0 = t0 / kBlockTok;
-      bool hit = false;
-      if (nb > 0 && k0 < cap) hit = table_contains(tables + (int64_t)i * slots, mask, keys[k0]);
-      hits[g] = hit ? 1 : 0;
-      more = hit && nb > 1;
+    if (tables) {
+      const int64_t row = (int64_t)s * n_inst;
+      for (int ib = 0; ib < n_inst; ib += NT) {
+        const int i = ib + threadIdx.x;
+        bool more = false;
+        if (i < n_inst) {
+          const bool hit = nb > 0 && k0 < cap && table_contains_v(tables + (int64_t)i * slots, mask, key0);
+          hits[row + i] = hit ? 1 : 0;
+          more = hit && nb > 1;
+        }
+        const unsigned bal = __ballot_sync(kFull, more);
+        int slot = 0;
+        if (lane == 0 && bal) slot = atomicAdd(work_n, __popc(bal));
+        slot = __shfl_sync(kFull, slot, 0);
+        if (more) work[slot + __popc(bal & ((1u << lane) - 1u))] = (uint32_t)(row + i);
+      }
     }
-    const unsigned bal = __ballot_sync(kFull, more);
-    int slot = 0;
-    if (lane == 0 && bal) slot = atomicAdd(work_n, __popc(bal));
-    slot = __shfl_sync(kFull, slot, 0);
-    if (more) work[slot + __popc(bal & ((1u << lane) - 1u))] = (uint32_t)g;
+    __syncthreads();
   }
 }
 
@@ -187,17 +199,18 @@ __global__ void k_probe_walk(int n_inst, const int64_t* __restrict__ tok_off,
   const int lane = threadIdx.x & 31;
   const int64_t warps = ((int64_t)gridDim.x * blockDim.x) >> 5;
   const int n = *work_n;
+  const int64_t tbase = tok_off[0];
   for (int64_t e = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; e < n; e += warps) {
     const uint32_t g = work[e];
     const int r = (int)(g / (uint32_t)n_inst), i = (int)(g - (uint32_t)r * (uint32_t)n_inst);
     const int64_t t0 = tok_off[r];
     const int64_t nb = (tok_off[r + 1] - t0) / kBlockTok;
-    const int64_t k0 = t0 / kBlockTok;
+    const int64_t k0 = (t0 - tbase) / kBlockTok;
     const uint64_t* tab = tables + (int64_t)i * slots;
     int64_t h = nb;
     for (int64_t p = 1; p < nb; p += 32) {
       const int64_t b = p + lane;
-      const bool miss = b < nb && (k0 + b >= cap || !table_contains(tab, mask, keys[k0 + b]));
+      const bool miss = b < nb && (k0 + b >= cap || !table_contains_v(tab, mask, keys[k0 + b]));
       const unsigned bal = __ballot_sync(kFull, miss);
       if (bal) {
         h = p + __ffs(bal) - 1;
@@ -287,7 +300,7 @@ __global__ void __launch_bounds__(kThreads) k_prefix_match(int n_req, const int3
 
       if (c0 == 0) {
         for (int i = t; i < n_inst; i += kThreads) {
-          const bool hit = table_contains(tables + (int64_t)i * slots, mask, keys[0]);
+          const bool hit = table_contains_v(tables + (int64_t)i * slots, mask, keys[0]);
           hv[i] = hit ? 1 : 0;
           dead[i] = hit ? 0 : 1;
         }
@@ -310,7 +323,7 @@ __global__ void __launch_bounds__(kThreads) k_prefix_match(int n_req, const int3
           const int k = e >> logw;
           const int i = lst[k];
           const int b = (int)(hv[i] - c0) + (e & (W - 1));
-          if (b < n && !table_contains(tables + (int64_t)i * slots, mask, keys[b])) atomicMin(&fm[k], b);
+          if (b < n && !table_contains_v(tables + (int64_t)i * slots, mask, keys[b])) atomicMin(&fm[k], b);
         }
         __syncthreads();
         if (t == 0) n_list = 0;
@@ -366,18 +379,20 @@ cudaError_t launch_hash_blocks(int n_seq, const int32_t* tok, const int64_t* tok
                                uint64_t* keys_out, const int64_t* key_off, int64_t cap, int* err,
                                cudaStream_t s) {
   if (n_seq <= 0) return cudaSuccess;
-  k_hash_blocks<<<grid_for(n_seq), kThreads, 0, s>>>(n_seq, tok, tok_off, keys_out, key_off, cap, err);
+  k_hash_blocks<kThreads><<<grid_for(n_seq), kThreads, 0, s>>>(n_seq, tok, tok_off, keys_out, key_off, cap, err,
+                                                             nullptr, 0, 0, 0, nullptr, nullptr, nullptr);
   return cudaGetLastError();
 }
 
-cudaError_t launch_probe_screen(int n_req, int n_inst, const int64_t* tok_off, const uint64_t* keys,
-                                int64_t cap, const uint64_t* tables, uint32_t mask, int64_t slots,
-                                int32_t* hits, uint32_t* work, int* work_n, int sms, cudaStream_t s) {
-  const int64_t pairs = (int64_t)n_req * n_inst;
-  if (pairs <= 0) return cudaSuccess;
-  const int grid = (int)std::min<int64_t>((pairs + 255) / 256, (int64_t)sms * 8);
-  k_probe_screen<<<grid, 256, 0, s>>>(n_req, n_inst, tok_off, keys, cap, tables, mask, slots, hits, work,
-                                      work_n);
+cudaError_t launch_hash_screen(int n_req, const int32_t* tok, const int64_t* tok_off, uint64_t* keys,
+                               int64_t cap, int* err, const uint64_t* tables, uint32_t mask, int64_t slots,
+                               int n_inst, int32_t* hits, uint32_t* work, int* work_n, int sms,
+                               cudaStream_t s) {
+  if (n_req <= 0) return cudaSuccess;
+  constexpr int NT = 128;
+  const int grid = std::min(n_req, sms * 16);
+  k_hash_blocks<NT><<<grid, NT, 0, s>>>(n_req, tok, tok_off, keys, nullptr, cap, err, tables, mask, slots, n_inst,
+                                        hits, work, work_n);
   return cudaGetLastError();
 }
 

@@ -152,22 +152,25 @@ __global__ void __launch_bounds__(1024) k_loss_grad(int B, const float* __restri
   }
 }
 
-// db[o] = sum_j dz[j, o] (unrounded dZ).  32 columns per CTA; the 32 rows of
-// threads stride over the batch, then the column partials are summed in order.
-__global__ void __launch_bounds__(1024) k_colsum(int B, int out, const float* __restrict__ dz,
-                                                 float* __restrict__ db) {
-  __shared__ float part[32][33];
+// db[o] = sum_j dz[j, o] (unrounded dZ), first stage: CTA (x, y) sums rows
+// y*rows_per .. of 32 columns into part[y][o]; k_reduce_partials adds the
+// partials in order.
+__global__ void __launch_bounds__(256) k_colsum(int B, int out, int rows_per, const float* __restrict__ dz,
+                                                float* __restrict__ part) {
+  __shared__ float red[8][33];
   const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
   const int o = blockIdx.x * 32 + tx;
+  const int j0 = blockIdx.y * rows_per, j1 = min(B, j0 + rows_per);
   float s = 0.0f;
   if (o < out)
-    for (int j = ty; j < B; j += 32) s += dz[(int64_t)j * out + o];
-  part[ty][tx] = s;
+    for (int j = j0 + ty; j < j1; j += 8) s += dz[(int64_t)j * out + o];
+  red[ty][tx] = s;
   __syncthreads();
   if (ty == 0 && o < out) {
     float t = 0.0f;
-    for (int k = 0; k < 32; ++k) t += part[k][tx];
-    db[o] = t;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) t += red[k][tx];
+    part[(int64_t)blockIdx.y * out + o] = t;
   }
 }
 
@@ -255,8 +258,19 @@ cudaError_t run_train_step(Ctx& c, int B, const int32_t* idx, int opt, float lr,
     a.act = a.hidden ? c.tx + xoff[l + 1] : nullptr;
     a.ld_act = m.w[l + 1];
     a.bf16 = m.bf16;
-    e = traced(c, TR_GEMM_FWD, 1, s, [&] { return gemm<false, true, EPI_FWD>(a, 1, s); });
-    if (e != cudaSuccess) return e;
+    bool done_tc = false;
+    if (m.bf16) {
+      e = traced(c, TR_GEMM_TC_FWD, 1, s, [&] {
+        return launch_gemm_tc(a.M, a.N, a.K, a.A, a.lda, 1, a.B, a.ldb, 1, 1, 1, a.C, a.ldc, 0, a.bias, a.act,
+                              a.ld_act, a.hidden, nullptr, 0, c.d_err, c.sms, s);
+      });
+      if (e == cudaSuccess) done_tc = true;
+      else if (e != cudaErrorInvalidValue) return e;
+    }
+    if (!done_tc) {
+      e = traced(c, TR_GEMM_FWD, 1, s, [&] { return gemm<false, true, EPI_FWD>(a, 1, s); });
+      if (e != cudaSuccess) return e;
+    }
   }
   e = traced(c, TR_LOSS, 1, s, [&] {
     k_loss_grad<<<1, 1024, 0, s>>>(B, c.tz + zoff[L - 1], c.ty, c.dz0,
@@ -279,20 +293,44 @@ cudaError_t run_train_step(Ctx& c, int B, const int32_t* idx, int opt, float lr,
     a.round_a = m.bf16; a.round_b = 0;
     a.kchunk = (((B + S - 1) / S + 15) / 16) * 16;
     const int Seff = (B + a.kchunk - 1) / a.kchunk;
-    e = traced(c, TR_GEMM_DW, 1, s, [&] { return gemm<true, false, EPI_STORE>(a, Seff, s); });
-    if (e != cudaSuccess) return e;
+    int nparts = Seff;
+    bool dw_tc = false;
+    if (m.bf16) {
+      const int tiles = ((out + 127) / 128) * ((in + 127) / 128);
+      const int S_tc = std::max(1, std::min({64, B / 64, (2 * c.sms + tiles - 1) / tiles}));
+      e = traced(c, TR_GEMM_TC_DW, 1, s, [&] {
+        return launch_gemm_tc(out, in, B, dz, 1, out, c.tx + xoff[l], 1, in, S_tc, 0, c.gpart, in,
+                              (int64_t)out * in, nullptr, nullptr, 0, 0, nullptr, 0, c.d_err, c.sms, s);
+      });
+      if (e == cudaSuccess) { dw_tc = true; nparts = gemm_tc_splits_used(B, S_tc); }
+      else if (e != cudaErrorInvalidValue) return e;
+    }
+    if (!dw_tc) {
+      e = traced(c, TR_GEMM_DW, 1, s, [&] { return gemm<true, false, EPI_STORE>(a, Seff, s); });
+      if (e != cudaSuccess) return e;
+    }
     const int64_t nw = (int64_t)out * in;
     e = traced(c, TR_REDUCE, 1, s, [&] {
       k_reduce_partials<<<(int)std::min<int64_t>((nw + 255) / 256, (int64_t)c.sms * 8), 256, 0, s>>>(
-          Seff, nw, c.gpart, c.grad + m.woff[l]);
+          nparts, nw, c.gpart, c.grad + m.woff[l]);
       return cudaGetLastError();
     });
     if (e != cudaSuccess) return e;
-    e = traced(c, TR_COLSUM, 1, s, [&] {
-      k_colsum<<<(out + 31) / 32, 1024, 0, s>>>(B, out, dz, c.grad + m.boff[l]);
-      return cudaGetLastError();
-    });
-    if (e != cudaSuccess) return e;
+    {
+      const int S2 = std::max(1, std::min(64, B / 64));
+      const int rows_per = (B + S2 - 1) / S2;
+      float* part = c.gpart + (int64_t)64 * out * in;  // after the dW partials
+      e = traced(c, TR_COLSUM, 1, s, [&] {
+        k_colsum<<<dim3((out + 31) / 32, S2), 256, 0, s>>>(B, out, rows_per, dz, part);
+        return cudaGetLastError();
+      });
+      if (e != cudaSuccess) return e;
+      e = traced(c, TR_REDUCE, 1, s, [&] {
+        k_reduce_partials<<<(out + 255) / 256, 256, 0, s>>>(S2, out, part, c.grad + m.boff[l]);
+        return cudaGetLastError();
+      });
+      if (e != cudaSuccess) return e;
+    }
     if (l > 0) {
       // dZ_{l-1} = (round(dZ_l) round(W_l)) * [z_{l-1} > 0]
       GemmArgs b{};
@@ -303,8 +341,19 @@ cudaError_t run_train_step(Ctx& c, int B, const int32_t* idx, int opt, float lr,
       b.round_a = m.bf16; b.round_b = m.bf16;
       b.kchunk = ((out + 15) / 16) * 16;
       b.zprev = c.tz + zoff[l - 1]; b.ld_zprev = in;
-      e = traced(c, TR_GEMM_DX, 1, s, [&] { return gemm<false, false, EPI_MASK>(b, 1, s); });
-      if (e != cudaSuccess) return e;
+      bool dx_tc = false;
+      if (m.bf16) {
+        e = traced(c, TR_GEMM_TC_DX, 1, s, [&] {
+          return launch_gemm_tc(B, in, out, dz, out, 1, c.master + m.woff[l], 1, in, 1, 2, dzn, in, 0, nullptr,
+                                nullptr, 0, 0, c.tz + zoff[l - 1], in, c.d_err, c.sms, s);
+        });
+        if (e == cudaSuccess) dx_tc = true;
+        else if (e != cudaErrorInvalidValue) return e;
+      }
+      if (!dx_tc) {
+        e = traced(c, TR_GEMM_DX, 1, s, [&] { return gemm<false, false, EPI_MASK>(b, 1, s); });
+        if (e != cudaSuccess) return e;
+      }
       float* t = dz; dz = dzn; dzn = t;
     }
   }

@@ -1,0 +1,223 @@
+// Tensor-core GEMM for the bf16 training step (Sec. 4.3.2 online learning):
+//   D[m, n] = sum_k A(m, k) * B(n, k),  A(m, k) = A[m*sam + k*sak],
+//                                      B(n, k) = B[n*sbn + k*sbk]
+// with fp32 operands in global memory rounded to bf16 (round to nearest even)
+// while they are staged into shared memory.  Arbitrary strides make the
+// transposed operands of the backward pass (dW = dZ^T A, dX = dZ W) plain
+// strided reads.  One CTA computes a 128 x ntile tile with the accumulator in
+// tensor memory; K runs in chunks of 64 through two staging buffers (the next
+// chunk is staged while the MMAs of the current one run); blockIdx.z splits
+// K (partials reduced by the caller).  Epilogues: store (partial), forward
+// (Z = D + bias, A_next = bf16(ReLU(Z))), or ReLU mask (dZ_prev = D * [Z > 0]).
+#include "common.cuh"
+#include "sm100.cuh"
+
+namespace ls {
+using namespace sm100;
+
+namespace {
+
+constexpr int kM = 128;
+constexpr int kT = 256;  // threads: 8 warps, 2 per TMEM lane quadrant
+
+struct TcGemmArgs {
+  int M, N, K;
+  const float* A;
+  int64_t sam, sak;
+  const float* B;
+  int64_t sbn, sbk;
+  int ntile, kper, epi;
+  float* C;
+  int64_t ldc, split_stride;
+  const float* bias;
+  float* act;
+  int64_t ld_act;
+  int hidden;
+  const float* zprev;
+  int64_t ld_zprev;
+  int* err;
+  uint32_t tmem_cols;
+};
+
+__device__ __forceinline__ uint32_t pack2(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+__device__ __forceinline__ void sts32(uint8_t* p, uint32_t v) {
+  asm volatile("st.shared.b32 [%0], %1;" ::"r"(smem_u32(p)), "r"(v) : "memory");
+}
+
+// Stage rows [row0, row0 + R) x k [k0, k0 + 64) of a strided fp32 operand as
+// a bf16 [R x 64] K-major 128B-swizzled tile; out-of-range elements are 0.
+__device__ __forceinline__ void stage(uint8_t* tile, int R, const float* src, int64_t s_row, int64_t s_k,
+                                      int row0, int nrow, int64_t k0, int64_t kend) {
+  if (s_k == 1) {  // k contiguous: consecutive threads take consecutive k pairs of a row
+    for (int e = threadIdx.x; e < R * 32; e += kT) {
+      const int r = e >> 5, k = (e & 31) * 2;
+      const int64_t kk = k0 + k;
+      float v0 = 0.0f, v1 = 0.0f;
+      if (row0 + r < nrow) {
+        const float* p = src + (int64_t)(row0 + r) * s_row + kk;
+        if (kk < kend) v0 = __ldg(p);
+        if (kk + 1 < kend) v1 = __ldg(p + 1);
+      }
+      sts32(tile + sw128_offset(r, k, R), pack2(v0, v1));
+    }
+  } else {  // rows contiguous: consecutive threads take consecutive rows
+    for (int e = threadIdx.x; e < R * 32; e += kT) {
+      const int r = e % R, k = (e / R) * 2;
+      const int64_t kk = k0 + k;
+      float v0 = 0.0f, v1 = 0.0f;
+      if (row0 + r < nrow) {
+        const float* p = src + (int64_t)(row0 + r) * s_row + kk * s_k;
+        if (kk < kend) v0 = __ldg(p);
+        if (kk + 1 < kend) v1 = __ldg(p + s_k);
+      }
+      sts32(tile + sw128_offset(r, k, R), pack2(v0, v1));
+    }
+  }
+}
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+
+__global__ void __launch_bounds__(kT) k_gemm_tc(const __grid_constant__ TcGemmArgs g) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int a_bytes = kM * 128, b_bytes = g.ntile * 128;
+  uint8_t* As[2] = {smem, smem + a_bytes};
+  uint8_t* Bs[2] = {smem + 2 * a_bytes, smem + 2 * a_bytes + b_bytes};
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + 2 * a_bytes + 2 * b_bytes);  // [2]
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bar + 2);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int m0 = blockIdx.y * kM, n0 = blockIdx.x * g.ntile;
+  const int64_t kbeg = (int64_t)blockIdx.z * g.kper;
+  const int64_t kend = kbeg + g.kper < g.K ? kbeg + g.kper : g.K;
+  const int nchunks = kend > kbeg ? (int)((kend - kbeg + 63) / 64) : 0;
+
+  if (tid == 0) {
+    mbar_init(&bar[0], 1);
+    mbar_init(&bar[1], 1);
+    fence_mbar_init();
+  }
+  if (warp == 0) {
+    tmem_alloc(tmem_holder, g.tmem_cols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_holder;
+  const uint32_t idesc = idesc_bf16_f32(kM, g.ntile);
+  bool ok = true;
+
+  for (int c = 0; c < nchunks; ++c) {
+    const int b = c & 1;
+    if (c >= 2 && !mbar_wait(&bar[b], (uint32_t)(((c - 2) >> 1) & 1))) ok = false;
+    const int64_t k0 = kbeg + (int64_t)c * 64;
+    stage(As[b], kM, g.A, g.sam, g.sak, m0, g.M, k0, kend);
+    stage(Bs[b], g.ntile, g.B, g.sbn, g.sbk, n0, g.N, k0, kend);
+    fence_async_smem();
+    __syncthreads();
+    if (tid == 0) {
+      tc_fence_after();
+      const uint32_t ab = smem_u32(As[b]), bb = smem_u32(Bs[b]);
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        umma_bf16(tmem, sdesc_sw128(ab + 32u * j), sdesc_sw128(bb + 32u * j), idesc, (c | j) ? 1u : 0u);
+      umma_commit(&bar[b]);
+    }
+    __syncwarp();
+  }
+  if (nchunks > 0) {
+    const int b = (nchunks - 1) & 1;
+    if (!mbar_wait(&bar[b], (uint32_t)(((nchunks - 1) >> 1) & 1))) ok = false;
+    // the other buffer's last commit (if any) completed before this one
+  }
+  if (!ok) latch_error(g.err, LS_ERR_TIMEOUT);
+  tc_fence_after();
+
+  const int q4 = warp & 3, ch = warp >> 2;
+  const int row = m0 + 32 * q4 + lane;
+  const int half = g.ntile / 2;
+  const uint32_t lane_addr = (uint32_t)(32 * q4) << 16;
+  for (int c0 = ch * half; c0 < (ch + 1) * half; c0 += 16) {
+    uint32_t v[16];
+    if (nchunks > 0) {
+      tmem_ld16(tmem + lane_addr + (uint32_t)c0, v);
+      tmem_wait_ld();
+    } else {
+#pragma unroll
+      for (int j = 0; j < 16; ++j) v[j] = 0u;
+    }
+    if (row >= g.M) continue;
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      const int n = n0 + c0 + j;
+      if (n >= g.N) break;
+      const float acc = __uint_as_float(v[j]);
+      if (g.epi == 0) {
+        g.C[(int64_t)blockIdx.z * g.split_stride + (int64_t)row * g.ldc + n] = acc;
+      } else if (g.epi == 1) {
+        const float z = acc + __ldg(g.bias + n);
+        g.C[(int64_t)row * g.ldc + n] = z;
+        if (g.hidden) g.act[(int64_t)row * g.ld_act + n] = round_bf16(z > 0.0f ? z : 0.0f);
+      } else {
+        g.C[(int64_t)row * g.ldc + n] = __ldg(g.zprev + (int64_t)row * g.ld_zprev + n) > 0.0f ? acc : 0.0f;
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tmem, g.tmem_cols);
+}
+
+}  // namespace
+
+// Picks the tile width and launches; returns cudaErrorInvalidValue when the
+// shape is not worth a tensor-core tile (the caller then uses CUDA cores).
+cudaError_t launch_gemm_tc(int M, int N, int K, const float* A, int64_t sam, int64_t sak, const float* B,
+                           int64_t sbn, int64_t sbk, int splits, int epi, float* C, int64_t ldc,
+                           int64_t split_stride, const float* bias, float* act, int64_t ld_act, int hidden,
+                           const float* zprev, int64_t ld_zprev, int* err, int sms, cudaStream_t s) {
+  if (M < 64 || N < 32 || K < 1) return cudaErrorInvalidValue;
+  const int mt = (M + kM - 1) / kM;
+  int ntile = 256;
+  while (ntile > 64 && (int64_t)mt * ((N + ntile - 1) / ntile) * splits < sms) ntile /= 2;
+  if (ntile > ((N + 31) / 32) * 32) ntile = ((N + 31) / 32) * 32;
+  TcGemmArgs g{};
+  g.M = M; g.N = N; g.K = K;
+  g.A = A; g.sam = sam; g.sak = sak;
+  g.B = B; g.sbn = sbn; g.sbk = sbk;
+  g.ntile = ntile;
+  g.kper = (int)((((int64_t)K + splits - 1) / splits + 63) / 64 * 64);
+  g.epi = epi;
+  g.C = C; g.ldc = ldc; g.split_stride = split_stride;
+  g.bias = bias; g.act = act; g.ld_act = ld_act; g.hidden = hidden;
+  g.zprev = zprev; g.ld_zprev = ld_zprev;
+  g.err = err;
+  g.tmem_cols = 32;
+  while ((int)g.tmem_cols < ntile) g.tmem_cols <<= 1;
+  const int zs = (int)(((int64_t)K + g.kper - 1) / g.kper);
+  const int smem = 1024 + 2 * kM * 128 + 2 * ntile * 128 + 64;
+  cudaError_t e = cudaFuncSetAttribute(k_gemm_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  dim3 grid((N + ntile - 1) / ntile, mt, zs);
+  k_gemm_tc<<<grid, kT, smem, s>>>(g);
+  return cudaGetLastError();
+}
+
+int gemm_tc_splits_used(int K, int splits) {
+  const int64_t kper = ((((int64_t)K + splits - 1) / splits + 63) / 64) * 64;
+  return (int)(((int64_t)K + kper - 1) / kper);
+}
+
+}  // namespace ls

@@ -147,11 +147,18 @@ def test_batch_over_token_capacity_is_latched_not_faulted():
     dw.load(small)
     small.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)   # ~20k tokens > 1000
     assert small.sync() == L.LS_ERR_ARG
-    n = 3                                                           # a batch that fits
-    ok = small.route(dw.tok, dw.tok_off[:n + 1], dw.req_feats[:n], wl.cfg.n_inst)
+    # a batch that fits, taken from the middle of the token buffer (slots are
+    # relative to the batch's first offset)
+    off = wl.tok_off
+    a = 10
+    b = a + 1
+    while b < len(off) - 1 and off[b + 1] - off[a] <= 1000:
+        b += 1
+    sub = dw.tok_off[a:b + 1]
+    ok = small.route(dw.tok, sub, dw.req_feats[a:b], wl.cfg.n_inst)
     assert small.sync() == L.LS_OK
-    ref = r.route(dw.tok, dw.tok_off[:n + 1], dw.req_feats[:n], wl.cfg.n_inst)
-    assert torch.equal(ok["hits"], ref["hits"])
+    ref = r.route(dw.tok, sub, dw.req_feats[a:b], wl.cfg.n_inst)
+    assert torch.equal(ok["hits"], ref["hits"]) and torch.equal(ok["scores"], ref["scores"])
     small.close()
 
 
