@@ -55,7 +55,7 @@ enum { LS_F32 = 0, LS_BF16 = 1 };      /* predictor arithmetic */
 enum { LS_REPLACE = 0, LS_INSERT = 1 };/* ls_snapshot_update key modes */
 enum { LS_SGD = 0, LS_ADAM = 1 };      /* ls_train_step optimisers */
 enum { LS_SCORER_AUTO = 0, LS_SCORER_CUDA_CORES = 1, LS_SCORER_TENSOR_CORES = 2 };
-enum { LS_PREFIX_AUTO = 0, LS_PREFIX_TWO_PHASE = 1, LS_PREFIX_FUSED = 2 };
+enum { LS_PREFIX_AUTO = 0, LS_PREFIX_TWO_PHASE = 1, LS_PREFIX_FUSED = 2, LS_PREFIX_INDEX = 3 };
 
 /* Predictor and capacity configuration, fixed at ls_create.
  * widths[0] = d = 6 + d_inst + d_req (pair features, instance state, request
@@ -74,10 +74,15 @@ typedef struct {
     int32_t max_train_batch;
     int64_t max_batch_tokens;            /* prompt tokens per ls_route_batch call (sizes the
                                             block-key scratch; more latches LS_ERR_ARG) */
-    int32_t prefix_mode;                 /* LS_PREFIX_*: TWO_PHASE (AUTO) hashes every block,
-                                            then screens block 0 per pair and walks the
-                                            survivors; FUSED hashes and probes per request and
-                                            stops hashing once no instance still matches */
+    int32_t prefix_mode;                 /* LS_PREFIX_*: INDEX keeps one table over all
+                                            instances (key -> instance bitmask; needs
+                                            max_instances <= 512) and looks each block up once
+                                            per request, stopping once no instance matches;
+                                            TWO_PHASE hashes every block, then screens block 0
+                                            per pair and walks the survivors in per-instance
+                                            tables; FUSED probes per-instance tables per request
+                                            with early exit.  AUTO = INDEX when possible, else
+                                            TWO_PHASE.  All modes give identical hits. */
     int32_t scorer;                      /* LS_SCORER_*: AUTO picks the tensor-core scorer
                                             for bf16 predictors whose hidden widths are
                                             multiples of 64 (<= 512), CUDA cores otherwise;

@@ -14,7 +14,8 @@ const char* const kTraceNames[TR_COUNT] = {
     "hash_blocks", "table_insert", "prefix_match", "score_simt", "argmin", "assemble_features",
     "ring_append", "publish", "train_gather", "gemm_fwd", "loss_grad", "gemm_dw", "reduce_dw",
     "colsum_db", "gemm_dx", "optimizer", "memset", "score_tc", "norm_rows", "publish_tc",
-    "hash_screen", "probe_screen", "probe_walk", "gemm_tc_fwd", "gemm_tc_dw", "gemm_tc_dx"};
+    "hash_screen", "probe_screen", "probe_walk", "gemm_tc_fwd", "gemm_tc_dw", "gemm_tc_dx", "prefix_index",
+    "index_insert"};
 }
 
 struct ls_ctx {
@@ -68,7 +69,11 @@ bool check_config(const ls_config* c, std::string& why) {
   if (c->ring_capacity < 1) { why = "ring_capacity must be >= 1"; return false; }
   if (c->max_train_batch < 1) { why = "max_train_batch must be >= 1"; return false; }
   if (c->scorer < LS_SCORER_AUTO || c->scorer > LS_SCORER_TENSOR_CORES) { why = "bad scorer"; return false; }
-  if (c->prefix_mode < LS_PREFIX_AUTO || c->prefix_mode > LS_PREFIX_FUSED) { why = "bad prefix_mode"; return false; }
+  if (c->prefix_mode < LS_PREFIX_AUTO || c->prefix_mode > LS_PREFIX_INDEX) { why = "bad prefix_mode"; return false; }
+  if (c->prefix_mode == LS_PREFIX_INDEX && c->max_instances > 512) {
+    why = "prefix_mode INDEX needs max_instances <= 512";
+    return false;
+  }
   if (c->max_batch_tokens < 1) { why = "max_batch_tokens must be >= 1"; return false; }
   const double need = std::ceil((double)c->max_keys_per_instance / (double)c->max_load);
   if (need > (double)(1ull << 31)) { why = "table would exceed 2^31 slots"; return false; }
@@ -94,7 +99,7 @@ void free_all(Ctx& c) {
                   c.adam_v, c.pub[0].params, c.pub[0].wt, c.pub[1].params, c.pub[1].wt,
                   c.ring_x, c.ring_y, c.hits, c.scores, c.tx, c.tz, c.ty, c.dz0, c.dz1, c.grad,
                   c.gpart, c.loss_tmp, c.d_err, c.pub[0].img, c.pub[1].img, c.xin, c.xrq,
-                  c.bkeys, c.work, c.work_n};
+                  c.bkeys, c.work, c.work_n, c.gkeys, c.gmask};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   for (int b = 0; b < 2; ++b) {
@@ -171,7 +176,19 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
   }
   cudaError_t e = cudaSuccess;
   auto A = [&](cudaError_t r) { if (e == cudaSuccess) e = r; };
-  A(dalloc(&c.tables, NI * c.slots));
+  c.use_index = cfg->prefix_mode == LS_PREFIX_INDEX ||
+                (cfg->prefix_mode == LS_PREFIX_AUTO && cfg->max_instances <= 512);
+  if (c.use_index) {
+    c.gW = index_words(cfg->max_instances);
+    const double need = std::ceil((double)cfg->max_instances * (double)cfg->max_keys_per_instance /
+                                  (double)cfg->max_load);
+    c.gslots = 16;
+    while ((double)c.gslots < need) c.gslots <<= 1;
+    A(dalloc(&c.gkeys, c.gslots));
+    A(dalloc(&c.gmask, c.gslots * c.gW));
+  } else {
+    A(dalloc(&c.tables, NI * c.slots));
+  }
   A(dalloc(&c.table_count, NI));
   A(dalloc(&c.inst_state, NI * std::max(1, cfg->d_inst)));
   A(dalloc(&c.mean, c.d));
@@ -185,7 +202,7 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
     if (c.use_tc) A(dalloc(&c.pub[b].img, c.tc.img_bytes));
   }
   c.bkeys_cap = cfg->max_batch_tokens / kBlockTok + 1;
-  if (cfg->prefix_mode != LS_PREFIX_FUSED) {
+  if (!c.use_index && cfg->prefix_mode != LS_PREFIX_FUSED) {
     A(dalloc(&c.bkeys, c.bkeys_cap));
     A(dalloc(&c.work, R * NI));
   }
@@ -211,7 +228,9 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
     A(cudaEventCreateWithFlags(&c.route_done[b], cudaEventDisableTiming));
   }
   if (e == cudaSuccess) {
-    A(cudaMemset(c.tables, 0, (size_t)NI * c.slots * sizeof(uint64_t)));
+    if (c.tables) A(cudaMemset(c.tables, 0, (size_t)NI * c.slots * sizeof(uint64_t)));
+    if (c.gkeys) A(cudaMemset(c.gkeys, 0, (size_t)c.gslots * sizeof(uint64_t)));
+    if (c.gmask) A(cudaMemset(c.gmask, 0, (size_t)c.gslots * c.gW * sizeof(uint64_t)));
     A(cudaMemset(c.table_count, 0, (size_t)NI * sizeof(int32_t)));
     A(cudaMemset(c.adam_m, 0, (size_t)c.n_params * sizeof(float)));
     A(cudaMemset(c.adam_v, 0, (size_t)c.n_params * sizeof(float)));
@@ -253,7 +272,7 @@ int ls_get_info(ls_ctx* h, ls_info* out) {
   out->n_inst = c.n_inst;
   out->d = c.d;
   out->n_params = c.n_params;
-  out->table_slots = c.slots;
+  out->table_slots = c.use_index ? c.gslots : c.slots;
   out->ring_count = c.ring_count;
   out->train_steps = c.step;
   out->weight_version = c.version;
@@ -322,7 +341,19 @@ int ls_snapshot_update(ls_ctx* h, int32_t n_inst, const float* inst_state, const
   if (c.cfg.d_inst > 0)
     LS_CK(cudaMemcpyAsync(c.inst_state, inst_state, (size_t)n_inst * c.cfg.d_inst * sizeof(float),
                           cudaMemcpyDeviceToDevice, S(stream)));
-  if (keys) {
+  if (keys && c.use_index) {
+    if (mode == LS_REPLACE) {
+      // the index holds every instance: replacing the listed instances
+      // (all of the snapshot) rebuilds it
+      LS_CK(cudaMemsetAsync(c.gkeys, 0, (size_t)c.gslots * sizeof(uint64_t), S(stream)));
+      LS_CK(cudaMemsetAsync(c.gmask, 0, (size_t)c.gslots * c.gW * sizeof(uint64_t), S(stream)));
+      LS_CK(cudaMemsetAsync(c.table_count, 0, (size_t)c.cfg.max_instances * sizeof(int32_t), S(stream)));
+    }
+    LS_CK(traced(c, TR_INDEX_INSERT, 1, S(stream), [&] {
+      return launch_index_insert(keys, key_off, n_inst, n_keys, c.gkeys, c.gmask, c.gW, (uint64_t)(c.gslots - 1),
+                                 c.table_count, c.cfg.max_keys_per_instance, c.d_err, c.sms, S(stream));
+    }));
+  } else if (keys) {
     if (mode == LS_REPLACE) {
       LS_CK(cudaMemsetAsync(c.tables, 0, (size_t)n_inst * c.slots * sizeof(uint64_t), S(stream)));
       LS_CK(cudaMemsetAsync(c.table_count, 0, (size_t)n_inst * sizeof(int32_t), S(stream)));
@@ -389,7 +420,12 @@ int ls_route_batch(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* 
   if (n_req == 0) return LS_OK;
   int32_t* hits = hits_opt ? hits_opt : c.hits;
   float* scores = scores_opt ? scores_opt : c.scores;
-  if (c.cfg.prefix_mode == LS_PREFIX_FUSED) {
+  if (c.use_index) {
+    LS_CK(traced(c, TR_PREFIX_INDEX, 1, s, [&] {
+      return launch_prefix_index(n_req, tok, tok_off, c.gkeys, c.gmask, c.gW, (uint64_t)(c.gslots - 1), c.n_inst,
+                                 hits, c.sms, s);
+    }));
+  } else if (c.cfg.prefix_mode == LS_PREFIX_FUSED) {
     LS_CK(traced(c, TR_PREFIX, 1, s, [&] {
       return launch_prefix_match(n_req, tok, tok_off, c.tables, c.mask, c.slots, c.n_inst, hits, s);
     }));

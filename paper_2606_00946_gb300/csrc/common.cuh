@@ -67,7 +67,7 @@ enum TraceId {
   TR_HASH, TR_INSERT, TR_PREFIX, TR_SCORE, TR_ARGMIN, TR_ASSEMBLE, TR_RING, TR_PUBLISH,
   TR_GATHER, TR_GEMM_FWD, TR_LOSS, TR_GEMM_DW, TR_REDUCE, TR_COLSUM, TR_GEMM_DX, TR_OPT,
   TR_MEMSET, TR_SCORE_TC, TR_NORM_ROWS, TR_PUBLISH_TC, TR_HASH_BATCH, TR_SCREEN, TR_WALK,
-  TR_GEMM_TC_FWD, TR_GEMM_TC_DW, TR_GEMM_TC_DX, TR_COUNT
+  TR_GEMM_TC_FWD, TR_GEMM_TC_DW, TR_GEMM_TC_DX, TR_PREFIX_INDEX, TR_INDEX_INSERT, TR_COUNT
 };
 extern const char* const kTraceNames[TR_COUNT];
 
@@ -143,6 +143,12 @@ struct Ctx {
   // route scratch
   int32_t* hits = nullptr;    // [max_requests, max_instances]
   float* scores = nullptr;    // [max_requests, max_instances]
+  // prefix index over all instances (LS_PREFIX_INDEX): key -> instance bitmask
+  bool use_index = false;
+  int gW = 0;                 // 64-bit mask words per slot
+  int64_t gslots = 0;
+  uint64_t* gkeys = nullptr;  // [gslots]
+  uint64_t* gmask = nullptr;  // [gslots, gW]
   uint64_t* bkeys = nullptr;  // block keys of the batch, slot tok_off[r]/16 + b
   int64_t bkeys_cap = 0;
   uint32_t* work = nullptr;   // (request, instance) pairs that hit block 0
@@ -265,5 +271,12 @@ cudaError_t launch_gemm_tc(int M, int N, int K, const float* A, int64_t sam, int
                            int64_t split_stride, const float* bias, float* act, int64_t ld_act, int hidden,
                            const float* zprev, int64_t ld_zprev, int* err, int sms, cudaStream_t s);
 int gemm_tc_splits_used(int K, int splits);
+int index_words(int max_instances);
+cudaError_t launch_prefix_index(int n_req, const int32_t* tok, const int64_t* tok_off, const uint64_t* gkeys,
+                                const uint64_t* gmask, int W, uint64_t gmask_slots, int n_inst, int32_t* hits,
+                                int sms, cudaStream_t s);
+cudaError_t launch_index_insert(const uint64_t* keys, const int64_t* key_off, int n_inst, int64_t n_keys,
+                                uint64_t* gkeys, uint64_t* gmask, int W, uint64_t gmask_slots, int32_t* counts,
+                                int64_t max_keys, int* err, int sms, cudaStream_t s);
 
 }  // namespace ls

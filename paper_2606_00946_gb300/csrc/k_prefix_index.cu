@@ -1,0 +1,197 @@
+// Prefix index over all instances: one open-addressing table maps a block key
+// to the bitmask of instances whose cache holds that block (the gateway's
+// single logical prefix index of Sec. 4.2, in hash-table form as Sec. 2
+// allows).  Hit lengths then need one lookup per (request, block) instead of
+// one per (request, block, instance):
+//   alive_b = AND_{b' <= b} mask(key_b')   (bits of instances still matching)
+//   h_i     = number of leading blocks b with bit i of alive_b set
+// which is exactly "leading blocks all cached on instance i, stop at the first
+// miss" (Sec. 2: prefix reuse is strictly sequential).
+//
+// One CTA per request hashes its prompt 128 blocks at a time; warp 0 walks
+// the chunk 32 blocks per round: each lane looks up one block's mask, a
+// warp-wide prefix AND gives alive_b per lane, and an instance that stops
+// matching in the round gets h from one ballot.  Hashing stops as soon as no
+// instance matches, so tokens past the longest hit are never read.
+#include "blockhash.cuh"
+
+namespace ls {
+namespace {
+using namespace bh;
+
+constexpr int kNT = 128;
+
+// Slot of `key` in the index (linear probing in aligned 4-slot buckets), -1 if absent.
+__device__ __forceinline__ int64_t index_find(const uint64_t* __restrict__ gkeys, uint64_t gmask_slots,
+                                              uint64_t key) {
+  uint64_t s = key & gmask_slots;
+  uint32_t first = (uint32_t)(s & 3u);
+  uint64_t b = s & ~(uint64_t)3;
+  for (uint64_t n = 0; n <= (gmask_slots >> 2) + 1; ++n) {
+    const ulonglong2* q = reinterpret_cast<const ulonglong2*>(gkeys + b);
+    const ulonglong2 v01 = __ldg(q), v23 = __ldg(q + 1);
+    const uint64_t v[4] = {v01.x, v01.y, v23.x, v23.y};
+#pragma unroll
+    for (uint32_t j = 0; j < 4; ++j) {
+      if (j < first) continue;
+      if (v[j] == key) return (int64_t)(b + j);
+      if (v[j] == 0) return -1;
+    }
+    first = 0;
+    b = (b + 4) & gmask_slots;
+  }
+  return -1;
+}
+
+template <int W>
+__global__ void __launch_bounds__(kNT) k_prefix_index(int n_req, const int32_t* __restrict__ tok,
+                                                      const int64_t* __restrict__ tok_off,
+                                                      const uint64_t* __restrict__ gkeys,
+                                                      const uint64_t* __restrict__ gmask, uint64_t gmask_slots,
+                                                      int n_inst, int32_t* __restrict__ hits) {
+  __shared__ uint64_t keys[kNT];
+  __shared__ uint64_t wtot[kNT / 32], wpre[kNT / 32], carry;
+  __shared__ int any_alive;
+  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+  for (int r = blockIdx.x; r < n_req; r += gridDim.x) {
+    const int64_t t0 = tok_off[r];
+    const int64_t nb = (tok_off[r + 1] - t0) / kBlockTok;
+    const int32_t* base = tok + t0;
+    const bool aligned = ((reinterpret_cast<uintptr_t>(base) & 15) == 0);
+    int32_t* hrow = hits + (int64_t)r * n_inst;
+    uint64_t alive[W];
+#pragma unroll
+    for (int w = 0; w < W; ++w) {
+      const int lo = 64 * w;
+      alive[w] = n_inst >= lo + 64 ? ~0ull : (n_inst > lo ? ((1ull << (n_inst - lo)) - 1ull) : 0ull);
+    }
+    if (t == 0) {
+      carry = kG;
+      any_alive = n_inst > 0;
+    }
+    __syncthreads();
+    for (int64_t c0 = 0; c0 < nb; c0 += kNT) {
+      if (!any_alive) break;  // uniform: read after a barrier
+      const int n = (int)(nb - c0 < kNT ? nb - c0 : kNT);
+      const uint64_t s_in = carry;
+      const uint64_t c = t < n ? block_content(base + (c0 + t) * kBlockTok, aligned) : 0ull;
+      const uint64_t st = chain_scan<kNT>(c, s_in, wtot, wpre);
+      if (t < n) keys[t] = key_of(st);
+      if (t == n - 1) carry = st;
+      __syncthreads();
+      if (warp == 0) {
+        bool any = true;
+        for (int p = 0; p < n && any; p += 32) {
+          const int b = p + lane;
+          uint64_t pa[W];
+          if (b < n) {
+            const int64_t slot = index_find(gkeys, gmask_slots, keys[b]);
+#pragma unroll
+            for (int w = 0; w < W; ++w) pa[w] = slot >= 0 ? __ldg(gmask + slot * W + w) : 0ull;
+          } else {
+#pragma unroll
+            for (int w = 0; w < W; ++w) pa[w] = 0ull;
+          }
+          any = false;
+#pragma unroll
+          for (int w = 0; w < W; ++w) {
+            uint64_t x = pa[w];
+#pragma unroll
+            for (int k = 0; k < 5; ++k) {
+              const uint64_t y = __shfl_up_sync(kFull, x, 1 << k);
+              if (lane >= (1 << k)) x &= y;
+            }
+            x &= alive[w];
+            const uint64_t end = __shfl_sync(kFull, x, 31);
+            uint64_t died = alive[w] & ~end;
+            while (died) {
+              const int bit = __ffsll((long long)died) - 1;
+              const int cnt = __popc(__ballot_sync(kFull, (x >> bit) & 1ull));
+              if (lane == 0) hrow[64 * w + bit] = (int32_t)(c0 + p + cnt);
+              died &= died - 1;
+            }
+            alive[w] = end;
+            any = any || end != 0;
+          }
+        }
+        if (lane == 0) any_alive = any;
+      }
+      __syncthreads();
+    }
+    if (warp == 0) {
+      // instances matching every full block (or requests without a full block)
+#pragma unroll
+      for (int w = 0; w < W; ++w)
+        for (int bit = lane; bit < 64; bit += 32)
+          if ((alive[w] >> bit) & 1ull) hrow[64 * w + bit] = (int32_t)nb;
+    }
+    __syncthreads();
+  }
+}
+
+// Insert (instance, key) pairs: thread per key, instance by binary search in
+// key_off.  A new key takes a slot (CAS on 0); the instance's bit is OR-ed into
+// the slot's mask; a bit set for the first time counts one distinct key of
+// that instance (more than max_keys latches LS_ERR_TABLE_FULL, as does a
+// probe sequence that finds no room).
+__global__ void k_index_insert(const uint64_t* __restrict__ keys, const int64_t* __restrict__ key_off,
+                               int n_inst, int64_t n_keys, uint64_t* gkeys, uint64_t* gmask, int W,
+                               uint64_t gmask_slots, int32_t* counts, int64_t max_keys, int* err) {
+  for (int64_t k = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; k < n_keys;
+       k += (int64_t)gridDim.x * blockDim.x) {
+    int lo = 0, hi = n_inst - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (key_off[mid] <= k) lo = mid; else hi = mid - 1;
+    }
+    uint64_t key = keys[k];
+    if (key == 0) key = 1;
+    unsigned long long* tab = reinterpret_cast<unsigned long long*>(gkeys);
+    uint64_t s = key & gmask_slots;
+    int64_t slot = -1;
+    for (uint64_t n = 0; n <= gmask_slots; ++n) {
+      const unsigned long long prev = atomicCAS(tab + s, 0ull, (unsigned long long)key);
+      if (prev == 0ull || prev == key) { slot = (int64_t)s; break; }
+      s = (s + 1) & gmask_slots;
+    }
+    if (slot < 0) { latch_error(err, LS_ERR_TABLE_FULL); continue; }
+    const unsigned long long bit = 1ull << (lo & 63);
+    const unsigned long long old =
+        atomicOr(reinterpret_cast<unsigned long long*>(gmask + slot * W + (lo >> 6)), bit);
+    if (!(old & bit)) {
+      const int cnt = atomicAdd(counts + lo, 1);
+      if (cnt >= max_keys) latch_error(err, LS_ERR_TABLE_FULL);
+    }
+  }
+}
+
+}  // namespace
+
+int index_words(int max_instances) { return max_instances <= 64 ? 1 : max_instances <= 128 ? 2 : max_instances <= 256 ? 4 : max_instances <= 512 ? 8 : 0; }
+
+cudaError_t launch_prefix_index(int n_req, const int32_t* tok, const int64_t* tok_off, const uint64_t* gkeys,
+                                const uint64_t* gmask, int W, uint64_t gmask_slots, int n_inst, int32_t* hits,
+                                int sms, cudaStream_t s) {
+  if (n_req <= 0) return cudaSuccess;
+  const int grid = std::min(n_req, sms * 16);
+  switch (W) {
+    case 1: k_prefix_index<1><<<grid, kNT, 0, s>>>(n_req, tok, tok_off, gkeys, gmask, gmask_slots, n_inst, hits); break;
+    case 2: k_prefix_index<2><<<grid, kNT, 0, s>>>(n_req, tok, tok_off, gkeys, gmask, gmask_slots, n_inst, hits); break;
+    case 4: k_prefix_index<4><<<grid, kNT, 0, s>>>(n_req, tok, tok_off, gkeys, gmask, gmask_slots, n_inst, hits); break;
+    case 8: k_prefix_index<8><<<grid, kNT, 0, s>>>(n_req, tok, tok_off, gkeys, gmask, gmask_slots, n_inst, hits); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_index_insert(const uint64_t* keys, const int64_t* key_off, int n_inst, int64_t n_keys,
+                                uint64_t* gkeys, uint64_t* gmask, int W, uint64_t gmask_slots, int32_t* counts,
+                                int64_t max_keys, int* err, int sms, cudaStream_t s) {
+  if (n_keys <= 0 || n_inst <= 0) return cudaSuccess;
+  const int64_t blocks = std::min<int64_t>((n_keys + 255) / 256, (int64_t)sms * 32);
+  k_index_insert<<<(int)blocks, 256, 0, s>>>(keys, key_off, n_inst, n_keys, gkeys, gmask, W, gmask_slots, counts,
+                                             max_keys, err);
+  return cudaGetLastError();
+}
+
+}  // namespace ls

@@ -66,15 +66,27 @@ __device__ __forceinline__ void st_shared_v4(uint8_t* p, uint32_t a, uint32_t b,
 // normalised values at their feature positions and zeros elsewhere, so a
 // 16-byte chunk of a feature row is the OR of the two templates' chunks (the
 // pair features, computed here, only occupy chunk 0).
-__device__ __forceinline__ void build_features(const TcArgs& a, uint8_t* A, int64_t row0) {
+__device__ __forceinline__ void build_features(const TcArgs& a, uint8_t* A, int64_t row0, const float (&mu)[kPair],
+                                               const float (&sd)[kPair]) {
   const int cpr = a.p.d_pad / 8;  // 16-byte chunks per row
+  const int total = kTileM * cpr;
   const int64_t r0 = row0 / a.n_inst;
   const int i0 = (int)(row0 - r0 * a.n_inst);
-  for (int e = threadIdx.x; e < kTileM * cpr; e += kThreadsTc) {
-    const int m = e / cpr, c = e - m * cpr;
-    const int64_t g = row0 + m;
-    uint4 v = make_uint4(0u, 0u, 0u, 0u);
-    if (g < a.rows) {
+  constexpr int U = 4;  // chunks per thread per pass; all their loads are issued first
+  for (int base = 0; base < total; base += U * kThreadsTc) {
+    uint4 ti[U], tr[U];
+    int64_t L[U];
+    int h[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int e = base + u * kThreadsTc + threadIdx.x;
+      ti[u] = tr[u] = make_uint4(0u, 0u, 0u, 0u);
+      L[u] = 0;
+      h[u] = 0;
+      if (e >= total) continue;
+      const int m = e / cpr, c = e - m * cpr;
+      const int64_t g = row0 + m;
+      if (g >= a.rows) continue;
       int i = i0 + m;
       int64_t r = r0;
       if (a.n_inst >= 16) {
@@ -83,22 +95,29 @@ __device__ __forceinline__ void build_features(const TcArgs& a, uint8_t* A, int6
         r += i / a.n_inst;
         i -= (i / a.n_inst) * a.n_inst;
       }
-      const uint4 ti = __ldg(reinterpret_cast<const uint4*>(a.xin + (int64_t)i * a.p.d_pad) + c);
-      const uint4 tr = __ldg(reinterpret_cast<const uint4*>(a.xrq + r * a.p.d_pad) + c);
-      v = make_uint4(ti.x | tr.x, ti.y | tr.y, ti.z | tr.z, ti.w | tr.w);
+      ti[u] = __ldg(reinterpret_cast<const uint4*>(a.xin + (int64_t)i * a.p.d_pad) + c);
+      tr[u] = __ldg(reinterpret_cast<const uint4*>(a.xrq + r * a.p.d_pad) + c);
       if (c == 0) {
-        const int64_t L = a.tok_off[r + 1] - a.tok_off[r];
-        const int h = a.hits[g];
+        L[u] = __ldg(a.tok_off + r + 1) - __ldg(a.tok_off + r);
+        h[u] = __ldg(a.hits + g);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int e = base + u * kThreadsTc + threadIdx.x;
+      if (e >= total) continue;
+      const int m = e / cpr, c = e - m * cpr;
+      uint4 v = make_uint4(ti[u].x | tr[u].x, ti[u].y | tr[u].y, ti[u].z | tr[u].z, ti[u].w | tr[u].w);
+      if (c == 0 && row0 + m < a.rows) {
         uint16_t f[kPair];
 #pragma unroll
-        for (int k = 0; k < kPair; ++k)
-          f[k] = bf16_bits(zscore(raw_feature(k, L, h, nullptr, 0, nullptr), a.mean[k], a.stdv[k]));
+        for (int k = 0; k < kPair; ++k) f[k] = bf16_bits(zscore(raw_feature(k, L[u], h[u], nullptr, 0, nullptr), mu[k], sd[k]));
         v.x = f[0] | ((uint32_t)f[1] << 16);
         v.y = f[2] | ((uint32_t)f[3] << 16);
         v.z = f[4] | ((uint32_t)f[5] << 16);
       }
+      st_shared_v4(A + sw128_offset(m, c * 8, kTileM), v.x, v.y, v.z, v.w);
     }
-    st_shared_v4(A + sw128_offset(m, c * 8, kTileM), v.x, v.y, v.z, v.w);
   }
 }
 
@@ -176,6 +195,12 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc(const __grid_constan
     }
   }
   uint32_t done_phase = 0;
+  float mu[kPair], sd[kPair];
+#pragma unroll
+  for (int k = 0; k < kPair; ++k) {
+    mu[k] = __ldg(a.mean + k);
+    sd[k] = __ldg(a.stdv + k);
+  }
   const int q4 = warp & 3;   // TMEM lane quadrant: rows 32*q4 .. 32*q4+31
   const int cq = warp >> 2;  // column quarter handled by this warp
   const int row = 32 * q4 + lane;
@@ -183,7 +208,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc(const __grid_constan
 
   for (int it = 0; it < my_tiles; ++it) {
     const int64_t row0 = (int64_t)(blockIdx.x + (int64_t)it * gridDim.x) * kTileM;
-    build_features(a, A, row0);
+    build_features(a, A, row0, mu, sd);
     fence_async_smem();
     __syncthreads();
     if (*abort_flag) break;

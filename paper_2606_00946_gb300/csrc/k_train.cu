@@ -174,6 +174,62 @@ __global__ void __launch_bounds__(256) k_colsum(int B, int out, int rows_per, co
   }
 }
 
+// Output layer (width 1) forward: z[j] = sum_k round(w[k]) a[j, k] + b, one
+// warp per row (a is already bf16-valued in bf16 mode).
+__global__ void k_out_fwd(int B, int K, const float* __restrict__ a, const float* __restrict__ w,
+                          const float* __restrict__ b, int bf16, float* __restrict__ z) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t j = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; j < B; j += warps) {
+    float s = 0.0f;
+    for (int k = lane; k < K; k += 32) {
+      const float wk = bf16 ? round_bf16(w[k]) : w[k];
+      s = fmaf(a[j * (int64_t)K + k], wk, s);
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if (lane == 0) z[j] = s + b[0];
+  }
+}
+
+// Output layer weight gradient, first stage: part[y][k] = sum over rows of
+// block y of round(dz[j]) a[j, k]; k_reduce_partials adds the partials.
+__global__ void __launch_bounds__(256) k_out_dw(int B, int K, int rows_per, const float* __restrict__ dz,
+                                                const float* __restrict__ a, int bf16,
+                                                float* __restrict__ part) {
+  __shared__ float red[8][33];
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+  const int k = blockIdx.x * 32 + tx;
+  const int j0 = blockIdx.y * rows_per, j1 = min(B, j0 + rows_per);
+  float s = 0.0f;
+  if (k < K)
+    for (int j = j0 + ty; j < j1; j += 8) {
+      const float g = bf16 ? round_bf16(dz[j]) : dz[j];
+      s = fmaf(g, a[(int64_t)j * K + k], s);
+    }
+  red[ty][tx] = s;
+  __syncthreads();
+  if (ty == 0 && k < K) {
+    float t = 0.0f;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) t += red[q][tx];
+    part[(int64_t)blockIdx.y * K + k] = t;
+  }
+}
+
+// Output layer input gradient: dz_prev[j, k] = round(dz[j]) round(w[k]) [z[j, k] > 0].
+__global__ void k_out_dx(int B, int K, const float* __restrict__ dz, const float* __restrict__ w,
+                         const float* __restrict__ zprev, int bf16, float* __restrict__ out) {
+  const int64_t n = (int64_t)B * K;
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n; e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t j = e / K;
+    const int k = (int)(e - j * K);
+    const float g = bf16 ? round_bf16(dz[j]) : dz[j];
+    const float wk = bf16 ? round_bf16(w[k]) : w[k];
+    out[e] = zprev[e] > 0.0f ? g * wk : 0.0f;
+  }
+}
+
 __global__ void k_reduce_partials(int S, int64_t n, const float* __restrict__ part,
                                   float* __restrict__ dst) {
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n;
@@ -259,7 +315,15 @@ cudaError_t run_train_step(Ctx& c, int B, const int32_t* idx, int opt, float lr,
     a.ld_act = m.w[l + 1];
     a.bf16 = m.bf16;
     bool done_tc = false;
-    if (m.bf16) {
+    if (m.w[l + 1] == 1) {
+      e = traced(c, TR_GEMM_FWD, 1, s, [&] {
+        const int grid = (int)std::min<int64_t>(((int64_t)B * 32 + 255) / 256, (int64_t)c.sms * 8);
+        k_out_fwd<<<grid, 256, 0, s>>>(B, m.w[l], a.A, a.B, a.bias, m.bf16, a.C);
+        return cudaGetLastError();
+      });
+      if (e != cudaSuccess) return e;
+      done_tc = true;
+    } else if (m.bf16) {
       e = traced(c, TR_GEMM_TC_FWD, 1, s, [&] {
         return launch_gemm_tc(a.M, a.N, a.K, a.A, a.lda, 1, a.B, a.ldb, 1, 1, 1, a.C, a.ldc, 0, a.bias, a.act,
                               a.ld_act, a.hidden, nullptr, 0, c.d_err, c.sms, s);
@@ -295,9 +359,19 @@ cudaError_t run_train_step(Ctx& c, int B, const int32_t* idx, int opt, float lr,
     const int Seff = (B + a.kchunk - 1) / a.kchunk;
     int nparts = Seff;
     bool dw_tc = false;
-    if (m.bf16) {
+    if (out == 1) {
+      const int S1 = std::max(1, std::min(64, B / 64));
+      const int rows_per = (B + S1 - 1) / S1;
+      e = traced(c, TR_GEMM_DW, 1, s, [&] {
+        k_out_dw<<<dim3((in + 31) / 32, S1), 256, 0, s>>>(B, in, rows_per, dz, c.tx + xoff[l], m.bf16, c.gpart);
+        return cudaGetLastError();
+      });
+      if (e != cudaSuccess) return e;
+      dw_tc = true;
+      nparts = S1;
+    } else if (m.bf16) {
       const int tiles = ((out + 127) / 128) * ((in + 127) / 128);
-      const int S_tc = std::max(1, std::min({64, B / 64, (2 * c.sms + tiles - 1) / tiles}));
+      const int S_tc = std::max(1, std::min({16, B / 64, (2 * c.sms + tiles - 1) / tiles}));
       e = traced(c, TR_GEMM_TC_DW, 1, s, [&] {
         return launch_gemm_tc(out, in, B, dz, 1, out, c.tx + xoff[l], 1, in, S_tc, 0, c.gpart, in,
                               (int64_t)out * in, nullptr, nullptr, 0, 0, nullptr, 0, c.d_err, c.sms, s);
@@ -342,7 +416,16 @@ cudaError_t run_train_step(Ctx& c, int B, const int32_t* idx, int opt, float lr,
       b.kchunk = ((out + 15) / 16) * 16;
       b.zprev = c.tz + zoff[l - 1]; b.ld_zprev = in;
       bool dx_tc = false;
-      if (m.bf16) {
+      if (out == 1) {
+        e = traced(c, TR_GEMM_DX, 1, s, [&] {
+          const int64_t n = (int64_t)B * in;
+          const int grid = (int)std::min<int64_t>((n + 255) / 256, (int64_t)c.sms * 8);
+          k_out_dx<<<grid, 256, 0, s>>>(B, in, dz, c.master + m.woff[l], c.tz + zoff[l - 1], m.bf16, dzn);
+          return cudaGetLastError();
+        });
+        if (e != cudaSuccess) return e;
+        dx_tc = true;
+      } else if (m.bf16) {
         e = traced(c, TR_GEMM_TC_DX, 1, s, [&] {
           return launch_gemm_tc(B, in, out, dz, out, 1, c.master + m.woff[l], 1, in, 1, 2, dzn, in, 0, nullptr,
                                 nullptr, 0, 0, c.tz + zoff[l - 1], in, c.d_err, c.sms, s);

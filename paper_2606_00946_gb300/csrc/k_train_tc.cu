@@ -50,31 +50,70 @@ __device__ __forceinline__ void sts32(uint8_t* p, uint32_t v) {
 
 // Stage rows [row0, row0 + R) x k [k0, k0 + 64) of a strided fp32 operand as
 // a bf16 [R x 64] K-major 128B-swizzled tile; out-of-range elements are 0.
-__device__ __forceinline__ void stage(uint8_t* tile, int R, const float* src, int64_t s_row, int64_t s_k,
-                                      int row0, int nrow, int64_t k0, int64_t kend) {
-  if (s_k == 1) {  // k contiguous: consecutive threads take consecutive k pairs of a row
-    for (int e = threadIdx.x; e < R * 32; e += kT) {
-      const int r = e >> 5, k = (e & 31) * 2;
+// Every thread first issues all of its loads (R/16 float4 or equivalent), then
+// converts and stores, so a chunk costs about one memory latency.
+template <int R>
+__device__ __forceinline__ void stage(uint8_t* tile, const float* src, int64_t s_row, int64_t s_k, int row0,
+                                      int nrow, int64_t k0, int64_t kend, bool vec) {
+  constexpr int PER = R * 16 / kT;  // float4-sized pieces per thread
+  if (s_k == 1) {
+    // piece = 4 consecutive k of one row: e -> (r = e / 16, q = e % 16)
+    float4 v[PER];
+#pragma unroll
+    for (int u = 0; u < PER; ++u) {
+      const int e = threadIdx.x + u * kT;
+      const int r = e >> 4, k = (e & 15) * 4;
       const int64_t kk = k0 + k;
-      float v0 = 0.0f, v1 = 0.0f;
+      v[u] = make_float4(0.f, 0.f, 0.f, 0.f);
       if (row0 + r < nrow) {
         const float* p = src + (int64_t)(row0 + r) * s_row + kk;
-        if (kk < kend) v0 = __ldg(p);
-        if (kk + 1 < kend) v1 = __ldg(p + 1);
+        if (vec && kk + 3 < kend) {
+          v[u] = __ldg(reinterpret_cast<const float4*>(p));
+        } else {
+          if (kk < kend) v[u].x = __ldg(p);
+          if (kk + 1 < kend) v[u].y = __ldg(p + 1);
+          if (kk + 2 < kend) v[u].z = __ldg(p + 2);
+          if (kk + 3 < kend) v[u].w = __ldg(p + 3);
+        }
       }
-      sts32(tile + sw128_offset(r, k, R), pack2(v0, v1));
     }
-  } else {  // rows contiguous: consecutive threads take consecutive rows
-    for (int e = threadIdx.x; e < R * 32; e += kT) {
-      const int r = e % R, k = (e / R) * 2;
+#pragma unroll
+    for (int u = 0; u < PER; ++u) {
+      const int e = threadIdx.x + u * kT;
+      const int r = e >> 4, k = (e & 15) * 4;
+      uint8_t* dst = tile + sw128_offset(r, k, R);
+      asm volatile("st.shared.v2.b32 [%0], {%1, %2};" ::"r"(smem_u32(dst)), "r"(pack2(v[u].x, v[u].y)),
+                   "r"(pack2(v[u].z, v[u].w))
+                   : "memory");
+    }
+  } else {
+    // rows contiguous: piece = k pair (k, k+1) of 2 consecutive rows:
+    // e -> (r = 2 * (e % (R/2)), k = 2 * (e / (R/2)))
+    float2 lo[PER], hi[PER];
+#pragma unroll
+    for (int u = 0; u < PER; ++u) {
+      const int e = threadIdx.x + u * kT;
+      const int r = 2 * (e % (R / 2)), k = 2 * (e / (R / 2));
       const int64_t kk = k0 + k;
-      float v0 = 0.0f, v1 = 0.0f;
-      if (row0 + r < nrow) {
-        const float* p = src + (int64_t)(row0 + r) * s_row + kk * s_k;
-        if (kk < kend) v0 = __ldg(p);
-        if (kk + 1 < kend) v1 = __ldg(p + s_k);
+      lo[u] = make_float2(0.f, 0.f);
+      hi[u] = make_float2(0.f, 0.f);
+      const float* p = src + (int64_t)(row0 + r) * s_row + kk * s_k;
+      const bool r0ok = row0 + r < nrow, r1ok = row0 + r + 1 < nrow;
+      if (kk < kend) {
+        if (r0ok) lo[u].x = __ldg(p);
+        if (r1ok) lo[u].y = __ldg(p + s_row);
       }
-      sts32(tile + sw128_offset(r, k, R), pack2(v0, v1));
+      if (kk + 1 < kend) {
+        if (r0ok) hi[u].x = __ldg(p + s_k);
+        if (r1ok) hi[u].y = __ldg(p + s_k + s_row);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < PER; ++u) {
+      const int e = threadIdx.x + u * kT;
+      const int r = 2 * (e % (R / 2)), k = 2 * (e / (R / 2));
+      sts32(tile + sw128_offset(r, k, R), pack2(lo[u].x, hi[u].x));
+      sts32(tile + sw128_offset(r + 1, k, R), pack2(lo[u].y, hi[u].y));
     }
   }
 }
@@ -88,10 +127,11 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
       : "r"(taddr));
 }
 
+template <int NTILE>
 __global__ void __launch_bounds__(kT) k_gemm_tc(const __grid_constant__ TcGemmArgs g) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const int a_bytes = kM * 128, b_bytes = g.ntile * 128;
+  const int a_bytes = kM * 128, b_bytes = NTILE * 128;
   uint8_t* As[2] = {smem, smem + a_bytes};
   uint8_t* Bs[2] = {smem + 2 * a_bytes, smem + 2 * a_bytes + b_bytes};
   uint64_t* bar = reinterpret_cast<uint64_t*>(smem + 2 * a_bytes + 2 * b_bytes);  // [2]
@@ -116,15 +156,17 @@ __global__ void __launch_bounds__(kT) k_gemm_tc(const __grid_constant__ TcGemmAr
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_holder;
-  const uint32_t idesc = idesc_bf16_f32(kM, g.ntile);
+  const uint32_t idesc = idesc_bf16_f32(kM, NTILE);
+  const bool vec_a = g.sak == 1 && (g.sam % 4) == 0 && (reinterpret_cast<uintptr_t>(g.A) & 15) == 0;
+  const bool vec_b = g.sbk == 1 && (g.sbn % 4) == 0 && (reinterpret_cast<uintptr_t>(g.B) & 15) == 0;
   bool ok = true;
 
   for (int c = 0; c < nchunks; ++c) {
     const int b = c & 1;
     if (c >= 2 && !mbar_wait(&bar[b], (uint32_t)(((c - 2) >> 1) & 1))) ok = false;
     const int64_t k0 = kbeg + (int64_t)c * 64;
-    stage(As[b], kM, g.A, g.sam, g.sak, m0, g.M, k0, kend);
-    stage(Bs[b], g.ntile, g.B, g.sbn, g.sbk, n0, g.N, k0, kend);
+    stage<kM>(As[b], g.A, g.sam, g.sak, m0, g.M, k0, kend, vec_a);
+    stage<NTILE>(Bs[b], g.B, g.sbn, g.sbk, n0, g.N, k0, kend, vec_b);
     fence_async_smem();
     __syncthreads();
     if (tid == 0) {
@@ -147,7 +189,7 @@ __global__ void __launch_bounds__(kT) k_gemm_tc(const __grid_constant__ TcGemmAr
 
   const int q4 = warp & 3, ch = warp >> 2;
   const int row = m0 + 32 * q4 + lane;
-  const int half = g.ntile / 2;
+  const int half = NTILE / 2;
   const uint32_t lane_addr = (uint32_t)(32 * q4) << 16;
   for (int c0 = ch * half; c0 < (ch + 1) * half; c0 += 16) {
     uint32_t v[16];
@@ -180,6 +222,14 @@ __global__ void __launch_bounds__(kT) k_gemm_tc(const __grid_constant__ TcGemmAr
   if (warp == 0) tmem_dealloc(tmem, g.tmem_cols);
 }
 
+template <int NTILE>
+cudaError_t run_tc(dim3 grid, int smem, const TcGemmArgs& g, cudaStream_t s) {
+  cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<NTILE>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  k_gemm_tc<NTILE><<<grid, kT, smem, s>>>(g);
+  return cudaGetLastError();
+}
+
 }  // namespace
 
 // Picks the tile width and launches; returns cudaErrorInvalidValue when the
@@ -192,7 +242,7 @@ cudaError_t launch_gemm_tc(int M, int N, int K, const float* A, int64_t sam, int
   const int mt = (M + kM - 1) / kM;
   int ntile = 256;
   while (ntile > 64 && (int64_t)mt * ((N + ntile - 1) / ntile) * splits < sms) ntile /= 2;
-  if (ntile > ((N + 31) / 32) * 32) ntile = ((N + 31) / 32) * 32;
+  while (ntile > 64 && ntile / 2 >= N) ntile /= 2;
   TcGemmArgs g{};
   g.M = M; g.N = N; g.K = K;
   g.A = A; g.sam = sam; g.sak = sak;
@@ -208,11 +258,15 @@ cudaError_t launch_gemm_tc(int M, int N, int K, const float* A, int64_t sam, int
   while ((int)g.tmem_cols < ntile) g.tmem_cols <<= 1;
   const int zs = (int)(((int64_t)K + g.kper - 1) / g.kper);
   const int smem = 1024 + 2 * kM * 128 + 2 * ntile * 128 + 64;
-  cudaError_t e = cudaFuncSetAttribute(k_gemm_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  if (e != cudaSuccess) return e;
   dim3 grid((N + ntile - 1) / ntile, mt, zs);
-  k_gemm_tc<<<grid, kT, smem, s>>>(g);
-  return cudaGetLastError();
+  cudaError_t e2 = cudaSuccess;
+  switch (ntile) {
+    case 256: e2 = run_tc<256>(grid, smem, g, s); break;
+    case 128: e2 = run_tc<128>(grid, smem, g, s); break;
+    case 64: e2 = run_tc<64>(grid, smem, g, s); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return e2;
 }
 
 int gemm_tc_splits_used(int K, int splits) {

@@ -21,8 +21,8 @@ LS_REPLACE, LS_INSERT = 0, 1
 LS_SGD, LS_ADAM = 0, 1
 LS_SCORER_AUTO, LS_SCORER_CUDA_CORES, LS_SCORER_TENSOR_CORES = 0, 1, 2
 SCORERS = {"auto": 0, "cuda_cores": 1, "tensor_cores": 2}
-LS_PREFIX_AUTO, LS_PREFIX_TWO_PHASE, LS_PREFIX_FUSED = 0, 1, 2
-PREFIX_MODES = {"auto": 0, "two_phase": 1, "fused": 2}
+LS_PREFIX_AUTO, LS_PREFIX_TWO_PHASE, LS_PREFIX_FUSED, LS_PREFIX_INDEX = 0, 1, 2, 3
+PREFIX_MODES = {"auto": 0, "two_phase": 1, "fused": 2, "index": 3}
 
 
 class ls_config(C.Structure):

@@ -83,3 +83,9 @@ def test_tensor_core_scorer_rejected_for_unsupported_predictors(lib):
     bad = _cfg()
     bad.scorer = 7
     assert L.ls_param_count(bad) == L.LS_ERR_ARG
+
+
+def test_prefix_index_mode_needs_at_most_512_instances(lib):
+    c = _cfg(max_instances=600, prefix_mode="index")
+    rc, h = L.ls_create(c)
+    assert rc == L.LS_ERR_ARG and "512" in L.last_error()

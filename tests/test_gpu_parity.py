@@ -129,11 +129,13 @@ def test_hits_parity(name):
     assert want.max() > 0 and (want == 0).any()
 
 
-@pytest.mark.parametrize("name", ["homogeneous", "heterogeneous"])
-def test_fused_prefix_mode_matches_two_phase(name):
+@pytest.mark.parametrize("name", ["tiny", "homogeneous", "heterogeneous"])
+@pytest.mark.parametrize("mode", ["two_phase", "fused"])
+def test_prefix_modes_agree(name, mode):
+    # the default (prefix index over all instances) against per-instance tables
     wl, dw, r = staged(name)
     out = r.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)
-    r2 = H.Router.for_config(wl.cfg, prefix_mode="fused")
+    r2 = H.Router.for_config(wl.cfg, prefix_mode=mode)
     dw.load(r2)
     out2 = r2.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)
     assert torch.equal(out["hits"], out2["hits"])
@@ -143,7 +145,7 @@ def test_fused_prefix_mode_matches_two_phase(name):
 
 def test_batch_over_token_capacity_is_latched_not_faulted():
     wl, dw, r = staged("tiny")
-    small = H.Router.for_config(wl.cfg, max_batch_tokens=1000)
+    small = H.Router.for_config(wl.cfg, max_batch_tokens=1000, prefix_mode="two_phase")
     dw.load(small)
     small.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)   # ~20k tokens > 1000
     assert small.sync() == L.LS_ERR_ARG
@@ -393,7 +395,8 @@ def test_train_adam_bf16(steps, batch):
         assert np.all(np.abs(dg - do)[clear] <= 0.1 * np.abs(do)[clear] + 0.05 * lr)
         assert np.mean(np.abs(dg - do)[clear] <= 0.02 * np.abs(do)[clear] + 0.01 * lr) > 0.99
         assert np.mean(np.sign(dg) == np.sign(do)) > 0.99
-        np.testing.assert_allclose(m1.cpu().numpy()[clear], tr.m[clear], rtol=5e-2, atol=1e-9)
+        mg, mo = m1.cpu().numpy().astype(np.float64), tr.m
+        assert np.all(np.abs(mg - mo)[clear] <= 5e-2 * np.maximum(np.abs(mo), 0.1 * np.sqrt(np.mean(mo ** 2)))[clear])
         assert np.abs(after - tr.params).max() <= 2.5 * lr
     assert r.sync() == L.LS_OK
     r.close()
