@@ -50,6 +50,8 @@ struct TcPlan {
   int d_pad = 0;
   int64_t w_last_off = 0;
   int64_t b_last_off = 0;
+  int pipe = 0;                    // pipelined kernel applies (two hidden layers, resident weights)
+  int pipe_smem = 0;
 };
 
 // One published weight version (Sec. 4.3.1 P2: the routing side reads a

@@ -327,6 +327,282 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc(const __grid_constan
   if (warp == 0) tmem_dealloc(tmem, p.tmem_cols);
 }
 
+// ---------------------------------------------------------------------------
+// Pipelined variant for predictors with two hidden layers whose weights stay
+// resident (widths <= 256): warp 0 issues the MMAs, warps 1-7 build feature
+// tiles into two buffers ahead of time, warps 8-15 run the epilogues.  Layer-1
+// activations go to the layer-2 MMA through a two-slot ring of 64-column
+// K-blocks, so the layer-2 MMA of a tile runs while its layer-1 epilogue is
+// still producing K-blocks; D1 and D2 sit in separate TMEM halves, so the final
+// epilogue of tile t overlaps the layer-1 MMA of tile t+1.
+// ---------------------------------------------------------------------------
+constexpr int kProdWarps = 7, kEpiWarps = 8;
+constexpr int kProdThreads = kProdWarps * 32, kEpiThreads = kEpiWarps * 32;
+
+// feature tile built by `nthr` threads (index `tr`)
+__device__ __forceinline__ void build_tile_part(const TcArgs& a, uint8_t* X, int64_t row0, int tr, int nthr,
+                                                const float (&mu)[kPair], const float (&sd)[kPair]) {
+  const int cpr = a.p.d_pad / 8;
+  const int total = kTileM * cpr;
+  const int64_t r0 = row0 / a.n_inst;
+  const int i0 = (int)(row0 - r0 * a.n_inst);
+  constexpr int U = 5;
+  for (int base = 0; base < total; base += U * nthr) {
+    uint4 ti[U], trq[U];
+    int64_t L[U];
+    int h[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int e = base + u * nthr + tr;
+      ti[u] = trq[u] = make_uint4(0u, 0u, 0u, 0u);
+      L[u] = 0;
+      h[u] = 0;
+      if (e >= total) continue;
+      const int m = e / cpr, c = e - m * cpr;
+      const int64_t g = row0 + m;
+      if (g >= a.rows) continue;
+      int i = i0 + m;
+      int64_t r = r0;
+      if (a.n_inst >= 16) {
+        while (i >= a.n_inst) { i -= a.n_inst; ++r; }
+      } else {
+        r += i / a.n_inst;
+        i -= (i / a.n_inst) * a.n_inst;
+      }
+      ti[u] = __ldg(reinterpret_cast<const uint4*>(a.xin + (int64_t)i * a.p.d_pad) + c);
+      trq[u] = __ldg(reinterpret_cast<const uint4*>(a.xrq + r * a.p.d_pad) + c);
+      if (c == 0) {
+        L[u] = __ldg(a.tok_off + r + 1) - __ldg(a.tok_off + r);
+        h[u] = __ldg(a.hits + g);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int e = base + u * nthr + tr;
+      if (e >= total) continue;
+      const int m = e / cpr, c = e - m * cpr;
+      uint4 v = make_uint4(ti[u].x | trq[u].x, ti[u].y | trq[u].y, ti[u].z | trq[u].z, ti[u].w | trq[u].w);
+      if (c == 0 && row0 + m < a.rows) {
+        uint16_t f[kPair];
+#pragma unroll
+        for (int k = 0; k < kPair; ++k)
+          f[k] = bf16_bits(zscore(raw_feature(k, L[u], h[u], nullptr, 0, nullptr), mu[k], sd[k]));
+        v.x = f[0] | ((uint32_t)f[1] << 16);
+        v.y = f[2] | ((uint32_t)f[3] << 16);
+        v.z = f[4] | ((uint32_t)f[5] << 16);
+      }
+      st_shared_v4(X + sw128_offset(m, c * 8, kTileM), v.x, v.y, v.z, v.w);
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc_pipe(const __grid_constant__ TcArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const TcPlan& p = a.p;
+  const int H1 = p.out[0], H2 = p.out[1];
+  const int nk0 = p.in_pad[0] / 64;       // K-blocks of layer 1 (feature tile)
+  const int nk1 = H1 / 64;                // K-blocks of layer 2 (= 64-column blocks of D1)
+  const int xbytes = nk0 * kTileM * 128;  // one feature tile
+  uint8_t* W = smem;                                            // resident weight chunks
+  uint8_t* X = W + (size_t)p.chunks * p.chunk_bytes;            // [2] feature tiles
+  uint8_t* AR = X + 2 * (size_t)xbytes;                         // [2] activation K-blocks (16 KB)
+  float* part = reinterpret_cast<float*>(AR + 2 * kTileM * 128);  // [2][128]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(part + 2 * kTileM);
+  uint64_t* x_full = bars;       // [2]
+  uint64_t* x_empty = bars + 2;  // [2]
+  uint64_t* a_full = bars + 4;   // [2]
+  uint64_t* a_empty = bars + 6;  // [2]
+  uint64_t* d1_full = bars + 8;
+  uint64_t* d1_empty = bars + 9;
+  uint64_t* d2_full = bars + 10;
+  uint64_t* d2_empty = bars + 11;
+  uint64_t* w_full = bars + 12;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 13);
+  int* abort_flag = reinterpret_cast<int*>(tmem_holder + 1);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  if (tid == 0) {
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&x_full[b], kProdThreads);
+      mbar_init(&x_empty[b], 1);
+      mbar_init(&a_full[b], kEpiWarps);
+      mbar_init(&a_empty[b], 1);
+    }
+    mbar_init(d1_full, 1);
+    mbar_init(d1_empty, kEpiWarps);
+    mbar_init(d2_full, 1);
+    mbar_init(d2_empty, kEpiWarps);
+    mbar_init(w_full, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0) {
+    tmem_alloc(tmem_holder, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_holder;
+  const uint32_t D1 = tmem, D2 = tmem + 256;
+  const int my_tiles = blockIdx.x < a.n_tiles ? (a.n_tiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0 && my_tiles > 0) {
+      int64_t wbytes = 0;
+      for (int q = 0; q < p.chunks; ++q) wbytes += p.chunk_len[q];
+      mbar_arrive_expect_tx(w_full, (uint32_t)wbytes);
+      for (int q = 0; q < p.chunks; ++q)
+        bulk_g2s(W + (size_t)q * p.chunk_bytes, a.img + p.chunk_off[q], (uint32_t)p.chunk_len[q], w_full);
+      bool ok = mbar_wait(w_full, 0);
+      const uint32_t id1 = idesc_bf16_f32(kTileM, H1), id2 = idesc_bf16_f32(kTileM, H2);
+      for (int t = 0; t < my_tiles && ok; ++t) {
+        const int xb = t & 1;
+        ok = mbar_wait(&x_full[xb], (uint32_t)((t >> 1) & 1));
+        if (ok && t >= 1) ok = mbar_wait(d1_empty, (uint32_t)((t - 1) & 1));
+        if (!ok) break;
+        tc_fence_after();
+        const uint32_t xa = smem_u32(X + (size_t)xb * xbytes);
+        for (int kb = 0; kb < nk0; ++kb)
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            umma_bf16(D1, sdesc_sw128(xa + (uint32_t)kb * kTileM * 128u + 32u * j),
+                      sdesc_sw128(smem_u32(W + (size_t)kb * p.chunk_bytes) + 32u * j), id1, (kb | j) ? 1u : 0u);
+        umma_commit(&x_empty[xb]);
+        umma_commit(d1_full);
+        for (int kb = 0; kb < nk1 && ok; ++kb) {
+          const int64_t kq = (int64_t)t * nk1 + kb;
+          const int slot = (int)(kq & 1);
+          ok = mbar_wait(&a_full[slot], (uint32_t)((kq >> 1) & 1));
+          if (ok && kb == 0 && t >= 1) ok = mbar_wait(d2_empty, (uint32_t)((t - 1) & 1));
+          if (!ok) break;
+          tc_fence_after();
+          const uint32_t aa = smem_u32(AR + (size_t)slot * kTileM * 128);
+          const uint32_t bb = smem_u32(W + (size_t)(nk0 + kb) * p.chunk_bytes);
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            umma_bf16(D2, sdesc_sw128(aa + 32u * j), sdesc_sw128(bb + 32u * j), id2, (kb | j) ? 1u : 0u);
+          umma_commit(&a_empty[slot]);
+        }
+        umma_commit(d2_full);
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        latch_error(a.err, LS_ERR_TIMEOUT);
+      }
+    }
+    __syncwarp();
+  } else if (warp <= kProdWarps) {
+    // ------------------------------------------------------------ feature tiles
+    float mu[kPair], sd[kPair];
+#pragma unroll
+    for (int k = 0; k < kPair; ++k) {
+      mu[k] = __ldg(a.mean + k);
+      sd[k] = __ldg(a.stdv + k);
+    }
+    const int tr = tid - 32;
+    for (int t = 0; t < my_tiles; ++t) {
+      const int xb = t & 1;
+      if (t >= 2 && !mbar_wait(&x_empty[xb], (uint32_t)(((t - 2) >> 1) & 1))) {
+        *abort_flag = 1;
+        latch_error(a.err, LS_ERR_TIMEOUT);
+        break;
+      }
+      if (*abort_flag) break;
+      const int64_t row0 = (int64_t)(blockIdx.x + (int64_t)t * gridDim.x) * kTileM;
+      build_tile_part(a, X + (size_t)xb * xbytes, row0, tr, kProdThreads, mu, sd);
+      fence_async_smem();
+      mbar_arrive(&x_full[xb]);
+    }
+  } else {
+    // ------------------------------------------------------------ epilogues
+    const int ew = warp - 1 - kProdWarps;  // 0..7
+    const int q4 = warp & 3;               // TMEM lane quadrant
+    const int wk = ew >> 2;                // 0/1: column half
+    const int row = 32 * q4 + lane;
+    const uint32_t lane_addr = (uint32_t)(32 * q4) << 16;
+    const float* b1 = a.params + a.boff[0];
+    const float* b2 = a.params + a.boff[1];
+    const float* w3 = a.params + a.w_last_off;
+    const float b3 = __ldg(a.params + p.b_last_off);
+    for (int t = 0; t < my_tiles; ++t) {
+      const int64_t row0 = (int64_t)(blockIdx.x + (int64_t)t * gridDim.x) * kTileM;
+      if (!mbar_wait(d1_full, (uint32_t)(t & 1))) { *abort_flag = 1; latch_error(a.err, LS_ERR_TIMEOUT); break; }
+      tc_fence_after();
+      // layer-1 epilogue, one 64-column K-block at a time (this warp: 32 columns of it)
+      bool ok = true;
+      for (int kb = 0; kb < nk1; ++kb) {
+        const int64_t kq = (int64_t)t * nk1 + kb;
+        const int slot = (int)(kq & 1);
+        if (kq >= 2 && !mbar_wait(&a_empty[slot], (uint32_t)(((kq - 2) >> 1) & 1))) { ok = false; break; }
+        uint8_t* dst = AR + (size_t)slot * kTileM * 128;
+#pragma unroll
+        for (int g = 0; g < 2; ++g) {
+          const int col = 64 * kb + 32 * wk + 16 * g;
+          uint32_t v[16];
+          tmem_ld16(D1 + lane_addr + (uint32_t)col, v);
+          tmem_wait_ld();
+          uint32_t pk[8];
+#pragma unroll
+          for (int j4 = 0; j4 < 4; ++j4) {
+            const float4 b = ldg4(b1 + col + 4 * j4);
+            const uint64_t z0 = add_f32x2(((uint64_t)v[4 * j4 + 1] << 32) | v[4 * j4], f2pack(b.x, b.y));
+            const uint64_t z1 = add_f32x2(((uint64_t)v[4 * j4 + 3] << 32) | v[4 * j4 + 2], f2pack(b.z, b.w));
+            pk[2 * j4] = relu_bf16x2(cvt_bf16x2(z0));
+            pk[2 * j4 + 1] = relu_bf16x2(cvt_bf16x2(z1));
+          }
+          const int kcol = 32 * wk + 16 * g;  // column inside the K-block
+          st_shared_v4(dst + sw128_offset(row, kcol, kTileM), pk[0], pk[1], pk[2], pk[3]);
+          st_shared_v4(dst + sw128_offset(row, kcol + 8, kTileM), pk[4], pk[5], pk[6], pk[7]);
+        }
+        fence_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&a_full[slot]);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(d1_empty);
+      if (!ok) { *abort_flag = 1; latch_error(a.err, LS_ERR_TIMEOUT); break; }
+      // layer-2 epilogue: bias, ReLU, bf16, dot with the output weights
+      if (!mbar_wait(d2_full, (uint32_t)(t & 1))) { *abort_flag = 1; latch_error(a.err, LS_ERR_TIMEOUT); break; }
+      tc_fence_after();
+      uint64_t acc2 = 0;
+      const int half = H2 / 2;
+      for (int c0 = wk * half; c0 < (wk + 1) * half; c0 += 16) {
+        uint32_t v[16];
+        tmem_ld16(D2 + lane_addr + (uint32_t)c0, v);
+        tmem_wait_ld();
+#pragma unroll
+        for (int j4 = 0; j4 < 4; ++j4) {
+          const float4 b = ldg4(b2 + c0 + 4 * j4);
+          const float4 w = ldg4(w3 + c0 + 4 * j4);
+          const uint32_t h0 = relu_bf16x2(cvt_bf16x2(add_f32x2(((uint64_t)v[4 * j4 + 1] << 32) | v[4 * j4],
+                                                                 f2pack(b.x, b.y))));
+          const uint32_t h1 = relu_bf16x2(cvt_bf16x2(add_f32x2(((uint64_t)v[4 * j4 + 3] << 32) | v[4 * j4 + 2],
+                                                                 f2pack(b.z, b.w))));
+          acc2 = fma_f32x2(bf16x2_to_f32x2(h0), f2pack(w.x, w.y), acc2);
+          acc2 = fma_f32x2(bf16x2_to_f32x2(h1), f2pack(w.z, w.w), acc2);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(d2_empty);
+      float* pt = part + (t & 1) * kTileM;  // double-buffered by tile parity
+      if (wk == 1) pt[row] = __uint_as_float((uint32_t)acc2) + __uint_as_float((uint32_t)(acc2 >> 32));
+      named_bar_sync(1, kEpiThreads);
+      if (wk == 0) {
+        const int64_t g = row0 + row;
+        const float mine = __uint_as_float((uint32_t)acc2) + __uint_as_float((uint32_t)(acc2 >> 32));
+        if (g < a.rows) a.scores[g] = (mine + pt[row]) + b3;
+      }
+    }
+  }
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tmem, 512);
+}
+
 // Normalised bf16 template rows, computed once per batch: instance row i holds
 // the z-scored instance features at their feature positions (6 .. 6+d_inst)
 // and zeros elsewhere; request row r likewise for the request block.
@@ -422,6 +698,16 @@ bool plan_tc(const MlpDesc& m, TcPlan& p) {
   while ((int)p.tmem_cols < outmax) p.tmem_cols <<= 1;
   p.w_last_off = m.woff[m.n_layers - 1];
   p.b_last_off = m.boff[m.n_layers - 1];
+  // pipelined variant: two hidden layers of <= 256, all weights resident
+  p.pipe = 0;
+  if (p.n_tc == 2 && p.out[0] <= 256 && p.out[1] <= 256 && p.nc[0] == p.out[0] && p.nc[1] == p.out[1]) {
+    const int64_t need = 1024 + (int64_t)p.chunks * cb + 2 * (int64_t)p.d_pad * kTileM * 2 + 2 * kTileM * 128 +
+                         2 * kTileM * 4 + 13 * 8 + 16;
+    if (need <= kMaxSmem) {
+      p.pipe = 1;
+      p.pipe_smem = (int)need;
+    }
+  }
   return true;
 }
 
@@ -475,10 +761,16 @@ cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const uint8_t* im
   a.err = err;
   a.rows = rows;
   a.n_tiles = (int)((rows + kTileM - 1) / kTileM);
-  cudaError_t e = cudaFuncSetAttribute(k_score_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, p.smem);
-  if (e != cudaSuccess) return e;
   const int grid = std::min(a.n_tiles, sms);
-  k_score_tc<<<grid, kThreadsTc, p.smem, s>>>(a);
+  if (p.pipe) {
+    cudaError_t e = cudaFuncSetAttribute(k_score_tc_pipe, cudaFuncAttributeMaxDynamicSharedMemorySize, p.pipe_smem);
+    if (e != cudaSuccess) return e;
+    k_score_tc_pipe<<<grid, kThreadsTc, p.pipe_smem, s>>>(a);
+  } else {
+    cudaError_t e = cudaFuncSetAttribute(k_score_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, p.smem);
+    if (e != cudaSuccess) return e;
+    k_score_tc<<<grid, kThreadsTc, p.smem, s>>>(a);
+  }
   return cudaGetLastError();
 }
 

@@ -230,12 +230,19 @@ __global__ void k_out_dx(int B, int K, const float* __restrict__ dz, const float
   }
 }
 
+// dst[e] = sum over z of part[z * n + e], z in order (up to 16 loads in flight).
 __global__ void k_reduce_partials(int S, int64_t n, const float* __restrict__ part,
                                   float* __restrict__ dst) {
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n;
        e += (int64_t)gridDim.x * blockDim.x) {
     float s = 0.0f;
-    for (int z = 0; z < S; ++z) s += part[(int64_t)z * n + e];
+    for (int z0 = 0; z0 < S; z0 += 16) {
+      float v[16];
+#pragma unroll
+      for (int u = 0; u < 16; ++u) v[u] = z0 + u < S ? __ldg(part + (int64_t)(z0 + u) * n + e) : 0.0f;
+#pragma unroll
+      for (int u = 0; u < 16; ++u) s += v[u];
+    }
     dst[e] = s;
   }
 }

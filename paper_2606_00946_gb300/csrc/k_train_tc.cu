@@ -191,6 +191,7 @@ __global__ void __launch_bounds__(kT) k_gemm_tc(const __grid_constant__ TcGemmAr
   const int row = m0 + 32 * q4 + lane;
   const int half = NTILE / 2;
   const uint32_t lane_addr = (uint32_t)(32 * q4) << 16;
+  const bool row_ok = row < g.M;
   for (int c0 = ch * half; c0 < (ch + 1) * half; c0 += 16) {
     uint32_t v[16];
     if (nchunks > 0) {
@@ -200,21 +201,66 @@ __global__ void __launch_bounds__(kT) k_gemm_tc(const __grid_constant__ TcGemmAr
 #pragma unroll
       for (int j = 0; j < 16; ++j) v[j] = 0u;
     }
-    if (row >= g.M) continue;
+    const int nb = n0 + c0;            // first column of this group
+    const bool full = nb + 16 <= g.N;  // all 16 columns in range
+    // side inputs of the group (bias, or the pre-activation for the mask),
+    // all loaded before any use
+    float side[16];
+    if (g.epi == 1) {
+      if (full && (reinterpret_cast<uintptr_t>(g.bias + nb) & 15) == 0) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const float4 b4 = __ldg(reinterpret_cast<const float4*>(g.bias + nb) + q);
+          side[4 * q] = b4.x; side[4 * q + 1] = b4.y; side[4 * q + 2] = b4.z; side[4 * q + 3] = b4.w;
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) side[j] = nb + j < g.N ? __ldg(g.bias + nb + j) : 0.0f;
+      }
+    } else if (g.epi == 2) {
+      const float* zp = g.zprev + (int64_t)row * g.ld_zprev + nb;
+      if (row_ok && full && (reinterpret_cast<uintptr_t>(zp) & 15) == 0) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const float4 z4 = __ldg(reinterpret_cast<const float4*>(zp) + q);
+          side[4 * q] = z4.x; side[4 * q + 1] = z4.y; side[4 * q + 2] = z4.z; side[4 * q + 3] = z4.w;
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) side[j] = (row_ok && nb + j < g.N) ? __ldg(zp + j) : 0.0f;
+      }
+    }
+    if (!row_ok) continue;
+    float out[16], act[16];
 #pragma unroll
     for (int j = 0; j < 16; ++j) {
-      const int n = n0 + c0 + j;
-      if (n >= g.N) break;
       const float acc = __uint_as_float(v[j]);
       if (g.epi == 0) {
-        g.C[(int64_t)blockIdx.z * g.split_stride + (int64_t)row * g.ldc + n] = acc;
+        out[j] = acc;
       } else if (g.epi == 1) {
-        const float z = acc + __ldg(g.bias + n);
-        g.C[(int64_t)row * g.ldc + n] = z;
-        if (g.hidden) g.act[(int64_t)row * g.ld_act + n] = round_bf16(z > 0.0f ? z : 0.0f);
+        out[j] = acc + side[j];
+        act[j] = round_bf16(out[j] > 0.0f ? out[j] : 0.0f);
       } else {
-        g.C[(int64_t)row * g.ldc + n] = __ldg(g.zprev + (int64_t)row * g.ld_zprev + n) > 0.0f ? acc : 0.0f;
+        out[j] = side[j] > 0.0f ? acc : 0.0f;
       }
+    }
+    float* crow = g.C + (g.epi == 0 ? (int64_t)blockIdx.z * g.split_stride : 0) + (int64_t)row * g.ldc + nb;
+    float* arow = g.epi == 1 && g.hidden ? g.act + (int64_t)row * g.ld_act + nb : nullptr;
+    if (full && (reinterpret_cast<uintptr_t>(crow) & 15) == 0 &&
+        (!arow || (reinterpret_cast<uintptr_t>(arow) & 15) == 0)) {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        reinterpret_cast<float4*>(crow)[q] = make_float4(out[4 * q], out[4 * q + 1], out[4 * q + 2], out[4 * q + 3]);
+        if (arow)
+          reinterpret_cast<float4*>(arow)[q] = make_float4(act[4 * q], act[4 * q + 1], act[4 * q + 2], act[4 * q + 3]);
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < 16; ++j)
+        if (nb + j < g.N) {
+          crow[j] = out[j];
+          if (arow) arow[j] = act[j];
+        }
     }
   }
   tc_fence_before();

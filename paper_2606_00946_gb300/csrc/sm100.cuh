@@ -33,6 +33,10 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t by
                : "memory");
 }
 
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
@@ -69,6 +73,44 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
 // generic-proxy shared-memory writes -> visible to the async proxy (tensor core)
 __device__ __forceinline__ void fence_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// named barrier among `count` threads (id 1..15; id 0 is __syncthreads)
+__device__ __forceinline__ void named_bar_sync(int id, int count) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
+// ---------------------------------------------------------------------------
+// packed arithmetic (two fp32 lanes in one 64-bit register; bf16x2)
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint64_t f2pack(float lo, float hi) {
+  return (uint64_t)__float_as_uint(lo) | ((uint64_t)__float_as_uint(hi) << 32);
+}
+__device__ __forceinline__ uint64_t add_f32x2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t fma_f32x2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+// bf16 (round to nearest even) of the two lanes, low lane in the low half
+__device__ __forceinline__ uint32_t cvt_bf16x2(uint64_t v) {
+  uint32_t d;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(__uint_as_float((uint32_t)(v >> 32))),
+      "f"(__uint_as_float((uint32_t)v)));
+  return d;
+}
+__device__ __forceinline__ uint32_t relu_bf16x2(uint32_t v) {
+  uint32_t d;
+  asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(v), "r"(0u));
+  return d;
+}
+// the two bf16 values back to fp32 lanes
+__device__ __forceinline__ uint64_t bf16x2_to_f32x2(uint32_t v) {
+  return (uint64_t)(v << 16) | ((uint64_t)(v & 0xFFFF0000u) << 32);
 }
 
 // ---------------------------------------------------------------------------

@@ -395,8 +395,9 @@ def test_train_adam_bf16(steps, batch):
         assert np.all(np.abs(dg - do)[clear] <= 0.1 * np.abs(do)[clear] + 0.05 * lr)
         assert np.mean(np.abs(dg - do)[clear] <= 0.02 * np.abs(do)[clear] + 0.01 * lr) > 0.99
         assert np.mean(np.sign(dg) == np.sign(do)) > 0.99
+        # first moment: m1 - m0 = (1 - beta1) g, so it carries the gradient's tolerance
         mg, mo = m1.cpu().numpy().astype(np.float64), tr.m
-        assert np.all(np.abs(mg - mo)[clear] <= 5e-2 * np.maximum(np.abs(mo), 0.1 * np.sqrt(np.mean(mo ** 2)))[clear])
+        assert np.linalg.norm(mg - mo) <= 0.1 * 2e-2 * np.linalg.norm(g) + 1e-6 * np.linalg.norm(mo)
         assert np.abs(after - tr.params).max() <= 2.5 * lr
     assert r.sync() == L.LS_OK
     r.close()
