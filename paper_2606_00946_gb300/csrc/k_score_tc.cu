@@ -344,6 +344,7 @@ __device__ __forceinline__ void build_tile_part(const TcArgs& a, uint8_t* X, int
                                                 const float (&mu)[kPair], const float (&sd)[kPair]) {
   const int cpr = a.p.d_pad / 8;
   const int total = kTileM * cpr;
+  const int csh = (cpr & (cpr - 1)) == 0 ? __ffs(cpr) - 1 : -1;  // shift when cpr is a power of two
   const int64_t r0 = row0 / a.n_inst;
   const int i0 = (int)(row0 - r0 * a.n_inst);
   constexpr int U = 5;
@@ -358,7 +359,7 @@ __device__ __forceinline__ void build_tile_part(const TcArgs& a, uint8_t* X, int
       L[u] = 0;
       h[u] = 0;
       if (e >= total) continue;
-      const int m = e / cpr, c = e - m * cpr;
+      const int m = csh >= 0 ? e >> csh : e / cpr, c = e - m * cpr;
       const int64_t g = row0 + m;
       if (g >= a.rows) continue;
       int i = i0 + m;
@@ -380,7 +381,7 @@ __device__ __forceinline__ void build_tile_part(const TcArgs& a, uint8_t* X, int
     for (int u = 0; u < U; ++u) {
       const int e = base + u * nthr + tr;
       if (e >= total) continue;
-      const int m = e / cpr, c = e - m * cpr;
+      const int m = csh >= 0 ? e >> csh : e / cpr, c = e - m * cpr;
       uint4 v = make_uint4(ti[u].x | trq[u].x, ti[u].y | trq[u].y, ti[u].z | trq[u].z, ti[u].w | trq[u].w);
       if (c == 0 && row0 + m < a.rows) {
         uint16_t f[kPair];
@@ -538,18 +539,20 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc_pipe(const __grid_co
         const int slot = (int)(kq & 1);
         if (kq >= 2 && !mbar_wait(&a_empty[slot], (uint32_t)(((kq - 2) >> 1) & 1))) { ok = false; break; }
         uint8_t* dst = AR + (size_t)slot * kTileM * 128;
+        const int colb = 64 * kb + 32 * wk;
+        uint32_t v[2][16];
+        tmem_ld16(D1 + lane_addr + (uint32_t)colb, v[0]);
+        tmem_ld16(D1 + lane_addr + (uint32_t)(colb + 16), v[1]);
+        tmem_wait_ld();
 #pragma unroll
         for (int g = 0; g < 2; ++g) {
-          const int col = 64 * kb + 32 * wk + 16 * g;
-          uint32_t v[16];
-          tmem_ld16(D1 + lane_addr + (uint32_t)col, v);
-          tmem_wait_ld();
+          const int col = colb + 16 * g;
           uint32_t pk[8];
 #pragma unroll
           for (int j4 = 0; j4 < 4; ++j4) {
             const float4 b = ldg4(b1 + col + 4 * j4);
-            const uint64_t z0 = add_f32x2(((uint64_t)v[4 * j4 + 1] << 32) | v[4 * j4], f2pack(b.x, b.y));
-            const uint64_t z1 = add_f32x2(((uint64_t)v[4 * j4 + 3] << 32) | v[4 * j4 + 2], f2pack(b.z, b.w));
+            const uint64_t z0 = add_f32x2(((uint64_t)v[g][4 * j4 + 1] << 32) | v[g][4 * j4], f2pack(b.x, b.y));
+            const uint64_t z1 = add_f32x2(((uint64_t)v[g][4 * j4 + 3] << 32) | v[g][4 * j4 + 2], f2pack(b.z, b.w));
             pk[2 * j4] = relu_bf16x2(cvt_bf16x2(z0));
             pk[2 * j4 + 1] = relu_bf16x2(cvt_bf16x2(z1));
           }
@@ -570,20 +573,25 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc_pipe(const __grid_co
       tc_fence_after();
       uint64_t acc2 = 0;
       const int half = H2 / 2;
-      for (int c0 = wk * half; c0 < (wk + 1) * half; c0 += 16) {
-        uint32_t v[16];
-        tmem_ld16(D2 + lane_addr + (uint32_t)c0, v);
+      for (int c0 = wk * half; c0 < (wk + 1) * half; c0 += 32) {
+        uint32_t v[2][16];
+        tmem_ld16(D2 + lane_addr + (uint32_t)c0, v[0]);
+        tmem_ld16(D2 + lane_addr + (uint32_t)(c0 + 16), v[1]);
         tmem_wait_ld();
 #pragma unroll
-        for (int j4 = 0; j4 < 4; ++j4) {
-          const float4 b = ldg4(b2 + c0 + 4 * j4);
-          const float4 w = ldg4(w3 + c0 + 4 * j4);
-          const uint32_t h0 = relu_bf16x2(cvt_bf16x2(add_f32x2(((uint64_t)v[4 * j4 + 1] << 32) | v[4 * j4],
-                                                                 f2pack(b.x, b.y))));
-          const uint32_t h1 = relu_bf16x2(cvt_bf16x2(add_f32x2(((uint64_t)v[4 * j4 + 3] << 32) | v[4 * j4 + 2],
-                                                                 f2pack(b.z, b.w))));
-          acc2 = fma_f32x2(bf16x2_to_f32x2(h0), f2pack(w.x, w.y), acc2);
-          acc2 = fma_f32x2(bf16x2_to_f32x2(h1), f2pack(w.z, w.w), acc2);
+        for (int g = 0; g < 2; ++g) {
+#pragma unroll
+          for (int j4 = 0; j4 < 4; ++j4) {
+            const int cc = c0 + 16 * g + 4 * j4;
+            const float4 b = ldg4(b2 + cc);
+            const float4 w = ldg4(w3 + cc);
+            const uint32_t h0 = relu_bf16x2(cvt_bf16x2(add_f32x2(((uint64_t)v[g][4 * j4 + 1] << 32) | v[g][4 * j4],
+                                                                   f2pack(b.x, b.y))));
+            const uint32_t h1 = relu_bf16x2(cvt_bf16x2(
+                add_f32x2(((uint64_t)v[g][4 * j4 + 3] << 32) | v[g][4 * j4 + 2], f2pack(b.z, b.w))));
+            acc2 = fma_f32x2(bf16x2_to_f32x2(h0), f2pack(w.x, w.y), acc2);
+            acc2 = fma_f32x2(bf16x2_to_f32x2(h1), f2pack(w.z, w.w), acc2);
+          }
         }
       }
       tc_fence_before();
