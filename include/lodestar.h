@@ -224,6 +224,56 @@ typedef struct {
 int ls_trace_enable(ls_ctx *ctx, int32_t on);
 int ls_trace_read(ls_ctx *ctx, ls_trace_entry *out, int32_t max_entries, int32_t *n_out);
 
+/* Prefix hit lengths without any device allocation (no counterpart in the
+ * paper: the paper's router calls into a Python service and never states how
+ * scratch memory is obtained).  Computes the same h[r, i] as the prefix
+ * stage of ls_route_batch (Sec. 2: the first miss ends reuse; Sec. 4.1
+ * Features (2)), using the two-phase kernels (hash + block-0 screen, then a
+ * walk of the pairs that hit block 0), but needs no context and takes its
+ * scratch from one statically sized device array compiled into the library.
+ *
+ * Who needs it: callers that must not allocate device memory while routing --
+ * a routing thread that is latency-critical (cudaMalloc/cudaFree can
+ * synchronise the device), code inside stream capture (allocation calls are
+ * not capturable), and plugins inside a host process whose memory pool owns
+ * all device memory.  The cost: LS_STATIC_SCRATCH_BYTES of device memory is
+ * reserved on every GPU the library is loaded on, for the life of the process.
+ *
+ *   n_req       requests (>= 0; 0 returns LS_OK with nothing enqueued)
+ *   tok         DEVICE int32 tokens of the batch (CSR values)
+ *   tok_off     DEVICE int64 [n_req + 1] CSR offsets (non-decreasing)
+ *   n_tokens    HOST copy of tok_off[n_req] - tok_off[0]; the call checks the
+ *               batch's block count against LS_STATIC_MAX_BLOCKS with it.  If
+ *               it understates the span, blocks past the static capacity
+ *               count as misses (hits come out short, nothing is written out
+ *               of bounds).
+ *   tables      DEVICE uint64 [n_inst * slots_per_instance]: per-instance
+ *               open-addressing tables of block keys (key 0 = empty slot,
+ *               linear probing from key & (slots - 1)), 16-byte aligned
+ *   slots_per_instance  power of two in [16, 2^31]
+ *   n_inst      instances (>= 1)
+ *   hits_out    DEVICE int32 [n_req, n_inst] row-major, fully overwritten
+ *   stream      cudaStream_t (NULL = legacy default stream)
+ *
+ * Scratch: keys [LS_STATIC_MAX_BLOCKS] uint64, a work list of
+ * [LS_STATIC_MAX_PAIRS] uint32, and two int32 counters that must start at
+ * zero for every call; the call zeroes them itself with cudaMemsetAsync on
+ * `stream`, before its kernels.  The scratch is shared by every caller on a
+ * device, so two calls whose kernels overlap in time (different streams,
+ * different host threads) race and may return wrong hit lengths: serialise
+ * them on one stream or with events.
+ * The first call on a device (with that device current) looks up the
+ * scratch address with cudaGetSymbolAddress; make that first call outside
+ * any stream capture.  Returns LS_ERR_ARG for bad arguments or a batch
+ * beyond the static limits (with a message in ls_last_error), LS_ERR_CUDA if
+ * the lookup or a launch fails, else LS_OK once the work is enqueued. */
+#define LS_STATIC_MAX_BLOCKS 262144 /* full 16-token blocks per batch */
+#define LS_STATIC_MAX_PAIRS 262144  /* n_req * n_inst per batch */
+#define LS_STATIC_SCRATCH_BYTES (LS_STATIC_MAX_BLOCKS * 8 + LS_STATIC_MAX_PAIRS * 4 + 256)
+int ls_prefix_hits_static(int32_t n_req, const int32_t *tok, const int64_t *tok_off, int64_t n_tokens,
+                          const uint64_t *tables, int64_t slots_per_instance, int32_t n_inst,
+                          int32_t *hits_out, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -36,6 +36,15 @@ int cuda_fail(cudaError_t e, const char* where) {
   return e == cudaErrorMemoryAllocation ? LS_ERR_OOM : LS_ERR_CUDA;
 }
 
+}  // namespace
+
+namespace ls {
+// Message for ls_last_error() from entry points defined in other files.
+void set_last_error(const char* msg) { g_err = msg; }
+}  // namespace ls
+
+namespace {
+
 #define LS_CK(call)                                   \
   do {                                                \
     cudaError_t e_ = (call);                          \

@@ -274,6 +274,7 @@ cudaError_t launch_gemm_tc(int M, int N, int K, const float* A, int64_t sam, int
                            const float* zprev, int64_t ld_zprev, int* err, int sms, cudaStream_t s);
 int gemm_tc_splits_used(int K, int splits);
 int index_words(int max_instances);
+void set_last_error(const char* msg);  // sets the text ls_last_error() returns
 cudaError_t launch_prefix_index(int n_req, const int32_t* tok, const int64_t* tok_off, const uint64_t* gkeys,
                                 const uint64_t* gmask, int W, uint64_t gmask_slots, int n_inst, int32_t* hits,
                                 int sms, cudaStream_t s);

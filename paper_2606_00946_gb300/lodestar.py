@@ -21,6 +21,7 @@ LS_REPLACE, LS_INSERT = 0, 1
 LS_SGD, LS_ADAM = 0, 1
 LS_SCORER_AUTO, LS_SCORER_CUDA_CORES, LS_SCORER_TENSOR_CORES = 0, 1, 2
 SCORERS = {"auto": 0, "cuda_cores": 1, "tensor_cores": 2}
+LS_STATIC_MAX_BLOCKS, LS_STATIC_MAX_PAIRS = 262144, 262144
 LS_PREFIX_AUTO, LS_PREFIX_TWO_PHASE, LS_PREFIX_FUSED, LS_PREFIX_INDEX = 0, 1, 2, 3
 PREFIX_MODES = {"auto": 0, "two_phase": 1, "fused": 2, "index": 3}
 
@@ -66,6 +67,7 @@ _SIGS = {
     "ls_publish": (C.c_int, [_P, _P]),
     "ls_trace_enable": (C.c_int, [_P, _i32]),
     "ls_trace_read": (C.c_int, [_P, C.POINTER(ls_trace_entry), _i32, C.POINTER(_i32)]),
+    "ls_prefix_hits_static": (C.c_int, [_i32, _P, _P, _i64, _P, _i64, _i32, _P, _P]),
 }
 
 _lib = None
@@ -250,3 +252,10 @@ def ls_trace_read(ctx, max_entries=64):
     n = _i32(0)
     rc = lib().ls_trace_read(ctx, arr, max_entries, C.byref(n))
     return rc, {arr[i].name.decode(): (arr[i].launches, arr[i].total_ms) for i in range(n.value)}
+
+
+def ls_prefix_hits_static(n_req, tok, tok_off, n_tokens, tables, slots_per_instance, n_inst, hits_out,
+                          stream=None) -> int:
+    return lib().ls_prefix_hits_static(int(n_req), ptr(tok), ptr(tok_off), int(n_tokens), ptr(tables),
+                                       int(slots_per_instance), int(n_inst), ptr(hits_out),
+                                       stream_handle(stream))
