@@ -25,6 +25,18 @@
  *    ls_route_batch (on one stream) may run concurrently with
  *    ls_log_samples / ls_train_step / ls_publish (on another stream).
  *  - Block size is 16 tokens; prompts are int32 token ids.
+ *  - The counters that advance every step (records in the sample ring,
+ *    optimiser steps, which published buffer routing reads, the weight
+ *    version) live in device memory and are read and advanced by the kernels
+ *    when they run.  So the calls of one step -- ls_snapshot_update,
+ *    ls_route_batch, ls_log_samples, ls_train_step, ls_publish -- can be
+ *    recorded once into a CUDA graph by stream capture and replayed; each
+ *    replay behaves like issuing the calls again.  While a stream is being
+ *    captured these calls skip their cross-stream ordering (the events that
+ *    make a publish wait for earlier routes and a route wait for the last
+ *    publish), so a replayed graph must be the context's only user while it
+ *    runs, on one stream.  Host-side argument checks and the version written
+ *    to *weight_version_out happen at capture time.
  */
 #ifndef LODESTAR_H
 #define LODESTAR_H
@@ -119,6 +131,8 @@ const char *ls_last_error(void);
  * the first error latched by device code (LS_OK if none). */
 int ls_sync_status(ls_ctx *ctx);
 
+/* Context facts; ring_count, train_steps and weight_version are read from the
+ * device after synchronising it. */
 int ls_get_info(ls_ctx *ctx, ls_info *out /* host */);
 
 /* Set the fp32 master parameters (device, ls_param_count floats: W1 [w1,w0]
@@ -128,7 +142,8 @@ int ls_set_params(ls_ctx *ctx, const float *params, void *stream);
 int ls_get_params(ls_ctx *ctx, float *params_out, void *stream);
 
 /* Optimiser state for checkpointing: Adam first and second moments (device,
- * n_params floats each) and the step count (host). */
+ * n_params floats each) and the step count (host value; both calls
+ * synchronise `stream` to move it). */
 int ls_get_opt_state(ls_ctx *ctx, float *m_out, float *v_out, int64_t *step_out, void *stream);
 int ls_set_opt_state(ls_ctx *ctx, const float *m, const float *v, int64_t step, void *stream);
 
@@ -190,11 +205,14 @@ int ls_route_batch(ls_ctx *ctx, int32_t n_req, const int32_t *tok, const int64_t
 
 /* Append n logged records (raw feature rows feats [n, d], observed TTFT in
  * seconds ttft [n]) to the sample ring: record j goes to slot
- * (count + j) mod ring_capacity, evicting the oldest (Sec. 4.3.2). */
+ * (count + j) mod ring_capacity, evicting the oldest (Sec. 4.3.2); count is
+ * the number of records appended before, kept on the device. */
 int ls_log_samples(ls_ctx *ctx, int32_t n, const float *feats, const float *ttft, void *stream);
 
 /* One minibatch step of the predictor on ring slots idx [batch] (int32 on the
- * device; NULL = slots (k*batch + j) mod min(count, capacity) at step k).
+ * device; NULL = slots (k*batch + j) mod min(count, capacity) at step k; k and
+ * count are the device counters when the step runs; an empty ring at that
+ * point latches LS_ERR_STATE).
  * Loss = mean squared error of the predicted TTFT (seconds).  opt LS_SGD:
  * theta -= lr g; LS_ADAM: beta1 0.9, beta2 0.999, eps 1e-8, bias-corrected.
  * Updates the master weights only; routing sees them after ls_publish.
@@ -205,20 +223,25 @@ int ls_train_step(ls_ctx *ctx, int32_t batch, const int32_t *idx, int32_t opt, f
                   float *loss_out, void *stream);
 
 /* Atomically publish the master weights to routing (Sec. 4.3.1 P2: swap of the
- * model pointer).  Route calls enqueued after this call (in host order) use
- * the new version once this stream reaches the publish point; earlier routes
- * keep the version they started with. */
+ * model pointer).  One kernel writes the buffer routing is not reading and,
+ * when all of it is written, switches the device-side buffer index.  Route
+ * calls enqueued after this call (in host order) use the new version once
+ * this stream reaches the publish point; earlier routes keep the version they
+ * started with (each route takes the index once, before it scores). */
 int ls_publish(ls_ctx *ctx, void *stream);
 
 /* Kernel tracing.  While enabled, each kernel launch of this context is
  * bracketed by CUDA events on its launching stream (a few microseconds of host
- * time per launch).  ls_trace_read synchronises the device, writes up to
- * max_entries per-kernel totals (name, launches, summed device time in ms)
- * to the HOST array out, sets *n_out, and resets the totals. */
+ * time per launch; launches recorded into a CUDA graph are not traced).
+ * ls_trace_read synchronises the device, writes up to max_entries per-kernel
+ * totals to the HOST array out, sets *n_out, and resets the totals: launches
+ * counted, total_ms summed over the timed_launches of them that got events
+ * (8192 events are pooled between reads; later launches are counted only). */
 typedef struct {
     char name[32];
     int64_t launches;
     double total_ms;
+    int64_t timed_launches;
 } ls_trace_entry;
 
 int ls_trace_enable(ls_ctx *ctx, int32_t on);

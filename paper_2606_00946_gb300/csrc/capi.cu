@@ -108,13 +108,11 @@ void free_all(Ctx& c) {
                   c.adam_v, c.pub[0].params, c.pub[0].wt, c.pub[1].params, c.pub[1].wt,
                   c.ring_x, c.ring_y, c.hits, c.scores, c.tx, c.tz, c.ty, c.dz0, c.dz1, c.grad,
                   c.gpart, c.loss_tmp, c.d_err, c.pub[0].img, c.pub[1].img, c.xin, c.xrq,
-                  c.bkeys, c.work, c.work_n, c.gkeys, c.gmask};
+                  c.bkeys, c.work, c.work_n, c.gkeys, c.gmask, c.st};
   for (void* p : ptrs)
     if (p) cudaFree(p);
-  for (int b = 0; b < 2; ++b) {
-    if (c.pub_ready[b]) cudaEventDestroy(c.pub_ready[b]);
-    if (c.route_done[b]) cudaEventDestroy(c.route_done[b]);
-  }
+  if (c.ev_pub) cudaEventDestroy(c.ev_pub);
+  if (c.ev_route) cudaEventDestroy(c.ev_route);
   if (c.tracer.ready)
     for (int i = 0; i < Tracer::kPool; ++i) cudaEventDestroy(c.tracer.ev[i]);
 }
@@ -232,9 +230,10 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
   A(dalloc(&c.gpart, c.gpart_floats));
   A(dalloc(&c.loss_tmp, 1));
   A(dalloc(&c.d_err, 1));
-  for (int b = 0; b < 2 && e == cudaSuccess; ++b) {
-    A(cudaEventCreateWithFlags(&c.pub_ready[b], cudaEventDisableTiming));
-    A(cudaEventCreateWithFlags(&c.route_done[b], cudaEventDisableTiming));
+  A(dalloc(&c.st, 1));
+  if (e == cudaSuccess) {
+    A(cudaEventCreateWithFlags(&c.ev_pub, cudaEventDisableTiming));
+    A(cudaEventCreateWithFlags(&c.ev_route, cudaEventDisableTiming));
   }
   if (e == cudaSuccess) {
     if (c.tables) A(cudaMemset(c.tables, 0, (size_t)NI * c.slots * sizeof(uint64_t)));
@@ -244,6 +243,10 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
     A(cudaMemset(c.adam_m, 0, (size_t)c.n_params * sizeof(float)));
     A(cudaMemset(c.adam_v, 0, (size_t)c.n_params * sizeof(float)));
     A(cudaMemset(c.d_err, 0, sizeof(int)));
+    DevState init{};
+    init.cur = -1;
+    init.route_b = 0;
+    A(cudaMemcpy(c.st, &init, sizeof(DevState), cudaMemcpyHostToDevice));
     A(cudaDeviceSynchronize());
   }
   if (e != cudaSuccess) {
@@ -277,14 +280,17 @@ int ls_sync_status(ls_ctx* h) {
 int ls_get_info(ls_ctx* h, ls_info* out) {
   if (!h || !out) return fail(LS_ERR_ARG, "NULL argument");
   Ctx& c = h->c;
+  DevState ds{};
+  LS_CK(cudaDeviceSynchronize());
+  LS_CK(cudaMemcpy(&ds, c.st, sizeof(DevState), cudaMemcpyDeviceToHost));
   std::lock_guard<std::mutex> g(c.mu);
   out->n_inst = c.n_inst;
   out->d = c.d;
   out->n_params = c.n_params;
   out->table_slots = c.use_index ? c.gslots : c.slots;
-  out->ring_count = c.ring_count;
-  out->train_steps = c.step;
-  out->weight_version = c.version;
+  out->ring_count = ds.ring_count;
+  out->train_steps = ds.step;
+  out->weight_version = ds.version;
   out->scorer = c.use_tc ? LS_SCORER_TENSOR_CORES : LS_SCORER_CUDA_CORES;
   return LS_OK;
 }
@@ -296,7 +302,7 @@ int ls_set_params(ls_ctx* h, const float* params, void* stream) {
   LS_CK(cudaMemcpyAsync(c.master, params, n, cudaMemcpyDeviceToDevice, S(stream)));
   LS_CK(cudaMemsetAsync(c.adam_m, 0, n, S(stream)));
   LS_CK(cudaMemsetAsync(c.adam_v, 0, n, S(stream)));
-  c.step = 0;
+  LS_CK(cudaMemsetAsync(&c.st->step, 0, sizeof(int64_t), S(stream)));
   c.have_params = true;
   return LS_OK;
 }
@@ -315,7 +321,10 @@ int ls_get_opt_state(ls_ctx* h, float* m_out, float* v_out, int64_t* step_out, v
   const size_t n = (size_t)c.n_params * sizeof(float);
   LS_CK(cudaMemcpyAsync(m_out, c.adam_m, n, cudaMemcpyDeviceToDevice, S(stream)));
   LS_CK(cudaMemcpyAsync(v_out, c.adam_v, n, cudaMemcpyDeviceToDevice, S(stream)));
-  *step_out = c.step;
+  int64_t step = 0;
+  LS_CK(cudaMemcpyAsync(&step, &c.st->step, sizeof(int64_t), cudaMemcpyDeviceToHost, S(stream)));
+  LS_CK(cudaStreamSynchronize(S(stream)));
+  *step_out = step;
   return LS_OK;
 }
 
@@ -325,7 +334,9 @@ int ls_set_opt_state(ls_ctx* h, const float* m, const float* v, int64_t step, vo
   const size_t n = (size_t)c.n_params * sizeof(float);
   LS_CK(cudaMemcpyAsync(c.adam_m, m, n, cudaMemcpyDeviceToDevice, S(stream)));
   LS_CK(cudaMemcpyAsync(c.adam_v, v, n, cudaMemcpyDeviceToDevice, S(stream)));
-  c.step = step;
+  const int64_t st_step = step;
+  LS_CK(cudaMemcpyAsync(&c.st->step, &st_step, sizeof(int64_t), cudaMemcpyHostToDevice, S(stream)));
+  LS_CK(cudaStreamSynchronize(S(stream)));
   return LS_OK;
 }
 
@@ -416,14 +427,14 @@ int ls_route_batch(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* 
   if (c.n_inst < 1) return fail(LS_ERR_STATE, "no snapshot");
   if (!c.have_norm) return fail(LS_ERR_STATE, "normaliser not set");
   cudaStream_t s = S(stream);
-  int b;
+  const bool cap = capturing(s);
   uint64_t v;
   {
     std::lock_guard<std::mutex> g(c.mu);
-    if (c.cur < 0) return fail(LS_ERR_STATE, "no weights published");
-    b = c.cur;
-    v = c.pub[b].version;
-    LS_CK(cudaStreamWaitEvent(s, c.pub_ready[b], 0));
+    if (!c.have_published) return fail(LS_ERR_STATE, "no weights published");
+    v = c.version;
+    // the route reads the latest publish enqueued before it (host order)
+    if (!cap && c.pub_recorded) LS_CK(cudaStreamWaitEvent(s, c.ev_pub, 0));
   }
   if (weight_version_out) *weight_version_out = v;
   if (n_req == 0) return LS_OK;
@@ -432,17 +443,17 @@ int ls_route_batch(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* 
   if (c.use_index) {
     LS_CK(traced(c, TR_PREFIX_INDEX, 1, s, [&] {
       return launch_prefix_index(n_req, tok, tok_off, c.gkeys, c.gmask, c.gW, (uint64_t)(c.gslots - 1), c.n_inst,
-                                 hits, c.sms, s);
+                                 hits, c.sms, c.st, s);
     }));
   } else if (c.cfg.prefix_mode == LS_PREFIX_FUSED) {
     LS_CK(traced(c, TR_PREFIX, 1, s, [&] {
-      return launch_prefix_match(n_req, tok, tok_off, c.tables, c.mask, c.slots, c.n_inst, hits, s);
+      return launch_prefix_match(n_req, tok, tok_off, c.tables, c.mask, c.slots, c.n_inst, hits, c.st, s);
     }));
   } else {
     LS_CK(traced(c, TR_MEMSET, 1, s, [&] { return cudaMemsetAsync(c.work_n, 0, sizeof(int), s); }));
     LS_CK(traced(c, TR_HASH_BATCH, 1, s, [&] {
       return launch_hash_screen(n_req, tok, tok_off, c.bkeys, c.bkeys_cap, c.d_err, c.tables, c.mask, c.slots,
-                                c.n_inst, hits, c.work, c.work_n, c.sms, s);
+                                c.n_inst, hits, c.work, c.work_n, c.sms, c.st, s);
     }));
     LS_CK(traced(c, TR_WALK, 1, s, [&] {
       return launch_probe_walk(c.n_inst, tok_off, c.bkeys, c.bkeys_cap, c.tables, c.mask, c.slots, hits,
@@ -455,20 +466,21 @@ int ls_route_batch(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* 
                               c.stdv, c.tc.d_pad, c.xin, c.xrq, c.sms, s);
     }));
     LS_CK(traced(c, TR_SCORE_TC, 1, s, [&] {
-      return launch_score_tc(c.mlp, c.tc, c.pub[b].img, c.pub[b].params, n_req, c.n_inst, tok_off, hits,
+      return launch_score_tc(c.mlp, c.tc, c.pub, &c.st->route_b, n_req, c.n_inst, tok_off, hits,
                              c.xin, c.xrq, c.cfg.d_inst, c.cfg.d_req, c.mean, c.stdv, scores, c.d_err, c.sms,
                              s);
     }));
   } else {
     LS_CK(traced(c, TR_SCORE, 1, s, [&] {
-      return launch_score_simt(c.mlp, c.pub[b], n_req, c.n_inst, tok_off, hits, c.inst_state,
+      return launch_score_simt(c.mlp, c.pub, &c.st->route_b, n_req, c.n_inst, tok_off, hits, c.inst_state,
                                c.cfg.d_inst, req_feats, c.cfg.d_req, c.mean, c.stdv, scores, s);
     }));
   }
   LS_CK(traced(c, TR_ARGMIN, 1, s, [&] { return launch_argmin(n_req, c.n_inst, scores, choice, best, s); }));
-  {
+  if (!cap) {
     std::lock_guard<std::mutex> g(c.mu);
-    LS_CK(cudaEventRecord(c.route_done[b], s));
+    LS_CK(cudaEventRecord(c.ev_route, s));
+    c.route_recorded = true;
   }
   return LS_OK;
 }
@@ -480,11 +492,10 @@ int ls_log_samples(ls_ctx* h, int32_t n, const float* feats, const float* ttft, 
   if (n == 0) return LS_OK;
   if (!feats || !ttft) return fail(LS_ERR_ARG, "NULL argument");
   LS_CK(traced(c, TR_RING, 1, S(stream), [&] {
-    return launch_ring_append(n, c.d, feats, ttft, c.ring_x, c.ring_y, c.ring_count,
-                              c.cfg.ring_capacity, S(stream));
+    return launch_ring_append(n, c.d, feats, ttft, c.ring_x, c.ring_y, c.st, c.cfg.ring_capacity, S(stream));
   }));
   std::lock_guard<std::mutex> g(c.mu);
-  c.ring_count += n;
+  c.ring_enqueued += n;
   return LS_OK;
 }
 
@@ -497,9 +508,8 @@ int ls_train_step(ls_ctx* h, int32_t batch, const int32_t* idx, int32_t opt, flo
   if (!std::isfinite(lr)) return fail(LS_ERR_ARG, "lr is not finite");
   if (!c.have_params) return fail(LS_ERR_STATE, "parameters not set");
   if (!c.have_norm) return fail(LS_ERR_STATE, "normaliser not set");
-  if (c.ring_count < 1) return fail(LS_ERR_STATE, "sample ring is empty");
+  if (c.ring_enqueued < 1) return fail(LS_ERR_STATE, "sample ring is empty");
   LS_CK(run_train_step(c, batch, idx, opt, lr, loss_out, S(stream)));
-  c.step += 1;
   return LS_OK;
 }
 
@@ -508,17 +518,21 @@ int ls_publish(ls_ctx* h, void* stream) {
   Ctx& c = h->c;
   if (!c.have_params) return fail(LS_ERR_STATE, "parameters not set");
   cudaStream_t s = S(stream);
+  const bool cap = capturing(s);
   std::lock_guard<std::mutex> g(c.mu);
-  const int target = c.cur < 0 ? 0 : 1 - c.cur;
-  LS_CK(cudaStreamWaitEvent(s, c.route_done[target], 0));
-  LS_CK(traced(c, TR_PUBLISH, c.mlp.n_layers, s, [&] { return launch_publish(c.mlp, c.master, c.pub[target], s); }));
-  if (c.use_tc)
-    LS_CK(traced(c, TR_PUBLISH_TC, c.tc.n_tc, s,
-                 [&] { return launch_publish_tc(c.mlp, c.tc, c.master, c.pub[target].img, s); }));
-  LS_CK(cudaEventRecord(c.pub_ready[target], s));
+  // the buffer written (1 - cur) may still be read by routes enqueued
+  // earlier, and publishes must not overlap one another
+  if (!cap && c.route_recorded) LS_CK(cudaStreamWaitEvent(s, c.ev_route, 0));
+  if (!cap && c.pub_recorded) LS_CK(cudaStreamWaitEvent(s, c.ev_pub, 0));
+  LS_CK(traced(c, TR_PUBLISH, 1, s, [&] {
+    return launch_publish(c.mlp, c.use_tc ? &c.tc : nullptr, c.master, c.pub, c.use_tc ? 0 : 1, c.st, c.sms, s);
+  }));
+  if (!cap) {
+    LS_CK(cudaEventRecord(c.ev_pub, s));
+    c.pub_recorded = true;
+  }
   c.version += 1;
-  c.pub[target].version = c.version;
-  c.cur = target;
+  c.have_published = true;
   return LS_OK;
 }
 
@@ -543,6 +557,7 @@ int ls_trace_read(ls_ctx* h, ls_trace_entry* out, int32_t max_entries, int32_t* 
     float ms = 0.0f;
     LS_CK(cudaEventElapsedTime(&ms, t.ev[p.a], t.ev[p.a + 1]));
     t.ms[p.id] += ms;
+    t.timed[p.id] += p.launches;
   }
   t.pend.clear();
   t.used = 0;
@@ -554,9 +569,11 @@ int ls_trace_read(ls_ctx* h, ls_trace_entry* out, int32_t max_entries, int32_t* 
       std::strncpy(out[n].name, kTraceNames[id], sizeof(out[n].name) - 1);
       out[n].launches = t.launches[id];
       out[n].total_ms = t.ms[id];
+      out[n].timed_launches = t.timed[id];
     }
     ++n;
     t.launches[id] = 0;
+    t.timed[id] = 0;
     t.ms[id] = 0.0;
   }
   *n_out = n < max_entries ? n : max_entries;

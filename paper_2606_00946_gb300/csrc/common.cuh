@@ -63,6 +63,20 @@ struct Published {
   uint64_t version = 0;
 };
 
+// Counters that change with every step live in device memory so that a whole
+// step (snapshot, route, log, train, publish) can be captured once in a CUDA
+// graph and replayed: kernels read and advance them at execution time.
+struct DevState {
+  int64_t ring_count;       // records appended to the sample ring so far
+  int64_t step;             // optimiser steps taken
+  int32_t cur;              // published buffer routes read (-1: none yet)
+  int32_t route_b;          // buffer chosen by the route in flight (set by its prefix kernel)
+  uint64_t version;         // publishes completed
+  uint64_t pub_version[2];  // version held by each buffer
+  uint32_t done[4];         // per-kernel block arrival counters (last-block updates)
+};
+enum { DONE_RING = 0, DONE_OPT = 1, DONE_PUB = 2 };
+
 // Kernel-level tracing: when enabled, every launch is bracketed by CUDA events
 // recorded on the launching stream; ls_trace_read() sums the elapsed times.
 enum TraceId {
@@ -82,6 +96,7 @@ struct Tracer {
   struct Pending { int id, a, launches; };
   std::vector<Pending> pend;
   int64_t launches[TR_COUNT] = {};
+  int64_t timed[TR_COUNT] = {};   // launches whose time is in ms[] (the rest found the event pool full)
   double ms[TR_COUNT] = {};
   int64_t dropped = 0;
   std::mutex mu;
@@ -127,20 +142,22 @@ struct Ctx {
   float* master = nullptr;
   float* adam_m = nullptr;
   float* adam_v = nullptr;
-  int64_t step = 0;
   bool have_params = false;
 
-  // publish / swap
+  // publish / swap: two buffers, the device-side index st->cur says which
+  // one routes read; a publish writes the other and flips it
   Published pub[2];
-  int cur = -1;
-  uint64_t version = 0;
-  cudaEvent_t pub_ready[2] = {nullptr, nullptr};
-  cudaEvent_t route_done[2] = {nullptr, nullptr};
+  bool have_published = false;   // a publish has been enqueued (host order)
+  uint64_t version = 0;          // publishes enqueued (host order)
+  cudaEvent_t ev_pub = nullptr;    // after the last publish enqueued
+  cudaEvent_t ev_route = nullptr;  // after the last route enqueued
+  bool pub_recorded = false, route_recorded = false;
+  DevState* st = nullptr;
 
   // sample ring (Sec. 4.3.2)
   float* ring_x = nullptr;
   float* ring_y = nullptr;
-  int64_t ring_count = 0;
+  int64_t ring_enqueued = 0;     // records appended (host order); the device count is st->ring_count
 
   // route scratch
   int32_t* hits = nullptr;    // [max_requests, max_instances]
@@ -177,9 +194,15 @@ struct Ctx {
   Tracer tracer;
 };
 
+inline bool capturing(cudaStream_t s) {
+  cudaStreamCaptureStatus st = cudaStreamCaptureStatusNone;
+  return cudaStreamIsCapturing(s, &st) == cudaSuccess && st != cudaStreamCaptureStatusNone;
+}
+
+// Launch bracketed by trace events (skipped while the stream is being captured).
 template <class F>
 cudaError_t traced(Ctx& c, int id, int n_launch, cudaStream_t s, F&& f) {
-  const int t = c.tracer.begin(s);
+  const int t = c.tracer.on && !capturing(s) ? c.tracer.begin(s) : -1;
   const cudaError_t e = f();
   c.tracer.end(t, id, n_launch, s);
   return e;
@@ -194,6 +217,30 @@ __device__ __forceinline__ float round_bf16(float x) {
 
 __device__ __forceinline__ void latch_error(int* err, int code) {
   atomicCAS(err, 0, code);
+}
+
+// The route's choice of published buffer, taken once per route (by thread 0
+// of block 0 of its prefix kernel) so that every scorer CTA reads one version.
+__device__ __forceinline__ void route_snapshot(DevState* st) {
+  if (st && blockIdx.x == 0 && threadIdx.x == 0)
+    st->route_b = *reinterpret_cast<volatile int32_t*>(&st->cur);
+}
+
+// True in exactly one block of the grid: the last to arrive at `done`, after
+// every block has passed this point (so every block's earlier reads of the
+// state it will update are done).  The counter is reset for the next launch.
+__device__ __forceinline__ bool last_block(uint32_t* done) {
+  __shared__ bool is_last;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    const uint32_t nb = gridDim.x * gridDim.y * gridDim.z;
+    const uint32_t t = atomicAdd(done, 1u);
+    is_last = (t == nb - 1);
+    if (is_last) *done = 0u;
+  }
+  __syncthreads();
+  return is_last;
 }
 
 // Raw feature k of pair (request with prompt length L and hit length h,
@@ -229,7 +276,7 @@ cudaError_t launch_hash_blocks(int n_seq, const int32_t* tok, const int64_t* tok
 cudaError_t launch_hash_screen(int n_req, const int32_t* tok, const int64_t* tok_off, uint64_t* keys,
                                int64_t cap, int* err, const uint64_t* tables, uint32_t mask, int64_t slots,
                                int n_inst, int32_t* hits, uint32_t* work, int* work_n, int sms,
-                               cudaStream_t s);
+                               DevState* st, cudaStream_t s);
 cudaError_t launch_probe_walk(int n_inst, const int64_t* tok_off, const uint64_t* keys, int64_t cap,
                               const uint64_t* tables, uint32_t mask, int64_t slots, int32_t* hits,
                               const uint32_t* work, const int* work_n, int sms, cudaStream_t s);
@@ -238,34 +285,35 @@ cudaError_t launch_table_insert(const uint64_t* keys, const int64_t* key_off, in
                                 int32_t* counts, int64_t max_keys, int* err, cudaStream_t s);
 cudaError_t launch_prefix_match(int n_req, const int32_t* tok, const int64_t* tok_off,
                                 const uint64_t* tables, uint32_t mask, int64_t slots, int n_inst,
-                                int32_t* hits, cudaStream_t s);
+                                int32_t* hits, DevState* st, cudaStream_t s);
 
 cudaError_t launch_assemble_features(int n_req, int n_inst, const int64_t* tok_off,
                                      const int32_t* hits, const float* inst_state, int d_inst,
                                      const float* req_feats, int d_req, const float* mean,
                                      const float* stdv, float* x_out, cudaStream_t s);
-cudaError_t launch_score_simt(const MlpDesc& mlp, const Published& pub, int n_req, int n_inst,
+cudaError_t launch_score_simt(const MlpDesc& mlp, const Published* pub, const int32_t* sel, int n_req, int n_inst,
                               const int64_t* tok_off, const int32_t* hits, const float* inst_state,
                               int d_inst, const float* req_feats, int d_req, const float* mean,
                               const float* stdv, float* scores, cudaStream_t s);
 cudaError_t launch_argmin(int n_req, int n_inst, const float* scores, int32_t* choice,
                           float* best, cudaStream_t s);
 
-cudaError_t launch_publish(const MlpDesc& mlp, const float* master, Published& pub,
-                           cudaStream_t s);
 bool plan_tc(const MlpDesc& m, TcPlan& p);
-cudaError_t launch_publish_tc(const MlpDesc& m, const TcPlan& p, const float* master, uint8_t* img,
-                              cudaStream_t s);
+// Publish the master weights into buffer 1 - st->cur (fp32 params, the
+// transposed copy when `want_wt`, the tensor-core image when `tc`), then flip
+// st->cur and bump the version; one launch.
+cudaError_t launch_publish(const MlpDesc& m, const TcPlan* tc, const float* master, const Published* pub,
+                           int want_wt, DevState* st, int sms, cudaStream_t s);
 cudaError_t launch_norm_rows(int n_inst, int d_inst, const float* inst, int n_req, int d_req,
                              const float* req, const float* mean, const float* stdv, int d_pad,
                              uint16_t* xin, uint16_t* xrq, int sms, cudaStream_t s);
-cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const uint8_t* img, const float* params,
+cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const Published* pub, const int32_t* sel,
                             int n_req, int n_inst, const int64_t* tok_off, const int32_t* hits,
                             const uint16_t* xin, const uint16_t* xrq, int d_inst, int d_req,
                             const float* mean, const float* stdv, float* scores, int* err, int sms,
                             cudaStream_t s);
 cudaError_t launch_ring_append(int n, int d, const float* x, const float* y, float* ring_x,
-                               float* ring_y, int64_t count, int64_t capacity, cudaStream_t s);
+                               float* ring_y, DevState* st, int64_t capacity, cudaStream_t s);
 cudaError_t run_train_step(Ctx& c, int batch, const int32_t* idx, int opt, float lr,
                            float* loss_out, cudaStream_t s);
 cudaError_t launch_gemm_tc(int M, int N, int K, const float* A, int64_t sam, int64_t sak, const float* B,
@@ -277,7 +325,7 @@ int index_words(int max_instances);
 void set_last_error(const char* msg);  // sets the text ls_last_error() returns
 cudaError_t launch_prefix_index(int n_req, const int32_t* tok, const int64_t* tok_off, const uint64_t* gkeys,
                                 const uint64_t* gmask, int W, uint64_t gmask_slots, int n_inst, int32_t* hits,
-                                int sms, cudaStream_t s);
+                                int sms, DevState* st, cudaStream_t s);
 cudaError_t launch_index_insert(const uint64_t* keys, const int64_t* key_off, int n_inst, int64_t n_keys,
                                 uint64_t* gkeys, uint64_t* gmask, int W, uint64_t gmask_slots, int32_t* counts,
                                 int64_t max_keys, int* err, int sms, cudaStream_t s);

@@ -37,9 +37,10 @@ __global__ void __launch_bounds__(NT) k_hash_blocks(int n_seq, const int32_t* __
                                                     const int64_t* __restrict__ key_off, int64_t cap, int* err,
                                                     const uint64_t* __restrict__ tables, uint32_t mask,
                                                     int64_t slots, int n_inst, int32_t* __restrict__ hits,
-                                                    uint32_t* __restrict__ work, int* work_n) {
+                                                    uint32_t* __restrict__ work, int* work_n, DevState* st) {
   constexpr int W = NT / 32;
   __shared__ uint64_t wtot[W], wpre[W], carry, key0;
+  route_snapshot(st);
   const int64_t tbase = tok_off[0];
   const int lane = threadIdx.x & 31;
   for (int s = blockIdx.x; s < n_seq; s += gridDim.x) {
@@ -163,8 +164,9 @@ __global__ void __launch_bounds__(kThreads) k_prefix_match(int n_req, const int3
                                                            const int64_t* __restrict__ tok_off,
                                                            const uint64_t* __restrict__ tables,
                                                            uint32_t mask, int64_t slots, int n_inst,
-                                                           int32_t* __restrict__ hits) {
+                                                           int32_t* __restrict__ hits, DevState* st) {
   __shared__ uint64_t keys[kThreads];
+  route_snapshot(st);
   __shared__ uint64_t wtot[kWarps], wpre[kWarps], carry;
   __shared__ int n_alive, n_list;
   extern __shared__ int32_t dyn[];
@@ -276,19 +278,19 @@ cudaError_t launch_hash_blocks(int n_seq, const int32_t* tok, const int64_t* tok
                                cudaStream_t s) {
   if (n_seq <= 0) return cudaSuccess;
   k_hash_blocks<kThreads><<<grid_for(n_seq), kThreads, 0, s>>>(n_seq, tok, tok_off, keys_out, key_off, cap, err,
-                                                             nullptr, 0, 0, 0, nullptr, nullptr, nullptr);
+                                                             nullptr, 0, 0, 0, nullptr, nullptr, nullptr, nullptr);
   return cudaGetLastError();
 }
 
 cudaError_t launch_hash_screen(int n_req, const int32_t* tok, const int64_t* tok_off, uint64_t* keys,
                                int64_t cap, int* err, const uint64_t* tables, uint32_t mask, int64_t slots,
                                int n_inst, int32_t* hits, uint32_t* work, int* work_n, int sms,
-                               cudaStream_t s) {
+                               DevState* st, cudaStream_t s) {
   if (n_req <= 0) return cudaSuccess;
   constexpr int NT = 128;
   const int grid = std::min(n_req, sms * 16);
   k_hash_blocks<NT><<<grid, NT, 0, s>>>(n_req, tok, tok_off, keys, nullptr, cap, err, tables, mask, slots, n_inst,
-                                        hits, work, work_n);
+                                        hits, work, work_n, st);
   return cudaGetLastError();
 }
 
@@ -315,7 +317,7 @@ cudaError_t launch_table_insert(const uint64_t* keys, const int64_t* key_off, in
 
 cudaError_t launch_prefix_match(int n_req, const int32_t* tok, const int64_t* tok_off,
                                 const uint64_t* tables, uint32_t mask, int64_t slots, int n_inst,
-                                int32_t* hits, cudaStream_t s) {
+                                int32_t* hits, DevState* st, cudaStream_t s) {
   if (n_req <= 0) return cudaSuccess;
   const size_t smem = (size_t)n_inst * 4 * sizeof(int32_t);
   if (smem > 48 * 1024) {
@@ -324,7 +326,7 @@ cudaError_t launch_prefix_match(int n_req, const int32_t* tok, const int64_t* to
     if (e != cudaSuccess) return e;
   }
   k_prefix_match<<<grid_for(n_req), kThreads, smem, s>>>(n_req, tok, tok_off, tables, mask, slots,
-                                                         n_inst, hits);
+                                                         n_inst, hits, st);
   return cudaGetLastError();
 }
 

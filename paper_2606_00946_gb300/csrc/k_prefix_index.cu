@@ -48,8 +48,9 @@ __global__ void __launch_bounds__(kNT) k_prefix_index(int n_req, const int32_t* 
                                                       const int64_t* __restrict__ tok_off,
                                                       const uint64_t* __restrict__ gkeys,
                                                       const uint64_t* __restrict__ gmask, uint64_t gmask_slots,
-                                                      int n_inst, int32_t* __restrict__ hits) {
+                                                      int n_inst, int32_t* __restrict__ hits, DevState* st) {
   __shared__ uint64_t keys[kNT];
+  route_snapshot(st);
   __shared__ uint64_t wtot[kNT / 32], wpre[kNT / 32], carry;
   __shared__ int any_alive;
   const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
@@ -171,14 +172,14 @@ int index_words(int max_instances) { return max_instances <= 64 ? 1 : max_instan
 
 cudaError_t launch_prefix_index(int n_req, const int32_t* tok, const int64_t* tok_off, const uint64_t* gkeys,
                                 const uint64_t* gmask, int W, uint64_t gmask_slots, int n_inst, int32_t* hits,
-                                int sms, cudaStream_t s) {
+                                int sms, DevState* st, cudaStream_t s) {
   if (n_req <= 0) return cudaSuccess;
   const int grid = std::min(n_req, sms * 16);
   switch (W) {
-    case 1: k_prefix_index<1><<<grid, kNT, 0, s>>>(n_req, tok, tok_off, gkeys, gmask, gmask_slots, n_inst, hits); break;
-    case 2: k_prefix_index<2><<<grid, kNT, 0, s>>>(n_req, tok, tok_off, gkeys, gmask, gmask_slots, n_inst, hits); break;
-    case 4: k_prefix_index<4><<<grid, kNT, 0, s>>>(n_req, tok, tok_off, gkeys, gmask, gmask_slots, n_inst, hits); break;
-    case 8: k_prefix_index<8><<<grid, kNT, 0, s>>>(n_req, tok, tok_off, gkeys, gmask, gmask_slots, n_inst, hits); break;
+    case 1: k_prefix_index<1><<<grid, kNT, 0, s>>>(n_req, tok, tok_off, gkeys, gmask, gmask_slots, n_inst, hits, st); break;
+    case 2: k_prefix_index<2><<<grid, kNT, 0, s>>>(n_req, tok, tok_off, gkeys, gmask, gmask_slots, n_inst, hits, st); break;
+    case 4: k_prefix_index<4><<<grid, kNT, 0, s>>>(n_req, tok, tok_off, gkeys, gmask, gmask_slots, n_inst, hits, st); break;
+    case 8: k_prefix_index<8><<<grid, kNT, 0, s>>>(n_req, tok, tok_off, gkeys, gmask, gmask_slots, n_inst, hits, st); break;
     default: return cudaErrorInvalidValue;
   }
   return cudaGetLastError();

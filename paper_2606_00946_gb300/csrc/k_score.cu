@@ -1,8 +1,7 @@
 // Scoring kernels on CUDA cores: feature assembly (Sec. 4.1 Features,
 // Algorithm 4 Normalize), the reward-model forward pass for small or fp32
 // predictors (Sec. 4.1 Model architecture), the greedy argmin selector
-// (Algorithm 4, argmax reward = argmin predicted TTFT), weight publishing and
-// the sample ring.
+// (Algorithm 4, argmax reward = argmin predicted TTFT) and the sample ring.
 #include "common.cuh"
 
 namespace ls {
@@ -48,8 +47,11 @@ __global__ void k_assemble(int n_req, int n_inst, const int64_t* __restrict__ to
 // from the transposed weights W^T [in, out] (coalesced across threads);
 // output layer (width 1): one warp per row, lanes split the dot product.
 template <int TR>
-__global__ void __launch_bounds__(256) k_score_simt(MlpDesc mlp, const float* __restrict__ pp,
-                                                    const float* __restrict__ wt, int n_req,
+__global__ void __launch_bounds__(256) k_score_simt(MlpDesc mlp, const float* __restrict__ pp0,
+                                                    const float* __restrict__ wt0,
+                                                    const float* __restrict__ pp1,
+                                                    const float* __restrict__ wt1,
+                                                    const int32_t* __restrict__ sel, int n_req,
                                                     int n_inst, const int64_t* __restrict__ tok_off,
                                                     const int32_t* __restrict__ hits,
                                                     const float* __restrict__ inst_state, int d_inst,
@@ -58,6 +60,9 @@ __global__ void __launch_bounds__(256) k_score_simt(MlpDesc mlp, const float* __
                                                     const float* __restrict__ stdv,
                                                     float* __restrict__ scores) {
   extern __shared__ float smem[];
+  const bool b1 = sel && *sel == 1;  // published buffer of this route
+  const float* __restrict__ pp = b1 ? pp1 : pp0;
+  const float* __restrict__ wt = b1 ? wt1 : wt0;
   const int H = mlp.max_width;
   float* a = smem;
   float* b = smem + TR * H;
@@ -140,29 +145,14 @@ __global__ void k_argmin(int n_req, int n_inst, const float* __restrict__ scores
   if (lane == 0) { choice[r] = bi; best[r] = bv; }
 }
 
-// Publish layer l: rounded weights (bf16 mode), biases, and the transposed copy.
-__global__ void k_publish_layer(const float* __restrict__ W, const float* __restrict__ bsrc,
-                                int out, int in, int bf16, float* __restrict__ Wdst,
-                                float* __restrict__ bdst, float* __restrict__ Wt) {
-  const int64_t n = (int64_t)out * in;
-  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n + out;
-       e += (int64_t)gridDim.x * blockDim.x) {
-    if (e < n) {
-      const int o = (int)(e / in), k = (int)(e - (int64_t)o * in);
-      const float v = bf16 ? round_bf16(W[e]) : W[e];
-      Wdst[e] = v;
-      Wt[(int64_t)k * out + o] = v;
-    } else {
-      bdst[e - n] = bsrc[e - n];
-    }
-  }
-}
-
-// Record j of the batch -> slot (count + j) mod capacity.  When a batch is
-// longer than the ring only its last `capacity` records are kept.
+// Record j of the batch -> slot (count + j) mod capacity, count = records
+// appended before this batch (device state); the last block advances the
+// count by n.  When a batch is longer than the ring only its last `capacity`
+// records are kept.
 __global__ void k_ring_append(int n, int d, const float* __restrict__ x, const float* __restrict__ y,
-                              float* __restrict__ ring_x, float* __restrict__ ring_y, int64_t count,
+                              float* __restrict__ ring_x, float* __restrict__ ring_y, DevState* st,
                               int64_t capacity) {
+  const int64_t count = *reinterpret_cast<volatile int64_t*>(&st->ring_count);
   const int64_t first = n > capacity ? n - capacity : 0;
   const int64_t total = (int64_t)(n - first) * (d + 1);
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
@@ -173,6 +163,7 @@ __global__ void k_ring_append(int n, int d, const float* __restrict__ x, const f
     if (k < d) ring_x[slot * d + k] = x[j * d + k];
     else ring_y[slot] = y[j];
   }
+  if (last_block(&st->done[DONE_RING]) && threadIdx.x == 0) st->ring_count = count + n;
 }
 
 int sm_count() {
@@ -201,7 +192,7 @@ cudaError_t launch_assemble_features(int n_req, int n_inst, const int64_t* tok_o
   return cudaGetLastError();
 }
 
-cudaError_t launch_score_simt(const MlpDesc& mlp, const Published& pub, int n_req, int n_inst,
+cudaError_t launch_score_simt(const MlpDesc& mlp, const Published* pub, const int32_t* sel, int n_req, int n_inst,
                               const int64_t* tok_off, const int32_t* hits, const float* inst_state,
                               int d_inst, const float* req_feats, int d_req, const float* mean,
                               const float* stdv, float* scores, cudaStream_t s) {
@@ -215,7 +206,8 @@ cudaError_t launch_score_simt(const MlpDesc& mlp, const Published& pub, int n_re
   int64_t tiles = (rows + TR - 1) / TR;
   const int64_t cap = (int64_t)sm_count() * 8;
   const int grid = (int)(tiles > cap ? cap : tiles);
-  k_score_simt<TR><<<grid, 256, smem, s>>>(mlp, pub.params, pub.wt, n_req, n_inst, tok_off, hits,
+  k_score_simt<TR><<<grid, 256, smem, s>>>(mlp, pub[0].params, pub[0].wt, pub[1].params, pub[1].wt, sel, n_req,
+                                           n_inst, tok_off, hits,
                                            inst_state, d_inst, req_feats, d_req, mean, stdv, scores);
   return cudaGetLastError();
 }
@@ -228,25 +220,12 @@ cudaError_t launch_argmin(int n_req, int n_inst, const float* scores, int32_t* c
   return cudaGetLastError();
 }
 
-cudaError_t launch_publish(const MlpDesc& mlp, const float* master, Published& pub, cudaStream_t s) {
-  for (int l = 0; l < mlp.n_layers; ++l) {
-    const int out = mlp.w[l + 1], in = mlp.w[l];
-    const int64_t n = (int64_t)out * in + out;
-    k_publish_layer<<<grid_1d(n, 256), 256, 0, s>>>(master + mlp.woff[l], master + mlp.boff[l], out, in,
-                                                   mlp.bf16, pub.params + mlp.woff[l],
-                                                   pub.params + mlp.boff[l], pub.wt + mlp.wtoff[l]);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-  }
-  return cudaSuccess;
-}
-
 cudaError_t launch_ring_append(int n, int d, const float* x, const float* y, float* ring_x,
-                               float* ring_y, int64_t count, int64_t capacity, cudaStream_t s) {
+                               float* ring_y, DevState* st, int64_t capacity, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
   const int64_t keep = n > capacity ? capacity : n;
   const int64_t total = keep * (d + 1);
-  k_ring_append<<<grid_1d(total, 256), 256, 0, s>>>(n, d, x, y, ring_x, ring_y, count, capacity);
+  k_ring_append<<<grid_1d(total, 256), 256, 0, s>>>(n, d, x, y, ring_x, ring_y, st, capacity);
   return cudaGetLastError();
 }
 

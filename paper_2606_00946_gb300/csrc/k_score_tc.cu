@@ -29,8 +29,11 @@ constexpr int kMaxSmem = 232448;  // 227 KB opt-in per CTA
 
 struct TcArgs {
   TcPlan p;
-  const uint8_t* img;
-  const float* params;
+  const uint8_t* img0;     // published buffer 0 / 1: tensor-core weight image
+  const uint8_t* img1;
+  const float* params0;    // published buffer 0 / 1: flat fp32 parameters
+  const float* params1;
+  const int32_t* sel;      // buffer this route reads (device), NULL: buffer 0
   int64_t boff[LS_MAX_LAYERS];
   int64_t w_last_off;
   int n_req, n_inst, d, d_inst, d_req;
@@ -134,6 +137,9 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
 __device__ __forceinline__ float4 ldg4(const float* p) { return __ldg(reinterpret_cast<const float4*>(p)); }
 
 __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc(const __grid_constant__ TcArgs a) {
+  const bool pb = a.sel && *a.sel == 1;  // published buffer of this route
+  const uint8_t* __restrict__ img = pb ? a.img1 : a.img0;
+  const float* __restrict__ params = pb ? a.params1 : a.params0;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const TcPlan& p = a.p;
@@ -177,7 +183,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc(const __grid_constan
     if (u >= 1 && !mbar_wait(&empty[s], (uint32_t)((u - 1) & 1))) return false;
     const int q = (int)(gq % p.chunks);
     mbar_arrive_expect_tx(&full[s], (uint32_t)p.chunk_len[q]);
-    bulk_g2s(ring + (size_t)s * p.chunk_bytes, a.img + p.chunk_off[q], (uint32_t)p.chunk_len[q], &full[s]);
+    bulk_g2s(ring + (size_t)s * p.chunk_bytes, img + p.chunk_off[q], (uint32_t)p.chunk_len[q], &full[s]);
     return true;
   };
 
@@ -185,7 +191,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc(const __grid_constan
     if (p.resident) {
       for (int q = 0; q < p.chunks; ++q) {
         mbar_arrive_expect_tx(&full[q], (uint32_t)p.chunk_len[q]);
-        bulk_g2s(ring + (size_t)q * p.chunk_bytes, a.img + p.chunk_off[q], (uint32_t)p.chunk_len[q], &full[q]);
+        bulk_g2s(ring + (size_t)q * p.chunk_bytes, img + p.chunk_off[q], (uint32_t)p.chunk_len[q], &full[q]);
       }
     } else {
       while (g_load < total && g_load < p.stages - 1) {
@@ -258,7 +264,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc(const __grid_constan
       tc_fence_after();
       const int qw = p.out[l] / 4;  // columns per warp
       const int cbeg = cq * qw;
-      const float* bias = a.params + a.boff[l];
+      const float* bias = params + a.boff[l];
       if (l + 1 < p.n_tc) {
         // hidden epilogue: bias, ReLU, bf16 -> next layer's operand tile
         for (int c0 = cbeg; c0 < cbeg + qw; c0 += 16) {
@@ -282,7 +288,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc(const __grid_constan
         __syncthreads();
       } else {
         // last hidden layer: bias, ReLU, bf16 rounding, then the width-1 output layer
-        const float* wl = a.params + a.w_last_off;
+        const float* wl = params + a.w_last_off;
         float sacc = 0.0f;
         for (int c0 = cbeg; c0 < cbeg + qw; c0 += 16) {
           uint32_t v[16];
@@ -309,7 +315,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc(const __grid_constan
           const int64_t g = row0 + tid;
           if (g < a.rows)
             a.scores[g] = ((part[tid] + part[kTileM + tid]) + (part[2 * kTileM + tid] + part[3 * kTileM + tid])) +
-                          __ldg(a.params + a.p.b_last_off);
+                          __ldg(params + a.p.b_last_off);
         }
         __syncthreads();
       }
@@ -398,6 +404,9 @@ __device__ __forceinline__ void build_tile_part(const TcArgs& a, uint8_t* X, int
 }
 
 __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc_pipe(const __grid_constant__ TcArgs a) {
+  const bool pb = a.sel && *a.sel == 1;  // published buffer of this route
+  const uint8_t* __restrict__ img = pb ? a.img1 : a.img0;
+  const float* __restrict__ params = pb ? a.params1 : a.params0;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const TcPlan& p = a.p;
@@ -456,7 +465,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc_pipe(const __grid_co
       for (int q = 0; q < p.chunks; ++q) wbytes += p.chunk_len[q];
       mbar_arrive_expect_tx(w_full, (uint32_t)wbytes);
       for (int q = 0; q < p.chunks; ++q)
-        bulk_g2s(W + (size_t)q * p.chunk_bytes, a.img + p.chunk_off[q], (uint32_t)p.chunk_len[q], w_full);
+        bulk_g2s(W + (size_t)q * p.chunk_bytes, img + p.chunk_off[q], (uint32_t)p.chunk_len[q], w_full);
       bool ok = mbar_wait(w_full, 0);
       const uint32_t id1 = idesc_bf16_f32(kTileM, H1), id2 = idesc_bf16_f32(kTileM, H2);
       for (int t = 0; t < my_tiles && ok; ++t) {
@@ -524,10 +533,10 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc_pipe(const __grid_co
     const int wk = ew >> 2;                // 0/1: column half
     const int row = 32 * q4 + lane;
     const uint32_t lane_addr = (uint32_t)(32 * q4) << 16;
-    const float* b1 = a.params + a.boff[0];
-    const float* b2 = a.params + a.boff[1];
-    const float* w3 = a.params + a.w_last_off;
-    const float b3 = __ldg(a.params + p.b_last_off);
+    const float* b1 = params + a.boff[0];
+    const float* b2 = params + a.boff[1];
+    const float* w3 = params + a.w_last_off;
+    const float b3 = __ldg(params + p.b_last_off);
     for (int t = 0; t < my_tiles; ++t) {
       const int64_t row0 = (int64_t)(blockIdx.x + (int64_t)t * gridDim.x) * kTileM;
       if (!mbar_wait(d1_full, (uint32_t)(t & 1))) { *abort_flag = 1; latch_error(a.err, LS_ERR_TIMEOUT); break; }
@@ -637,21 +646,6 @@ __global__ void k_norm_rows(int n_inst, int d_inst, const float* __restrict__ in
   }
 }
 
-// Pre-swizzled bf16 image of hidden layer l: N-chunks of nc rows, each split into
-// K-blocks of 64 columns laid out exactly as the MMA reads them from shared memory.
-__global__ void k_publish_tc(const float* __restrict__ W, int out, int in, int in_pad, int nc,
-                             uint8_t* __restrict__ img) {
-  const int64_t n = (int64_t)out * in_pad;
-  const int nk = in_pad / 64;
-  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n; e += (int64_t)gridDim.x * blockDim.x) {
-    const int o = (int)(e / in_pad), k = (int)(e - (int64_t)o * in_pad);
-    const float v = k < in ? W[(int64_t)o * in + k] : 0.0f;
-    const int nci = o / nc, orow = o - nci * nc;
-    const int64_t off = (int64_t)nci * nk * nc * 128 + sw128_offset(orow, k, nc);
-    *reinterpret_cast<uint16_t*>(img + off) = bf16_bits(v);
-  }
-}
-
 }  // namespace
 
 bool plan_tc(const MlpDesc& m, TcPlan& p) {
@@ -719,19 +713,6 @@ bool plan_tc(const MlpDesc& m, TcPlan& p) {
   return true;
 }
 
-cudaError_t launch_publish_tc(const MlpDesc& m, const TcPlan& p, const float* master, uint8_t* img,
-                              cudaStream_t s) {
-  for (int l = 0; l < p.n_tc; ++l) {
-    const int64_t n = (int64_t)p.out[l] * p.in_pad[l];
-    const int grid = (int)std::min<int64_t>((n + 255) / 256, 1024);
-    k_publish_tc<<<grid, 256, 0, s>>>(master + m.woff[l], p.out[l], m.w[l], p.in_pad[l], p.nc[l],
-                                      img + p.img_off[l]);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-  }
-  return cudaSuccess;
-}
-
 cudaError_t launch_norm_rows(int n_inst, int d_inst, const float* inst, int n_req, int d_req, const float* req,
                              const float* mean, const float* stdv, int d_pad, uint16_t* xin, uint16_t* xrq,
                              int sms, cudaStream_t s) {
@@ -742,7 +723,7 @@ cudaError_t launch_norm_rows(int n_inst, int d_inst, const float* inst, int n_re
   return cudaGetLastError();
 }
 
-cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const uint8_t* img, const float* params,
+cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const Published* pub, const int32_t* sel,
                             int n_req, int n_inst, const int64_t* tok_off, const int32_t* hits,
                             const uint16_t* xin, const uint16_t* xrq, int d_inst, int d_req, const float* mean,
                             const float* stdv, float* scores, int* err, int sms, cudaStream_t s) {
@@ -750,8 +731,11 @@ cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const uint8_t* im
   if (rows <= 0) return cudaSuccess;
   TcArgs a{};
   a.p = p;
-  a.img = img;
-  a.params = params;
+  a.img0 = pub[0].img;
+  a.img1 = pub[1].img;
+  a.params0 = pub[0].params;
+  a.params1 = pub[1].params;
+  a.sel = sel;
   for (int l = 0; l < m.n_layers; ++l) a.boff[l] = m.boff[l];
   a.w_last_off = p.w_last_off;
   a.n_req = n_req;

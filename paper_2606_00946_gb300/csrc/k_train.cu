@@ -103,12 +103,18 @@ __global__ void __launch_bounds__(256) k_gemm(GemmArgs g) {
 }
 
 // Minibatch rows: slot = idx[j] (checked against the filled part of the ring)
-// or (step*B + j) mod valid; z-score in fp32, bf16-rounded in bf16 mode.
-__global__ void k_train_gather(int B, int d, const int32_t* __restrict__ idx, int64_t step,
-                               int64_t valid, const float* __restrict__ ring_x,
+// or (step*B + j) mod valid, with step and the ring's fill read from the device
+// state; z-score in fp32, bf16-rounded in bf16 mode.  An empty ring latches
+// LS_ERR_STATE (rows then come from slot 0).
+__global__ void k_train_gather(int B, int d, const int32_t* __restrict__ idx, const DevState* st,
+                               int64_t capacity, const float* __restrict__ ring_x,
                                const float* __restrict__ ring_y, const float* __restrict__ mean,
                                const float* __restrict__ stdv, int bf16, float* __restrict__ x0,
                                float* __restrict__ y, int* err) {
+  const int64_t step = st->step;
+  const int64_t count = st->ring_count;
+  const int64_t valid = count < capacity ? count : capacity;
+  if (valid < 1 && blockIdx.x == 0 && threadIdx.x == 0) latch_error(err, LS_ERR_STATE);
   const int64_t total = (int64_t)B * d;
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
        e += (int64_t)gridDim.x * blockDim.x) {
@@ -121,7 +127,7 @@ __global__ void k_train_gather(int B, int d, const int32_t* __restrict__ idx, in
         slot = 0;
       }
     } else {
-      slot = (step * (int64_t)B + j) % valid;
+      slot = valid > 0 ? (step * (int64_t)B + j) % valid : 0;
     }
     const float v = zscore(ring_x[slot * d + k], mean[k], stdv[k]);
     x0[e] = bf16 ? round_bf16(v) : v;
@@ -247,14 +253,27 @@ __global__ void k_reduce_partials(int S, int64_t n, const float* __restrict__ pa
   }
 }
 
-__global__ void k_sgd(int64_t n, float lr, const float* __restrict__ g, float* __restrict__ p) {
+// Optimiser updates.  Each advances the device step counter once (last block),
+// after every block has read it.
+__global__ void k_sgd(int64_t n, float lr, const float* __restrict__ g, float* __restrict__ p, DevState* st) {
+  const int64_t t = st->step + 1;
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n;
        e += (int64_t)gridDim.x * blockDim.x)
     p[e] = p[e] - lr * g[e];
+  if (last_block(&st->done[DONE_OPT]) && threadIdx.x == 0) st->step = t;
 }
 
-__global__ void k_adam(int64_t n, float lr, float bc1, float bc2, const float* __restrict__ g,
-                       float* __restrict__ p, float* __restrict__ m, float* __restrict__ v) {
+// Adam, t = steps taken + 1: bias corrections 1 - beta^t formed in fp64.
+__global__ void k_adam(int64_t n, float lr, const float* __restrict__ g, float* __restrict__ p,
+                       float* __restrict__ m, float* __restrict__ v, DevState* st) {
+  __shared__ float bc[2];
+  const int64_t t = st->step + 1;
+  if (threadIdx.x == 0) {
+    bc[0] = (float)(1.0 - pow(0.9, (double)t));
+    bc[1] = (float)(1.0 - pow(0.999, (double)t));
+  }
+  __syncthreads();
+  const float bc1 = bc[0], bc2 = bc[1];
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n;
        e += (int64_t)gridDim.x * blockDim.x) {
     const float ge = g[e];
@@ -265,6 +284,7 @@ __global__ void k_adam(int64_t n, float lr, float bc1, float bc2, const float* _
     const float mh = me / bc1, vh = ve / bc2;
     p[e] = p[e] - lr * mh / (sqrtf(vh) + 1e-8f);
   }
+  if (last_block(&st->done[DONE_OPT]) && threadIdx.x == 0) st->step = t;
 }
 
 template <bool TA, bool TB, int EPI>
@@ -287,7 +307,6 @@ cudaError_t run_train_step(Ctx& c, int B, const int32_t* idx, int opt, float lr,
                            cudaStream_t s) {
   const MlpDesc& m = c.mlp;
   const int L = m.n_layers;
-  const int64_t valid = std::min<int64_t>(c.ring_count, c.cfg.ring_capacity);
   int64_t xoff[LS_MAX_LAYERS + 1], zoff[LS_MAX_LAYERS + 1];
   xoff[0] = zoff[0] = 0;
   for (int l = 0; l < L; ++l) {
@@ -299,7 +318,7 @@ cudaError_t run_train_step(Ctx& c, int B, const int32_t* idx, int opt, float lr,
     const int64_t total = (int64_t)B * m.w[0];
     int grid = (int)std::min<int64_t>((total + 255) / 256, (int64_t)c.sms * 8);
     e = traced(c, TR_GATHER, 1, s, [&] {
-      k_train_gather<<<std::max(grid, 1), 256, 0, s>>>(B, m.w[0], idx, c.step, valid, c.ring_x,
+      k_train_gather<<<std::max(grid, 1), 256, 0, s>>>(B, m.w[0], idx, c.st, c.cfg.ring_capacity, c.ring_x,
                                                        c.ring_y, c.mean, c.stdv, m.bf16, c.tx, c.ty,
                                                        c.d_err);
       return cudaGetLastError();
@@ -449,14 +468,8 @@ cudaError_t run_train_step(Ctx& c, int B, const int32_t* idx, int opt, float lr,
   }
   const int grid = (int)std::min<int64_t>((c.n_params + 255) / 256, (int64_t)c.sms * 8);
   return traced(c, TR_OPT, 1, s, [&] {
-    if (opt == LS_SGD) {
-      k_sgd<<<grid, 256, 0, s>>>(c.n_params, lr, c.grad, c.master);
-    } else {
-      const double t = (double)(c.step + 1);
-      const float bc1 = (float)(1.0 - std::pow(0.9, t));
-      const float bc2 = (float)(1.0 - std::pow(0.999, t));
-      k_adam<<<grid, 256, 0, s>>>(c.n_params, lr, bc1, bc2, c.grad, c.master, c.adam_m, c.adam_v);
-    }
+    if (opt == LS_SGD) k_sgd<<<grid, 256, 0, s>>>(c.n_params, lr, c.grad, c.master, c.st);
+    else k_adam<<<grid, 256, 0, s>>>(c.n_params, lr, c.grad, c.master, c.adam_m, c.adam_v, c.st);
     return cudaGetLastError();
   });
 }

@@ -102,7 +102,7 @@ extern "C" int ls_prefix_hits_static(int32_t n_req, const int32_t* tok, const in
   cudaError_t e = cudaMemsetAsync(work_n, 0, 2 * sizeof(int), s);
   if (e == cudaSuccess)
     e = launch_hash_screen(n_req, tok, tok_off, keys, kStaticBlocks, err, tables, mask, slots_per_instance, n_inst,
-                           hits_out, work, work_n, d.sms, s);
+                           hits_out, work, work_n, d.sms, nullptr, s);
   if (e == cudaSuccess)
     e = launch_probe_walk(n_inst, tok_off, keys, kStaticBlocks, tables, mask, slots_per_instance, hits_out, work,
                           work_n, d.sms, s);

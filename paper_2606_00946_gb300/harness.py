@@ -123,6 +123,29 @@ class Router:
         L.check(L.ls_publish(self.h, stream))
 
 
+class StepGraph:
+    """ABI calls of one step recorded once by stream capture, then replayed.
+
+    `body` issues the calls (on the current stream, which is the capture stream
+    while recording); every pointer it passes is baked into the graph, so new
+    inputs of a step are copied into the same buffers before `replay()`.  The
+    library keeps its per-step counters on the device, so a replay behaves
+    like issuing the calls again.  Run `body` eagerly at least once first
+    (kernel loading and shared-memory attributes happen outside capture).
+    """
+
+    def __init__(self, body, stream=None):
+        self.graph = torch.cuda.CUDAGraph()
+        s = stream if stream is not None else torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.graph(self.graph, stream=s):
+            body()
+        torch.cuda.current_stream().wait_stream(s)
+
+    def replay(self):
+        self.graph.replay()
+
+
 class DeviceWorkload:
     """A workload's arrays resident in HBM, plus each instance's key CSR."""
 

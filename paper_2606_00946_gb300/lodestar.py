@@ -42,7 +42,8 @@ class ls_info(C.Structure):
 
 
 class ls_trace_entry(C.Structure):
-    _fields_ = [("name", C.c_char * 32), ("launches", C.c_int64), ("total_ms", C.c_double)]
+    _fields_ = [("name", C.c_char * 32), ("launches", C.c_int64), ("total_ms", C.c_double),
+                ("timed_launches", C.c_int64)]
 
 
 _P, _i32, _i64 = C.c_void_p, C.c_int32, C.c_int64
@@ -247,11 +248,12 @@ def ls_trace_enable(ctx, on=True) -> int:
 
 
 def ls_trace_read(ctx, max_entries=64):
-    """Returns (status, {name: (launches, total_ms)})."""
+    """Returns (status, {name: (launches, total_ms, timed_launches)})."""
     arr = (ls_trace_entry * max_entries)()
     n = _i32(0)
     rc = lib().ls_trace_read(ctx, arr, max_entries, C.byref(n))
-    return rc, {arr[i].name.decode(): (arr[i].launches, arr[i].total_ms) for i in range(n.value)}
+    return rc, {arr[i].name.decode(): (arr[i].launches, arr[i].total_ms, arr[i].timed_launches)
+                for i in range(n.value)}
 
 
 def ls_prefix_hits_static(n_req, tok, tok_off, n_tokens, tables, slots_per_instance, n_inst, hits_out,

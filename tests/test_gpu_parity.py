@@ -474,3 +474,91 @@ def test_table_full_and_bad_slot_are_latched():
     r.train(2, torch.tensor([1, 9], dtype=torch.int32, device="cuda"), opt="sgd", lr=0.0)
     assert r.sync() == L.LS_ERR_ARG
     r.close()
+
+
+# ----------------------------------------------------------------------------
+# a whole step captured in a CUDA graph; tracing
+# ----------------------------------------------------------------------------
+
+def test_graph_replay_matches_eager_steps():
+    # Two contexts fed the same inputs: one issues snapshot/route/log/train/
+    # publish eagerly every step, the other replays one captured graph.  The
+    # device counters make each replay a new step, so routes, losses, weights
+    # and counters agree bit for bit.
+    wl = W.generate("homogeneous")
+    cfg = wl.cfg
+    Bt = 512
+    ctxs = []
+    for _ in range(2):
+        r = H.Router.for_config(cfg, ring_capacity=8 * Bt, max_train_batch=Bt)
+        dw = H.DeviceWorkload(wl)
+        dw.load(r)
+        ctxs.append((r, dw))
+    R, N = cfg.n_req, cfg.n_inst
+    sx = torch.from_numpy(wl.samples_x[: 6 * Bt]).cuda()
+    sy = torch.from_numpy(wl.samples_y[: 6 * Bt]).cuda()
+    states = [ctxs[0][1].inst_state,
+              torch.from_numpy(W.instance_state(np.random.default_rng(99), cfg)).cuda()]
+
+    def make(r, dw):
+        bufs = dict(state=torch.empty_like(states[0]), x=torch.empty(Bt, cfg.d, device="cuda"),
+                    y=torch.empty(Bt, device="cuda"), loss=torch.zeros(1, device="cuda"),
+                    out={"choice": torch.empty(R, dtype=torch.int32, device="cuda"),
+                         "best": torch.empty(R, device="cuda"),
+                         "scores": torch.empty(R, N, device="cuda"), "hits": None})
+
+        def feed(k):
+            bufs["state"].copy_(states[k & 1])
+            a = (k * Bt) % len(sy)
+            bufs["x"].copy_(sx[a:a + Bt])
+            bufs["y"].copy_(sy[a:a + Bt])
+
+        def body():
+            r.snapshot(N, bufs["state"])
+            r.route(dw.tok, dw.tok_off, dw.req_feats, N, out=bufs["out"])
+            r.log(bufs["x"], bufs["y"])
+            r.train(Bt, None, opt="adam", lr=1e-3, loss_out=bufs["loss"])
+            r.publish()
+        return bufs, feed, body
+
+    (ra, dwa), (rb, dwb) = ctxs
+    A, feed_a, body_a = make(ra, dwa)
+    Bb, feed_b, body_b = make(rb, dwb)
+    feed_a(0); body_a()
+    feed_b(0); body_b()                     # eager warm-up step on both
+    g = H.StepGraph(body_b)                 # recording runs nothing
+    prev = ra.get_params().cpu().numpy()    # published at the end of step 0
+    sample = np.arange(0, R, R // 8)
+    for k in range(1, 6):
+        feed_a(k); body_a()
+        feed_b(k); g.replay()
+        torch.cuda.synchronize()
+        assert torch.equal(A["out"]["choice"], Bb["out"]["choice"])
+        assert torch.equal(A["out"]["scores"], Bb["out"]["scores"])
+        assert torch.equal(A["loss"], Bb["loss"])
+        if k % 2 == 0:
+            # step k routed with the weights published by step k - 1 and the
+            # workload's own instance state
+            ref = oracle.route(wl, params=prev, req_idx=sample, inst_keys=oracle_inst_keys("homogeneous", wl))
+            assert_scores_close(Bb["out"]["scores"].cpu().numpy()[sample], ref["scores"], TOL["bf16"])
+        prev = ra.get_params().cpu().numpy()
+    assert torch.equal(ra.get_params(), rb.get_params())
+    ia, ib = ra.info(), rb.info()
+    assert (ia.ring_count, ia.train_steps, ia.weight_version) == (6 * Bt, 6, 7)
+    assert (ib.ring_count, ib.train_steps, ib.weight_version) == (6 * Bt, 6, 7)
+    assert ra.sync() == L.LS_OK and rb.sync() == L.LS_OK
+    ra.close(); rb.close()
+
+
+def test_trace_counts_and_times_launches():
+    wl, dw, r = staged("tiny")
+    L.check(L.ls_trace_enable(r.h, True))
+    L.ls_trace_read(r.h)
+    for _ in range(3):
+        r.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)
+    rc, tr = L.ls_trace_read(r.h)
+    L.check(L.ls_trace_enable(r.h, False))
+    assert rc == L.LS_OK and tr
+    for name, (launches, ms, timed) in tr.items():
+        assert launches == timed == 3, (name, launches, timed)
+        assert ms > 0.0
