@@ -108,7 +108,7 @@ void free_all(Ctx& c) {
                   c.adam_v, c.pub[0].params, c.pub[0].wt, c.pub[1].params, c.pub[1].wt,
                   c.ring_x, c.ring_y, c.hits, c.scores, c.tx, c.tz, c.ty, c.dz0, c.dz1, c.grad,
                   c.gpart, c.loss_tmp, c.d_err, c.pub[0].img, c.pub[1].img, c.xin, c.xrq,
-                  c.bkeys, c.work, c.work_n, c.gkeys, c.gmask, c.st};
+                  c.bkeys, c.work, c.work_n, c.gkeys, c.gmask, c.st, c.tf.base, c.tf.parts};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   if (c.ev_pub) cudaEventDestroy(c.ev_pub);
@@ -231,6 +231,14 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
   A(dalloc(&c.loss_tmp, 1));
   A(dalloc(&c.d_err, 1));
   A(dalloc(&c.st, 1));
+  int64_t tf_bytes = 0;
+  if (plan_train_fast(m, cfg->max_train_batch, c.tf)) {
+    int64_t pf = 0;
+    tf_bytes = train_fast_bytes(m, c.tf, &pf);
+    A(dalloc(&c.tf.base, tf_bytes));
+    A(dalloc(&c.tf.parts, pf));
+    if (e == cudaSuccess) train_fast_bind(m, c.tf, c.tf.base, c.tf.parts);
+  }
   if (e == cudaSuccess) {
     A(cudaEventCreateWithFlags(&c.ev_pub, cudaEventDisableTiming));
     A(cudaEventCreateWithFlags(&c.ev_route, cudaEventDisableTiming));
@@ -243,6 +251,7 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
     A(cudaMemset(c.adam_m, 0, (size_t)c.n_params * sizeof(float)));
     A(cudaMemset(c.adam_v, 0, (size_t)c.n_params * sizeof(float)));
     A(cudaMemset(c.d_err, 0, sizeof(int)));
+    if (c.tf.base) A(cudaMemset(c.tf.base, 0, (size_t)tf_bytes));
     DevState init{};
     init.cur = -1;
     init.route_b = 0;
@@ -303,6 +312,7 @@ int ls_set_params(ls_ctx* h, const float* params, void* stream) {
   LS_CK(cudaMemsetAsync(c.adam_m, 0, n, S(stream)));
   LS_CK(cudaMemsetAsync(c.adam_v, 0, n, S(stream)));
   LS_CK(cudaMemsetAsync(&c.st->step, 0, sizeof(int64_t), S(stream)));
+  if (c.tf.on) LS_CK(train_fast_images(c, S(stream)));
   c.have_params = true;
   return LS_OK;
 }
@@ -509,7 +519,8 @@ int ls_train_step(ls_ctx* h, int32_t batch, const int32_t* idx, int32_t opt, flo
   if (!c.have_params) return fail(LS_ERR_STATE, "parameters not set");
   if (!c.have_norm) return fail(LS_ERR_STATE, "normaliser not set");
   if (c.ring_enqueued < 1) return fail(LS_ERR_STATE, "sample ring is empty");
-  LS_CK(run_train_step(c, batch, idx, opt, lr, loss_out, S(stream)));
+  LS_CK(c.tf.on ? run_train_fast(c, batch, idx, opt, lr, loss_out, S(stream))
+                : run_train_step(c, batch, idx, opt, lr, loss_out, S(stream)));
   return LS_OK;
 }
 

@@ -120,6 +120,30 @@ struct Tracer {
   }
 };
 
+// Buffers of the tensor-core training step (k_train_fast.cu): bf16 operand
+// images of activations, gradients and weights, ReLU mask bits, and the
+// fp32 partials the optimiser sums.
+struct TrainFast {
+  bool on = false;
+  int rows_max = 0;                        // max_train_batch rounded up to 128
+  int in_pad[LS_MAX_LAYERS] = {};          // K of layer l (input width padded to 64)
+  uint8_t* imgA[LS_MAX_LAYERS] = {};       // A_l  [rows, in_pad[l]]
+  uint8_t* imgAT[LS_MAX_LAYERS] = {};      // A_l^T [in_pad[l], rows]
+  uint8_t* imgDZ[2] = {};                  // dz of a hidden layer [rows, width], by layer parity
+  uint8_t* imgDZT[2] = {};                 // its transpose [width padded to 128, rows]
+  uint32_t* mask[LS_MAX_LAYERS + 1] = {};  // bits of [A_l > 0] as [width/32][rows]
+  uint8_t* imgW[LS_MAX_LAYERS] = {};       // bf16 W_l  [out, in_pad]
+  uint8_t* imgWT[LS_MAX_LAYERS] = {};      // bf16 W_l^T [in_pad, out]
+  float* partW[LS_MAX_LAYERS] = {};        // dW split partials [splits][out][in_pad]
+  float* partB[LS_MAX_LAYERS] = {};        // db tile partials [tiles][out]
+  float* partWL = nullptr;                 // output-layer dW tile partials [tiles][in]
+  float* partBL = nullptr;                 // output-layer db tile partials [tiles]
+  float* partLoss = nullptr;               // squared-error tile partials [tiles]
+  int splits[LS_MAX_LAYERS] = {};
+  uint8_t* base = nullptr;                 // allocations
+  float* parts = nullptr;
+};
+
 struct Ctx {
   ls_config cfg{};
   MlpDesc mlp{};
@@ -187,6 +211,7 @@ struct Ctx {
   float* gpart = nullptr;     // split-K partials (also column-sum partials)
   int64_t gpart_floats = 0;
   float* loss_tmp = nullptr;  // [1]
+  TrainFast tf;               // tensor-core training buffers (when tf.on)
 
   int* d_err = nullptr;       // first device-side error (0 = none)
   int sms = 148;              // SM count of the context's device
@@ -322,6 +347,12 @@ cudaError_t launch_gemm_tc(int M, int N, int K, const float* A, int64_t sam, int
                            const float* zprev, int64_t ld_zprev, int* err, int sms, cudaStream_t s);
 int gemm_tc_splits_used(int K, int splits);
 int index_words(int max_instances);
+bool plan_train_fast(const MlpDesc& m, int max_batch, TrainFast& f);
+int64_t train_fast_bytes(const MlpDesc& m, const TrainFast& f, int64_t* parts_floats);
+void train_fast_bind(const MlpDesc& m, TrainFast& f, uint8_t* base, float* parts);
+cudaError_t train_fast_images(Ctx& c, cudaStream_t s);
+cudaError_t run_train_fast(Ctx& c, int batch, const int32_t* idx, int opt, float lr, float* loss_out,
+                           cudaStream_t s);
 void set_last_error(const char* msg);  // sets the text ls_last_error() returns
 cudaError_t launch_prefix_index(int n_req, const int32_t* tok, const int64_t* tok_off, const uint64_t* gkeys,
                                 const uint64_t* gmask, int W, uint64_t gmask_slots, int n_inst, int32_t* hits,

@@ -154,14 +154,26 @@ __global__ void k_ring_append(int n, int d, const float* __restrict__ x, const f
                               int64_t capacity) {
   const int64_t count = *reinterpret_cast<volatile int64_t*>(&st->ring_count);
   const int64_t first = n > capacity ? n - capacity : 0;
-  const int64_t total = (int64_t)(n - first) * (d + 1);
+  // piece = 4 consecutive columns of one record (the last piece of a record
+  // may be short); pieces of a record share its slot
+  const int per = (d + 3) / 4;
+  const int64_t total = (int64_t)(n - first) * per;
+  const bool vec = (d & 3) == 0 && (reinterpret_cast<uintptr_t>(x) & 15) == 0 &&
+                   (reinterpret_cast<uintptr_t>(ring_x) & 15) == 0;
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
        e += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t j = first + e / (d + 1);
-    const int k = (int)(e % (d + 1));
+    const int64_t jj = e / per;
+    const int k = (int)(e - jj * per) * 4;
+    const int64_t j = first + jj;
     const int64_t slot = (count + j) % capacity;
-    if (k < d) ring_x[slot * d + k] = x[j * d + k];
-    else ring_y[slot] = y[j];
+    const float* src = x + j * d + k;
+    float* dst = ring_x + slot * d + k;
+    if (vec) {
+      *reinterpret_cast<float4*>(dst) = __ldg(reinterpret_cast<const float4*>(src));
+    } else {
+      for (int u = 0; u < 4 && k + u < d; ++u) dst[u] = __ldg(src + u);
+    }
+    if (k == 0) ring_y[slot] = y[j];
   }
   if (last_block(&st->done[DONE_RING]) && threadIdx.x == 0) st->ring_count = count + n;
 }
@@ -224,7 +236,7 @@ cudaError_t launch_ring_append(int n, int d, const float* x, const float* y, flo
                                float* ring_y, DevState* st, int64_t capacity, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
   const int64_t keep = n > capacity ? capacity : n;
-  const int64_t total = keep * (d + 1);
+  const int64_t total = keep * ((d + 3) / 4);
   k_ring_append<<<grid_1d(total, 256), 256, 0, s>>>(n, d, x, y, ring_x, ring_y, st, capacity);
   return cudaGetLastError();
 }
