@@ -131,7 +131,7 @@ struct TrainFast {
   uint8_t* imgAT[LS_MAX_LAYERS] = {};      // A_l^T [in_pad[l], rows]
   uint8_t* imgDZ[2] = {};                  // dz of a hidden layer [rows, width], by layer parity
   uint8_t* imgDZT[2] = {};                 // its transpose [width padded to 128, rows]
-  uint32_t* mask[LS_MAX_LAYERS + 1] = {};  // bits of [A_l > 0] as [width/32][rows]
+  uint16_t* mask[LS_MAX_LAYERS + 1] = {};  // bits of [A_l > 0] as [width/16][rows]
   uint8_t* imgW[LS_MAX_LAYERS] = {};       // bf16 W_l  [out, in_pad]
   uint8_t* imgWT[LS_MAX_LAYERS] = {};      // bf16 W_l^T [in_pad, out]
   float* partW[LS_MAX_LAYERS] = {};        // dW split partials [splits][out][in_pad]

@@ -32,18 +32,22 @@ using namespace sm100;
 
 namespace {
 
-constexpr int kT = 256;        // threads: 8 warps, 2 per TMEM lane quadrant
+constexpr int kT = 512;        // 16 warps: TMEM lane quadrant = warp % 4, column quarter = warp / 4
 constexpr int kM = 128;        // rows per tile
 constexpr int kMaxChunks = 4;  // K-blocks of 64 per CTA (all resident)
 
 enum { TE_STORE = 0, TE_FWD = 1, TE_FWD_OUT = 2, TE_DX = 3 };
 
+// One product D = A B^T over a K range, tiled as 128-row tiles x n_split
+// column parts x splits of K; CTA li -> (column part li % n_split, row tile,
+// split), so the column parts of a tile are adjacent (a cluster for TE_FWD_OUT).
 struct TrJob {
   int epi;
-  int m_tiles, splits, nchunks, NT;  // CTA (m_tile, split) computes rows m_tile*128.., K-blocks split*nchunks..
+  int m_tiles, n_split, splits, nchunks;
+  int NT;                            // columns per CTA; the product's N = NT * n_split
   const uint8_t* A;                  // image, rA rows
   int rA;
-  const uint8_t* B;                  // image, NT rows
+  const uint8_t* B;                  // image, N rows
   int M;                             // valid rows of D
   // TE_STORE: fp32 partial D to C[split][row][col]
   float* C;
@@ -52,18 +56,18 @@ struct TrJob {
   // TE_FWD / TE_FWD_OUT / TE_DX
   const float* bias;                 // layer bias (TE_FWD, TE_FWD_OUT)
   uint8_t* out;                      // row-major image of the result, rows = rows_pad (nullable)
-  uint8_t* outT;                     // transposed image, rows = rT (nullable)
+  uint8_t* outT;                     // transposed image, rows = rT
   int rT;
-  uint32_t* mask_out;                // TE_FWD: [NT/32][rows_pad] bits of [Z > 0]
-  const uint32_t* mask_in;           // TE_FWD_OUT keeps its own; TE_DX: bits of the previous layer
-  float* colpart;                    // [m_tiles][NT] column sums of dz (TE_FWD_OUT, TE_DX)
+  uint16_t* mask_out;                // TE_FWD: bits of [Z > 0] as [N/16][rows_pad]
+  const uint16_t* mask_in;           // TE_DX: bits of the layer input's ReLU
+  float* colpart;                    // [m_tiles][N] column sums of dz (TE_FWD_OUT, TE_DX)
   int rows_pad;                      // padded batch (multiple of 128)
   // TE_FWD_OUT: width-1 output layer
-  const float* wL;                   // [NT] fp32 master weights of the output layer
+  const float* wL;                   // [N] fp32 master weights of the output layer
   const float* bL;                   // [1]
   const float* y;                    // [batch] targets
   int batch;
-  float* partWL;                     // [m_tiles][NT]
+  float* partWL;                     // [m_tiles][N]
   float* partBL;                     // [m_tiles]
   float* partLoss;                   // [m_tiles]
 };
@@ -84,12 +88,12 @@ __device__ __forceinline__ uint32_t pack2(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
-// Sum over the warp's 32 lanes of each of 32 per-lane values: afterwards lane
-// u holds the sum for column u.  Fixed order (butterfly), 31 shuffles.
-__device__ __forceinline__ float col_reduce32(float (&v)[32]) {
+// Sum over the warp's 32 lanes of each of 16 per-lane values: afterwards
+// lanes u and u + 16 hold the sum for column u.  Fixed order (butterfly).
+__device__ __forceinline__ float col_reduce16(float (&v)[16]) {
   const int lane = threadIdx.x & 31;
 #pragma unroll
-  for (int s = 16; s >= 1; s >>= 1) {
+  for (int s = 8; s >= 1; s >>= 1) {
     const bool up = (lane & s) != 0;
 #pragma unroll
     for (int i = 0; i < s; ++i) {
@@ -98,28 +102,28 @@ __device__ __forceinline__ float col_reduce32(float (&v)[32]) {
       v[i] = keep + __shfl_xor_sync(0xffffffffu, send, s);
     }
   }
-  return v[0];
+  return v[0] + __shfl_xor_sync(0xffffffffu, v[0], 16);
 }
 
-// Row-major image: 32 bf16 values of row j, columns c0..c0+31 (c0 % 32 == 0).
-__device__ __forceinline__ void store_row32(uint8_t* img, int rows, int j, int c0, const float (&v)[32]) {
+// Row-major image: 16 bf16 values of row j, columns c..c+15 (c % 16 == 0).
+__device__ __forceinline__ void store_row16(uint8_t* img, int rows, int j, int c, const float (&v)[16]) {
 #pragma unroll
-  for (int g = 0; g < 4; ++g) {
+  for (int g = 0; g < 2; ++g) {
     uint4 q;
     q.x = pack2(v[8 * g], v[8 * g + 1]);
     q.y = pack2(v[8 * g + 2], v[8 * g + 3]);
     q.z = pack2(v[8 * g + 4], v[8 * g + 5]);
     q.w = pack2(v[8 * g + 6], v[8 * g + 7]);
-    *reinterpret_cast<uint4*>(img + sw128_offset(j, c0 + 8 * g, rows)) = q;
+    *reinterpret_cast<uint4*>(img + sw128_offset(j, c + 8 * g, rows)) = q;
   }
 }
 
-// Transposed image: element (c0 + u, j) for u < 32; lanes hold consecutive j,
+// Transposed image: element (c + u, j) for u < 16; lanes hold consecutive j,
 // so each column is written as 2-byte pieces of one 64-byte run per warp.
-__device__ __forceinline__ void store_col32(uint8_t* imgT, int rowsT, int j, int c0, const float (&v)[32]) {
+__device__ __forceinline__ void store_col16(uint8_t* imgT, int rowsT, int j, int c, const float (&v)[16]) {
 #pragma unroll
-  for (int u = 0; u < 32; ++u)
-    *reinterpret_cast<uint16_t*>(imgT + sw128_offset(c0 + u, j, rowsT)) = bf16_bits(v[u]);
+  for (int u = 0; u < 16; ++u)
+    *reinterpret_cast<uint16_t*>(imgT + sw128_offset(c + u, j, rowsT)) = bf16_bits(v[u]);
 }
 
 __global__ void __launch_bounds__(kT, 1) k_tr_gemm(const __grid_constant__ TrArgs args) {
@@ -128,17 +132,24 @@ __global__ void __launch_bounds__(kT, 1) k_tr_gemm(const __grid_constant__ TrArg
   const bool second = (int)blockIdx.x >= args.n_cta0;
   const TrJob& J = args.job[second ? 1 : 0];
   const int li = second ? (int)blockIdx.x - args.n_cta0 : (int)blockIdx.x;
-  const int mt = li % J.m_tiles, split = li / J.m_tiles;
+  const int ns = li % J.n_split, rest = li / J.n_split;
+  const int mt = rest % J.m_tiles, split = rest / J.m_tiles;
   const int m0 = mt * kM;
-  const int NT = J.NT, nch = J.nchunks;
+  const int NT = J.NT, N = NT * J.n_split, n0 = ns * NT, nch = J.nchunks;
   const uint32_t a_bytes = kM * 128, b_bytes = (uint32_t)NT * 128;
   const uint32_t stage_bytes = a_bytes + b_bytes;
   uint8_t* tail = smem + (size_t)kMaxChunks * (kM * 128 + 256 * 128);
   uint64_t* full = reinterpret_cast<uint64_t*>(tail);           // [kMaxChunks]
   uint64_t* done = full + kMaxChunks;
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(done + 1);
-  float* red = reinterpret_cast<float*>(tail + 128);            // [2][4][256]
-  float* xch = red + 2 * 4 * 256;                               // [2][128] row exchange
+  float* s_bias = reinterpret_cast<float*>(tail + 128);         // [256]
+  float* s_w = s_bias + 256;                                    // [256] bf16-rounded output weights
+  float* red = s_w + 256;                                       // [4][256] column sums by lane quadrant
+  float* red2 = red + 4 * 256;                                  // [4][256]
+  float* rowq = red2 + 4 * 256;                                 // [4][128] row dots by column quarter
+  float* rowdot = rowq + 4 * 128;                               // [128] this CTA's row dots
+  float* yrow = rowdot + 128;                                   // [128] predictions
+  float* wsum = yrow + 128;                                     // [8] warp partials
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   uint32_t tcols = 32;
@@ -163,7 +174,7 @@ __global__ void __launch_bounds__(kT, 1) k_tr_gemm(const __grid_constant__ TrArg
       uint8_t* sa = smem + (size_t)c * stage_bytes;
       mbar_arrive_expect_tx(&full[c], stage_bytes);
       bulk_g2s(sa, J.A + (size_t)kb * J.rA * 128 + (size_t)m0 * 128, a_bytes, &full[c]);
-      bulk_g2s(sa + a_bytes, J.B + (size_t)kb * NT * 128, b_bytes, &full[c]);
+      bulk_g2s(sa + a_bytes, J.B + (size_t)kb * N * 128 + (size_t)n0 * 128, b_bytes, &full[c]);
     }
     const uint32_t idesc = idesc_bf16_f32(kM, NT);
     for (int c = 0; c < nch; ++c) {
@@ -175,6 +186,11 @@ __global__ void __launch_bounds__(kT, 1) k_tr_gemm(const __grid_constant__ TrArg
         umma_bf16(tmem, sdesc_sw128(sa + 32u * k), sdesc_sw128(sb + 32u * k), idesc, (c | k) ? 1u : 0u);
     }
     umma_commit(done);  // arrives once everything issued so far has completed
+  }
+  // side inputs of the epilogue, staged while the copies and MMAs run
+  for (int t = tid; t < NT; t += kT) {
+    if (J.bias) s_bias[t] = __ldg(J.bias + n0 + t);
+    if (J.epi == TE_FWD_OUT) s_w[t] = round_bf16(__ldg(J.wL + n0 + t));
   }
   __syncwarp();
   if (!mbar_wait(done, 0)) ok = false;
@@ -188,129 +204,142 @@ __global__ void __launch_bounds__(kT, 1) k_tr_gemm(const __grid_constant__ TrArg
   }
   tc_fence_after();
 
-  const int q = warp & 3, h = warp >> 2;
+  const int q = warp & 3, cq = warp >> 2;
   const int r = 32 * q + lane, j = m0 + r;
-  const int half = NT / 2;
+  const int cw = NT / 4, cbeg = cq * cw;  // this warp's columns (CTA-local)
   const uint32_t lane_addr = (uint32_t)(32 * q) << 16;
-  float* redA = red;              // [4][256]
-  float* redB = red + 4 * 256;    // [4][256]
 
   if (ok && J.epi == TE_STORE) {
     if (j < J.M) {
-      float* crow = J.C + (int64_t)split * J.split_stride + (int64_t)j * J.ldc;
-      for (int c0 = h * half; c0 < (h + 1) * half; c0 += 32) {
-        uint32_t v[32];
-        tmem_ld32(tmem + lane_addr + (uint32_t)c0, v);
+      float* crow = J.C + (int64_t)split * J.split_stride + (int64_t)j * J.ldc + n0;
+      for (int c = cbeg; c < cbeg + cw; c += 16) {
+        uint32_t v[16];
+        tmem_ld16x(tmem + lane_addr + (uint32_t)c, v);
         tmem_wait_ld();
 #pragma unroll
-        for (int g = 0; g < 8; ++g)
-          reinterpret_cast<float4*>(crow + c0)[g] =
+        for (int g = 0; g < 4; ++g)
+          reinterpret_cast<float4*>(crow + c)[g] =
               make_float4(__uint_as_float(v[4 * g]), __uint_as_float(v[4 * g + 1]), __uint_as_float(v[4 * g + 2]),
                           __uint_as_float(v[4 * g + 3]));
       }
     }
   } else if (ok && J.epi == TE_FWD) {
-    for (int c0 = h * half; c0 < (h + 1) * half; c0 += 32) {
-      uint32_t v[32];
-      tmem_ld32(tmem + lane_addr + (uint32_t)c0, v);
+    for (int c = cbeg; c < cbeg + cw; c += 16) {
+      uint32_t v[16];
+      tmem_ld16x(tmem + lane_addr + (uint32_t)c, v);
       tmem_wait_ld();
-      float a[32];
+      float a[16];
       uint32_t bits = 0;
 #pragma unroll
-      for (int u = 0; u < 32; ++u) {
-        const float z = __uint_as_float(v[u]) + __ldg(J.bias + c0 + u);
+      for (int u = 0; u < 16; ++u) {
+        const float z = __uint_as_float(v[u]) + s_bias[c + u];
         bits |= (z > 0.0f ? 1u : 0u) << u;
         a[u] = round_bf16(z > 0.0f ? z : 0.0f);
       }
-      J.mask_out[(int64_t)(c0 >> 5) * J.rows_pad + j] = bits;
-      store_row32(J.out, J.rows_pad, j, c0, a);
-      store_col32(J.outT, J.rT, j, c0, a);
-    }
-  } else if (ok && J.epi == TE_FWD_OUT) {
-    // pass 1: activations, mask bits, this half's part of the output dot product
-    uint32_t mbits[4];
-    float dot = 0.0f;
-    int w = 0;
-    for (int c0 = h * half; c0 < (h + 1) * half; c0 += 32, ++w) {
-      uint32_t v[32];
-      tmem_ld32(tmem + lane_addr + (uint32_t)c0, v);
-      tmem_wait_ld();
-      uint32_t bits = 0;
-#pragma unroll
-      for (int u = 0; u < 32; ++u) {
-        const float z = __uint_as_float(v[u]) + __ldg(J.bias + c0 + u);
-        bits |= (z > 0.0f ? 1u : 0u) << u;
-        const float a = round_bf16(z > 0.0f ? z : 0.0f);
-        dot = fmaf(a, round_bf16(__ldg(J.wL + c0 + u)), dot);
-      }
-      mbits[w] = bits;
-    }
-    xch[h * kM + r] = dot;
-    __syncthreads();
-    const float yhat = (xch[r] + xch[kM + r]) + __ldg(J.bL);
-    const bool valid = j < J.batch;
-    const float e = valid ? yhat - __ldg(J.y + j) : 0.0f;
-    const float dzL = valid ? 2.0f * e / (float)J.batch : 0.0f;
-    const float rd = round_bf16(dzL);
-    // loss and db_L partials: warp sums, then quadrants in order (half 0 only)
-    float e2 = e * e, dsum = dzL;
-#pragma unroll
-    for (int o = 16; o; o >>= 1) {
-      e2 += __shfl_xor_sync(0xffffffffu, e2, o);
-      dsum += __shfl_xor_sync(0xffffffffu, dsum, o);
-    }
-    __syncthreads();  // xch reused below
-    if (h == 0 && lane == 0) {
-      xch[q] = e2;
-      xch[4 + q] = dsum;
-    }
-    // pass 2: dW_L partial (sum_j bf16(dz_L[j]) a[j, c]) and dz_l = bf16(dz_L) bf16(w_L) [Z > 0]
-    w = 0;
-    for (int c0 = h * half; c0 < (h + 1) * half; c0 += 32, ++w) {
-      uint32_t v[32];
-      tmem_ld32(tmem + lane_addr + (uint32_t)c0, v);
-      tmem_wait_ld();
-      float pw[32], dz[32];
-#pragma unroll
-      for (int u = 0; u < 32; ++u) {
-        const float z = __uint_as_float(v[u]) + __ldg(J.bias + c0 + u);
-        const float a = round_bf16(z > 0.0f ? z : 0.0f);
-        pw[u] = rd * a;
-        dz[u] = ((mbits[w] >> u) & 1u) ? rd * round_bf16(__ldg(J.wL + c0 + u)) : 0.0f;
-      }
-      if (J.out) store_row32(J.out, J.rows_pad, j, c0, dz);
-      store_col32(J.outT, J.rT, j, c0, dz);
-      const float sw = col_reduce32(pw);
-      redA[q * 256 + c0 + lane] = sw;
-      const float sb = col_reduce32(dz);
-      redB[q * 256 + c0 + lane] = sb;
-    }
-    __syncthreads();
-    for (int c = tid; c < NT; c += kT) {
-      J.partWL[(int64_t)mt * NT + c] = ((redA[c] + redA[256 + c]) + redA[512 + c]) + redA[768 + c];
-      J.colpart[(int64_t)mt * NT + c] = ((redB[c] + redB[256 + c]) + redB[512 + c]) + redB[768 + c];
-    }
-    if (tid == 0) {
-      J.partLoss[mt] = ((xch[0] + xch[1]) + xch[2]) + xch[3];
-      J.partBL[mt] = ((xch[4] + xch[5]) + xch[6]) + xch[7];
+      J.mask_out[(int64_t)((n0 + c) >> 4) * J.rows_pad + j] = (uint16_t)bits;
+      store_row16(J.out, J.rows_pad, j, n0 + c, a);
+      store_col16(J.outT, J.rT, j, n0 + c, a);
     }
   } else if (ok && J.epi == TE_DX) {
-    for (int c0 = h * half; c0 < (h + 1) * half; c0 += 32) {
-      uint32_t v[32];
-      tmem_ld32(tmem + lane_addr + (uint32_t)c0, v);
+    for (int c = cbeg; c < cbeg + cw; c += 16) {
+      uint32_t v[16];
+      tmem_ld16x(tmem + lane_addr + (uint32_t)c, v);
       tmem_wait_ld();
-      const uint32_t bits = J.mask_in[(int64_t)(c0 >> 5) * J.rows_pad + j];
-      float dz[32];
+      const uint32_t bits = J.mask_in[(int64_t)((n0 + c) >> 4) * J.rows_pad + j];
+      float dz[16];
 #pragma unroll
-      for (int u = 0; u < 32; ++u) dz[u] = ((bits >> u) & 1u) ? __uint_as_float(v[u]) : 0.0f;
-      if (J.out) store_row32(J.out, J.rows_pad, j, c0, dz);
-      store_col32(J.outT, J.rT, j, c0, dz);
-      const float sb = col_reduce32(dz);
-      redB[q * 256 + c0 + lane] = sb;
+      for (int u = 0; u < 16; ++u) dz[u] = ((bits >> u) & 1u) ? __uint_as_float(v[u]) : 0.0f;
+      if (J.out) store_row16(J.out, J.rows_pad, j, n0 + c, dz);
+      store_col16(J.outT, J.rT, j, n0 + c, dz);
+      const float sb = col_reduce16(dz);
+      if (lane < 16) red[q * 256 + c + lane] = sb;
     }
     __syncthreads();
     for (int c = tid; c < NT; c += kT)
-      J.colpart[(int64_t)mt * NT + c] = ((redB[c] + redB[256 + c]) + redB[512 + c]) + redB[768 + c];
+      J.colpart[(int64_t)mt * N + n0 + c] = ((red[c] + red[256 + c]) + red[512 + c]) + red[768 + c];
+  }
+  if (J.epi == TE_FWD_OUT) {
+    // pass 1: activations and this warp's part of the output dot product
+    if (ok) {
+      float dot = 0.0f;
+      for (int c = cbeg; c < cbeg + cw; c += 16) {
+        uint32_t v[16];
+        tmem_ld16x(tmem + lane_addr + (uint32_t)c, v);
+        tmem_wait_ld();
+#pragma unroll
+        for (int u = 0; u < 16; ++u) {
+          const float z = __uint_as_float(v[u]) + s_bias[c + u];
+          dot = fmaf(round_bf16(z > 0.0f ? z : 0.0f), s_w[c + u], dot);
+        }
+      }
+      rowq[cq * 128 + r] = dot;
+    }
+    __syncthreads();
+    if (ok && tid < kM) rowdot[tid] = ((rowq[tid] + rowq[128 + tid]) + rowq[256 + tid]) + rowq[384 + tid];
+    if (J.n_split > 1) cluster_sync();
+    else __syncthreads();
+    if (ok && tid < kM) {
+      float tot = rowdot[tid];
+      if (J.n_split > 1) {
+        const uint32_t me = cluster_ctarank();
+        const float other = ld_dsmem_f32(rowdot + tid, me ^ 1u);
+        tot = me == 0 ? tot + other : other + tot;  // rank 0's part first on both
+      }
+      yrow[tid] = tot + __ldg(J.bL);
+    }
+    if (J.n_split > 1) cluster_sync();  // the partner has read this CTA's rowdot
+    else __syncthreads();
+    if (ok) {
+      const bool valid = j < J.batch;
+      const float yhat = yrow[r];
+      const float e = valid ? yhat - __ldg(J.y + j) : 0.0f;
+      const float dzL = valid ? 2.0f * e / (float)J.batch : 0.0f;
+      const float rd = round_bf16(dzL);
+      if (ns == 0 && cq == 0) {
+        float e2 = e * e, dsum = dzL;
+#pragma unroll
+        for (int o = 16; o; o >>= 1) {
+          e2 += __shfl_xor_sync(0xffffffffu, e2, o);
+          dsum += __shfl_xor_sync(0xffffffffu, dsum, o);
+        }
+        if (lane == 0) {
+          wsum[q] = e2;
+          wsum[4 + q] = dsum;
+        }
+      }
+      // pass 2 (Z re-read from TMEM, so [Z > 0] is the same test as in pass 1):
+      // dW_L partial (sum_j bf16(dz_L[j]) a[j, c]) and dz = bf16(dz_L) bf16(w_L) [Z > 0]
+      for (int c = cbeg; c < cbeg + cw; c += 16) {
+        uint32_t v[16];
+        tmem_ld16x(tmem + lane_addr + (uint32_t)c, v);
+        tmem_wait_ld();
+        float pw[16], dz[16];
+#pragma unroll
+        for (int u = 0; u < 16; ++u) {
+          const float z = __uint_as_float(v[u]) + s_bias[c + u];
+          const bool pos = z > 0.0f;
+          pw[u] = rd * round_bf16(pos ? z : 0.0f);
+          dz[u] = pos ? rd * s_w[c + u] : 0.0f;
+        }
+        if (J.out) store_row16(J.out, J.rows_pad, j, n0 + c, dz);
+        store_col16(J.outT, J.rT, j, n0 + c, dz);
+        const float sw = col_reduce16(pw);
+        if (lane < 16) red2[q * 256 + c + lane] = sw;
+        const float sb = col_reduce16(dz);
+        if (lane < 16) red[q * 256 + c + lane] = sb;
+      }
+    }
+    __syncthreads();
+    if (ok) {
+      for (int c = tid; c < NT; c += kT) {
+        J.partWL[(int64_t)mt * N + n0 + c] = ((red2[c] + red2[256 + c]) + red2[512 + c]) + red2[768 + c];
+        J.colpart[(int64_t)mt * N + n0 + c] = ((red[c] + red[256 + c]) + red[512 + c]) + red[768 + c];
+      }
+      if (ns == 0 && tid == 0) {
+        J.partLoss[mt] = ((wsum[0] + wsum[1]) + wsum[2]) + wsum[3];
+        J.partBL[mt] = ((wsum[4] + wsum[5]) + wsum[6]) + wsum[7];
+      }
+    }
   }
   tc_fence_before();
   __syncthreads();
@@ -478,24 +507,44 @@ __global__ void __launch_bounds__(256) k_tr_opt(const __grid_constant__ OptArgs 
   if (a.mode != 0 && last_block(&a.st->done[DONE_OPT]) && threadIdx.x == 0) a.st->step = t;
 }
 
-int gemm_smem_bytes() { return 1024 + kMaxChunks * (kM * 128 + 256 * 128) + 128 + (2 * 4 * 256 + 2 * kM) * 4; }
+int gemm_smem_bytes() {
+  return 1024 + kMaxChunks * (kM * 128 + 256 * 128) + 128 + (256 + 256 + 8 * 256 + 4 * 128 + 128 + 128 + 8) * 4;
+}
 
 cudaError_t launch_tr_gemm(const TrJob& j0, const TrJob* j1, int* err, cudaStream_t s) {
   TrArgs a{};
   a.job[0] = j0;
-  a.n_cta0 = j0.m_tiles * j0.splits;
+  a.n_cta0 = j0.m_tiles * j0.n_split * j0.splits;
   int n = a.n_cta0;
   if (j1) {
     a.job[1] = *j1;
-    n += j1->m_tiles * j1->splits;
+    n += j1->m_tiles * j1->n_split * j1->splits;
   }
   a.err = err;
   const int smem = gemm_smem_bytes();
   cudaError_t e = cudaFuncSetAttribute(k_tr_gemm, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  k_tr_gemm<<<n, kT, smem, s>>>(a);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(n);
+  cfg.blockDim = dim3(kT);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  // the column parts of a TE_FWD_OUT tile exchange row sums through
+  // distributed shared memory: one cluster per tile
+  const int cl = (j0.epi == TE_FWD_OUT && !j1) ? j0.n_split : 1;
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = cl;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, k_tr_gemm, a);
 }
+
+// Column parts per tile: two when the columns split into halves that are
+// multiples of 64 (each warp then owns a multiple of 16 columns).
+int n_split_for(int N) { return N % 128 == 0 ? 2 : 1; }
 
 }  // namespace
 
@@ -556,7 +605,7 @@ void train_fast_bind(const MlpDesc& m, TrainFast& f, uint8_t* base, float* parts
     p += hpad * R * 2;
   }
   for (int l = 1; l <= nh; ++l) {
-    f.mask[l] = reinterpret_cast<uint32_t*>(p);
+    f.mask[l] = reinterpret_cast<uint16_t*>(p);
     p += (int64_t)(m.w[l] / 32) * R * 4;
   }
   for (int l = 0; l < nh; ++l) {
@@ -621,9 +670,10 @@ cudaError_t run_train_fast(Ctx& c, int B, const int32_t* idx, int opt, float lr,
     TrJob J{};
     J.epi = last ? TE_FWD_OUT : TE_FWD;
     J.m_tiles = T;
+    J.n_split = n_split_for(m.w[l + 1]);
     J.splits = 1;
     J.nchunks = f.in_pad[l] / 64;
-    J.NT = m.w[l + 1];
+    J.NT = m.w[l + 1] / J.n_split;
     J.A = f.imgA[l];
     J.rA = R;
     J.B = f.imgW[l];
@@ -652,15 +702,18 @@ cudaError_t run_train_fast(Ctx& c, int B, const int32_t* idx, int opt, float lr,
     if (e != cudaSuccess) return e;
   }
   // backward: dW_l (split over the batch) and, for l > 0, dz_{l-1} in the same launch
-  const int kpc = 2;  // K-blocks (of 64 rows) per dW CTA
   for (int l = nh - 1; l >= 0; --l) {
     const int out = m.w[l + 1];
     TrJob W{};
     W.epi = TE_STORE;
     W.m_tiles = (out + kM - 1) / kM;
+    W.n_split = n_split_for(f.in_pad[l]);
+    // K-blocks (of 64 batch rows) per CTA: 4 when that still gives 48 CTAs,
+    // else 2 (more CTAs, more partials for the optimiser to add)
+    const int kpc = W.m_tiles * W.n_split * (R / 256) >= 48 ? 4 : 2;
     W.nchunks = std::min(kpc, R / 64);
     W.splits = (R / 64) / W.nchunks;
-    W.NT = f.in_pad[l];
+    W.NT = f.in_pad[l] / W.n_split;
     W.A = f.imgDZT[l & 1];
     W.rA = ((out + 127) / 128) * 128;
     W.B = f.imgAT[l];
@@ -673,9 +726,10 @@ cudaError_t run_train_fast(Ctx& c, int B, const int32_t* idx, int opt, float lr,
     if (l > 0) {
       X.epi = TE_DX;
       X.m_tiles = T;
+      X.n_split = n_split_for(m.w[l]);
       X.splits = 1;
       X.nchunks = out / 64;
-      X.NT = m.w[l];
+      X.NT = m.w[l] / X.n_split;
       X.A = f.imgDZ[l & 1];
       X.rA = R;
       X.B = f.imgWT[l];
