@@ -107,7 +107,7 @@ void free_all(Ctx& c) {
   void* ptrs[] = {c.tables, c.table_count, c.inst_state, c.mean, c.stdv, c.master, c.adam_m,
                   c.adam_v, c.pub[0].params, c.pub[0].wt, c.pub[1].params, c.pub[1].wt,
                   c.ring_x, c.ring_y, c.hits, c.scores, c.tx, c.tz, c.ty, c.dz0, c.dz1, c.grad,
-                  c.gpart, c.loss_tmp, c.d_err, c.pub[0].img, c.pub[1].img, c.xin, c.xrq,
+                  c.gpart, c.loss_tmp, c.d_err, c.pub[0].img, c.pub[1].img, c.xin, c.xrq, c.pairx,
                   c.bkeys, c.work, c.work_n, c.gkeys, c.gmask, c.st, c.tf.base, c.tf.parts};
   for (void* p : ptrs)
     if (p) cudaFree(p);
@@ -216,6 +216,7 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
   A(dalloc(&c.work_n, 1));
   A(dalloc(&c.xin, NI * std::max(1, c.tc.d_pad)));
   A(dalloc(&c.xrq, R * std::max(1, c.tc.d_pad)));
+  if (c.use_tc) A(dalloc(&c.pairx, R * NI));
   A(dalloc(&c.ring_x, cfg->ring_capacity * c.d));
   A(dalloc(&c.ring_y, cfg->ring_capacity));
   A(dalloc(&c.hits, R * NI));
@@ -472,11 +473,12 @@ int ls_route_batch(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* 
   }
   if (c.use_tc) {
     LS_CK(traced(c, TR_NORM_ROWS, 1, s, [&] {
-      return launch_norm_rows(c.n_inst, c.cfg.d_inst, c.inst_state, n_req, c.cfg.d_req, req_feats, c.mean,
+      return launch_norm_rows(tok_off, hits, c.pairx, c.n_inst, c.cfg.d_inst, c.inst_state, n_req, c.cfg.d_req,
+                              req_feats, c.mean,
                               c.stdv, c.tc.d_pad, c.xin, c.xrq, c.sms, s);
     }));
     LS_CK(traced(c, TR_SCORE_TC, 1, s, [&] {
-      return launch_score_tc(c.mlp, c.tc, c.pub, &c.st->route_b, n_req, c.n_inst, tok_off, hits,
+      return launch_score_tc(c.mlp, c.tc, c.pub, &c.st->route_b, n_req, c.n_inst, c.pairx,
                              c.xin, c.xrq, c.cfg.d_inst, c.cfg.d_req, c.mean, c.stdv, scores, c.d_err, c.sms,
                              s);
     }));

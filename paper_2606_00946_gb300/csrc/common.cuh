@@ -198,6 +198,7 @@ struct Ctx {
   int* work_n = nullptr;
   uint16_t* xin = nullptr;    // bf16 instance template rows [max_instances, d_pad]
   uint16_t* xrq = nullptr;    // bf16 request template rows [max_requests, d_pad]
+  uint4* pairx = nullptr;     // bf16 pair features of each (request, instance), 16 bytes: chunk 0 of its row
   bool use_tc = false;
   TcPlan tc;
 
@@ -329,11 +330,12 @@ bool plan_tc(const MlpDesc& m, TcPlan& p);
 // st->cur and bump the version; one launch.
 cudaError_t launch_publish(const MlpDesc& m, const TcPlan* tc, const float* master, const Published* pub,
                            int want_wt, DevState* st, int sms, cudaStream_t s);
-cudaError_t launch_norm_rows(int n_inst, int d_inst, const float* inst, int n_req, int d_req,
+cudaError_t launch_norm_rows(const int64_t* tok_off, const int32_t* hits, uint4* pairx, int n_inst, int d_inst,
+                             const float* inst, int n_req, int d_req,
                              const float* req, const float* mean, const float* stdv, int d_pad,
                              uint16_t* xin, uint16_t* xrq, int sms, cudaStream_t s);
 cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const Published* pub, const int32_t* sel,
-                            int n_req, int n_inst, const int64_t* tok_off, const int32_t* hits,
+                            int n_req, int n_inst, const uint4* pairx,
                             const uint16_t* xin, const uint16_t* xrq, int d_inst, int d_req,
                             const float* mean, const float* stdv, float* scores, int* err, int sms,
                             cudaStream_t s);

@@ -37,8 +37,7 @@ struct TcArgs {
   int64_t boff[LS_MAX_LAYERS];
   int64_t w_last_off;
   int n_req, n_inst, d, d_inst, d_req;
-  const int64_t* tok_off;
-  const int32_t* hits;
+  const uint4* pairx;    // [rows] bf16 pair features (chunk 0 of each feature row, zeros past column 5)
   const uint16_t* xin;   // [n_inst, d_pad] bf16 instance template rows (zero outside inst columns)
   const uint16_t* xrq;   // [n_req, d_pad]  bf16 request template rows (zero outside req columns)
   const float* mean;
@@ -59,6 +58,16 @@ __device__ __forceinline__ uint16_t bf16_bits(float x) {
   return *reinterpret_cast<uint16_t*>(&v);
 }
 
+// 16-byte global load that leaves L1 alone (streamed feature inputs must not
+// evict the epilogue's bias and weight lines)
+__device__ __forceinline__ uint4 ldg_stream(const void* p) {
+  uint4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+
 __device__ __forceinline__ void st_shared_v4(uint8_t* p, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
   asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(smem_u32(p)), "r"(a), "r"(b), "r"(c), "r"(d)
                : "memory");
@@ -66,28 +75,25 @@ __device__ __forceinline__ void st_shared_v4(uint8_t* p, uint32_t a, uint32_t b,
 
 // Feature tile of rows row0..row0+127: [pair(6) || inst || req || 0-pad] as bf16.
 // The instance and request blocks come from template rows that hold the
-// normalised values at their feature positions and zeros elsewhere, so a
-// 16-byte chunk of a feature row is the OR of the two templates' chunks (the
-// pair features, computed here, only occupy chunk 0).
-__device__ __forceinline__ void build_features(const TcArgs& a, uint8_t* A, int64_t row0, const float (&mu)[kPair],
-                                               const float (&sd)[kPair]) {
+// normalised values at their feature positions and zeros elsewhere, and the
+// pair features of each row come as one 16-byte chunk with zeros past column
+// 5 (k_norm_rows), so a 16-byte chunk of a feature row is the OR of at most
+// three loaded chunks.  `nthr` threads (index `tr`) share the tile.
+template <int U>
+__device__ __forceinline__ void build_tile(const TcArgs& a, uint8_t* X, int64_t row0, int tr, int nthr) {
   const int cpr = a.p.d_pad / 8;  // 16-byte chunks per row
   const int total = kTileM * cpr;
+  const int csh = (cpr & (cpr - 1)) == 0 ? __ffs(cpr) - 1 : -1;  // shift when cpr is a power of two
   const int64_t r0 = row0 / a.n_inst;
   const int i0 = (int)(row0 - r0 * a.n_inst);
-  constexpr int U = 4;  // chunks per thread per pass; all their loads are issued first
-  for (int base = 0; base < total; base += U * kThreadsTc) {
-    uint4 ti[U], tr[U];
-    int64_t L[U];
-    int h[U];
+  for (int base = 0; base < total; base += U * nthr) {
+    uint4 v[U];
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      const int e = base + u * kThreadsTc + threadIdx.x;
-      ti[u] = tr[u] = make_uint4(0u, 0u, 0u, 0u);
-      L[u] = 0;
-      h[u] = 0;
+      const int e = base + u * nthr + tr;
+      v[u] = make_uint4(0u, 0u, 0u, 0u);
       if (e >= total) continue;
-      const int m = e / cpr, c = e - m * cpr;
+      const int m = csh >= 0 ? e >> csh : e / cpr, c = e - m * cpr;
       const int64_t g = row0 + m;
       if (g >= a.rows) continue;
       int i = i0 + m;
@@ -98,28 +104,17 @@ __device__ __forceinline__ void build_features(const TcArgs& a, uint8_t* A, int6
         r += i / a.n_inst;
         i -= (i / a.n_inst) * a.n_inst;
       }
-      ti[u] = __ldg(reinterpret_cast<const uint4*>(a.xin + (int64_t)i * a.p.d_pad) + c);
-      tr[u] = __ldg(reinterpret_cast<const uint4*>(a.xrq + r * a.p.d_pad) + c);
-      if (c == 0) {
-        L[u] = __ldg(a.tok_off + r + 1) - __ldg(a.tok_off + r);
-        h[u] = __ldg(a.hits + g);
-      }
+      const uint4 ti = ldg_stream(reinterpret_cast<const uint4*>(a.xin + (int64_t)i * a.p.d_pad) + c);
+      const uint4 tq = ldg_stream(reinterpret_cast<const uint4*>(a.xrq + r * a.p.d_pad) + c);
+      const uint4 tp = c == 0 ? ldg_stream(a.pairx + g) : make_uint4(0u, 0u, 0u, 0u);
+      v[u] = make_uint4(ti.x | tq.x | tp.x, ti.y | tq.y | tp.y, ti.z | tq.z | tp.z, ti.w | tq.w | tp.w);
     }
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      const int e = base + u * kThreadsTc + threadIdx.x;
+      const int e = base + u * nthr + tr;
       if (e >= total) continue;
-      const int m = e / cpr, c = e - m * cpr;
-      uint4 v = make_uint4(ti[u].x | tr[u].x, ti[u].y | tr[u].y, ti[u].z | tr[u].z, ti[u].w | tr[u].w);
-      if (c == 0 && row0 + m < a.rows) {
-        uint16_t f[kPair];
-#pragma unroll
-        for (int k = 0; k < kPair; ++k) f[k] = bf16_bits(zscore(raw_feature(k, L[u], h[u], nullptr, 0, nullptr), mu[k], sd[k]));
-        v.x = f[0] | ((uint32_t)f[1] << 16);
-        v.y = f[2] | ((uint32_t)f[3] << 16);
-        v.z = f[4] | ((uint32_t)f[5] << 16);
-      }
-      st_shared_v4(A + sw128_offset(m, c * 8, kTileM), v.x, v.y, v.z, v.w);
+      const int m = csh >= 0 ? e >> csh : e / cpr, c = e - m * cpr;
+      st_shared_v4(X + sw128_offset(m, c * 8, kTileM), v[u].x, v[u].y, v[u].z, v[u].w);
     }
   }
 }
@@ -201,12 +196,6 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc(const __grid_constan
     }
   }
   uint32_t done_phase = 0;
-  float mu[kPair], sd[kPair];
-#pragma unroll
-  for (int k = 0; k < kPair; ++k) {
-    mu[k] = __ldg(a.mean + k);
-    sd[k] = __ldg(a.stdv + k);
-  }
   const int q4 = warp & 3;   // TMEM lane quadrant: rows 32*q4 .. 32*q4+31
   const int cq = warp >> 2;  // column quarter handled by this warp
   const int row = 32 * q4 + lane;
@@ -214,7 +203,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc(const __grid_constan
 
   for (int it = 0; it < my_tiles; ++it) {
     const int64_t row0 = (int64_t)(blockIdx.x + (int64_t)it * gridDim.x) * kTileM;
-    build_features(a, A, row0, mu, sd);
+    build_tile<4>(a, A, row0, threadIdx.x, kThreadsTc);
     fence_async_smem();
     __syncthreads();
     if (*abort_flag) break;
@@ -345,64 +334,6 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc(const __grid_constan
 constexpr int kProdWarps = 7, kEpiWarps = 8;
 constexpr int kProdThreads = kProdWarps * 32, kEpiThreads = kEpiWarps * 32;
 
-// feature tile built by `nthr` threads (index `tr`)
-__device__ __forceinline__ void build_tile_part(const TcArgs& a, uint8_t* X, int64_t row0, int tr, int nthr,
-                                                const float (&mu)[kPair], const float (&sd)[kPair]) {
-  const int cpr = a.p.d_pad / 8;
-  const int total = kTileM * cpr;
-  const int csh = (cpr & (cpr - 1)) == 0 ? __ffs(cpr) - 1 : -1;  // shift when cpr is a power of two
-  const int64_t r0 = row0 / a.n_inst;
-  const int i0 = (int)(row0 - r0 * a.n_inst);
-  constexpr int U = 5;
-  for (int base = 0; base < total; base += U * nthr) {
-    uint4 ti[U], trq[U];
-    int64_t L[U];
-    int h[U];
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int e = base + u * nthr + tr;
-      ti[u] = trq[u] = make_uint4(0u, 0u, 0u, 0u);
-      L[u] = 0;
-      h[u] = 0;
-      if (e >= total) continue;
-      const int m = csh >= 0 ? e >> csh : e / cpr, c = e - m * cpr;
-      const int64_t g = row0 + m;
-      if (g >= a.rows) continue;
-      int i = i0 + m;
-      int64_t r = r0;
-      if (a.n_inst >= 16) {
-        while (i >= a.n_inst) { i -= a.n_inst; ++r; }
-      } else {
-        r += i / a.n_inst;
-        i -= (i / a.n_inst) * a.n_inst;
-      }
-      ti[u] = __ldg(reinterpret_cast<const uint4*>(a.xin + (int64_t)i * a.p.d_pad) + c);
-      trq[u] = __ldg(reinterpret_cast<const uint4*>(a.xrq + r * a.p.d_pad) + c);
-      if (c == 0) {
-        L[u] = __ldg(a.tok_off + r + 1) - __ldg(a.tok_off + r);
-        h[u] = __ldg(a.hits + g);
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int e = base + u * nthr + tr;
-      if (e >= total) continue;
-      const int m = csh >= 0 ? e >> csh : e / cpr, c = e - m * cpr;
-      uint4 v = make_uint4(ti[u].x | trq[u].x, ti[u].y | trq[u].y, ti[u].z | trq[u].z, ti[u].w | trq[u].w);
-      if (c == 0 && row0 + m < a.rows) {
-        uint16_t f[kPair];
-#pragma unroll
-        for (int k = 0; k < kPair; ++k)
-          f[k] = bf16_bits(zscore(raw_feature(k, L[u], h[u], nullptr, 0, nullptr), mu[k], sd[k]));
-        v.x = f[0] | ((uint32_t)f[1] << 16);
-        v.y = f[2] | ((uint32_t)f[3] << 16);
-        v.z = f[4] | ((uint32_t)f[5] << 16);
-      }
-      st_shared_v4(X + sw128_offset(m, c * 8, kTileM), v.x, v.y, v.z, v.w);
-    }
-  }
-}
-
 __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc_pipe(const __grid_constant__ TcArgs a) {
   const bool pb = a.sel && *a.sel == 1;  // published buffer of this route
   const uint8_t* __restrict__ img = pb ? a.img1 : a.img0;
@@ -506,12 +437,6 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc_pipe(const __grid_co
     __syncwarp();
   } else if (warp <= kProdWarps) {
     // ------------------------------------------------------------ feature tiles
-    float mu[kPair], sd[kPair];
-#pragma unroll
-    for (int k = 0; k < kPair; ++k) {
-      mu[k] = __ldg(a.mean + k);
-      sd[k] = __ldg(a.stdv + k);
-    }
     const int tr = tid - 32;
     for (int t = 0; t < my_tiles; ++t) {
       const int xb = t & 1;
@@ -522,7 +447,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc_pipe(const __grid_co
       }
       if (*abort_flag) break;
       const int64_t row0 = (int64_t)(blockIdx.x + (int64_t)t * gridDim.x) * kTileM;
-      build_tile_part(a, X + (size_t)xb * xbytes, row0, tr, kProdThreads, mu, sd);
+      build_tile<5>(a, X + (size_t)xb * xbytes, row0, tr, kProdThreads);
       fence_async_smem();
       mbar_arrive(&x_full[xb]);
     }
@@ -578,11 +503,11 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc_pipe(const __grid_co
       if (lane == 0) mbar_arrive(d1_empty);
       if (!ok) { *abort_flag = 1; latch_error(a.err, LS_ERR_TIMEOUT); break; }
       // layer-2 epilogue: bias, ReLU, bf16, dot with the output weights
-      if (!mbar_wait(d2_full, (uint32_t)(t & 1))) { *abort_flag = 1; latch_error(a.err, LS_ERR_TIMEOUT); break; }
+      const bool ok2 = mbar_wait(d2_full, (uint32_t)(t & 1));
       tc_fence_after();
       uint64_t acc2 = 0;
       const int half = H2 / 2;
-      for (int c0 = wk * half; c0 < (wk + 1) * half; c0 += 32) {
+      for (int c0 = wk * half; ok2 && c0 < (wk + 1) * half; c0 += 32) {
         uint32_t v[2][16];
         tmem_ld16(D2 + lane_addr + (uint32_t)c0, v[0]);
         tmem_ld16(D2 + lane_addr + (uint32_t)(c0 + 16), v[1]);
@@ -608,7 +533,12 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc_pipe(const __grid_co
       if (lane == 0) mbar_arrive(d2_empty);
       float* pt = part + (t & 1) * kTileM;  // double-buffered by tile parity
       if (wk == 1) pt[row] = __uint_as_float((uint32_t)acc2) + __uint_as_float((uint32_t)(acc2 >> 32));
-      named_bar_sync(1, kEpiThreads);
+      // all epilogue warps continue, or all stop (a timeout here or elsewhere)
+      if (!named_bar_and(1, kEpiThreads, ok2 && !*reinterpret_cast<volatile int*>(abort_flag))) {
+        *abort_flag = 1;
+        latch_error(a.err, LS_ERR_TIMEOUT);
+        break;
+      }
       if (wk == 0) {
         const int64_t g = row0 + row;
         const float mine = __uint_as_float((uint32_t)acc2) + __uint_as_float((uint32_t)(acc2 >> 32));
@@ -620,28 +550,44 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc_pipe(const __grid_co
   if (warp == 0) tmem_dealloc(tmem, 512);
 }
 
-// Normalised bf16 template rows, computed once per batch: instance row i holds
-// the z-scored instance features at their feature positions (6 .. 6+d_inst)
-// and zeros elsewhere; request row r likewise for the request block.
-__global__ void k_norm_rows(int n_inst, int d_inst, const float* __restrict__ inst, int n_req, int d_req,
-                            const float* __restrict__ req, const float* __restrict__ mean,
+// Per batch, before the scorer: normalised bf16 template rows (instance row i
+// holds the z-scored instance features at their feature positions 6 ..
+// 6+d_inst and zeros elsewhere; request row r likewise for the request block)
+// and, for every (request, instance) pair, the 16-byte first chunk of its
+// feature row holding the six z-scored pair features (Sec. 4.1 Features;
+// Algorithm 4 Normalize) with zeros in columns 6 and 7.
+__global__ void k_norm_rows(const int64_t* __restrict__ tok_off, const int32_t* __restrict__ hits,
+                            uint4* __restrict__ pairx, int n_inst, int d_inst, const float* __restrict__ inst,
+                            int n_req, int d_req, const float* __restrict__ req, const float* __restrict__ mean,
                             const float* __restrict__ stdv, int d_pad, uint16_t* __restrict__ xin,
                             uint16_t* __restrict__ xrq) {
   const int64_t ni = (int64_t)n_inst * d_pad, nr = (int64_t)n_req * d_pad;
-  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < ni + nr;
+  const int64_t np = (int64_t)n_req * n_inst;
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < ni + nr + np;
        e += (int64_t)gridDim.x * blockDim.x) {
     if (e < ni) {
       const int64_t i = e / d_pad;
       const int k = (int)(e - i * d_pad) - kPair;
       xin[e] = (k >= 0 && k < d_inst) ? bf16_bits(zscore(inst[i * d_inst + k], mean[kPair + k], stdv[kPair + k]))
                                       : (uint16_t)0;
-    } else {
+    } else if (e < ni + nr) {
       const int64_t f = e - ni;
       const int64_t r = f / d_pad;
       const int k = (int)(f - r * d_pad) - kPair - d_inst;
       xrq[f] = (k >= 0 && k < d_req)
                    ? bf16_bits(zscore(req[r * d_req + k], mean[kPair + d_inst + k], stdv[kPair + d_inst + k]))
                    : (uint16_t)0;
+    } else {
+      const int64_t g = e - ni - nr;
+      const int64_t r = g / n_inst;
+      const int64_t L = __ldg(tok_off + r + 1) - __ldg(tok_off + r);
+      const int h = __ldg(hits + g);
+      uint16_t f[kPair];
+#pragma unroll
+      for (int k = 0; k < kPair; ++k)
+        f[k] = bf16_bits(zscore(raw_feature(k, L, h, nullptr, 0, nullptr), __ldg(mean + k), __ldg(stdv + k)));
+      pairx[g] = make_uint4(f[0] | ((uint32_t)f[1] << 16), f[2] | ((uint32_t)f[3] << 16),
+                            f[4] | ((uint32_t)f[5] << 16), 0u);
     }
   }
 }
@@ -713,18 +659,19 @@ bool plan_tc(const MlpDesc& m, TcPlan& p) {
   return true;
 }
 
-cudaError_t launch_norm_rows(int n_inst, int d_inst, const float* inst, int n_req, int d_req, const float* req,
-                             const float* mean, const float* stdv, int d_pad, uint16_t* xin, uint16_t* xrq,
-                             int sms, cudaStream_t s) {
-  const int64_t n = (int64_t)(n_inst + n_req) * d_pad;
+cudaError_t launch_norm_rows(const int64_t* tok_off, const int32_t* hits, uint4* pairx, int n_inst, int d_inst,
+                             const float* inst, int n_req, int d_req, const float* req, const float* mean,
+                             const float* stdv, int d_pad, uint16_t* xin, uint16_t* xrq, int sms, cudaStream_t s) {
+  const int64_t n = (int64_t)(n_inst + n_req) * d_pad + (int64_t)n_req * n_inst;
   if (n <= 0) return cudaSuccess;
   const int grid = (int)std::min<int64_t>((n + 255) / 256, (int64_t)sms * 8);
-  k_norm_rows<<<grid, 256, 0, s>>>(n_inst, d_inst, inst, n_req, d_req, req, mean, stdv, d_pad, xin, xrq);
+  k_norm_rows<<<grid, 256, 0, s>>>(tok_off, hits, pairx, n_inst, d_inst, inst, n_req, d_req, req, mean, stdv, d_pad,
+                                   xin, xrq);
   return cudaGetLastError();
 }
 
 cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const Published* pub, const int32_t* sel,
-                            int n_req, int n_inst, const int64_t* tok_off, const int32_t* hits,
+                            int n_req, int n_inst, const uint4* pairx,
                             const uint16_t* xin, const uint16_t* xrq, int d_inst, int d_req, const float* mean,
                             const float* stdv, float* scores, int* err, int sms, cudaStream_t s) {
   const int64_t rows = (int64_t)n_req * n_inst;
@@ -743,8 +690,7 @@ cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const Published* 
   a.d = m.w[0];
   a.d_inst = d_inst;
   a.d_req = d_req;
-  a.tok_off = tok_off;
-  a.hits = hits;
+  a.pairx = pairx;
   a.xin = xin;
   a.xrq = xrq;
   a.mean = mean;
