@@ -474,17 +474,20 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc_pipe(const __grid_co
         if (kq >= 2 && !mbar_wait(&a_empty[slot], (uint32_t)(((kq - 2) >> 1) & 1))) { ok = false; break; }
         uint8_t* dst = AR + (size_t)slot * kTileM * 128;
         const int colb = 64 * kb + 32 * wk;
+        // all loads of the block first: none waits behind this block's stores
+        float4 bq[8];
+#pragma unroll
+        for (int j4 = 0; j4 < 8; ++j4) bq[j4] = ldg4(b1 + colb + 4 * j4);
         uint32_t v[2][16];
         tmem_ld16(D1 + lane_addr + (uint32_t)colb, v[0]);
         tmem_ld16(D1 + lane_addr + (uint32_t)(colb + 16), v[1]);
         tmem_wait_ld();
 #pragma unroll
         for (int g = 0; g < 2; ++g) {
-          const int col = colb + 16 * g;
           uint32_t pk[8];
 #pragma unroll
           for (int j4 = 0; j4 < 4; ++j4) {
-            const float4 b = ldg4(b1 + col + 4 * j4);
+            const float4 b = bq[4 * g + j4];
             const uint64_t z0 = add_f32x2(((uint64_t)v[g][4 * j4 + 1] << 32) | v[g][4 * j4], f2pack(b.x, b.y));
             const uint64_t z1 = add_f32x2(((uint64_t)v[g][4 * j4 + 3] << 32) | v[g][4 * j4 + 2], f2pack(b.z, b.w));
             pk[2 * j4] = relu_bf16x2(cvt_bf16x2(z0));
@@ -508,6 +511,12 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc_pipe(const __grid_co
       uint64_t acc2 = 0;
       const int half = H2 / 2;
       for (int c0 = wk * half; ok2 && c0 < (wk + 1) * half; c0 += 32) {
+        float4 bq[8], wq[8];  // loaded before the TMEM wait
+#pragma unroll
+        for (int j4 = 0; j4 < 8; ++j4) {
+          bq[j4] = ldg4(b2 + c0 + 4 * j4);
+          wq[j4] = ldg4(w3 + c0 + 4 * j4);
+        }
         uint32_t v[2][16];
         tmem_ld16(D2 + lane_addr + (uint32_t)c0, v[0]);
         tmem_ld16(D2 + lane_addr + (uint32_t)(c0 + 16), v[1]);
@@ -516,9 +525,8 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc_pipe(const __grid_co
         for (int g = 0; g < 2; ++g) {
 #pragma unroll
           for (int j4 = 0; j4 < 4; ++j4) {
-            const int cc = c0 + 16 * g + 4 * j4;
-            const float4 b = ldg4(b2 + cc);
-            const float4 w = ldg4(w3 + cc);
+            const float4 b = bq[4 * g + j4];
+            const float4 w = wq[4 * g + j4];
             const uint32_t h0 = relu_bf16x2(cvt_bf16x2(add_f32x2(((uint64_t)v[g][4 * j4 + 1] << 32) | v[g][4 * j4],
                                                                    f2pack(b.x, b.y))));
             const uint32_t h1 = relu_bf16x2(cvt_bf16x2(
