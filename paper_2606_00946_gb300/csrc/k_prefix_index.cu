@@ -8,11 +8,15 @@
 // which is exactly "leading blocks all cached on instance i, stop at the first
 // miss" (Sec. 2: prefix reuse is strictly sequential).
 //
-// One CTA per request hashes its prompt 128 blocks at a time; warp 0 walks
-// the chunk 32 blocks per round: each lane looks up one block's mask, a
-// warp-wide prefix AND gives alive_b per lane, and an instance that stops
-// matching in the round gets h from one ballot.  Hashing stops as soon as no
-// instance matches, so tokens past the longest hit are never read.
+// One warp per request: each round hashes the next 32 blocks of the prompt
+// (one per lane; the chained prefix state is a warp-wide scan of the linear
+// recurrence), looks the 32 keys up at once, and a warp-wide prefix AND of
+// their instance masks gives, per lane, the instances still matching every
+// block up to it.  An instance that stops matching in the round gets its hit
+// length from one ballot; the lane that owns the instance keeps it and the
+// row is written once, coalesced, at the end.  The walk stops at the first
+// round after which no instance matches, so tokens past the longest hit plus
+// one round are never read.
 #include "blockhash.cuh"
 
 namespace ls {
@@ -49,84 +53,90 @@ __global__ void __launch_bounds__(kNT) k_prefix_index(int n_req, const int32_t* 
                                                       const uint64_t* __restrict__ gkeys,
                                                       const uint64_t* __restrict__ gmask, uint64_t gmask_slots,
                                                       int n_inst, int32_t* __restrict__ hits, DevState* st) {
-  __shared__ uint64_t keys[kNT];
   route_snapshot(st);
-  __shared__ uint64_t wtot[kNT / 32], wpre[kNT / 32], carry;
-  __shared__ int any_alive;
-  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
-  for (int r = blockIdx.x; r < n_req; r += gridDim.x) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  // G^(lane+1): the factor by which the state entering a round reaches this lane
+  uint64_t glane = 1;
+  {
+    uint64_t b = kG;
+    for (unsigned e = (unsigned)lane + 1; e; e >>= 1) {
+      if (e & 1) glane *= b;
+      b *= b;
+    }
+  }
+  for (int64_t r = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; r < n_req; r += warps) {
     const int64_t t0 = tok_off[r];
     const int64_t nb = (tok_off[r + 1] - t0) / kBlockTok;
     const int32_t* base = tok + t0;
     const bool aligned = ((reinterpret_cast<uintptr_t>(base) & 15) == 0);
-    int32_t* hrow = hits + (int64_t)r * n_inst;
     uint64_t alive[W];
+    int32_t hreg[W][2];  // hit length of instances 64w + lane and 64w + 32 + lane
 #pragma unroll
     for (int w = 0; w < W; ++w) {
       const int lo = 64 * w;
       alive[w] = n_inst >= lo + 64 ? ~0ull : (n_inst > lo ? ((1ull << (n_inst - lo)) - 1ull) : 0ull);
+      hreg[w][0] = hreg[w][1] = 0;
     }
-    if (t == 0) {
-      carry = kG;
-      any_alive = n_inst > 0;
-    }
-    __syncthreads();
-    for (int64_t c0 = 0; c0 < nb; c0 += kNT) {
-      if (!any_alive) break;  // uniform: read after a barrier
-      const int n = (int)(nb - c0 < kNT ? nb - c0 : kNT);
-      const uint64_t s_in = carry;
-      const uint64_t c = t < n ? block_content(base + (c0 + t) * kBlockTok, aligned) : 0ull;
-      const uint64_t st = chain_scan<kNT>(c, s_in, wtot, wpre);
-      if (t < n) keys[t] = key_of(st);
-      if (t == n - 1) carry = st;
-      __syncthreads();
-      if (warp == 0) {
-        bool any = true;
-        for (int p = 0; p < n && any; p += 32) {
-          const int b = p + lane;
-          uint64_t pa[W];
-          if (b < n) {
-            const int64_t slot = index_find(gkeys, gmask_slots, keys[b]);
+    uint64_t state = kG;  // s_{-1}
+    bool any = n_inst > 0;
+    for (int64_t p = 0; p < nb && any; p += 32) {
+      const int64_t b = p + lane;
+      const bool in = b < nb;
+      // inclusive scan: B = sum_{j <= lane} G^(lane - j) c_j, then s = G^(lane+1) s_in + B
+      uint64_t B = in ? block_content(base + b * kBlockTok, aligned) : 0ull;
 #pragma unroll
-            for (int w = 0; w < W; ++w) pa[w] = slot >= 0 ? __ldg(gmask + slot * W + w) : 0ull;
-          } else {
-#pragma unroll
-            for (int w = 0; w < W; ++w) pa[w] = 0ull;
-          }
-          any = false;
-#pragma unroll
-          for (int w = 0; w < W; ++w) {
-            uint64_t x = pa[w];
-#pragma unroll
-            for (int k = 0; k < 5; ++k) {
-              const uint64_t y = __shfl_up_sync(kFull, x, 1 << k);
-              if (lane >= (1 << k)) x &= y;
-            }
-            x &= alive[w];
-            const uint64_t end = __shfl_sync(kFull, x, 31);
-            uint64_t died = alive[w] & ~end;
-            while (died) {
-              const int bit = __ffsll((long long)died) - 1;
-              const int cnt = __popc(__ballot_sync(kFull, (x >> bit) & 1ull));
-              if (lane == 0) hrow[64 * w + bit] = (int32_t)(c0 + p + cnt);
-              died &= died - 1;
-            }
-            alive[w] = end;
-            any = any || end != 0;
-          }
-        }
-        if (lane == 0) any_alive = any;
+      for (int k = 0; k < 5; ++k) {
+        const int off = 1 << k;
+        const uint64_t o = __shfl_up_sync(kFull, B, off);
+        if (lane >= off) B = gpow(off) * o + B;
       }
-      __syncthreads();
-    }
-    if (warp == 0) {
-      // instances matching every full block (or requests without a full block)
+      const uint64_t s = glane * state + B;
+      const int last = (int)(nb - p < 32 ? nb - p : 32) - 1;
+      state = __shfl_sync(kFull, s, last);
+      uint64_t pa[W];
+      if (in) {
+        const int64_t slot = index_find(gkeys, gmask_slots, key_of(s));
 #pragma unroll
-      for (int w = 0; w < W; ++w)
-        for (int bit = lane; bit < 64; bit += 32)
-          if ((alive[w] >> bit) & 1ull) hrow[64 * w + bit] = (int32_t)nb;
+        for (int w = 0; w < W; ++w) pa[w] = slot >= 0 ? __ldg(gmask + slot * W + w) : 0ull;
+      } else {
+#pragma unroll
+        for (int w = 0; w < W; ++w) pa[w] = 0ull;
+      }
+      any = false;
+#pragma unroll
+      for (int w = 0; w < W; ++w) {
+        uint64_t x = pa[w];
+#pragma unroll
+        for (int k = 0; k < 5; ++k) {
+          const uint64_t y = __shfl_up_sync(kFull, x, 1 << k);
+          if (lane >= (1 << k)) x &= y;
+        }
+        x &= alive[w];
+        const uint64_t end = __shfl_sync(kFull, x, 31);
+        uint64_t died = alive[w] & ~end;
+        while (died) {
+          const int bit = __ffsll((long long)died) - 1;
+          const int cnt = __popc(__ballot_sync(kFull, (x >> bit) & 1ull));
+          if (lane == (bit & 31)) {
+            if (bit >> 5) hreg[w][1] = (int32_t)(p + cnt);
+            else hreg[w][0] = (int32_t)(p + cnt);
+          }
+          died &= died - 1;
+        }
+        alive[w] = end;
+        any = any || end != 0;
+      }
     }
-    __syncthreads();
+    int32_t* hrow = hits + (int64_t)r * n_inst;
+#pragma unroll
+    for (int w = 0; w < W; ++w)
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int bit = 32 * h + lane, i = 64 * w + bit;
+        // instances matching every full block (or requests without a full block)
+        if (i < n_inst) hrow[i] = ((alive[w] >> bit) & 1ull) ? (int32_t)nb : hreg[w][h];
+      }
   }
 }
 
@@ -174,7 +184,7 @@ cudaError_t launch_prefix_index(int n_req, const int32_t* tok, const int64_t* to
                                 const uint64_t* gmask, int W, uint64_t gmask_slots, int n_inst, int32_t* hits,
                                 int sms, DevState* st, cudaStream_t s) {
   if (n_req <= 0) return cudaSuccess;
-  const int grid = std::min(n_req, sms * 16);
+  const int grid = std::max(1, std::min((n_req + kNT / 32 - 1) / (kNT / 32), sms * 16));  // one warp per request
   switch (W) {
     case 1: k_prefix_index<1><<<grid, kNT, 0, s>>>(n_req, tok, tok_off, gkeys, gmask, gmask_slots, n_inst, hits, st); break;
     case 2: k_prefix_index<2><<<grid, kNT, 0, s>>>(n_req, tok, tok_off, gkeys, gmask, gmask_slots, n_inst, hits, st); break;
