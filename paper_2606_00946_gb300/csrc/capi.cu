@@ -191,8 +191,9 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
                                   (double)cfg->max_load);
     c.gslots = 16;
     while ((double)c.gslots < need) c.gslots <<= 1;
-    A(dalloc(&c.gkeys, c.gslots));
-    A(dalloc(&c.gmask, c.gslots * c.gW));
+    // one mask word: (key, mask) entries interleaved in gkeys; else separate arrays
+    A(dalloc(&c.gkeys, c.gW == 1 ? 2 * c.gslots : c.gslots));
+    if (c.gW > 1) A(dalloc(&c.gmask, c.gslots * c.gW));
   } else {
     A(dalloc(&c.tables, NI * c.slots));
   }
@@ -246,7 +247,7 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
   }
   if (e == cudaSuccess) {
     if (c.tables) A(cudaMemset(c.tables, 0, (size_t)NI * c.slots * sizeof(uint64_t)));
-    if (c.gkeys) A(cudaMemset(c.gkeys, 0, (size_t)c.gslots * sizeof(uint64_t)));
+    if (c.gkeys) A(cudaMemset(c.gkeys, 0, (size_t)c.gslots * (c.gW == 1 ? 2 : 1) * sizeof(uint64_t)));
     if (c.gmask) A(cudaMemset(c.gmask, 0, (size_t)c.gslots * c.gW * sizeof(uint64_t)));
     A(cudaMemset(c.table_count, 0, (size_t)NI * sizeof(int32_t)));
     A(cudaMemset(c.adam_m, 0, (size_t)c.n_params * sizeof(float)));
@@ -376,8 +377,8 @@ int ls_snapshot_update(ls_ctx* h, int32_t n_inst, const float* inst_state, const
     if (mode == LS_REPLACE) {
       // the index holds every instance: replacing the listed instances
       // (all of the snapshot) rebuilds it
-      LS_CK(cudaMemsetAsync(c.gkeys, 0, (size_t)c.gslots * sizeof(uint64_t), S(stream)));
-      LS_CK(cudaMemsetAsync(c.gmask, 0, (size_t)c.gslots * c.gW * sizeof(uint64_t), S(stream)));
+      LS_CK(cudaMemsetAsync(c.gkeys, 0, (size_t)c.gslots * (c.gW == 1 ? 2 : 1) * sizeof(uint64_t), S(stream)));
+      if (c.gmask) LS_CK(cudaMemsetAsync(c.gmask, 0, (size_t)c.gslots * c.gW * sizeof(uint64_t), S(stream)));
       LS_CK(cudaMemsetAsync(c.table_count, 0, (size_t)c.cfg.max_instances * sizeof(int32_t), S(stream)));
     }
     LS_CK(traced(c, TR_INDEX_INSERT, 1, S(stream), [&] {

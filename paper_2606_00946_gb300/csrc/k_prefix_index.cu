@@ -47,6 +47,28 @@ __device__ __forceinline__ int64_t index_find(const uint64_t* __restrict__ gkeys
   return -1;
 }
 
+// With one mask word (at most 64 instances) the index stores each key next to
+// its mask, entry e = (ent[2e], ent[2e+1]) = (key, mask), so one 32-byte
+// bucket of two entries answers a probe: mask of `key`, 0 if absent.
+__device__ __forceinline__ uint64_t index_mask_w1(const uint64_t* __restrict__ ent, uint64_t mslots, uint64_t key) {
+  uint64_t s = key & mslots;
+  uint32_t first = (uint32_t)(s & 1);
+  uint64_t b = s & ~(uint64_t)1;
+  for (uint64_t n = 0; n <= (mslots >> 1) + 1; ++n) {
+    const ulonglong2* q = reinterpret_cast<const ulonglong2*>(ent + 2 * b);
+    const ulonglong2 e0 = __ldg(q), e1 = __ldg(q + 1);
+    if (first == 0) {
+      if (e0.x == key) return e0.y;
+      if (e0.x == 0) return 0;
+    }
+    if (e1.x == key) return e1.y;
+    if (e1.x == 0) return 0;
+    first = 0;
+    b = (b + 2) & mslots;
+  }
+  return 0;
+}
+
 template <int W>
 __global__ void __launch_bounds__(kNT) k_prefix_index(int n_req, const int32_t* __restrict__ tok,
                                                       const int64_t* __restrict__ tok_off,
@@ -95,7 +117,9 @@ __global__ void __launch_bounds__(kNT) k_prefix_index(int n_req, const int32_t* 
       const int last = (int)(nb - p < 32 ? nb - p : 32) - 1;
       state = __shfl_sync(kFull, s, last);
       uint64_t pa[W];
-      if (in) {
+      if (in && W == 1) {
+        pa[0] = index_mask_w1(gkeys, gmask_slots, key_of(s));
+      } else if (in) {
         const int64_t slot = index_find(gkeys, gmask_slots, key_of(s));
 #pragma unroll
         for (int w = 0; w < W; ++w) pa[w] = slot >= 0 ? __ldg(gmask + slot * W + w) : 0ull;
@@ -144,7 +168,8 @@ __global__ void __launch_bounds__(kNT) k_prefix_index(int n_req, const int32_t* 
 // key_off.  A new key takes a slot (CAS on 0); the instance's bit is OR-ed into
 // the slot's mask; a bit set for the first time counts one distinct key of
 // that instance (more than max_keys latches LS_ERR_TABLE_FULL, as does a
-// probe sequence that finds no room).
+// probe sequence that finds no room).  With W == 1 keys and masks share the
+// interleaved entry array gkeys (gmask unused).
 __global__ void k_index_insert(const uint64_t* __restrict__ keys, const int64_t* __restrict__ key_off,
                                int n_inst, int64_t n_keys, uint64_t* gkeys, uint64_t* gmask, int W,
                                uint64_t gmask_slots, int32_t* counts, int64_t max_keys, int* err) {
@@ -158,17 +183,19 @@ __global__ void k_index_insert(const uint64_t* __restrict__ keys, const int64_t*
     uint64_t key = keys[k];
     if (key == 0) key = 1;
     unsigned long long* tab = reinterpret_cast<unsigned long long*>(gkeys);
+    const int kstride = W == 1 ? 2 : 1;
     uint64_t s = key & gmask_slots;
     int64_t slot = -1;
     for (uint64_t n = 0; n <= gmask_slots; ++n) {
-      const unsigned long long prev = atomicCAS(tab + s, 0ull, (unsigned long long)key);
+      const unsigned long long prev = atomicCAS(tab + s * kstride, 0ull, (unsigned long long)key);
       if (prev == 0ull || prev == key) { slot = (int64_t)s; break; }
       s = (s + 1) & gmask_slots;
     }
     if (slot < 0) { latch_error(err, LS_ERR_TABLE_FULL); continue; }
     const unsigned long long bit = 1ull << (lo & 63);
-    const unsigned long long old =
-        atomicOr(reinterpret_cast<unsigned long long*>(gmask + slot * W + (lo >> 6)), bit);
+    unsigned long long* mword = W == 1 ? tab + 2 * slot + 1
+                                       : reinterpret_cast<unsigned long long*>(gmask + slot * W + (lo >> 6));
+    const unsigned long long old = atomicOr(mword, bit);
     if (!(old & bit)) {
       const int cnt = atomicAdd(counts + lo, 1);
       if (cnt >= max_keys) latch_error(err, LS_ERR_TABLE_FULL);
