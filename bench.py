@@ -179,6 +179,26 @@ class ClockSampler:
                 "power_w_max": float(np.nanmax([num(r[3]) for r in self.rows]))}
 
 
+def profiled_traffic(kernel):
+    """DRAM bytes per launch of `kernel` from the committed ncu summary, if the
+    summary was taken on the kernel's current source (else None)."""
+    import glob
+    import hashlib
+    src = os.path.join(ROOT, "paper_2606_00946_gb300", "csrc")
+    h = hashlib.sha256()
+    for f in ("k_score_tc.cu", "sm100.cuh"):
+        with open(os.path.join(src, f), "rb") as fh:
+            h.update(fh.read())
+    sha = h.hexdigest()[:16]
+    for path in glob.glob(os.path.join(ROOT, "profiles", "*.md")):
+        for line in open(path):
+            if line.startswith("roofline-traffic:"):
+                kv = dict(p.split("=", 1) for p in line.split()[1:])
+                if kv.get("kernel") == kernel and kv.get("source_sha256") == sha:
+                    return float(kv["bytes_per_launch"])
+    return None
+
+
 def measured_peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -377,7 +397,7 @@ def main():
         alg, peak, unit, bound = train_flops(cfg.widths, Bt) / 1e12 / 5, peaks["bf16_tflops"], "TFLOP/s", "tensor"
     achieved = alg / (per[dom] / 1e3)
     roofline = {"kernel": dom, "bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
-                "frac": achieved / peak, "traffic": None, "peak_source": f"{peak_src} (burst)",
+                "frac": achieved / peak, "traffic": profiled_traffic(dom) if dom == "score_tc" else None, "peak_source": f"{peak_src} (burst)",
                 "avg_launch_ms": per[dom],
                 "timing": "kernel durations from CUDA events around each launch over steps issued call by "
                           "call (instrumented); value and ms_per_step from the K graph replays"}

@@ -136,8 +136,9 @@ int ls_sync_status(ls_ctx *ctx);
 int ls_get_info(ls_ctx *ctx, ls_info *out /* host */);
 
 /* Set the fp32 master parameters (device, ls_param_count floats: W1 [w1,w0]
- * row-major, b1 [w1], W2, b2, ...), reset optimiser state and step count.
- * Routing keeps using the previously published weights until ls_publish. */
+ * row-major, b1 [w1], W2, b2, ...), reset optimiser state and step count
+ * (synchronises `stream`).  Routing keeps using the previously published
+ * weights until ls_publish. */
 int ls_set_params(ls_ctx *ctx, const float *params, void *stream);
 int ls_get_params(ls_ctx *ctx, float *params_out, void *stream);
 

@@ -257,6 +257,7 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
     DevState init{};
     init.cur = -1;
     init.route_b = 0;
+    init.beta_pow[0] = init.beta_pow[1] = 1.0;
     A(cudaMemcpy(c.st, &init, sizeof(DevState), cudaMemcpyHostToDevice));
     A(cudaDeviceSynchronize());
   }
@@ -313,7 +314,13 @@ int ls_set_params(ls_ctx* h, const float* params, void* stream) {
   LS_CK(cudaMemcpyAsync(c.master, params, n, cudaMemcpyDeviceToDevice, S(stream)));
   LS_CK(cudaMemsetAsync(c.adam_m, 0, n, S(stream)));
   LS_CK(cudaMemsetAsync(c.adam_v, 0, n, S(stream)));
-  LS_CK(cudaMemsetAsync(&c.st->step, 0, sizeof(int64_t), S(stream)));
+  {
+    const int64_t zero = 0;
+    const double ones[2] = {1.0, 1.0};
+    LS_CK(cudaMemcpyAsync(&c.st->step, &zero, sizeof(zero), cudaMemcpyHostToDevice, S(stream)));
+    LS_CK(cudaMemcpyAsync(c.st->beta_pow, ones, sizeof(ones), cudaMemcpyHostToDevice, S(stream)));
+    LS_CK(cudaStreamSynchronize(S(stream)));  // the host values above are locals
+  }
   if (c.tf.on) LS_CK(train_fast_images(c, S(stream)));
   c.have_params = true;
   return LS_OK;
@@ -347,7 +354,9 @@ int ls_set_opt_state(ls_ctx* h, const float* m, const float* v, int64_t step, vo
   LS_CK(cudaMemcpyAsync(c.adam_m, m, n, cudaMemcpyDeviceToDevice, S(stream)));
   LS_CK(cudaMemcpyAsync(c.adam_v, v, n, cudaMemcpyDeviceToDevice, S(stream)));
   const int64_t st_step = step;
+  const double pw[2] = {std::pow(0.9, (double)step), std::pow(0.999, (double)step)};
   LS_CK(cudaMemcpyAsync(&c.st->step, &st_step, sizeof(int64_t), cudaMemcpyHostToDevice, S(stream)));
+  LS_CK(cudaMemcpyAsync(c.st->beta_pow, pw, sizeof(pw), cudaMemcpyHostToDevice, S(stream)));
   LS_CK(cudaStreamSynchronize(S(stream)));
   return LS_OK;
 }

@@ -74,7 +74,23 @@ struct DevState {
   uint64_t version;         // publishes completed
   uint64_t pub_version[2];  // version held by each buffer
   uint32_t done[4];         // per-kernel block arrival counters (last-block updates)
+  float adam_bc[2];         // 1 - beta1^t, 1 - beta2^t of the step in flight, t = step + 1
+  double beta_pow[2];       // beta1^step, beta2^step (fp64 running products)
 };
+
+// Adam bias corrections of the coming step, 1 - beta^(step+1), from the fp64
+// running powers (one multiply each, by one thread of the step's first kernel).
+__device__ __forceinline__ void set_adam_bc(DevState* st) {
+  st->adam_bc[0] = (float)(1.0 - st->beta_pow[0] * 0.9);
+  st->adam_bc[1] = (float)(1.0 - st->beta_pow[1] * 0.999);
+}
+
+// The optimiser's last block, after a step: advance the counter and the powers.
+__device__ __forceinline__ void advance_step(DevState* st, int64_t t) {
+  st->step = t;
+  st->beta_pow[0] *= 0.9;
+  st->beta_pow[1] *= 0.999;
+}
 enum { DONE_RING = 0, DONE_OPT = 1, DONE_PUB = 2 };
 
 // Kernel-level tracing: when enabled, every launch is bracketed by CUDA events

@@ -83,7 +83,8 @@ __global__ void __launch_bounds__(256) k_publish(const __grid_constant__ PubArgs
       *reinterpret_cast<uint4*>(img + off) = q;
     }
   }
-  __threadfence();
+  // last_block: barrier, then thread 0 fences (cumulative over the block's
+  // writes) before it arrives; the flip below comes after every block's writes
   if (last_block(&a.st->done[DONE_PUB]) && threadIdx.x == 0) {
     const uint64_t ver = a.st->version + 1;
     a.st->pub_version[tgt] = ver;

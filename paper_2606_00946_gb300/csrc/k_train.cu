@@ -106,7 +106,7 @@ __global__ void __launch_bounds__(256) k_gemm(GemmArgs g) {
 // or (step*B + j) mod valid, with step and the ring's fill read from the device
 // state; z-score in fp32, bf16-rounded in bf16 mode.  An empty ring latches
 // LS_ERR_STATE (rows then come from slot 0).
-__global__ void k_train_gather(int B, int d, const int32_t* __restrict__ idx, const DevState* st,
+__global__ void k_train_gather(int B, int d, const int32_t* __restrict__ idx, DevState* st,
                                int64_t capacity, const float* __restrict__ ring_x,
                                const float* __restrict__ ring_y, const float* __restrict__ mean,
                                const float* __restrict__ stdv, int bf16, float* __restrict__ x0,
@@ -115,6 +115,7 @@ __global__ void k_train_gather(int B, int d, const int32_t* __restrict__ idx, co
   const int64_t count = st->ring_count;
   const int64_t valid = count < capacity ? count : capacity;
   if (valid < 1 && blockIdx.x == 0 && threadIdx.x == 0) latch_error(err, LS_ERR_STATE);
+  if (blockIdx.x == 0 && threadIdx.x == 0) set_adam_bc(st);
   const int64_t total = (int64_t)B * d;
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
        e += (int64_t)gridDim.x * blockDim.x) {
@@ -260,20 +261,15 @@ __global__ void k_sgd(int64_t n, float lr, const float* __restrict__ g, float* _
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n;
        e += (int64_t)gridDim.x * blockDim.x)
     p[e] = p[e] - lr * g[e];
-  if (last_block(&st->done[DONE_OPT]) && threadIdx.x == 0) st->step = t;
+  if (last_block(&st->done[DONE_OPT]) && threadIdx.x == 0) advance_step(st, t);
 }
 
-// Adam, t = steps taken + 1: bias corrections 1 - beta^t formed in fp64.
+// Adam, t = steps taken + 1: bias corrections 1 - beta^t formed in fp64 by
+// the gather kernel of this step.
 __global__ void k_adam(int64_t n, float lr, const float* __restrict__ g, float* __restrict__ p,
                        float* __restrict__ m, float* __restrict__ v, DevState* st) {
-  __shared__ float bc[2];
   const int64_t t = st->step + 1;
-  if (threadIdx.x == 0) {
-    bc[0] = (float)(1.0 - pow(0.9, (double)t));
-    bc[1] = (float)(1.0 - pow(0.999, (double)t));
-  }
-  __syncthreads();
-  const float bc1 = bc[0], bc2 = bc[1];
+  const float bc1 = st->adam_bc[0], bc2 = st->adam_bc[1];
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n;
        e += (int64_t)gridDim.x * blockDim.x) {
     const float ge = g[e];
@@ -284,7 +280,7 @@ __global__ void k_adam(int64_t n, float lr, const float* __restrict__ g, float* 
     const float mh = me / bc1, vh = ve / bc2;
     p[e] = p[e] - lr * mh / (sqrtf(vh) + 1e-8f);
   }
-  if (last_block(&st->done[DONE_OPT]) && threadIdx.x == 0) st->step = t;
+  if (last_block(&st->done[DONE_OPT]) && threadIdx.x == 0) advance_step(st, t);
 }
 
 template <bool TA, bool TB, int EPI>

@@ -350,7 +350,7 @@ __global__ void __launch_bounds__(kT, 1) k_tr_gemm(const __grid_constant__ TrArg
 // valid) z-scored and rounded to bf16 into img(A_0) and img(A_0^T); rows past
 // the batch and columns past d are zero.  Thread = (row j, 8 columns).
 __global__ void k_tr_gather(int B, int rows_pad, int d, int d_pad, const int32_t* __restrict__ idx,
-                            const DevState* st, int64_t capacity, const float* __restrict__ ring_x,
+                            DevState* st, int64_t capacity, const float* __restrict__ ring_x,
                             const float* __restrict__ ring_y, const float* __restrict__ mean,
                             const float* __restrict__ stdv, uint8_t* __restrict__ a0, uint8_t* __restrict__ a0t,
                             float* __restrict__ y, int* err) {
@@ -358,6 +358,7 @@ __global__ void k_tr_gather(int B, int rows_pad, int d, int d_pad, const int32_t
   const int64_t count = st->ring_count;
   const int64_t valid = count < capacity ? count : capacity;
   if (valid < 1 && blockIdx.x == 0 && threadIdx.x == 0) latch_error(err, LS_ERR_STATE);
+  if (blockIdx.x == 0 && threadIdx.x == 0) set_adam_bc(st);
   const int64_t total = (int64_t)rows_pad * (d_pad / 8);
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
        e += (int64_t)gridDim.x * blockDim.x) {
@@ -439,13 +440,8 @@ struct OptArgs {
 // optimiser update of the fp32 master, and the bf16 images of the updated
 // hidden-layer weights.  Block 0 also forms the minibatch loss.
 __global__ void __launch_bounds__(256) k_tr_opt(const __grid_constant__ OptArgs a) {
-  __shared__ float bc[2];
   const int64_t t = a.st->step + 1;
-  if (threadIdx.x == 0) {
-    bc[0] = (float)(1.0 - pow(0.9, (double)t));
-    bc[1] = (float)(1.0 - pow(0.999, (double)t));
-  }
-  __syncthreads();
+  const float bc1 = a.st->adam_bc[0], bc2 = a.st->adam_bc[1];  // set by the gather kernel
   const MlpDesc& m = a.m;
   const int nl = m.n_layers;
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < a.n;
@@ -484,7 +480,7 @@ __global__ void __launch_bounds__(256) k_tr_opt(const __grid_constant__ OptArgs 
         const float ve = 0.999f * a.vo[e] + 0.001f * g * g;
         a.mo[e] = me;
         a.vo[e] = ve;
-        const float mh = me / bc[0], vh = ve / bc[1];
+        const float mh = me / bc1, vh = ve / bc2;
         p = p - a.lr * mh / (sqrtf(vh) + 1e-8f);
       }
       a.p[e] = p;
@@ -504,7 +500,7 @@ __global__ void __launch_bounds__(256) k_tr_opt(const __grid_constant__ OptArgs 
     for (int tt = 0; tt < a.T; ++tt) s += a.partLoss[tt];
     *a.loss_out = s / (float)a.B;
   }
-  if (a.mode != 0 && last_block(&a.st->done[DONE_OPT]) && threadIdx.x == 0) a.st->step = t;
+  if (a.mode != 0 && last_block(&a.st->done[DONE_OPT]) && threadIdx.x == 0) advance_step(a.st, t);
 }
 
 int gemm_smem_bytes() {
