@@ -13,7 +13,7 @@ namespace ls {
 const char* const kTraceNames[TR_COUNT] = {
     "hash_blocks", "table_insert", "prefix_match", "score_simt", "argmin", "assemble_features",
     "ring_append", "publish", "train_gather", "gemm_fwd", "loss_grad", "gemm_dw", "reduce_dw",
-    "colsum_db", "gemm_dx", "optimizer", "memset", "score_tc", "norm_rows", "publish_tc",
+    "colsum_db", "gemm_dx", "optimizer", "memset", "score_tc", "features", "publish_tc",
     "hash_screen", "probe_screen", "probe_walk", "gemm_tc_fwd", "gemm_tc_dw", "gemm_tc_dx", "prefix_index",
     "index_insert"};
 }
@@ -107,7 +107,7 @@ void free_all(Ctx& c) {
   void* ptrs[] = {c.tables, c.table_count, c.inst_state, c.mean, c.stdv, c.master, c.adam_m,
                   c.adam_v, c.pub[0].params, c.pub[0].wt, c.pub[1].params, c.pub[1].wt,
                   c.ring_x, c.ring_y, c.hits, c.scores, c.tx, c.tz, c.ty, c.dz0, c.dz1, c.grad,
-                  c.gpart, c.loss_tmp, c.d_err, c.pub[0].img, c.pub[1].img, c.xin, c.xrq, c.pairx,
+                  c.gpart, c.loss_tmp, c.d_err, c.pub[0].img, c.pub[1].img, c.xin, c.xrq, c.pairx, c.ximg,
                   c.bkeys, c.work, c.work_n, c.gkeys, c.gmask, c.st, c.tf.base, c.tf.parts};
   for (void* p : ptrs)
     if (p) cudaFree(p);
@@ -217,7 +217,9 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
   A(dalloc(&c.work_n, 1));
   A(dalloc(&c.xin, NI * std::max(1, c.tc.d_pad)));
   A(dalloc(&c.xrq, R * std::max(1, c.tc.d_pad)));
-  if (c.use_tc) A(dalloc(&c.pairx, R * NI));
+  if (c.use_tc && !c.tc.pipe) A(dalloc(&c.pairx, R * NI));
+  if (c.use_tc && c.tc.pipe)
+    A(dalloc(&c.ximg, (R * NI + 127) / 128 * ((int64_t)c.tc.d_pad / 64) * 16384));
   A(dalloc(&c.ring_x, cfg->ring_capacity * c.d));
   A(dalloc(&c.ring_y, cfg->ring_capacity));
   A(dalloc(&c.hits, R * NI));
@@ -367,6 +369,9 @@ int ls_set_normalizer(ls_ctx* h, const float* mean, const float* stdv, void* str
   LS_CK(cudaMemcpyAsync(c.mean, mean, (size_t)c.d * sizeof(float), cudaMemcpyDeviceToDevice, S(stream)));
   LS_CK(cudaMemcpyAsync(c.stdv, stdv, (size_t)c.d * sizeof(float), cudaMemcpyDeviceToDevice, S(stream)));
   c.have_norm = true;
+  if (c.use_tc && c.tc.pipe && c.n_inst > 0)  // instance template rows follow the normaliser
+    LS_CK(launch_inst_templates(c.n_inst, c.cfg.d_inst, c.inst_state, c.mean, c.stdv, c.tc.d_pad, c.xin, c.sms,
+                                S(stream)));
   return LS_OK;
 }
 
@@ -382,6 +387,11 @@ int ls_snapshot_update(ls_ctx* h, int32_t n_inst, const float* inst_state, const
   if (c.cfg.d_inst > 0)
     LS_CK(cudaMemcpyAsync(c.inst_state, inst_state, (size_t)n_inst * c.cfg.d_inst * sizeof(float),
                           cudaMemcpyDeviceToDevice, S(stream)));
+  if (c.use_tc && c.tc.pipe && c.have_norm)  // instance template rows follow the snapshot
+    LS_CK(traced(c, TR_NORM_ROWS, 1, S(stream), [&] {
+      return launch_inst_templates(n_inst, c.cfg.d_inst, c.inst_state, c.mean, c.stdv, c.tc.d_pad, c.xin, c.sms,
+                                   S(stream));
+    }));
   if (keys && c.use_index) {
     if (mode == LS_REPLACE) {
       // the index holds every instance: replacing the listed instances
@@ -483,12 +493,15 @@ int ls_route_batch(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* 
   }
   if (c.use_tc) {
     LS_CK(traced(c, TR_NORM_ROWS, 1, s, [&] {
+      if (c.tc.pipe)
+        return launch_feature_image(tok_off, hits, c.n_inst, c.xin, c.cfg.d_inst, n_req, c.cfg.d_req, req_feats,
+                                    c.mean, c.stdv, c.tc.d_pad, c.ximg, c.sms, s);
       return launch_norm_rows(tok_off, hits, c.pairx, c.n_inst, c.cfg.d_inst, c.inst_state, n_req, c.cfg.d_req,
                               req_feats, c.mean,
                               c.stdv, c.tc.d_pad, c.xin, c.xrq, c.sms, s);
     }));
     LS_CK(traced(c, TR_SCORE_TC, 1, s, [&] {
-      return launch_score_tc(c.mlp, c.tc, c.pub, &c.st->route_b, n_req, c.n_inst, c.pairx,
+      return launch_score_tc(c.mlp, c.tc, c.pub, &c.st->route_b, n_req, c.n_inst, c.pairx, c.ximg,
                              c.xin, c.xrq, c.cfg.d_inst, c.cfg.d_req, c.mean, c.stdv, scores, c.d_err, c.sms,
                              s);
     }));

@@ -215,6 +215,7 @@ struct Ctx {
   uint16_t* xin = nullptr;    // bf16 instance template rows [max_instances, d_pad]
   uint16_t* xrq = nullptr;    // bf16 request template rows [max_requests, d_pad]
   uint4* pairx = nullptr;     // bf16 pair features of each (request, instance), 16 bytes: chunk 0 of its row
+  uint8_t* ximg = nullptr;    // pipelined scorer: bf16 feature rows of the batch as MMA-layout tiles
   bool use_tc = false;
   TcPlan tc;
 
@@ -350,8 +351,13 @@ cudaError_t launch_norm_rows(const int64_t* tok_off, const int32_t* hits, uint4*
                              const float* inst, int n_req, int d_req,
                              const float* req, const float* mean, const float* stdv, int d_pad,
                              uint16_t* xin, uint16_t* xrq, int sms, cudaStream_t s);
+cudaError_t launch_inst_templates(int n_inst, int d_inst, const float* inst, const float* mean, const float* stdv,
+                                  int d_pad, uint16_t* xin, int sms, cudaStream_t s);
+cudaError_t launch_feature_image(const int64_t* tok_off, const int32_t* hits, int n_inst, const uint16_t* xin,
+                                 int d_inst, int n_req, int d_req, const float* req, const float* mean,
+                                 const float* stdv, int d_pad, uint8_t* ximg, int sms, cudaStream_t s);
 cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const Published* pub, const int32_t* sel,
-                            int n_req, int n_inst, const uint4* pairx,
+                            int n_req, int n_inst, const uint4* pairx, const uint8_t* ximg,
                             const uint16_t* xin, const uint16_t* xrq, int d_inst, int d_req,
                             const float* mean, const float* stdv, float* scores, int* err, int sms,
                             cudaStream_t s);

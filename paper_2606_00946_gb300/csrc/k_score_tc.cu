@@ -38,6 +38,7 @@ struct TcArgs {
   int64_t w_last_off;
   int n_req, n_inst, d, d_inst, d_req;
   const uint4* pairx;    // [rows] bf16 pair features (chunk 0 of each feature row, zeros past column 5)
+  const uint8_t* ximg;   // pipelined kernel: feature tiles, tile t = xbytes at t * xbytes, in the MMA layout
   const uint16_t* xin;   // [n_inst, d_pad] bf16 instance template rows (zero outside inst columns)
   const uint16_t* xrq;   // [n_req, d_pad]  bf16 request template rows (zero outside req columns)
   const float* mean;
@@ -331,10 +332,18 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc(const __grid_constan
 // still producing K-blocks; D1 and D2 sit in separate TMEM halves, so the final
 // epilogue of tile t overlaps the layer-1 MMA of tile t+1.
 // ---------------------------------------------------------------------------
-constexpr int kProdWarps = 7, kEpiWarps = 8;
-constexpr int kProdThreads = kProdWarps * 32, kEpiThreads = kEpiWarps * 32;
+// Warp roles: 0 = MMA issuer, 1 = feature-tile loader (one bulk copy per
+// tile from the feature image), 2..9 = layer-1 epilogue (E1), 10..17 =
+// layer-2 + output epilogue (E2).  E1 of tile t+1 runs while E2 finishes tile
+// t.  18 warps = at most 5 per SM sub-partition: 96 registers per thread.
+constexpr int kEpiWarps = 8, kEpiThreads = kEpiWarps * 32;
+constexpr int kE1Warp0 = 2, kE2Warp0 = kE1Warp0 + kEpiWarps;
+constexpr int kThreadsPipe = (kE2Warp0 + kEpiWarps) * 32;  // 576
+// Feature tiles in flight.  One suffices: the copy of tile t+1 starts when the
+// layer-1 MMA of tile t completes and has the rest of tile t to land.
+constexpr int kXB = 1;
 
-__global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc_pipe(const __grid_constant__ TcArgs a) {
+__global__ void __launch_bounds__(kThreadsPipe, 1) k_score_tc_pipe(const __grid_constant__ TcArgs a) {
   const bool pb = a.sel && *a.sel == 1;  // published buffer of this route
   const uint8_t* __restrict__ img = pb ? a.img1 : a.img0;
   const float* __restrict__ params = pb ? a.params1 : a.params0;
@@ -346,10 +355,13 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc_pipe(const __grid_co
   const int nk1 = H1 / 64;                // K-blocks of layer 2 (= 64-column blocks of D1)
   const int xbytes = nk0 * kTileM * 128;  // one feature tile
   uint8_t* W = smem;                                            // resident weight chunks
-  uint8_t* X = W + (size_t)p.chunks * p.chunk_bytes;            // [2] feature tiles
-  uint8_t* AR = X + 2 * (size_t)xbytes;                         // [2] activation K-blocks (16 KB)
+  uint8_t* X = W + (size_t)p.chunks * p.chunk_bytes;            // [kXB] feature tiles
+  uint8_t* AR = X + kXB * (size_t)xbytes;                       // [2] activation K-blocks (16 KB)
   float* part = reinterpret_cast<float*>(AR + 2 * kTileM * 128);  // [2][128]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(part + 2 * kTileM);
+  float* sb1 = part + 2 * kTileM;                               // [256] layer-1 bias
+  float* sb2 = sb1 + 256;                                       // [256] layer-2 bias
+  float* sw3 = sb2 + 256;                                       // [256] output-layer weights
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sw3 + 256);
   uint64_t* x_full = bars;       // [2]
   uint64_t* x_empty = bars + 2;  // [2]
   uint64_t* a_full = bars + 4;   // [2]
@@ -365,7 +377,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc_pipe(const __grid_co
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (tid == 0) {
     for (int b = 0; b < 2; ++b) {
-      mbar_init(&x_full[b], kProdThreads);
+      mbar_init(&x_full[b], 1);  // only the first kXB are used
       mbar_init(&x_empty[b], 1);
       mbar_init(&a_full[b], kEpiWarps);
       mbar_init(&a_empty[b], 1);
@@ -381,6 +393,11 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc_pipe(const __grid_co
   if (warp == 0) {
     tmem_alloc(tmem_holder, 512);
     tmem_relinquish();
+  }
+  for (int k = tid; k < H1; k += blockDim.x) sb1[k] = __ldg(params + a.boff[0] + k);
+  for (int k = tid; k < H2; k += blockDim.x) {
+    sb2[k] = __ldg(params + a.boff[1] + k);
+    sw3[k] = __ldg(params + a.w_last_off + k);
   }
   tc_fence_before();
   __syncthreads();
@@ -400,8 +417,8 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc_pipe(const __grid_co
       bool ok = mbar_wait(w_full, 0);
       const uint32_t id1 = idesc_bf16_f32(kTileM, H1), id2 = idesc_bf16_f32(kTileM, H2);
       for (int t = 0; t < my_tiles && ok; ++t) {
-        const int xb = t & 1;
-        ok = mbar_wait(&x_full[xb], (uint32_t)((t >> 1) & 1));
+        const int xb = t % kXB;
+        ok = mbar_wait(&x_full[xb], (uint32_t)((t / kXB) & 1));
         if (ok && t >= 1) ok = mbar_wait(d1_empty, (uint32_t)((t - 1) & 1));
         if (!ok) break;
         tc_fence_after();
@@ -435,53 +452,53 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc_pipe(const __grid_co
       }
     }
     __syncwarp();
-  } else if (warp <= kProdWarps) {
-    // ------------------------------------------------------------ feature tiles
-    const int tr = tid - 32;
-    for (int t = 0; t < my_tiles; ++t) {
-      const int xb = t & 1;
-      if (t >= 2 && !mbar_wait(&x_empty[xb], (uint32_t)(((t - 2) >> 1) & 1))) {
-        *abort_flag = 1;
-        latch_error(a.err, LS_ERR_TIMEOUT);
-        break;
+  } else if (warp < kE1Warp0) {
+    // ------------------------------------------------------------ feature-tile loader
+    if (lane == 0) {
+      int last[2] = {-1, -1};
+      for (int t = 0; t < my_tiles; ++t) {
+        const int xb = t % kXB;
+        if (t >= kXB && !mbar_wait(&x_empty[xb], (uint32_t)(((t - kXB) / kXB) & 1))) {
+          *abort_flag = 1;
+          latch_error(a.err, LS_ERR_TIMEOUT);
+          break;
+        }
+        if (*reinterpret_cast<volatile int*>(abort_flag)) break;
+        const int64_t tile = blockIdx.x + (int64_t)t * gridDim.x;
+        mbar_arrive_expect_tx(&x_full[xb], (uint32_t)xbytes);
+        bulk_g2s(X + (size_t)xb * xbytes, a.ximg + tile * xbytes, (uint32_t)xbytes, &x_full[xb]);
+        last[xb] = t;
       }
-      if (*abort_flag) break;
-      const int64_t row0 = (int64_t)(blockIdx.x + (int64_t)t * gridDim.x) * kTileM;
-      build_tile<5>(a, X + (size_t)xb * xbytes, row0, tr, kProdThreads);
-      fence_async_smem();
-      mbar_arrive(&x_full[xb]);
+      // copies still in flight land in this CTA's shared memory: wait for them
+      // (bounded) before the CTA can exit
+      for (int b = 0; b < kXB; ++b)
+        if (last[b] >= 0) mbar_wait(&x_full[b], (uint32_t)((last[b] / kXB) & 1));
     }
-  } else {
-    // ------------------------------------------------------------ epilogues
-    const int ew = warp - 1 - kProdWarps;  // 0..7
+    __syncwarp();
+  } else if (warp < kE2Warp0) {
+    // ------------------------------------------------------------ E1: layer-1 epilogue
+    const int ew = warp - kE1Warp0;        // 0..7
     const int q4 = warp & 3;               // TMEM lane quadrant
-    const int wk = ew >> 2;                // 0/1: column half
+    const int wk = ew >> 2;                // which 32 columns of each 64-column K-block
     const int row = 32 * q4 + lane;
     const uint32_t lane_addr = (uint32_t)(32 * q4) << 16;
-    const float* b1 = params + a.boff[0];
-    const float* b2 = params + a.boff[1];
-    const float* w3 = params + a.w_last_off;
-    const float b3 = __ldg(params + p.b_last_off);
     for (int t = 0; t < my_tiles; ++t) {
-      const int64_t row0 = (int64_t)(blockIdx.x + (int64_t)t * gridDim.x) * kTileM;
       if (!mbar_wait(d1_full, (uint32_t)(t & 1))) { *abort_flag = 1; latch_error(a.err, LS_ERR_TIMEOUT); break; }
       tc_fence_after();
-      // layer-1 epilogue, one 64-column K-block at a time (this warp: 32 columns of it)
       bool ok = true;
       for (int kb = 0; kb < nk1; ++kb) {
         const int64_t kq = (int64_t)t * nk1 + kb;
         const int slot = (int)(kq & 1);
-        if (kq >= 2 && !mbar_wait(&a_empty[slot], (uint32_t)(((kq - 2) >> 1) & 1))) { ok = false; break; }
-        uint8_t* dst = AR + (size_t)slot * kTileM * 128;
         const int colb = 64 * kb + 32 * wk;
-        // all loads of the block first: none waits behind this block's stores
-        float4 bq[8];
+        float4 bq[8];  // bias of the 32 columns (shared memory), in flight during the TMEM load
 #pragma unroll
-        for (int j4 = 0; j4 < 8; ++j4) bq[j4] = ldg4(b1 + colb + 4 * j4);
+        for (int j4 = 0; j4 < 8; ++j4) bq[j4] = *reinterpret_cast<const float4*>(sb1 + colb + 4 * j4);
         uint32_t v[2][16];
         tmem_ld16(D1 + lane_addr + (uint32_t)colb, v[0]);
         tmem_ld16(D1 + lane_addr + (uint32_t)(colb + 16), v[1]);
         tmem_wait_ld();
+        if (kq >= 2 && !mbar_wait(&a_empty[slot], (uint32_t)(((kq - 2) >> 1) & 1))) { ok = false; break; }
+        uint8_t* dst = AR + (size_t)slot * kTileM * 128;
 #pragma unroll
         for (int g = 0; g < 2; ++g) {
           uint32_t pk[8];
@@ -505,35 +522,41 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc_pipe(const __grid_co
       __syncwarp();
       if (lane == 0) mbar_arrive(d1_empty);
       if (!ok) { *abort_flag = 1; latch_error(a.err, LS_ERR_TIMEOUT); break; }
-      // layer-2 epilogue: bias, ReLU, bf16, dot with the output weights
+      if (*abort_flag) break;
+    }
+  } else {
+    // ------------------------------------------------------------ E2: layer-2 epilogue + output layer
+    const int ew = warp - kE2Warp0;        // 0..7
+    const int q4 = warp & 3;
+    const int wk = ew >> 2;                // column half of D2
+    const int row = 32 * q4 + lane;
+    const uint32_t lane_addr = (uint32_t)(32 * q4) << 16;
+    const float b3 = __ldg(params + p.b_last_off);
+    const int half = H2 / 2;
+    for (int t = 0; t < my_tiles; ++t) {
+      const int64_t row0 = (int64_t)(blockIdx.x + (int64_t)t * gridDim.x) * kTileM;
       const bool ok2 = mbar_wait(d2_full, (uint32_t)(t & 1));
       tc_fence_after();
       uint64_t acc2 = 0;
-      const int half = H2 / 2;
-      for (int c0 = wk * half; ok2 && c0 < (wk + 1) * half; c0 += 32) {
-        float4 bq[8], wq[8];  // loaded before the TMEM wait
+      for (int c0 = wk * half; ok2 && c0 < (wk + 1) * half; c0 += 16) {
+        float4 bq[4], wq[4];  // shared memory, in flight during the TMEM load
 #pragma unroll
-        for (int j4 = 0; j4 < 8; ++j4) {
-          bq[j4] = ldg4(b2 + c0 + 4 * j4);
-          wq[j4] = ldg4(w3 + c0 + 4 * j4);
+        for (int j4 = 0; j4 < 4; ++j4) {
+          bq[j4] = *reinterpret_cast<const float4*>(sb2 + c0 + 4 * j4);
+          wq[j4] = *reinterpret_cast<const float4*>(sw3 + c0 + 4 * j4);
         }
-        uint32_t v[2][16];
-        tmem_ld16(D2 + lane_addr + (uint32_t)c0, v[0]);
-        tmem_ld16(D2 + lane_addr + (uint32_t)(c0 + 16), v[1]);
+        uint32_t v[16];
+        tmem_ld16(D2 + lane_addr + (uint32_t)c0, v);
         tmem_wait_ld();
 #pragma unroll
-        for (int g = 0; g < 2; ++g) {
-#pragma unroll
-          for (int j4 = 0; j4 < 4; ++j4) {
-            const float4 b = bq[4 * g + j4];
-            const float4 w = wq[4 * g + j4];
-            const uint32_t h0 = relu_bf16x2(cvt_bf16x2(add_f32x2(((uint64_t)v[g][4 * j4 + 1] << 32) | v[g][4 * j4],
-                                                                   f2pack(b.x, b.y))));
-            const uint32_t h1 = relu_bf16x2(cvt_bf16x2(
-                add_f32x2(((uint64_t)v[g][4 * j4 + 3] << 32) | v[g][4 * j4 + 2], f2pack(b.z, b.w))));
-            acc2 = fma_f32x2(bf16x2_to_f32x2(h0), f2pack(w.x, w.y), acc2);
-            acc2 = fma_f32x2(bf16x2_to_f32x2(h1), f2pack(w.z, w.w), acc2);
-          }
+        for (int j4 = 0; j4 < 4; ++j4) {
+          const float4 b = bq[j4], w = wq[j4];
+          const uint32_t h0 =
+              relu_bf16x2(cvt_bf16x2(add_f32x2(((uint64_t)v[4 * j4 + 1] << 32) | v[4 * j4], f2pack(b.x, b.y))));
+          const uint32_t h1 =
+              relu_bf16x2(cvt_bf16x2(add_f32x2(((uint64_t)v[4 * j4 + 3] << 32) | v[4 * j4 + 2], f2pack(b.z, b.w))));
+          acc2 = fma_f32x2(bf16x2_to_f32x2(h0), f2pack(w.x, w.y), acc2);
+          acc2 = fma_f32x2(bf16x2_to_f32x2(h1), f2pack(w.z, w.w), acc2);
         }
       }
       tc_fence_before();
@@ -541,7 +564,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc_pipe(const __grid_co
       if (lane == 0) mbar_arrive(d2_empty);
       float* pt = part + (t & 1) * kTileM;  // double-buffered by tile parity
       if (wk == 1) pt[row] = __uint_as_float((uint32_t)acc2) + __uint_as_float((uint32_t)(acc2 >> 32));
-      // all epilogue warps continue, or all stop (a timeout here or elsewhere)
+      // all E2 warps continue, or all stop (a timeout here or elsewhere)
       if (!named_bar_and(1, kEpiThreads, ok2 && !*reinterpret_cast<volatile int*>(abort_flag))) {
         *abort_flag = 1;
         latch_error(a.err, LS_ERR_TIMEOUT);
@@ -597,6 +620,92 @@ __global__ void k_norm_rows(const int64_t* __restrict__ tok_off, const int32_t* 
       pairx[g] = make_uint4(f[0] | ((uint32_t)f[1] << 16), f[2] | ((uint32_t)f[3] << 16),
                             f[4] | ((uint32_t)f[5] << 16), 0u);
     }
+  }
+}
+
+// Instance template rows (computed when the snapshot or the normaliser
+// changes): row i holds the z-scored instance features of instance i, bf16,
+// at their feature positions 6 .. 6+d_inst, zeros elsewhere (Algorithm 4
+// Normalize).
+__global__ void k_inst_templates(int n_inst, int d_inst, const float* __restrict__ inst,
+                                 const float* __restrict__ mean, const float* __restrict__ stdv, int d_pad,
+                                 uint16_t* __restrict__ xin) {
+  const int n = n_inst * d_pad;
+  for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < n; e += gridDim.x * blockDim.x) {
+    const int i = e / d_pad, k = e - i * d_pad - kPair;
+    xin[e] = (k >= 0 && k < d_inst)
+                 ? bf16_bits(zscore(inst[(int64_t)i * d_inst + k], mean[kPair + k], stdv[kPair + k]))
+                 : (uint16_t)0;
+  }
+}
+
+// Feature image for the pipelined scorer: row g = r * n_inst + i of the batch
+// as its bf16 feature row [pair(6) || inst || req || 0-pad] (Sec. 4.1
+// Features; Algorithm 4 Normalize), tile t of 128 rows at t * xbytes in the
+// 128-byte-swizzled K-major layout of the MMA operand, rows past the batch
+// zero.  One CTA per tile: it forms the request template rows of the requests
+// it touches and the pair-feature chunk of each row in shared memory; a
+// 16-byte chunk of a feature row is then the OR of an instance-template chunk
+// (computed with the snapshot), a request-template chunk and, for chunk 0,
+// the pair chunk.  Values are bit-identical to the template path.
+__global__ void __launch_bounds__(256) k_feature_image(const int64_t* __restrict__ tok_off,
+                                                       const int32_t* __restrict__ hits, int n_inst,
+                                                       const uint16_t* __restrict__ xin, int d_inst, int d_req,
+                                                       const float* __restrict__ req, const float* __restrict__ mean,
+                                                       const float* __restrict__ stdv, int d_pad, int64_t rows,
+                                                       int64_t n_tiles, int nr_max, uint8_t* __restrict__ ximg) {
+  extern __shared__ uint4 fz4[];
+  uint4* zr = fz4;                                     // [nr_max][d_pad / 8] request template chunks
+  __shared__ uint4 zp[kTileM];                         // pair chunk of each row
+  __shared__ int row_i[kTileM];                        // instance of each tile row
+  __shared__ int row_q[kTileM];                        // its request, relative to the tile's first
+  const int cpr = d_pad / 8;
+  const int64_t xbytes = (int64_t)kTileM * d_pad * 2;
+  for (int64_t t = blockIdx.x; t < n_tiles; t += gridDim.x) {
+    const int64_t g0 = t * kTileM;
+    const int nrow = (int)(g0 + kTileM < rows ? kTileM : rows - g0);
+    const int64_t r_lo = g0 / n_inst;
+    const int i0 = (int)(g0 - r_lo * n_inst);
+    if (threadIdx.x < kTileM) {
+      const int m = threadIdx.x, q = (i0 + m) / n_inst;
+      row_q[m] = q;
+      row_i[m] = i0 + m - q * n_inst;
+      uint16_t f[kPair];
+#pragma unroll
+      for (int k = 0; k < kPair; ++k) f[k] = 0;
+      if (m < nrow) {
+        const int64_t r = r_lo + q;
+        const int64_t L = __ldg(tok_off + r + 1) - __ldg(tok_off + r);
+        const int h = __ldg(hits + g0 + m);
+#pragma unroll
+        for (int k = 0; k < kPair; ++k)
+          f[k] = bf16_bits(zscore(raw_feature(k, L, h, nullptr, 0, nullptr), __ldg(mean + k), __ldg(stdv + k)));
+      }
+      zp[m] = make_uint4(f[0] | ((uint32_t)f[1] << 16), f[2] | ((uint32_t)f[3] << 16), f[4] | ((uint32_t)f[5] << 16),
+                         0u);
+    }
+    const int q_last = (i0 + nrow - 1) / n_inst;  // requests r_lo .. r_lo + q_last
+    uint16_t* zr16 = reinterpret_cast<uint16_t*>(zr);
+    for (int e = threadIdx.x; e < (q_last + 1) * d_pad; e += blockDim.x) {
+      const int rl = e / d_pad, k = e - rl * d_pad - kPair - d_inst;
+      zr16[e] = (k >= 0 && k < d_req) ? bf16_bits(zscore(__ldg(req + (r_lo + rl) * d_req + k),
+                                                         __ldg(mean + kPair + d_inst + k),
+                                                         __ldg(stdv + kPair + d_inst + k)))
+                                      : (uint16_t)0;
+    }
+    __syncthreads();
+    for (int e = threadIdx.x; e < kTileM * cpr; e += blockDim.x) {
+      const int m = e / cpr, c = e - m * cpr;
+      uint4 v = make_uint4(0u, 0u, 0u, 0u);
+      if (m < nrow) {
+        const uint4 ti = __ldg(reinterpret_cast<const uint4*>(xin + (int64_t)row_i[m] * d_pad) + c);
+        const uint4 tq = zr[row_q[m] * cpr + c];
+        const uint4 tp = c == 0 ? zp[m] : make_uint4(0u, 0u, 0u, 0u);
+        v = make_uint4(ti.x | tq.x | tp.x, ti.y | tq.y | tp.y, ti.z | tq.z | tp.z, ti.w | tq.w | tp.w);
+      }
+      *reinterpret_cast<uint4*>(ximg + t * xbytes + sw128_offset(m, 8 * c, kTileM)) = v;
+    }
+    __syncthreads();
   }
 }
 
@@ -657,8 +766,8 @@ bool plan_tc(const MlpDesc& m, TcPlan& p) {
   // pipelined variant: two hidden layers of <= 256, all weights resident
   p.pipe = 0;
   if (p.n_tc == 2 && p.out[0] <= 256 && p.out[1] <= 256 && p.nc[0] == p.out[0] && p.nc[1] == p.out[1]) {
-    const int64_t need = 1024 + (int64_t)p.chunks * cb + 2 * (int64_t)p.d_pad * kTileM * 2 + 2 * kTileM * 128 +
-                         2 * kTileM * 4 + 13 * 8 + 16;
+    const int64_t need = 1024 + (int64_t)p.chunks * cb + kXB * (int64_t)p.d_pad * kTileM * 2 + 2 * kTileM * 128 +
+                         2 * kTileM * 4 + 3 * 256 * 4 + 13 * 8 + 16;
     if (need <= kMaxSmem) {
       p.pipe = 1;
       p.pipe_smem = (int)need;
@@ -678,8 +787,35 @@ cudaError_t launch_norm_rows(const int64_t* tok_off, const int32_t* hits, uint4*
   return cudaGetLastError();
 }
 
+cudaError_t launch_inst_templates(int n_inst, int d_inst, const float* inst, const float* mean, const float* stdv,
+                                  int d_pad, uint16_t* xin, int sms, cudaStream_t s) {
+  const int n = n_inst * d_pad;
+  if (n <= 0) return cudaSuccess;
+  const int grid = std::min((n + 255) / 256, sms * 4);
+  k_inst_templates<<<grid, 256, 0, s>>>(n_inst, d_inst, inst, mean, stdv, d_pad, xin);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_feature_image(const int64_t* tok_off, const int32_t* hits, int n_inst, const uint16_t* xin,
+                                 int d_inst, int n_req, int d_req, const float* req, const float* mean,
+                                 const float* stdv, int d_pad, uint8_t* ximg, int sms, cudaStream_t s) {
+  const int64_t rows = (int64_t)n_req * n_inst;
+  if (rows <= 0) return cudaSuccess;
+  const int64_t n_tiles = (rows + kTileM - 1) / kTileM;
+  const int nr_max = (kTileM + n_inst - 1) / n_inst + 1;  // requests a tile can touch
+  const size_t smem = (size_t)nr_max * d_pad * sizeof(uint16_t);
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(k_feature_image, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+  }
+  const int grid = (int)std::min<int64_t>(n_tiles, (int64_t)sms * 8);
+  k_feature_image<<<grid, 256, smem, s>>>(tok_off, hits, n_inst, xin, d_inst, d_req, req, mean, stdv, d_pad, rows,
+                                          n_tiles, nr_max, ximg);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const Published* pub, const int32_t* sel,
-                            int n_req, int n_inst, const uint4* pairx,
+                            int n_req, int n_inst, const uint4* pairx, const uint8_t* ximg,
                             const uint16_t* xin, const uint16_t* xrq, int d_inst, int d_req, const float* mean,
                             const float* stdv, float* scores, int* err, int sms, cudaStream_t s) {
   const int64_t rows = (int64_t)n_req * n_inst;
@@ -699,6 +835,7 @@ cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const Published* 
   a.d_inst = d_inst;
   a.d_req = d_req;
   a.pairx = pairx;
+  a.ximg = ximg;
   a.xin = xin;
   a.xrq = xrq;
   a.mean = mean;
@@ -711,7 +848,7 @@ cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const Published* 
   if (p.pipe) {
     cudaError_t e = cudaFuncSetAttribute(k_score_tc_pipe, cudaFuncAttributeMaxDynamicSharedMemorySize, p.pipe_smem);
     if (e != cudaSuccess) return e;
-    k_score_tc_pipe<<<grid, kThreadsTc, p.pipe_smem, s>>>(a);
+    k_score_tc_pipe<<<grid, kThreadsPipe, p.pipe_smem, s>>>(a);
   } else {
     cudaError_t e = cudaFuncSetAttribute(k_score_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, p.smem);
     if (e != cudaSuccess) return e;

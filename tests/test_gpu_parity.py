@@ -234,6 +234,27 @@ def test_tensor_core_scorer_matches_cuda_core_scorer(name):
     r2.close()
 
 
+@pytest.mark.parametrize("n_inst", [24, 200])
+def test_pipelined_scorer_with_tiles_across_requests(n_inst):
+    # instance counts that do not divide the 128-row tile (tiles span request
+    # boundaries), and more instances than rows in a tile
+    import dataclasses
+    cfg = dataclasses.replace(W.CONFIGS["homogeneous"], n_inst=n_inst, n_req=64, cache_blocks=1024,
+                              n_samples=0)
+    wl = W.generate(cfg)
+    r = H.Router.for_config(cfg)
+    dw = H.DeviceWorkload(wl)
+    dw.load(r)
+    assert r.info().scorer == L.LS_SCORER_TENSOR_CORES
+    out = r.route(dw.tok, dw.tok_off, dw.req_feats, n_inst)
+    ref = oracle.route(wl)
+    assert np.array_equal(out["hits"].cpu().numpy(), ref["hits"])
+    sg = out["scores"].cpu().numpy()
+    assert_scores_close(sg, ref["scores"], TOL["bf16"])
+    assert_choices(out["choice"].cpu().numpy(), sg, ref["scores"], TOL["bf16"])
+    r.close()
+
+
 def test_optional_outputs_do_not_change_the_result():
     wl, dw, r = staged("homogeneous")
     full = r.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)
