@@ -470,7 +470,8 @@ int ls_route_batch(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* 
   if (weight_version_out) *weight_version_out = v;
   if (n_req == 0) return LS_OK;
   int32_t* hits = hits_opt ? hits_opt : c.hits;
-  float* scores = scores_opt ? scores_opt : c.scores;
+  const bool fused_select = c.use_tc && scorer_selects(c.tc, c.n_inst);
+  float* scores = scores_opt ? scores_opt : (fused_select ? nullptr : c.scores);
   if (c.use_index) {
     LS_CK(traced(c, TR_PREFIX_INDEX, 1, s, [&] {
       return launch_prefix_index(n_req, tok, tok_off, c.gkeys, c.gmask, c.gW, (uint64_t)(c.gslots - 1), c.n_inst,
@@ -502,6 +503,7 @@ int ls_route_batch(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* 
     }));
     LS_CK(traced(c, TR_SCORE_TC, 1, s, [&] {
       return launch_score_tc(c.mlp, c.tc, c.pub, &c.st->route_b, n_req, c.n_inst, c.pairx, c.ximg,
+                             fused_select ? choice : nullptr, fused_select ? best : nullptr,
                              c.xin, c.xrq, c.cfg.d_inst, c.cfg.d_req, c.mean, c.stdv, scores, c.d_err, c.sms,
                              s);
     }));
@@ -511,7 +513,8 @@ int ls_route_batch(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* 
                                c.cfg.d_inst, req_feats, c.cfg.d_req, c.mean, c.stdv, scores, s);
     }));
   }
-  LS_CK(traced(c, TR_ARGMIN, 1, s, [&] { return launch_argmin(n_req, c.n_inst, scores, choice, best, s); }));
+  if (!fused_select)
+    LS_CK(traced(c, TR_ARGMIN, 1, s, [&] { return launch_argmin(n_req, c.n_inst, scores, choice, best, s); }));
   if (!cap) {
     std::lock_guard<std::mutex> g(c.mu);
     LS_CK(cudaEventRecord(c.ev_route, s));

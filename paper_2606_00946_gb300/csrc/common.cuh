@@ -356,8 +356,12 @@ cudaError_t launch_inst_templates(int n_inst, int d_inst, const float* inst, con
 cudaError_t launch_feature_image(const int64_t* tok_off, const int32_t* hits, int n_inst, const uint16_t* xin,
                                  int d_inst, int n_req, int d_req, const float* req, const float* mean,
                                  const float* stdv, int d_pad, uint8_t* ximg, int sms, cudaStream_t s);
+// With the pipelined kernel and n_inst dividing 32 the selector runs inside the
+// scorer (choice/best written, scores only when non-NULL); see scorer_selects().
+inline bool scorer_selects(const TcPlan& p, int n_inst) { return p.pipe && n_inst <= 32 && 32 % n_inst == 0; }
 cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const Published* pub, const int32_t* sel,
-                            int n_req, int n_inst, const uint4* pairx, const uint8_t* ximg,
+                            int n_req, int n_inst, const uint4* pairx, const uint8_t* ximg, int32_t* choice,
+                            float* best,
                             const uint16_t* xin, const uint16_t* xrq, int d_inst, int d_req,
                             const float* mean, const float* stdv, float* scores, int* err, int sms,
                             cudaStream_t s);

@@ -39,6 +39,9 @@ struct TcArgs {
   int n_req, n_inst, d, d_inst, d_req;
   const uint4* pairx;    // [rows] bf16 pair features (chunk 0 of each feature row, zeros past column 5)
   const uint8_t* ximg;   // pipelined kernel: feature tiles, tile t = xbytes at t * xbytes, in the MMA layout
+  int32_t* choice;       // pipelined kernel with n_inst dividing 32: the selector runs in the epilogue
+  float* best;
+  int fuse_argmin;
   const uint16_t* xin;   // [n_inst, d_pad] bf16 instance template rows (zero outside inst columns)
   const uint16_t* xrq;   // [n_req, d_pad]  bf16 request template rows (zero outside req columns)
   const float* mean;
@@ -573,7 +576,28 @@ __global__ void __launch_bounds__(kThreadsPipe, 1) k_score_tc_pipe(const __grid_
       if (wk == 0) {
         const int64_t g = row0 + row;
         const float mine = __uint_as_float((uint32_t)acc2) + __uint_as_float((uint32_t)(acc2 >> 32));
-        if (g < a.rows) a.scores[g] = (mine + pt[row]) + b3;
+        const float yhat = (mine + pt[row]) + b3;
+        if (g < a.rows && a.scores) a.scores[g] = yhat;
+        if (a.fuse_argmin) {
+          // n_inst divides 32 and tiles start at request boundaries: the
+          // request's scores sit in n_inst consecutive lanes; lexicographic
+          // (score, index) minimum, NaN last (Algorithm 4, greedy selection)
+          const int n = a.n_inst;
+          float bv = yhat;
+          int bi = g < a.rows ? (lane & (n - 1)) : -1;
+          for (int o = 1; o < n; o <<= 1) {
+            const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+            const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+            const bool an = isnan(ov), bn = isnan(bv);
+            const bool first = an != bn ? bn : (!an && ov != bv ? ov < bv : oi < bi);
+            if (oi >= 0 && (bi < 0 || first)) { bv = ov; bi = oi; }
+          }
+          if ((lane & (n - 1)) == 0 && g < a.rows) {
+            const int64_t r = g / n;
+            a.choice[r] = bi;
+            a.best[r] = bv;
+          }
+        }
       }
     }
   }
@@ -815,7 +839,8 @@ cudaError_t launch_feature_image(const int64_t* tok_off, const int32_t* hits, in
 }
 
 cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const Published* pub, const int32_t* sel,
-                            int n_req, int n_inst, const uint4* pairx, const uint8_t* ximg,
+                            int n_req, int n_inst, const uint4* pairx, const uint8_t* ximg, int32_t* choice,
+                            float* best,
                             const uint16_t* xin, const uint16_t* xrq, int d_inst, int d_req, const float* mean,
                             const float* stdv, float* scores, int* err, int sms, cudaStream_t s) {
   const int64_t rows = (int64_t)n_req * n_inst;
@@ -836,6 +861,9 @@ cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const Published* 
   a.d_req = d_req;
   a.pairx = pairx;
   a.ximg = ximg;
+  a.choice = choice;
+  a.best = best;
+  a.fuse_argmin = (p.pipe && choice && best && n_inst <= 32 && 32 % n_inst == 0) ? 1 : 0;
   a.xin = xin;
   a.xrq = xrq;
   a.mean = mean;
