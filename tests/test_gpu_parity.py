@@ -501,7 +501,8 @@ def test_table_full_and_bad_slot_are_latched():
 # a whole step captured in a CUDA graph; tracing
 # ----------------------------------------------------------------------------
 
-def test_graph_replay_matches_eager_steps():
+@pytest.mark.parametrize("branches", [1, 2])
+def test_graph_replay_matches_eager_steps(branches):
     # Two contexts fed the same inputs: one issues snapshot/route/log/train/
     # publish eagerly every step, the other replays one captured graph.  The
     # device counters make each replay a new step, so routes, losses, weights
@@ -534,11 +535,19 @@ def test_graph_replay_matches_eager_steps():
             bufs["x"].copy_(sx[a:a + Bt])
             bufs["y"].copy_(sy[a:a + Bt])
 
+        side = torch.cuda.Stream()
+
         def body():
+            # branches == 2: log + train on a second stream beside the route,
+            # joined before the publish
+            main = torch.cuda.current_stream()
+            side.wait_stream(main)
             r.snapshot(N, bufs["state"])
             r.route(dw.tok, dw.tok_off, dw.req_feats, N, out=bufs["out"])
-            r.log(bufs["x"], bufs["y"])
-            r.train(Bt, None, opt="adam", lr=1e-3, loss_out=bufs["loss"])
+            with torch.cuda.stream(side if branches == 2 else main):
+                r.log(bufs["x"], bufs["y"])
+                r.train(Bt, None, opt="adam", lr=1e-3, loss_out=bufs["loss"])
+            main.wait_stream(side)
             r.publish()
         return bufs, feed, body
 
