@@ -72,6 +72,11 @@ def lib():
             L.or_train_step.argtypes = [C.c_int, C.c_int, P, P, P, P, i64, C.c_int, dbl,
                                         C.c_int, P, P, P, P, P, P, P]
             L.or_loss.argtypes = [C.c_int, C.c_int, P, P, C.c_int, P, P, P, P, P, P]
+            L.or_ring_bounds.argtypes = [i64, C.c_int, P, i64, P, P]
+            L.or_hrw_candidates.restype = i32
+            L.or_hrw_candidates.argtypes = [C.c_uint64, i32, i32, P]
+            L.or_guards.argtypes = [i64, i32, P, P, P, P, C.c_int, P, C.c_int, P, P, P, i64, i64,
+                                    C.c_int, i32, i32, C.c_float, C.c_float, P, P, P]
             _lib = L
     return _lib
 
@@ -288,3 +293,62 @@ def loss(mode, widths, params, ring_x, ring_y, idx, mean, std) -> float:
                          _p(idx), _p(_c(mean, np.float32)), _p(_c(std, np.float32)), _p(out)),
            "loss")
     return float(out[0])
+
+
+# --------------------------------------------------------------------------
+# Algorithm 4 guards
+# --------------------------------------------------------------------------
+
+ROUTE_OK, ROUTE_COLD_START, ROUTE_OOD, ROUTE_KFILTER = 0, 1, 2, 4
+
+
+def ring_bounds(ring_x, count):
+    """Per-feature [lo, hi] over the records the ring holds (NaN skipped)."""
+    rx = _c(ring_x, np.float32)
+    cap, d = rx.shape
+    lo = np.zeros(d, np.float32)
+    hi = np.zeros(d, np.float32)
+    _check(lib().or_ring_bounds(cap, d, _p(rx), int(count), _p(lo), _p(hi)), "ring_bounds")
+    return lo, hi
+
+
+def hrw_candidates(gkey: int, n_inst: int, K: int) -> np.ndarray:
+    """ConsistentHash_K of one prefix-group key, in rank order."""
+    out = np.zeros(max(K, 1), np.int32)
+    m = lib().or_hrw_candidates(C.c_uint64(gkey & (2**64 - 1)), n_inst, K, _p(out))
+    return out[:m]
+
+
+def group_keys(tok, tok_off) -> np.ndarray:
+    """Prefix-group key of every prompt: the key of its first full block
+    (0 where the prompt has none)."""
+    keys, ko = hash_blocks(tok, tok_off)
+    L = np.diff(np.asarray(tok_off, np.int64))
+    g = np.zeros(len(L), np.uint64)
+    has = L >= BLOCK
+    g[has] = keys[ko[:-1][has]]
+    return g
+
+
+def guards(L, gkey, hits, inst_state, req_feats, scores, lo, hi, n, *, n_min=0, ood=False,
+           k=0, kv_col=4, tau_sat=0.8, tau_ben=0.0):
+    """Guarded selection of Algorithm 4 over given scores.
+    Returns (choice int32 [R], best f32 [R], status int32 [R])."""
+    L = _c(L, np.int64)
+    gkey = _c(gkey, np.uint64)
+    hits = _c(hits, np.int32)
+    s = _c(scores, np.float32)
+    inst = _c(inst_state, np.float32)
+    req = _c(req_feats, np.float32)
+    R, N = s.shape
+    d_inst, d_req = inst.shape[1], (req.shape[1] if req.ndim == 2 else 0)
+    choice = np.zeros(R, np.int32)
+    best = np.zeros(R, np.float32)
+    status = np.zeros(R, np.int32)
+    one = np.zeros(1, np.float32)
+    _check(lib().or_guards(R, N, _p(L), _p(gkey), _p(hits), _p(inst if inst.size else one), d_inst,
+                           _p(req if req.size else one), d_req, _p(s), _p(_c(lo, np.float32)),
+                           _p(_c(hi, np.float32)), int(n), int(n_min), int(bool(ood)), int(k),
+                           int(kv_col), float(tau_sat), float(tau_ben), _p(choice), _p(best),
+                           _p(status)), "guards")
+    return choice, best, status

@@ -21,6 +21,9 @@
  *   Algorithm 4: per-feature z-score normalisation, batched forward, argmax.
  *   Sec. 4.3.2 (Online learning): periodic retraining on logged
  *          (features, TTFT) records; FIFO buffer of recent samples.
+ *   Sec. 4.3.1 (Fallback) and Algorithm 4: cold-start and out-of-range
+ *          guards; Sec. 4.1 (Consistent hashing based filtering): the
+ *          K-filter of Algorithm 4.
  *
  * Readings where the paper is silent (each also listed in the design notes):
  *   - block hash: SplitMix64 finaliser based content hash, prefix state chained
@@ -31,7 +34,11 @@
  *     defaults beta1 = 0.9, beta2 = 0.999, eps = 1e-8);
  *   - bf16 mode: weights, layer-1 input and hidden activations rounded to
  *     bf16 (round to nearest even); biases and accumulation stay wide;
- *   - argmin ties -> lowest index, -0 == +0, NaN after every number.
+ *   - argmin ties -> lowest index, -0 == +0, NaN after every number;
+ *   - guards: n = records ever appended; bounds = NaN-skipping min / max over
+ *     the records the ring holds; prefix group = key of the first full block;
+ *     ConsistentHash_K = top-K rendezvous hashing; gpu_kv mean in fp64 in
+ *     index order; kappa_i |r| = 16 h_i; epsilon = 0, no random tiebreak.
  */
 #include <math.h>
 #include <stdint.h>
@@ -475,5 +482,136 @@ int or_loss(int mode, int n_layers, const int *w, const double *params, int batc
     }
     *loss_out = loss / (double)batch;
     free(ba); free(bb); free(xr); free(xf);
+    return 0;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Algorithm 4 guards (Sec. 4.3.1 fallback; Sec. 4.1 consistent hashing)    */
+/* ------------------------------------------------------------------------ */
+
+/* Feature bounds [l_j, u_j] of the training buffer (Algorithm 4 input; the
+ * fallback paragraph of Sec. 4.3.1: the ranges observed in the buffer).  The
+ * buffer is the sample ring: its first min(count, capacity) slots hold the
+ * records it keeps.  l_j / u_j = smallest / largest value of column j over
+ * those rows, NaN values skipped; a column with no number keeps the empty
+ * range l = +inf, u = -inf. */
+int or_ring_bounds(int64_t capacity, int d, const float *ring_x, int64_t count,
+                   float *lo, float *hi) {
+    int64_t rows = count < capacity ? count : capacity;
+    for (int j = 0; j < d; ++j) {
+        lo[j] = INFINITY;
+        hi[j] = -INFINITY;
+    }
+    for (int64_t r = 0; r < rows; ++r)
+        for (int j = 0; j < d; ++j) {
+            float v = ring_x[r * d + j];
+            if (isnan(v)) continue;
+            if (v < lo[j]) lo[j] = v;
+            if (v > hi[j]) hi[j] = v;
+        }
+    return 0;
+}
+
+/* Rendezvous weight of instance i for prefix-group key g. */
+static uint64_t hrw_weight(uint64_t g, int32_t i) {
+    return or_mix64(g ^ or_mix64((uint64_t)(i + 1) * OR_G));
+}
+
+/* (w_a, a) ranks before (w_b, b): larger weight first, then lower index. */
+static int hrw_before(uint64_t wa, int32_t a, uint64_t wb, int32_t b) {
+    if (wa != wb) return wa > wb;
+    return a < b;
+}
+
+/* ConsistentHash_K (Algorithm 4; Sec. 4.1 "Consistent hashing based
+ * filtering"): the K instances with the largest rendezvous weights for key g
+ * (highest-random-weight hashing), in rank order.  Writes min(K, n_inst)
+ * indices to cand and returns that count.  Selection sort: pass k takes the
+ * best instance not yet taken. */
+int32_t or_hrw_candidates(uint64_t g, int32_t n_inst, int32_t K, int32_t *cand) {
+    int32_t m = K < n_inst ? K : n_inst;
+    for (int32_t k = 0; k < m; ++k) {
+        int32_t b = -1;
+        for (int32_t i = 0; i < n_inst; ++i) {
+            int taken = 0;
+            for (int32_t q = 0; q < k; ++q) taken |= cand[q] == i;
+            if (taken) continue;
+            if (b < 0 || hrw_before(hrw_weight(g, i), i, hrw_weight(g, b), b)) b = i;
+        }
+        cand[k] = b;
+    }
+    return m < 0 ? 0 : m;
+}
+
+/* Guarded selection of Algorithm 4, given the predicted TTFT of every pair.
+ *   status 1 (cold start): n < n_min                       -> choice -1, best NaN
+ *   status 2 (OOD)       : ood_on and some raw feature of some pair of the
+ *                          request lies outside [lo, hi] (NaN counts as
+ *                          outside)                         -> choice -1, best NaN
+ *   otherwise status 0 and choice = argmin over instances (= argmax of the
+ *   reward -TTFT; order of or_argmin), then the K-filter: when K >= 1, the
+ *   prompt has a full block (its group key gkey[r] is the key of block 0),
+ *     mean_i inst[i, kv_col] > tau_sat   (fp64 sum in index order, / N) and
+ *     max_i 16 h_i > tau_ben             (kappa_i |r| = 16 h_i hit tokens),
+ *   status gains bit 4 and a choice outside the candidates is replaced by the
+ *   argmin over the candidates.  best = scores of the final choice.
+ * Cold start is tested before OOD (Algorithm 4 order).  Exploration and the
+ * random tiebreak are not taken (epsilon = 0; equal scores go to the lowest
+ * index). */
+int or_guards(int64_t n_req, int32_t n_inst, const int64_t *L, const uint64_t *gkey,
+              const int32_t *hits, const float *inst, int d_inst, const float *req, int d_req,
+              const float *scores, const float *lo, const float *hi, int64_t n, int64_t n_min,
+              int ood_on, int32_t K, int32_t kv_col, float tau_sat, float tau_ben,
+              int32_t *choice, float *best, int32_t *status) {
+    int d = 6 + d_inst + d_req;
+    float *x = (float *)malloc((size_t)d * sizeof(float));
+    int32_t *cand = (int32_t *)malloc((size_t)(K > 0 ? K : 1) * sizeof(int32_t));
+    if (!x || !cand) { free(x); free(cand); return -1; }
+    double kv_sum = 0.0;
+    if (K >= 1 && kv_col >= 0 && kv_col < d_inst)
+        for (int32_t i = 0; i < n_inst; ++i) kv_sum += (double)inst[(int64_t)i * d_inst + kv_col];
+    double kv_mean = kv_sum / (double)n_inst;
+    for (int64_t r = 0; r < n_req; ++r) {
+        const float *sr = scores + r * n_inst;
+        const int32_t *hr = hits + r * n_inst;
+        if (n < n_min) {
+            choice[r] = -1; best[r] = NAN; status[r] = 1;
+            continue;
+        }
+        if (ood_on) {
+            int out = 0;
+            for (int32_t i = 0; i < n_inst && !out; ++i) {
+                or_raw_features_row(L[r], hr[i], inst + (int64_t)i * d_inst, d_inst,
+                                    req + r * d_req, d_req, x);
+                for (int j = 0; j < d; ++j)
+                    if (!(x[j] >= lo[j] && x[j] <= hi[j])) { out = 1; break; }
+            }
+            if (out) {
+                choice[r] = -1; best[r] = NAN; status[r] = 2;
+                continue;
+            }
+        }
+        int32_t c = 0;
+        for (int32_t i = 1; i < n_inst; ++i)
+            if (precedes(sr[i], i, sr[c], c)) c = i;
+        int32_t st = 0;
+        if (K >= 1 && L[r] >= OR_BLOCK && kv_col >= 0 && kv_col < d_inst) {
+            int32_t hmax = 0;
+            for (int32_t i = 0; i < n_inst; ++i) if (hr[i] > hmax) hmax = hr[i];
+            if (kv_mean > (double)tau_sat && 16.0 * (double)hmax > (double)tau_ben) {
+                int32_t m = or_hrw_candidates(gkey[r], n_inst, K, cand);
+                int in = 0;
+                for (int32_t q = 0; q < m; ++q) in |= cand[q] == c;
+                if (!in) {
+                    c = cand[0];
+                    for (int32_t q = 1; q < m; ++q)
+                        if (precedes(sr[cand[q]], cand[q], sr[c], c)) c = cand[q];
+                }
+                st = 4;
+            }
+        }
+        choice[r] = c; best[r] = sr[c]; status[r] = st;
+    }
+    free(x); free(cand);
     return 0;
 }
