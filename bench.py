@@ -43,8 +43,73 @@ def parse():
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-guards", action="store_true", help="skip the guarded-route measurement")
     p.add_argument("--cpu-seconds", type=float, default=12.0, help="target oracle work for cpu_baseline")
     return p.parse_args()
+
+
+def measure_guards(L, r, dw, N, R, d, ring_rows, d_req, flush, stream, peaks, n=60):
+    """Guarded route of Algorithm 4 (cold start, out-of-range bounds, K-filter
+    with K = 2) on the bench batch, beside the plain route: event-timed route
+    calls (call by call, L2 flushed before each) and per-launch times of the
+    guard kernel and of the ring-bounds reduction."""
+    import torch
+    dev = dw.tok.device
+    o_plain = {"choice": torch.empty(R, dtype=torch.int32, device=dev),
+               "best": torch.empty(R, dtype=torch.float32, device=dev), "scores": None, "hits": None}
+    o_g = dict(o_plain, status=torch.empty(R, dtype=torch.int32, device=dev))
+    r.refresh_bounds()
+    r.publish()
+    # tau_sat = 0 keeps the K-filter on for every request with a hit (the
+    # paper's 0.8 would switch it off on this snapshot: mean KV use ~0.5)
+    r.set_guards(n_min=1, ood=True, k=2, kv_col=4, tau_sat=0.0, tau_ben=0.0)
+
+    def timed(fn):
+        ts = []
+        for k in range(n):
+            flush.fill_(k & 0xFF)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            fn()
+            e1.record(stream)
+            e1.synchronize()
+            ts.append(e0.elapsed_time(e1))
+        return float(np.mean(ts[3:]))
+
+    plain_ms = timed(lambda: r.route(dw.tok, dw.tok_off, dw.req_feats, N, out=o_plain))
+    guarded_ms = timed(lambda: r.route_guarded(dw.tok, dw.tok_off, dw.req_feats, N, out=o_g))
+    L.ls_trace_enable(r.h, True)
+    L.ls_trace_read(r.h)
+    for k in range(n):
+        flush.fill_(k & 0xFF)
+        r.route_guarded(dw.tok, dw.tok_off, dw.req_feats, N, out=o_g)
+        flush.fill_(k & 0xFF)
+        r.refresh_bounds()
+    torch.cuda.synchronize()
+    rc, trace = L.ls_trace_read(r.h)
+    L.ls_trace_enable(r.h, False)
+    r.set_guards()                                   # all guards off again
+    st = o_g["status"].cpu().numpy()
+    agree = bool(torch.equal(o_g["choice"][st == 0], o_plain["choice"][torch.from_numpy(st == 0).to(dev)]))
+    per = {k: v[1] / max(v[2], 1) for k, v in trace.items()}
+    g_bytes = R * N * 8 + R * (16 + 64 + 4 * d_req + 12)
+    b_bytes = ring_rows * d * 4
+    hbm = peaks["hbm_gbs"]
+    g_gbs = g_bytes / 1e9 / (per["guards"] / 1e3)
+    b_gbs = b_bytes / 1e9 / (per["ring_bounds"] / 1e3)
+    return {
+        "route_plain_ms": plain_ms, "route_guarded_ms": guarded_ms,
+        "guards_kernel": {"avg_launch_ms": per["guards"], "bytes_per_launch": g_bytes, "achieved": g_gbs,
+                          "peak": hbm, "unit": "GB/s", "frac": g_gbs / hbm, "bound": "hbm"},
+        "ring_bounds_kernel": {"avg_launch_ms": per["ring_bounds"], "bytes_per_launch": b_bytes,
+                               "achieved": b_gbs, "peak": hbm, "unit": "GB/s", "frac": b_gbs / hbm,
+                               "bound": "hbm", "rows": ring_rows},
+        "status_counts": {"ok": int((st == 0).sum()), "k_filtered": int((st == 4).sum()),
+                          "cold_start": int((st == 1).sum()), "out_of_range": int((st == 2).sum())},
+        "unfiltered_choices_equal_plain_route": agree,
+        "settings": "n_min 1, out-of-range check on, K 2, kv column 4, tau_sat 0, tau_ben 0",
+    }
 
 
 def dist_setup(n_gpus):
@@ -408,6 +473,11 @@ def main():
                 "timing": "kernel durations from CUDA events around each launch over steps issued call by "
                           "call (instrumented); value and ms_per_step from the K graph replays"}
 
+    guards = None
+    if not args.no_guards:
+        guards = measure_guards(L, r, dw, N, R, cfg.d, min(ring, int(r.info().ring_count)), cfg.d_req, flush,
+                                stream, peaks)
+
     # end to end through the C ABI with host buffers
     e2e = None
     if not args.no_e2e:
@@ -517,6 +587,7 @@ def main():
             "gpu_launches_per_step": launches / args.steps,
             "clocks": clk,
             "algorithmic": costs,
+            "guarded_route": guards,
         }
         print(json.dumps(line))
     r.close()

@@ -231,6 +231,69 @@ int ls_train_step(ls_ctx *ctx, int32_t batch, const int32_t *idx, int32_t opt, f
  * started with (each route takes the index once, before it scores). */
 int ls_publish(ls_ctx *ctx, void *stream);
 
+/* ---- Algorithm 4 guards (Sec. 4.3.1 fallback; Sec. 4.1 consistent hashing) ----
+ * Per-request status of a guarded route.  The low bits say whether the
+ * router decided (OK) or hands the request back to the gateway's fallback
+ * heuristic (Algorithm 3) with choice -1 and best NaN:
+ *   LS_ROUTE_COLD_START  fewer than n_min records were ever logged;
+ *   LS_ROUTE_OOD         some raw feature of some (request, instance) pair
+ *                        lies outside the published bounds [lo_j, hi_j]
+ *                        (a NaN feature is outside).
+ * LS_ROUTE_KFILTER is added to OK when the K-filter applied to the request. */
+enum { LS_ROUTE_OK = 0, LS_ROUTE_COLD_START = 1, LS_ROUTE_OOD = 2, LS_ROUTE_KFILTER = 4 };
+
+typedef struct {
+    int64_t n_min;     /* cold start while records logged < n_min (<= 0: off) */
+    int32_t ood;       /* nonzero: out-of-range check against the published bounds */
+    int32_t k;         /* K-filter candidates (0: filter off) */
+    int32_t kv_col;    /* instance-state column holding KV-cache utilisation */
+    float tau_sat;     /* filter when mean_i inst[i, kv_col] > tau_sat ... */
+    float tau_ben;     /* ... and max_i 16 h[r,i] (kappa_i |r|, hit tokens) > tau_ben */
+} ls_guards;
+
+/* Set the guard parameters used by later ls_route_batch_guarded calls (host
+ * state, read when a route is enqueued or captured).  All off after
+ * ls_create.  LS_ERR_ARG for k < 0, k > max_instances, or k > 0 with kv_col
+ * outside [0, d_inst). */
+int ls_set_guards(ls_ctx *ctx, const ls_guards *g /* host */);
+
+/* Feature bounds of the training buffer (Algorithm 4 input [l, u]): one kernel
+ * takes, for every feature column j, the smallest and largest value over the
+ * records the sample ring holds when it runs (its first min(count,
+ * ring_capacity) slots; NaN values skipped; a column without a number gets
+ * the empty range lo = +inf, hi = -inf) into a staging copy.  The next
+ * ls_publish publishes the staged bounds together with the weights, so a
+ * route sees the bounds of the data its weights were trained beside.  Before
+ * the first refresh the staging copy holds the empty range in every column. */
+int ls_refresh_bounds(ls_ctx *ctx, void *stream);
+
+/* Copy bounds to DEVICE lo_out [d], hi_out [d]: which = 0 the staging copy,
+ * 1 the bounds routing reads now (synchronises the device). */
+int ls_get_bounds(ls_ctx *ctx, int32_t which, float *lo_out, float *hi_out, void *stream);
+
+/* ls_route_batch with the guards of Algorithm 4 and a status per request
+ * (DEVICE int32 status [n_req]).  Per request, in order:
+ *   1. cold start: records logged (device count when the route runs) < n_min;
+ *   2. out of range (when ood): any raw feature [L, h, 16h, 16h/L, L-16h,
+ *      ceil(L/16)-h || inst_state[i] || req_feats[r]] of any instance i
+ *      outside [lo, hi] of the bounds published with the weights this route
+ *      reads;
+ *   3. choice = argmin_i yhat[r,i] as in ls_route_batch, then the K-filter
+ *      (when k >= 1 and the prompt has a full block): if the fp64 mean of
+ *      inst_state[:, kv_col] (summed in instance order) exceeds tau_sat and
+ *      16 max_i h[r,i] exceeds tau_ben, the candidates are the k instances
+ *      with the largest rendezvous weights mix64(g ^ mix64((i+1) G)) (ties
+ *      to the lower index), g = key of the prompt's first block (the prefix
+ *      group, as ls_hash_blocks defines keys); a choice outside them is
+ *      replaced by the argmin over them (same order).
+ * Exploration and the random tiebreak of Algorithm 4 are not taken
+ * (epsilon = 0, equal scores go to the lowest index).  Other arguments, the
+ * stream rules and errors are those of ls_route_batch. */
+int ls_route_batch_guarded(ls_ctx *ctx, int32_t n_req, const int32_t *tok, const int64_t *tok_off,
+                           const float *req_feats, int32_t *choice, float *best, int32_t *status,
+                           float *scores_opt, int32_t *hits_opt, uint64_t *weight_version_out,
+                           void *stream);
+
 /* Kernel tracing.  While enabled, each kernel launch of this context is
  * bracketed by CUDA events on its launching stream (a few microseconds of host
  * time per launch; launches recorded into a CUDA graph are not traced).

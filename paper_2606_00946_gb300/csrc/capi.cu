@@ -4,6 +4,7 @@
 #include <cmath>
 #include <cstring>
 #include <string>
+#include <vector>
 
 #include "common.cuh"
 
@@ -15,7 +16,7 @@ const char* const kTraceNames[TR_COUNT] = {
     "ring_append", "publish", "train_gather", "gemm_fwd", "loss_grad", "gemm_dw", "reduce_dw",
     "colsum_db", "gemm_dx", "optimizer", "memset", "score_tc", "features", "publish_tc",
     "hash_screen", "probe_screen", "probe_walk", "gemm_tc_fwd", "gemm_tc_dw", "gemm_tc_dx", "prefix_index",
-    "index_insert"};
+    "index_insert", "guards", "ring_bounds"};
 }
 
 struct ls_ctx {
@@ -108,7 +109,8 @@ void free_all(Ctx& c) {
                   c.adam_v, c.pub[0].params, c.pub[0].wt, c.pub[1].params, c.pub[1].wt,
                   c.ring_x, c.ring_y, c.hits, c.scores, c.tx, c.tz, c.ty, c.dz0, c.dz1, c.grad,
                   c.gpart, c.loss_tmp, c.d_err, c.pub[0].img, c.pub[1].img, c.xin, c.xrq, c.pairx, c.ximg,
-                  c.bkeys, c.work, c.work_n, c.gkeys, c.gmask, c.st, c.tf.base, c.tf.parts};
+                  c.bkeys, c.work, c.work_n, c.gkeys, c.gmask, c.st, c.tf.base, c.tf.parts,
+                  c.pub[0].bounds, c.pub[1].bounds, c.bounds_stage, c.bpart};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   if (c.ev_pub) cudaEventDestroy(c.ev_pub);
@@ -208,7 +210,10 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
     A(dalloc(&c.pub[b].params, c.n_params));
     A(dalloc(&c.pub[b].wt, c.wt_total));
     if (c.use_tc) A(dalloc(&c.pub[b].img, c.tc.img_bytes));
+    A(dalloc(&c.pub[b].bounds, 2 * (int64_t)c.d));
   }
+  A(dalloc(&c.bounds_stage, 2 * (int64_t)c.d));
+  A(dalloc(&c.bpart, (int64_t)kBoundsBlocks * 2 * c.d));
   c.bkeys_cap = cfg->max_batch_tokens / kBlockTok + 1;
   if (!c.use_index && cfg->prefix_mode != LS_PREFIX_FUSED) {
     A(dalloc(&c.bkeys, c.bkeys_cap));
@@ -256,6 +261,15 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
     A(cudaMemset(c.adam_v, 0, (size_t)c.n_params * sizeof(float)));
     A(cudaMemset(c.d_err, 0, sizeof(int)));
     if (c.tf.base) A(cudaMemset(c.tf.base, 0, (size_t)tf_bytes));
+    {  // no record seen yet: the empty range in every column
+      std::vector<float> empty(2 * (size_t)c.d);
+      std::fill(empty.begin(), empty.begin() + c.d, INFINITY);
+      std::fill(empty.begin() + c.d, empty.end(), -INFINITY);
+      const size_t nb = empty.size() * sizeof(float);
+      A(cudaMemcpy(c.bounds_stage, empty.data(), nb, cudaMemcpyHostToDevice));
+      A(cudaMemcpy(c.pub[0].bounds, empty.data(), nb, cudaMemcpyHostToDevice));
+      A(cudaMemcpy(c.pub[1].bounds, empty.data(), nb, cudaMemcpyHostToDevice));
+    }
     DevState init{};
     init.cur = -1;
     init.route_b = 0;
@@ -447,13 +461,20 @@ int ls_assemble_features(ls_ctx* h, int32_t n_req, const int64_t* tok_off, const
   return LS_OK;
 }
 
-int ls_route_batch(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* tok_off,
-                   const float* req_feats, int32_t* choice, float* best, float* scores_opt,
-                   int32_t* hits_opt, uint64_t* weight_version_out, void* stream) {
+}  // extern "C"
+
+namespace {
+
+// One route; `status` non-NULL selects the guarded selection of Algorithm 4
+// (scores are then always materialised and the guard kernel replaces argmin).
+int route_impl(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* tok_off, const float* req_feats,
+               int32_t* choice, float* best, int32_t* status, bool guarded, float* scores_opt, int32_t* hits_opt,
+               uint64_t* weight_version_out, void* stream) {
   if (!h) return fail(LS_ERR_ARG, "ctx is NULL");
   Ctx& c = h->c;
   if (n_req < 0 || n_req > c.cfg.max_requests) return fail(LS_ERR_ARG, "n_req out of range");
-  if (n_req > 0 && (!tok || !tok_off || !choice || !best || (c.cfg.d_req > 0 && !req_feats)))
+  if (n_req > 0 && (!tok || !tok_off || !choice || !best || (c.cfg.d_req > 0 && !req_feats) ||
+                    (guarded && !status)))
     return fail(LS_ERR_ARG, "NULL argument");
   if (c.n_inst < 1) return fail(LS_ERR_STATE, "no snapshot");
   if (!c.have_norm) return fail(LS_ERR_STATE, "normaliser not set");
@@ -470,7 +491,7 @@ int ls_route_batch(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* 
   if (weight_version_out) *weight_version_out = v;
   if (n_req == 0) return LS_OK;
   int32_t* hits = hits_opt ? hits_opt : c.hits;
-  const bool fused_select = c.use_tc && scorer_selects(c.tc, c.n_inst);
+  const bool fused_select = !guarded && c.use_tc && scorer_selects(c.tc, c.n_inst);
   float* scores = scores_opt ? scores_opt : (fused_select ? nullptr : c.scores);
   if (c.use_index) {
     LS_CK(traced(c, TR_PREFIX_INDEX, 1, s, [&] {
@@ -513,13 +534,75 @@ int ls_route_batch(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* 
                                c.cfg.d_inst, req_feats, c.cfg.d_req, c.mean, c.stdv, scores, s);
     }));
   }
-  if (!fused_select)
+  if (guarded)
+    LS_CK(traced(c, TR_GUARDS, 1, s, [&] {
+      return launch_guards(c.guards, n_req, c.n_inst, tok, tok_off, hits, scores, c.inst_state, c.cfg.d_inst,
+                           req_feats, c.cfg.d_req, c.pub, c.st, choice, best, status, c.sms, s);
+    }));
+  else if (!fused_select)
     LS_CK(traced(c, TR_ARGMIN, 1, s, [&] { return launch_argmin(n_req, c.n_inst, scores, choice, best, s); }));
   if (!cap) {
     std::lock_guard<std::mutex> g(c.mu);
     LS_CK(cudaEventRecord(c.ev_route, s));
     c.route_recorded = true;
   }
+  return LS_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int ls_route_batch(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* tok_off,
+                   const float* req_feats, int32_t* choice, float* best, float* scores_opt,
+                   int32_t* hits_opt, uint64_t* weight_version_out, void* stream) {
+  return route_impl(h, n_req, tok, tok_off, req_feats, choice, best, nullptr, false, scores_opt, hits_opt,
+                    weight_version_out, stream);
+}
+
+int ls_route_batch_guarded(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* tok_off,
+                           const float* req_feats, int32_t* choice, float* best, int32_t* status,
+                           float* scores_opt, int32_t* hits_opt, uint64_t* weight_version_out, void* stream) {
+  return route_impl(h, n_req, tok, tok_off, req_feats, choice, best, status, true, scores_opt, hits_opt,
+                    weight_version_out, stream);
+}
+
+int ls_set_guards(ls_ctx* h, const ls_guards* g) {
+  if (!h || !g) return fail(LS_ERR_ARG, "NULL argument");
+  Ctx& c = h->c;
+  if (g->k < 0 || g->k > c.cfg.max_instances) return fail(LS_ERR_ARG, "k out of range");
+  if (g->k > 0 && (g->kv_col < 0 || g->kv_col >= c.cfg.d_inst))
+    return fail(LS_ERR_ARG, "kv_col outside the instance-state columns");
+  c.guards = *g;
+  return LS_OK;
+}
+
+int ls_refresh_bounds(ls_ctx* h, void* stream) {
+  if (!h) return fail(LS_ERR_ARG, "ctx is NULL");
+  Ctx& c = h->c;
+  LS_CK(traced(c, TR_BOUNDS, 1, S(stream), [&] {
+    return launch_ring_bounds(c.d, c.ring_x, c.cfg.ring_capacity, c.bpart, c.bounds_stage, c.st, c.sms,
+                              S(stream));
+  }));
+  return LS_OK;
+}
+
+int ls_get_bounds(ls_ctx* h, int32_t which, float* lo_out, float* hi_out, void* stream) {
+  if (!h || !lo_out || !hi_out) return fail(LS_ERR_ARG, "NULL argument");
+  if (which != 0 && which != 1) return fail(LS_ERR_ARG, "which must be 0 or 1");
+  Ctx& c = h->c;
+  const float* src = c.bounds_stage;
+  if (which == 1) {
+    int32_t cur = -1;
+    LS_CK(cudaDeviceSynchronize());
+    LS_CK(cudaMemcpy(&cur, &c.st->cur, sizeof(cur), cudaMemcpyDeviceToHost));
+    if (cur < 0) return fail(LS_ERR_STATE, "no weights published");
+    src = c.pub[cur].bounds;
+  }
+  const size_t nb = (size_t)c.d * sizeof(float);
+  LS_CK(cudaMemcpyAsync(lo_out, src, nb, cudaMemcpyDeviceToDevice, S(stream)));
+  LS_CK(cudaMemcpyAsync(hi_out, src + c.d, nb, cudaMemcpyDeviceToDevice, S(stream)));
+  LS_CK(cudaStreamSynchronize(S(stream)));
   return LS_OK;
 }
 
@@ -564,7 +647,8 @@ int ls_publish(ls_ctx* h, void* stream) {
   if (!cap && c.route_recorded) LS_CK(cudaStreamWaitEvent(s, c.ev_route, 0));
   if (!cap && c.pub_recorded) LS_CK(cudaStreamWaitEvent(s, c.ev_pub, 0));
   LS_CK(traced(c, TR_PUBLISH, 1, s, [&] {
-    return launch_publish(c.mlp, c.use_tc ? &c.tc : nullptr, c.master, c.pub, c.use_tc ? 0 : 1, c.st, c.sms, s);
+    return launch_publish(c.mlp, c.use_tc ? &c.tc : nullptr, c.master, c.pub, c.use_tc ? 0 : 1, c.bounds_stage,
+                          c.st, c.sms, s);
   }));
   if (!cap) {
     LS_CK(cudaEventRecord(c.ev_pub, s));

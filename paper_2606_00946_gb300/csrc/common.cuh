@@ -60,6 +60,7 @@ struct Published {
   float* params = nullptr;  // flat, same layout as the master; weights rounded in bf16 mode
   float* wt = nullptr;      // per-layer transposed weights [in, out]
   uint8_t* img = nullptr;   // pre-swizzled bf16 hidden-layer weights (tensor-core scorer)
+  float* bounds = nullptr;  // feature bounds published with the weights: lo [d], then hi [d]
   uint64_t version = 0;
 };
 
@@ -91,7 +92,7 @@ __device__ __forceinline__ void advance_step(DevState* st, int64_t t) {
   st->beta_pow[0] *= 0.9;
   st->beta_pow[1] *= 0.999;
 }
-enum { DONE_RING = 0, DONE_OPT = 1, DONE_PUB = 2 };
+enum { DONE_RING = 0, DONE_OPT = 1, DONE_PUB = 2, DONE_BOUNDS = 3 };
 
 // Kernel-level tracing: when enabled, every launch is bracketed by CUDA events
 // recorded on the launching stream; ls_trace_read() sums the elapsed times.
@@ -99,7 +100,8 @@ enum TraceId {
   TR_HASH, TR_INSERT, TR_PREFIX, TR_SCORE, TR_ARGMIN, TR_ASSEMBLE, TR_RING, TR_PUBLISH,
   TR_GATHER, TR_GEMM_FWD, TR_LOSS, TR_GEMM_DW, TR_REDUCE, TR_COLSUM, TR_GEMM_DX, TR_OPT,
   TR_MEMSET, TR_SCORE_TC, TR_NORM_ROWS, TR_PUBLISH_TC, TR_HASH_BATCH, TR_SCREEN, TR_WALK,
-  TR_GEMM_TC_FWD, TR_GEMM_TC_DW, TR_GEMM_TC_DX, TR_PREFIX_INDEX, TR_INDEX_INSERT, TR_COUNT
+  TR_GEMM_TC_FWD, TR_GEMM_TC_DW, TR_GEMM_TC_DX, TR_PREFIX_INDEX, TR_INDEX_INSERT,
+  TR_GUARDS, TR_BOUNDS, TR_COUNT
 };
 extern const char* const kTraceNames[TR_COUNT];
 
@@ -197,7 +199,12 @@ struct Ctx {
   // sample ring (Sec. 4.3.2)
   float* ring_x = nullptr;
   float* ring_y = nullptr;
-  int64_t ring_enqueued = 0;     // records appended (host order); the device count is st->ring_count
+  int64_t ring_enqueued = 0;
+  // feature bounds of the ring (Algorithm 4 [l, u]): staged by ls_refresh_bounds,
+  // published by ls_publish into pub[b].bounds
+  float* bounds_stage = nullptr;  // lo [d], hi [d]
+  float* bpart = nullptr;         // per-block partial bounds [kBoundsBlocks][2][d]
+  ls_guards guards{};     // records appended (host order); the device count is st->ring_count
 
   // route scratch
   int32_t* hits = nullptr;    // [max_requests, max_instances]
@@ -286,6 +293,15 @@ __device__ __forceinline__ bool last_block(uint32_t* done) {
   return is_last;
 }
 
+// (a, i) precedes (b, j) in the order (score, index): NaN after every number,
+// -0 == +0, ties to the lower index (the greedy selection of Algorithm 4).
+__device__ __forceinline__ bool score_precedes(float a, int i, float b, int j) {
+  const bool an = isnan(a), bn = isnan(b);
+  if (an != bn) return bn;
+  if (!an && a != b) return a < b;
+  return i < j;
+}
+
 // Raw feature k of pair (request with prompt length L and hit length h,
 // instance row inst, request extras req):  [L, h, 16h, 16h/L, L-16h,
 // ceil(L/16)-h || inst[0..d_inst) || req[0..d_req)]  (Sec. 4.1 Features).
@@ -340,13 +356,21 @@ cudaError_t launch_score_simt(const MlpDesc& mlp, const Published* pub, const in
                               const float* stdv, float* scores, cudaStream_t s);
 cudaError_t launch_argmin(int n_req, int n_inst, const float* scores, int32_t* choice,
                           float* best, cudaStream_t s);
+// Algorithm 4 guards: per-block bounds partials are combined by the last block.
+constexpr int kBoundsBlocks = 256;
+cudaError_t launch_ring_bounds(int d, const float* ring_x, int64_t capacity, float* bpart, float* stage,
+                               DevState* st, int sms, cudaStream_t s);
+cudaError_t launch_guards(const ls_guards& g, int n_req, int n_inst, const int32_t* tok, const int64_t* tok_off,
+                          const int32_t* hits, const float* scores, const float* inst, int d_inst,
+                          const float* req, int d_req, const Published* pub, const DevState* st,
+                          int32_t* choice, float* best, int32_t* status, int sms, cudaStream_t s);
 
 bool plan_tc(const MlpDesc& m, TcPlan& p);
 // Publish the master weights into buffer 1 - st->cur (fp32 params, the
-// transposed copy when `want_wt`, the tensor-core image when `tc`), then flip
-// st->cur and bump the version; one launch.
+// transposed copy when `want_wt`, the tensor-core image when `tc`, the staged
+// feature bounds), then flip st->cur and bump the version; one launch.
 cudaError_t launch_publish(const MlpDesc& m, const TcPlan* tc, const float* master, const Published* pub,
-                           int want_wt, DevState* st, int sms, cudaStream_t s);
+                           int want_wt, const float* bounds_stage, DevState* st, int sms, cudaStream_t s);
 cudaError_t launch_norm_rows(const int64_t* tok_off, const int32_t* hits, uint4* pairx, int n_inst, int d_inst,
                              const float* inst, int n_req, int d_req,
                              const float* req, const float* mean, const float* stdv, int d_pad,

@@ -7,7 +7,8 @@
 //   wt      per-layer transposed weights W^T [in, out] (CUDA-core scorer only);
 //   img     bf16 hidden-layer weights pre-swizzled into the tensor-core operand
 //           layout: N-chunks of nc rows x K-blocks of 64 columns, 128-byte
-//           swizzle, one 16-byte chunk (8 columns) per thread.
+//           swizzle, one 16-byte chunk (8 columns) per thread;
+//   bounds  the staged feature bounds (Algorithm 4 [l, u]), lo [d] then hi [d].
 // The last block to finish bumps the version and then flips st->cur, so a
 // route that sees the new index sees a complete buffer.
 #include "common.cuh"
@@ -22,6 +23,9 @@ struct PubArgs {
   float* params[2];
   float* wt[2];
   uint8_t* img[2];
+  float* bounds[2];
+  const float* bounds_stage;
+  int64_t n_bounds;                      // 2 d
   int64_t n_params;
   int64_t n_wt;                          // elements of the transposed copy (0: not kept)
   int n_tc;                              // tensor-core layers (0: no image)
@@ -43,8 +47,9 @@ __global__ void __launch_bounds__(256) k_publish(const __grid_constant__ PubArgs
   float* __restrict__ pp = a.params[tgt];
   float* __restrict__ wt = a.wt[tgt];
   uint8_t* __restrict__ img = a.img[tgt];
+  float* __restrict__ bnd = a.bounds[tgt];
   const int64_t n_img = a.n_tc ? a.grp_end[a.n_tc - 1] : 0;
-  const int64_t total = a.n_params + a.n_wt + n_img;
+  const int64_t total = a.n_params + a.n_wt + n_img + a.n_bounds;
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
        e += (int64_t)gridDim.x * blockDim.x) {
     if (e < a.n_params) {
@@ -61,6 +66,9 @@ __global__ void __launch_bounds__(256) k_publish(const __grid_constant__ PubArgs
       const int k = (int)(u / out), o = (int)(u - (int64_t)k * out);
       const float v = __ldg(a.master + m.woff[l] + (int64_t)o * in + k);
       wt[t] = m.bf16 ? round_bf16(v) : v;
+    } else if (e >= a.n_params + a.n_wt + n_img) {
+      const int64_t t = e - (a.n_params + a.n_wt + n_img);
+      bnd[t] = __ldg(a.bounds_stage + t);
     } else {
       const int64_t g = e - a.n_params - a.n_wt;
       int l = 0;
@@ -97,7 +105,7 @@ __global__ void __launch_bounds__(256) k_publish(const __grid_constant__ PubArgs
 }  // namespace
 
 cudaError_t launch_publish(const MlpDesc& m, const TcPlan* tc, const float* master, const Published* pub,
-                           int want_wt, DevState* st, int sms, cudaStream_t s) {
+                           int want_wt, const float* bounds_stage, DevState* st, int sms, cudaStream_t s) {
   PubArgs a{};
   a.m = m;
   a.master = master;
@@ -105,7 +113,10 @@ cudaError_t launch_publish(const MlpDesc& m, const TcPlan* tc, const float* mast
     a.params[b] = pub[b].params;
     a.wt[b] = pub[b].wt;
     a.img[b] = pub[b].img;
+    a.bounds[b] = pub[b].bounds;
   }
+  a.bounds_stage = bounds_stage;
+  a.n_bounds = 2 * (int64_t)m.w[0];
   int64_t n_params = 0, n_wt = 0;
   for (int l = 0; l < m.n_layers; ++l) {
     n_params += (int64_t)m.w[l + 1] * m.w[l] + m.w[l + 1];
@@ -123,7 +134,7 @@ cudaError_t launch_publish(const MlpDesc& m, const TcPlan* tc, const float* mast
     a.grp_end[l] = groups;
   }
   a.st = st;
-  const int64_t total = a.n_params + a.n_wt + groups;
+  const int64_t total = a.n_params + a.n_wt + groups + a.n_bounds;
   const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((total + 255) / 256, (int64_t)sms * 4));
   k_publish<<<grid, 256, 0, s>>>(a);
   return cudaGetLastError();

@@ -9,15 +9,6 @@ namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
 
-// (a, i) precedes (b, j) in the order (score, index): NaN after every number,
-// -0 == +0, ties to the lower index.
-__device__ __forceinline__ bool precedes(float a, int i, float b, int j) {
-  const bool an = isnan(a), bn = isnan(b);
-  if (an != bn) return bn;
-  if (!an && a != b) return a < b;
-  return i < j;
-}
-
 __device__ __forceinline__ float norm_feature(int k, int64_t L, int h, const float* inst,
                                              int d_inst, const float* req, const float* mean,
                                              const float* stdv) {
@@ -134,13 +125,13 @@ __global__ void k_argmin(int n_req, int n_inst, const float* __restrict__ scores
   int bi = -1;
   for (int i = lane; i < n_inst; i += 32) {
     const float v = s[i];
-    if (bi < 0 || precedes(v, i, bv, bi)) { bv = v; bi = i; }
+    if (bi < 0 || score_precedes(v, i, bv, bi)) { bv = v; bi = i; }
   }
 #pragma unroll
   for (int o = 16; o; o >>= 1) {
     const float ov = __shfl_xor_sync(kFull, bv, o);
     const int oi = __shfl_xor_sync(kFull, bi, o);
-    if (oi >= 0 && (bi < 0 || precedes(ov, oi, bv, bi))) { bv = ov; bi = oi; }
+    if (oi >= 0 && (bi < 0 || score_precedes(ov, oi, bv, bi))) { bv = ov; bi = oi; }
   }
   if (lane == 0) { choice[r] = bi; best[r] = bv; }
 }

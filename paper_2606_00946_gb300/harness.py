@@ -112,6 +112,35 @@ class Router:
         L.check(rc)
         return dict(choice=choice, best=best, scores=scores, hits=hits, version=ver)
 
+    def route_guarded(self, tok, tok_off, req_feats, n_inst, want_scores=True, want_hits=True, stream=None,
+                      out=None):
+        """Guarded route (Algorithm 4): adds a per-request status."""
+        n_req = tok_off.numel() - 1
+        o = out or {}
+        choice = o.get("choice", torch.empty(n_req, dtype=torch.int32, device="cuda"))
+        best = o.get("best", torch.empty(n_req, dtype=torch.float32, device="cuda"))
+        status = o.get("status", torch.empty(n_req, dtype=torch.int32, device="cuda"))
+        scores = o.get("scores") if "scores" in o else (
+            torch.empty(n_req, n_inst, dtype=torch.float32, device="cuda") if want_scores else None)
+        hits = o.get("hits") if "hits" in o else (
+            torch.empty(n_req, n_inst, dtype=torch.int32, device="cuda") if want_hits else None)
+        rc, ver = L.ls_route_batch_guarded(self.h, n_req, tok, tok_off, req_feats, choice, best, status,
+                                           scores, hits, stream)
+        L.check(rc)
+        return dict(choice=choice, best=best, status=status, scores=scores, hits=hits, version=ver)
+
+    def set_guards(self, **kw):
+        L.check(L.ls_set_guards(self.h, **kw))
+
+    def refresh_bounds(self, stream=None):
+        L.check(L.ls_refresh_bounds(self.h, stream))
+
+    def bounds(self, which=1):
+        lo = torch.empty(self.widths[0], dtype=torch.float32, device="cuda")
+        hi = torch.empty_like(lo)
+        L.check(L.ls_get_bounds(self.h, which, lo, hi))
+        return lo, hi
+
     def log(self, feats, ttft, stream=None):
         L.check(L.ls_log_samples(self.h, ttft.numel(), feats, ttft, stream))
 

@@ -24,6 +24,7 @@ SCORERS = {"auto": 0, "cuda_cores": 1, "tensor_cores": 2}
 LS_STATIC_MAX_BLOCKS, LS_STATIC_MAX_PAIRS = 262144, 262144
 LS_PREFIX_AUTO, LS_PREFIX_TWO_PHASE, LS_PREFIX_FUSED, LS_PREFIX_INDEX = 0, 1, 2, 3
 PREFIX_MODES = {"auto": 0, "two_phase": 1, "fused": 2, "index": 3}
+LS_ROUTE_OK, LS_ROUTE_COLD_START, LS_ROUTE_OOD, LS_ROUTE_KFILTER = 0, 1, 2, 4
 
 
 class ls_config(C.Structure):
@@ -39,6 +40,11 @@ class ls_info(C.Structure):
     _fields_ = [("n_inst", C.c_int32), ("d", C.c_int32), ("n_params", C.c_int64),
                 ("table_slots", C.c_int64), ("ring_count", C.c_int64),
                 ("train_steps", C.c_int64), ("weight_version", C.c_uint64), ("scorer", C.c_int32)]
+
+
+class ls_guards(C.Structure):
+    _fields_ = [("n_min", C.c_int64), ("ood", C.c_int32), ("k", C.c_int32), ("kv_col", C.c_int32),
+                ("tau_sat", C.c_float), ("tau_ben", C.c_float)]
 
 
 class ls_trace_entry(C.Structure):
@@ -66,6 +72,11 @@ _SIGS = {
     "ls_log_samples": (C.c_int, [_P, _i32, _P, _P, _P]),
     "ls_train_step": (C.c_int, [_P, _i32, _P, _i32, C.c_float, _P, _P]),
     "ls_publish": (C.c_int, [_P, _P]),
+    "ls_set_guards": (C.c_int, [_P, C.POINTER(ls_guards)]),
+    "ls_refresh_bounds": (C.c_int, [_P, _P]),
+    "ls_get_bounds": (C.c_int, [_P, _i32, _P, _P, _P]),
+    "ls_route_batch_guarded": (C.c_int, [_P, _i32, _P, _P, _P, _P, _P, _P, _P, _P,
+                                         C.POINTER(C.c_uint64), _P]),
     "ls_trace_enable": (C.c_int, [_P, _i32]),
     "ls_trace_read": (C.c_int, [_P, C.POINTER(ls_trace_entry), _i32, C.POINTER(_i32)]),
     "ls_prefix_hits_static": (C.c_int, [_i32, _P, _P, _i64, _P, _i64, _i32, _P, _P]),
@@ -241,6 +252,29 @@ def ls_train_step(ctx, batch, idx, opt, lr, loss_out=None, stream=None) -> int:
 
 def ls_publish(ctx, stream=None) -> int:
     return lib().ls_publish(ctx, stream_handle(stream))
+
+
+def ls_set_guards(ctx, n_min=0, ood=False, k=0, kv_col=0, tau_sat=0.8, tau_ben=0.0) -> int:
+    g = ls_guards(int(n_min), 1 if ood else 0, int(k), int(kv_col), float(tau_sat), float(tau_ben))
+    return lib().ls_set_guards(ctx, C.byref(g))
+
+
+def ls_refresh_bounds(ctx, stream=None) -> int:
+    return lib().ls_refresh_bounds(ctx, stream_handle(stream))
+
+
+def ls_get_bounds(ctx, which, lo_out, hi_out, stream=None) -> int:
+    return lib().ls_get_bounds(ctx, int(which), ptr(lo_out), ptr(hi_out), stream_handle(stream))
+
+
+def ls_route_batch_guarded(ctx, n_req, tok, tok_off, req_feats, choice, best, status, scores_opt=None,
+                           hits_opt=None, stream=None):
+    """Returns (status code of the call, weight_version)."""
+    v = C.c_uint64(0)
+    rc = lib().ls_route_batch_guarded(ctx, int(n_req), ptr(tok), ptr(tok_off), ptr(req_feats), ptr(choice),
+                                      ptr(best), ptr(status), ptr(scores_opt), ptr(hits_opt), C.byref(v),
+                                      stream_handle(stream))
+    return rc, v.value
 
 
 def ls_trace_enable(ctx, on=True) -> int:

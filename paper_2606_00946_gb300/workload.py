@@ -179,9 +179,9 @@ def instance_state(rng, cfg: Config, n: int | None = None) -> np.ndarray:
 def records(rng, cfg: Config, n: int):
     """Synthetic logged (raw feature row, observed TTFT) records.
 
-    Columns are drawn directly, not assembled: f0 = prompt length L, f1 = hit
-    blocks h ~ U{0..floor(L/16)}, f2..f5 are independent draws in the ranges of
-    hit tokens, hit ratio, miss tokens and miss blocks; instance columns follow
+    Pair columns are those of a routed pair (Sec. 4.1 Features): f0 = prompt
+    length L, f1 = hit blocks h ~ U{0..floor(L/16)}, f2 = 16h, f3 = 16h/L
+    (fp32), f4 = L - 16h, f5 = ceil(L/16) - h; instance columns follow
     instance_state(); request extras are N(0,1).
     TTFT models (seconds):
       linear    : y = sum_k w_k * (x_k - m_k)/s_k + 0.05 N(0,1), w_k ~ N(0, 0.1^2),
@@ -196,11 +196,12 @@ def records(rng, cfg: Config, n: int):
     nb = L // BLOCK
     x = np.zeros((n, cfg.d), np.float64)
     x[:, 0] = L
-    x[:, 1] = np.floor(rng.random(n) * (nb + 1))
-    x[:, 2] = BLOCK * np.floor(rng.random(n) * (nb + 1))
-    x[:, 3] = rng.random(n)
-    x[:, 4] = np.floor(rng.random(n) * (L + 1))
-    x[:, 5] = np.floor(rng.random(n) * (nb + 2))
+    h = np.floor(rng.random(n) * (nb + 1))
+    x[:, 1] = h
+    x[:, 2] = BLOCK * h
+    x[:, 3] = (BLOCK * h).astype(np.float32) / L.astype(np.float32)
+    x[:, 4] = L - BLOCK * h
+    x[:, 5] = -(-L // BLOCK) - h
     x[:, PAIR_DIMS:PAIR_DIMS + cfg.d_inst] = instance_state(rng, cfg, n)
     if cfg.d_req:
         x[:, PAIR_DIMS + cfg.d_inst:] = rng.standard_normal((n, cfg.d_req))
