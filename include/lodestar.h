@@ -279,8 +279,9 @@ int ls_get_bounds(ls_ctx *ctx, int32_t which, float *lo_out, float *hi_out, void
  *      outside [lo, hi] of the bounds published with the weights this route
  *      reads;
  *   3. choice = argmin_i yhat[r,i] as in ls_route_batch, then the K-filter
- *      (when k >= 1 and the prompt has a full block): if the fp64 mean of
- *      inst_state[:, kv_col] (summed in instance order) exceeds tau_sat and
+ *      (when k >= 1 and the prompt has a full block): if the mean of
+ *      inst_state[:, kv_col] exceeds tau_sat (decided as S > N tau_sat in
+ *      fp64, S the fp32 sum in instance order) and
  *      16 max_i h[r,i] exceeds tau_ben, the candidates are the k instances
  *      with the largest rendezvous weights mix64(g ^ mix64((i+1) G)) (ties
  *      to the lower index), g = key of the prompt's first block (the prefix

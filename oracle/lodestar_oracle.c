@@ -37,7 +37,7 @@
  *   - argmin ties -> lowest index, -0 == +0, NaN after every number;
  *   - guards: n = records ever appended; bounds = NaN-skipping min / max over
  *     the records the ring holds; prefix group = key of the first full block;
- *     ConsistentHash_K = top-K rendezvous hashing; gpu_kv mean in fp64 in
+ *     ConsistentHash_K = top-K rendezvous hashing; gpu_kv sum in fp32 in
  *     index order; kappa_i |r| = 16 h_i; epsilon = 0, no random tiebreak.
  */
 #include <math.h>
@@ -551,7 +551,9 @@ int32_t or_hrw_candidates(uint64_t g, int32_t n_inst, int32_t K, int32_t *cand) 
  *   otherwise status 0 and choice = argmin over instances (= argmax of the
  *   reward -TTFT; order of or_argmin), then the K-filter: when K >= 1, the
  *   prompt has a full block (its group key gkey[r] is the key of block 0),
- *     mean_i inst[i, kv_col] > tau_sat   (fp64 sum in index order, / N) and
+ *     mean_i inst[i, kv_col] > tau_sat   (S = fp32 sum in index order; the
+ *                                         test is S > N tau_sat in fp64, the
+ *                                         product exact for N < 2^29) and
  *     max_i 16 h_i > tau_ben             (kappa_i |r| = 16 h_i hit tokens),
  *   status gains bit 4 and a choice outside the candidates is replaced by the
  *   argmin over the candidates.  best = scores of the final choice.
@@ -567,10 +569,9 @@ int or_guards(int64_t n_req, int32_t n_inst, const int64_t *L, const uint64_t *g
     float *x = (float *)malloc((size_t)d * sizeof(float));
     int32_t *cand = (int32_t *)malloc((size_t)(K > 0 ? K : 1) * sizeof(int32_t));
     if (!x || !cand) { free(x); free(cand); return -1; }
-    double kv_sum = 0.0;
+    float kv_sum = 0.0f;
     if (K >= 1 && kv_col >= 0 && kv_col < d_inst)
-        for (int32_t i = 0; i < n_inst; ++i) kv_sum += (double)inst[(int64_t)i * d_inst + kv_col];
-    double kv_mean = kv_sum / (double)n_inst;
+        for (int32_t i = 0; i < n_inst; ++i) kv_sum += inst[(int64_t)i * d_inst + kv_col];
     for (int64_t r = 0; r < n_req; ++r) {
         const float *sr = scores + r * n_inst;
         const int32_t *hr = hits + r * n_inst;
@@ -598,7 +599,7 @@ int or_guards(int64_t n_req, int32_t n_inst, const int64_t *L, const uint64_t *g
         if (K >= 1 && L[r] >= OR_BLOCK && kv_col >= 0 && kv_col < d_inst) {
             int32_t hmax = 0;
             for (int32_t i = 0; i < n_inst; ++i) if (hr[i] > hmax) hmax = hr[i];
-            if (kv_mean > (double)tau_sat && 16.0 * (double)hmax > (double)tau_ben) {
+            if ((double)kv_sum > (double)n_inst * (double)tau_sat && 16.0 * (double)hmax > (double)tau_ben) {
                 int32_t m = or_hrw_candidates(gkey[r], n_inst, K, cand);
                 int in = 0;
                 for (int32_t q = 0; q < m; ++q) in |= cand[q] == c;

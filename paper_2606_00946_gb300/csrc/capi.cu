@@ -110,7 +110,7 @@ void free_all(Ctx& c) {
                   c.ring_x, c.ring_y, c.hits, c.scores, c.tx, c.tz, c.ty, c.dz0, c.dz1, c.grad,
                   c.gpart, c.loss_tmp, c.d_err, c.pub[0].img, c.pub[1].img, c.xin, c.xrq, c.pairx, c.ximg,
                   c.bkeys, c.work, c.work_n, c.gkeys, c.gmask, c.st, c.tf.base, c.tf.parts,
-                  c.pub[0].bounds, c.pub[1].bounds, c.bounds_stage, c.bpart};
+                  c.pub[0].bounds, c.pub[1].bounds, c.bounds_stage, c.benc};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   if (c.ev_pub) cudaEventDestroy(c.ev_pub);
@@ -213,7 +213,7 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
     A(dalloc(&c.pub[b].bounds, 2 * (int64_t)c.d));
   }
   A(dalloc(&c.bounds_stage, 2 * (int64_t)c.d));
-  A(dalloc(&c.bpart, (int64_t)kBoundsBlocks * 2 * c.d));
+  A(dalloc(&c.benc, 2 * (int64_t)c.d));
   c.bkeys_cap = cfg->max_batch_tokens / kBlockTok + 1;
   if (!c.use_index && cfg->prefix_mode != LS_PREFIX_FUSED) {
     A(dalloc(&c.bkeys, c.bkeys_cap));
@@ -269,6 +269,9 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
       A(cudaMemcpy(c.bounds_stage, empty.data(), nb, cudaMemcpyHostToDevice));
       A(cudaMemcpy(c.pub[0].bounds, empty.data(), nb, cudaMemcpyHostToDevice));
       A(cudaMemcpy(c.pub[1].bounds, empty.data(), nb, cudaMemcpyHostToDevice));
+      std::vector<uint32_t> ident(2 * (size_t)c.d, 0xff800000u);  // codes of +inf, then -inf
+      std::fill(ident.begin() + c.d, ident.end(), 0x007fffffu);
+      A(cudaMemcpy(c.benc, ident.data(), ident.size() * sizeof(uint32_t), cudaMemcpyHostToDevice));
     }
     DevState init{};
     init.cur = -1;
@@ -581,7 +584,7 @@ int ls_refresh_bounds(ls_ctx* h, void* stream) {
   if (!h) return fail(LS_ERR_ARG, "ctx is NULL");
   Ctx& c = h->c;
   LS_CK(traced(c, TR_BOUNDS, 1, S(stream), [&] {
-    return launch_ring_bounds(c.d, c.ring_x, c.cfg.ring_capacity, c.bpart, c.bounds_stage, c.st, c.sms,
+    return launch_ring_bounds(c.d, c.ring_x, c.cfg.ring_capacity, c.benc, c.bounds_stage, c.st, c.sms,
                               S(stream));
   }));
   return LS_OK;

@@ -203,7 +203,7 @@ struct Ctx {
   // feature bounds of the ring (Algorithm 4 [l, u]): staged by ls_refresh_bounds,
   // published by ls_publish into pub[b].bounds
   float* bounds_stage = nullptr;  // lo [d], hi [d]
-  float* bpart = nullptr;         // per-block partial bounds [kBoundsBlocks][2][d]
+  uint32_t* benc = nullptr;       // bounds being reduced, order-preserving codes [2][d]
   ls_guards guards{};     // records appended (host order); the device count is st->ring_count
 
   // route scratch
@@ -356,9 +356,10 @@ cudaError_t launch_score_simt(const MlpDesc& mlp, const Published* pub, const in
                               const float* stdv, float* scores, cudaStream_t s);
 cudaError_t launch_argmin(int n_req, int n_inst, const float* scores, int32_t* choice,
                           float* best, cudaStream_t s);
-// Algorithm 4 guards: per-block bounds partials are combined by the last block.
-constexpr int kBoundsBlocks = 256;
-cudaError_t launch_ring_bounds(int d, const float* ring_x, int64_t capacity, float* bpart, float* stage,
+// Algorithm 4 guards.  benc must hold the identity codes (0xff800000 in
+// [0, d), 0x007fffff in [d, 2d)) before a bounds launch; each launch leaves
+// them so.
+cudaError_t launch_ring_bounds(int d, const float* ring_x, int64_t capacity, uint32_t* benc, float* stage,
                                DevState* st, int sms, cudaStream_t s);
 cudaError_t launch_guards(const ls_guards& g, int n_req, int n_inst, const int32_t* tok, const int64_t* tok_off,
                           const int32_t* hits, const float* scores, const float* inst, int d_inst,

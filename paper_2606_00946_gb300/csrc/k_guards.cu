@@ -6,15 +6,20 @@
 //
 //   k_ring_bounds  feature bounds [l, u] of the training buffer: column-wise
 //                  minimum / maximum over the records the ring holds (NaN
-//                  skipped), block partials combined by the last block into
-//                  the staging copy that the next publish makes visible.
+//                  skipped), block results met by atomic min / max on
+//                  order-preserving codes, decoded by the last block into the
+//                  staging copy that the next publish makes visible.
 //                  Bound: HBM, 4 d bytes per held record.
 //   k_guards       one warp per request: cold-start test, out-of-range test of
 //                  every raw feature of every pair, argmin, K-filter.  Reads
 //                  the hits and scores of the request (8 bytes per pair), its
 //                  first 64 prompt bytes and its extras; writes 12 bytes.
+#include <climits>
+#include <cmath>
+
 #include "blockhash.cuh"
 #include "common.cuh"
+#include "sm100.cuh"
 
 namespace ls {
 namespace {
@@ -25,79 +30,118 @@ constexpr unsigned kFull = 0xffffffffu;
 // feature bounds of the sample ring
 // ---------------------------------------------------------------------------
 
-// Rows [0, min(count, capacity)) split into gridDim.x contiguous ranges.  For
-// d <= 256 the block reads P = 256 / d rows per pass (thread t: column t % d,
-// row phase t / d), so one pass reads a contiguous run of P d floats; wider
-// rows take columns t, t + 256, ... of every row.
+// Order-preserving 32-bit code of a float (unsigned comparison of codes =
+// float comparison, -0 below +0): the block minima / maxima meet in global
+// memory through atomicMin / atomicMax on codes, so the result does not
+// depend on which block finishes first.
+__device__ __forceinline__ uint32_t ord_code(float f) {
+  const uint32_t u = __float_as_uint(f);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float ord_float(uint32_t e) {
+  return __uint_as_float((e & 0x80000000u) ? (e & 0x7fffffffu) : ~e);
+}
+constexpr uint32_t kCodePosInf = 0xff800000u;  // ord_code(+inf): identity of the minimum
+constexpr uint32_t kCodeNegInf = 0x007fffffu;  // ord_code(-inf): identity of the maximum
+
+__device__ __forceinline__ void fold(float v, float& lo, float& hi) {  // NaN fails both tests: skipped
+  lo = v < lo ? v : lo;
+  hi = v > hi ? v : hi;
+}
+
+// Rows [0, min(count, capacity)) split into gridDim.x contiguous ranges.
+// d % 4 == 0: thread t reads 16-byte groups g = t % (d/4) of rows t / (d/4),
+// t / (d/4) + P, ... (P = 256 / (d/4) rows per pass, so a pass is one
+// contiguous run of P d floats), eight loads in flight.  Other d: the same
+// with single floats (d <= 256), or columns t, t + 256, ... of every row.
+// Block results go to the per-column codes in benc [2][d]; the last block
+// decodes them into the staging copy and resets them for the next launch.
 __global__ void __launch_bounds__(256) k_ring_bounds(int d, const float* __restrict__ ring_x, int64_t capacity,
-                                                     float* __restrict__ bpart, float* __restrict__ stage,
+                                                     uint32_t* __restrict__ benc, float* __restrict__ stage,
                                                      DevState* st) {
-  __shared__ float s_lo[256], s_hi[256];
+  __shared__ float s_lo[1024], s_hi[1024];
   const int64_t count = *reinterpret_cast<volatile int64_t*>(&st->ring_count);
   const int64_t rows = count < capacity ? count : capacity;
   const int64_t per = (rows + gridDim.x - 1) / gridDim.x;
   const int64_t r0 = (int64_t)blockIdx.x * per;
   const int64_t r1 = r0 + per < rows ? r0 + per : rows;
-  const bool narrow = d <= 256;
-  const int P = narrow ? 256 / d : 1;
-  const int p = narrow ? (int)threadIdx.x / d : 0;
-  float* part = bpart + (int64_t)blockIdx.x * 2 * d;
-  for (int c = narrow ? (int)threadIdx.x % d : (int)threadIdx.x; c < d; c += narrow ? d : 256) {
-    float lo = INFINITY, hi = -INFINITY;
+  const int t = threadIdx.x;
+  if ((d & 3) == 0) {
+    const int G = d >> 2, P = 256 / G, g = t % G, p = t / G;
+    float lo[4] = {INFINITY, INFINITY, INFINITY, INFINITY};
+    float hi[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
     if (p < P) {
-      const float* col = ring_x + c;
-      int64_t r = r0 + p;
-      // four rows in flight per thread
-      for (; r + 3 * (int64_t)P < r1; r += 4 * (int64_t)P) {
-        float v[4];
+      const float4* base = reinterpret_cast<const float4*>(ring_x) + g;
+      const float4 none = make_float4(NAN, NAN, NAN, NAN);  // rows past the range: folded as NaN, i.e. skipped
+      for (int64_t r = r0 + p; r < r1; r += 8 * (int64_t)P) {
+        float4 v[8];
 #pragma unroll
-        for (int u = 0; u < 4; ++u) v[u] = __ldcs(col + (r + (int64_t)u * P) * d);
+        for (int u = 0; u < 8; ++u) v[u] = r + (int64_t)u * P < r1 ? __ldcs(base + (r + (int64_t)u * P) * G) : none;
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {  // NaN fails both comparisons: skipped
-          lo = v[u] < lo ? v[u] : lo;
-          hi = v[u] > hi ? v[u] : hi;
+        for (int u = 0; u < 8; ++u) {
+          fold(v[u].x, lo[0], hi[0]);
+          fold(v[u].y, lo[1], hi[1]);
+          fold(v[u].z, lo[2], hi[2]);
+          fold(v[u].w, lo[3], hi[3]);
         }
       }
-      for (; r < r1; r += P) {
-        const float v = __ldcs(col + r * d);
-        lo = v < lo ? v : lo;
-        hi = v > hi ? v : hi;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        s_lo[p * d + 4 * g + k] = lo[k];
+        s_hi[p * d + 4 * g + k] = hi[k];
+      }
+    }
+    __syncthreads();
+    for (int c = t; c < d; c += 256) {
+      float l = s_lo[c], h = s_hi[c];
+      for (int q = 1; q < P; ++q) {
+        l = fminf(l, s_lo[q * d + c]);  // +inf / -inf mark phases without a number
+        h = fmaxf(h, s_hi[q * d + c]);
+      }
+      atomicMin(benc + c, ord_code(l));
+      atomicMax(benc + d + c, ord_code(h));
+    }
+  } else {
+    const bool narrow = d <= 256;
+    const int P = narrow ? 256 / d : 1;
+    const int p = narrow ? t / d : 0;
+    for (int c = narrow ? t % d : t; c < d; c += narrow ? d : 256) {
+      float lo = INFINITY, hi = -INFINITY;
+      if (p < P)
+        for (int64_t r = r0 + p; r < r1; r += 4 * (int64_t)P) {
+          float v[4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) v[u] = r + (int64_t)u * P < r1 ? __ldcs(ring_x + (r + (int64_t)u * P) * d + c) : NAN;
+#pragma unroll
+          for (int u = 0; u < 4; ++u) fold(v[u], lo, hi);
+        }
+      if (narrow) {
+        if (p < P) {
+          s_lo[t] = lo;
+          s_hi[t] = hi;
+        }
+      } else {
+        atomicMin(benc + c, ord_code(lo));
+        atomicMax(benc + d + c, ord_code(hi));
       }
     }
     if (narrow) {
-      if (p < P) {
-        s_lo[threadIdx.x] = lo;
-        s_hi[threadIdx.x] = hi;
+      __syncthreads();
+      if (t < d) {
+        float l = s_lo[t], h = s_hi[t];
+        for (int q = 1; q < P; ++q) {
+          l = fminf(l, s_lo[q * d + t]);
+          h = fmaxf(h, s_hi[q * d + t]);
+        }
+        atomicMin(benc + t, ord_code(l));
+        atomicMax(benc + d + t, ord_code(h));
       }
-    } else {
-      part[c] = lo;
-      part[d + c] = hi;
-    }
-  }
-  if (narrow) {
-    __syncthreads();
-    if ((int)threadIdx.x < d) {
-      float lo = s_lo[threadIdx.x], hi = s_hi[threadIdx.x];
-      for (int q = 1; q < P; ++q) {
-        const float l2 = s_lo[q * d + threadIdx.x], h2 = s_hi[q * d + threadIdx.x];
-        lo = l2 < lo ? l2 : lo;
-        hi = h2 > hi ? h2 : hi;
-      }
-      part[threadIdx.x] = lo;
-      part[d + threadIdx.x] = hi;
     }
   }
   if (last_block(&st->done[DONE_BOUNDS])) {
-    for (int c = threadIdx.x; c < d; c += blockDim.x) {
-      float lo = INFINITY, hi = -INFINITY;
-      for (int b = 0; b < (int)gridDim.x; ++b) {
-        const float l2 = __ldcg(bpart + (int64_t)b * 2 * d + c);
-        const float h2 = __ldcg(bpart + (int64_t)b * 2 * d + d + c);
-        lo = l2 < lo ? l2 : lo;
-        hi = h2 > hi ? h2 : hi;
-      }
-      stage[c] = lo;
-      stage[d + c] = hi;
+    for (int c = t; c < d; c += blockDim.x) {
+      stage[c] = ord_float(atomicExch(benc + c, kCodePosInf));
+      stage[d + c] = ord_float(atomicExch(benc + d + c, kCodeNegInf));
     }
   }
 }
@@ -117,8 +161,9 @@ struct GuardArgs {
   const float* bounds[2];
   const DevState* st;
   int64_t n_min;
+  int64_t h_ben;       // 16 h > tau_ben  <=>  h >= h_ben (h an integer; set on the host)
   int ood, K, kv_col;
-  float tau_sat, tau_ben;
+  float tau_sat;
   int32_t* choice;
   float* best;
   int32_t* status;
@@ -131,143 +176,241 @@ __device__ __forceinline__ bool hrw_before(uint64_t wa, int a, uint64_t wb, int 
 
 __device__ __forceinline__ bool in_range(float x, float lo, float hi) { return x >= lo && x <= hi; }
 
-__global__ void __launch_bounds__(256) k_guards(const __grid_constant__ GuardArgs a) {
-  __shared__ float s_lo[kPair], s_hi[kPair];
-  __shared__ int s_kv;
+constexpr int kHashedInst = 1024;  // instance hashes kept in shared memory up to this count
+constexpr int kGuardThreads = 256;  // warp 0: batch-wide terms; warps 1..7: requests
+constexpr int kBarBatch = 1, kBarInst = 2;
+
+// Warp 0 of a block computes the terms shared by the whole batch and hands
+// them over through named barriers, while warps 1..7 work on requests:
+//   kBarBatch  instance hashes mix64((i + 1) G) and the gpu_kv decision;
+//   kBarInst   whether some instance-state value lies outside its bounds.
+// Requests: S lanes per request (a group; 32 / S requests per warp).  Lane j
+// of a group takes instances j, j + S, ...; group results meet through
+// log2(S) xor shuffles.  The out-of-range test of the pair features needs
+// only the smallest and largest hit length of the request: every pair
+// feature is a monotone function of h for a fixed L (L, h, 16h, 16h/L
+// rounded, L - 16h, ceil(L/16) - h), so its extremes over the instances sit
+// at those two.
+template <int S>
+__global__ void __launch_bounds__(kGuardThreads) k_guards(const __grid_constant__ GuardArgs a) {
+  __shared__ uint64_t s_ih[kHashedInst];  // mix64((i + 1) G): the instance half of the rendezvous weight
+  __shared__ int s_kv, s_inst_bad;
   const int N = a.n_inst, d = kPair + a.d_inst + a.d_req;
   const int b = *reinterpret_cast<const volatile int32_t*>(&a.st->route_b);
   const float* lo = a.bounds[b == 1 ? 1 : 0];
   const float* hi = lo + d;
   const bool cold = *reinterpret_cast<const volatile int64_t*>(&a.st->ring_count) < a.n_min;
-  int inst_bad = 0;
-  if (!cold && a.ood) {
-    // instance rows are the same for every request of the batch
-    for (int e = threadIdx.x; e < N * a.d_inst; e += blockDim.x) {
-      const int k = kPair + e % a.d_inst;
-      inst_bad |= !in_range(__ldg(a.inst + e), __ldg(lo + k), __ldg(hi + k));
-    }
-    if (threadIdx.x < kPair) {
-      s_lo[threadIdx.x] = __ldg(lo + threadIdx.x);
-      s_hi[threadIdx.x] = __ldg(hi + threadIdx.x);
-    }
-  }
-  if (threadIdx.x == 0) {
-    int kv = 0;
-    if (!cold && a.K >= 1) {  // gpu_kv mean: fp64, instance order
-      double sum = 0.0;
-      for (int i = 0; i < N; ++i) sum += (double)__ldg(a.inst + (int64_t)i * a.d_inst + a.kv_col);
-      kv = sum / (double)N > (double)a.tau_sat;
-    }
-    s_kv = kv;
-  }
-  inst_bad = __syncthreads_or(inst_bad);
-  const bool kv_ok = s_kv != 0;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const bool hashed = !cold && a.K >= 1 && a.K < N && N <= kHashedInst;
 
-  const int lane = threadIdx.x & 31, warps = blockDim.x >> 5;
-  for (int64_t r = (int64_t)blockIdx.x * warps + (threadIdx.x >> 5); r < a.n_req;
-       r += (int64_t)gridDim.x * warps) {
+  if (warp == 0) {
+    if (cold) return;  // no request warp waits when the batch is cold
+    if (hashed)
+      for (int i = lane; i < N; i += 32) s_ih[i] = bh::mix64((uint64_t)(i + 1) * kG);
+    // gpu_kv: fp32 sum in instance order (lanes load 32 values at a time, the
+    // sum takes them one by one); mean > tau_sat decided as sum > N tau_sat,
+    // the product exact in fp64
+    int kv = 0;
+    if (a.K >= 1) {
+      float sum = 0.0f;
+      for (int base = 0; base < N; base += 32) {
+        const int i = base + lane;
+        const float v = i < N ? __ldg(a.inst + (int64_t)i * a.d_inst + a.kv_col) : 0.0f;
+        const int m = N - base < 32 ? N - base : 32;
+#pragma unroll 8
+        for (int q = 0; q < m; ++q) sum += __shfl_sync(kFull, v, q);
+      }
+      kv = (double)sum > (double)N * (double)a.tau_sat;
+    }
+    if (lane == 0) s_kv = kv;
+    sm100::named_bar_arrive(kBarBatch, kGuardThreads);
+    // instance rows are the same for every request of the batch: lane t takes
+    // elements t, t + 32, ... of the N x d_inst block, 16 loads in flight
+    int bad = 0;
+    if (a.ood && a.d_inst > 0) {
+      const int total = N * a.d_inst;
+      const int step_i = 32 / a.d_inst, step_k = 32 % a.d_inst;
+      int ei = lane / a.d_inst, ek = lane % a.d_inst;
+      for (int e0 = lane; e0 < total; e0 += 16 * 32) {
+        float v[16], l[16], h[16];
+#pragma unroll
+        for (int u = 0; u < 16; ++u) {
+          const bool ok = e0 + u * 32 < total;
+          v[u] = ok ? __ldg(a.inst + (int64_t)ei * a.d_inst + ek) : 0.0f;
+          l[u] = ok ? __ldg(lo + kPair + ek) : 0.0f;
+          h[u] = ok ? __ldg(hi + kPair + ek) : 0.0f;
+          ei += step_i;
+          ek += step_k;
+          if (ek >= a.d_inst) { ek -= a.d_inst; ++ei; }
+        }
+#pragma unroll
+        for (int u = 0; u < 16; ++u) bad |= !in_range(v[u], l[u], h[u]);
+      }
+    }
+    bad = __any_sync(kFull, bad);
+    if (lane == 0) s_inst_bad = bad;
+    sm100::named_bar_arrive(kBarInst, kGuardThreads);
+    return;
+  }
+
+  constexpr int kPerWarp = 32 / S;
+  const int j = lane & (S - 1);  // lane within the group
+  const int64_t groups = (int64_t)gridDim.x * (kGuardThreads / 32 - 1) * kPerWarp;
+  // every lane of a warp runs the same number of iterations (shuffles stay converged)
+  const int64_t iters = ((int64_t)a.n_req + groups - 1) / groups;
+  float plo[kPair], phi[kPair];
+  if (a.ood) {
+#pragma unroll
+    for (int k = 0; k < kPair; ++k) {
+      plo[k] = __ldg(lo + k);
+      phi[k] = __ldg(hi + k);
+    }
+  }
+  bool kv_ok = false, inst_bad = false;
+  for (int64_t it = 0; it < iters; ++it) {
+    const int64_t r = it * groups + ((int64_t)blockIdx.x * (kGuardThreads / 32 - 1) + (warp - 1)) * kPerWarp +
+                      lane / S;
+    const bool live = r < a.n_req;
     if (cold) {
-      if (lane == 0) {
+      if (live && j == 0) {
         a.choice[r] = -1;
         a.best[r] = __int_as_float(0x7fc00000);
         a.status[r] = LS_ROUTE_COLD_START;
       }
       continue;
     }
-    const int64_t off = __ldg(a.tok_off + r);
-    const int64_t L = __ldg(a.tok_off + r + 1) - off;
+    // --- loads: offsets, then the first block's tokens; hits, scores, extras
+    int64_t off = 0, L = 0;
+    if (live) {
+      off = __ldg(a.tok_off + r);
+      L = __ldg(a.tok_off + r + 1) - off;
+    }
+    uint64_t part = 0;  // the group's lanes mix the 8 words of block 0 between them
+    if (live && L >= kBlockTok)
+      for (int w = j; w < 8; w += S) {
+        const int32_t* p = a.tok + off + 2 * w;
+        part ^= bh::word_mix((uint32_t)__ldg(p), (uint32_t)__ldg(p + 1), w);
+      }
     const int32_t* hr = a.hits + r * N;
     const float* sr = a.scores + r * N;
     float bv = 0.0f;
-    int bi = -1, hmax = 0, bad = inst_bad;
-    for (int i = lane; i < N; i += 32) {
-      const int h = __ldg(hr + i);
-      const float v = __ldg(sr + i);
-      if (bi < 0 || score_precedes(v, i, bv, bi)) { bv = v; bi = i; }
-      hmax = h > hmax ? h : hmax;
-      if (a.ood) {
+    int bi = -1, hmax = 0, hmin = INT_MAX, bad = 0;
+    if (live)
+#pragma unroll 4
+      for (int i = j; i < N; i += S) {
+        const int h = __ldg(hr + i);
+        const float v = __ldg(sr + i);
+        if (bi < 0 || score_precedes(v, i, bv, bi)) { bv = v; bi = i; }
+        hmax = h > hmax ? h : hmax;
+        hmin = h < hmin ? h : hmin;
+      }
+    if (live && a.ood)
+      for (int k = j; k < a.d_req; k += S) {
+        const int q = kPair + a.d_inst + k;
+        bad |= !in_range(__ldg(a.req + r * a.d_req + k), __ldg(lo + q), __ldg(hi + q));
+      }
 #pragma unroll
-        for (int k = 0; k < kPair; ++k)
-          bad |= !in_range(raw_feature(k, L, h, nullptr, 0, nullptr), s_lo[k], s_hi[k]);
-      }
-    }
-    if (a.ood)
-      for (int k = lane; k < a.d_req; k += 32) {
-        const int j = kPair + a.d_inst + k;
-        bad |= !in_range(__ldg(a.req + r * a.d_req + k), __ldg(lo + j), __ldg(hi + j));
-      }
-    if (__any_sync(kFull, bad)) {
-      if (lane == 0) {
-        a.choice[r] = -1;
-        a.best[r] = __int_as_float(0x7fc00000);
-        a.status[r] = LS_ROUTE_OOD;
-      }
-      continue;
-    }
-#pragma unroll
-    for (int o = 16; o; o >>= 1) {
+    for (int o = 1; o < S; o <<= 1) {
       const float ov = __shfl_xor_sync(kFull, bv, o);
       const int oi = __shfl_xor_sync(kFull, bi, o);
       if (oi >= 0 && (bi < 0 || score_precedes(ov, oi, bv, bi))) { bv = ov; bi = oi; }
+      const int oh = __shfl_xor_sync(kFull, hmax, o), ol = __shfl_xor_sync(kFull, hmin, o);
+      hmax = oh > hmax ? oh : hmax;
+      hmin = ol < hmin ? ol : hmin;
+      part ^= __shfl_xor_sync(kFull, part, o);
     }
-    hmax = __reduce_max_sync(kFull, hmax);
-    int code = LS_ROUTE_OK;
-    if (a.K >= 1 && L >= kBlockTok && kv_ok && 16.0 * (double)hmax > (double)a.tau_ben) {
-      code = LS_ROUTE_KFILTER;
-      if (a.K < N) {
-        // prefix group g = key of block 0: s_0 = G * G + c_0 (s_{-1} = G)
-        uint64_t part = 0;
-        if (lane < 8) {
-          const int32_t* p = a.tok + off + 2 * lane;
-          part = bh::word_mix((uint32_t)__ldg(p), (uint32_t)__ldg(p + 1), lane);
-        }
+    if (live && a.ood && j < 2) {  // lane 0 tests the pair features at hmin, lane 1 at hmax
+      const int h = j == 0 ? hmin : hmax;
 #pragma unroll
-        for (int o = 4; o; o >>= 1) part ^= __shfl_xor_sync(kFull, part, o);
-        const uint64_t g = bh::key_of(kG * kG + bh::mix64(__shfl_sync(kFull, part, 0)));
-        // K rounds: each takes the best-ranked instance after the one taken last
-        uint64_t tw = 0;
-        int ti = -1, ci = -1;
-        float cv = 0.0f;
-        bool in = false;
-        for (int k = 0; k < a.K; ++k) {
-          uint64_t lw = 0;
-          int li = -1;
-          for (int i = lane; i < N; i += 32) {
-            const uint64_t w = bh::mix64(g ^ bh::mix64((uint64_t)(i + 1) * kG));
+      for (int k = 0; k < kPair; ++k) bad |= !in_range(raw_feature(k, L, h, nullptr, 0, nullptr), plo[k], phi[k]);
+    }
+#pragma unroll
+    for (int o = 1; o < S; o <<= 1) bad |= __shfl_xor_sync(kFull, bad, o);
+    if (it == 0) {  // the batch-wide terms from warp 0
+      sm100::named_bar_sync(kBarBatch, kGuardThreads);
+      kv_ok = s_kv != 0;
+    }
+    const bool filter = live && !bad && a.K >= 1 && L >= kBlockTok && kv_ok && (int64_t)hmax >= a.h_ben;
+    // (a group filters or not as a whole; groups of one warp may differ, so
+    // the shuffles below run in every group and only filtering groups use them)
+    if (__any_sync(kFull, filter && a.K < N)) {
+      // prefix group g = key of block 0: s_0 = G * G + c_0 (s_{-1} = G)
+      const uint64_t g = bh::key_of(kG * kG + bh::mix64(part));
+      // K rounds: each takes the best-ranked instance after the one taken
+      // last.  The lane's weights are computed once (kept in registers for up
+      // to kCached instances per lane, recomputed per round beyond that).
+      constexpr int kCached = 32 / S < 4 ? 4 : 32 / S;
+      uint64_t wc[kCached];
+#pragma unroll
+      for (int m = 0; m < kCached; ++m) {
+        const int i = j + m * S;
+        wc[m] = filter && i < N ? bh::mix64(g ^ (hashed ? s_ih[i] : bh::mix64((uint64_t)(i + 1) * kG))) : 0;
+      }
+      uint64_t tw = 0;
+      int ti = -1, ci = -1;
+      float cv = 0.0f;
+      bool in = false;
+      const int rounds = filter && a.K < N ? a.K : 0;  // K < N: every round finds an instance
+      const int all_rounds = __reduce_max_sync(kFull, rounds);
+      for (int k = 0; k < all_rounds; ++k) {
+        uint64_t lw = 0;
+        int li = -1;
+        if (k < rounds) {
+#pragma unroll
+          for (int m = 0; m < kCached; ++m) {
+            const int i = j + m * S;
+            if (i < N && (ti < 0 || hrw_before(tw, ti, wc[m], i)) && (li < 0 || hrw_before(wc[m], i, lw, li))) {
+              lw = wc[m];
+              li = i;
+            }
+          }
+          for (int i = j + kCached * S; i < N; i += S) {
+            const uint64_t w = bh::mix64(g ^ (hashed ? s_ih[i] : bh::mix64((uint64_t)(i + 1) * kG)));
             if ((ti < 0 || hrw_before(tw, ti, w, i)) && (li < 0 || hrw_before(w, i, lw, li))) { lw = w; li = i; }
           }
+        }
 #pragma unroll
-          for (int o = 16; o; o >>= 1) {
-            const uint64_t ow = __shfl_xor_sync(kFull, lw, o);
-            const int oi = __shfl_xor_sync(kFull, li, o);
-            if (oi >= 0 && (li < 0 || hrw_before(ow, oi, lw, li))) { lw = ow; li = oi; }
-          }
+        for (int o = 1; o < S; o <<= 1) {
+          const uint64_t ow = __shfl_xor_sync(kFull, lw, o);
+          const int oi = __shfl_xor_sync(kFull, li, o);
+          if (oi >= 0 && (li < 0 || hrw_before(ow, oi, lw, li))) { lw = ow; li = oi; }
+        }
+        if (k < rounds) {
           tw = lw;
           ti = li;
           in |= ti == bi;
           const float v = __ldg(sr + ti);
           if (ci < 0 || score_precedes(v, ti, cv, ci)) { cv = v; ci = ti; }
         }
-        if (!in) { bv = cv; bi = ci; }
       }
+      if (filter && a.K < N && !in) { bv = cv; bi = ci; }
     }
-    if (lane == 0) {
-      a.choice[r] = bi;
-      a.best[r] = bv;
-      a.status[r] = code;
+    if (it == 0) {  // out-of-range instance state puts every request out of range
+      sm100::named_bar_sync(kBarInst, kGuardThreads);
+      inst_bad = s_inst_bad != 0;
+    }
+    if (live && j == 0) {
+      if (bad || inst_bad) {
+        a.choice[r] = -1;
+        a.best[r] = __int_as_float(0x7fc00000);
+        a.status[r] = LS_ROUTE_OOD;
+      } else {
+        a.choice[r] = bi;
+        a.best[r] = bv;
+        a.status[r] = filter ? LS_ROUTE_KFILTER : LS_ROUTE_OK;
+      }
     }
   }
 }
 
 }  // namespace
 
-cudaError_t launch_ring_bounds(int d, const float* ring_x, int64_t capacity, float* bpart, float* stage,
+cudaError_t launch_ring_bounds(int d, const float* ring_x, int64_t capacity, uint32_t* benc, float* stage,
                                DevState* st, int sms, cudaStream_t s) {
-  // about 64 rows per block at least; never more blocks than partial slots
-  int64_t grid = (capacity + 63) / 64;
-  grid = std::min<int64_t>(grid, std::min<int64_t>(kBoundsBlocks, 2 * (int64_t)sms));
+  // at least 64 rows per block, at most four blocks per SM
+  int64_t grid = std::min<int64_t>((capacity + 63) / 64, 4 * (int64_t)sms);
   grid = std::max<int64_t>(grid, 1);
-  k_ring_bounds<<<(int)grid, 256, 0, s>>>(d, ring_x, capacity, bpart, stage, st);
+  k_ring_bounds<<<(int)grid, 256, 0, s>>>(d, ring_x, capacity, benc, stage, st);
   return cudaGetLastError();
 }
 
@@ -295,13 +438,19 @@ cudaError_t launch_guards(const ls_guards& g, int n_req, int n_inst, const int32
   a.K = g.k;
   a.kv_col = g.kv_col;
   a.tau_sat = g.tau_sat;
-  a.tau_ben = g.tau_ben;
+  {  // 16 h > tau_ben for an integer h  <=>  h >= floor(tau_ben / 16) + 1 (exact: a power-of-two divide)
+    const double t = (double)g.tau_ben / 16.0;
+    if (std::isnan(t) || t >= 9.0e18) a.h_ben = INT64_MAX;  // never
+    else if (t < 0.0) a.h_ben = 0;                            // every h >= 0
+    else a.h_ben = (int64_t)std::floor(t) + 1;
+  }
   a.choice = choice;
   a.best = best;
   a.status = status;
-  const int64_t blocks = ((int64_t)n_req + 7) / 8;
-  const int grid = (int)std::min<int64_t>(blocks, (int64_t)sms * 8);
-  k_guards<<<grid, 256, 0, s>>>(a);
+  constexpr int S = 8;
+  const int64_t per_block = (kGuardThreads / 32 - 1) * (32 / S);
+  const int grid = (int)std::min<int64_t>(((int64_t)n_req + per_block - 1) / per_block, (int64_t)sms * 8);
+  k_guards<S><<<grid, kGuardThreads, 0, s>>>(a);
   return cudaGetLastError();
 }
 

@@ -82,6 +82,12 @@ __device__ __forceinline__ void named_bar_sync(int id, int count) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
 
+// arrive at a named barrier without waiting (the producer side of a
+// producer / consumer hand-off; consumers bar.sync with the same count)
+__device__ __forceinline__ void named_bar_arrive(int id, int count) {
+  asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
 // named barrier that also ANDs a predicate over the `count` threads: every
 // participant gets the same answer, so a decision to stop is taken together
 __device__ __forceinline__ bool named_bar_and(int id, int count, bool pred) {
