@@ -44,6 +44,8 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-guards", action="store_true", help="skip the guarded-route measurement")
+    p.add_argument("--guards-only", action="store_true",
+                   help="only the guarded-route measurement (--steps routes; for kernel profiling)")
     p.add_argument("--cpu-seconds", type=float, default=12.0, help="target oracle work for cpu_baseline")
     return p.parse_args()
 
@@ -362,6 +364,13 @@ def main():
     loss = torch.zeros(1, device=dev)
     flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
+    if args.guards_only:
+        g = measure_guards(L, r, dw, N, R, cfg.d, min(ring, int(r.info().ring_count)), cfg.d_req, flush, stream,
+                           measured_peaks()[0], n=max(args.steps, 4))
+        if rank == 0:
+            print(json.dumps({"workload": WORKLOAD, "guarded_route": g}))
+        r.close()
+        return 0
     # the step's inputs arrive in fixed buffers (new instance state, new logged records)
     stage_state = torch.empty_like(states[0])
     stage_x = torch.empty(Bt, cfg.d, device=dev)

@@ -75,6 +75,8 @@ def lib():
             L.or_ring_bounds.argtypes = [i64, C.c_int, P, i64, P, P]
             L.or_hrw_candidates.restype = i32
             L.or_hrw_candidates.argtypes = [C.c_uint64, i32, i32, P]
+            L.or_heuristic.argtypes = [i64, i32, P, P, P, C.c_int, C.c_int, C.c_int, C.c_int, C.c_float,
+                                       C.c_float, C.c_float, P]
             L.or_guards.argtypes = [i64, i32, P, P, P, P, C.c_int, P, C.c_int, P, P, P, i64, i64,
                                     C.c_int, i32, i32, C.c_float, C.c_float, P, P, P]
             _lib = L
@@ -352,3 +354,16 @@ def guards(L, gkey, hits, inst_state, req_feats, scores, lo, hi, n, *, n_min=0, 
                            int(kv_col), float(tau_sat), float(tau_ben), _p(choice), _p(best),
                            _p(status)), "guards")
     return choice, best, status
+
+
+def heuristic(L, hits, inst_state, *, mode=1, count_cols=(0, 1), theta_imbal=8.0, k=1.0, tau=0.5):
+    """Fallback heuristic choice per request (Algorithm 1: mode 1; Algorithm 2: mode 2)."""
+    L = _c(L, np.int64)
+    hits = _c(hits, np.int32)
+    inst = _c(inst_state, np.float32)
+    R, N = hits.shape
+    out = np.zeros(R, np.int32)
+    c1 = count_cols[1] if len(count_cols) > 1 else -1
+    _check(lib().or_heuristic(R, N, _p(L), _p(hits), _p(inst), inst.shape[1], int(mode), int(count_cols[0]),
+                              int(c1), float(theta_imbal), float(k), float(tau), _p(out)), "heuristic")
+    return out

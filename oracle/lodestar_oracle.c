@@ -24,6 +24,8 @@
  *   Sec. 4.3.1 (Fallback) and Algorithm 4: cold-start and out-of-range
  *          guards; Sec. 4.1 (Consistent hashing based filtering): the
  *          K-filter of Algorithm 4.
+ *   Algorithms 1 and 2 (the comparison heuristics), which Algorithm 3
+ *          pre-computes as the gateway's fallback choice.
  *
  * Readings where the paper is silent (each also listed in the design notes):
  *   - block hash: SplitMix64 finaliser based content hash, prefix state chained
@@ -38,7 +40,9 @@
  *   - guards: n = records ever appended; bounds = NaN-skipping min / max over
  *     the records the ring holds; prefix group = key of the first full block;
  *     ConsistentHash_K = top-K rendezvous hashing; gpu_kv sum in fp32 in
- *     index order; kappa_i |r| = 16 h_i; epsilon = 0, no random tiebreak.
+ *     index order; kappa_i |r| = 16 h_i; epsilon = 0, no random tiebreak;
+ *   - heuristics: request count = queued + running columns, population
+ *     standard deviation, sort ties to the lowest index.
  */
 #include <math.h>
 #include <stdint.h>
@@ -614,5 +618,74 @@ int or_guards(int64_t n_req, int32_t n_inst, const int64_t *L, const uint64_t *g
         choice[r] = c; best[r] = sr[c]; status[r] = st;
     }
     free(x); free(cand);
+    return 0;
+}
+
+/* ------------------------------------------------------------------------ */
+/* fallback heuristics (Algorithms 1 and 2; Algorithm 3 pre-computes one)   */
+/* ------------------------------------------------------------------------ */
+
+/* The heuristic choice of every request.  Inputs per instance: the request
+ * count c_i = inst[i, c_col0] (+ inst[i, c_col1] when c_col1 >= 0), in fp32,
+ * and per pair the prefix match ratio m_i = kappa = 16 h / L (fp32, 0 when
+ * L = 0).
+ *   mode 1, Algorithm 1 (prefix-cache and load aware):
+ *     if c_max - c_min > theta_imbal (fp64): argmin_i c_i;
+ *     else mu = mean c, sigma = population standard deviation (fp64 sums in
+ *     index order, two passes, sqrt correctly rounded), and among the
+ *     instances with c_i <= mu + k sigma the first in the order (m desc,
+ *     c asc, index asc); none: argmin_i c_i.
+ *   mode 2, Algorithm 2 (prefix aware, threshold tau): i* = argmax m_i
+ *     (ties to the lowest index); i* if m_{i*} > tau, else argmin_i c_i.
+ * argmin_i c_i takes the lowest index among equal counts. */
+int or_heuristic(int64_t n_req, int32_t n_inst, const int64_t *L, const int32_t *hits,
+                 const float *inst, int d_inst, int mode, int c_col0, int c_col1,
+                 float theta_imbal, float k_over, float tau, int32_t *out) {
+    float *c = (float *)malloc((size_t)n_inst * sizeof(float));
+    float *m = (float *)malloc((size_t)n_inst * sizeof(float));
+    if (!c || !m) { free(c); free(m); return -1; }
+    for (int32_t i = 0; i < n_inst; ++i) {
+        c[i] = inst[(int64_t)i * d_inst + c_col0];
+        if (c_col1 >= 0) c[i] = c[i] + inst[(int64_t)i * d_inst + c_col1];
+    }
+    int32_t least = 0;
+    float cmin = c[0], cmax = c[0];
+    for (int32_t i = 1; i < n_inst; ++i) {
+        if (c[i] < c[least]) least = i;
+        if (c[i] < cmin) cmin = c[i];
+        if (c[i] > cmax) cmax = c[i];
+    }
+    double mu = 0.0, var = 0.0;
+    for (int32_t i = 0; i < n_inst; ++i) mu += (double)c[i];
+    mu = mu / (double)n_inst;
+    for (int32_t i = 0; i < n_inst; ++i) {
+        double dv = (double)c[i] - mu;
+        var += dv * dv;
+    }
+    var = var / (double)n_inst;
+    double thr = mu + (double)k_over * sqrt(var);
+    int imbalanced = (double)cmax - (double)cmin > (double)theta_imbal;
+    for (int64_t r = 0; r < n_req; ++r) {
+        const int32_t *hr = hits + r * n_inst;
+        for (int32_t i = 0; i < n_inst; ++i) {
+            float ht = (float)((int64_t)OR_BLOCK * hr[i]);
+            m[i] = L[r] > 0 ? ht / (float)L[r] : 0.0f;
+        }
+        int32_t pick = least;
+        if (mode == 1 && !imbalanced) {
+            int32_t b = -1;
+            for (int32_t i = 0; i < n_inst; ++i) {
+                if (!((double)c[i] <= thr)) continue;
+                if (b < 0 || m[i] > m[b] || (m[i] == m[b] && c[i] < c[b])) b = i;
+            }
+            if (b >= 0) pick = b;
+        } else if (mode == 2) {
+            int32_t b = 0;
+            for (int32_t i = 1; i < n_inst; ++i) if (m[i] > m[b]) b = i;
+            if (m[b] > tau) pick = b;
+        }
+        out[r] = pick;
+    }
+    free(c); free(m);
     return 0;
 }
