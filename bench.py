@@ -52,19 +52,22 @@ def parse():
 
 def measure_guards(L, r, dw, N, R, d, ring_rows, d_req, flush, stream, peaks, n=60):
     """Guarded route of Algorithm 4 (cold start, out-of-range bounds, K-filter
-    with K = 2) on the bench batch, beside the plain route: event-timed route
+    with K = 2) with the fallback heuristic of Algorithm 1 pre-computed (as
+    Algorithm 3 does) on the bench batch, beside the plain route: event-timed route
     calls (call by call, L2 flushed before each) and per-launch times of the
     guard kernel and of the ring-bounds reduction."""
     import torch
     dev = dw.tok.device
     o_plain = {"choice": torch.empty(R, dtype=torch.int32, device=dev),
                "best": torch.empty(R, dtype=torch.float32, device=dev), "scores": None, "hits": None}
-    o_g = dict(o_plain, status=torch.empty(R, dtype=torch.int32, device=dev))
+    o_g = dict(o_plain, status=torch.empty(R, dtype=torch.int32, device=dev),
+               fallback=torch.empty(R, dtype=torch.int32, device=dev))
     r.refresh_bounds()
     r.publish()
     # tau_sat = 0 keeps the K-filter on for every request with a hit (the
     # paper's 0.8 would switch it off on this snapshot: mean KV use ~0.5)
-    r.set_guards(n_min=1, ood=True, k=2, kv_col=4, tau_sat=0.0, tau_ben=0.0)
+    r.set_guards(n_min=1, ood=True, k=2, kv_col=4, tau_sat=0.0, tau_ben=0.0, heuristic=1, count_cols=(0, 1),
+                 theta_imbal=8.0, k_overload=1.0)
 
     def timed(fn):
         ts = []
@@ -110,7 +113,9 @@ def measure_guards(L, r, dw, N, R, d, ring_rows, d_req, flush, stream, peaks, n=
         "status_counts": {"ok": int((st == 0).sum()), "k_filtered": int((st == 4).sum()),
                           "cold_start": int((st == 1).sum()), "out_of_range": int((st == 2).sum())},
         "unfiltered_choices_equal_plain_route": agree,
-        "settings": "n_min 1, out-of-range check on, K 2, kv column 4, tau_sat 0, tau_ben 0",
+        "fallback_distinct_instances": int(torch.unique(o_g["fallback"]).numel()),
+        "settings": "n_min 1, out-of-range check on, K 2, kv column 4, tau_sat 0, tau_ben 0; fallback "
+                    "heuristic of Algorithm 1 (counts = queued + running, theta_imbal 8, k 1)",
     }
 
 

@@ -249,12 +249,26 @@ typedef struct {
     int32_t kv_col;    /* instance-state column holding KV-cache utilisation */
     float tau_sat;     /* filter when mean_i inst[i, kv_col] > tau_sat ... */
     float tau_ben;     /* ... and max_i 16 h[r,i] (kappa_i |r|, hit tokens) > tau_ben */
+    /* Fallback heuristic written to fallback_opt (Algorithm 3 pre-computes it
+     * so that a cold-start / out-of-range status costs the gateway nothing):
+     * LS_HEUR_NONE, LS_HEUR_PREFIX_LOAD (Algorithm 1) or LS_HEUR_PREFIX
+     * (Algorithm 2). */
+    int32_t heuristic;
+    int32_t count_col[2];  /* request count c_i = inst[i, count_col[0]] (+ inst[i, count_col[1]]
+                              when count_col[1] >= 0), fp32 */
+    float theta_imbal;     /* Algorithm 1: c_max - c_min > theta_imbal -> least loaded */
+    float k_overload;      /* Algorithm 1: eligible when c_i <= mean + k_overload * std */
+    float tau_prefix;      /* Algorithm 2: best prefix match kept when m > tau_prefix */
 } ls_guards;
+
+enum { LS_HEUR_NONE = 0, LS_HEUR_PREFIX_LOAD = 1, LS_HEUR_PREFIX = 2 };
 
 /* Set the guard parameters used by later ls_route_batch_guarded calls (host
  * state, read when a route is enqueued or captured).  All off after
- * ls_create.  LS_ERR_ARG for k < 0, k > max_instances, or k > 0 with kv_col
- * outside [0, d_inst). */
+ * ls_create.  LS_ERR_ARG for k < 0, k > max_instances, k > 0 with kv_col
+ * outside [0, d_inst), an unknown heuristic, a heuristic with count_col[0]
+ * outside [0, d_inst) or count_col[1] outside [-1, d_inst), or a heuristic
+ * with max_instances > 1024. */
 int ls_set_guards(ls_ctx *ctx, const ls_guards *g /* host */);
 
 /* Feature bounds of the training buffer (Algorithm 4 input [l, u]): one kernel
@@ -288,12 +302,23 @@ int ls_get_bounds(ls_ctx *ctx, int32_t which, float *lo_out, float *hi_out, void
  *      group, as ls_hash_blocks defines keys); a choice outside them is
  *      replaced by the argmin over them (same order).
  * Exploration and the random tiebreak of Algorithm 4 are not taken
- * (epsilon = 0, equal scores go to the lowest index).  Other arguments, the
- * stream rules and errors are those of ls_route_batch. */
+ * (epsilon = 0, equal scores go to the lowest index).
+ * fallback_opt (DEVICE int32 [n_req], nullable; written when a heuristic is
+ * set): the heuristic's instance for every request, whatever its status.
+ * With m_i = 16 h[r,i] / L (fp32) and c_i the request counts:
+ *   Algorithm 1: if c_max - c_min > theta_imbal (fp64) the least-loaded
+ *     instance; else, with mu and sigma the mean and population standard
+ *     deviation of c (fp64 sums in instance order, two passes), the first
+ *     instance with c_i <= mu + k_overload sigma in the order (m desc, c asc,
+ *     index asc); none: the least loaded.
+ *   Algorithm 2: the largest m (lowest index) if it exceeds tau_prefix, else
+ *     the least loaded.
+ * Least loaded = smallest c_i, lowest index among equals, NaN last.
+ * Other arguments, the stream rules and errors are those of ls_route_batch. */
 int ls_route_batch_guarded(ls_ctx *ctx, int32_t n_req, const int32_t *tok, const int64_t *tok_off,
                            const float *req_feats, int32_t *choice, float *best, int32_t *status,
-                           float *scores_opt, int32_t *hits_opt, uint64_t *weight_version_out,
-                           void *stream);
+                           int32_t *fallback_opt, float *scores_opt, int32_t *hits_opt,
+                           uint64_t *weight_version_out, void *stream);
 
 /* Kernel tracing.  While enabled, each kernel launch of this context is
  * bracketed by CUDA events on its launching stream (a few microseconds of host

@@ -637,7 +637,8 @@ int or_guards(int64_t n_req, int32_t n_inst, const int64_t *L, const uint64_t *g
  *     c asc, index asc); none: argmin_i c_i.
  *   mode 2, Algorithm 2 (prefix aware, threshold tau): i* = argmax m_i
  *     (ties to the lowest index); i* if m_{i*} > tau, else argmin_i c_i.
- * argmin_i c_i takes the lowest index among equal counts. */
+ * argmin_i c_i takes the lowest index among equal counts, NaN after every
+ * number; c_min / c_max skip NaN counts. */
 int or_heuristic(int64_t n_req, int32_t n_inst, const int64_t *L, const int32_t *hits,
                  const float *inst, int d_inst, int mode, int c_col0, int c_col1,
                  float theta_imbal, float k_over, float tau, int32_t *out) {
@@ -649,9 +650,9 @@ int or_heuristic(int64_t n_req, int32_t n_inst, const int64_t *L, const int32_t 
         if (c_col1 >= 0) c[i] = c[i] + inst[(int64_t)i * d_inst + c_col1];
     }
     int32_t least = 0;
-    float cmin = c[0], cmax = c[0];
-    for (int32_t i = 1; i < n_inst; ++i) {
-        if (c[i] < c[least]) least = i;
+    float cmin = INFINITY, cmax = -INFINITY;       /* NaN counts skipped here */
+    for (int32_t i = 0; i < n_inst; ++i) {
+        if (precedes(c[i], i, c[least], least)) least = i;   /* NaN after numbers */
         if (c[i] < cmin) cmin = c[i];
         if (c[i] > cmax) cmax = c[i];
     }

@@ -471,8 +471,8 @@ namespace {
 // One route; `status` non-NULL selects the guarded selection of Algorithm 4
 // (scores are then always materialised and the guard kernel replaces argmin).
 int route_impl(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* tok_off, const float* req_feats,
-               int32_t* choice, float* best, int32_t* status, bool guarded, float* scores_opt, int32_t* hits_opt,
-               uint64_t* weight_version_out, void* stream) {
+               int32_t* choice, float* best, int32_t* status, int32_t* fallback, bool guarded, float* scores_opt,
+               int32_t* hits_opt, uint64_t* weight_version_out, void* stream) {
   if (!h) return fail(LS_ERR_ARG, "ctx is NULL");
   Ctx& c = h->c;
   if (n_req < 0 || n_req > c.cfg.max_requests) return fail(LS_ERR_ARG, "n_req out of range");
@@ -540,7 +540,7 @@ int route_impl(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* tok_
   if (guarded)
     LS_CK(traced(c, TR_GUARDS, 1, s, [&] {
       return launch_guards(c.guards, n_req, c.n_inst, tok, tok_off, hits, scores, c.inst_state, c.cfg.d_inst,
-                           req_feats, c.cfg.d_req, c.pub, c.st, choice, best, status, c.sms, s);
+                           req_feats, c.cfg.d_req, c.pub, c.st, choice, best, status, fallback, c.sms, s);
     }));
   else if (!fused_select)
     LS_CK(traced(c, TR_ARGMIN, 1, s, [&] { return launch_argmin(n_req, c.n_inst, scores, choice, best, s); }));
@@ -559,15 +559,16 @@ extern "C" {
 int ls_route_batch(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* tok_off,
                    const float* req_feats, int32_t* choice, float* best, float* scores_opt,
                    int32_t* hits_opt, uint64_t* weight_version_out, void* stream) {
-  return route_impl(h, n_req, tok, tok_off, req_feats, choice, best, nullptr, false, scores_opt, hits_opt,
+  return route_impl(h, n_req, tok, tok_off, req_feats, choice, best, nullptr, nullptr, false, scores_opt, hits_opt,
                     weight_version_out, stream);
 }
 
 int ls_route_batch_guarded(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* tok_off,
                            const float* req_feats, int32_t* choice, float* best, int32_t* status,
-                           float* scores_opt, int32_t* hits_opt, uint64_t* weight_version_out, void* stream) {
-  return route_impl(h, n_req, tok, tok_off, req_feats, choice, best, status, true, scores_opt, hits_opt,
-                    weight_version_out, stream);
+                           int32_t* fallback_opt, float* scores_opt, int32_t* hits_opt, uint64_t* weight_version_out,
+                           void* stream) {
+  return route_impl(h, n_req, tok, tok_off, req_feats, choice, best, status, fallback_opt, true, scores_opt,
+                    hits_opt, weight_version_out, stream);
 }
 
 int ls_set_guards(ls_ctx* h, const ls_guards* g) {
@@ -576,6 +577,13 @@ int ls_set_guards(ls_ctx* h, const ls_guards* g) {
   if (g->k < 0 || g->k > c.cfg.max_instances) return fail(LS_ERR_ARG, "k out of range");
   if (g->k > 0 && (g->kv_col < 0 || g->kv_col >= c.cfg.d_inst))
     return fail(LS_ERR_ARG, "kv_col outside the instance-state columns");
+  if (g->heuristic < LS_HEUR_NONE || g->heuristic > LS_HEUR_PREFIX) return fail(LS_ERR_ARG, "unknown heuristic");
+  if (g->heuristic != LS_HEUR_NONE) {
+    if (g->count_col[0] < 0 || g->count_col[0] >= c.cfg.d_inst || g->count_col[1] < -1 ||
+        g->count_col[1] >= c.cfg.d_inst)
+      return fail(LS_ERR_ARG, "count_col outside the instance-state columns");
+    if (c.cfg.max_instances > kGuardHeurMaxInst) return fail(LS_ERR_ARG, "heuristic needs max_instances <= 1024");
+  }
   c.guards = *g;
   return LS_OK;
 }

@@ -364,7 +364,9 @@ cudaError_t launch_ring_bounds(int d, const float* ring_x, int64_t capacity, uin
 cudaError_t launch_guards(const ls_guards& g, int n_req, int n_inst, const int32_t* tok, const int64_t* tok_off,
                           const int32_t* hits, const float* scores, const float* inst, int d_inst,
                           const float* req, int d_req, const Published* pub, const DevState* st,
-                          int32_t* choice, float* best, int32_t* status, int sms, cudaStream_t s);
+                          int32_t* choice, float* best, int32_t* status, int32_t* fallback, int sms,
+                          cudaStream_t s);
+constexpr int kGuardHeurMaxInst = 1024;  // instances the heuristic keeps in shared memory
 
 bool plan_tc(const MlpDesc& m, TcPlan& p);
 // Publish the master weights into buffer 1 - st->cur (fp32 params, the

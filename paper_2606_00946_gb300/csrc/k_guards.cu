@@ -164,9 +164,13 @@ struct GuardArgs {
   int64_t h_ben;       // 16 h > tau_ben  <=>  h >= h_ben (h an integer; set on the host)
   int ood, K, kv_col;
   float tau_sat;
+  // fallback heuristic (Algorithm 1: heur 1; Algorithm 2: heur 2; 0 = none)
+  int heur, c_col0, c_col1;
+  float theta_imbal, k_over, tau_prefix;
   int32_t* choice;
   float* best;
   int32_t* status;
+  int32_t* fallback;
 };
 
 // (wa, a) ranks before (wb, b) in rendezvous order: larger weight, then lower index.
@@ -176,14 +180,21 @@ __device__ __forceinline__ bool hrw_before(uint64_t wa, int a, uint64_t wb, int 
 
 __device__ __forceinline__ bool in_range(float x, float lo, float hi) { return x >= lo && x <= hi; }
 
-constexpr int kHashedInst = 1024;  // instance hashes kept in shared memory up to this count
+constexpr int kHashedInst = kGuardHeurMaxInst;  // instance hashes kept in shared memory up to this count
 constexpr int kGuardThreads = 256;  // warp 0: batch-wide terms; warps 1..7: requests
-constexpr int kBarBatch = 1, kBarInst = 2;
+constexpr int kBarBatch = 1, kBarInst = 2, kBarHeur = 3;
 
 // Warp 0 of a block computes the terms shared by the whole batch and hands
 // them over through named barriers, while warps 1..7 work on requests:
 //   kBarBatch  instance hashes mix64((i + 1) G) and the gpu_kv decision;
+//   kBarHeur   the heuristic's request counts, the least-loaded instance,
+//              imbalance and which instances are within mu + k sigma;
 //   kBarInst   whether some instance-state value lies outside its bounds.
+// The heuristic (Algorithm 3 pre-computes it for the gateway's fallback) is
+// formed for every request, cold or not.  Its prefix match ratio
+// m_i = 16 h_i / L orders instances exactly as h_i does for a fixed L (fp32
+// division is monotone, and distinct h < 2^24 give distinct ratios), so the
+// kernel compares hit lengths.
 // Requests: S lanes per request (a group; 32 / S requests per warp).  Lane j
 // of a group takes instances j, j + S, ...; group results meet through
 // log2(S) xor shuffles.  The out-of-range test of the pair features needs
@@ -194,7 +205,9 @@ constexpr int kBarBatch = 1, kBarInst = 2;
 template <int S>
 __global__ void __launch_bounds__(kGuardThreads) k_guards(const __grid_constant__ GuardArgs a) {
   __shared__ uint64_t s_ih[kHashedInst];  // mix64((i + 1) G): the instance half of the rendezvous weight
-  __shared__ int s_kv, s_inst_bad;
+  __shared__ float s_c[kHashedInst];      // heuristic request counts
+  __shared__ uint8_t s_elig[kHashedInst]; // c_i <= mu + k sigma
+  __shared__ int s_kv, s_inst_bad, s_least, s_imb;
   const int N = a.n_inst, d = kPair + a.d_inst + a.d_req;
   const int b = *reinterpret_cast<const volatile int32_t*>(&a.st->route_b);
   const float* lo = a.bounds[b == 1 ? 1 : 0];
@@ -202,9 +215,49 @@ __global__ void __launch_bounds__(kGuardThreads) k_guards(const __grid_constant_
   const bool cold = *reinterpret_cast<const volatile int64_t*>(&a.st->ring_count) < a.n_min;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const bool hashed = !cold && a.K >= 1 && a.K < N && N <= kHashedInst;
+  const bool heur = a.heur != 0 && a.fallback != nullptr;  // the host keeps N <= kHashedInst then
 
   if (warp == 0) {
-    if (cold) return;  // no request warp waits when the batch is cold
+    if (heur) {
+      // request counts, the least-loaded instance (lowest index on ties),
+      // imbalance, and mu + k sigma: fp64 sums in instance order, two passes
+      float cmin = INFINITY, cmax = -INFINITY, cl = INFINITY;
+      int least = N;
+      for (int i = lane; i < N; i += 32) {
+        float c = __ldg(a.inst + (int64_t)i * a.d_inst + a.c_col0);
+        if (a.c_col1 >= 0) c = __fadd_rn(c, __ldg(a.inst + (int64_t)i * a.d_inst + a.c_col1));
+        s_c[i] = c;
+        cmin = fminf(cmin, c);  // NaN counts are skipped by min / max
+        cmax = fmaxf(cmax, c);
+        if (least == N || score_precedes(c, i, cl, least)) { cl = c; least = i; }  // NaN after numbers
+      }
+#pragma unroll
+      for (int o = 16; o; o >>= 1) {
+        cmin = fminf(cmin, __shfl_xor_sync(kFull, cmin, o));
+        cmax = fmaxf(cmax, __shfl_xor_sync(kFull, cmax, o));
+        const float oc = __shfl_xor_sync(kFull, cl, o);
+        const int oi = __shfl_xor_sync(kFull, least, o);
+        if (oi < N && (least == N || score_precedes(oc, oi, cl, least))) { cl = oc; least = oi; }
+      }
+      __syncwarp();
+      double mu = 0.0;
+      for (int i = 0; i < N; ++i) mu = __dadd_rn(mu, (double)s_c[i]);
+      mu = __ddiv_rn(mu, (double)N);
+      double var = 0.0;
+      for (int i = 0; i < N; ++i) {
+        const double dv = __dsub_rn((double)s_c[i], mu);
+        var = __dadd_rn(var, __dmul_rn(dv, dv));
+      }
+      var = __ddiv_rn(var, (double)N);
+      const double thr = __dadd_rn(mu, __dmul_rn((double)a.k_over, __dsqrt_rn(var)));
+      for (int i = lane; i < N; i += 32) s_elig[i] = (double)s_c[i] <= thr;
+      if (lane == 0) {
+        s_least = least;
+        s_imb = __dsub_rn((double)cmax, (double)cmin) > (double)a.theta_imbal;
+      }
+      sm100::named_bar_arrive(kBarHeur, kGuardThreads);
+    }
+    if (cold) return;  // no request warp waits for the rest when the batch is cold
     if (hashed)
       for (int i = lane; i < N; i += 32) s_ih[i] = bh::mix64((uint64_t)(i + 1) * kG);
     // gpu_kv: fp32 sum in instance order (lanes load 32 values at a time, the
@@ -271,14 +324,12 @@ __global__ void __launch_bounds__(kGuardThreads) k_guards(const __grid_constant_
     const int64_t r = it * groups + ((int64_t)blockIdx.x * (kGuardThreads / 32 - 1) + (warp - 1)) * kPerWarp +
                       lane / S;
     const bool live = r < a.n_req;
-    if (cold) {
-      if (live && j == 0) {
-        a.choice[r] = -1;
-        a.best[r] = __int_as_float(0x7fc00000);
-        a.status[r] = LS_ROUTE_COLD_START;
-      }
-      continue;
+    if (cold && live && j == 0) {
+      a.choice[r] = -1;
+      a.best[r] = __int_as_float(0x7fc00000);
+      a.status[r] = LS_ROUTE_COLD_START;
     }
+    if (cold && !heur) continue;
     // --- loads: offsets, then the first block's tokens; hits, scores, extras
     int64_t off = 0, L = 0;
     if (live) {
@@ -326,11 +377,11 @@ __global__ void __launch_bounds__(kGuardThreads) k_guards(const __grid_constant_
     }
 #pragma unroll
     for (int o = 1; o < S; o <<= 1) bad |= __shfl_xor_sync(kFull, bad, o);
-    if (it == 0) {  // the batch-wide terms from warp 0
+    if (it == 0 && !cold) {  // the batch-wide terms from warp 0
       sm100::named_bar_sync(kBarBatch, kGuardThreads);
       kv_ok = s_kv != 0;
     }
-    const bool filter = live && !bad && a.K >= 1 && L >= kBlockTok && kv_ok && (int64_t)hmax >= a.h_ben;
+    const bool filter = live && !cold && !bad && a.K >= 1 && L >= kBlockTok && kv_ok && (int64_t)hmax >= a.h_ben;
     // (a group filters or not as a whole; groups of one warp may differ, so
     // the shuffles below run in every group and only filtering groups use them)
     if (__any_sync(kFull, filter && a.K < N)) {
@@ -385,6 +436,43 @@ __global__ void __launch_bounds__(kGuardThreads) k_guards(const __grid_constant_
       }
       if (filter && a.K < N && !in) { bv = cv; bi = ci; }
     }
+    if (heur) {
+      if (it == 0) sm100::named_bar_sync(kBarHeur, kGuardThreads);
+      // Algorithm 1: the first eligible instance in the order (m desc, c asc,
+      // index asc); Algorithm 2: argmax m (lowest index), kept if m > tau
+      int hh = -1, hx = -1;
+      float hc = 0.0f;
+      if (live)
+        for (int i = j; i < N; i += S) {
+          if (a.heur == 1 && !s_elig[i]) continue;
+          const int h = __ldg(hr + i);
+          const float c = s_c[i];
+          if (hx < 0 || h > hh || (h == hh && a.heur == 1 && (c < hc || (c == hc && i < hx))) ||
+              (h == hh && a.heur == 2 && i < hx)) {
+            hh = h;
+            hc = c;
+            hx = i;
+          }
+        }
+#pragma unroll
+      for (int o = 1; o < S; o <<= 1) {
+        const int oh = __shfl_xor_sync(kFull, hh, o), oi = __shfl_xor_sync(kFull, hx, o);
+        const float oc = __shfl_xor_sync(kFull, hc, o);
+        if (oi >= 0 && (hx < 0 || oh > hh || (oh == hh && a.heur == 1 && (oc < hc || (oc == hc && oi < hx))) ||
+                        (oh == hh && a.heur == 2 && oi < hx))) {
+          hh = oh;
+          hc = oc;
+          hx = oi;
+        }
+      }
+      if (live && j == 0) {
+        int pick = s_least;
+        if (a.heur == 1 && !s_imb && hx >= 0) pick = hx;
+        if (a.heur == 2 && raw_feature(3, L, hh, nullptr, 0, nullptr) > a.tau_prefix) pick = hx;
+        a.fallback[r] = pick;
+      }
+    }
+    if (cold) continue;
     if (it == 0) {  // out-of-range instance state puts every request out of range
       sm100::named_bar_sync(kBarInst, kGuardThreads);
       inst_bad = s_inst_bad != 0;
@@ -417,7 +505,8 @@ cudaError_t launch_ring_bounds(int d, const float* ring_x, int64_t capacity, uin
 cudaError_t launch_guards(const ls_guards& g, int n_req, int n_inst, const int32_t* tok, const int64_t* tok_off,
                           const int32_t* hits, const float* scores, const float* inst, int d_inst,
                           const float* req, int d_req, const Published* pub, const DevState* st,
-                          int32_t* choice, float* best, int32_t* status, int sms, cudaStream_t s) {
+                          int32_t* choice, float* best, int32_t* status, int32_t* fallback, int sms,
+                          cudaStream_t s) {
   if (n_req <= 0) return cudaSuccess;
   GuardArgs a{};
   a.n_req = n_req;
@@ -447,6 +536,13 @@ cudaError_t launch_guards(const ls_guards& g, int n_req, int n_inst, const int32
   a.choice = choice;
   a.best = best;
   a.status = status;
+  a.fallback = fallback;
+  a.heur = g.heuristic;
+  a.c_col0 = g.count_col[0];
+  a.c_col1 = g.count_col[1];
+  a.theta_imbal = g.theta_imbal;
+  a.k_over = g.k_overload;
+  a.tau_prefix = g.tau_prefix;
   constexpr int S = 8;
   const int64_t per_block = (kGuardThreads / 32 - 1) * (32 / S);
   const int grid = (int)std::min<int64_t>(((int64_t)n_req + per_block - 1) / per_block, (int64_t)sms * 8);

@@ -120,14 +120,16 @@ class Router:
         choice = o.get("choice", torch.empty(n_req, dtype=torch.int32, device="cuda"))
         best = o.get("best", torch.empty(n_req, dtype=torch.float32, device="cuda"))
         status = o.get("status", torch.empty(n_req, dtype=torch.int32, device="cuda"))
+        fallback = o.get("fallback", torch.empty(n_req, dtype=torch.int32, device="cuda"))
         scores = o.get("scores") if "scores" in o else (
             torch.empty(n_req, n_inst, dtype=torch.float32, device="cuda") if want_scores else None)
         hits = o.get("hits") if "hits" in o else (
             torch.empty(n_req, n_inst, dtype=torch.int32, device="cuda") if want_hits else None)
         rc, ver = L.ls_route_batch_guarded(self.h, n_req, tok, tok_off, req_feats, choice, best, status,
-                                           scores, hits, stream)
+                                           fallback, scores, hits, stream)
         L.check(rc)
-        return dict(choice=choice, best=best, status=status, scores=scores, hits=hits, version=ver)
+        return dict(choice=choice, best=best, status=status, fallback=fallback, scores=scores, hits=hits,
+                    version=ver)
 
     def set_guards(self, **kw):
         L.check(L.ls_set_guards(self.h, **kw))

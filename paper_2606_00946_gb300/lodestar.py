@@ -25,6 +25,7 @@ LS_STATIC_MAX_BLOCKS, LS_STATIC_MAX_PAIRS = 262144, 262144
 LS_PREFIX_AUTO, LS_PREFIX_TWO_PHASE, LS_PREFIX_FUSED, LS_PREFIX_INDEX = 0, 1, 2, 3
 PREFIX_MODES = {"auto": 0, "two_phase": 1, "fused": 2, "index": 3}
 LS_ROUTE_OK, LS_ROUTE_COLD_START, LS_ROUTE_OOD, LS_ROUTE_KFILTER = 0, 1, 2, 4
+LS_HEUR_NONE, LS_HEUR_PREFIX_LOAD, LS_HEUR_PREFIX = 0, 1, 2
 
 
 class ls_config(C.Structure):
@@ -44,7 +45,9 @@ class ls_info(C.Structure):
 
 class ls_guards(C.Structure):
     _fields_ = [("n_min", C.c_int64), ("ood", C.c_int32), ("k", C.c_int32), ("kv_col", C.c_int32),
-                ("tau_sat", C.c_float), ("tau_ben", C.c_float)]
+                ("tau_sat", C.c_float), ("tau_ben", C.c_float), ("heuristic", C.c_int32),
+                ("count_col", C.c_int32 * 2), ("theta_imbal", C.c_float), ("k_overload", C.c_float),
+                ("tau_prefix", C.c_float)]
 
 
 class ls_trace_entry(C.Structure):
@@ -75,7 +78,7 @@ _SIGS = {
     "ls_set_guards": (C.c_int, [_P, C.POINTER(ls_guards)]),
     "ls_refresh_bounds": (C.c_int, [_P, _P]),
     "ls_get_bounds": (C.c_int, [_P, _i32, _P, _P, _P]),
-    "ls_route_batch_guarded": (C.c_int, [_P, _i32, _P, _P, _P, _P, _P, _P, _P, _P,
+    "ls_route_batch_guarded": (C.c_int, [_P, _i32, _P, _P, _P, _P, _P, _P, _P, _P, _P,
                                          C.POINTER(C.c_uint64), _P]),
     "ls_trace_enable": (C.c_int, [_P, _i32]),
     "ls_trace_read": (C.c_int, [_P, C.POINTER(ls_trace_entry), _i32, C.POINTER(_i32)]),
@@ -254,8 +257,11 @@ def ls_publish(ctx, stream=None) -> int:
     return lib().ls_publish(ctx, stream_handle(stream))
 
 
-def ls_set_guards(ctx, n_min=0, ood=False, k=0, kv_col=0, tau_sat=0.8, tau_ben=0.0) -> int:
-    g = ls_guards(int(n_min), 1 if ood else 0, int(k), int(kv_col), float(tau_sat), float(tau_ben))
+def ls_set_guards(ctx, n_min=0, ood=False, k=0, kv_col=0, tau_sat=0.8, tau_ben=0.0, heuristic=0,
+                  count_cols=(0, 1), theta_imbal=8.0, k_overload=1.0, tau_prefix=0.5) -> int:
+    g = ls_guards(int(n_min), 1 if ood else 0, int(k), int(kv_col), float(tau_sat), float(tau_ben),
+                  int(heuristic), (C.c_int32 * 2)(int(count_cols[0]), int(count_cols[1])), float(theta_imbal),
+                  float(k_overload), float(tau_prefix))
     return lib().ls_set_guards(ctx, C.byref(g))
 
 
@@ -267,13 +273,13 @@ def ls_get_bounds(ctx, which, lo_out, hi_out, stream=None) -> int:
     return lib().ls_get_bounds(ctx, int(which), ptr(lo_out), ptr(hi_out), stream_handle(stream))
 
 
-def ls_route_batch_guarded(ctx, n_req, tok, tok_off, req_feats, choice, best, status, scores_opt=None,
-                           hits_opt=None, stream=None):
+def ls_route_batch_guarded(ctx, n_req, tok, tok_off, req_feats, choice, best, status, fallback_opt=None,
+                           scores_opt=None, hits_opt=None, stream=None):
     """Returns (status code of the call, weight_version)."""
     v = C.c_uint64(0)
     rc = lib().ls_route_batch_guarded(ctx, int(n_req), ptr(tok), ptr(tok_off), ptr(req_feats), ptr(choice),
-                                      ptr(best), ptr(status), ptr(scores_opt), ptr(hits_opt), C.byref(v),
-                                      stream_handle(stream))
+                                      ptr(best), ptr(status), ptr(fallback_opt), ptr(scores_opt), ptr(hits_opt),
+                                      C.byref(v), stream_handle(stream))
     return rc, v.value
 
 

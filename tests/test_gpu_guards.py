@@ -238,3 +238,77 @@ def test_set_guards_rejects_bad_arguments():
     assert L.ls_set_guards(r.h, k=2, kv_col=cfg.d_inst) == L.LS_ERR_ARG
     assert L.ls_set_guards(r.h, k=2, kv_col=KV_COL) == L.LS_OK
     r.close()
+
+
+# ----------------------------------------------------------------------------
+# fallback heuristics (Algorithms 1 and 2, pre-computed as Algorithm 3 does)
+# ----------------------------------------------------------------------------
+
+HEUR_CASES = [
+    ("tiny", {}),
+    ("homogeneous", {}),
+    ("homogeneous", {"n_inst": 24, "n_req": 512, "cache_blocks": 1024}),
+    ("homogeneous", {"n_inst": 40, "n_req": 512, "cache_blocks": 1024}),
+    ("homogeneous", {"n_inst": 7, "n_req": 300, "cache_blocks": 1024}),
+]
+
+
+@pytest.mark.parametrize("name,over", HEUR_CASES)
+def test_fallback_heuristic_parity(name, over):
+    cfg = _cfg(name, n_samples=0, **over)
+    g = dict(n_min=1, ood=True, k=2, kv_col=KV_COL, tau_sat=0.3, tau_ben=0.0)
+    wl, dw, r, out, lo, hi, count = _guard_case(cfg, 4096, g)
+    L_ = np.diff(wl.tok_off)
+    c = wl.inst_state[:, 0] + wl.inst_state[:, 1]
+    spread = float(c.max() - c.min())
+    settings = [
+        dict(heuristic=1, count_cols=(0, 1), theta_imbal=spread + 1.0, k_overload=1.0),   # balanced
+        dict(heuristic=1, count_cols=(0, 1), theta_imbal=spread + 1.0, k_overload=-0.5),
+        dict(heuristic=1, count_cols=(0, 1), theta_imbal=spread - 0.5, k_overload=1.0),   # imbalanced
+        dict(heuristic=1, count_cols=(1, -1), theta_imbal=1e9, k_overload=0.0),
+        dict(heuristic=2, count_cols=(0, 1), tau_prefix=0.5),
+        dict(heuristic=2, count_cols=(0, -1), tau_prefix=0.05),
+    ]
+    picks = set()
+    for hs in settings:
+        r.set_guards(**g, **hs)
+        got = r.route_guarded(dw.tok, dw.tok_off, dw.req_feats, cfg.n_inst)
+        want = oracle.heuristic(L_, got["hits"].cpu().numpy(), wl.inst_state, mode=hs["heuristic"],
+                                count_cols=hs["count_cols"], theta_imbal=hs.get("theta_imbal", 8.0),
+                                k=hs.get("k_overload", 1.0), tau=hs.get("tau_prefix", 0.5))
+        np.testing.assert_array_equal(got["fallback"].cpu().numpy(), want)
+        # the guarded selection itself is unchanged by the heuristic
+        _assert_same(got, _oracle_guards(wl, got, lo, hi, count, g))
+        picks.add(len(np.unique(want)))
+    assert max(picks) > 1                              # some setting spreads the requests
+    # cold batch: the heuristic is still formed for every request
+    r.set_guards(**dict(g, n_min=count + 1), **settings[0])
+    got = r.route_guarded(dw.tok, dw.tok_off, dw.req_feats, cfg.n_inst)
+    assert (got["status"] == L.LS_ROUTE_COLD_START).all()
+    want = oracle.heuristic(L_, got["hits"].cpu().numpy(), wl.inst_state, mode=1, count_cols=(0, 1),
+                            theta_imbal=spread + 1.0, k=1.0)
+    np.testing.assert_array_equal(got["fallback"].cpu().numpy(), want)
+    r.close()
+
+
+def test_fallback_heuristic_nan_counts_and_bad_arguments():
+    cfg = _cfg("tiny", n_samples=0)
+    wl, dw, r = _staged(cfg, 1024)
+    st = wl.inst_state.copy()
+    st[0, 0] = np.nan                                  # NaN count: never least loaded, never eligible
+    st[3, 0] = st[5, 0] = 0.0
+    st[3, 1] = st[5, 1] = 0.0
+    r.snapshot(cfg.n_inst, torch.from_numpy(st).cuda())
+    L_ = np.diff(wl.tok_off)
+    for hs in (dict(heuristic=1, theta_imbal=1e9, k_overload=1.0), dict(heuristic=1, theta_imbal=0.0),
+               dict(heuristic=2, tau_prefix=0.99)):
+        r.set_guards(**hs)
+        got = r.route_guarded(dw.tok, dw.tok_off, dw.req_feats, cfg.n_inst)
+        want = oracle.heuristic(L_, got["hits"].cpu().numpy(), st, mode=hs["heuristic"],
+                                theta_imbal=hs.get("theta_imbal", 8.0), k=hs.get("k_overload", 1.0),
+                                tau=hs.get("tau_prefix", 0.5))
+        np.testing.assert_array_equal(got["fallback"].cpu().numpy(), want)
+    assert L.ls_set_guards(r.h, heuristic=3) == L.LS_ERR_ARG
+    assert L.ls_set_guards(r.h, heuristic=1, count_cols=(cfg.d_inst, -1)) == L.LS_ERR_ARG
+    assert L.ls_set_guards(r.h, heuristic=1, count_cols=(0, -2)) == L.LS_ERR_ARG
+    r.close()
