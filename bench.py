@@ -67,7 +67,7 @@ def measure_guards(L, r, dw, N, R, d, ring_rows, d_req, flush, stream, peaks, n=
     # tau_sat = 0 keeps the K-filter on for every request with a hit (the
     # paper's 0.8 would switch it off on this snapshot: mean KV use ~0.5)
     r.set_guards(n_min=1, ood=True, k=2, kv_col=4, tau_sat=0.0, tau_ben=0.0, heuristic=1, count_cols=(0, 1),
-                 theta_imbal=8.0, k_overload=1.0)
+                 theta_imbal=128.0, k_overload=1.0)
 
     def timed(fn):
         ts = []
@@ -115,7 +115,8 @@ def measure_guards(L, r, dw, N, R, d, ring_rows, d_req, flush, stream, peaks, n=
         "unfiltered_choices_equal_plain_route": agree,
         "fallback_distinct_instances": int(torch.unique(o_g["fallback"]).numel()),
         "settings": "n_min 1, out-of-range check on, K 2, kv column 4, tau_sat 0, tau_ben 0; fallback "
-                    "heuristic of Algorithm 1 (counts = queued + running, theta_imbal 8, k 1)",
+                    "heuristic of Algorithm 1 (counts = queued + running, theta_imbal 128 so that the per-request "
+                    "order decides, k 1)",
     }
 
 

@@ -306,9 +306,10 @@ int ls_get_bounds(ls_ctx *ctx, int32_t which, float *lo_out, float *hi_out, void
  * fallback_opt (DEVICE int32 [n_req], nullable; written when a heuristic is
  * set): the heuristic's instance for every request, whatever its status.
  * With m_i = 16 h[r,i] / L (fp32) and c_i the request counts:
- *   Algorithm 1: if c_max - c_min > theta_imbal (fp64) the least-loaded
+ *   Algorithm 1: if c_max - c_min > theta_imbal (fp32) the least-loaded
  *     instance; else, with mu and sigma the mean and population standard
- *     deviation of c (fp64 sums in instance order, two passes), the first
+ *     deviation of c (fp32, sums in instance order, two passes, each
+ *     operation rounded on its own, sqrt correctly rounded), the first
  *     instance with c_i <= mu + k_overload sigma in the order (m desc, c asc,
  *     index asc); none: the least loaded.
  *   Algorithm 2: the largest m (lowest index) if it exceeds tau_prefix, else

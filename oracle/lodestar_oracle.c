@@ -630,11 +630,11 @@ int or_guards(int64_t n_req, int32_t n_inst, const int64_t *L, const uint64_t *g
  * and per pair the prefix match ratio m_i = kappa = 16 h / L (fp32, 0 when
  * L = 0).
  *   mode 1, Algorithm 1 (prefix-cache and load aware):
- *     if c_max - c_min > theta_imbal (fp64): argmin_i c_i;
- *     else mu = mean c, sigma = population standard deviation (fp64 sums in
- *     index order, two passes, sqrt correctly rounded), and among the
- *     instances with c_i <= mu + k sigma the first in the order (m desc,
- *     c asc, index asc); none: argmin_i c_i.
+ *     if c_max - c_min > theta_imbal (fp32): argmin_i c_i;
+ *     else mu = mean c, sigma = population standard deviation (fp32: sums in
+ *     index order, two passes, every operation rounded on its own, sqrt
+ *     correctly rounded), and among the instances with c_i <= mu + k sigma
+ *     the first in the order (m desc, c asc, index asc); none: argmin_i c_i.
  *   mode 2, Algorithm 2 (prefix aware, threshold tau): i* = argmax m_i
  *     (ties to the lowest index); i* if m_{i*} > tau, else argmin_i c_i.
  * argmin_i c_i takes the lowest index among equal counts, NaN after every
@@ -656,16 +656,16 @@ int or_heuristic(int64_t n_req, int32_t n_inst, const int64_t *L, const int32_t 
         if (c[i] < cmin) cmin = c[i];
         if (c[i] > cmax) cmax = c[i];
     }
-    double mu = 0.0, var = 0.0;
-    for (int32_t i = 0; i < n_inst; ++i) mu += (double)c[i];
-    mu = mu / (double)n_inst;
+    float mu = 0.0f, var = 0.0f;
+    for (int32_t i = 0; i < n_inst; ++i) mu += c[i];
+    mu = mu / (float)n_inst;
     for (int32_t i = 0; i < n_inst; ++i) {
-        double dv = (double)c[i] - mu;
+        float dv = c[i] - mu;
         var += dv * dv;
     }
-    var = var / (double)n_inst;
-    double thr = mu + (double)k_over * sqrt(var);
-    int imbalanced = (double)cmax - (double)cmin > (double)theta_imbal;
+    var = var / (float)n_inst;
+    float thr = mu + k_over * sqrtf(var);
+    int imbalanced = cmax - cmin > theta_imbal;
     for (int64_t r = 0; r < n_req; ++r) {
         const int32_t *hr = hits + r * n_inst;
         for (int32_t i = 0; i < n_inst; ++i) {
@@ -676,7 +676,7 @@ int or_heuristic(int64_t n_req, int32_t n_inst, const int64_t *L, const int32_t 
         if (mode == 1 && !imbalanced) {
             int32_t b = -1;
             for (int32_t i = 0; i < n_inst; ++i) {
-                if (!((double)c[i] <= thr)) continue;
+                if (!(c[i] <= thr)) continue;
                 if (b < 0 || m[i] > m[b] || (m[i] == m[b] && c[i] < c[b])) b = i;
             }
             if (b >= 0) pick = b;

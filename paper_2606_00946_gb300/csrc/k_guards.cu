@@ -220,7 +220,8 @@ __global__ void __launch_bounds__(kGuardThreads) k_guards(const __grid_constant_
   if (warp == 0) {
     if (heur) {
       // request counts, the least-loaded instance (lowest index on ties),
-      // imbalance, and mu + k sigma: fp64 sums in instance order, two passes
+      // imbalance, and mu + k sigma: fp32 sums in instance order, two passes,
+      // every operation rounded on its own (no fused multiply-add)
       float cmin = INFINITY, cmax = -INFINITY, cl = INFINITY;
       int least = N;
       for (int i = lane; i < N; i += 32) {
@@ -240,20 +241,22 @@ __global__ void __launch_bounds__(kGuardThreads) k_guards(const __grid_constant_
         if (oi < N && (least == N || score_precedes(oc, oi, cl, least))) { cl = oc; least = oi; }
       }
       __syncwarp();
-      double mu = 0.0;
-      for (int i = 0; i < N; ++i) mu = __dadd_rn(mu, (double)s_c[i]);
-      mu = __ddiv_rn(mu, (double)N);
-      double var = 0.0;
+      float mu = 0.0f;
+#pragma unroll 8
+      for (int i = 0; i < N; ++i) mu = __fadd_rn(mu, s_c[i]);
+      mu = __fdiv_rn(mu, (float)N);
+      float var = 0.0f;
+#pragma unroll 8
       for (int i = 0; i < N; ++i) {
-        const double dv = __dsub_rn((double)s_c[i], mu);
-        var = __dadd_rn(var, __dmul_rn(dv, dv));
+        const float dv = __fsub_rn(s_c[i], mu);
+        var = __fadd_rn(var, __fmul_rn(dv, dv));
       }
-      var = __ddiv_rn(var, (double)N);
-      const double thr = __dadd_rn(mu, __dmul_rn((double)a.k_over, __dsqrt_rn(var)));
-      for (int i = lane; i < N; i += 32) s_elig[i] = (double)s_c[i] <= thr;
+      var = __fdiv_rn(var, (float)N);
+      const float thr = __fadd_rn(mu, __fmul_rn(a.k_over, __fsqrt_rn(var)));
+      for (int i = lane; i < N; i += 32) s_elig[i] = s_c[i] <= thr;
       if (lane == 0) {
         s_least = least;
-        s_imb = __dsub_rn((double)cmax, (double)cmin) > (double)a.theta_imbal;
+        s_imb = __fsub_rn(cmax, cmin) > a.theta_imbal;
       }
       sm100::named_bar_arrive(kBarHeur, kGuardThreads);
     }

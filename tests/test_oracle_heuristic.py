@@ -65,7 +65,7 @@ def test_alg1_overload_bound_is_inclusive():
     hits = np.array([[0, 0, 4, 1]], np.int32)        # best prefix match on instance 2 (c = 3)
     inst = np.array([[1, 0], [1, 0], [3, 0], [3, 0]], np.float32)
     assert oracle.heuristic(L, hits, inst, mode=1, count_cols=(0, -1), theta_imbal=99, k=1.0)[0] == 2
-    k_less = float(np.nextafter(np.float32(1.0), np.float32(0)))
+    k_less = 1.0 - 2.0 ** -22     # 2 + k_less = 3 - ulp(3) in fp32: the bound falls just below 3
     # just below: instances 2 and 3 are overloaded; the best of 0 and 1 (m equal, c equal) is 0
     assert oracle.heuristic(L, hits, inst, mode=1, count_cols=(0, -1), theta_imbal=99, k=k_less)[0] == 0
 
