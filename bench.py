@@ -469,24 +469,49 @@ def main():
     ms = max_over_ranks(world, float(np.mean(times)), dev if world > 1 and torch.distributed.get_backend() == "nccl" else None)
     value = world * R / (ms / 1e3)
 
-    # roofline of the dominant kernel (largest device time in the timed region)
+    # roofline of the dominant kernel: the largest device time per step on the
+    # step's critical branch (snapshot + route runs beside log + train, and is
+    # the longer branch); the training branch's largest kernel is reported too
     peaks, peak_src = measured_peaks()
     per = {k: v[1] / max(v[2], 1) for k, v in trace.items()}          # ms per timed launch
     per_step = {k: per[k] * v[0] / n_traced for k, v in trace.items()}  # ms per step
-    dom = max(per_step, key=lambda k: per_step[k])
+    n_per_step = {k: v[0] / n_traced for k, v in trace.items()}         # launches per step
     launches = int(round(sum(v[0] for v in trace.values()) * args.steps / n_traced))
-    if dom == "prefix_match":
-        alg, peak, unit, bound = costs["prefix_bytes"] / 1e9, peaks["hbm_gbs"], "GB/s", "hbm"
-    elif dom in ("score_simt", "score_tc"):
-        alg, peak, unit, bound = costs["score_flops"] / 1e12, peaks["bf16_tflops"], "TFLOP/s", "tensor"
-    else:
-        alg, peak, unit, bound = train_flops(cfg.widths, Bt) / 1e12 / 5, peaks["bf16_tflops"], "TFLOP/s", "tensor"
-    achieved = alg / (per[dom] / 1e3)
-    roofline = {"kernel": dom, "bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
-                "frac": achieved / peak, "traffic": profiled_traffic(dom) if dom == "score_tc" else None, "peak_source": f"{peak_src} (burst)",
-                "avg_launch_ms": per[dom],
-                "timing": "kernel durations from CUDA events around each launch over steps issued call by "
-                          "call (instrumented); value and ms_per_step from the K graph replays"}
+    timing = ("kernel durations from CUDA events around each launch over steps issued call by call "
+              "(instrumented); value and ms_per_step from the K graph replays")
+
+    def kernel_roofline(k):
+        d_pad = 64 * ((cfg.d + 63) // 64)
+        if k in ("prefix_index", "prefix_match"):
+            alg, peak, unit, bound = costs["prefix_bytes"] / 1e9, peaks["hbm_gbs"], "GB/s", "hbm"
+        elif k == "features":     # feature image written + hits and offsets read
+            alg = (R * N * (2 * d_pad + 4) + R * 8) / 1e9
+            peak, unit, bound = peaks["hbm_gbs"], "GB/s", "hbm"
+        elif k in ("score_simt", "score_tc"):
+            alg, peak, unit, bound = costs["score_flops"] / 1e12, peaks["bf16_tflops"], "TFLOP/s", "tensor"
+        else:                      # training products: the kind's flops per step over its launches per step
+            # forward launches: every layer's product plus the output layer's dW
+            # (in the last hidden layer's epilogue); dW + dX launches for hidden
+            # layers l >= 1; the dW-only launch for layer 0
+            w, Bk = cfg.widths, Bt
+            nh = len(w) - 2
+            per_kind = {"gemm_tc_fwd": sum(2 * Bk * w[l] * w[l + 1] for l in range(nh + 1)) + 2 * Bk * w[nh],
+                        "gemm_tc_dx": sum(4 * Bk * w[l] * w[l + 1] for l in range(1, nh)),
+                        "gemm_tc_dw": 2 * Bk * w[0] * w[1]}
+            alg = per_kind.get(k, 0.0) / max(n_per_step[k], 1e-9) / 1e12
+            peak, unit, bound = peaks["bf16_tflops"], "TFLOP/s", "tensor"
+        achieved = alg / (per[k] / 1e3)
+        return {"kernel": k, "bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
+                "frac": achieved / peak, "traffic": profiled_traffic(k) if k == "score_tc" else None,
+                "peak_source": f"{peak_src} (burst)", "avg_launch_ms": per[k], "timing": timing}
+
+    route_kernels = [k for k in per_step if k in ("prefix_index", "prefix_match", "hash_screen", "probe_walk",
+                                                  "features", "score_tc", "score_simt", "argmin")]
+    dom = max(route_kernels, key=lambda k: per_step[k])
+    roofline = dict(kernel_roofline(dom), branch="route (the step's critical branch)")
+    train_kernels = [k for k in per_step if k in ("gemm_tc_fwd", "gemm_tc_dw", "gemm_tc_dx")]
+    train_roofline = (dict(kernel_roofline(max(train_kernels, key=lambda k: per_step[k])), branch="train")
+                      if train_kernels else None)
 
     guards = None
     if not args.no_guards:
@@ -589,6 +614,7 @@ def main():
             "train_samples_per_s": world * Bt / (ms / 1e3),
             "scores_per_s": world * R * N / (ms / 1e3),
             "roofline": roofline,
+            "train_roofline": train_roofline,
             "kernels_ms_per_step": {k: per_step[k] for k in sorted(per_step, key=lambda k: -per_step[k])},
             "cpu_baseline": cpu,
             "e2e": e2e,
