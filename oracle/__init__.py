@@ -75,6 +75,9 @@ def lib():
             L.or_ring_bounds.argtypes = [i64, C.c_int, P, i64, P, P]
             L.or_hrw_candidates.restype = i32
             L.or_hrw_candidates.argtypes = [C.c_uint64, i32, i32, P]
+            L.or_replay_embed.argtypes = [C.c_int, C.c_int, P, P, i64, P, P, P, P, P]
+            L.or_replay_distances.argtypes = [i64, P, i64, P, C.c_int, P, P]
+            L.or_replay_select.argtypes = [i64, P, i64, P, i64, P, P]
             L.or_heuristic.argtypes = [i64, i32, P, P, P, C.c_int, C.c_int, C.c_int, C.c_int, C.c_float,
                                        C.c_float, C.c_float, P]
             L.or_guards.argtypes = [i64, i32, P, P, P, P, C.c_int, P, C.c_int, P, P, P, i64, i64,
@@ -367,3 +370,47 @@ def heuristic(L, hits, inst_state, *, mode=1, count_cols=(0, 1), theta_imbal=8.0
     _check(lib().or_heuristic(R, N, _p(L), _p(hits), _p(inst), inst.shape[1], int(mode), int(count_cols[0]),
                               int(c1), float(theta_imbal), float(k), float(tau), _p(out)), "heuristic")
     return out
+
+
+# --------------------------------------------------------------------------
+# two-pool training data (FIFO + replay pool)
+# --------------------------------------------------------------------------
+
+def replay_embed(mode, widths, params, x, y, mean, std) -> np.ndarray:
+    """Gradient embeddings g = (yhat - y) * last hidden activation, [M, H] fp64."""
+    mode = MODES.get(mode, mode)
+    w = _c(widths, np.int32)
+    x = _c(x, np.float32)
+    y = _c(y, np.float32)
+    M = len(y)
+    H = int(w[-2])
+    g = np.zeros((max(M, 1), H), np.float64)
+    _check(lib().or_replay_embed(mode, len(w) - 1, _p(w), _p(_c(params, np.float64)), M,
+                                 _p(x if M else np.zeros(1, np.float32)), _p(y if M else np.zeros(1, np.float32)),
+                                 _p(_c(mean, np.float32)), _p(_c(std, np.float32)), _p(g)), "replay_embed")
+    return g[:M]
+
+
+def replay_distances(gc, gk):
+    """(d per candidate, n per kept): nearest kept squared distance, nearest other kept."""
+    gc = _c(gc, np.float64).reshape(len(gc), -1) if len(gc) else np.zeros((0, 1))
+    gk = _c(gk, np.float64).reshape(len(gk), -1) if len(gk) else np.zeros((0, 1))
+    H = gc.shape[1] if len(gc) else gk.shape[1]
+    d = np.zeros(max(len(gc), 1))
+    n = np.zeros(max(len(gk), 1))
+    one = np.zeros(1)
+    _check(lib().or_replay_distances(len(gc), _p(gc if len(gc) else one), len(gk), _p(gk if len(gk) else one),
+                                     int(H), _p(d), _p(n)), "replay_distances")
+    return d[:len(gc)], n[:len(gk)]
+
+
+def replay_select(d, n, cap):
+    """Admission round: (src per slot of the new pool, new count); src >= 0 is a
+    candidate index, -1 - j keeps kept sample j."""
+    d = _c(d, np.float64)
+    n = _c(n, np.float64)
+    src = np.zeros(max(int(cap), 1), np.int64)
+    cnt = np.zeros(1, np.int64)
+    _check(lib().or_replay_select(len(d), _p(d if len(d) else np.zeros(1)), len(n),
+                                  _p(n if len(n) else np.zeros(1)), int(cap), _p(src), _p(cnt)), "replay_select")
+    return src[:int(cnt[0])], int(cnt[0])

@@ -26,6 +26,8 @@
  *          K-filter of Algorithm 4.
  *   Algorithms 1 and 2 (the comparison heuristics), which Algorithm 3
  *          pre-computes as the gateway's fallback choice.
+ *   Sec. 4.3.2 (Training-data selection): FIFO + replay pool, admission of
+ *          evicted samples by the diversity of their gradient embeddings.
  *
  * Readings where the paper is silent (each also listed in the design notes):
  *   - block hash: SplitMix64 finaliser based content hash, prefix state chained
@@ -42,7 +44,10 @@
  *     ConsistentHash_K = top-K rendezvous hashing; gpu_kv sum in fp32 in
  *     index order; kappa_i |r| = 16 h_i; epsilon = 0, no random tiebreak;
  *   - heuristics: request count = queued + running columns, population
- *     standard deviation, sort ties to the lowest index.
+ *     standard deviation, sort ties to the lowest index;
+ *   - replay admission: one round per call, candidates ranked by distance to
+ *     the nearest kept embedding, kept samples by distance to their nearest
+ *     other kept sample, pairing while it raises diversity (or_replay_select).
  */
 #include <math.h>
 #include <stdint.h>
@@ -688,5 +693,122 @@ int or_heuristic(int64_t n_req, int32_t n_inst, const int64_t *L, const int32_t 
         out[r] = pick;
     }
     free(c); free(m);
+    return 0;
+}
+
+/* ------------------------------------------------------------------------ */
+/* two-pool training data (Sec. 4.3.2 Training-data selection)              */
+/* ------------------------------------------------------------------------ */
+
+/* Gradient embedding of logged records: each raw row is z-scored (fp32) and
+ * run forward (rounding per mode); with a the last hidden activation (the
+ * output layer's input, width H = w[n_layers - 1]) and yhat the prediction,
+ * g = (yhat - y) a, the per-record gradient of the squared error with respect
+ * to the output layer's weights up to the factor 2 ("last-hidden-layer
+ * activations, weighted by prediction residual").  g is [M, H]. */
+int or_replay_embed(int mode, int n_layers, const int *w, const double *params, int64_t M,
+                    const float *x, const float *y, const float *mean, const float *std, double *g) {
+    int d = w[0], m = max_width(n_layers, w), H = w[n_layers - 1];
+    int64_t act_off[17];
+    act_off[0] = 0;
+    for (int l = 0; l < n_layers; ++l) act_off[l + 1] = act_off[l] + w[l];
+    double *ba = (double *)malloc((size_t)m * sizeof(double));
+    double *bb = (double *)malloc((size_t)m * sizeof(double));
+    double *xr = (double *)malloc((size_t)d * sizeof(double));
+    double *acts = (double *)malloc((size_t)act_off[n_layers] * sizeof(double));
+    float *xf = (float *)malloc((size_t)d * sizeof(float));
+    if (!ba || !bb || !xr || !acts || !xf) {
+        free(ba); free(bb); free(xr); free(acts); free(xf);
+        return -1;
+    }
+    for (int64_t s = 0; s < M; ++s) {
+        or_zscore(d, x + s * d, mean, std, xf);
+        for (int k = 0; k < d; ++k) xr[k] = (double)xf[k];
+        double yhat = forward_row(mode, n_layers, w, params, xr, NULL, acts, act_off, ba, bb);
+        double res = yhat - (double)y[s];
+        for (int k = 0; k < H; ++k) g[s * H + k] = res * acts[act_off[n_layers - 1] + k];
+    }
+    free(ba); free(bb); free(xr); free(acts); free(xf);
+    return 0;
+}
+
+/* Squared Euclidean distances between embeddings, written out:
+ *   dcand[e] = min_j ||gc_e - gk_j||^2 over the nk kept embeddings (+inf if none);
+ *   nkept[j] = min_{k != j} ||gk_j - gk_k||^2 (+inf if there is no other). */
+int or_replay_distances(int64_t mc, const double *gc, int64_t nk, const double *gk, int H,
+                        double *dcand, double *nkept) {
+    for (int64_t e = 0; e < mc; ++e) {
+        double best = INFINITY;
+        for (int64_t j = 0; j < nk; ++j) {
+            double s = 0.0;
+            for (int k = 0; k < H; ++k) {
+                double t = gc[e * H + k] - gk[j * H + k];
+                s += t * t;
+            }
+            if (s < best) best = s;
+        }
+        dcand[e] = best;
+    }
+    for (int64_t j = 0; j < nk; ++j) {
+        double best = INFINITY;
+        for (int64_t q = 0; q < nk; ++q) {
+            if (q == j) continue;
+            double s = 0.0;
+            for (int k = 0; k < H; ++k) {
+                double t = gk[j * H + k] - gk[q * H + k];
+                s += t * t;
+            }
+            if (s < best) best = s;
+        }
+        nkept[j] = best;
+    }
+    return 0;
+}
+
+/* key for ranking: NaN counts as -inf (no diversity) */
+static double div_key(double v) { return isnan(v) ? -INFINITY : v; }
+
+/* One admission round of the replay pool (reading of the two-pool design:
+ * evicted samples are admitted when they are the most diverse with respect
+ * to those kept).  Candidates are ranked by (dcand desc, index asc), kept
+ * samples by (nkept asc, slot asc); free = cap - nk.  The candidate of rank
+ * t < free fills slot nk + t; the candidate of rank free + q replaces the
+ * kept sample of rank q when its dcand exceeds that sample's nkept (both
+ * sequences are monotone, so the replacements are a prefix).
+ * src[s] for the new pool's slots s < *new_count: c >= 0 = candidate c,
+ * -1 - j = kept sample j stays. */
+int or_replay_select(int64_t mc, const double *dcand, int64_t nk, const double *nkept, int64_t cap,
+                     int64_t *src, int64_t *new_count) {
+    int64_t *oc = (int64_t *)malloc((size_t)(mc > 0 ? mc : 1) * sizeof(int64_t));
+    int64_t *ok = (int64_t *)malloc((size_t)(nk > 0 ? nk : 1) * sizeof(int64_t));
+    if (!oc || !ok) { free(oc); free(ok); return -1; }
+    /* rank by counting: rank_e = #{e' ranked before e} */
+    for (int64_t e = 0; e < mc; ++e) {
+        int64_t r = 0;
+        for (int64_t f = 0; f < mc; ++f) {
+            double a = div_key(dcand[f]), b = div_key(dcand[e]);
+            if (a > b || (a == b && f < e)) ++r;
+        }
+        oc[r] = e;
+    }
+    for (int64_t j = 0; j < nk; ++j) {
+        int64_t r = 0;
+        for (int64_t q = 0; q < nk; ++q) {
+            double a = div_key(nkept[q]), b = div_key(nkept[j]);
+            if (a < b || (a == b && q < j)) ++r;
+        }
+        ok[r] = j;
+    }
+    for (int64_t s = 0; s < nk; ++s) src[s] = -1 - s;
+    int64_t free_slots = cap - nk, t = 0;
+    for (; t < mc && t < free_slots; ++t) src[nk + t] = oc[t];
+    int64_t count = nk + t;
+    for (int64_t q = 0; t + q < mc && q < nk; ++q) {
+        int64_t c = oc[t + q], j = ok[q];
+        if (!(div_key(dcand[c]) > div_key(nkept[j]))) break;
+        src[j] = c;
+    }
+    *new_count = count;
+    free(oc); free(ok);
     return 0;
 }
