@@ -99,6 +99,13 @@ typedef struct {
                                             for bf16 predictors whose hidden widths are
                                             multiples of 64 (<= 512), CUDA cores otherwise;
                                             TENSOR_CORES on an unsupported shape -> LS_ERR_ARG */
+    /* Two-pool training data (Sec. 4.3.2): the sample ring is the FIFO pool;
+     * replay_capacity > 0 adds a replay pool of that many records, fed by
+     * ls_replay_admit from the records the FIFO evicted, which wait in a
+     * pending ring of pending_capacity records (>= 1 with a replay pool, 0
+     * without).  0 / 0: FIFO only. */
+    int64_t replay_capacity;
+    int64_t pending_capacity;
 } ls_config;
 
 typedef struct {
@@ -110,6 +117,8 @@ typedef struct {
     int64_t train_steps;         /* training steps taken */
     uint64_t weight_version;     /* version of the last published weights, 0 = none */
     int32_t scorer;              /* LS_SCORER_CUDA_CORES or LS_SCORER_TENSOR_CORES in use */
+    int64_t replay_count;        /* records in the replay pool */
+    int64_t pending_count;       /* evicted records waiting for ls_replay_admit */
 } ls_info;
 
 /* Number of predictor parameters: sum over layers of out*in + out. */
@@ -207,13 +216,20 @@ int ls_route_batch(ls_ctx *ctx, int32_t n_req, const int32_t *tok, const int64_t
 /* Append n logged records (raw feature rows feats [n, d], observed TTFT in
  * seconds ttft [n]) to the sample ring: record j goes to slot
  * (count + j) mod ring_capacity, evicting the oldest (Sec. 4.3.2); count is
- * the number of records appended before, kept on the device. */
+ * the number of records appended before, kept on the device.  With a replay
+ * pool, every record the call evicts is first copied to the pending ring
+ * (the record at stream position p to pending slot p mod pending_capacity,
+ * overwriting the oldest pending record when full), and n must not exceed
+ * ring_capacity (LS_ERR_ARG). */
 int ls_log_samples(ls_ctx *ctx, int32_t n, const float *feats, const float *ttft, void *stream);
 
-/* One minibatch step of the predictor on ring slots idx [batch] (int32 on the
- * device; NULL = slots (k*batch + j) mod min(count, capacity) at step k; k and
- * count are the device counters when the step runs; an empty ring at that
- * point latches LS_ERR_STATE).
+/* One minibatch step of the predictor on the training buffer F u R (Sec.
+ * 4.3.2): index u < nF is ring slot u, nF <= u < nF + nR is replay record
+ * u - nF (nF = min(count, ring_capacity), nR = records in the replay pool,
+ * 0 without one).  idx [batch] int32 on the device; NULL = indices
+ * (k*batch + j) mod (nF + nR) at step k; k, count and nR are the device
+ * counters when the step runs; an empty buffer at that point latches
+ * LS_ERR_STATE).
  * Loss = mean squared error of the predicted TTFT (seconds).  opt LS_SGD:
  * theta -= lr g; LS_ADAM: beta1 0.9, beta2 0.999, eps 1e-8, bias-corrected.
  * Updates the master weights only; routing sees them after ls_publish.
@@ -273,13 +289,38 @@ int ls_set_guards(ls_ctx *ctx, const ls_guards *g /* host */);
 
 /* Feature bounds of the training buffer (Algorithm 4 input [l, u]): one kernel
  * takes, for every feature column j, the smallest and largest value over the
- * records the sample ring holds when it runs (its first min(count,
- * ring_capacity) slots; NaN values skipped; a column without a number gets
- * the empty range lo = +inf, hi = -inf) into a staging copy.  The next
+ * records the training buffer holds when it runs (the sample ring's first
+ * min(count, ring_capacity) slots and the replay pool's records; NaN values
+ * skipped; a column without a number gets the empty range lo = +inf,
+ * hi = -inf) into a staging copy.  The next
  * ls_publish publishes the staged bounds together with the weights, so a
  * route sees the bounds of the data its weights were trained beside.  Before
  * the first refresh the staging copy holds the empty range in every column. */
 int ls_refresh_bounds(ls_ctx *ctx, void *stream);
+
+/* One admission round of the replay pool (Sec. 4.3.2: evicted samples are
+ * admitted only if their last-hidden-layer activations weighted by the
+ * prediction residual are the most diverse with respect to those kept).
+ * Candidates: the pending records not yet considered (stream order), m of
+ * them.  With the current master weights every candidate and kept record
+ * gets the embedding g = (yhat - y) a (a = last hidden activation); then
+ *   d_e = min over kept j of |g_e - g_j|^2        (+inf with nothing kept),
+ *   n_j = min over kept k != j of |g_j - g_k|^2   (+inf without another),
+ * candidates ranked by (d desc, stream order), kept records by (n asc, slot);
+ * the first free = replay_capacity - nR candidates fill the free slots, then
+ * the candidate of rank free + q replaces the kept record of rank q while
+ * d > n (NaN counts as -inf).  All candidates count as considered.
+ * Distances are formed as |g_e|^2 + |g_j|^2 - 2 g_e.g_j with bf16 products
+ * and fp32 sums on tensor cores (shapes of at least 64 x 32), else fp32.
+ * d_out [pending_capacity] / n_out [replay_capacity] (DEVICE, nullable):
+ * d of candidate t (t < m) and n of replay slot j (j < nR, before the round).
+ * LS_ERR_STATE without a replay pool or without parameters / normaliser. */
+int ls_replay_admit(ls_ctx *ctx, float *d_out, float *n_out, void *stream);
+
+/* Copy the replay pool: DEVICE x_out [replay_capacity, d], y_out
+ * [replay_capacity] (slots >= *n_out are left as they are), HOST *n_out
+ * (synchronises the device). */
+int ls_get_replay(ls_ctx *ctx, float *x_out, float *y_out, int64_t *n_out, void *stream);
 
 /* Copy bounds to DEVICE lo_out [d], hi_out [d]: which = 0 the staging copy,
  * 1 the bounds routing reads now (synchronises the device). */

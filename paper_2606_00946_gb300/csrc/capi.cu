@@ -16,7 +16,7 @@ const char* const kTraceNames[TR_COUNT] = {
     "ring_append", "publish", "train_gather", "gemm_fwd", "loss_grad", "gemm_dw", "reduce_dw",
     "colsum_db", "gemm_dx", "optimizer", "memset", "score_tc", "features", "publish_tc",
     "hash_screen", "probe_screen", "probe_walk", "gemm_tc_fwd", "gemm_tc_dw", "gemm_tc_dx", "prefix_index",
-    "index_insert", "guards", "ring_bounds"};
+    "index_insert", "guards", "ring_bounds", "replay_admit"};
 }
 
 struct ls_ctx {
@@ -85,6 +85,10 @@ bool check_config(const ls_config* c, std::string& why) {
     return false;
   }
   if (c->max_batch_tokens < 1) { why = "max_batch_tokens must be >= 1"; return false; }
+  if (c->replay_capacity < 0 || c->pending_capacity < 0 || ((c->replay_capacity > 0) != (c->pending_capacity > 0))) {
+    why = "replay_capacity and pending_capacity must both be 0 or both be >= 1";
+    return false;
+  }
   const double need = std::ceil((double)c->max_keys_per_instance / (double)c->max_load);
   if (need > (double)(1ull << 31)) { why = "table would exceed 2^31 slots"; return false; }
   return true;
@@ -110,7 +114,8 @@ void free_all(Ctx& c) {
                   c.ring_x, c.ring_y, c.hits, c.scores, c.tx, c.tz, c.ty, c.dz0, c.dz1, c.grad,
                   c.gpart, c.loss_tmp, c.d_err, c.pub[0].img, c.pub[1].img, c.xin, c.xrq, c.pairx, c.ximg,
                   c.bkeys, c.work, c.work_n, c.gkeys, c.gmask, c.st, c.tf.base, c.tf.parts,
-                  c.pub[0].bounds, c.pub[1].bounds, c.bounds_stage, c.benc};
+                  c.pub[0].bounds, c.pub[1].bounds, c.bounds_stage, c.benc, c.remb, c.rnorm, c.rpart, c.rd,
+                  c.rn, c.rinv};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   if (c.ev_pub) cudaEventDestroy(c.ev_pub);
@@ -225,8 +230,20 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
   if (c.use_tc && !c.tc.pipe) A(dalloc(&c.pairx, R * NI));
   if (c.use_tc && c.tc.pipe)
     A(dalloc(&c.ximg, (R * NI + 127) / 128 * ((int64_t)c.tc.d_pad / 64) * 16384));
-  A(dalloc(&c.ring_x, cfg->ring_capacity * c.d));
-  A(dalloc(&c.ring_y, cfg->ring_capacity));
+  // FIFO, pending ring, replay pool (Sec. 4.3.2 two-pool training data)
+  const int64_t ring_rows = cfg->ring_capacity + cfg->pending_capacity + cfg->replay_capacity;
+  c.replay_base = cfg->ring_capacity + cfg->pending_capacity;
+  A(dalloc(&c.ring_x, ring_rows * c.d));
+  A(dalloc(&c.ring_y, ring_rows));
+  if (cfg->replay_capacity > 0) {
+    const int64_t er = cfg->pending_capacity + cfg->replay_capacity;
+    A(dalloc(&c.remb, er * m.w[m.n_layers - 1]));
+    A(dalloc(&c.rnorm, er));
+    A(dalloc(&c.rpart, std::max(cfg->pending_capacity, cfg->replay_capacity) * kRowMinParts));
+    A(dalloc(&c.rd, cfg->pending_capacity));
+    A(dalloc(&c.rn, cfg->replay_capacity));
+    A(dalloc(&c.rinv, er));
+  }
   A(dalloc(&c.hits, R * NI));
   A(dalloc(&c.scores, R * NI));
   A(dalloc(&c.tx, B * sum_in));
@@ -323,6 +340,13 @@ int ls_get_info(ls_ctx* h, ls_info* out) {
   out->train_steps = ds.step;
   out->weight_version = ds.version;
   out->scorer = c.use_tc ? LS_SCORER_TENSOR_CORES : LS_SCORER_CUDA_CORES;
+  out->replay_count = ds.replay_count;
+  out->pending_count = 0;
+  if (c.cfg.replay_capacity > 0) {  // evicted positions [lo, hi) not yet considered
+    const int64_t hi = std::max<int64_t>(0, ds.ring_count - c.cfg.ring_capacity);
+    const int64_t lo = std::min(hi, std::max(ds.admitted, hi - c.cfg.pending_capacity));
+    out->pending_count = hi - lo;
+  }
   return LS_OK;
 }
 
@@ -592,9 +616,38 @@ int ls_refresh_bounds(ls_ctx* h, void* stream) {
   if (!h) return fail(LS_ERR_ARG, "ctx is NULL");
   Ctx& c = h->c;
   LS_CK(traced(c, TR_BOUNDS, 1, S(stream), [&] {
-    return launch_ring_bounds(c.d, c.ring_x, c.cfg.ring_capacity, c.benc, c.bounds_stage, c.st, c.sms,
+    return launch_ring_bounds(c.d, c.ring_x, c.cfg.ring_capacity, c.replay_base, c.cfg.replay_capacity, c.benc,
+                              c.bounds_stage, c.st, c.sms,
                               S(stream));
   }));
+  return LS_OK;
+}
+
+int ls_replay_admit(ls_ctx* h, float* d_out, float* n_out, void* stream) {
+  if (!h) return fail(LS_ERR_ARG, "ctx is NULL");
+  Ctx& c = h->c;
+  if (c.cfg.replay_capacity < 1) return fail(LS_ERR_STATE, "no replay pool configured");
+  if (!c.have_params) return fail(LS_ERR_STATE, "parameters not set");
+  if (!c.have_norm) return fail(LS_ERR_STATE, "normaliser not set");
+  LS_CK(run_replay_admit(c, d_out, n_out, S(stream)));
+  return LS_OK;
+}
+
+int ls_get_replay(ls_ctx* h, float* x_out, float* y_out, int64_t* n_out, void* stream) {
+  if (!h || !x_out || !y_out || !n_out) return fail(LS_ERR_ARG, "NULL argument");
+  Ctx& c = h->c;
+  if (c.cfg.replay_capacity < 1) return fail(LS_ERR_STATE, "no replay pool configured");
+  int64_t nr = 0;
+  LS_CK(cudaDeviceSynchronize());
+  LS_CK(cudaMemcpy(&nr, &c.st->replay_count, sizeof(nr), cudaMemcpyDeviceToHost));
+  if (nr > 0) {
+    LS_CK(cudaMemcpyAsync(x_out, c.ring_x + c.replay_base * c.d, (size_t)nr * c.d * sizeof(float),
+                          cudaMemcpyDeviceToDevice, S(stream)));
+    LS_CK(cudaMemcpyAsync(y_out, c.ring_y + c.replay_base, (size_t)nr * sizeof(float), cudaMemcpyDeviceToDevice,
+                          S(stream)));
+    LS_CK(cudaStreamSynchronize(S(stream)));
+  }
+  *n_out = nr;
   return LS_OK;
 }
 
@@ -623,8 +676,11 @@ int ls_log_samples(ls_ctx* h, int32_t n, const float* feats, const float* ttft, 
   if (n < 0) return fail(LS_ERR_ARG, "n < 0");
   if (n == 0) return LS_OK;
   if (!feats || !ttft) return fail(LS_ERR_ARG, "NULL argument");
+  if (c.cfg.pending_capacity > 0 && n > c.cfg.ring_capacity)
+    return fail(LS_ERR_ARG, "with a replay pool a log call holds at most ring_capacity records");
   LS_CK(traced(c, TR_RING, 1, S(stream), [&] {
-    return launch_ring_append(n, c.d, feats, ttft, c.ring_x, c.ring_y, c.st, c.cfg.ring_capacity, S(stream));
+    return launch_ring_append(n, c.d, feats, ttft, c.ring_x, c.ring_y, c.st, c.cfg.ring_capacity,
+                              c.cfg.pending_capacity, S(stream));
   }));
   std::lock_guard<std::mutex> g(c.mu);
   c.ring_enqueued += n;

@@ -74,10 +74,18 @@ struct DevState {
   int32_t route_b;          // buffer chosen by the route in flight (set by its prefix kernel)
   uint64_t version;         // publishes completed
   uint64_t pub_version[2];  // version held by each buffer
-  uint32_t done[4];         // per-kernel block arrival counters (last-block updates)
+  uint32_t done[6];         // per-kernel block arrival counters (last-block updates)
   float adam_bc[2];         // 1 - beta1^t, 1 - beta2^t of the step in flight, t = step + 1
   double beta_pow[2];       // beta1^step, beta2^step (fp64 running products)
+  int64_t replay_count;     // records in the replay pool
+  int64_t admitted;         // evicted stream positions below this were considered for the replay pool
 };
+
+// Row of training-buffer index u (Sec. 4.3.2: a round trains on F u R): ring
+// slot u for u < nF, else replay record u - nF at row replay_base + u - nF.
+__host__ __device__ __forceinline__ int64_t union_row(int64_t u, int64_t nF, int64_t replay_base) {
+  return u < nF ? u : replay_base + (u - nF);
+}
 
 // Adam bias corrections of the coming step, 1 - beta^(step+1), from the fp64
 // running powers (one multiply each, by one thread of the step's first kernel).
@@ -93,6 +101,7 @@ __device__ __forceinline__ void advance_step(DevState* st, int64_t t) {
   st->beta_pow[1] *= 0.999;
 }
 enum { DONE_RING = 0, DONE_OPT = 1, DONE_PUB = 2, DONE_BOUNDS = 3 };
+enum { DONE_REPLAY = 4 };  // DevState::done has 6 entries
 
 // Kernel-level tracing: when enabled, every launch is bracketed by CUDA events
 // recorded on the launching stream; ls_trace_read() sums the elapsed times.
@@ -101,7 +110,7 @@ enum TraceId {
   TR_GATHER, TR_GEMM_FWD, TR_LOSS, TR_GEMM_DW, TR_REDUCE, TR_COLSUM, TR_GEMM_DX, TR_OPT,
   TR_MEMSET, TR_SCORE_TC, TR_NORM_ROWS, TR_PUBLISH_TC, TR_HASH_BATCH, TR_SCREEN, TR_WALK,
   TR_GEMM_TC_FWD, TR_GEMM_TC_DW, TR_GEMM_TC_DX, TR_PREFIX_INDEX, TR_INDEX_INSERT,
-  TR_GUARDS, TR_BOUNDS, TR_COUNT
+  TR_GUARDS, TR_BOUNDS, TR_REPLAY, TR_COUNT
 };
 extern const char* const kTraceNames[TR_COUNT];
 
@@ -196,9 +205,18 @@ struct Ctx {
   bool pub_recorded = false, route_recorded = false;
   DevState* st = nullptr;
 
-  // sample ring (Sec. 4.3.2)
+  // sample ring (Sec. 4.3.2): rows [0, C) the FIFO pool, [C, C + P) the
+  // pending ring of evicted records, [C + P, C + P + Rc) the replay pool
   float* ring_x = nullptr;
   float* ring_y = nullptr;
+  int64_t replay_base = 0;        // C + P
+  // replay admission scratch
+  float* remb = nullptr;          // embeddings [P + Rc, H] fp32 (candidates, then kept)
+  float* rnorm = nullptr;         // |bf16(g)|^2 [P + Rc] (+inf for rows not in use)
+  float* rpart = nullptr;         // row-min partials [max(P, Rc), kRowMinParts]
+  float* rd = nullptr;            // d per candidate [P]
+  float* rn = nullptr;            // n per kept record [Rc]
+  int32_t* rinv = nullptr;        // rank -> candidate [P], then rank -> kept slot [Rc]
   int64_t ring_enqueued = 0;
   // feature bounds of the ring (Algorithm 4 [l, u]): staged by ls_refresh_bounds,
   // published by ls_publish into pub[b].bounds
@@ -359,8 +377,9 @@ cudaError_t launch_argmin(int n_req, int n_inst, const float* scores, int32_t* c
 // Algorithm 4 guards.  benc must hold the identity codes (0xff800000 in
 // [0, d), 0x007fffff in [d, 2d)) before a bounds launch; each launch leaves
 // them so.
-cudaError_t launch_ring_bounds(int d, const float* ring_x, int64_t capacity, uint32_t* benc, float* stage,
-                               DevState* st, int sms, cudaStream_t s);
+cudaError_t launch_ring_bounds(int d, const float* ring_x, int64_t capacity, int64_t replay_base,
+                               int64_t replay_capacity, uint32_t* benc, float* stage, DevState* st, int sms,
+                               cudaStream_t s);
 cudaError_t launch_guards(const ls_guards& g, int n_req, int n_inst, const int32_t* tok, const int64_t* tok_off,
                           const int32_t* hits, const float* scores, const float* inst, int d_inst,
                           const float* req, int d_req, const Published* pub, const DevState* st,
@@ -393,7 +412,16 @@ cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const Published* 
                             const float* mean, const float* stdv, float* scores, int* err, int sms,
                             cudaStream_t s);
 cudaError_t launch_ring_append(int n, int d, const float* x, const float* y, float* ring_x,
-                               float* ring_y, DevState* st, int64_t capacity, cudaStream_t s);
+                               float* ring_y, DevState* st, int64_t capacity, int64_t pending, cudaStream_t s);
+// forward of B rows already in c.tx (layer inputs), keeping z_l in c.tz and a_l in c.tx
+cudaError_t forward_rows(Ctx& c, int B, cudaStream_t s);
+cudaError_t run_replay_admit(Ctx& c, float* d_out, float* n_out, cudaStream_t s);
+// row-min distance GEMM: out[row * ldp + part] = min over this CTA's columns n of
+// na[row] + nb[n] - 2 sum_k A(row, k) B(n, k), skipping n == row + self_off
+cudaError_t launch_rowmin_tc(int M, int N, int K, const float* A, int64_t lda, const float* B, int64_t ldb,
+                             const float* na, const float* nb, int64_t self_off, float* part, int64_t ldp,
+                             int* parts_used, int* err, int sms, cudaStream_t s);
+constexpr int kRowMinParts = 256;  // partial columns per row of rpart
 cudaError_t run_train_step(Ctx& c, int batch, const int32_t* idx, int opt, float lr,
                            float* loss_out, cudaStream_t s);
 cudaError_t launch_gemm_tc(int M, int N, int K, const float* A, int64_t sam, int64_t sak, const float* B,

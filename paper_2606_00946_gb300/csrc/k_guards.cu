@@ -49,7 +49,8 @@ __device__ __forceinline__ void fold(float v, float& lo, float& hi) {  // NaN fa
   hi = v > hi ? v : hi;
 }
 
-// Rows [0, min(count, capacity)) split into gridDim.x contiguous ranges.
+// Records of the training buffer F u R (union index u -> row union_row(u))
+// split into gridDim.x contiguous ranges of u.
 // d % 4 == 0: thread t reads 16-byte groups g = t % (d/4) of rows t / (d/4),
 // t / (d/4) + P, ... (P = 256 / (d/4) rows per pass, so a pass is one
 // contiguous run of P d floats), eight loads in flight.  Other d: the same
@@ -57,11 +58,12 @@ __device__ __forceinline__ void fold(float v, float& lo, float& hi) {  // NaN fa
 // Block results go to the per-column codes in benc [2][d]; the last block
 // decodes them into the staging copy and resets them for the next launch.
 __global__ void __launch_bounds__(256) k_ring_bounds(int d, const float* __restrict__ ring_x, int64_t capacity,
-                                                     uint32_t* __restrict__ benc, float* __restrict__ stage,
-                                                     DevState* st) {
+                                                     int64_t replay_base, uint32_t* __restrict__ benc,
+                                                     float* __restrict__ stage, DevState* st) {
   __shared__ float s_lo[1024], s_hi[1024];
   const int64_t count = *reinterpret_cast<volatile int64_t*>(&st->ring_count);
-  const int64_t rows = count < capacity ? count : capacity;
+  const int64_t nF = count < capacity ? count : capacity;
+  const int64_t rows = nF + *reinterpret_cast<volatile int64_t*>(&st->replay_count);
   const int64_t per = (rows + gridDim.x - 1) / gridDim.x;
   const int64_t r0 = (int64_t)blockIdx.x * per;
   const int64_t r1 = r0 + per < rows ? r0 + per : rows;
@@ -76,7 +78,8 @@ __global__ void __launch_bounds__(256) k_ring_bounds(int d, const float* __restr
       for (int64_t r = r0 + p; r < r1; r += 8 * (int64_t)P) {
         float4 v[8];
 #pragma unroll
-        for (int u = 0; u < 8; ++u) v[u] = r + (int64_t)u * P < r1 ? __ldcs(base + (r + (int64_t)u * P) * G) : none;
+        for (int u = 0; u < 8; ++u)
+          v[u] = r + (int64_t)u * P < r1 ? __ldcs(base + union_row(r + (int64_t)u * P, nF, replay_base) * G) : none;
 #pragma unroll
         for (int u = 0; u < 8; ++u) {
           fold(v[u].x, lo[0], hi[0]);
@@ -111,7 +114,9 @@ __global__ void __launch_bounds__(256) k_ring_bounds(int d, const float* __restr
         for (int64_t r = r0 + p; r < r1; r += 4 * (int64_t)P) {
           float v[4];
 #pragma unroll
-          for (int u = 0; u < 4; ++u) v[u] = r + (int64_t)u * P < r1 ? __ldcs(ring_x + (r + (int64_t)u * P) * d + c) : NAN;
+          for (int u = 0; u < 4; ++u)
+            v[u] = r + (int64_t)u * P < r1 ? __ldcs(ring_x + union_row(r + (int64_t)u * P, nF, replay_base) * d + c)
+                                           : NAN;
 #pragma unroll
           for (int u = 0; u < 4; ++u) fold(v[u], lo, hi);
         }
@@ -496,12 +501,13 @@ __global__ void __launch_bounds__(kGuardThreads) k_guards(const __grid_constant_
 
 }  // namespace
 
-cudaError_t launch_ring_bounds(int d, const float* ring_x, int64_t capacity, uint32_t* benc, float* stage,
-                               DevState* st, int sms, cudaStream_t s) {
+cudaError_t launch_ring_bounds(int d, const float* ring_x, int64_t capacity, int64_t replay_base,
+                               int64_t replay_capacity, uint32_t* benc, float* stage, DevState* st, int sms,
+                               cudaStream_t s) {
   // at least 64 rows per block, at most four blocks per SM
-  int64_t grid = std::min<int64_t>((capacity + 63) / 64, 4 * (int64_t)sms);
+  int64_t grid = std::min<int64_t>((capacity + replay_capacity + 63) / 64, 4 * (int64_t)sms);
   grid = std::max<int64_t>(grid, 1);
-  k_ring_bounds<<<(int)grid, 256, 0, s>>>(d, ring_x, capacity, benc, stage, st);
+  k_ring_bounds<<<(int)grid, 256, 0, s>>>(d, ring_x, capacity, replay_base, benc, stage, st);
   return cudaGetLastError();
 }
 

@@ -139,10 +139,13 @@ __global__ void k_argmin(int n_req, int n_inst, const float* __restrict__ scores
 // Record j of the batch -> slot (count + j) mod capacity, count = records
 // appended before this batch (device state); the last block advances the
 // count by n.  When a batch is longer than the ring only its last `capacity`
-// records are kept.
+// records are kept.  With a pending ring (pending > 0; then n <= capacity)
+// the record a slot held, stream position p - capacity, is first copied to
+// pending row capacity + (p - capacity) mod pending by the thread that then
+// overwrites the same piece; of the records one call evicts only the newest
+// `pending` are copied, so no two copies share a row.
 __global__ void k_ring_append(int n, int d, const float* __restrict__ x, const float* __restrict__ y,
-                              float* __restrict__ ring_x, float* __restrict__ ring_y, DevState* st,
-                              int64_t capacity) {
+                              float* ring_x, float* ring_y, DevState* st, int64_t capacity, int64_t pending) {
   const int64_t count = *reinterpret_cast<volatile int64_t*>(&st->ring_count);
   const int64_t first = n > capacity ? n - capacity : 0;
   // piece = 4 consecutive columns of one record (the last piece of a record
@@ -159,6 +162,18 @@ __global__ void k_ring_append(int n, int d, const float* __restrict__ x, const f
     const int64_t slot = (count + j) % capacity;
     const float* src = x + j * d + k;
     float* dst = ring_x + slot * d + k;
+    // only the newest `pending` records this call evicts are kept (older ones
+    // would land on the same pending rows)
+    if (pending > 0 && count + j >= capacity && count + j - capacity >= count + n - capacity - pending) {
+      const int64_t prow = capacity + (count + j - capacity) % pending;
+      float* pdst = ring_x + prow * d + k;
+      if (vec) {
+        *reinterpret_cast<float4*>(pdst) = *reinterpret_cast<const float4*>(dst);
+      } else {
+        for (int u = 0; u < 4 && k + u < d; ++u) pdst[u] = dst[u];
+      }
+      if (k == 0) ring_y[prow] = ring_y[slot];
+    }
     if (vec) {
       *reinterpret_cast<float4*>(dst) = __ldg(reinterpret_cast<const float4*>(src));
     } else {
@@ -224,11 +239,11 @@ cudaError_t launch_argmin(int n_req, int n_inst, const float* scores, int32_t* c
 }
 
 cudaError_t launch_ring_append(int n, int d, const float* x, const float* y, float* ring_x,
-                               float* ring_y, DevState* st, int64_t capacity, cudaStream_t s) {
+                               float* ring_y, DevState* st, int64_t capacity, int64_t pending, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
   const int64_t keep = n > capacity ? capacity : n;
   const int64_t total = keep * ((d + 3) / 4);
-  k_ring_append<<<grid_1d(total, 256), 256, 0, s>>>(n, d, x, y, ring_x, ring_y, st, capacity);
+  k_ring_append<<<grid_1d(total, 256), 256, 0, s>>>(n, d, x, y, ring_x, ring_y, st, capacity, pending);
   return cudaGetLastError();
 }
 

@@ -107,13 +107,14 @@ __global__ void __launch_bounds__(256) k_gemm(GemmArgs g) {
 // state; z-score in fp32, bf16-rounded in bf16 mode.  An empty ring latches
 // LS_ERR_STATE (rows then come from slot 0).
 __global__ void k_train_gather(int B, int d, const int32_t* __restrict__ idx, DevState* st,
-                               int64_t capacity, const float* __restrict__ ring_x,
+                               int64_t capacity, int64_t replay_base, const float* __restrict__ ring_x,
                                const float* __restrict__ ring_y, const float* __restrict__ mean,
                                const float* __restrict__ stdv, int bf16, float* __restrict__ x0,
                                float* __restrict__ y, int* err) {
   const int64_t step = st->step;
   const int64_t count = st->ring_count;
-  const int64_t valid = count < capacity ? count : capacity;
+  const int64_t nF = count < capacity ? count : capacity;
+  const int64_t valid = nF + st->replay_count;  // F u R
   if (valid < 1 && blockIdx.x == 0 && threadIdx.x == 0) latch_error(err, LS_ERR_STATE);
   if (blockIdx.x == 0 && threadIdx.x == 0) set_adam_bc(st);
   const int64_t total = (int64_t)B * d;
@@ -130,6 +131,7 @@ __global__ void k_train_gather(int B, int d, const int32_t* __restrict__ idx, De
     } else {
       slot = valid > 0 ? (step * (int64_t)B + j) % valid : 0;
     }
+    slot = union_row(slot, nF, replay_base);
     const float v = zscore(ring_x[slot * d + k], mean[k], stdv[k]);
     x0[e] = bf16 ? round_bf16(v) : v;
     if (k == 0) y[j] = ring_y[slot];
@@ -299,8 +301,10 @@ int train_splits(int out, int in, int B, int n_sm) {
   return std::max(1, std::min(S, 64));
 }
 
-cudaError_t run_train_step(Ctx& c, int B, const int32_t* idx, int opt, float lr, float* loss_out,
-                           cudaStream_t s) {
+// Forward of B rows whose layer-0 inputs are in c.tx (z-scored, rounded in
+// bf16 mode): z_l into c.tz, hidden activations a_l into c.tx (the training
+// step's layout: layer l's input at c.tx + B * sum_{k<l} w_k).
+cudaError_t forward_rows(Ctx& c, int B, cudaStream_t s) {
   const MlpDesc& m = c.mlp;
   const int L = m.n_layers;
   int64_t xoff[LS_MAX_LAYERS + 1], zoff[LS_MAX_LAYERS + 1];
@@ -309,19 +313,7 @@ cudaError_t run_train_step(Ctx& c, int B, const int32_t* idx, int opt, float lr,
     xoff[l + 1] = xoff[l] + (int64_t)B * m.w[l];
     zoff[l + 1] = zoff[l] + (int64_t)B * m.w[l + 1];
   }
-  cudaError_t e;
-  {
-    const int64_t total = (int64_t)B * m.w[0];
-    int grid = (int)std::min<int64_t>((total + 255) / 256, (int64_t)c.sms * 8);
-    e = traced(c, TR_GATHER, 1, s, [&] {
-      k_train_gather<<<std::max(grid, 1), 256, 0, s>>>(B, m.w[0], idx, c.st, c.cfg.ring_capacity, c.ring_x,
-                                                       c.ring_y, c.mean, c.stdv, m.bf16, c.tx, c.ty,
-                                                       c.d_err);
-      return cudaGetLastError();
-    });
-    if (e != cudaSuccess) return e;
-  }
-  // forward, keeping z_l and a_l
+  cudaError_t e = cudaSuccess;
   for (int l = 0; l < L; ++l) {
     GemmArgs a{};
     a.M = B; a.N = m.w[l + 1]; a.K = m.w[l];
@@ -358,6 +350,35 @@ cudaError_t run_train_step(Ctx& c, int B, const int32_t* idx, int opt, float lr,
       if (e != cudaSuccess) return e;
     }
   }
+  return cudaSuccess;
+}
+
+cudaError_t run_train_step(Ctx& c, int B, const int32_t* idx, int opt, float lr, float* loss_out,
+                           cudaStream_t s) {
+  const MlpDesc& m = c.mlp;
+  const int L = m.n_layers;
+  int64_t xoff[LS_MAX_LAYERS + 1], zoff[LS_MAX_LAYERS + 1];
+  xoff[0] = zoff[0] = 0;
+  for (int l = 0; l < L; ++l) {
+    xoff[l + 1] = xoff[l] + (int64_t)B * m.w[l];
+    zoff[l + 1] = zoff[l] + (int64_t)B * m.w[l + 1];
+  }
+  cudaError_t e;
+  {
+    const int64_t total = (int64_t)B * m.w[0];
+    int grid = (int)std::min<int64_t>((total + 255) / 256, (int64_t)c.sms * 8);
+    e = traced(c, TR_GATHER, 1, s, [&] {
+      k_train_gather<<<std::max(grid, 1), 256, 0, s>>>(B, m.w[0], idx, c.st, c.cfg.ring_capacity, c.replay_base,
+                                                       c.ring_x,
+                                                       c.ring_y, c.mean, c.stdv, m.bf16, c.tx, c.ty,
+                                                       c.d_err);
+      return cudaGetLastError();
+    });
+    if (e != cudaSuccess) return e;
+  }
+  // forward, keeping z_l and a_l
+  e = forward_rows(c, B, s);
+  if (e != cudaSuccess) return e;
   e = traced(c, TR_LOSS, 1, s, [&] {
     k_loss_grad<<<1, 1024, 0, s>>>(B, c.tz + zoff[L - 1], c.ty, c.dz0,
                                    loss_out ? loss_out : c.loss_tmp);

@@ -350,13 +350,14 @@ __global__ void __launch_bounds__(kT, 1) k_tr_gemm(const __grid_constant__ TrArg
 // valid) z-scored and rounded to bf16 into img(A_0) and img(A_0^T); rows past
 // the batch and columns past d are zero.  Thread = (row j, 8 columns).
 __global__ void k_tr_gather(int B, int rows_pad, int d, int d_pad, const int32_t* __restrict__ idx,
-                            DevState* st, int64_t capacity, const float* __restrict__ ring_x,
+                            DevState* st, int64_t capacity, int64_t replay_base, const float* __restrict__ ring_x,
                             const float* __restrict__ ring_y, const float* __restrict__ mean,
                             const float* __restrict__ stdv, uint8_t* __restrict__ a0, uint8_t* __restrict__ a0t,
                             float* __restrict__ y, int* err) {
   const int64_t step = st->step;
   const int64_t count = st->ring_count;
-  const int64_t valid = count < capacity ? count : capacity;
+  const int64_t nF = count < capacity ? count : capacity;
+  const int64_t valid = nF + st->replay_count;  // F u R
   if (valid < 1 && blockIdx.x == 0 && threadIdx.x == 0) latch_error(err, LS_ERR_STATE);
   if (blockIdx.x == 0 && threadIdx.x == 0) set_adam_bc(st);
   const int64_t total = (int64_t)rows_pad * (d_pad / 8);
@@ -377,6 +378,7 @@ __global__ void k_tr_gather(int B, int rows_pad, int d, int d_pad, const int32_t
       } else {
         slot = valid > 0 ? (step * (int64_t)B + j) % valid : 0;
       }
+      slot = union_row(slot, nF, replay_base);
       const float* row = ring_x + slot * d;
 #pragma unroll
       for (int u = 0; u < 8; ++u)
@@ -655,7 +657,8 @@ cudaError_t run_train_fast(Ctx& c, int B, const int32_t* idx, int opt, float lr,
   e = traced(c, TR_GATHER, 1, s, [&] {
     const int64_t total = (int64_t)R * (f.in_pad[0] / 8);
     const int grid = (int)std::min<int64_t>((total + 255) / 256, (int64_t)c.sms * 8);
-    k_tr_gather<<<grid, 256, 0, s>>>(B, R, m.w[0], f.in_pad[0], idx, c.st, c.cfg.ring_capacity, c.ring_x, c.ring_y,
+    k_tr_gather<<<grid, 256, 0, s>>>(B, R, m.w[0], f.in_pad[0], idx, c.st, c.cfg.ring_capacity, c.replay_base,
+                                     c.ring_x, c.ring_y,
                                      c.mean, c.stdv, f.imgA[0], f.imgAT[0], c.ty, c.d_err);
     return cudaGetLastError();
   });

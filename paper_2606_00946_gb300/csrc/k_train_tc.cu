@@ -8,7 +8,9 @@
 // tensor memory; K runs in chunks of 64 through two staging buffers (the next
 // chunk is staged while the MMAs of the current one run); blockIdx.z splits
 // K (partials reduced by the caller).  Epilogues: store (partial), forward
-// (Z = D + bias, A_next = bf16(ReLU(Z))), or ReLU mask (dZ_prev = D * [Z > 0]).
+// (Z = D + bias, A_next = bf16(ReLU(Z))), ReLU mask (dZ_prev = D * [Z > 0]),
+// or row minimum of squared distances na[m] + nb[n] - 2 D[m, n] over the
+// CTA's columns (the replay pool's nearest-neighbour search, Sec. 4.3.2).
 #include "common.cuh"
 #include "sm100.cuh"
 
@@ -35,6 +37,9 @@ struct TcGemmArgs {
   int hidden;
   const float* zprev;
   int64_t ld_zprev;
+  const float* na;   // epilogue 3: row and column squared norms
+  const float* nb;
+  int64_t self_off;  // epilogue 3: column row + self_off is skipped
   int* err;
   uint32_t tmem_cols;
 };
@@ -192,6 +197,8 @@ __global__ void __launch_bounds__(kT) k_gemm_tc(const __grid_constant__ TcGemmAr
   const int half = NTILE / 2;
   const uint32_t lane_addr = (uint32_t)(32 * q4) << 16;
   const bool row_ok = row < g.M;
+  float rmin = INFINITY;
+  const float row_norm = g.epi == 3 && row_ok ? __ldg(g.na + row) : 0.0f;
   for (int c0 = ch * half; c0 < (ch + 1) * half; c0 += 16) {
     uint32_t v[16];
     if (nchunks > 0) {
@@ -217,6 +224,9 @@ __global__ void __launch_bounds__(kT) k_gemm_tc(const __grid_constant__ TcGemmAr
 #pragma unroll
         for (int j = 0; j < 16; ++j) side[j] = nb + j < g.N ? __ldg(g.bias + nb + j) : 0.0f;
       }
+    } else if (g.epi == 3) {
+#pragma unroll
+      for (int j = 0; j < 16; ++j) side[j] = nb + j < g.N ? __ldg(g.nb + nb + j) : INFINITY;
     } else if (g.epi == 2) {
       const float* zp = g.zprev + (int64_t)row * g.ld_zprev + nb;
       if (row_ok && full && (reinterpret_cast<uintptr_t>(zp) & 15) == 0) {
@@ -231,6 +241,14 @@ __global__ void __launch_bounds__(kT) k_gemm_tc(const __grid_constant__ TcGemmAr
       }
     }
     if (!row_ok) continue;
+    if (g.epi == 3) {
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const float dist = row_norm + side[j] - 2.0f * __uint_as_float(v[j]);
+        if ((int64_t)(nb + j) != (int64_t)row + g.self_off) rmin = fminf(rmin, dist);
+      }
+      continue;
+    }
     float out[16], act[16];
 #pragma unroll
     for (int j = 0; j < 16; ++j) {
@@ -263,6 +281,7 @@ __global__ void __launch_bounds__(kT) k_gemm_tc(const __grid_constant__ TcGemmAr
         }
     }
   }
+  if (g.epi == 3 && row_ok) g.C[(int64_t)row * g.ldc + 2 * blockIdx.x + ch] = rmin;
   tc_fence_before();
   __syncthreads();
   if (warp == 0) tmem_dealloc(tmem, g.tmem_cols);
@@ -313,6 +332,39 @@ cudaError_t launch_gemm_tc(int M, int N, int K, const float* A, int64_t sam, int
     default: return cudaErrorInvalidValue;
   }
   return e2;
+}
+
+cudaError_t launch_rowmin_tc(int M, int N, int K, const float* A, int64_t lda, const float* B, int64_t ldb,
+                             const float* na, const float* nb, int64_t self_off, float* part, int64_t ldp,
+                             int* parts_used, int* err, int sms, cudaStream_t s) {
+  if (M < 64 || N < 32 || K < 1) return cudaErrorInvalidValue;
+  const int mt = (M + kM - 1) / kM;
+  int ntile = 256;
+  while (ntile > 64 && (int64_t)mt * ((N + ntile - 1) / ntile) < sms) ntile /= 2;
+  while (ntile > 64 && ntile / 2 >= N) ntile /= 2;
+  const int nt = (N + ntile - 1) / ntile;
+  if (2 * nt > ldp) return cudaErrorInvalidValue;
+  TcGemmArgs g{};
+  g.M = M; g.N = N; g.K = K;
+  g.A = A; g.sam = lda; g.sak = 1;
+  g.B = B; g.sbn = ldb; g.sbk = 1;
+  g.ntile = ntile;
+  g.kper = (int)(((int64_t)K + 63) / 64 * 64);
+  g.epi = 3;
+  g.C = part; g.ldc = ldp;
+  g.na = na; g.nb = nb; g.self_off = self_off;
+  g.err = err;
+  g.tmem_cols = 32;
+  while ((int)g.tmem_cols < ntile) g.tmem_cols <<= 1;
+  const int smem = 1024 + 2 * kM * 128 + 2 * ntile * 128 + 64;
+  dim3 grid(nt, mt, 1);
+  *parts_used = 2 * nt;
+  switch (ntile) {
+    case 256: return run_tc<256>(grid, smem, g, s);
+    case 128: return run_tc<128>(grid, smem, g, s);
+    case 64: return run_tc<64>(grid, smem, g, s);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 int gemm_tc_splits_used(int K, int splits) {

@@ -131,6 +131,25 @@ class Router:
         return dict(choice=choice, best=best, status=status, fallback=fallback, scores=scores, hits=hits,
                     version=ver)
 
+    def replay_admit(self, diag=False, stream=None):
+        """One admission round of the replay pool; with diag, returns (d, n)
+        per candidate / kept slot (device tensors of the pools' capacities)."""
+        d = n = None
+        if diag:
+            d = torch.empty(max(int(self.cfg.pending_capacity), 1), dtype=torch.float32, device="cuda")
+            n = torch.empty(max(int(self.cfg.replay_capacity), 1), dtype=torch.float32, device="cuda")
+        L.check(L.ls_replay_admit(self.h, d, n, stream))
+        return (d, n) if diag else None
+
+    def replay(self):
+        """Records in the replay pool: (x [n, d], y [n])."""
+        cap = max(int(self.cfg.replay_capacity), 1)
+        x = torch.empty(cap, self.widths[0], dtype=torch.float32, device="cuda")
+        y = torch.empty(cap, dtype=torch.float32, device="cuda")
+        rc, n = L.ls_get_replay(self.h, x, y)
+        L.check(rc)
+        return x[:n], y[:n]
+
     def set_guards(self, **kw):
         L.check(L.ls_set_guards(self.h, **kw))
 

@@ -34,13 +34,15 @@ class ls_config(C.Structure):
                 ("max_instances", C.c_int32), ("max_requests", C.c_int32),
                 ("max_keys_per_instance", C.c_int64), ("max_load", C.c_float),
                 ("ring_capacity", C.c_int64), ("max_train_batch", C.c_int32),
-                ("max_batch_tokens", C.c_int64), ("prefix_mode", C.c_int32), ("scorer", C.c_int32)]
+                ("max_batch_tokens", C.c_int64), ("prefix_mode", C.c_int32), ("scorer", C.c_int32),
+                ("replay_capacity", C.c_int64), ("pending_capacity", C.c_int64)]
 
 
 class ls_info(C.Structure):
     _fields_ = [("n_inst", C.c_int32), ("d", C.c_int32), ("n_params", C.c_int64),
                 ("table_slots", C.c_int64), ("ring_count", C.c_int64),
-                ("train_steps", C.c_int64), ("weight_version", C.c_uint64), ("scorer", C.c_int32)]
+                ("train_steps", C.c_int64), ("weight_version", C.c_uint64), ("scorer", C.c_int32),
+                ("replay_count", C.c_int64), ("pending_count", C.c_int64)]
 
 
 class ls_guards(C.Structure):
@@ -76,6 +78,8 @@ _SIGS = {
     "ls_train_step": (C.c_int, [_P, _i32, _P, _i32, C.c_float, _P, _P]),
     "ls_publish": (C.c_int, [_P, _P]),
     "ls_set_guards": (C.c_int, [_P, C.POINTER(ls_guards)]),
+    "ls_replay_admit": (C.c_int, [_P, _P, _P, _P]),
+    "ls_get_replay": (C.c_int, [_P, _P, _P, C.POINTER(_i64), _P]),
     "ls_refresh_bounds": (C.c_int, [_P, _P]),
     "ls_get_bounds": (C.c_int, [_P, _i32, _P, _P, _P]),
     "ls_route_batch_guarded": (C.c_int, [_P, _i32, _P, _P, _P, _P, _P, _P, _P, _P, _P,
@@ -147,7 +151,7 @@ def check(rc: int) -> int:
 def make_config(widths, d_inst, d_req, dtype="bf16", max_instances=64, max_requests=4096,
                 max_keys_per_instance=16384, max_load=0.5, ring_capacity=65536,
                 max_train_batch=4096, scorer="auto", max_batch_tokens=1 << 24,
-                prefix_mode="auto") -> ls_config:
+                prefix_mode="auto", replay_capacity=0, pending_capacity=0) -> ls_config:
     c = ls_config()
     c.n_layers = len(widths) - 1
     for i, w in enumerate(widths):
@@ -160,6 +164,7 @@ def make_config(widths, d_inst, d_req, dtype="bf16", max_instances=64, max_reque
     c.scorer = SCORERS.get(scorer, scorer)
     c.max_batch_tokens = int(max_batch_tokens)
     c.prefix_mode = PREFIX_MODES.get(prefix_mode, prefix_mode)
+    c.replay_capacity, c.pending_capacity = int(replay_capacity), int(pending_capacity)
     return c
 
 
@@ -263,6 +268,17 @@ def ls_set_guards(ctx, n_min=0, ood=False, k=0, kv_col=0, tau_sat=0.8, tau_ben=0
                   int(heuristic), (C.c_int32 * 2)(int(count_cols[0]), int(count_cols[1])), float(theta_imbal),
                   float(k_overload), float(tau_prefix))
     return lib().ls_set_guards(ctx, C.byref(g))
+
+
+def ls_replay_admit(ctx, d_out=None, n_out=None, stream=None) -> int:
+    return lib().ls_replay_admit(ctx, ptr(d_out), ptr(n_out), stream_handle(stream))
+
+
+def ls_get_replay(ctx, x_out, y_out, stream=None):
+    """Returns (status, records in the replay pool)."""
+    n = _i64(0)
+    rc = lib().ls_get_replay(ctx, ptr(x_out), ptr(y_out), C.byref(n), stream_handle(stream))
+    return rc, n.value
 
 
 def ls_refresh_bounds(ctx, stream=None) -> int:
