@@ -44,6 +44,9 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-guards", action="store_true", help="skip the guarded-route measurement")
+    p.add_argument("--no-replay", action="store_true", help="skip the replay-pool admission measurement")
+    p.add_argument("--replay-only", action="store_true",
+                   help="only the replay-pool admission measurement (for kernel profiling)")
     p.add_argument("--guards-only", action="store_true",
                    help="only the guarded-route measurement (--steps routes; for kernel profiling)")
     p.add_argument("--cpu-seconds", type=float, default=12.0, help="target oracle work for cpu_baseline")
@@ -118,6 +121,57 @@ def measure_guards(L, r, dw, N, R, d, ring_rows, d_req, flush, stream, peaks, n=
                     "heuristic of Algorithm 1 (counts = queued + running, theta_imbal 128 so that the per-request "
                     "order decides, k 1)",
     }
+
+
+def measure_replay(L, H, W, wl, dev, flush, stream, peaks, n=20):
+    """Two-pool training data (Sec. 4.3.2) at the paper's sizes: FIFO 5000,
+    replay pool 5000, pending ring 5000, records logged in flushes of 100.
+    Each timed round logs one flush (100 evictions) and runs one admission
+    round; a second series logs 4096 records per round."""
+    import torch
+    cfg = wl.cfg
+    r = H.Router.for_config(cfg, ring_capacity=5000, pending_capacity=5000, replay_capacity=5000,
+                            max_train_batch=4096)
+    dw = H.DeviceWorkload(wl, device=dev)
+    dw.load(r)
+    rng = np.random.default_rng(11)
+    x, y = W.records(rng, cfg, 20000)
+    xs, ys = torch.from_numpy(x).to(dev), torch.from_numpy(y).to(dev)
+    pos = 0
+
+    def log(k):
+        nonlocal pos
+        for a in range(0, k, 100):
+            b = min(k, a + 100)
+            i = pos % (len(ys) - 100)
+            r.log(xs[i:i + b - a], ys[i:i + b - a])
+            pos += b - a
+
+    log(10000)                                   # FIFO full, 5000 evicted and pending
+    r.replay_admit()                             # fills the replay pool
+    out = {"fifo": 5000, "replay": 5000, "pending": 5000, "hidden": cfg.widths[-2]}
+    for label, k in (("flush_100", 100), ("batch_4096", 4096)):
+        ts = []
+        for it in range(n + 3):
+            log(k)
+            flush.fill_(it & 0xFF)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            r.replay_admit()
+            e1.record(stream)
+            e1.synchronize()
+            ts.append(e0.elapsed_time(e1))
+        ms = float(np.mean(ts[3:]))
+        Hd, nR = cfg.widths[-2], 5000
+        flops = 2.0 * k * nR * Hd + 2.0 * nR * nR * Hd      # useful distance products
+        out[label] = {"ms_per_round": ms, "candidates": k, "useful_distance_gflop": flops / 1e9,
+                      "achieved_tflops": flops / 1e12 / (ms / 1e3),
+                      "frac_of_bf16_peak": flops / 1e12 / (ms / 1e3) / peaks["bf16_tflops"]}
+    info = r.info()
+    out["replay_count"] = int(info.replay_count)
+    r.close()
+    return out
 
 
 def dist_setup(n_gpus):
@@ -370,6 +424,12 @@ def main():
     loss = torch.zeros(1, device=dev)
     flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
+    if args.replay_only:
+        rp = measure_replay(L, H, W, wl, dev, flush, stream, measured_peaks()[0], n=max(args.steps, 4))
+        if rank == 0:
+            print(json.dumps({"workload": WORKLOAD, "replay_admission": rp}))
+        r.close()
+        return 0
     if args.guards_only:
         g = measure_guards(L, r, dw, N, R, cfg.d, min(ring, int(r.info().ring_count)), cfg.d_req, flush, stream,
                            measured_peaks()[0], n=max(args.steps, 4))
@@ -513,6 +573,9 @@ def main():
     train_roofline = (dict(kernel_roofline(max(train_kernels, key=lambda k: per_step[k])), branch="train")
                       if train_kernels else None)
 
+    replay = None
+    if not args.no_replay:
+        replay = measure_replay(L, H, W, wl, dev, flush, stream, peaks)
     guards = None
     if not args.no_guards:
         guards = measure_guards(L, r, dw, N, R, cfg.d, min(ring, int(r.info().ring_count)), cfg.d_req, flush,
@@ -629,6 +692,7 @@ def main():
             "clocks": clk,
             "algorithmic": costs,
             "guarded_route": guards,
+            "replay_admission": replay,
         }
         print(json.dumps(line))
     r.close()

@@ -115,7 +115,7 @@ void free_all(Ctx& c) {
                   c.gpart, c.loss_tmp, c.d_err, c.pub[0].img, c.pub[1].img, c.xin, c.xrq, c.pairx, c.ximg,
                   c.bkeys, c.work, c.work_n, c.gkeys, c.gmask, c.st, c.tf.base, c.tf.parts,
                   c.pub[0].bounds, c.pub[1].bounds, c.bounds_stage, c.benc, c.remb, c.rnorm, c.rpart, c.rd,
-                  c.rn, c.rinv};
+                  c.rn, c.rinv, c.rcount};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   if (c.ev_pub) cudaEventDestroy(c.ev_pub);
@@ -243,6 +243,7 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
     A(dalloc(&c.rd, cfg->pending_capacity));
     A(dalloc(&c.rn, cfg->replay_capacity));
     A(dalloc(&c.rinv, er));
+    A(dalloc(&c.rcount, 2));
   }
   A(dalloc(&c.hits, R * NI));
   A(dalloc(&c.scores, R * NI));

@@ -217,6 +217,7 @@ struct Ctx {
   float* rd = nullptr;            // d per candidate [P]
   float* rn = nullptr;            // n per kept record [Rc]
   int32_t* rinv = nullptr;        // rank -> candidate [P], then rank -> kept slot [Rc]
+  int64_t* rcount = nullptr;      // candidates and kept records of the round in flight [2]
   int64_t ring_enqueued = 0;
   // feature bounds of the ring (Algorithm 4 [l, u]): staged by ls_refresh_bounds,
   // published by ls_publish into pub[b].bounds
@@ -309,6 +310,13 @@ __device__ __forceinline__ bool last_block(uint32_t* done) {
   }
   __syncthreads();
   return is_last;
+}
+
+// Order-preserving 32-bit code of a float: unsigned comparison of codes is
+// the float comparison, -0 below +0.
+__device__ __forceinline__ uint32_t ord_code(float f) {
+  const uint32_t u = __float_as_uint(f);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
 // (a, i) precedes (b, j) in the order (score, index): NaN after every number,
@@ -418,9 +426,12 @@ cudaError_t forward_rows(Ctx& c, int B, cudaStream_t s);
 cudaError_t run_replay_admit(Ctx& c, float* d_out, float* n_out, cudaStream_t s);
 // row-min distance GEMM: out[row * ldp + part] = min over this CTA's columns n of
 // na[row] + nb[n] - 2 sum_k A(row, k) B(n, k), skipping n == row + self_off
+// rows_dev / cols_dev (device, nullable): rows / columns in use; CTAs whose
+// tile starts past them write +inf partials and stop.
 cudaError_t launch_rowmin_tc(int M, int N, int K, const float* A, int64_t lda, const float* B, int64_t ldb,
                              const float* na, const float* nb, int64_t self_off, float* part, int64_t ldp,
-                             int* parts_used, int* err, int sms, cudaStream_t s);
+                             const int64_t* rows_dev, const int64_t* cols_dev, int* parts_used, int* err, int sms,
+                             cudaStream_t s);
 constexpr int kRowMinParts = 256;  // partial columns per row of rpart
 cudaError_t run_train_step(Ctx& c, int batch, const int32_t* idx, int opt, float lr,
                            float* loss_out, cudaStream_t s);

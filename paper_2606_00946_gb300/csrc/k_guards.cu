@@ -30,14 +30,9 @@ constexpr unsigned kFull = 0xffffffffu;
 // feature bounds of the sample ring
 // ---------------------------------------------------------------------------
 
-// Order-preserving 32-bit code of a float (unsigned comparison of codes =
-// float comparison, -0 below +0): the block minima / maxima meet in global
-// memory through atomicMin / atomicMax on codes, so the result does not
+// The block minima / maxima meet in global memory through atomicMin /
+// atomicMax on order-preserving codes (ord_code), so the result does not
 // depend on which block finishes first.
-__device__ __forceinline__ uint32_t ord_code(float f) {
-  const uint32_t u = __float_as_uint(f);
-  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
-}
 __device__ __forceinline__ float ord_float(uint32_t e) {
   return __uint_as_float((e & 0x80000000u) ? (e & 0x7fffffffu) : ~e);
 }

@@ -13,7 +13,9 @@
 //   2. nearest-neighbour distances on tensor cores (launch_rowmin_tc: bf16
 //      products, fp32 sums, row minima per CTA) or on CUDA cores for small
 //      shapes (k_rowmin_simt), minima combined by k_rowmin_reduce;
-//   3. k_replay_rank: ranks by counting (candidates by d desc, kept by n asc);
+//   3. ranks (candidates by d desc, kept by n asc): k_replay_sort (bitonic,
+//      one block per pool) when a pool fits 16384 keys, else k_replay_rank
+//      (counting);
 //   4. k_replay_apply: free slots filled, then pairs replaced while d > n;
 //      the last block advances the pool size and the considered position.
 #include "common.cuh"
@@ -50,7 +52,13 @@ __device__ __forceinline__ int64_t embed_row_slot(int64_t r, const DevState* st,
 __global__ void k_replay_gather(int B, int64_t row0, int d, ReplayGeom g, const DevState* st,
                                 const float* __restrict__ ring_x, const float* __restrict__ ring_y,
                                 const float* __restrict__ mean, const float* __restrict__ stdv, int bf16,
-                                float* __restrict__ x0, float* __restrict__ y) {
+                                float* __restrict__ x0, float* __restrict__ y, int64_t* __restrict__ counts) {
+  if (row0 == 0 && blockIdx.x == 0 && threadIdx.x == 0) {  // the round's candidates and kept records
+    int64_t lo, hi;
+    pending_range(st, g, lo, hi);
+    counts[0] = hi - lo;
+    counts[1] = *reinterpret_cast<const volatile int64_t*>(&st->replay_count);
+  }
   const int64_t total = (int64_t)B * d;
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
     const int j = (int)(e / d), k = (int)(e - (int64_t)j * d);
@@ -159,6 +167,46 @@ __global__ void __launch_bounds__(256) k_replay_rank(ReplayGeom g, const DevStat
   if (i < cnt) inv[(cand ? 0 : g.P) + rank] = (int32_t)i;
 }
 
+// The same ranks by sorting, one block per pool (block 0 candidates, block 1
+// kept records): 64-bit keys (order code << 32 | index; the candidates' code
+// complemented for the descending order) sorted ascending in shared memory
+// by a bitonic network over n2 (a power of two) keys, padding keys all ones.
+__global__ void __launch_bounds__(1024) k_replay_sort(ReplayGeom g, const DevState* st, const float* __restrict__ dc,
+                                                      const float* __restrict__ nk, int32_t* __restrict__ inv,
+                                                      int n2c, int n2k) {
+  extern __shared__ uint64_t key[];
+  int64_t lo, hi;
+  pending_range(st, g, lo, hi);
+  const bool cand = blockIdx.x == 0;
+  const int64_t cnt = cand ? hi - lo : *reinterpret_cast<const volatile int64_t*>(&st->replay_count);
+  const int n2 = cand ? n2c : n2k;
+  const float* v = cand ? dc : nk;
+  for (int i = threadIdx.x; i < n2; i += blockDim.x) {
+    uint64_t k = ~0ull;
+    if (i < cnt) {
+      const uint32_t code = ord_code(div_key(v[i]));
+      k = ((uint64_t)(cand ? ~code : code) << 32) | (uint32_t)i;
+    }
+    key[i] = k;
+  }
+  __syncthreads();
+  for (int k = 2; k <= n2; k <<= 1)
+    for (int j = k >> 1; j > 0; j >>= 1) {
+      for (int i = threadIdx.x; i < n2; i += blockDim.x) {
+        const int p = i ^ j;
+        if (p > i) {
+          const uint64_t a = key[i], b = key[p];
+          if ((a > b) == ((i & k) == 0)) {
+            key[i] = b;
+            key[p] = a;
+          }
+        }
+      }
+      __syncthreads();
+    }
+  for (int r = threadIdx.x; r < cnt; r += blockDim.x) inv[(cand ? 0 : g.P) + r] = (int32_t)(key[r] & 0xffffffffu);
+}
+
 // One warp per candidate rank t: free slots first, then pairs while d > n.
 __global__ void __launch_bounds__(256) k_replay_apply(int d, ReplayGeom g, DevState* st, const float* __restrict__ dc,
                                                       const float* __restrict__ nk, const int32_t* __restrict__ inv,
@@ -190,6 +238,8 @@ __global__ void __launch_bounds__(256) k_replay_apply(int d, ReplayGeom g, DevSt
   }
 }
 
+constexpr int kSortMax = 16384;  // keys a block sorts in shared memory (128 KB)
+
 int grid_for(int64_t threads, int sms) {
   const int64_t b = (threads + 255) / 256;
   return (int)std::max<int64_t>(1, std::min<int64_t>(b, (int64_t)sms * 8));
@@ -210,7 +260,7 @@ cudaError_t run_replay_admit(Ctx& c, float* d_out, float* n_out, cudaStream_t s)
     const int B = (int)std::min<int64_t>(Bc, rows - row0);
     e = traced(c, TR_REPLAY, 1, s, [&] {
       k_replay_gather<<<grid_for((int64_t)B * m.w[0], c.sms), 256, 0, s>>>(
-          B, row0, m.w[0], g, c.st, c.ring_x, c.ring_y, c.mean, c.stdv, m.bf16, c.tx, c.ty);
+          B, row0, m.w[0], g, c.st, c.ring_x, c.ring_y, c.mean, c.stdv, m.bf16, c.tx, c.ty, c.rcount);
       return cudaGetLastError();
     });
     if (e != cudaSuccess) return e;
@@ -234,11 +284,12 @@ cudaError_t run_replay_admit(Ctx& c, float* d_out, float* n_out, cudaStream_t s)
   const float* nc = c.rnorm;
   const float* nkp = c.rnorm + g.P;
   const int64_t kNoSelf = -(int64_t(1) << 62);
-  auto rowmin = [&](int M, const float* A, const float* na, int64_t self_off, float* out) -> cudaError_t {
+  auto rowmin = [&](int M, const float* A, const float* na, int64_t self_off, const int64_t* rows_in_use,
+                    float* out) -> cudaError_t {
     int parts = 0;
     cudaError_t r = traced(c, TR_REPLAY, 1, s, [&] {
-      return launch_rowmin_tc(M, (int)g.Rc, H, A, H, Ek, H, na, nkp, self_off, c.rpart, kRowMinParts, &parts,
-                              c.d_err, c.sms, s);
+      return launch_rowmin_tc(M, (int)g.Rc, H, A, H, Ek, H, na, nkp, self_off, c.rpart, kRowMinParts, rows_in_use,
+                              c.rcount + 1, &parts, c.d_err, c.sms, s);
     });
     if (r == cudaSuccess) {
       return traced(c, TR_REPLAY, 1, s, [&] {
@@ -253,9 +304,9 @@ cudaError_t run_replay_admit(Ctx& c, float* d_out, float* n_out, cudaStream_t s)
       return cudaGetLastError();
     });
   };
-  e = rowmin((int)g.P, Ec, nc, kNoSelf, c.rd);
+  e = rowmin((int)g.P, Ec, nc, kNoSelf, c.rcount, c.rd);
   if (e != cudaSuccess) return e;
-  e = rowmin((int)g.Rc, Ek, nkp, 0, c.rn);
+  e = rowmin((int)g.Rc, Ek, nkp, 0, c.rcount + 1, c.rn);
   if (e != cudaSuccess) return e;
   if (d_out) {
     e = cudaMemcpyAsync(d_out, c.rd, (size_t)g.P * sizeof(float), cudaMemcpyDeviceToDevice, s);
@@ -267,8 +318,19 @@ cudaError_t run_replay_admit(Ctx& c, float* d_out, float* n_out, cudaStream_t s)
   }
   // 3. ranks, 4. admission
   e = traced(c, TR_REPLAY, 1, s, [&] {
-    const int blocks = (int)((g.P + 255) / 256 + (g.Rc + 255) / 256);
-    k_replay_rank<<<blocks, 256, 0, s>>>(g, c.st, c.rd, c.rn, c.rinv);
+    int n2c = 1, n2k = 1;
+    while (n2c < g.P) n2c <<= 1;
+    while (n2k < g.Rc) n2k <<= 1;
+    const int n2 = std::max(n2c, n2k);
+    if (n2 <= kSortMax) {
+      const int smem = n2 * (int)sizeof(uint64_t);
+      cudaError_t a = cudaFuncSetAttribute(k_replay_sort, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+      if (a != cudaSuccess) return a;
+      k_replay_sort<<<2, 1024, smem, s>>>(g, c.st, c.rd, c.rn, c.rinv, n2c, n2k);
+    } else {
+      const int blocks = (int)((g.P + 255) / 256 + (g.Rc + 255) / 256);
+      k_replay_rank<<<blocks, 256, 0, s>>>(g, c.st, c.rd, c.rn, c.rinv);
+    }
     return cudaGetLastError();
   });
   if (e != cudaSuccess) return e;

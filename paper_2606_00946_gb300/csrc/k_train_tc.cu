@@ -40,6 +40,8 @@ struct TcGemmArgs {
   const float* na;   // epilogue 3: row and column squared norms
   const float* nb;
   int64_t self_off;  // epilogue 3: column row + self_off is skipped
+  const int64_t* rows_dev;  // epilogue 3: rows / columns in use (device, nullable)
+  const int64_t* cols_dev;
   int* err;
   uint32_t tmem_cols;
 };
@@ -144,6 +146,12 @@ __global__ void __launch_bounds__(kT) k_gemm_tc(const __grid_constant__ TcGemmAr
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int m0 = blockIdx.y * kM, n0 = blockIdx.x * g.ntile;
+  if (g.epi == 3 && ((g.rows_dev && m0 >= *g.rows_dev) || (g.cols_dev && n0 >= *g.cols_dev))) {
+    // nothing of this tile is in use: its partial minima are +inf
+    const int r = m0 + 32 * (warp & 3) + lane;
+    if (r < g.M) g.C[(int64_t)r * g.ldc + 2 * blockIdx.x + (warp >> 2)] = INFINITY;
+    return;
+  }
   const int64_t kbeg = (int64_t)blockIdx.z * g.kper;
   const int64_t kend = kbeg + g.kper < g.K ? kbeg + g.kper : g.K;
   const int nchunks = kend > kbeg ? (int)((kend - kbeg + 63) / 64) : 0;
@@ -336,7 +344,8 @@ cudaError_t launch_gemm_tc(int M, int N, int K, const float* A, int64_t sam, int
 
 cudaError_t launch_rowmin_tc(int M, int N, int K, const float* A, int64_t lda, const float* B, int64_t ldb,
                              const float* na, const float* nb, int64_t self_off, float* part, int64_t ldp,
-                             int* parts_used, int* err, int sms, cudaStream_t s) {
+                             const int64_t* rows_dev, const int64_t* cols_dev, int* parts_used, int* err, int sms,
+                             cudaStream_t s) {
   if (M < 64 || N < 32 || K < 1) return cudaErrorInvalidValue;
   const int mt = (M + kM - 1) / kM;
   int ntile = 256;
@@ -353,6 +362,7 @@ cudaError_t launch_rowmin_tc(int M, int N, int K, const float* A, int64_t lda, c
   g.epi = 3;
   g.C = part; g.ldc = ldp;
   g.na = na; g.nb = nb; g.self_off = self_off;
+  g.rows_dev = rows_dev; g.cols_dev = cols_dev;
   g.err = err;
   g.tmem_cols = 32;
   while ((int)g.tmem_cols < ntile) g.tmem_cols <<= 1;
