@@ -70,7 +70,9 @@ def lib():
             L.or_argmin.argtypes = [i64, i32, P, P, P]
             L.or_ring_append.argtypes = [i64, C.c_int, P, P, i64, i64, P, P]
             L.or_train_step.argtypes = [C.c_int, C.c_int, P, P, P, P, i64, C.c_int, dbl,
-                                        C.c_int, P, P, P, P, P, P, P]
+                                        C.c_int, P, P, P, P, P, P, P, C.c_float, C.c_uint64]
+            L.or_drop_keep.restype = C.c_int
+            L.or_drop_keep.argtypes = [C.c_uint64, C.c_float, i64, C.c_int, i64, C.c_int]
             L.or_loss.argtypes = [C.c_int, C.c_int, P, P, C.c_int, P, P, P, P, P, P]
             L.or_ring_bounds.argtypes = [i64, C.c_int, P, i64, P, P]
             L.or_hrw_candidates.restype = i32
@@ -266,7 +268,8 @@ def ring_append(ring_x, ring_y, count, x, y):
 class Trainer:
     """Oracle optimiser state: fp32-valued params, Adam moments, step count."""
 
-    def __init__(self, widths, params, mode="f32"):
+    def __init__(self, widths, params, mode="f32", dropout=0.0, dropout_seed=0):
+        self.dropout, self.dropout_seed = float(dropout), int(dropout_seed)
         self.w = _c(widths, np.int32)
         self.mode = MODES.get(mode, mode)
         self.params = _c(params, np.float64).copy()
@@ -284,7 +287,8 @@ class Trainer:
                                  float(lr), len(idx), _p(_c(ring_x, np.float32)),
                                  _p(_c(ring_y, np.float32)), _p(idx), _p(_c(mean, np.float32)),
                                  _p(_c(std, np.float32)), _p(loss),
-                                 _p(g) if g is not None else None)
+                                 _p(g) if g is not None else None, self.dropout,
+                                 C.c_uint64(self.dropout_seed & (2**64 - 1)))
         _check(rc, "train_step")
         return (float(loss[0]), g) if want_grad else float(loss[0])
 
@@ -414,3 +418,8 @@ def replay_select(d, n, cap):
     _check(lib().or_replay_select(len(d), _p(d if len(d) else np.zeros(1)), len(n),
                                   _p(n if len(n) else np.zeros(1)), int(cap), _p(src), _p(cnt)), "replay_select")
     return src[:int(cnt[0])], int(cnt[0])
+
+
+def drop_keep(seed, p, t, h, j, o) -> bool:
+    """Dropout keep decision of unit o of hidden activation h, minibatch row j, step t."""
+    return bool(lib().or_drop_keep(C.c_uint64(seed & (2**64 - 1)), float(p), int(t), int(h), int(j), int(o)))

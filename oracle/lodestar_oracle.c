@@ -275,15 +275,45 @@ int64_t or_param_count(int n_layers, const int *w) {
     return param_offset(n_layers, w, n_layers, 0);
 }
 
+/* Dropout between hidden layers (Sec. 4.1 Model architecture: dropout 0.1
+ * between hidden layers; training only).  The keep decision of unit o of
+ * hidden activation h (1-based layer output) for minibatch row j at optimiser
+ * step t comes from a counter-based generator built on mix64:
+ *   h1 = mix64(seed ^ ((t << 16) | h)),  u = mix64(h1 ^ ((j << 20) | o)),
+ *   keep  <=>  (u >> 11) >= ceil(p 2^53)      (a uniform on [0, 1) >= p),
+ * and kept units are scaled by s = fp32(1 / (1 - p)).  Hidden activations
+ * that feed another hidden layer are dropped; the last one is not. */
+typedef struct {
+    uint64_t seed, thr;  /* thr = ceil(p 2^53); 0 = no dropout */
+    float scale;         /* fp32 1 / (1 - p) (fp32 and bf16 modes) */
+    double p;            /* the rate (fp64 mode scales by 1 / (1 - p) exactly) */
+    int64_t t, j;
+} or_drop;
+
+static int drop_keep(const or_drop *dr, int h, int o) {
+    uint64_t h1 = or_mix64(dr->seed ^ (((uint64_t)dr->t << 16) | (uint64_t)h));
+    uint64_t u = or_mix64(h1 ^ (((uint64_t)dr->j << 20) | (uint64_t)o));
+    return (u >> 11) >= dr->thr;
+}
+
+uint64_t or_drop_threshold(float p) { return (uint64_t)ceil((double)p * 9007199254740992.0); }
+float or_drop_scale(float p) { return (float)(1.0 / (1.0 - (double)p)); }
+
+/* keep decision for the pins: 1 kept, 0 dropped */
+int or_drop_keep(uint64_t seed, float p, int64_t t, int h, int64_t j, int o) {
+    or_drop dr = {seed, or_drop_threshold(p), or_drop_scale(p), (double)p, t, j};
+    return drop_keep(&dr, h, o);
+}
+
 /* Forward pass of one row.  z_l = W_l a_{l-1} + b_l summed in fp64; a_l = relu(z_l)
  * for hidden layers; the last layer is linear.  Rounding per mode:
  *   F64 : none;  F32 : each z_l rounded to fp32;
  *   BF16: additionally W_l, a_0 = x and every hidden a_l rounded to bf16.
  * If z_save / a_save are given, z_l and a_l of every layer are stored at
  * offsets act_off[l] (the input a_0 at a_save + 0). */
-static double forward_row(int mode, int n_layers, const int *w, const double *params,
-                          const double *x, double *z_save, double *a_save, const int64_t *act_off,
-                          double *buf_a, double *buf_b) {
+static double forward_row_drop(int mode, int n_layers, const int *w, const double *params,
+                               const double *x, double *z_save, double *a_save, const int64_t *act_off,
+                               double *buf_a, double *buf_b, const or_drop *dr) {
     double *a = buf_a, *z = buf_b;
     for (int k = 0; k < w[0]; ++k) a[k] = rnd_op(mode, x[k]);
     if (a_save) for (int k = 0; k < w[0]; ++k) a_save[k] = a[k];
@@ -297,8 +327,13 @@ static double forward_row(int mode, int n_layers, const int *w, const double *pa
         }
         if (z_save) for (int o = 0; o < w[l + 1]; ++o) z_save[act_off[l + 1] + o] = z[o];
         if (l + 1 < n_layers) {
+            int dropped = dr && dr->thr > 0 && l + 2 < n_layers;
             for (int o = 0; o < w[l + 1]; ++o) {
                 double r = z[o] > 0.0 ? z[o] : 0.0;
+                if (dropped) {  /* scale in the mode's working precision, then round the operand */
+                    if (!drop_keep(dr, l + 1, o)) r = 0.0;
+                    else r = mode == OR_F64 ? r * (1.0 / (1.0 - dr->p)) : (double)((float)r * dr->scale);
+                }
                 z[o] = rnd_op(mode, r);
             }
             if (a_save) for (int o = 0; o < w[l + 1]; ++o) a_save[act_off[l + 1] + o] = z[o];
@@ -306,6 +341,12 @@ static double forward_row(int mode, int n_layers, const int *w, const double *pa
         double *t = a; a = z; z = t;
     }
     return a[0];
+}
+
+static double forward_row(int mode, int n_layers, const int *w, const double *params,
+                          const double *x, double *z_save, double *a_save, const int64_t *act_off,
+                          double *buf_a, double *buf_b) {
+    return forward_row_drop(mode, n_layers, w, params, x, z_save, a_save, act_off, buf_a, buf_b, NULL);
 }
 
 static int max_width(int n_layers, const int *w) {
@@ -387,7 +428,8 @@ int or_ring_append(int64_t capacity, int d, float *ring_x, float *ring_y, int64_
 int or_train_step(int mode, int n_layers, const int *w, double *params, double *adam_m,
                   double *adam_v, int64_t t, int opt, double lr, int batch,
                   const float *ring_x, const float *ring_y, const int32_t *idx,
-                  const float *mean, const float *std, double *loss_out, double *grad_out) {
+                  const float *mean, const float *std, double *loss_out, double *grad_out,
+                  float drop_p, uint64_t drop_seed) {
     const double b1 = 0.9, b2 = 0.999, eps = 1e-8;
     int d = w[0];
     int64_t P = or_param_count(n_layers, w);
@@ -407,14 +449,17 @@ int or_train_step(int mode, int n_layers, const int *w, double *params, double *
     float *xf = (float *)malloc((size_t)d * sizeof(float));
     double *yhat = (double *)malloc((size_t)(batch > 0 ? batch : 1) * sizeof(double));
     if (!Z || !A || !g || !dz || !dz_prev || !ba || !bb || !xr || !xf || !yhat) return -1;
+    or_drop dr = {drop_seed, drop_p > 0.0f ? or_drop_threshold(drop_p) : 0, or_drop_scale(drop_p),
+                  (double)drop_p, t, 0};
 
     /* forward */
     double loss = 0.0;
     for (int j = 0; j < batch; ++j) {
         or_zscore(d, ring_x + (int64_t)idx[j] * d, mean, std, xf);
         for (int k = 0; k < d; ++k) xr[k] = (double)xf[k];
-        yhat[j] = forward_row(mode, n_layers, w, params, xr, Z + (int64_t)j * act_row,
-                              A + (int64_t)j * act_row, act_off, ba, bb);
+        dr.j = j;
+        yhat[j] = forward_row_drop(mode, n_layers, w, params, xr, Z + (int64_t)j * act_row,
+                                   A + (int64_t)j * act_row, act_off, ba, bb, &dr);
         double e = yhat[j] - (double)ring_y[idx[j]];
         loss += e * e;
     }
@@ -441,14 +486,23 @@ int or_train_step(int mode, int n_layers, const int *w, double *params, double *
             }
         }
         if (l > 0) {
-            for (int j = 0; j < batch; ++j)
+            /* input a_l is hidden activation h = l; it was dropped when it feeds
+             * another hidden layer (l < n_layers - 1) */
+            int dropped = dr.thr > 0 && l < n_layers - 1;
+            for (int j = 0; j < batch; ++j) {
+                dr.j = j;
                 for (int k = 0; k < fi; ++k) {
                     double s = 0.0;
                     for (int o = 0; o < fo; ++o)
                         s += rnd_op(mode, dz[(int64_t)j * m + o]) * rnd_op(mode, W[(int64_t)o * fi + k]);
                     double zprev = Z[(int64_t)j * act_row + act_off[l] + k];
-                    dz_prev[(int64_t)j * m + k] = zprev > 0.0 ? rnd(mode, s) : 0.0;
+                    double v = zprev > 0.0 ? rnd(mode, s) : 0.0;
+                    if (dropped && v != 0.0)
+                        v = !drop_keep(&dr, l, k) ? 0.0
+                            : (mode == OR_F64 ? v * (1.0 / (1.0 - dr.p)) : (double)((float)v * dr.scale));
+                    dz_prev[(int64_t)j * m + k] = v;
                 }
+            }
             double *tmp = dz; dz = dz_prev; dz_prev = tmp;
         }
     }
