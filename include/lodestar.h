@@ -106,6 +106,16 @@ typedef struct {
      * without).  0 / 0: FIFO only. */
     int64_t replay_capacity;
     int64_t pending_capacity;
+    /* Dropout between hidden layers during training (Sec. 4.1 Model
+     * architecture: 0.1), 0 <= dropout < 1; 0 = none.  Unit o of hidden
+     * activation h (one that feeds another hidden layer) in minibatch row j
+     * at optimiser step t is kept when (u >> 11) >= ceil(dropout 2^53), u =
+     * mix64(mix64(dropout_seed ^ ((t << 16) | h)) ^ ((j << 20) | o)), and
+     * kept units are scaled by fp32(1 / (1 - dropout)).  Needs the
+     * tensor-core training path (bf16, hidden widths <= 256): LS_ERR_ARG
+     * otherwise. */
+    float dropout;
+    uint64_t dropout_seed;
 } ls_config;
 
 typedef struct {

@@ -85,6 +85,7 @@ bool check_config(const ls_config* c, std::string& why) {
     return false;
   }
   if (c->max_batch_tokens < 1) { why = "max_batch_tokens must be >= 1"; return false; }
+  if (!(c->dropout >= 0.0f && c->dropout < 1.0f)) { why = "dropout must be in [0, 1)"; return false; }
   if (c->replay_capacity < 0 || c->pending_capacity < 0 || ((c->replay_capacity > 0) != (c->pending_capacity > 0))) {
     why = "replay_capacity and pending_capacity must both be 0 or both be >= 1";
     return false;
@@ -259,7 +260,13 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
   A(dalloc(&c.d_err, 1));
   A(dalloc(&c.st, 1));
   int64_t tf_bytes = 0;
-  if (plan_train_fast(m, cfg->max_train_batch, c.tf)) {
+  const bool fast_train = plan_train_fast(m, cfg->max_train_batch, c.tf);
+  if (cfg->dropout > 0.0f && !fast_train) {
+    free_all(c);
+    delete h;
+    return fail(LS_ERR_ARG, "dropout needs the tensor-core training path (bf16, hidden widths <= 256)");
+  }
+  if (fast_train) {
     int64_t pf = 0;
     tf_bytes = train_fast_bytes(m, c.tf, &pf);
     A(dalloc(&c.tf.base, tf_bytes));

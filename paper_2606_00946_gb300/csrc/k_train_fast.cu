@@ -24,6 +24,7 @@
 #include <algorithm>
 #include <cmath>
 
+#include "blockhash.cuh"
 #include "common.cuh"
 #include "sm100.cuh"
 
@@ -70,12 +71,19 @@ struct TrJob {
   float* partWL;                     // [m_tiles][N]
   float* partBL;                     // [m_tiles]
   float* partLoss;                   // [m_tiles]
+  // dropout between hidden layers (0 = none): TE_FWD drops units of hidden
+  // activation drop_h and scales the kept ones; TE_DX scales the gradient of
+  // the dropped activation drop_h (its keep bits are in mask_in)
+  int drop_h;
 };
 
 struct TrArgs {
   TrJob job[2];
   int n_cta0;                        // CTAs of job 0; the rest run job 1
   int* err;
+  const DevState* st;                // optimiser step counter (dropout stream)
+  uint64_t drop_seed, drop_thr;      // keep <=> (u >> 11) >= drop_thr
+  float drop_scale;                  // fp32 1 / (1 - p)
 };
 
 __device__ __forceinline__ uint16_t bf16_bits(float x) {
@@ -224,6 +232,14 @@ __global__ void __launch_bounds__(kT, 1) k_tr_gemm(const __grid_constant__ TrArg
       }
     }
   } else if (ok && J.epi == TE_FWD) {
+    // dropout stream of this activation at step t = step + 1 (Sec. 4.1: dropout
+    // between hidden layers): h1 = mix64(seed ^ ((t << 16) | h)),
+    // u = mix64(h1 ^ ((row << 20) | unit)), kept when (u >> 11) >= thr
+    uint64_t h1 = 0;
+    if (J.drop_h > 0) {
+      const uint64_t t = (uint64_t)(*reinterpret_cast<const volatile int64_t*>(&args.st->step) + 1);
+      h1 = bh::mix64(args.drop_seed ^ ((t << 16) | (uint64_t)J.drop_h));
+    }
     for (int c = cbeg; c < cbeg + cw; c += 16) {
       uint32_t v[16];
       tmem_ld16x(tmem + lane_addr + (uint32_t)c, v);
@@ -233,8 +249,16 @@ __global__ void __launch_bounds__(kT, 1) k_tr_gemm(const __grid_constant__ TrArg
 #pragma unroll
       for (int u = 0; u < 16; ++u) {
         const float z = __uint_as_float(v[u]) + s_bias[c + u];
-        bits |= (z > 0.0f ? 1u : 0u) << u;
-        a[u] = round_bf16(z > 0.0f ? z : 0.0f);
+        float r = z > 0.0f ? z : 0.0f;
+        bool on = z > 0.0f;
+        if (J.drop_h > 0) {
+          const uint64_t hu = bh::mix64(h1 ^ (((uint64_t)j << 20) | (uint64_t)(n0 + c + u)));
+          const bool keep = (hu >> 11) >= args.drop_thr;
+          on = on && keep;
+          r = keep ? r * args.drop_scale : 0.0f;
+        }
+        bits |= (on ? 1u : 0u) << u;
+        a[u] = round_bf16(r);
       }
       J.mask_out[(int64_t)((n0 + c) >> 4) * J.rows_pad + j] = (uint16_t)bits;
       store_row16(J.out, J.rows_pad, j, n0 + c, a);
@@ -247,8 +271,9 @@ __global__ void __launch_bounds__(kT, 1) k_tr_gemm(const __grid_constant__ TrArg
       tmem_wait_ld();
       const uint32_t bits = J.mask_in[(int64_t)((n0 + c) >> 4) * J.rows_pad + j];
       float dz[16];
+      const float sc = J.drop_h > 0 ? args.drop_scale : 1.0f;
 #pragma unroll
-      for (int u = 0; u < 16; ++u) dz[u] = ((bits >> u) & 1u) ? __uint_as_float(v[u]) : 0.0f;
+      for (int u = 0; u < 16; ++u) dz[u] = ((bits >> u) & 1u) ? __uint_as_float(v[u]) * sc : 0.0f;
       if (J.out) store_row16(J.out, J.rows_pad, j, n0 + c, dz);
       store_col16(J.outT, J.rT, j, n0 + c, dz);
       const float sb = col_reduce16(dz);
@@ -509,8 +534,12 @@ int gemm_smem_bytes() {
   return 1024 + kMaxChunks * (kM * 128 + 256 * 128) + 128 + (256 + 256 + 8 * 256 + 4 * 128 + 128 + 128 + 8) * 4;
 }
 
-cudaError_t launch_tr_gemm(const TrJob& j0, const TrJob* j1, int* err, cudaStream_t s) {
+cudaError_t launch_tr_gemm(const Ctx& c, const TrJob& j0, const TrJob* j1, int* err, cudaStream_t s) {
   TrArgs a{};
+  a.st = c.st;
+  a.drop_seed = c.cfg.dropout_seed;
+  a.drop_thr = c.cfg.dropout > 0.0f ? (uint64_t)std::ceil((double)c.cfg.dropout * 9007199254740992.0) : 0;
+  a.drop_scale = (float)(1.0 / (1.0 - (double)c.cfg.dropout));
   a.job[0] = j0;
   a.n_cta0 = j0.m_tiles * j0.n_split * j0.splits;
   int n = a.n_cta0;
@@ -697,7 +726,9 @@ cudaError_t run_train_fast(Ctx& c, int B, const int32_t* idx, int opt, float lr,
       J.partBL = f.partBL;
       J.partLoss = f.partLoss;
     }
-    e = traced(c, TR_GEMM_TC_FWD, 1, s, [&] { return launch_tr_gemm(J, nullptr, c.d_err, s); });
+    // dropout on hidden activation l + 1 when it feeds another hidden layer
+    J.drop_h = (c.cfg.dropout > 0.0f && l + 2 < m.n_layers) ? l + 1 : 0;
+    e = traced(c, TR_GEMM_TC_FWD, 1, s, [&] { return launch_tr_gemm(c, J, nullptr, c.d_err, s); });
     if (e != cudaSuccess) return e;
   }
   // backward: dW_l (split over the batch) and, for l > 0, dz_{l-1} in the same launch
@@ -739,9 +770,10 @@ cudaError_t run_train_fast(Ctx& c, int B, const int32_t* idx, int opt, float lr,
       X.outT = f.imgDZT[(l - 1) & 1];
       X.rT = ((m.w[l] + 127) / 128) * 128;
       X.colpart = f.partB[l - 1];
+      X.drop_h = (c.cfg.dropout > 0.0f && l < m.n_layers - 1) ? l : 0;  // input a_l was dropped
     }
     e = traced(c, l > 0 ? TR_GEMM_TC_DX : TR_GEMM_TC_DW, 1, s,
-               [&] { return launch_tr_gemm(W, l > 0 ? &X : nullptr, c.d_err, s); });
+               [&] { return launch_tr_gemm(c, W, l > 0 ? &X : nullptr, c.d_err, s); });
     if (e != cudaSuccess) return e;
   }
   OptArgs a{};

@@ -61,7 +61,7 @@ def _torch_grad(widths, params, x, y, idx, mean, std, p, seed, t):
     for l in range(L):
         g.append(Ws[l].grad.numpy().ravel())
         g.append(bs[l].grad.numpy())
-    return float(loss), np.concatenate(g)
+    return float(loss.detach()), np.concatenate(g)
 
 
 @pytest.mark.parametrize("widths", [(16, 32, 32, 32, 1), (16, 24, 24, 1)])
