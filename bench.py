@@ -45,6 +45,8 @@ def parse():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-guards", action="store_true", help="skip the guarded-route measurement")
     p.add_argument("--no-replay", action="store_true", help="skip the replay-pool admission measurement")
+    p.add_argument("--no-paper-point", action="store_true", help="skip the paper operating-point measurement")
+    p.add_argument("--paper-point-only", action="store_true", help="only the paper operating-point measurement")
     p.add_argument("--replay-only", action="store_true",
                    help="only the replay-pool admission measurement (for kernel profiling)")
     p.add_argument("--guards-only", action="store_true",
@@ -172,6 +174,89 @@ def measure_replay(L, H, W, wl, dev, flush, stream, peaks, n=20):
     out["replay_count"] = int(info.replay_count)
     r.close()
     return out
+
+
+def measure_paper_point(L, H, W, dev, stream, n=400):
+    """The paper's operating point (Sec. 4.3.1 P1, Sec. 5.5 overhead): one
+    request routed over 16 instances by the 3 x 128 predictor, and its
+    training recipe (FIFO 5000 + replay 5000, dropout 0.1, Adam).  Latency of
+    a single-request route: host wall clock of the call through the C ABI
+    until its result is on the host, device time of the call (events), and
+    one replay of the route captured in a CUDA graph."""
+    import time
+    import torch
+    wl = W.generate("paper")
+    cfg = wl.cfg
+    r = H.Router.for_config(cfg, max_requests=1, ring_capacity=5000, pending_capacity=5000, replay_capacity=5000,
+                            max_train_batch=4096, dropout=0.1, dropout_seed=1)
+    dw = H.DeviceWorkload(wl, device=dev)
+    dw.load(r)
+    N = cfg.n_inst
+    out = {"choice": torch.empty(1, dtype=torch.int32, device=dev), "best": torch.empty(1, device=dev),
+           "scores": None, "hits": None}
+    h_choice = torch.empty(1, dtype=torch.int32).pin_memory()
+    offs = [dw.tok_off[i:i + 2] for i in range(cfg.n_req)]
+    reqs = [dw.req_feats[i:i + 1] for i in range(cfg.n_req)]
+    wall, dev_ms = [], []
+    for k in range(n + 20):
+        i = k % cfg.n_req
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        e0.record(stream)
+        r.route(dw.tok, offs[i], reqs[i], N, out=out)
+        e1.record(stream)
+        h_choice.copy_(out["choice"], non_blocking=True)
+        stream.synchronize()
+        t1 = time.perf_counter()
+        if k >= 20:
+            wall.append(1e6 * (t1 - t0))
+            dev_ms.append(1e3 * e0.elapsed_time(e1))
+    g_off, g_req = offs[0].clone(), reqs[0].clone()
+    graph = H.StepGraph(lambda: r.route(dw.tok, g_off, g_req, N, out=out))
+    gt = []
+    for k in range(n + 20):
+        i = k % cfg.n_req
+        g_off.copy_(offs[i])
+        g_req.copy_(reqs[i])
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        graph.replay()
+        e1.record(stream)
+        e1.synchronize()
+        if k >= 20:
+            gt.append(1e3 * e0.elapsed_time(e1))
+    # training recipe: a round over F u R in minibatches of 4096 (Adam, dropout 0.1)
+    x, y = W.records(np.random.default_rng(3), cfg, 15000)
+    r.log(torch.from_numpy(x[:5000]).to(dev), torch.from_numpy(y[:5000]).to(dev))
+    r.log(torch.from_numpy(x[5000:10000]).to(dev), torch.from_numpy(y[5000:10000]).to(dev))
+    r.replay_admit()
+    r.log(torch.from_numpy(x[10000:]).to(dev), torch.from_numpy(y[10000:]).to(dev))
+    r.replay_admit()
+    info = r.info()
+    buf = min(info.ring_count, 5000) + info.replay_count
+    ts = []
+    for k in range(23):
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        r.train(4096, None, opt="adam", lr=3e-4)
+        e1.record(stream)
+        e1.synchronize()
+        if k >= 3:
+            ts.append(e0.elapsed_time(e1))
+    r.close()
+    pct = lambda v, q: float(np.percentile(v, q))
+    return {"instances": N, "predictor": "x".join(str(w) for w in cfg.widths),
+            "route_host_us": {"p50": pct(wall, 50), "p99": pct(wall, 99)},
+            "route_device_us": {"p50": pct(dev_ms, 50), "p99": pct(dev_ms, 99)},
+            "route_graph_replay_us": {"p50": pct(gt, 50), "p99": pct(gt, 99)},
+            "train_buffer_records": int(buf), "train_step_ms_batch_4096": float(np.mean(ts)),
+            "train_samples_per_s": 4096 / (float(np.mean(ts)) / 1e3),
+            "note": "the paper reports a few milliseconds of router overhead per request (Fig. overhead); "
+                    "host time here is the C-ABI call from Python until the choice is in pinned host memory"}
 
 
 def dist_setup(n_gpus):
@@ -424,6 +509,12 @@ def main():
     loss = torch.zeros(1, device=dev)
     flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
+    if args.paper_point_only:
+        pp = measure_paper_point(L, H, W, dev, stream)
+        if rank == 0:
+            print(json.dumps({"paper_point": pp}))
+        r.close()
+        return 0
     if args.replay_only:
         rp = measure_replay(L, H, W, wl, dev, flush, stream, measured_peaks()[0], n=max(args.steps, 4))
         if rank == 0:
@@ -573,6 +664,9 @@ def main():
     train_roofline = (dict(kernel_roofline(max(train_kernels, key=lambda k: per_step[k])), branch="train")
                       if train_kernels else None)
 
+    paper_point = None
+    if not args.no_paper_point:
+        paper_point = measure_paper_point(L, H, W, dev, stream)
     replay = None
     if not args.no_replay:
         replay = measure_replay(L, H, W, wl, dev, flush, stream, peaks)
@@ -693,6 +787,7 @@ def main():
             "algorithmic": costs,
             "guarded_route": guards,
             "replay_admission": replay,
+            "paper_point": paper_point,
         }
         print(json.dumps(line))
     r.close()

@@ -78,6 +78,10 @@ CONFIGS = {
     "training": Config("training", 4, 64, 8192, ("loguniform", 8192, 32768), 256,
                        1.1, 65536, 66, 56, (256, 256, 256), "bf16", 3,
                        n_samples=1 << 20),
+    # the paper's operating point: one request at a time over 16 instances, its
+    # predictor size (3 hidden layers of 128, Sec. 4.1), a pool of 256 requests
+    "paper": Config("paper", 6, 16, 256, ("uniform", 64, 4096), 256, 1.1, 16384, 34, 24,
+                    (128, 128, 128), "bf16", 1, n_samples=10000),
     # 256 instances x 16384 requests, 1M cached blocks each, bf16 128->512->512->1
     "large": Config("large", 5, 256, 16384, ("uniform", 128, 16384), 4096, 1.1,
                     1 << 20, 66, 56, (512, 512), "bf16", 3),
