@@ -177,7 +177,7 @@ def measure_replay(L, H, W, wl, dev, flush, stream, peaks, n=20):
 
 
 def measure_paper_point(L, H, W, dev, stream, n=400):
-    """The paper's operating point (Sec. 4.3.1 P1, Sec. 5.5 overhead): one
+    """The paper's operating point (Sec. 4.3.1 P1, Sec. 5.4 overhead): one
     request routed over 16 instances by the 3 x 128 predictor, and its
     training recipe (FIFO 5000 + replay 5000, dropout 0.1, Adam).  Latency of
     a single-request route: host wall clock of the call through the C ABI
