@@ -116,7 +116,7 @@ void free_all(Ctx& c) {
                   c.gpart, c.loss_tmp, c.d_err, c.pub[0].img, c.pub[1].img, c.xin, c.xrq, c.pairx, c.ximg,
                   c.bkeys, c.work, c.work_n, c.gkeys, c.gmask, c.st, c.tf.base, c.tf.parts,
                   c.pub[0].bounds, c.pub[1].bounds, c.bounds_stage, c.benc, c.remb, c.rnorm, c.rpart, c.rd,
-                  c.rn, c.rinv, c.rcount};
+                  c.rn, c.rinv, c.rcount, c.rimg, c.rrank};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   if (c.ev_pub) cudaEventDestroy(c.ev_pub);
@@ -240,11 +240,15 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
     const int64_t er = cfg->pending_capacity + cfg->replay_capacity;
     A(dalloc(&c.remb, er * m.w[m.n_layers - 1]));
     A(dalloc(&c.rnorm, er));
-    A(dalloc(&c.rpart, std::max(cfg->pending_capacity, cfg->replay_capacity) * kRowMinParts));
+    A(dalloc(&c.rpart, er * kRowMinParts));
+    const int H = m.w[m.n_layers - 1];
+    if (m.bf16 && H % 64 == 0 && H <= 256)  // tensor-core distances from a bf16 image
+      A(dalloc(&c.rimg, ((cfg->pending_capacity + 127) / 128 + (cfg->replay_capacity + 127) / 128) * 128 * H * 2));
     A(dalloc(&c.rd, cfg->pending_capacity));
     A(dalloc(&c.rn, cfg->replay_capacity));
     A(dalloc(&c.rinv, er));
-    A(dalloc(&c.rcount, 2));
+    A(dalloc(&c.rrank, er));
+    A(dalloc(&c.rcount, 2 + (er + cfg->max_train_batch - 1) / cfg->max_train_batch));
   }
   A(dalloc(&c.hits, R * NI));
   A(dalloc(&c.scores, R * NI));

@@ -217,7 +217,9 @@ struct Ctx {
   float* rd = nullptr;            // d per candidate [P]
   float* rn = nullptr;            // n per kept record [Rc]
   int32_t* rinv = nullptr;        // rank -> candidate [P], then rank -> kept slot [Rc]
+  int32_t* rrank = nullptr;       // rank of each candidate [P], then of each kept record [Rc]
   int64_t* rcount = nullptr;      // candidates and kept records of the round in flight [2]
+  uint8_t* rimg = nullptr;        // bf16 embedding image (128-row tiles, MMA layout) for bf16 predictors
   int64_t ring_enqueued = 0;
   // feature bounds of the ring (Algorithm 4 [l, u]): staged by ls_refresh_bounds,
   // published by ls_publish into pub[b].bounds
@@ -421,8 +423,9 @@ cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const Published* 
                             cudaStream_t s);
 cudaError_t launch_ring_append(int n, int d, const float* x, const float* y, float* ring_x,
                                float* ring_y, DevState* st, int64_t capacity, int64_t pending, cudaStream_t s);
-// forward of B rows already in c.tx (layer inputs), keeping z_l in c.tz and a_l in c.tx
-cudaError_t forward_rows(Ctx& c, int B, cudaStream_t s);
+// forward of B rows already in c.tx (layer inputs), keeping z_l in c.tz and a_l in c.tx;
+// rows_dev (device, nullable): rows in use, the tensor-core products skip tiles past it
+cudaError_t forward_rows(Ctx& c, int B, cudaStream_t s, const int64_t* rows_dev = nullptr);
 cudaError_t run_replay_admit(Ctx& c, float* d_out, float* n_out, cudaStream_t s);
 // row-min distance GEMM: out[row * ldp + part] = min over this CTA's columns n of
 // na[row] + nb[n] - 2 sum_k A(row, k) B(n, k), skipping n == row + self_off
@@ -438,7 +441,8 @@ cudaError_t run_train_step(Ctx& c, int batch, const int32_t* idx, int opt, float
 cudaError_t launch_gemm_tc(int M, int N, int K, const float* A, int64_t sam, int64_t sak, const float* B,
                            int64_t sbn, int64_t sbk, int splits, int epi, float* C, int64_t ldc,
                            int64_t split_stride, const float* bias, float* act, int64_t ld_act, int hidden,
-                           const float* zprev, int64_t ld_zprev, int* err, int sms, cudaStream_t s);
+                           const float* zprev, int64_t ld_zprev, int* err, int sms, cudaStream_t s,
+                           const int64_t* rows_dev = nullptr);  // rows in use (device): later tiles skip
 int gemm_tc_splits_used(int K, int splits);
 int index_words(int max_instances);
 bool plan_train_fast(const MlpDesc& m, int max_batch, TrainFast& f);

@@ -13,15 +13,17 @@
 //   2. nearest-neighbour distances on tensor cores (launch_rowmin_tc: bf16
 //      products, fp32 sums, row minima per CTA) or on CUDA cores for small
 //      shapes (k_rowmin_simt), minima combined by k_rowmin_reduce;
-//   3. ranks (candidates by d desc, kept by n asc): k_replay_sort (bitonic,
-//      one block per pool) when a pool fits 16384 keys, else k_replay_rank
-//      (counting);
+//   3. ranks (candidates by d desc, kept by n asc) by counting over
+//      (element tile, key tile) blocks (k_replay_rank), inverted by
+//      k_replay_inv;
 //   4. k_replay_apply: free slots filled, then pairs replaced while d > n;
 //      the last block advances the pool size and the considered position.
 #include "common.cuh"
+#include "sm100.cuh"
 
 namespace ls {
 namespace {
+using namespace sm100;
 
 constexpr unsigned kFull = 0xffffffffu;
 
@@ -39,30 +41,47 @@ __device__ __forceinline__ void pending_range(const DevState* st, const ReplayGe
   if (lo > hi) lo = hi;
 }
 
-// Ring row of embedding row r (candidates, then kept records), -1 if unused.
-__device__ __forceinline__ int64_t embed_row_slot(int64_t r, const DevState* st, const ReplayGeom& g) {
+// The forward runs over compact rows u: candidates t = u < m, then kept
+// records k = u - m < nR.  Embedding row (the image's and the norms' index):
+// candidate t -> t, kept record k -> P + k.
+__device__ __forceinline__ int64_t compact_slot(int64_t u, const int64_t* counts, const ReplayGeom& g,
+                                                int64_t lo) {
+  const int64_t m = counts[0], nr = counts[1];
+  if (u < m) return g.C + (lo + u) % g.P;
+  return u < m + nr ? g.base + (u - m) : -1;
+}
+
+// The round's counts (candidates, kept records, rows in use per forward
+// chunk of B) and every norm reset to +inf (rows the round does not use).
+__global__ void k_replay_prep(ReplayGeom g, const DevState* st, int B, int nchunks, int64_t* __restrict__ counts,
+                              float* __restrict__ norm, int32_t* __restrict__ rank) {
   int64_t lo, hi;
   pending_range(st, g, lo, hi);
-  if (r < g.P) return lo + r < hi ? g.C + (lo + r) % g.P : -1;
-  const int64_t k = r - g.P;
-  const int64_t nr = *reinterpret_cast<const volatile int64_t*>(&st->replay_count);
-  return k < nr ? g.base + k : -1;
+  const int64_t m = hi - lo, nr = *reinterpret_cast<const volatile int64_t*>(&st->replay_count);
+  if (threadIdx.x == 0) {
+    counts[0] = m;
+    counts[1] = nr;
+    for (int c = 0; c < nchunks; ++c) {
+      const int64_t v = m + nr - (int64_t)c * B;
+      counts[2 + c] = v < 0 ? 0 : (v > B ? B : v);
+    }
+  }
+  for (int64_t r = threadIdx.x; r < g.P + g.Rc; r += blockDim.x) {
+    norm[r] = INFINITY;
+    rank[r] = 0;
+  }
 }
 
 __global__ void k_replay_gather(int B, int64_t row0, int d, ReplayGeom g, const DevState* st,
                                 const float* __restrict__ ring_x, const float* __restrict__ ring_y,
                                 const float* __restrict__ mean, const float* __restrict__ stdv, int bf16,
-                                float* __restrict__ x0, float* __restrict__ y, int64_t* __restrict__ counts) {
-  if (row0 == 0 && blockIdx.x == 0 && threadIdx.x == 0) {  // the round's candidates and kept records
-    int64_t lo, hi;
-    pending_range(st, g, lo, hi);
-    counts[0] = hi - lo;
-    counts[1] = *reinterpret_cast<const volatile int64_t*>(&st->replay_count);
-  }
+                                float* __restrict__ x0, float* __restrict__ y, const int64_t* __restrict__ counts) {
+  int64_t lo, hi;
+  pending_range(st, g, lo, hi);
   const int64_t total = (int64_t)B * d;
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
     const int j = (int)(e / d), k = (int)(e - (int64_t)j * d);
-    const int64_t slot = embed_row_slot(row0 + j, st, g);
+    const int64_t slot = compact_slot(row0 + j, counts, g, lo);
     float v = 0.0f;
     if (slot >= 0) {
       v = zscore(__ldg(ring_x + slot * d + k), __ldg(mean + k), __ldg(stdv + k));
@@ -73,27 +92,41 @@ __global__ void k_replay_gather(int B, int64_t row0, int d, ReplayGeom g, const 
   }
 }
 
-// One warp per row: g = (yhat - y) a_last (fp32), |bf16(g)|^2 summed in a
-// fixed shuffle order; rows not in use get norm +inf (never nearest).
-__global__ void k_replay_embed(int B, int64_t row0, int H, ReplayGeom g, const DevState* st,
+// One warp per compact row: g = (yhat - y) a_last (fp32) and |bf16(g)|^2
+// (summed in a fixed shuffle order) at its embedding row; rows the round does
+// not use keep the +inf norm k_replay_prep gave them (never nearest).  With an
+// image (bf16 distances on tensor cores) the bf16 row also goes to its
+// 128-row tile: candidate tiles first, then kept tiles.
+__global__ void k_replay_embed(int B, int64_t row0, int H, ReplayGeom g, const int64_t* __restrict__ counts,
                                const float* __restrict__ a_last, const float* __restrict__ yhat,
-                               const float* __restrict__ y, float* __restrict__ emb, float* __restrict__ norm) {
+                               const float* __restrict__ y, float* __restrict__ emb, float* __restrict__ norm,
+                               uint8_t* __restrict__ img, int tilesC) {
   const int lane = threadIdx.x & 31;
+  const int64_t m = counts[0], nr = counts[1];
   for (int64_t j = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; j < B;
        j += ((int64_t)gridDim.x * blockDim.x) >> 5) {
-    const int64_t r = row0 + j;
-    const bool used = embed_row_slot(r, st, g) >= 0;
-    const float res = used ? yhat[j] - y[j] : 0.0f;
+    const int64_t u = row0 + j;
+    if (u >= m + nr) break;                 // rows past the round's records (warp-uniform)
+    const int64_t r = u < m ? u : g.P + (u - m);
+    const float res = yhat[j] - y[j];
     float s = 0.0f;
+    uint8_t* trow = nullptr;
+    int rr = 0;
+    if (img) {
+      const int64_t tl = r < g.P ? r / 128 : tilesC + (r - g.P) / 128;
+      rr = (int)(r < g.P ? r % 128 : (r - g.P) % 128);
+      trow = img + tl * (int64_t)128 * H * 2;
+    }
     for (int k = lane; k < H; k += 32) {
       const float v = res * a_last[j * H + k];
       emb[r * H + k] = v;
       const float b = round_bf16(v);
       s = fmaf(b, b, s);
+      if (trow) *reinterpret_cast<__nv_bfloat16*>(trow + sm100::sw128_offset(rr, k, 128)) = __float2bfloat16_rn(v);
     }
 #pragma unroll
     for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(kFull, s, o);
-    if (lane == 0) norm[r] = used ? s : INFINITY;
+    if (lane == 0) norm[r] = s;
   }
 }
 
@@ -131,80 +164,206 @@ __global__ void k_rowmin_reduce(int M, int parts, const float* __restrict__ part
   }
 }
 
-__device__ __forceinline__ float div_key(float v) { return isnan(v) ? -INFINITY : v; }
-
-// Ranks by counting.  Candidate t < m: #{f < m : (d_f, f) before (d_t, t)}
-// with larger d first; kept j < nR: #{q < nR : (n_q, q) before (n_j, j)} with
-// smaller n first.  inv[rank] = t (candidates), inv[P + rank] = j (kept).
-__global__ void __launch_bounds__(256) k_replay_rank(ReplayGeom g, const DevState* st, const float* __restrict__ dc,
-                                                     const float* __restrict__ nk, int32_t* __restrict__ inv) {
-  __shared__ float tile[1024];
-  int64_t lo, hi;
-  pending_range(st, g, lo, hi);
-  const int64_t m = hi - lo;
-  const int64_t nr = *reinterpret_cast<const volatile int64_t*>(&st->replay_count);
-  // blocks [0, cb) rank candidates, the rest rank kept records
-  const int64_t cb = (g.P + blockDim.x - 1) / blockDim.x;
-  const bool cand = blockIdx.x < cb;
-  const int64_t i = (cand ? blockIdx.x : blockIdx.x - cb) * (int64_t)blockDim.x + threadIdx.x;
-  const int64_t cnt = cand ? m : nr;
-  const float* keys = cand ? dc : nk;
-  const float mine = i < cnt ? div_key(keys[i]) : 0.0f;
-  int64_t rank = 0;
-  for (int64_t base = 0; base < cnt; base += 1024) {
-    __syncthreads();
-    for (int q = threadIdx.x; q < 1024; q += blockDim.x)
-      tile[q] = base + q < cnt ? div_key(keys[base + q]) : 0.0f;
-    __syncthreads();
-    const int lim = cnt - base < 1024 ? (int)(cnt - base) : 1024;
-    if (i < cnt)
-      for (int q = 0; q < lim; ++q) {
-        const float o = tile[q];
-        const int64_t f = base + q;
-        rank += cand ? (o > mine || (o == mine && f < i)) : (o < mine || (o == mine && f < i));
-      }
+// Both pools' partial minima (rows [0, P) candidates, [P, P + Rc) kept).
+__global__ void k_rowmin_reduce2(int P, int rows, int parts, const float* __restrict__ part, int64_t ldp,
+                                 float* __restrict__ dc, float* __restrict__ nk) {
+  for (int64_t r = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; r < rows; r += (int64_t)gridDim.x * blockDim.x) {
+    float best = INFINITY;
+    for (int q = 0; q < parts; ++q) best = fminf(best, part[r * ldp + q]);
+    if (r < P) dc[r] = best;
+    else nk[r - P] = best;
   }
-  if (i < cnt) inv[(cand ? 0 : g.P) + rank] = (int32_t)i;
 }
 
-// The same ranks by sorting, one block per pool (block 0 candidates, block 1
-// kept records): 64-bit keys (order code << 32 | index; the candidates' code
-// complemented for the descending order) sorted ascending in shared memory
-// by a bitonic network over n2 (a power of two) keys, padding keys all ones.
-__global__ void __launch_bounds__(1024) k_replay_sort(ReplayGeom g, const DevState* st, const float* __restrict__ dc,
-                                                      const float* __restrict__ nk, int32_t* __restrict__ inv,
-                                                      int n2c, int n2k) {
-  extern __shared__ uint64_t key[];
-  int64_t lo, hi;
-  pending_range(st, g, lo, hi);
-  const bool cand = blockIdx.x == 0;
-  const int64_t cnt = cand ? hi - lo : *reinterpret_cast<const volatile int64_t*>(&st->replay_count);
-  const int n2 = cand ? n2c : n2k;
-  const float* v = cand ? dc : nk;
-  for (int i = threadIdx.x; i < n2; i += blockDim.x) {
-    uint64_t k = ~0ull;
-    if (i < cnt) {
-      const uint32_t code = ord_code(div_key(v[i]));
-      k = ((uint64_t)(cand ? ~code : code) << 32) | (uint32_t)i;
-    }
-    key[i] = k;
+__device__ __forceinline__ float div_key(float v) { return isnan(v) ? -INFINITY : v; }
+
+// ---------------------------------------------------------------------------
+// nearest-neighbour distances on tensor cores from a bf16 embedding image
+// ---------------------------------------------------------------------------
+// The image holds the embeddings as 128-row tiles (candidate tiles, then kept
+// tiles) of H/64 K-major 128-byte-swizzled slabs of 16 KB, so one bulk copy
+// per slab lands a tile in the MMA layout.  CTA (row tile, column split):
+// its 128 rows against a range of kept 128-row column tiles; warp 0 issues
+// the MMAs into two TMEM accumulators, warp 1 bulk-copies the row tile once
+// and the column tiles through two buffers, warps 2..5 (one TMEM lane
+// quadrant each) turn each accumulator into the row minima of
+// |g_r|^2 + |g_c|^2 - 2 g_r.g_c (the row's own kept column skipped).
+constexpr int kDistThreads = 192;
+constexpr int kSlab = 16384;       // 128 rows x 64 bf16
+
+struct DistArgs {
+  const uint8_t* img;
+  const float* norm;               // [P + Rc] (+inf for rows not in use)
+  float* part;                     // [(P + Rc), ldp]
+  int64_t ldp;
+  const int64_t* counts;           // [candidates, kept] of the round
+  int P, Rc, H;
+  int tilesC, tilesK, splits, per_split;  // column tiles per split
+  int* err;
+};
+
+__global__ void __launch_bounds__(kDistThreads, 1) k_dist_rowmin(const __grid_constant__ DistArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int kb = a.H / 64;
+  uint8_t* sA = smem;
+  uint8_t* sB[2] = {smem + kb * kSlab, smem + 2 * kb * kSlab};
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + 3 * kb * kSlab);
+  uint64_t *a_full = bar, *b_full = bar + 1, *b_empty = bar + 3, *acc_full = bar + 5, *acc_empty = bar + 7;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bar + 9);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int tile = blockIdx.x / a.splits, split = blockIdx.x - tile * a.splits;
+  const bool kept_rows = tile >= a.tilesC;
+  const int rtile = kept_rows ? tile - a.tilesC : tile;       // row tile inside its region
+  const int64_t rows_used = kept_rows ? a.counts[1] : a.counts[0];
+  const int64_t ktiles_used = (a.counts[1] + 127) / 128;
+  const int t0 = split * a.per_split;
+  int T = (int)(ktiles_used - t0);
+  T = T < 0 ? 0 : (T > a.per_split ? a.per_split : T);
+  const int base_row = kept_rows ? a.P : 0;                   // first norm / partial row of the region
+  // epilogue thread -> row: warps 2..5 own TMEM lane quadrants warp & 3
+  const int q = warp & 3;
+  const int row = rtile * 128 + 32 * q + lane;                // row inside the region
+  const int region_rows = kept_rows ? a.Rc : a.P;
+  if ((int64_t)rtile * 128 >= rows_used || T == 0) {          // nothing of this CTA is in use
+    if (warp >= 2 && row < region_rows) a.part[(int64_t)(base_row + row) * a.ldp + split] = INFINITY;
+    return;
   }
+  if (tid == 0) {
+    mbar_init(a_full, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(b_full + i, 1);
+      mbar_init(b_empty + i, 1);
+      mbar_init(acc_full + i, 1);
+      mbar_init(acc_empty + i, 4);
+    }
+    fence_mbar_init();
+  }
+  if (warp == 0) {
+    tmem_alloc(tmem_holder, 256);
+    tmem_relinquish();
+  }
+  tc_fence_before();
   __syncthreads();
-  for (int k = 2; k <= n2; k <<= 1)
-    for (int j = k >> 1; j > 0; j >>= 1) {
-      for (int i = threadIdx.x; i < n2; i += blockDim.x) {
-        const int p = i ^ j;
-        if (p > i) {
-          const uint64_t a = key[i], b = key[p];
-          if ((a > b) == ((i & k) == 0)) {
-            key[i] = b;
-            key[p] = a;
-          }
+  tc_fence_after();
+  const uint32_t tmem = *tmem_holder;
+  const uint32_t tile_bytes = (uint32_t)kb * kSlab;
+  const uint8_t* imgA = a.img + (int64_t)tile * tile_bytes;
+  const uint8_t* imgB = a.img + (int64_t)(a.tilesC + t0) * tile_bytes;
+  bool ok = true;
+
+  if (warp == 1) {
+    if (lane == 0) {
+      mbar_arrive_expect_tx(a_full, tile_bytes);
+      for (int k = 0; k < kb; ++k) bulk_g2s(sA + k * kSlab, imgA + k * kSlab, kSlab, a_full);
+      for (int t = 0; t < T && ok; ++t) {
+        const int b = t & 1;
+        if (t >= 2 && !mbar_wait(b_empty + b, (uint32_t)(((t - 2) >> 1) & 1))) ok = false;
+        if (!ok) break;
+        mbar_arrive_expect_tx(b_full + b, tile_bytes);
+        for (int k = 0; k < kb; ++k)
+          bulk_g2s(sB[b] + k * kSlab, imgB + (int64_t)t * tile_bytes + k * kSlab, kSlab, b_full + b);
+      }
+      if (!ok) latch_error(a.err, LS_ERR_TIMEOUT);
+    }
+  } else if (warp == 0) {
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16_f32(128, 128);
+      if (!mbar_wait(a_full, 0)) ok = false;
+      for (int t = 0; t < T && ok; ++t) {
+        const int b = t & 1;
+        if (!mbar_wait(b_full + b, (uint32_t)((t >> 1) & 1))) { ok = false; break; }
+        if (t >= 2 && !mbar_wait(acc_empty + b, (uint32_t)(((t - 2) >> 1) & 1))) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t ab = smem_u32(sA), bb = smem_u32(sB[b]);
+        for (int k = 0; k < kb; ++k)
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            umma_bf16(tmem + (uint32_t)(128 * b), sdesc_sw128(ab + k * kSlab + 32u * j),
+                      sdesc_sw128(bb + k * kSlab + 32u * j), idesc, (k | j) ? 1u : 0u);
+        umma_commit(b_empty + b);
+        umma_commit(acc_full + b);
+      }
+      if (!ok) latch_error(a.err, LS_ERR_TIMEOUT);
+    }
+  } else {
+    const float na = row < region_rows ? __ldg(a.norm + base_row + row) : INFINITY;
+    const int self = kept_rows ? row : -1;                    // the row's own kept column
+    const uint32_t lane_addr = (uint32_t)(32 * q) << 16;
+    float rmin = INFINITY;
+    for (int t = 0; t < T; ++t) {
+      const int b = t & 1;
+      const int col0 = (t0 + t) * 128;
+      if (!mbar_wait(acc_full + b, (uint32_t)((t >> 1) & 1))) {
+        if (lane == 0) latch_error(a.err, LS_ERR_TIMEOUT);
+        break;
+      }
+      tc_fence_after();
+      for (int c = 0; c < 128; c += 32) {
+        float nb[32];
+#pragma unroll
+        for (int u = 0; u < 32; ++u) nb[u] = col0 + c + u < a.Rc ? __ldg(a.norm + a.P + col0 + c + u) : INFINITY;
+        uint32_t v[32];
+        tmem_ld32(tmem + lane_addr + (uint32_t)(128 * b + c), v);
+        tmem_wait_ld();
+#pragma unroll
+        for (int u = 0; u < 32; ++u) {
+          const float dist = na + nb[u] - 2.0f * __uint_as_float(v[u]);
+          if (col0 + c + u != self) rmin = fminf(rmin, dist);
         }
       }
-      __syncthreads();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(acc_empty + b);
     }
-  for (int r = threadIdx.x; r < cnt; r += blockDim.x) inv[(cand ? 0 : g.P) + r] = (int32_t)(key[r] & 0xffffffffu);
+    if (row < region_rows) a.part[(int64_t)(base_row + row) * a.ldp + split] = rmin;
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tmem, 256);
+}
+
+// Ranks by counting, tiled over (element tile, key tile): each block counts,
+// for its 256 elements, the keys of one 1024-key tile that come before them
+// (candidates: larger d first; kept records: smaller n first; equal keys by
+// index) and adds the count to rank[] (integer sums: the order of the
+// additions does not matter).  rank[] was zeroed by k_replay_prep.
+__global__ void __launch_bounds__(256) k_replay_rank(ReplayGeom g, const int64_t* __restrict__ counts,
+                                                     const float* __restrict__ dc, const float* __restrict__ nk,
+                                                     int32_t* __restrict__ rank) {
+  __shared__ float tile[1024];
+  const int64_t cb = (g.P + 255) / 256;               // element tiles of the candidates
+  const bool cand = blockIdx.x < cb;
+  const int64_t i = (cand ? blockIdx.x : blockIdx.x - cb) * 256 + threadIdx.x;
+  const int64_t cnt = cand ? counts[0] : counts[1];
+  const int64_t base = (int64_t)blockIdx.y * 1024;
+  if ((cand ? blockIdx.x : blockIdx.x - cb) * 256 >= cnt || base >= cnt) return;   // block-uniform
+  const float* keys = cand ? dc : nk;
+  for (int q = threadIdx.x; q < 1024; q += 256) tile[q] = base + q < cnt ? div_key(keys[base + q]) : 0.0f;
+  __syncthreads();
+  if (i >= cnt) return;
+  const float mine = div_key(keys[i]);
+  const int lim = cnt - base < 1024 ? (int)(cnt - base) : 1024;
+  int r = 0;
+  for (int q = 0; q < lim; ++q) {
+    const float o = tile[q];
+    const int64_t f = base + q;
+    r += cand ? (o > mine || (o == mine && f < i)) : (o < mine || (o == mine && f < i));
+  }
+  if (r) atomicAdd(rank + (cand ? 0 : g.P) + i, r);
+}
+
+// inv[rank] = element (candidates at [0, P), kept records at [P, P + Rc)).
+__global__ void k_replay_inv(ReplayGeom g, const int64_t* __restrict__ counts, const int32_t* __restrict__ rank,
+                             int32_t* __restrict__ inv) {
+  const int64_t m = counts[0], nr = counts[1];
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < g.P + g.Rc;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const bool cand = e < g.P;
+    const int64_t i = cand ? e : e - g.P;
+    if (i < (cand ? m : nr)) inv[(cand ? 0 : g.P) + rank[e]] = (int32_t)i;
+  }
 }
 
 // One warp per candidate rank t: free slots first, then pairs while d > n.
@@ -238,8 +397,6 @@ __global__ void __launch_bounds__(256) k_replay_apply(int d, ReplayGeom g, DevSt
   }
 }
 
-constexpr int kSortMax = 16384;  // keys a block sorts in shared memory (128 KB)
-
 int grid_for(int64_t threads, int sms) {
   const int64_t b = (threads + 255) / 256;
   return (int)std::max<int64_t>(1, std::min<int64_t>(b, (int64_t)sms * 8));
@@ -254,17 +411,25 @@ cudaError_t run_replay_admit(Ctx& c, float* d_out, float* n_out, cudaStream_t s)
   ReplayGeom g{c.cfg.ring_capacity, c.cfg.pending_capacity, c.cfg.replay_capacity, c.replay_base};
   const int64_t rows = g.P + g.Rc;
   const int Bc = c.cfg.max_train_batch;
+  const int tilesC = (int)((g.P + 127) / 128), tilesK = (int)((g.Rc + 127) / 128);
   cudaError_t e = cudaSuccess;
-  // 1. embeddings, in chunks of the training batch size
+  // 1. embeddings of the round's records (compact rows), in chunks of the training batch size
+  const int nchunks = (int)((rows + Bc - 1) / Bc);
+  e = traced(c, TR_REPLAY, 1, s, [&] {
+    k_replay_prep<<<1, 1024, 0, s>>>(g, c.st, Bc, nchunks, c.rcount, c.rnorm, c.rrank);
+    return cudaGetLastError();
+  });
+  if (e != cudaSuccess) return e;
   for (int64_t row0 = 0; row0 < rows; row0 += Bc) {
     const int B = (int)std::min<int64_t>(Bc, rows - row0);
+    const int64_t* chunk_rows = c.rcount + 2 + row0 / Bc;
     e = traced(c, TR_REPLAY, 1, s, [&] {
       k_replay_gather<<<grid_for((int64_t)B * m.w[0], c.sms), 256, 0, s>>>(
           B, row0, m.w[0], g, c.st, c.ring_x, c.ring_y, c.mean, c.stdv, m.bf16, c.tx, c.ty, c.rcount);
       return cudaGetLastError();
     });
     if (e != cudaSuccess) return e;
-    e = forward_rows(c, B, s);
+    e = forward_rows(c, B, s, chunk_rows);
     if (e != cudaSuccess) return e;
     int64_t xoff = 0, zoff = 0;
     for (int l = 0; l < L - 1; ++l) {
@@ -272,13 +437,44 @@ cudaError_t run_replay_admit(Ctx& c, float* d_out, float* n_out, cudaStream_t s)
       zoff += (int64_t)B * m.w[l + 1];
     }
     e = traced(c, TR_REPLAY, 1, s, [&] {
-      k_replay_embed<<<grid_for((int64_t)B * 32, c.sms), 256, 0, s>>>(B, row0, H, g, c.st, c.tx + xoff, c.tz + zoff,
-                                                                        c.ty, c.remb, c.rnorm);
+      k_replay_embed<<<grid_for((int64_t)B * 32, c.sms), 256, 0, s>>>(B, row0, H, g, c.rcount, c.tx + xoff,
+                                                                        c.tz + zoff, c.ty, c.remb, c.rnorm, c.rimg,
+                                                                        tilesC);
       return cudaGetLastError();
     });
     if (e != cudaSuccess) return e;
   }
   // 2. nearest kept embedding of every candidate, nearest other kept of every kept record
+  if (c.rimg) {  // bf16 image: one launch for both, then one reduction
+    DistArgs da{};
+    da.img = c.rimg;
+    da.norm = c.rnorm;
+    da.part = c.rpart;
+    da.ldp = kRowMinParts;
+    da.counts = c.rcount;
+    da.P = (int)g.P;
+    da.Rc = (int)g.Rc;
+    da.H = H;
+    da.tilesC = tilesC;
+    da.tilesK = tilesK;
+    da.splits = std::max(1, std::min(std::min(tilesK, kRowMinParts), 2 * c.sms / (tilesC + tilesK)));
+    da.per_split = (tilesK + da.splits - 1) / da.splits;
+    da.err = c.d_err;
+    const int smem = 1024 + 3 * (H / 64) * kSlab + 128;
+    e = traced(c, TR_REPLAY, 1, s, [&] {
+      cudaError_t a = cudaFuncSetAttribute(k_dist_rowmin, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+      if (a != cudaSuccess) return a;
+      k_dist_rowmin<<<(tilesC + tilesK) * da.splits, kDistThreads, smem, s>>>(da);
+      return cudaGetLastError();
+    });
+    if (e != cudaSuccess) return e;
+    e = traced(c, TR_REPLAY, 1, s, [&] {
+      k_rowmin_reduce2<<<grid_for(rows, c.sms), 256, 0, s>>>((int)g.P, (int)rows, da.splits, c.rpart, kRowMinParts,
+                                                             c.rd, c.rn);
+      return cudaGetLastError();
+    });
+    if (e != cudaSuccess) return e;
+  }
   const float* Ec = c.remb;
   const float* Ek = c.remb + g.P * H;
   const float* nc = c.rnorm;
@@ -304,10 +500,12 @@ cudaError_t run_replay_admit(Ctx& c, float* d_out, float* n_out, cudaStream_t s)
       return cudaGetLastError();
     });
   };
-  e = rowmin((int)g.P, Ec, nc, kNoSelf, c.rcount, c.rd);
-  if (e != cudaSuccess) return e;
-  e = rowmin((int)g.Rc, Ek, nkp, 0, c.rcount + 1, c.rn);
-  if (e != cudaSuccess) return e;
+  if (!c.rimg) {
+    e = rowmin((int)g.P, Ec, nc, kNoSelf, c.rcount, c.rd);
+    if (e != cudaSuccess) return e;
+    e = rowmin((int)g.Rc, Ek, nkp, 0, c.rcount + 1, c.rn);
+    if (e != cudaSuccess) return e;
+  }
   if (d_out) {
     e = cudaMemcpyAsync(d_out, c.rd, (size_t)g.P * sizeof(float), cudaMemcpyDeviceToDevice, s);
     if (e != cudaSuccess) return e;
@@ -318,19 +516,14 @@ cudaError_t run_replay_admit(Ctx& c, float* d_out, float* n_out, cudaStream_t s)
   }
   // 3. ranks, 4. admission
   e = traced(c, TR_REPLAY, 1, s, [&] {
-    int n2c = 1, n2k = 1;
-    while (n2c < g.P) n2c <<= 1;
-    while (n2k < g.Rc) n2k <<= 1;
-    const int n2 = std::max(n2c, n2k);
-    if (n2 <= kSortMax) {
-      const int smem = n2 * (int)sizeof(uint64_t);
-      cudaError_t a = cudaFuncSetAttribute(k_replay_sort, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-      if (a != cudaSuccess) return a;
-      k_replay_sort<<<2, 1024, smem, s>>>(g, c.st, c.rd, c.rn, c.rinv, n2c, n2k);
-    } else {
-      const int blocks = (int)((g.P + 255) / 256 + (g.Rc + 255) / 256);
-      k_replay_rank<<<blocks, 256, 0, s>>>(g, c.st, c.rd, c.rn, c.rinv);
-    }
+    const dim3 grid((unsigned)((g.P + 255) / 256 + (g.Rc + 255) / 256),
+                    (unsigned)((std::max(g.P, g.Rc) + 1023) / 1024));
+    k_replay_rank<<<grid, 256, 0, s>>>(g, c.rcount, c.rd, c.rn, c.rrank);
+    return cudaGetLastError();
+  });
+  if (e != cudaSuccess) return e;
+  e = traced(c, TR_REPLAY, 1, s, [&] {
+    k_replay_inv<<<grid_for(g.P + g.Rc, c.sms), 256, 0, s>>>(g, c.rcount, c.rrank, c.rinv);
     return cudaGetLastError();
   });
   if (e != cudaSuccess) return e;

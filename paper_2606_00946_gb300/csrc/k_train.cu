@@ -304,7 +304,7 @@ int train_splits(int out, int in, int B, int n_sm) {
 // Forward of B rows whose layer-0 inputs are in c.tx (z-scored, rounded in
 // bf16 mode): z_l into c.tz, hidden activations a_l into c.tx (the training
 // step's layout: layer l's input at c.tx + B * sum_{k<l} w_k).
-cudaError_t forward_rows(Ctx& c, int B, cudaStream_t s) {
+cudaError_t forward_rows(Ctx& c, int B, cudaStream_t s, const int64_t* rows_dev) {
   const MlpDesc& m = c.mlp;
   const int L = m.n_layers;
   int64_t xoff[LS_MAX_LAYERS + 1], zoff[LS_MAX_LAYERS + 1];
@@ -340,7 +340,7 @@ cudaError_t forward_rows(Ctx& c, int B, cudaStream_t s) {
     } else if (m.bf16) {
       e = traced(c, TR_GEMM_TC_FWD, 1, s, [&] {
         return launch_gemm_tc(a.M, a.N, a.K, a.A, a.lda, 1, a.B, a.ldb, 1, 1, 1, a.C, a.ldc, 0, a.bias, a.act,
-                              a.ld_act, a.hidden, nullptr, 0, c.d_err, c.sms, s);
+                              a.ld_act, a.hidden, nullptr, 0, c.d_err, c.sms, s, rows_dev);
       });
       if (e == cudaSuccess) done_tc = true;
       else if (e != cudaErrorInvalidValue) return e;

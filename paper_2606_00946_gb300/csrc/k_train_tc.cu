@@ -146,10 +146,10 @@ __global__ void __launch_bounds__(kT) k_gemm_tc(const __grid_constant__ TcGemmAr
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int m0 = blockIdx.y * kM, n0 = blockIdx.x * g.ntile;
-  if (g.epi == 3 && ((g.rows_dev && m0 >= *g.rows_dev) || (g.cols_dev && n0 >= *g.cols_dev))) {
-    // nothing of this tile is in use: its partial minima are +inf
+  if ((g.rows_dev && m0 >= *g.rows_dev) || (g.epi == 3 && g.cols_dev && n0 >= *g.cols_dev)) {
+    // nothing of this tile is in use (row-minimum partials: +inf)
     const int r = m0 + 32 * (warp & 3) + lane;
-    if (r < g.M) g.C[(int64_t)r * g.ldc + 2 * blockIdx.x + (warp >> 2)] = INFINITY;
+    if (g.epi == 3 && r < g.M) g.C[(int64_t)r * g.ldc + 2 * blockIdx.x + (warp >> 2)] = INFINITY;
     return;
   }
   const int64_t kbeg = (int64_t)blockIdx.z * g.kper;
@@ -310,7 +310,8 @@ cudaError_t run_tc(dim3 grid, int smem, const TcGemmArgs& g, cudaStream_t s) {
 cudaError_t launch_gemm_tc(int M, int N, int K, const float* A, int64_t sam, int64_t sak, const float* B,
                            int64_t sbn, int64_t sbk, int splits, int epi, float* C, int64_t ldc,
                            int64_t split_stride, const float* bias, float* act, int64_t ld_act, int hidden,
-                           const float* zprev, int64_t ld_zprev, int* err, int sms, cudaStream_t s) {
+                           const float* zprev, int64_t ld_zprev, int* err, int sms, cudaStream_t s,
+                           const int64_t* rows_dev) {
   if (M < 64 || N < 32 || K < 1) return cudaErrorInvalidValue;
   const int mt = (M + kM - 1) / kM;
   int ntile = 256;
@@ -326,6 +327,7 @@ cudaError_t launch_gemm_tc(int M, int N, int K, const float* A, int64_t sam, int
   g.C = C; g.ldc = ldc; g.split_stride = split_stride;
   g.bias = bias; g.act = act; g.ld_act = ld_act; g.hidden = hidden;
   g.zprev = zprev; g.ld_zprev = ld_zprev;
+  g.rows_dev = rows_dev;
   g.err = err;
   g.tmem_cols = 32;
   while ((int)g.tmem_cols < ntile) g.tmem_cols <<= 1;
