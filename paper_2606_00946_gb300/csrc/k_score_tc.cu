@@ -327,6 +327,18 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc(const __grid_constan
 }
 
 // ---------------------------------------------------------------------------
+// Output-layer partial of 16 columns: the fp32 pair accumulator gains
+// bf16(relu(z_c)) * w_c for the even and odd columns (w_c bf16, 8 per uint4).
+__device__ __forceinline__ uint64_t out_dot16(const uint32_t (&v)[16], uint4 w0, uint4 w1, uint64_t acc) {
+  const uint32_t wp[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const uint32_t h = relu_bf16x2(cvt_bf16x2(((uint64_t)v[2 * j + 1] << 32) | v[2 * j]));
+    acc = fma_f32x2(bf16x2_to_f32x2(h), bf16x2_to_f32x2(wp[j]), acc);
+  }
+  return acc;
+}
+
 // Pipelined variant for predictors with two hidden layers whose weights stay
 // resident (widths <= 256): warp 0 issues the MMAs, warps 1-7 build feature
 // tiles into two buffers ahead of time, warps 8-15 run the epilogues.  Layer-1
@@ -360,10 +372,14 @@ __global__ void __launch_bounds__(kThreadsPipe, 1) k_score_tc_pipe(const __grid_
   uint8_t* W = smem;                                            // resident weight chunks
   uint8_t* X = W + (size_t)p.chunks * p.chunk_bytes;            // [kXB] feature tiles
   uint8_t* AR = X + kXB * (size_t)xbytes;                       // [2] activation K-blocks (16 KB)
-  float* part = reinterpret_cast<float*>(AR + 2 * kTileM * 128);  // [2][128]
+  // layer-2 bias as one K = 16 product, D2 = ONE B2^T before the K-blocks:
+  // ONE [128 x 16] has ones in columns 0..2, B2 [256 x 16] holds the three
+  // bf16 terms hi + mid + lo of each fp32 b2 (their sum is b2 exactly)
+  uint8_t* ONE = AR + 2 * kTileM * 128;                         // 4 KB, no swizzle
+  uint8_t* B2 = ONE + kTileM * 32;                              // 8 KB, no swizzle
+  float* part = reinterpret_cast<float*>(B2 + 256 * 32);        // [2][128]
   float* sb1 = part + 2 * kTileM;                               // [256] layer-1 bias
-  float* sb2 = sb1 + 256;                                       // [256] layer-2 bias
-  float* sw3 = sb2 + 256;                                       // [256] output-layer weights
+  uint16_t* sw3 = reinterpret_cast<uint16_t*>(sb1 + 256);       // [256] bf16 output-layer weights
   uint64_t* bars = reinterpret_cast<uint64_t*>(sw3 + 256);
   uint64_t* x_full = bars;       // [2]
   uint64_t* x_empty = bars + 2;  // [2]
@@ -398,10 +414,29 @@ __global__ void __launch_bounds__(kThreadsPipe, 1) k_score_tc_pipe(const __grid_
     tmem_relinquish();
   }
   for (int k = tid; k < H1; k += blockDim.x) sb1[k] = __ldg(params + a.boff[0] + k);
-  for (int k = tid; k < H2; k += blockDim.x) {
-    sb2[k] = __ldg(params + a.boff[1] + k);
-    sw3[k] = __ldg(params + a.w_last_off + k);
+  for (int k = tid; k < H2; k += blockDim.x) sw3[k] = bf16_bits(__ldg(params + a.w_last_off + k));
+  for (int e = tid; e < kTileM * 2; e += blockDim.x) {  // 16-byte chunks: row e / 2, K half e % 2
+    const uint4 q = (e & 1) ? make_uint4(0u, 0u, 0u, 0u) : make_uint4(0x3F803F80u, 0x3F80u, 0u, 0u);
+    *reinterpret_cast<uint4*>(ONE + nosw16_offset(e >> 1, 8 * (e & 1))) = q;
   }
+  for (int e = tid; e < 256 * 2; e += blockDim.x) {
+    const int n = e >> 1;
+    uint4 q = make_uint4(0u, 0u, 0u, 0u);
+    if (!(e & 1) && n < H2) {
+      const float b = __ldg(params + a.boff[1] + n);
+      const uint16_t hi = bf16_bits(b);
+      uint16_t mid = 0, lo = 0;
+      if (!isinf(b)) {  // b - hi and (b - hi) - mid are exact in fp32; lo holds the last 8 bits
+        const float r1 = b - __uint_as_float((uint32_t)hi << 16);
+        mid = bf16_bits(r1);
+        lo = bf16_bits(r1 - __uint_as_float((uint32_t)mid << 16));
+      }
+      q.x = (uint32_t)hi | ((uint32_t)mid << 16);
+      q.y = lo;
+    }
+    *reinterpret_cast<uint4*>(B2 + nosw16_offset(n, 8 * (e & 1))) = q;
+  }
+  fence_async_smem();  // the bias operands are read by the tensor cores (async proxy)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -433,18 +468,20 @@ __global__ void __launch_bounds__(kThreadsPipe, 1) k_score_tc_pipe(const __grid_
                       sdesc_sw128(smem_u32(W + (size_t)kb * p.chunk_bytes) + 32u * j), id1, (kb | j) ? 1u : 0u);
         umma_commit(&x_empty[xb]);
         umma_commit(d1_full);
+        if (t >= 1 && !mbar_wait(d2_empty, (uint32_t)((t - 1) & 1))) { ok = false; break; }
+        tc_fence_after();
+        umma_bf16(D2, sdesc_nosw(smem_u32(ONE), 128, 256), sdesc_nosw(smem_u32(B2), 128, 256), id2, 0u);
         for (int kb = 0; kb < nk1 && ok; ++kb) {
           const int64_t kq = (int64_t)t * nk1 + kb;
           const int slot = (int)(kq & 1);
           ok = mbar_wait(&a_full[slot], (uint32_t)((kq >> 1) & 1));
-          if (ok && kb == 0 && t >= 1) ok = mbar_wait(d2_empty, (uint32_t)((t - 1) & 1));
           if (!ok) break;
           tc_fence_after();
           const uint32_t aa = smem_u32(AR + (size_t)slot * kTileM * 128);
           const uint32_t bb = smem_u32(W + (size_t)(nk0 + kb) * p.chunk_bytes);
 #pragma unroll
           for (int j = 0; j < 4; ++j)
-            umma_bf16(D2, sdesc_sw128(aa + 32u * j), sdesc_sw128(bb + 32u * j), id2, (kb | j) ? 1u : 0u);
+            umma_bf16(D2, sdesc_sw128(aa + 32u * j), sdesc_sw128(bb + 32u * j), id2, 1u);
           umma_commit(&a_empty[slot]);
         }
         umma_commit(d2_full);
@@ -541,25 +578,24 @@ __global__ void __launch_bounds__(kThreadsPipe, 1) k_score_tc_pipe(const __grid_
       const bool ok2 = mbar_wait(d2_full, (uint32_t)(t & 1));
       tc_fence_after();
       uint64_t acc2 = 0;
-      for (int c0 = wk * half; ok2 && c0 < (wk + 1) * half; c0 += 16) {
-        float4 bq[4], wq[4];  // shared memory, in flight during the TMEM load
-#pragma unroll
-        for (int j4 = 0; j4 < 4; ++j4) {
-          bq[j4] = *reinterpret_cast<const float4*>(sb2 + c0 + 4 * j4);
-          wq[j4] = *reinterpret_cast<const float4*>(sw3 + c0 + 4 * j4);
-        }
-        uint32_t v[16];
-        tmem_ld16(D2 + lane_addr + (uint32_t)c0, v);
-        tmem_wait_ld();
-#pragma unroll
-        for (int j4 = 0; j4 < 4; ++j4) {
-          const float4 b = bq[j4], w = wq[j4];
-          const uint32_t h0 =
-              relu_bf16x2(cvt_bf16x2(add_f32x2(((uint64_t)v[4 * j4 + 1] << 32) | v[4 * j4], f2pack(b.x, b.y))));
-          const uint32_t h1 =
-              relu_bf16x2(cvt_bf16x2(add_f32x2(((uint64_t)v[4 * j4 + 3] << 32) | v[4 * j4 + 2], f2pack(b.z, b.w))));
-          acc2 = fma_f32x2(bf16x2_to_f32x2(h0), f2pack(w.x, w.y), acc2);
-          acc2 = fma_f32x2(bf16x2_to_f32x2(h1), f2pack(w.z, w.w), acc2);
+      if (ok2) {
+        // D2 already holds z + b2: two 16-column loads in flight, one consumed
+        // while the next lands
+        const uint32_t base = D2 + lane_addr;
+        const int cb = wk * half, ce = cb + half;  // half is a multiple of 32
+        uint32_t va[16], vb[16];
+        tmem_ld16(base + (uint32_t)cb, va);
+        for (int c0 = cb; c0 < ce; c0 += 32) {
+          uint4 w0 = *reinterpret_cast<const uint4*>(sw3 + c0);
+          uint4 w1 = *reinterpret_cast<const uint4*>(sw3 + c0 + 8);
+          tmem_wait_ld_regs(va);
+          tmem_ld16(base + (uint32_t)(c0 + 16), vb);
+          acc2 = out_dot16(va, w0, w1, acc2);
+          w0 = *reinterpret_cast<const uint4*>(sw3 + c0 + 16);
+          w1 = *reinterpret_cast<const uint4*>(sw3 + c0 + 24);
+          tmem_wait_ld_regs(vb);
+          if (c0 + 32 < ce) tmem_ld16(base + (uint32_t)(c0 + 32), va);
+          acc2 = out_dot16(vb, w0, w1, acc2);
         }
       }
       tc_fence_before();
@@ -791,7 +827,7 @@ bool plan_tc(const MlpDesc& m, TcPlan& p) {
   p.pipe = 0;
   if (p.n_tc == 2 && p.out[0] <= 256 && p.out[1] <= 256 && p.nc[0] == p.out[0] && p.nc[1] == p.out[1]) {
     const int64_t need = 1024 + (int64_t)p.chunks * cb + kXB * (int64_t)p.d_pad * kTileM * 2 + 2 * kTileM * 128 +
-                         2 * kTileM * 4 + 3 * 256 * 4 + 13 * 8 + 16;
+                         kTileM * 32 + 256 * 32 + 2 * kTileM * 4 + 256 * 4 + 256 * 2 + 13 * 8 + 16;
     if (need <= kMaxSmem) {
       p.pipe = 1;
       p.pipe_smem = (int)need;

@@ -207,6 +207,17 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
 __device__ __forceinline__ void tmem_wait_ld() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
+// The same wait, with the 16 destination registers of the load it completes
+// as operands, so that no use of them can be scheduled above the wait (needed
+// when another load is in flight while earlier registers are consumed).
+__device__ __forceinline__ void tmem_wait_ld_regs(uint32_t (&r)[16]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
+                 "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]),
+                 "+r"(r[15])
+               :
+               : "memory");
+}
 
 // ---------------------------------------------------------------------------
 // UMMA (tcgen05.mma, kind::f16: bf16 x bf16 -> fp32 in TMEM)
@@ -231,6 +242,24 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
   d |= (uint64_t)1 << 46;            // version
   d |= (uint64_t)2 << 61;            // SWIZZLE_128B
   return d;
+}
+
+// Shared-memory descriptor of a K-major operand without swizzle: 8-row x
+// 16-byte core matrices of 128 contiguous bytes; `lbo` = byte distance between
+// core matrices adjacent along K, `sbo` = between 8-row groups along M/N.
+__device__ __forceinline__ uint64_t sdesc_nosw(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+  d |= (uint64_t)1 << 46;  // version; layout type 0 (no swizzle)
+  return d;
+}
+
+// Byte offset of element (row, k), k < 16, in such an operand with lbo = 128,
+// sbo = 256: row group (row / 8) holds its two K core matrices side by side.
+__host__ __device__ __forceinline__ uint32_t nosw16_offset(int row, int k) {
+  return (uint32_t)(row >> 3) * 256u + (uint32_t)(k >> 3) * 128u + (uint32_t)(row & 7) * 16u + (uint32_t)(k & 7) * 2u;
 }
 
 __device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
