@@ -372,14 +372,15 @@ __global__ void __launch_bounds__(kThreadsPipe, 1) k_score_tc_pipe(const __grid_
   uint8_t* W = smem;                                            // resident weight chunks
   uint8_t* X = W + (size_t)p.chunks * p.chunk_bytes;            // [kXB] feature tiles
   uint8_t* AR = X + kXB * (size_t)xbytes;                       // [2] activation K-blocks (16 KB)
-  // layer-2 bias as one K = 16 product, D2 = ONE B2^T before the K-blocks:
-  // ONE [128 x 16] has ones in columns 0..2, B2 [256 x 16] holds the three
-  // bf16 terms hi + mid + lo of each fp32 b2 (their sum is b2 exactly)
-  uint8_t* ONE = AR + 2 * kTileM * 128;                         // 4 KB, no swizzle
-  uint8_t* B2 = ONE + kTileM * 32;                              // 8 KB, no swizzle
+  // biases as one K = 16 product per layer, D = ONE Bl^T ahead of the K-blocks:
+  // ONE [128 x 16] has ones in columns 0..2 (all row groups read the same 8
+  // rows: stride 0), Bl [256 x 16] holds the three bf16 terms hi + mid + lo
+  // of each fp32 bias (their sum is the bias exactly)
+  uint8_t* ONE = AR + 2 * kTileM * 128;                         // 256 B, no swizzle
+  uint8_t* B1 = ONE + 8 * 32;                                   // 8 KB, no swizzle
+  uint8_t* B2 = B1 + 256 * 32;                                  // 8 KB, no swizzle
   float* part = reinterpret_cast<float*>(B2 + 256 * 32);        // [2][128]
-  float* sb1 = part + 2 * kTileM;                               // [256] layer-1 bias
-  uint16_t* sw3 = reinterpret_cast<uint16_t*>(sb1 + 256);       // [256] bf16 output-layer weights
+  uint16_t* sw3 = reinterpret_cast<uint16_t*>(part + 2 * kTileM);  // [256] bf16 output-layer weights
   uint64_t* bars = reinterpret_cast<uint64_t*>(sw3 + 256);
   uint64_t* x_full = bars;       // [2]
   uint64_t* x_empty = bars + 2;  // [2]
@@ -413,17 +414,16 @@ __global__ void __launch_bounds__(kThreadsPipe, 1) k_score_tc_pipe(const __grid_
     tmem_alloc(tmem_holder, 512);
     tmem_relinquish();
   }
-  for (int k = tid; k < H1; k += blockDim.x) sb1[k] = __ldg(params + a.boff[0] + k);
   for (int k = tid; k < H2; k += blockDim.x) sw3[k] = bf16_bits(__ldg(params + a.w_last_off + k));
-  for (int e = tid; e < kTileM * 2; e += blockDim.x) {  // 16-byte chunks: row e / 2, K half e % 2
+  for (int e = tid; e < 8 * 2; e += blockDim.x) {  // 16-byte chunks: row e / 2, K half e % 2
     const uint4 q = (e & 1) ? make_uint4(0u, 0u, 0u, 0u) : make_uint4(0x3F803F80u, 0x3F80u, 0u, 0u);
     *reinterpret_cast<uint4*>(ONE + nosw16_offset(e >> 1, 8 * (e & 1))) = q;
   }
-  for (int e = tid; e < 256 * 2; e += blockDim.x) {
-    const int n = e >> 1;
+  for (int e = tid; e < 2 * 256 * 2; e += blockDim.x) {  // layer (e / 512), row n, K half
+    const int l = e >> 9, n = (e >> 1) & 255;
     uint4 q = make_uint4(0u, 0u, 0u, 0u);
-    if (!(e & 1) && n < H2) {
-      const float b = __ldg(params + a.boff[1] + n);
+    if (!(e & 1) && n < (l ? H2 : H1)) {
+      const float b = __ldg(params + a.boff[l] + n);
       const uint16_t hi = bf16_bits(b);
       uint16_t mid = 0, lo = 0;
       if (!isinf(b)) {  // b - hi and (b - hi) - mid are exact in fp32; lo holds the last 8 bits
@@ -434,7 +434,7 @@ __global__ void __launch_bounds__(kThreadsPipe, 1) k_score_tc_pipe(const __grid_
       q.x = (uint32_t)hi | ((uint32_t)mid << 16);
       q.y = lo;
     }
-    *reinterpret_cast<uint4*>(B2 + nosw16_offset(n, 8 * (e & 1))) = q;
+    *reinterpret_cast<uint4*>((l ? B2 : B1) + nosw16_offset(n, 8 * (e & 1))) = q;
   }
   fence_async_smem();  // the bias operands are read by the tensor cores (async proxy)
   tc_fence_before();
@@ -461,16 +461,17 @@ __global__ void __launch_bounds__(kThreadsPipe, 1) k_score_tc_pipe(const __grid_
         if (!ok) break;
         tc_fence_after();
         const uint32_t xa = smem_u32(X + (size_t)xb * xbytes);
+        umma_bf16(D1, sdesc_nosw(smem_u32(ONE), 128, 0), sdesc_nosw(smem_u32(B1), 128, 256), id1, 0u);
         for (int kb = 0; kb < nk0; ++kb)
 #pragma unroll
           for (int j = 0; j < 4; ++j)
             umma_bf16(D1, sdesc_sw128(xa + (uint32_t)kb * kTileM * 128u + 32u * j),
-                      sdesc_sw128(smem_u32(W + (size_t)kb * p.chunk_bytes) + 32u * j), id1, (kb | j) ? 1u : 0u);
+                      sdesc_sw128(smem_u32(W + (size_t)kb * p.chunk_bytes) + 32u * j), id1, 1u);
         umma_commit(&x_empty[xb]);
         umma_commit(d1_full);
         if (t >= 1 && !mbar_wait(d2_empty, (uint32_t)((t - 1) & 1))) { ok = false; break; }
         tc_fence_after();
-        umma_bf16(D2, sdesc_nosw(smem_u32(ONE), 128, 256), sdesc_nosw(smem_u32(B2), 128, 256), id2, 0u);
+        umma_bf16(D2, sdesc_nosw(smem_u32(ONE), 128, 0), sdesc_nosw(smem_u32(B2), 128, 256), id2, 0u);
         for (int kb = 0; kb < nk1 && ok; ++kb) {
           const int64_t kq = (int64_t)t * nk1 + kb;
           const int slot = (int)(kq & 1);
@@ -530,10 +531,7 @@ __global__ void __launch_bounds__(kThreadsPipe, 1) k_score_tc_pipe(const __grid_
         const int64_t kq = (int64_t)t * nk1 + kb;
         const int slot = (int)(kq & 1);
         const int colb = 64 * kb + 32 * wk;
-        float4 bq[8];  // bias of the 32 columns (shared memory), in flight during the TMEM load
-#pragma unroll
-        for (int j4 = 0; j4 < 8; ++j4) bq[j4] = *reinterpret_cast<const float4*>(sb1 + colb + 4 * j4);
-        uint32_t v[2][16];
+        uint32_t v[2][16];  // D1 already holds z + b1
         tmem_ld16(D1 + lane_addr + (uint32_t)colb, v[0]);
         tmem_ld16(D1 + lane_addr + (uint32_t)(colb + 16), v[1]);
         tmem_wait_ld();
@@ -543,13 +541,8 @@ __global__ void __launch_bounds__(kThreadsPipe, 1) k_score_tc_pipe(const __grid_
         for (int g = 0; g < 2; ++g) {
           uint32_t pk[8];
 #pragma unroll
-          for (int j4 = 0; j4 < 4; ++j4) {
-            const float4 b = bq[4 * g + j4];
-            const uint64_t z0 = add_f32x2(((uint64_t)v[g][4 * j4 + 1] << 32) | v[g][4 * j4], f2pack(b.x, b.y));
-            const uint64_t z1 = add_f32x2(((uint64_t)v[g][4 * j4 + 3] << 32) | v[g][4 * j4 + 2], f2pack(b.z, b.w));
-            pk[2 * j4] = relu_bf16x2(cvt_bf16x2(z0));
-            pk[2 * j4 + 1] = relu_bf16x2(cvt_bf16x2(z1));
-          }
+          for (int j = 0; j < 8; ++j)
+            pk[j] = relu_bf16x2(cvt_bf16x2(((uint64_t)v[g][2 * j + 1] << 32) | v[g][2 * j]));
           const int kcol = 32 * wk + 16 * g;  // column inside the K-block
           st_shared_v4(dst + sw128_offset(row, kcol, kTileM), pk[0], pk[1], pk[2], pk[3]);
           st_shared_v4(dst + sw128_offset(row, kcol + 8, kTileM), pk[4], pk[5], pk[6], pk[7]);
@@ -827,7 +820,7 @@ bool plan_tc(const MlpDesc& m, TcPlan& p) {
   p.pipe = 0;
   if (p.n_tc == 2 && p.out[0] <= 256 && p.out[1] <= 256 && p.nc[0] == p.out[0] && p.nc[1] == p.out[1]) {
     const int64_t need = 1024 + (int64_t)p.chunks * cb + kXB * (int64_t)p.d_pad * kTileM * 2 + 2 * kTileM * 128 +
-                         kTileM * 32 + 256 * 32 + 2 * kTileM * 4 + 256 * 4 + 256 * 2 + 13 * 8 + 16;
+                         8 * 32 + 2 * 256 * 32 + 2 * kTileM * 4 + 256 * 2 + 13 * 8 + 16;
     if (need <= kMaxSmem) {
       p.pipe = 1;
       p.pipe_smem = (int)need;
