@@ -357,6 +357,9 @@ constexpr int kThreadsPipe = (kE2Warp0 + kEpiWarps) * 32;  // 576
 // Feature tiles in flight.  One suffices: the copy of tile t+1 starts when the
 // layer-1 MMA of tile t completes and has the rest of tile t to land.
 constexpr int kXB = 1;
+// Barriers for the resident weight chunks (the last one takes every chunk past it).
+constexpr int kWBars = 8;
+__device__ __forceinline__ int wbar_of(int q) { return q < kWBars - 1 ? q : kWBars - 1; }
 
 __global__ void __launch_bounds__(kThreadsPipe, 1) k_score_tc_pipe(const __grid_constant__ TcArgs a) {
   const bool pb = a.sel && *a.sel == 1;  // published buffer of this route
@@ -390,11 +393,12 @@ __global__ void __launch_bounds__(kThreadsPipe, 1) k_score_tc_pipe(const __grid_
   uint64_t* d1_empty = bars + 9;
   uint64_t* d2_full = bars + 10;
   uint64_t* d2_empty = bars + 11;
-  uint64_t* w_full = bars + 12;
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 13);
+  uint64_t* w_full = bars + 12;  // [kWBars]: weight chunk q lands on barrier min(q, kWBars - 1)
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 12 + kWBars);
   int* abort_flag = reinterpret_cast<int*>(tmem_holder + 1);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int my_tiles = blockIdx.x < a.n_tiles ? (a.n_tiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
   if (tid == 0) {
     for (int b = 0; b < 2; ++b) {
       mbar_init(&x_full[b], 1);  // only the first kXB are used
@@ -406,9 +410,27 @@ __global__ void __launch_bounds__(kThreadsPipe, 1) k_score_tc_pipe(const __grid_
     mbar_init(d1_empty, kEpiWarps);
     mbar_init(d2_full, 1);
     mbar_init(d2_empty, kEpiWarps);
-    mbar_init(w_full, 1);
+    for (int b = 0; b < kWBars; ++b) mbar_init(&w_full[b], 1);
     *abort_flag = 0;
     fence_mbar_init();
+    if (my_tiles > 0) {
+      // the weight chunks (in the order the first tile uses them, each K-block
+      // of tile 0 waiting only for its own chunk) and the first feature tile
+      // are requested before anything else, so they land during the prologue
+      // first tile's features, then the weight image: the K-blocks of layer 1
+      // (H1 x 128 B each) followed by those of layer 2 (H2 x 128 B each), one
+      // resident chunk each (offsets from the widths, not from indexed tables)
+      mbar_arrive_expect_tx(&x_full[0], (uint32_t)xbytes);
+      bulk_g2s(X, a.ximg + (int64_t)blockIdx.x * xbytes, (uint32_t)xbytes, &x_full[0]);
+      const int64_t l1_bytes = (int64_t)nk0 * H1 * 128;
+      for (int q = 0; q < nk0 + nk1; ++q) {
+        const uint32_t len = (uint32_t)(q < nk0 ? H1 : H2) * 128u;
+        const int64_t off = q < nk0 ? (int64_t)q * H1 * 128 : l1_bytes + (int64_t)(q - nk0) * H2 * 128;
+        mbar_expect_tx(&w_full[wbar_of(q)], len);
+        bulk_g2s(W + (size_t)q * p.chunk_bytes, img + off, len, &w_full[wbar_of(q)]);
+      }
+      for (int b = 0; b < kWBars; ++b) mbar_arrive(&w_full[b]);  // a barrier without chunks completes here
+    }
   }
   if (warp == 0) {
     tmem_alloc(tmem_holder, 512);
@@ -442,22 +464,18 @@ __global__ void __launch_bounds__(kThreadsPipe, 1) k_score_tc_pipe(const __grid_
   tc_fence_after();
   const uint32_t tmem = *tmem_holder;
   const uint32_t D1 = tmem, D2 = tmem + 256;
-  const int my_tiles = blockIdx.x < a.n_tiles ? (a.n_tiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
 
   if (warp == 0) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0 && my_tiles > 0) {
-      int64_t wbytes = 0;
-      for (int q = 0; q < p.chunks; ++q) wbytes += p.chunk_len[q];
-      mbar_arrive_expect_tx(w_full, (uint32_t)wbytes);
-      for (int q = 0; q < p.chunks; ++q)
-        bulk_g2s(W + (size_t)q * p.chunk_bytes, img + p.chunk_off[q], (uint32_t)p.chunk_len[q], w_full);
-      bool ok = mbar_wait(w_full, 0);
+      bool ok = true, x0_used = false;
       const uint32_t id1 = idesc_bf16_f32(kTileM, H1), id2 = idesc_bf16_f32(kTileM, H2);
       for (int t = 0; t < my_tiles && ok; ++t) {
         const int xb = t % kXB;
         ok = mbar_wait(&x_full[xb], (uint32_t)((t / kXB) & 1));
+        x0_used = x0_used || ok;
         if (ok && t >= 1) ok = mbar_wait(d1_empty, (uint32_t)((t - 1) & 1));
+        for (int kb = 0; ok && t == 0 && kb < nk0; ++kb) ok = mbar_wait(&w_full[wbar_of(kb)], 0);
         if (!ok) break;
         tc_fence_after();
         const uint32_t xa = smem_u32(X + (size_t)xb * xbytes);
@@ -476,6 +494,7 @@ __global__ void __launch_bounds__(kThreadsPipe, 1) k_score_tc_pipe(const __grid_
           const int64_t kq = (int64_t)t * nk1 + kb;
           const int slot = (int)(kq & 1);
           ok = mbar_wait(&a_full[slot], (uint32_t)((kq >> 1) & 1));
+          if (ok && t == 0) ok = mbar_wait(&w_full[wbar_of(nk0 + kb)], 0);
           if (!ok) break;
           tc_fence_after();
           const uint32_t aa = smem_u32(AR + (size_t)slot * kTileM * 128);
@@ -491,13 +510,17 @@ __global__ void __launch_bounds__(kThreadsPipe, 1) k_score_tc_pipe(const __grid_
         *abort_flag = 1;
         latch_error(a.err, LS_ERR_TIMEOUT);
       }
+      // copies issued at the start and still in flight land in this CTA's
+      // shared memory: wait for them (bounded) before the CTA can exit
+      for (int b = 0; b < kWBars; ++b) mbar_wait(&w_full[b], 0);
+      if (!x0_used) mbar_wait(&x_full[0], 0);
     }
     __syncwarp();
   } else if (warp < kE1Warp0) {
     // ------------------------------------------------------------ feature-tile loader
     if (lane == 0) {
       int last[2] = {-1, -1};
-      for (int t = 0; t < my_tiles; ++t) {
+      for (int t = 1; t < my_tiles; ++t) {  // tile 0 was requested by thread 0
         const int xb = t % kXB;
         if (t >= kXB && !mbar_wait(&x_empty[xb], (uint32_t)(((t - kXB) / kXB) & 1))) {
           *abort_flag = 1;
@@ -820,7 +843,7 @@ bool plan_tc(const MlpDesc& m, TcPlan& p) {
   p.pipe = 0;
   if (p.n_tc == 2 && p.out[0] <= 256 && p.out[1] <= 256 && p.nc[0] == p.out[0] && p.nc[1] == p.out[1]) {
     const int64_t need = 1024 + (int64_t)p.chunks * cb + kXB * (int64_t)p.d_pad * kTileM * 2 + 2 * kTileM * 128 +
-                         8 * 32 + 2 * 256 * 32 + 2 * kTileM * 4 + 256 * 2 + 13 * 8 + 16;
+                         8 * 32 + 2 * 256 * 32 + 2 * kTileM * 4 + 256 * 2 + (12 + kWBars) * 8 + 16;
     if (need <= kMaxSmem) {
       p.pipe = 1;
       p.pipe_smem = (int)need;
