@@ -436,14 +436,20 @@ class ClockSampler:
                 "power_w_max": float(np.nanmax([num(r[3]) for r in self.rows]))}
 
 
+KERNEL_SOURCES = {"score_tc": ("k_score_tc.cu", "sm100.cuh"),
+                  "prefix_index": ("k_prefix_index.cu", "blockhash.cuh")}
+
+
 def profiled_traffic(kernel):
-    """DRAM bytes per launch of `kernel` from the committed ncu summary, if the
+    """DRAM bytes per launch of `kernel` from the committed ncu summaries, if the
     summary was taken on the kernel's current source (else None)."""
     import glob
     import hashlib
+    if kernel not in KERNEL_SOURCES:
+        return None
     src = os.path.join(ROOT, "paper_2606_00946_gb300", "csrc")
     h = hashlib.sha256()
-    for f in ("k_score_tc.cu", "sm100.cuh"):
+    for f in KERNEL_SOURCES[kernel]:
         with open(os.path.join(src, f), "rb") as fh:
             h.update(fh.read())
     sha = h.hexdigest()[:16]
@@ -724,13 +730,14 @@ def main():
             peak, unit, bound = peaks["bf16_tflops"], "TFLOP/s", "tensor"
         achieved = alg / (per[k] / 1e3)
         return {"kernel": k, "bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
-                "frac": achieved / peak, "traffic": profiled_traffic(k) if k == "score_tc" else None,
+                "frac": achieved / peak, "traffic": profiled_traffic(k),
                 "peak_source": f"{peak_src} (burst)", "avg_launch_ms": per[k], "timing": timing}
 
     route_kernels = [k for k in per_step if k in ("prefix_index", "prefix_match", "hash_screen", "probe_walk",
                                                   "features", "score_tc", "score_simt", "argmin")]
     dom = max(route_kernels, key=lambda k: per_step[k])
     roofline = dict(kernel_roofline(dom), branch="route (the step's critical branch)")
+    route_rooflines = {k: kernel_roofline(k) for k in route_kernels}
     train_kernels = [k for k in per_step if k in ("gemm_tc_fwd", "gemm_tc_dw", "gemm_tc_dx")]
     train_roofline = (dict(kernel_roofline(max(train_kernels, key=lambda k: per_step[k])), branch="train")
                       if train_kernels else None)
@@ -895,6 +902,7 @@ def main():
             "algorithmic": costs,
             "guarded_route": guards,
             "replay_admission": replay,
+            "route_rooflines": route_rooflines,
             "paper_point": paper_point,
             "training_config": training_config,
         }
