@@ -52,6 +52,40 @@ __device__ __forceinline__ uint64_t block_content(const int32_t* p, bool aligned
   return mix64(acc);
 }
 
+// The same content hash in two steps, so that a block's tokens can be
+// requested well before they are hashed.  `align`: 16, 8 or 4, the largest
+// power of two (up to 16) dividing the byte address of p.
+__device__ __forceinline__ void block_load(const int32_t* p, int align, uint32_t (&w)[16]) {
+  if (align == 16) {
+    const int4* q = reinterpret_cast<const int4*>(p);
+#pragma unroll
+    for (int v = 0; v < 4; ++v) {
+      const int4 t = __ldg(q + v);
+      w[4 * v] = (uint32_t)t.x;
+      w[4 * v + 1] = (uint32_t)t.y;
+      w[4 * v + 2] = (uint32_t)t.z;
+      w[4 * v + 3] = (uint32_t)t.w;
+    }
+  } else if (align == 8) {
+    const int2* q = reinterpret_cast<const int2*>(p);
+#pragma unroll
+    for (int v = 0; v < 8; ++v) {
+      const int2 t = __ldg(q + v);
+      w[2 * v] = (uint32_t)t.x;
+      w[2 * v + 1] = (uint32_t)t.y;
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < 16; ++j) w[j] = (uint32_t)__ldg(p + j);
+  }
+}
+__device__ __forceinline__ uint64_t block_hash(const uint32_t (&w)[16]) {
+  uint64_t acc = 0;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) acc ^= word_mix(w[2 * j], w[2 * j + 1], j);
+  return mix64(acc);
+}
+
 // Prefix state after this thread's block, for a chunk whose first block
 // follows state s_in.  Thread t holds content c (0 for threads past the last
 // block: they come after every real block, so they change nothing).

@@ -70,7 +70,7 @@ __device__ __forceinline__ uint64_t index_mask_w1(const uint64_t* __restrict__ e
 }
 
 template <int W>
-__global__ void __launch_bounds__(kNT) k_prefix_index(int n_req, const int32_t* __restrict__ tok,
+__global__ void __launch_bounds__(kNT, W <= 2 ? 7 : 1) k_prefix_index(int n_req, const int32_t* __restrict__ tok,
                                                       const int64_t* __restrict__ tok_off,
                                                       const uint64_t* __restrict__ gkeys,
                                                       const uint64_t* __restrict__ gmask, uint64_t gmask_slots,
@@ -91,7 +91,8 @@ __global__ void __launch_bounds__(kNT) k_prefix_index(int n_req, const int32_t* 
     const int64_t t0 = tok_off[r];
     const int64_t nb = (tok_off[r + 1] - t0) / kBlockTok;
     const int32_t* base = tok + t0;
-    const bool aligned = ((reinterpret_cast<uintptr_t>(base) & 15) == 0);
+    const uintptr_t ab = reinterpret_cast<uintptr_t>(base);
+    const int align = (ab & 15) == 0 ? 16 : (ab & 7) == 0 ? 8 : 4;
     uint64_t alive[W];
     int32_t hreg[W][2];  // hit length of instances 64w + lane and 64w + 32 + lane
 #pragma unroll
@@ -102,11 +103,16 @@ __global__ void __launch_bounds__(kNT) k_prefix_index(int n_req, const int32_t* 
     }
     uint64_t state = kG;  // s_{-1}
     bool any = n_inst > 0;
+    // tokens of the lane's block in the coming round, requested one round
+    // ahead so that their load overlaps the index probes of the current round
+    uint32_t tw[16];
+    if (lane < nb) block_load(base + (int64_t)lane * kBlockTok, align, tw);
     for (int64_t p = 0; p < nb && any; p += 32) {
       const int64_t b = p + lane;
       const bool in = b < nb;
       // inclusive scan: B = sum_{j <= lane} G^(lane - j) c_j, then s = G^(lane+1) s_in + B
-      uint64_t B = in ? block_content(base + b * kBlockTok, aligned) : 0ull;
+      uint64_t B = in ? block_hash(tw) : 0ull;
+      if (b + 32 < nb) block_load(base + (b + 32) * kBlockTok, align, tw);
 #pragma unroll
       for (int k = 0; k < 5; ++k) {
         const int off = 1 << k;
