@@ -2,6 +2,8 @@
 // helpers shared by the kernels, and the launchers each .cu file provides.
 #pragma once
 
+#include <utility>
+
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 #include <algorithm>
@@ -352,6 +354,34 @@ __device__ __forceinline__ float raw_feature(int k, int64_t L, int h, const floa
 __device__ __forceinline__ float zscore(float x, float mu, float sd) {
   float s = sd < 1e-12f ? 1.0f : sd;
   return (x - mu) / s;
+}
+
+// Launch of a kernel of the route or training chain with programmatic
+// dependent launch: it may start (and run what precedes its pdl_wait()) while
+// the previous kernel of the stream finishes.  `cluster` > 1 adds a cluster
+// dimension.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_chained(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                           int cluster, Args&&... args) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  int n = 1;
+  if (cluster > 1) {
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = cluster;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    n = 2;
+  }
+  cfg.attrs = attr;
+  cfg.numAttrs = n;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
 }
 
 // ---------------------------------------------------------------------------

@@ -18,6 +18,7 @@
 // round after which no instance matches, so tokens past the longest hit plus
 // one round are never read.
 #include "blockhash.cuh"
+#include "sm100.cuh"
 
 namespace ls {
 namespace {
@@ -75,6 +76,7 @@ __global__ void __launch_bounds__(kNT, W <= 2 ? 7 : 1) k_prefix_index(int n_req,
                                                       const uint64_t* __restrict__ gkeys,
                                                       const uint64_t* __restrict__ gmask, uint64_t gmask_slots,
                                                       int n_inst, int32_t* __restrict__ hits, DevState* st) {
+  sm100::pdl_wait();  // the previous kernel of the stream is complete
   route_snapshot(st);
   const int lane = threadIdx.x & 31;
   const int64_t warps = ((int64_t)gridDim.x * blockDim.x) >> 5;
@@ -168,6 +170,7 @@ __global__ void __launch_bounds__(kNT, W <= 2 ? 7 : 1) k_prefix_index(int n_req,
         if (i < n_inst) hrow[i] = ((alive[w] >> bit) & 1ull) ? (int32_t)nb : hreg[w][h];
       }
   }
+  sm100::pdl_trigger();  // the next kernel may start once every CTA is here
 }
 
 // Insert (instance, key) pairs: thread per key, instance by binary search in
@@ -218,14 +221,17 @@ cudaError_t launch_prefix_index(int n_req, const int32_t* tok, const int64_t* to
                                 int sms, DevState* st, cudaStream_t s) {
   if (n_req <= 0) return cudaSuccess;
   const int grid = std::max(1, std::min((n_req + kNT / 32 - 1) / (kNT / 32), sms * 16));  // one warp per request
+  void (*k)(int, const int32_t*, const int64_t*, const uint64_t*, const uint64_t*, uint64_t, int, int32_t*,
+            DevState*) = nullptr;
   switch (W) {
-    case 1: k_prefix_index<1><<<grid, kNT, 0, s>>>(n_req, tok, tok_off, gkeys, gmask, gmask_slots, n_inst, hits, st); break;
-    case 2: k_prefix_index<2><<<grid, kNT, 0, s>>>(n_req, tok, tok_off, gkeys, gmask, gmask_slots, n_inst, hits, st); break;
-    case 4: k_prefix_index<4><<<grid, kNT, 0, s>>>(n_req, tok, tok_off, gkeys, gmask, gmask_slots, n_inst, hits, st); break;
-    case 8: k_prefix_index<8><<<grid, kNT, 0, s>>>(n_req, tok, tok_off, gkeys, gmask, gmask_slots, n_inst, hits, st); break;
+    case 1: k = k_prefix_index<1>; break;
+    case 2: k = k_prefix_index<2>; break;
+    case 4: k = k_prefix_index<4>; break;
+    case 8: k = k_prefix_index<8>; break;
     default: return cudaErrorInvalidValue;
   }
-  return cudaGetLastError();
+  return launch_chained(k, dim3(grid), dim3(kNT), 0, s, 1, n_req, tok, tok_off, gkeys, gmask, gmask_slots, n_inst,
+                        hits, st);
 }
 
 cudaError_t launch_index_insert(const uint64_t* keys, const int64_t* key_off, int n_inst, int64_t n_keys,

@@ -49,14 +49,37 @@ __global__ void __launch_bounds__(256) k_publish(const __grid_constant__ PubArgs
   uint8_t* __restrict__ img = a.img[tgt];
   float* __restrict__ bnd = a.bounds[tgt];
   const int64_t n_img = a.n_tc ? a.grp_end[a.n_tc - 1] : 0;
-  const int64_t total = a.n_params + a.n_wt + n_img + a.n_bounds;
-  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
-       e += (int64_t)gridDim.x * blockDim.x) {
-    if (e < a.n_params) {
-      int l = 0;
-      while (l + 1 < m.n_layers && e >= m.woff[l + 1]) ++l;
-      const float v = __ldg(a.master + e);
-      pp[e] = (m.bf16 && e < m.boff[l]) ? round_bf16(v) : v;
+  // work items: the flat parameters 4 at a time, then the transposed copy,
+  // the image groups and the bounds one at a time
+  const int64_t n_p4 = (a.n_params + 3) / 4;
+  const int64_t total = n_p4 + a.n_wt + n_img + a.n_bounds;
+  for (int64_t it = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; it < total;
+       it += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t e = it - n_p4 + a.n_params;  // element index of the items past the parameters
+    if (it < n_p4) {
+      const int64_t e0 = 4 * it;
+      float v[4];
+      if (e0 + 4 <= a.n_params) {
+        const float4 q = __ldg(reinterpret_cast<const float4*>(a.master + e0));
+        v[0] = q.x; v[1] = q.y; v[2] = q.z; v[3] = q.w;
+      } else {
+#pragma unroll
+        for (int j = 0; j < 4; ++j) v[j] = e0 + j < a.n_params ? __ldg(a.master + e0 + j) : 0.0f;
+      }
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int64_t ej = e0 + j;
+        int l = 0;
+        while (l + 1 < m.n_layers && ej >= m.woff[l + 1]) ++l;
+        if (m.bf16 && ej < m.boff[l]) v[j] = round_bf16(v[j]);
+      }
+      if (e0 + 4 <= a.n_params) {
+        *reinterpret_cast<float4*>(pp + e0) = make_float4(v[0], v[1], v[2], v[3]);
+      } else {
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          if (e0 + j < a.n_params) pp[e0 + j] = v[j];
+      }
     } else if (e < a.n_params + a.n_wt) {
       const int64_t t = e - a.n_params;
       int l = 0;
@@ -134,7 +157,7 @@ cudaError_t launch_publish(const MlpDesc& m, const TcPlan* tc, const float* mast
     a.grp_end[l] = groups;
   }
   a.st = st;
-  const int64_t total = a.n_params + a.n_wt + groups + a.n_bounds;
+  const int64_t total = (a.n_params + 3) / 4 + a.n_wt + groups + a.n_bounds;
   const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((total + 255) / 256, (int64_t)sms * 4));
   k_publish<<<grid, 256, 0, s>>>(a);
   return cudaGetLastError();

@@ -414,14 +414,11 @@ __global__ void __launch_bounds__(kThreadsPipe, 1) k_score_tc_pipe(const __grid_
     *abort_flag = 0;
     fence_mbar_init();
     if (my_tiles > 0) {
-      // the weight chunks (in the order the first tile uses them, each K-block
-      // of tile 0 waiting only for its own chunk) and the first feature tile
-      // are requested before anything else, so they land during the prologue
-      // first tile's features, then the weight image: the K-blocks of layer 1
-      // (H1 x 128 B each) followed by those of layer 2 (H2 x 128 B each), one
-      // resident chunk each (offsets from the widths, not from indexed tables)
-      mbar_arrive_expect_tx(&x_full[0], (uint32_t)xbytes);
-      bulk_g2s(X, a.ximg + (int64_t)blockIdx.x * xbytes, (uint32_t)xbytes, &x_full[0]);
+      // the weight image is requested before anything else, so that it lands
+      // during the prologue: the K-blocks of layer 1 (H1 x 128 B each), then
+      // those of layer 2 (H2 x 128 B each), one resident chunk and barrier
+      // each, so that tile 0's K-block kb waits only for its own chunk
+      // (offsets from the widths, not from indexed tables)
       const int64_t l1_bytes = (int64_t)nk0 * H1 * 128;
       for (int q = 0; q < nk0 + nk1; ++q) {
         const uint32_t len = (uint32_t)(q < nk0 ? H1 : H2) * 128u;
@@ -459,6 +456,14 @@ __global__ void __launch_bounds__(kThreadsPipe, 1) k_score_tc_pipe(const __grid_
     *reinterpret_cast<uint4*>((l ? B2 : B1) + nosw16_offset(n, 8 * (e & 1))) = q;
   }
   fence_async_smem();  // the bias operands are read by the tensor cores (async proxy)
+  // everything above reads only the published weights; the feature tiles come
+  // from the previous kernel of the stream
+  pdl_wait();
+  pdl_trigger();
+  if (tid == 0 && my_tiles > 0) {
+    mbar_arrive_expect_tx(&x_full[0], (uint32_t)xbytes);
+    bulk_g2s(X, a.ximg + (int64_t)blockIdx.x * xbytes, (uint32_t)xbytes, &x_full[0]);
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -737,6 +742,7 @@ __global__ void __launch_bounds__(256) k_feature_image(const int64_t* __restrict
   __shared__ int row_q[kTileM];                        // its request, relative to the tile's first
   const int cpr = d_pad / 8;
   const int64_t xbytes = (int64_t)kTileM * d_pad * 2;
+  pdl_wait();  // hit lengths from the prefix kernel
   for (int64_t t = blockIdx.x; t < n_tiles; t += gridDim.x) {
     const int64_t g0 = t * kTileM;
     const int nrow = (int)(g0 + kTileM < rows ? kTileM : rows - g0);
@@ -783,6 +789,7 @@ __global__ void __launch_bounds__(256) k_feature_image(const int64_t* __restrict
     }
     __syncthreads();
   }
+  pdl_trigger();  // the scorer may start once every CTA is here
 }
 
 }  // namespace
@@ -885,9 +892,8 @@ cudaError_t launch_feature_image(const int64_t* tok_off, const int32_t* hits, in
     if (e != cudaSuccess) return e;
   }
   const int grid = (int)std::min<int64_t>(n_tiles, (int64_t)sms * 8);
-  k_feature_image<<<grid, 256, smem, s>>>(tok_off, hits, n_inst, xin, d_inst, d_req, req, mean, stdv, d_pad, rows,
-                                          n_tiles, nr_max, ximg);
-  return cudaGetLastError();
+  return launch_chained(k_feature_image, dim3(grid), dim3(256), smem, s, 1, tok_off, hits, n_inst, xin, d_inst, d_req,
+                        req, mean, stdv, d_pad, rows, n_tiles, nr_max, ximg);
 }
 
 cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const Published* pub, const int32_t* sel,
@@ -928,7 +934,7 @@ cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const Published* 
   if (p.pipe) {
     cudaError_t e = cudaFuncSetAttribute(k_score_tc_pipe, cudaFuncAttributeMaxDynamicSharedMemorySize, p.pipe_smem);
     if (e != cudaSuccess) return e;
-    k_score_tc_pipe<<<grid, kThreadsPipe, p.pipe_smem, s>>>(a);
+    return launch_chained(k_score_tc_pipe, dim3(grid), dim3(kThreadsPipe), (size_t)p.pipe_smem, s, 1, a);
   } else {
     cudaError_t e = cudaFuncSetAttribute(k_score_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, p.smem);
     if (e != cudaSuccess) return e;

@@ -171,6 +171,8 @@ __global__ void __launch_bounds__(kT, 1) k_tr_gemm(const __grid_constant__ TrArg
     tmem_alloc(tmem_holder, tcols);
     tmem_relinquish();
   }
+  // operands and side inputs come from the previous kernels of the stream
+  pdl_wait();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -368,6 +370,9 @@ __global__ void __launch_bounds__(kT, 1) k_tr_gemm(const __grid_constant__ TrArg
   }
   tc_fence_before();
   __syncthreads();
+  // the next kernel may start once every CTA is here (a waiting CTA of it
+  // holds a whole SM, so it is not let in earlier)
+  pdl_trigger();
   if (warp == 0) tmem_dealloc(tmem, tcols);
 }
 
@@ -379,6 +384,7 @@ __global__ void k_tr_gather(int B, int rows_pad, int d, int d_pad, const int32_t
                             const float* __restrict__ ring_y, const float* __restrict__ mean,
                             const float* __restrict__ stdv, uint8_t* __restrict__ a0, uint8_t* __restrict__ a0t,
                             float* __restrict__ y, int* err) {
+  pdl_wait();  // the ring and the device counters from the previous kernels of the stream
   const int64_t step = st->step;
   const int64_t count = st->ring_count;
   const int64_t nF = count < capacity ? count : capacity;
@@ -420,6 +426,7 @@ __global__ void k_tr_gather(int B, int rows_pad, int d, int d_pad, const int32_t
     for (int u = 0; u < 8; ++u)
       *reinterpret_cast<uint16_t*>(a0t + sw128_offset(c0 + u, j, d_pad)) = bf16_bits(v[u]);
   }
+  pdl_trigger();
 }
 
 // sum_{s < n} src[s * stride], added in order, eight loads in flight.
@@ -467,6 +474,8 @@ struct OptArgs {
 // optimiser update of the fp32 master, and the bf16 images of the updated
 // hidden-layer weights.  Block 0 also forms the minibatch loss.
 __global__ void __launch_bounds__(256) k_tr_opt(const __grid_constant__ OptArgs a) {
+  pdl_wait();  // gradient partials from the previous kernels of the stream
+  pdl_trigger();
   const int64_t t = a.st->step + 1;
   const float bc1 = a.st->adam_bc[0], bc2 = a.st->adam_bc[1];  // set by the gather kernel
   const MlpDesc& m = a.m;
@@ -551,22 +560,10 @@ cudaError_t launch_tr_gemm(const Ctx& c, const TrJob& j0, const TrJob* j1, int* 
   const int smem = gemm_smem_bytes();
   cudaError_t e = cudaFuncSetAttribute(k_tr_gemm, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  cudaLaunchConfig_t cfg{};
-  cfg.gridDim = dim3(n);
-  cfg.blockDim = dim3(kT);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = s;
-  cudaLaunchAttribute attr[1];
   // the column parts of a TE_FWD_OUT tile exchange row sums through
   // distributed shared memory: one cluster per tile
   const int cl = (j0.epi == TE_FWD_OUT && !j1) ? j0.n_split : 1;
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = cl;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, k_tr_gemm, a);
+  return launch_chained(k_tr_gemm, dim3(n), dim3(kT), (size_t)smem, s, cl, a);
 }
 
 // Column parts per tile: two when the columns split into halves that are
@@ -686,10 +683,9 @@ cudaError_t run_train_fast(Ctx& c, int B, const int32_t* idx, int opt, float lr,
   e = traced(c, TR_GATHER, 1, s, [&] {
     const int64_t total = (int64_t)R * (f.in_pad[0] / 8);
     const int grid = (int)std::min<int64_t>((total + 255) / 256, (int64_t)c.sms * 8);
-    k_tr_gather<<<grid, 256, 0, s>>>(B, R, m.w[0], f.in_pad[0], idx, c.st, c.cfg.ring_capacity, c.replay_base,
-                                     c.ring_x, c.ring_y,
-                                     c.mean, c.stdv, f.imgA[0], f.imgAT[0], c.ty, c.d_err);
-    return cudaGetLastError();
+    return launch_chained(k_tr_gather, dim3(grid), dim3(256), 0, s, 1, B, R, m.w[0], f.in_pad[0], idx, c.st,
+                          c.cfg.ring_capacity, c.replay_base, (const float*)c.ring_x, (const float*)c.ring_y,
+                          (const float*)c.mean, (const float*)c.stdv, f.imgA[0], f.imgAT[0], c.ty, c.d_err);
   });
   if (e != cudaSuccess) return e;
   // forward: hidden layers; the last one also runs the output layer and the loss
@@ -803,8 +799,7 @@ cudaError_t run_train_fast(Ctx& c, int B, const int32_t* idx, int opt, float lr,
   a.loss_out = loss_out ? loss_out : c.loss_tmp;
   return traced(c, TR_OPT, 1, s, [&] {
     const int grid = (int)std::min<int64_t>((c.n_params + 255) / 256, (int64_t)c.sms * 4);
-    k_tr_opt<<<grid, 256, 0, s>>>(a);
-    return cudaGetLastError();
+    return launch_chained(k_tr_opt, dim3(grid), dim3(256), 0, s, 1, a);
   });
 }
 
