@@ -116,6 +116,13 @@ typedef struct {
      * otherwise. */
     float dropout;
     uint64_t dropout_seed;
+    /* Launch shape of a tensor-core training step (bf16, hidden widths <=
+     * 256): <= 0 uses one launch per phase (gather, each product, optimiser;
+     * the default and the faster one measured), > 0 runs the whole step as
+     * one persistent launch of that many CTAs (at most the SM count) that
+     * meet at a grid barrier between phases.  Results are the same bits
+     * either way. */
+    int32_t train_ctas;
 } ls_config;
 
 typedef struct {

@@ -16,7 +16,7 @@ const char* const kTraceNames[TR_COUNT] = {
     "ring_append", "publish", "train_gather", "gemm_fwd", "loss_grad", "gemm_dw", "reduce_dw",
     "colsum_db", "gemm_dx", "optimizer", "memset", "score_tc", "features", "publish_tc",
     "hash_screen", "probe_screen", "probe_walk", "gemm_tc_fwd", "gemm_tc_dw", "gemm_tc_dx", "prefix_index",
-    "index_insert", "guards", "ring_bounds", "replay_admit"};
+    "index_insert", "guards", "ring_bounds", "replay_admit", "train_step"};
 }
 
 struct ls_ctx {
@@ -116,7 +116,7 @@ void free_all(Ctx& c) {
                   c.gpart, c.loss_tmp, c.d_err, c.pub[0].img, c.pub[1].img, c.xin, c.xrq, c.pairx, c.ximg,
                   c.bkeys, c.work, c.work_n, c.gkeys, c.gmask, c.st, c.tf.base, c.tf.parts,
                   c.pub[0].bounds, c.pub[1].bounds, c.bounds_stage, c.benc, c.remb, c.rnorm, c.rpart, c.rd,
-                  c.rn, c.rinv, c.rcount, c.rimg, c.rrank};
+                  c.rn, c.rinv, c.rcount, c.rimg, c.rrank, c.tr_bar};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   if (c.ev_pub) cudaEventDestroy(c.ev_pub);
@@ -275,7 +275,9 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
     tf_bytes = train_fast_bytes(m, c.tf, &pf);
     A(dalloc(&c.tf.base, tf_bytes));
     A(dalloc(&c.tf.parts, pf));
+    A(dalloc(&c.tr_bar, 2));
     if (e == cudaSuccess) train_fast_bind(m, c.tf, c.tf.base, c.tf.parts);
+    c.train_ctas = cfg->train_ctas > 0 ? std::min(cfg->train_ctas, c.sms) : 0;
   }
   if (e == cudaSuccess) {
     A(cudaEventCreateWithFlags(&c.ev_pub, cudaEventDisableTiming));

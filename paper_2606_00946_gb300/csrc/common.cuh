@@ -112,7 +112,7 @@ enum TraceId {
   TR_GATHER, TR_GEMM_FWD, TR_LOSS, TR_GEMM_DW, TR_REDUCE, TR_COLSUM, TR_GEMM_DX, TR_OPT,
   TR_MEMSET, TR_SCORE_TC, TR_NORM_ROWS, TR_PUBLISH_TC, TR_HASH_BATCH, TR_SCREEN, TR_WALK,
   TR_GEMM_TC_FWD, TR_GEMM_TC_DW, TR_GEMM_TC_DX, TR_PREFIX_INDEX, TR_INDEX_INSERT,
-  TR_GUARDS, TR_BOUNDS, TR_REPLAY, TR_COUNT
+  TR_GUARDS, TR_BOUNDS, TR_REPLAY, TR_TRAIN_STEP, TR_COUNT
 };
 extern const char* const kTraceNames[TR_COUNT];
 
@@ -260,6 +260,8 @@ struct Ctx {
   int64_t gpart_floats = 0;
   float* loss_tmp = nullptr;  // [1]
   TrainFast tf;               // tensor-core training buffers (when tf.on)
+  int train_ctas = 0;         // > 0: persistent training step of that many CTAs
+  uint32_t* tr_bar = nullptr; // [2]: its grid-barrier arrivals and abort flag
 
   int* d_err = nullptr;       // first device-side error (0 = none)
   int sms = 148;              // SM count of the context's device

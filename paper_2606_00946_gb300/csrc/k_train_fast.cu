@@ -80,6 +80,7 @@ struct TrJob {
 struct TrArgs {
   TrJob job[2];
   int n_cta0;                        // CTAs of job 0; the rest run job 1
+  int n_cta;                         // CTAs of both jobs
   int* err;
   const DevState* st;                // optimiser step counter (dropout stream)
   uint64_t drop_seed, drop_thr;      // keep <=> (u >> 11) >= drop_thr
@@ -134,49 +135,40 @@ __device__ __forceinline__ void store_col16(uint8_t* imgT, int rowsT, int j, int
     *reinterpret_cast<uint16_t*>(imgT + sw128_offset(c + u, j, rowsT)) = bf16_bits(v[u]);
 }
 
-__global__ void __launch_bounds__(kT, 1) k_tr_gemm(const __grid_constant__ TrArgs args) {
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const bool second = (int)blockIdx.x >= args.n_cta0;
+// Shared memory of a training-product CTA: kMaxChunks stages of one 128-row A
+// tile and one (<= 256)-row B tile, then the barriers and epilogue scratch.
+__device__ __forceinline__ uint8_t* tr_tail(uint8_t* smem) {
+  return smem + (size_t)kMaxChunks * (kM * 128 + 256 * 128);
+}
+
+// One output tile (part `bid` of the products in `args`) on this CTA's shared
+// memory and TMEM accumulator.  Every mbarrier advances by one phase per tile
+// (parity `par`): chunk barriers the tile does not use are arrived on with no
+// bytes.  Returns false after a timed-out wait (error latched, copies in
+// flight waited for).
+__device__ __forceinline__ bool tr_tile(const TrArgs& args, int bid, uint8_t* smem, uint32_t tmem, uint32_t par) {
+  const bool second = bid >= args.n_cta0;
   const TrJob& J = args.job[second ? 1 : 0];
-  const int li = second ? (int)blockIdx.x - args.n_cta0 : (int)blockIdx.x;
+  const int li = second ? bid - args.n_cta0 : bid;
   const int ns = li % J.n_split, rest = li / J.n_split;
   const int mt = rest % J.m_tiles, split = rest / J.m_tiles;
   const int m0 = mt * kM;
   const int NT = J.NT, N = NT * J.n_split, n0 = ns * NT, nch = J.nchunks;
   const uint32_t a_bytes = kM * 128, b_bytes = (uint32_t)NT * 128;
   const uint32_t stage_bytes = a_bytes + b_bytes;
-  uint8_t* tail = smem + (size_t)kMaxChunks * (kM * 128 + 256 * 128);
+  uint8_t* tail = tr_tail(smem);
   uint64_t* full = reinterpret_cast<uint64_t*>(tail);           // [kMaxChunks]
   uint64_t* done = full + kMaxChunks;
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(done + 1);
   float* s_bias = reinterpret_cast<float*>(tail + 128);         // [256]
   float* s_w = s_bias + 256;                                    // [256] bf16-rounded output weights
   float* red = s_w + 256;                                       // [4][256] column sums by lane quadrant
   float* red2 = red + 4 * 256;                                  // [4][256]
-  float* rowq = red2 + 4 * 256;                                 // [4][128] row dots by column quarter
-  float* rowdot = rowq + 4 * 128;                               // [128] this CTA's row dots
+  float* rowq = red2 + 4 * 256;                                 // [8][128] row dots by column group
+  float* rowdot = rowq + 8 * 128;                               // [128] this CTA's row dots
   float* yrow = rowdot + 128;                                   // [128] predictions
   float* wsum = yrow + 128;                                     // [8] warp partials
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  uint32_t tcols = 32;
-  while ((int)tcols < NT) tcols <<= 1;
-  if (tid == 0) {
-    for (int c = 0; c < kMaxChunks; ++c) mbar_init(&full[c], 1);
-    mbar_init(done, 1);
-    fence_mbar_init();
-  }
-  if (warp == 0) {
-    tmem_alloc(tmem_holder, tcols);
-    tmem_relinquish();
-  }
-  // operands and side inputs come from the previous kernels of the stream
-  pdl_wait();
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = *tmem_holder;
   bool ok = true;
   if (tid == 0) {
     for (int c = 0; c < nch; ++c) {
@@ -186,9 +178,10 @@ __global__ void __launch_bounds__(kT, 1) k_tr_gemm(const __grid_constant__ TrArg
       bulk_g2s(sa, J.A + (size_t)kb * J.rA * 128 + (size_t)m0 * 128, a_bytes, &full[c]);
       bulk_g2s(sa + a_bytes, J.B + (size_t)kb * N * 128 + (size_t)n0 * 128, b_bytes, &full[c]);
     }
+    for (int c = nch; c < kMaxChunks; ++c) mbar_arrive(&full[c]);
     const uint32_t idesc = idesc_bf16_f32(kM, NT);
     for (int c = 0; c < nch; ++c) {
-      if (!mbar_wait(&full[c], 0)) { ok = false; break; }
+      if (!mbar_wait(&full[c], par)) { ok = false; break; }
       tc_fence_after();
       const uint32_t sa = smem_u32(smem + (size_t)c * stage_bytes), sb = sa + a_bytes;
 #pragma unroll
@@ -203,14 +196,14 @@ __global__ void __launch_bounds__(kT, 1) k_tr_gemm(const __grid_constant__ TrArg
     if (J.epi == TE_FWD_OUT) s_w[t] = round_bf16(__ldg(J.wL + n0 + t));
   }
   __syncwarp();
-  if (!mbar_wait(done, 0)) ok = false;
+  if (!mbar_wait(done, par)) ok = false;
   ok = __syncthreads_and(ok) != 0;  // one decision for the whole CTA
   if (!ok) {
     latch_error(args.err, LS_ERR_TIMEOUT);
     // copies that may still be in flight land in this CTA's own shared memory;
     // wait (bounded) for them before the CTA exits
     if (tid == 0)
-      for (int c = 0; c < nch; ++c) mbar_wait(&full[c], 0);
+      for (int c = 0; c < nch; ++c) mbar_wait(&full[c], par);
   }
   tc_fence_after();
 
@@ -287,22 +280,35 @@ __global__ void __launch_bounds__(kT, 1) k_tr_gemm(const __grid_constant__ TrArg
   }
   if (J.epi == TE_FWD_OUT) {
     // pass 1: activations and this warp's part of the output dot product
+    // With all 256 columns in one CTA (no cluster), each warp keeps its two
+    // 32-column halves apart and the row dot is added as the two 128-column
+    // CTAs of the cluster form add it: the same order, the same bits.
+    const bool whole = NT == 256;
     if (ok) {
-      float dot = 0.0f;
+      float dot[2] = {0.0f, 0.0f};
       for (int c = cbeg; c < cbeg + cw; c += 16) {
         uint32_t v[16];
         tmem_ld16x(tmem + lane_addr + (uint32_t)c, v);
         tmem_wait_ld();
+        const int hh = whole && c >= cbeg + 32 ? 1 : 0;
 #pragma unroll
         for (int u = 0; u < 16; ++u) {
           const float z = __uint_as_float(v[u]) + s_bias[c + u];
-          dot = fmaf(round_bf16(z > 0.0f ? z : 0.0f), s_w[c + u], dot);
+          dot[hh] = fmaf(round_bf16(z > 0.0f ? z : 0.0f), s_w[c + u], dot[hh]);
         }
       }
-      rowq[cq * 128 + r] = dot;
+      if (whole) {
+        rowq[(2 * cq) * 128 + r] = dot[0];
+        rowq[(2 * cq + 1) * 128 + r] = dot[1];
+      } else {
+        rowq[cq * 128 + r] = dot[0];
+      }
     }
     __syncthreads();
-    if (ok && tid < kM) rowdot[tid] = ((rowq[tid] + rowq[128 + tid]) + rowq[256 + tid]) + rowq[384 + tid];
+    if (ok && tid < kM) {
+      const float lo = ((rowq[tid] + rowq[128 + tid]) + rowq[256 + tid]) + rowq[384 + tid];
+      rowdot[tid] = whole ? lo + (((rowq[512 + tid] + rowq[640 + tid]) + rowq[768 + tid]) + rowq[896 + tid]) : lo;
+    }
     if (J.n_split > 1) cluster_sync();
     else __syncthreads();
     if (ok && tid < kM) {
@@ -370,30 +376,80 @@ __global__ void __launch_bounds__(kT, 1) k_tr_gemm(const __grid_constant__ TrArg
   }
   tc_fence_before();
   __syncthreads();
+  return ok;
+}
+
+// One launch per product (or pair of products): CTA b runs tile b.
+__global__ void __launch_bounds__(kT, 1) k_tr_gemm(const __grid_constant__ TrArgs args) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(tr_tail(smem));
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(full + kMaxChunks + 1);
+  const int NT = args.job[(int)blockIdx.x >= args.n_cta0 ? 1 : 0].NT;
+  uint32_t tcols = 32;
+  while ((int)tcols < NT) tcols <<= 1;
+  if (threadIdx.x == 0) {
+    for (int c = 0; c <= kMaxChunks; ++c) mbar_init(&full[c], 1);  // chunk barriers, then `done`
+    fence_mbar_init();
+  }
+  if (threadIdx.x < 32) {
+    tmem_alloc(tmem_holder, tcols);
+    tmem_relinquish();
+  }
+  // operands and side inputs come from the previous kernels of the stream
+  pdl_wait();
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_holder;
+  tr_tile(args, (int)blockIdx.x, smem, tmem, 0);
   // the next kernel may start once every CTA is here (a waiting CTA of it
   // holds a whole SM, so it is not let in earlier)
   pdl_trigger();
-  if (warp == 0) tmem_dealloc(tmem, tcols);
+  if (threadIdx.x < 32) tmem_dealloc(tmem, tcols);
 }
 
 // Minibatch gather: row j of the batch (slot idx[j], or (step*B + j) mod
 // valid) z-scored and rounded to bf16 into img(A_0) and img(A_0^T); rows past
 // the batch and columns past d are zero.  Thread = (row j, 8 columns).
-__global__ void k_tr_gather(int B, int rows_pad, int d, int d_pad, const int32_t* __restrict__ idx,
-                            DevState* st, int64_t capacity, int64_t replay_base, const float* __restrict__ ring_x,
-                            const float* __restrict__ ring_y, const float* __restrict__ mean,
-                            const float* __restrict__ stdv, uint8_t* __restrict__ a0, uint8_t* __restrict__ a0t,
-                            float* __restrict__ y, int* err) {
-  pdl_wait();  // the ring and the device counters from the previous kernels of the stream
+struct GatherArgs {
+  int B, rows_pad, d, d_pad;
+  const int32_t* idx;
+  DevState* st;
+  int64_t capacity, replay_base;
+  const float* ring_x;
+  const float* ring_y;
+  const float* mean;
+  const float* stdv;
+  uint8_t* a0;
+  uint8_t* a0t;
+  float* y;
+  int* err;
+};
+
+// Items [first, total) with stride `stride` of the minibatch gather; `lead`:
+// this thread also checks the buffer and sets the Adam bias corrections.
+__device__ __forceinline__ void tr_gather_items(const GatherArgs& g, int64_t first, int64_t stride, bool lead) {
+  const int B = g.B, rows_pad = g.rows_pad, d = g.d, d_pad = g.d_pad;
+  const int32_t* __restrict__ idx = g.idx;
+  const float* __restrict__ ring_x = g.ring_x;
+  const float* __restrict__ ring_y = g.ring_y;
+  const float* __restrict__ mean = g.mean;
+  const float* __restrict__ stdv = g.stdv;
+  uint8_t* __restrict__ a0 = g.a0;
+  uint8_t* __restrict__ a0t = g.a0t;
+  float* __restrict__ y = g.y;
+  int* err = g.err;
+  DevState* st = g.st;
   const int64_t step = st->step;
   const int64_t count = st->ring_count;
-  const int64_t nF = count < capacity ? count : capacity;
+  const int64_t nF = count < g.capacity ? count : g.capacity;
   const int64_t valid = nF + st->replay_count;  // F u R
-  if (valid < 1 && blockIdx.x == 0 && threadIdx.x == 0) latch_error(err, LS_ERR_STATE);
-  if (blockIdx.x == 0 && threadIdx.x == 0) set_adam_bc(st);
+  const int64_t replay_base = g.replay_base;
+  if (valid < 1 && lead) latch_error(err, LS_ERR_STATE);
+  if (lead) set_adam_bc(st);
   const int64_t total = (int64_t)rows_pad * (d_pad / 8);
-  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
-       e += (int64_t)gridDim.x * blockDim.x) {
+  for (int64_t e = first; e < total; e += stride) {
     const int j = (int)(e % rows_pad), c0 = (int)(e / rows_pad) * 8;
     float v[8];
 #pragma unroll
@@ -426,6 +482,12 @@ __global__ void k_tr_gather(int B, int rows_pad, int d, int d_pad, const int32_t
     for (int u = 0; u < 8; ++u)
       *reinterpret_cast<uint16_t*>(a0t + sw128_offset(c0 + u, j, d_pad)) = bf16_bits(v[u]);
   }
+}
+
+__global__ void k_tr_gather(const __grid_constant__ GatherArgs g) {
+  pdl_wait();  // the ring and the device counters from the previous kernels of the stream
+  tr_gather_items(g, blockIdx.x * (int64_t)blockDim.x + threadIdx.x, (int64_t)gridDim.x * blockDim.x,
+                  blockIdx.x == 0 && threadIdx.x == 0);
   pdl_trigger();
 }
 
@@ -472,16 +534,12 @@ struct OptArgs {
 
 // Gradient of every parameter as an ordered sum of its partials, the
 // optimiser update of the fp32 master, and the bf16 images of the updated
-// hidden-layer weights.  Block 0 also forms the minibatch loss.
-__global__ void __launch_bounds__(256) k_tr_opt(const __grid_constant__ OptArgs a) {
-  pdl_wait();  // gradient partials from the previous kernels of the stream
-  pdl_trigger();
-  const int64_t t = a.st->step + 1;
+// hidden-layer weights, for parameters [first, n) with stride `stride`.
+__device__ __forceinline__ void tr_opt_items(const OptArgs& a, int64_t first, int64_t stride) {
   const float bc1 = a.st->adam_bc[0], bc2 = a.st->adam_bc[1];  // set by the gather kernel
   const MlpDesc& m = a.m;
   const int nl = m.n_layers;
-  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < a.n;
-       e += (int64_t)gridDim.x * blockDim.x) {
+  for (int64_t e = first; e < a.n; e += stride) {
     int l = 0;
     while (l + 1 < nl && e >= m.woff[l + 1]) ++l;
     const int out = m.w[l + 1], in = m.w[l];
@@ -531,19 +589,135 @@ __global__ void __launch_bounds__(256) k_tr_opt(const __grid_constant__ OptArgs 
       *reinterpret_cast<uint16_t*>(P.imgWT + sw128_offset(i, o, P.in_pad)) = b;
     }
   }
-  if (a.mode != 0 && blockIdx.x == 0 && threadIdx.x == 0 && a.loss_out) {
+}
+
+// The minibatch loss (sum of the tile partials in order), by one thread.
+__device__ __forceinline__ void tr_loss(const OptArgs& a) {
+  if (a.mode != 0 && a.loss_out) {
     float s = 0.0f;
     for (int tt = 0; tt < a.T; ++tt) s += a.partLoss[tt];
     *a.loss_out = s / (float)a.B;
   }
+}
+
+__global__ void __launch_bounds__(256) k_tr_opt(const __grid_constant__ OptArgs a) {
+  pdl_wait();  // gradient partials from the previous kernels of the stream
+  pdl_trigger();
+  const int64_t t = a.st->step + 1;
+  tr_opt_items(a, blockIdx.x * (int64_t)blockDim.x + threadIdx.x, (int64_t)gridDim.x * blockDim.x);
+  if (blockIdx.x == 0 && threadIdx.x == 0) tr_loss(a);
   if (a.mode != 0 && last_block(&a.st->done[DONE_OPT]) && threadIdx.x == 0) advance_step(a.st, t);
 }
 
-int gemm_smem_bytes() {
-  return 1024 + kMaxChunks * (kM * 128 + 256 * 128) + 128 + (256 + 256 + 8 * 256 + 4 * 128 + 128 + 128 + 8) * 4;
+// ---------------------------------------------------------------------------
+// The whole step as one persistent launch of a few CTAs (the rest of the GPU
+// stays with routing): the gather, each product of the forward and backward
+// passes (a phase: its tiles spread over the CTAs) and the optimiser, with a
+// grid barrier between phases.  Same tiles, same epilogues and same order of
+// every sum as the launch-per-phase path, so the same bits.
+// ---------------------------------------------------------------------------
+constexpr int kMaxPhases = 2 * (LS_MAX_LAYERS - 1);
+constexpr uint32_t kGridSpin = 1u << 21;  // barrier polls before giving up (~0.2 s)
+
+struct StepArgs {
+  GatherArgs g;
+  TrArgs ph[kMaxPhases];
+  int n_ph;
+  OptArgs opt;
+  uint32_t* bar;  // [0] arrivals, [1] abort flag; zero at launch
+};
+static_assert(sizeof(StepArgs) <= 32000, "kernel parameters of the persistent step");
+
+__device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
 }
 
-cudaError_t launch_tr_gemm(const Ctx& c, const TrJob& j0, const TrJob* j1, int* err, cudaStream_t s) {
+// All CTAs meet (arrival `k` of each CTA: target k * gridDim.x).  Generic
+// writes before it are visible to every read after it, bulk copies included.
+// False for every CTA once one has given up (bounded wait) or failed a tile.
+__device__ __forceinline__ bool tr_grid_sync(uint32_t* bar, uint32_t target, int* err) {
+  __shared__ int s_go;
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    volatile uint32_t* abort = bar + 1;
+    __threadfence();
+    atomicAdd(bar, 1u);
+    int go = 1;
+    for (uint32_t it = 0; ld_acquire_u32(bar) < target; ++it) {
+      if (*abort || it >= kGridSpin) {
+        if (!*abort) {
+          atomicExch(bar + 1, 1u);
+          latch_error(err, LS_ERR_TIMEOUT);
+        }
+        go = 0;
+        break;
+      }
+      __nanosleep(64);
+    }
+    if (*abort) go = 0;
+    s_go = go;
+  }
+  __syncthreads();
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+  return s_go != 0;
+}
+
+__global__ void __launch_bounds__(kT, 1) k_tr_step(const __grid_constant__ StepArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(tr_tail(smem));
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(full + kMaxChunks + 1);
+  const int tid = threadIdx.x;
+  if (tid == 0) {
+    for (int c = 0; c <= kMaxChunks; ++c) mbar_init(&full[c], 1);  // chunk barriers, then `done`
+    fence_mbar_init();
+  }
+  if (tid < 32) {
+    tmem_alloc(tmem_holder, 256);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_holder;
+  int* err = a.g.err;
+  const int64_t first = blockIdx.x * (int64_t)kT + tid, stride = (int64_t)gridDim.x * kT;
+  uint32_t arrivals = 0;
+  tr_gather_items(a.g, first, stride, blockIdx.x == 0 && tid == 0);
+  bool go = tr_grid_sync(a.bar, ++arrivals * gridDim.x, err);
+  uint32_t par = 0;
+  for (int ph = 0; go && ph < a.n_ph; ++ph) {
+    const TrArgs& P = a.ph[ph];
+    for (int b = blockIdx.x; b < P.n_cta; b += gridDim.x) {
+      if (!tr_tile(P, b, smem, tmem, par)) {
+        if (tid == 0) atomicExch(a.bar + 1, 1u);
+        go = false;
+        break;
+      }
+      par ^= 1u;
+    }
+    if (go) go = tr_grid_sync(a.bar, ++arrivals * gridDim.x, err);
+  }
+  if (go) {
+    tr_opt_items(a.opt, first, stride);
+    if (tr_grid_sync(a.bar, ++arrivals * gridDim.x, err) && blockIdx.x == 0 && tid == 0) {
+      tr_loss(a.opt);
+      if (a.opt.mode != 0) advance_step(a.opt.st, a.opt.st->step + 1);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (tid < 32) tmem_dealloc(tmem, 256);
+}
+
+int gemm_smem_bytes() {
+  return 1024 + kMaxChunks * (kM * 128 + 256 * 128) + 128 + (256 + 256 + 8 * 256 + 8 * 128 + 128 + 128 + 8) * 4;
+}
+
+TrArgs tr_args(const Ctx& c, const TrJob& j0, const TrJob* j1, int* err) {
   TrArgs a{};
   a.st = c.st;
   a.drop_seed = c.cfg.dropout_seed;
@@ -557,6 +731,13 @@ cudaError_t launch_tr_gemm(const Ctx& c, const TrJob& j0, const TrJob* j1, int* 
     n += j1->m_tiles * j1->n_split * j1->splits;
   }
   a.err = err;
+  a.n_cta = n;
+  return a;
+}
+
+cudaError_t launch_tr_gemm(const Ctx& c, const TrJob& j0, const TrJob* j1, int* err, cudaStream_t s) {
+  const TrArgs a = tr_args(c, j0, j1, err);
+  const int n = a.n_cta;
   const int smem = gemm_smem_bytes();
   cudaError_t e = cudaFuncSetAttribute(k_tr_gemm, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
@@ -673,28 +854,57 @@ cudaError_t train_fast_images(Ctx& c, cudaStream_t s) {
   return cudaGetLastError();
 }
 
+namespace {
+GatherArgs gather_args(const Ctx& c, int B, const int32_t* idx) {
+  GatherArgs g{};
+  g.B = B;
+  g.rows_pad = ((B + kM - 1) / kM) * kM;
+  g.d = c.mlp.w[0];
+  g.d_pad = c.tf.in_pad[0];
+  g.idx = idx;
+  g.st = c.st;
+  g.capacity = c.cfg.ring_capacity;
+  g.replay_base = c.replay_base;
+  g.ring_x = c.ring_x;
+  g.ring_y = c.ring_y;
+  g.mean = c.mean;
+  g.stdv = c.stdv;
+  g.a0 = c.tf.imgA[0];
+  g.a0t = c.tf.imgAT[0];
+  g.y = c.ty;
+  g.err = c.d_err;
+  return g;
+}
+}  // namespace
+
 cudaError_t run_train_fast(Ctx& c, int B, const int32_t* idx, int opt, float lr, float* loss_out, cudaStream_t s) {
   const MlpDesc& m = c.mlp;
   TrainFast& f = c.tf;
   const int nh = m.n_layers - 1;  // hidden layers 0..nh-1, output layer nh
   const int R = ((B + kM - 1) / kM) * kM;
   const int T = R / kM;
-  cudaError_t e;
-  e = traced(c, TR_GATHER, 1, s, [&] {
-    const int64_t total = (int64_t)R * (f.in_pad[0] / 8);
-    const int grid = (int)std::min<int64_t>((total + 255) / 256, (int64_t)c.sms * 8);
-    return launch_chained(k_tr_gather, dim3(grid), dim3(256), 0, s, 1, B, R, m.w[0], f.in_pad[0], idx, c.st,
-                          c.cfg.ring_capacity, c.replay_base, (const float*)c.ring_x, (const float*)c.ring_y,
-                          (const float*)c.mean, (const float*)c.stdv, f.imgA[0], f.imgAT[0], c.ty, c.d_err);
-  });
-  if (e != cudaSuccess) return e;
+  // one persistent launch (the products become its phases) or one launch each
+  const bool one = c.train_ctas > 0;
+  static thread_local StepArgs step;
+  step = StepArgs{};
+  cudaError_t e = cudaSuccess;
+  if (!one) {
+    e = traced(c, TR_GATHER, 1, s, [&] {
+      const int64_t total = (int64_t)R * (f.in_pad[0] / 8);
+      const int grid = (int)std::min<int64_t>((total + 255) / 256, (int64_t)c.sms * 8);
+      return launch_chained(k_tr_gather, dim3(grid), dim3(256), 0, s, 1, gather_args(c, B, idx));
+    });
+    if (e != cudaSuccess) return e;
+  }
   // forward: hidden layers; the last one also runs the output layer and the loss
   for (int l = 0; l < nh; ++l) {
     const bool last = l == nh - 1;
     TrJob J{};
     J.epi = last ? TE_FWD_OUT : TE_FWD;
     J.m_tiles = T;
-    J.n_split = n_split_for(m.w[l + 1]);
+    // the persistent launch has no clusters: the output layer's row dot
+    // products stay within one CTA (all columns of the tile)
+    J.n_split = (last && one) ? 1 : n_split_for(m.w[l + 1]);
     J.splits = 1;
     J.nchunks = f.in_pad[l] / 64;
     J.NT = m.w[l + 1] / J.n_split;
@@ -724,6 +934,10 @@ cudaError_t run_train_fast(Ctx& c, int B, const int32_t* idx, int opt, float lr,
     }
     // dropout on hidden activation l + 1 when it feeds another hidden layer
     J.drop_h = (c.cfg.dropout > 0.0f && l + 2 < m.n_layers) ? l + 1 : 0;
+    if (one) {
+      step.ph[step.n_ph++] = tr_args(c, J, nullptr, c.d_err);
+      continue;
+    }
     e = traced(c, TR_GEMM_TC_FWD, 1, s, [&] { return launch_tr_gemm(c, J, nullptr, c.d_err, s); });
     if (e != cudaSuccess) return e;
   }
@@ -768,6 +982,10 @@ cudaError_t run_train_fast(Ctx& c, int B, const int32_t* idx, int opt, float lr,
       X.colpart = f.partB[l - 1];
       X.drop_h = (c.cfg.dropout > 0.0f && l < m.n_layers - 1) ? l : 0;  // input a_l was dropped
     }
+    if (one) {
+      step.ph[step.n_ph++] = tr_args(c, W, l > 0 ? &X : nullptr, c.d_err);
+      continue;
+    }
     e = traced(c, l > 0 ? TR_GEMM_TC_DX : TR_GEMM_TC_DW, 1, s,
                [&] { return launch_tr_gemm(c, W, l > 0 ? &X : nullptr, c.d_err, s); });
     if (e != cudaSuccess) return e;
@@ -797,6 +1015,29 @@ cudaError_t run_train_fast(Ctx& c, int B, const int32_t* idx, int opt, float lr,
   a.partLoss = f.partLoss;
   a.B = B;
   a.loss_out = loss_out ? loss_out : c.loss_tmp;
+  if (one) {
+    step.g = gather_args(c, B, idx);
+    step.opt = a;
+    step.bar = c.tr_bar;
+    return traced(c, TR_TRAIN_STEP, 1, s, [&] {
+      cudaError_t e2 = cudaMemsetAsync(c.tr_bar, 0, 2 * sizeof(uint32_t), s);
+      if (e2 != cudaSuccess) return e2;
+      const int smem = gemm_smem_bytes();
+      e2 = cudaFuncSetAttribute(k_tr_step, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+      if (e2 != cudaSuccess) return e2;
+      cudaLaunchConfig_t cfg{};
+      cfg.gridDim = dim3(c.train_ctas);
+      cfg.blockDim = dim3(kT);
+      cfg.dynamicSmemBytes = smem;
+      cfg.stream = s;
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeCooperative;  // every CTA resident: the grid barrier needs it
+      attr[0].val.cooperative = 1;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      return cudaLaunchKernelEx(&cfg, k_tr_step, step);
+    });
+  }
   return traced(c, TR_OPT, 1, s, [&] {
     const int grid = (int)std::min<int64_t>((c.n_params + 255) / 256, (int64_t)c.sms * 4);
     return launch_chained(k_tr_opt, dim3(grid), dim3(256), 0, s, 1, a);

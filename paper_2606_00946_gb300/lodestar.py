@@ -36,7 +36,7 @@ class ls_config(C.Structure):
                 ("ring_capacity", C.c_int64), ("max_train_batch", C.c_int32),
                 ("max_batch_tokens", C.c_int64), ("prefix_mode", C.c_int32), ("scorer", C.c_int32),
                 ("replay_capacity", C.c_int64), ("pending_capacity", C.c_int64), ("dropout", C.c_float),
-                ("dropout_seed", C.c_uint64)]
+                ("dropout_seed", C.c_uint64), ("train_ctas", C.c_int32)]
 
 
 class ls_info(C.Structure):
@@ -153,7 +153,7 @@ def make_config(widths, d_inst, d_req, dtype="bf16", max_instances=64, max_reque
                 max_keys_per_instance=16384, max_load=0.5, ring_capacity=65536,
                 max_train_batch=4096, scorer="auto", max_batch_tokens=1 << 24,
                 prefix_mode="auto", replay_capacity=0, pending_capacity=0, dropout=0.0,
-                dropout_seed=0) -> ls_config:
+                dropout_seed=0, train_ctas=0) -> ls_config:
     c = ls_config()
     c.n_layers = len(widths) - 1
     for i, w in enumerate(widths):
@@ -168,6 +168,7 @@ def make_config(widths, d_inst, d_req, dtype="bf16", max_instances=64, max_reque
     c.prefix_mode = PREFIX_MODES.get(prefix_mode, prefix_mode)
     c.replay_capacity, c.pending_capacity = int(replay_capacity), int(pending_capacity)
     c.dropout, c.dropout_seed = float(dropout), int(dropout_seed) & (2**64 - 1)
+    c.train_ctas = int(train_ctas)
     return c
 
 

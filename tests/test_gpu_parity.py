@@ -424,6 +424,42 @@ def test_train_adam_bf16(steps, batch):
     r.close()
 
 
+@pytest.mark.parametrize("cfg_name,dropout", [("training", 0.0), ("homogeneous", 0.2)])
+def test_persistent_train_step_same_bits(cfg_name, dropout):
+    # The one-launch step (phases met at a grid barrier, the output layer's
+    # 256 columns in one CTA) against one launch per phase: parameters, Adam
+    # moments and loss equal bit for bit after several steps.
+    cfg = W.CONFIGS[cfg_name]
+    rng = np.random.default_rng(31)
+    n = 9000
+    x, y = W.records(rng, cfg, n)
+    mean, std = W.normaliser(np.random.default_rng(32), cfg)
+    params = W.xavier_params(cfg.widths, 5)
+    out = []
+    for tc in (-1, 24):
+        r = H.Router(cfg.widths, cfg.d_inst, cfg.d_req, cfg.dtype, max_instances=4, max_requests=16,
+                     max_keys_per_instance=64, ring_capacity=n, max_train_batch=4096, dropout=dropout,
+                     dropout_seed=77, train_ctas=tc)
+        r.set_normalizer(torch.from_numpy(mean).cuda(), torch.from_numpy(std).cuda())
+        r.set_params(torch.from_numpy(params).cuda())
+        r.log(torch.from_numpy(x).cuda(), torch.from_numpy(y).cuda())
+        loss = torch.zeros(1, device="cuda")
+        losses = []
+        for k, batch in enumerate((4096, 1000, 300)):
+            idx = W.minibatch_indices(6, k, n, batch)
+            r.train(batch, torch.from_numpy(idx).cuda(), opt="adam", lr=1e-3, loss_out=loss)
+            losses.append(loss.item())
+        r.train(2048, None, opt="adam", lr=1e-3, loss_out=loss)  # sequential slots
+        losses.append(loss.item())
+        m, v, t = r.get_opt_state()
+        out.append((r.get_params().cpu(), m.cpu(), v.cpu(), t, losses))
+        assert r.sync() == L.LS_OK
+        r.close()
+    (p0, m0, v0, t0, l0), (p1, m1, v1, t1, l1) = out
+    assert t0 == t1 == 4 and l0 == l1
+    assert torch.equal(p0, p1) and torch.equal(m0, m1) and torch.equal(v0, v1)
+
+
 def test_train_gradient_bf16_via_sgd():
     # SGD with lr 0.1 exposes the bf16 gradient as (w - w') / 0.1.
     cfg = W.CONFIGS["training"]
