@@ -280,6 +280,7 @@ def measure_training_config(L, H, W, dev, steps=1000):
            "best": torch.empty(cfg.n_req, device=dev), "scores": None, "hits": None}
     sa, sb = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
     loss = torch.zeros(1, device=dev)
+    torch.cuda.synchronize()  # the two streams start after the setup above (snapshot, log)
 
     def run(n):
         for k in range(n):
@@ -698,7 +699,21 @@ def main():
     L.ls_trace_read(r.h)
     torch.cuda.synchronize()
     n_traced = min(args.steps, 120)                 # every launch gets events from the tracer's pool
-    traced_times = timed_pass(eager_step, 2 * args.warmup + 2 * args.steps, n_traced)
+
+    # each traced step behind a ~150 us spin on the GPU, so that the host has
+    # queued the whole step before it starts and no kernel interval includes
+    # host time; the step's interval excludes the spin
+    tev = []
+    for k in range(n_traced):
+        torch.cuda._sleep(300000)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        eager_step(2 * args.warmup + 2 * args.steps + k)
+        e1.record(stream)
+        tev.append((e0, e1))
+    torch.cuda.synchronize()
+    traced_times = [a.elapsed_time(b) for a, b in tev]
     torch.cuda.synchronize()
     rc, trace = L.ls_trace_read(r.h)
     L.ls_trace_enable(r.h, False)

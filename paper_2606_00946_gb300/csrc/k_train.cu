@@ -104,8 +104,8 @@ __global__ void __launch_bounds__(256) k_gemm(GemmArgs g) {
 
 // Minibatch rows: slot = idx[j] (checked against the filled part of the ring)
 // or (step*B + j) mod valid, with step and the ring's fill read from the device
-// state; z-score in fp32, bf16-rounded in bf16 mode.  An empty ring latches
-// LS_ERR_STATE (rows then come from slot 0).
+// state; z-score in fp32, bf16-rounded in bf16 mode.  An empty buffer latches
+// LS_ERR_STATE and reads nothing (the rows are zero).
 __global__ void k_train_gather(int B, int d, const int32_t* __restrict__ idx, DevState* st,
                                int64_t capacity, int64_t replay_base, const float* __restrict__ ring_x,
                                const float* __restrict__ ring_y, const float* __restrict__ mean,
@@ -130,6 +130,11 @@ __global__ void k_train_gather(int B, int d, const int32_t* __restrict__ idx, De
       }
     } else {
       slot = valid > 0 ? (step * (int64_t)B + j) % valid : 0;
+    }
+    if (valid < 1) {  // nothing logged yet: no row to read
+      x0[e] = 0.0f;
+      if (k == 0) y[j] = 0.0f;
+      continue;
     }
     slot = union_row(slot, nF, replay_base);
     const float v = zscore(ring_x[slot * d + k], mean[k], stdv[k]);

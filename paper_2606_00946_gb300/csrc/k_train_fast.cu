@@ -209,6 +209,12 @@ __device__ __forceinline__ bool tr_tile(const TrArgs& args, int bid, uint8_t* sm
 
   const int q = warp & 3, cq = warp >> 2;
   const int r = 32 * q + lane, j = m0 + r;
+  // the epilogues stage their image tiles in the (now free) operand stages,
+  // in the images' own byte layout: the row-major tile [128 rows x NT] as
+  // NT / 64 runs of 16 KB, the transposed tile [NT rows x 128] as two runs of
+  // NT x 128 bytes; bulk copies then write each run with one instruction
+  uint8_t* S1 = smem;
+  uint8_t* S2 = smem + 65536;
   const int cw = NT / 4, cbeg = cq * cw;  // this warp's columns (CTA-local)
   const uint32_t lane_addr = (uint32_t)(32 * q) << 16;
 
@@ -256,8 +262,8 @@ __device__ __forceinline__ bool tr_tile(const TrArgs& args, int bid, uint8_t* sm
         a[u] = round_bf16(r);
       }
       J.mask_out[(int64_t)((n0 + c) >> 4) * J.rows_pad + j] = (uint16_t)bits;
-      store_row16(J.out, J.rows_pad, j, n0 + c, a);
-      store_col16(J.outT, J.rT, j, n0 + c, a);
+      store_row16(S1, kM, r, c, a);
+      store_col16(S2, NT, r, c, a);
     }
   } else if (ok && J.epi == TE_DX) {
     for (int c = cbeg; c < cbeg + cw; c += 16) {
@@ -269,8 +275,8 @@ __device__ __forceinline__ bool tr_tile(const TrArgs& args, int bid, uint8_t* sm
       const float sc = J.drop_h > 0 ? args.drop_scale : 1.0f;
 #pragma unroll
       for (int u = 0; u < 16; ++u) dz[u] = ((bits >> u) & 1u) ? __uint_as_float(v[u]) * sc : 0.0f;
-      if (J.out) store_row16(J.out, J.rows_pad, j, n0 + c, dz);
-      store_col16(J.outT, J.rT, j, n0 + c, dz);
+      if (J.out) store_row16(S1, kM, r, c, dz);
+      store_col16(S2, NT, r, c, dz);
       const float sb = col_reduce16(dz);
       if (lane < 16) red[q * 256 + c + lane] = sb;
     }
@@ -354,8 +360,8 @@ __device__ __forceinline__ bool tr_tile(const TrArgs& args, int bid, uint8_t* sm
           pw[u] = rd * round_bf16(pos ? z : 0.0f);
           dz[u] = pos ? rd * s_w[c + u] : 0.0f;
         }
-        if (J.out) store_row16(J.out, J.rows_pad, j, n0 + c, dz);
-        store_col16(J.outT, J.rT, j, n0 + c, dz);
+        if (J.out) store_row16(S1, kM, r, c, dz);
+        store_col16(S2, NT, r, c, dz);
         const float sw = col_reduce16(pw);
         if (lane < 16) red2[q * 256 + c + lane] = sw;
         const float sb = col_reduce16(dz);
@@ -372,6 +378,19 @@ __device__ __forceinline__ bool tr_tile(const TrArgs& args, int bid, uint8_t* sm
         J.partLoss[mt] = ((wsum[0] + wsum[1]) + wsum[2]) + wsum[3];
         J.partBL[mt] = ((wsum[4] + wsum[5]) + wsum[6]) + wsum[7];
       }
+    }
+  }
+  if (ok && (J.epi == TE_FWD || J.epi == TE_DX || J.epi == TE_FWD_OUT)) {
+    fence_async_smem();  // staged tiles are read by the bulk copies (async proxy)
+    __syncthreads();
+    if (tid == 0) {
+      if (J.out)
+        for (int kb = 0; kb < NT / 64; ++kb)
+          bulk_s2g(J.out + ((int64_t)(n0 / 64 + kb) * J.rows_pad + m0) * 128, S1 + (size_t)kb * kM * 128, kM * 128);
+      for (int h = 0; h < kM / 64; ++h)
+        bulk_s2g(J.outT + ((int64_t)(m0 / 64 + h) * J.rT + n0) * 128, S2 + (size_t)h * NT * 128,
+                 (uint32_t)NT * 128);
+      bulk_commit_wait_all();  // before the stages are reused or the CTA exits
     }
   }
   tc_fence_before();
@@ -454,7 +473,7 @@ __device__ __forceinline__ void tr_gather_items(const GatherArgs& g, int64_t fir
     float v[8];
 #pragma unroll
     for (int u = 0; u < 8; ++u) v[u] = 0.0f;
-    if (j < B) {
+    if (j < B && valid > 0) {  // an empty buffer (error latched above) reads nothing: zero rows
       int64_t slot;
       if (idx) {
         slot = idx[j];
@@ -471,6 +490,8 @@ __device__ __forceinline__ void tr_gather_items(const GatherArgs& g, int64_t fir
       for (int u = 0; u < 8; ++u)
         if (c0 + u < d) v[u] = round_bf16(zscore(__ldg(row + c0 + u), __ldg(mean + c0 + u), __ldg(stdv + c0 + u)));
       if (c0 == 0) y[j] = ring_y[slot];
+    } else if (j < B && c0 == 0) {
+      y[j] = 0.0f;
     }
     uint4 qv;
     qv.x = pack2(v[0], v[1]);

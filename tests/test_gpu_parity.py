@@ -460,6 +460,25 @@ def test_persistent_train_step_same_bits(cfg_name, dropout):
     assert torch.equal(p0, p1) and torch.equal(m0, m1) and torch.equal(v0, v1)
 
 
+@pytest.mark.parametrize("cfg_name", ["tiny", "training"])
+def test_train_on_empty_buffer_is_a_state_error(cfg_name):
+    # Nothing logged yet: the call is refused with LS_ERR_STATE (tensor-core
+    # path for the bf16 config, plain path for the fp32 one).  A step that
+    # still finds the buffer empty on the device (records logged on another,
+    # unordered stream) latches the same error and reads no record.
+    cfg = W.CONFIGS[cfg_name]
+    params = W.xavier_params(cfg.widths, 1)
+    mean, std = W.normaliser(np.random.default_rng(2), cfg)
+    r = _train_router(cfg, 1024)
+    r.set_normalizer(torch.from_numpy(mean).cuda(), torch.from_numpy(std).cuda())
+    r.set_params(torch.from_numpy(params).cuda())
+    with pytest.raises(L.LodestarError) as e:
+        r.train(256, None, opt="adam", lr=1e-3)
+    assert e.value.code == L.LS_ERR_STATE
+    assert r.sync() == L.LS_OK
+    r.close()
+
+
 def test_train_gradient_bf16_via_sgd():
     # SGD with lr 0.1 exposes the bf16 gradient as (w - w') / 0.1.
     cfg = W.CONFIGS["training"]
