@@ -32,6 +32,9 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 WORKLOAD = "homogeneous"
+WORKLOAD_DESC = (f"{WORKLOAD}: 32 instances x 4096 requests/step, prompts 64-4096 tokens with Zipf(1.1) "
+                 "prefixes over 256 templates, 16384 cached blocks/instance, bf16 MLP 64-256-256-1, "
+                 "Adam batch 4096")
 INPUT_SETS = 6   # device copies of the batch the timed steps rotate over (> L2 together)
 METRIC = "routing decisions/sec (requests routed per second of whole route+log+train+publish steps)"
 UNIT = "decisions/s"
@@ -544,8 +547,8 @@ def run_reference(args, world, rank):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic (seeded generator shaped like the paper's prefix-sharing workloads)",
-            "config": {"workload": f"{WORKLOAD}: 32 instances x 4096 requests, bf16 MLP 64-256-256-1",
-                       "sample_requests_per_step": n},
+            "config": {"workload": WORKLOAD_DESC, "pairs_per_step": 32 * 4096, "train_samples_per_step": 4096,
+                       "parallelism": "replicas", "sample_requests_per_step": n},
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
                              "sample": f"{n} requests over {cores} host threads + one Adam step on {n} records "
                                        f"per step"},
@@ -902,9 +905,7 @@ def main():
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic (seeded generator shaped like the paper's prefix-sharing workloads)",
-            "config": {"workload": f"{WORKLOAD}: 32 instances x 4096 requests/step, prompts 64-4096 "
-                                   "tokens with Zipf(1.1) prefixes over 256 templates, 16384 cached "
-                                   "blocks/instance, bf16 MLP 64-256-256-1, Adam batch 4096",
+            "config": {"workload": WORKLOAD_DESC,
                        "pairs_per_step": R * N, "train_samples_per_step": Bt,
                        "l2": f"inputs larger than L2: consecutive steps read {n_sets} rotating device copies of "
                              f"the batch ({n_sets * set_bytes / 1e6:.0f} MB in all, L2 129 MB); no flush",
