@@ -411,7 +411,12 @@ int ls_set_opt_state(ls_ctx* h, const float* m, const float* v, int64_t step, vo
   LS_CK(cudaMemcpyAsync(c.adam_m, m, n, cudaMemcpyDeviceToDevice, S(stream)));
   LS_CK(cudaMemcpyAsync(c.adam_v, v, n, cudaMemcpyDeviceToDevice, S(stream)));
   const int64_t st_step = step;
-  const double pw[2] = {std::pow(0.9, (double)step), std::pow(0.999, (double)step)};
+  // the running powers exactly as the device forms them, one multiply per step
+  double pw[2] = {1.0, 1.0};
+  for (int64_t t = 0; t < step; ++t) {
+    pw[0] *= 0.9;
+    pw[1] *= 0.999;
+  }
   LS_CK(cudaMemcpyAsync(&c.st->step, &st_step, sizeof(int64_t), cudaMemcpyHostToDevice, S(stream)));
   LS_CK(cudaMemcpyAsync(c.st->beta_pow, pw, sizeof(pw), cudaMemcpyHostToDevice, S(stream)));
   LS_CK(cudaStreamSynchronize(S(stream)));

@@ -30,6 +30,7 @@ class Router:
         rc, h = L.ls_create(self.cfg)
         L.check(rc)
         self.h = h
+        self._norm = None
         self.widths = list(widths)
         self.dtype = dtype
         self.n_params = L.ls_param_count(self.cfg)
@@ -78,8 +79,32 @@ class Router:
         L.check(rc)
         return m, v, step
 
+    def set_opt_state(self, m, v, step, stream=None):
+        L.check(L.ls_set_opt_state(self.h, m, v, int(step), stream))
+
     def set_normalizer(self, mean, std, stream=None):
         L.check(L.ls_set_normalizer(self.h, mean, std, stream))
+        self._norm = (mean.detach().clone(), std.detach().clone())
+
+    def save_checkpoint(self, path):
+        """Master weights, Adam moments, step count and normaliser to an .npz."""
+        if self._norm is None:
+            raise ValueError("set_normalizer has not been called")
+        m, v, step = self.get_opt_state()
+        mean, std = self._norm
+        np.savez(path, params=self.get_params().cpu().numpy(), m=m.cpu().numpy(), v=v.cpu().numpy(),
+                 step=np.int64(step), mean=mean.cpu().numpy(), std=std.cpu().numpy())
+
+    def load_checkpoint(self, path, publish=True):
+        """Restore what save_checkpoint wrote; the next training step continues
+        the saved run (same bits, given the same records and minibatch)."""
+        z = np.load(path)
+        t = lambda a: torch.from_numpy(np.ascontiguousarray(a)).cuda()
+        self.set_normalizer(t(z["mean"]), t(z["std"]))
+        self.set_params(t(z["params"]))
+        self.set_opt_state(t(z["m"]), t(z["v"]), int(z["step"]))
+        if publish:
+            self.publish()
 
     def snapshot(self, n_inst, inst_state, keys=None, key_off=None, mode=L.LS_REPLACE, stream=None):
         n_keys = int(keys.numel()) if keys is not None else 0
