@@ -446,24 +446,34 @@ KERNEL_SOURCES = {"score_tc": ("k_score_tc.cu", "sm100.cuh"),
                   "prefix_index": ("k_prefix_index.cu", "blockhash.cuh")}
 
 
+def code_digest(files):
+    """Hash of the code of the given sources (comments and whitespace removed,
+    so that an edit of a comment keeps a capture of the same code valid)."""
+    import hashlib
+    import re
+    src = os.path.join(ROOT, "paper_2606_00946_gb300", "csrc")
+    h = hashlib.sha256()
+    for f in files:
+        with open(os.path.join(src, f)) as fh:
+            text = fh.read()
+        text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+        text = re.sub(r"//[^\n]*", " ", text)
+        h.update(" ".join(text.split()).encode())
+    return h.hexdigest()[:16]
+
+
 def profiled_traffic(kernel):
     """DRAM bytes per launch of `kernel` from the committed ncu summaries, if the
     summary was taken on the kernel's current source (else None)."""
     import glob
-    import hashlib
     if kernel not in KERNEL_SOURCES:
         return None
-    src = os.path.join(ROOT, "paper_2606_00946_gb300", "csrc")
-    h = hashlib.sha256()
-    for f in KERNEL_SOURCES[kernel]:
-        with open(os.path.join(src, f), "rb") as fh:
-            h.update(fh.read())
-    sha = h.hexdigest()[:16]
+    sha = code_digest(KERNEL_SOURCES[kernel])
     for path in glob.glob(os.path.join(ROOT, "profiles", "*.md")):
         for line in open(path):
             if line.startswith("roofline-traffic:"):
                 kv = dict(p.split("=", 1) for p in line.split()[1:])
-                if kv.get("kernel") == kernel and kv.get("source_sha256") == sha:
+                if kv.get("kernel") == kernel and kv.get("code_sha256") == sha:
                     return float(kv["bytes_per_launch"])
     return None
 

@@ -340,17 +340,19 @@ __device__ __forceinline__ uint64_t out_dot16(const uint32_t (&v)[16], uint4 w0,
 }
 
 // Pipelined variant for predictors with two hidden layers whose weights stay
-// resident (widths <= 256): warp 0 issues the MMAs, warps 1-7 build feature
-// tiles into two buffers ahead of time, warps 8-15 run the epilogues.  Layer-1
-// activations go to the layer-2 MMA through a two-slot ring of 64-column
-// K-blocks, so the layer-2 MMA of a tile runs while its layer-1 epilogue is
-// still producing K-blocks; D1 and D2 sit in separate TMEM halves, so the final
-// epilogue of tile t overlaps the layer-1 MMA of tile t+1.
+// resident (widths <= 256), one persistent CTA per SM over 128-row tiles of
+// the feature image.  Layer-1 activations go to the layer-2 MMA through a
+// two-slot ring of 64-column K-blocks, so the layer-2 MMA of a tile runs while
+// its layer-1 epilogue is still producing K-blocks; D1 and D2 sit in separate
+// TMEM halves, so the output epilogue of tile t overlaps the layer-1 MMA and
+// epilogue of tile t+1.  Each layer's accumulator starts from its bias (one
+// K = 16 product), so the epilogues read no bias.
 // ---------------------------------------------------------------------------
-// Warp roles: 0 = MMA issuer, 1 = feature-tile loader (one bulk copy per
-// tile from the feature image), 2..9 = layer-1 epilogue (E1), 10..17 =
-// layer-2 + output epilogue (E2).  E1 of tile t+1 runs while E2 finishes tile
-// t.  18 warps = at most 5 per SM sub-partition: 96 registers per thread.
+// Warp roles: 0 = MMA issuer (thread 0 also requests the weights and the
+// first feature tile at the start), 1 = feature-tile loader (one bulk copy
+// per later tile), 2..9 = layer-1 epilogue (E1), 10..17 = layer-2 + output
+// epilogue (E2).  18 warps = at most 5 per SM sub-partition: 96 registers per
+// thread at most.
 constexpr int kEpiWarps = 8, kEpiThreads = kEpiWarps * 32;
 constexpr int kE1Warp0 = 2, kE2Warp0 = kE1Warp0 + kEpiWarps;
 constexpr int kThreadsPipe = (kE2Warp0 + kEpiWarps) * 32;  // 576
