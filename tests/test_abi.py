@@ -89,3 +89,28 @@ def test_prefix_index_mode_needs_at_most_512_instances(lib):
     c = _cfg(max_instances=600, prefix_mode="index")
     rc, h = L.ls_create(c)
     assert rc == L.LS_ERR_ARG and "512" in L.last_error()
+
+
+@pytest.mark.parametrize("struct", [L.ls_config, L.ls_info, L.ls_guards])
+def test_struct_layouts_match_the_header(struct, tmp_path):
+    # sizeof and every field offset as gcc lays out the header's struct, against
+    # the ctypes binding (a field added on one side only would shift the rest)
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    name = struct.__name__
+    lines = [f'printf("size %zu\\n", sizeof({name}));']
+    for f, _ in struct._fields_:
+        lines.append(f'printf("{f} %zu\\n", offsetof({name}, {f}));')
+    src = tmp_path / "layout.c"
+    src.write_text('#include <stddef.h>\n#include <stdio.h>\n#include "lodestar.h"\nint main(void) {\n  '
+                   + "\n  ".join(lines) + "\n  return 0;\n}\n")
+    exe = tmp_path / "layout"
+    subprocess.run([cc, "-I", os.path.dirname(HEADER), str(src), "-o", str(exe)], check=True)
+    got = dict(line.split() for line in subprocess.run([str(exe)], capture_output=True, text=True,
+                                                          check=True).stdout.splitlines())
+    assert int(got["size"]) == C.sizeof(struct)
+    for f, _ in struct._fields_:
+        assert int(got[f]) == getattr(struct, f).offset, f
