@@ -245,8 +245,10 @@ int ls_log_samples(ls_ctx *ctx, int32_t n, const float *feats, const float *ttft
  * u - nF (nF = min(count, ring_capacity), nR = records in the replay pool,
  * 0 without one).  idx [batch] int32 on the device; NULL = indices
  * (k*batch + j) mod (nF + nR) at step k; k, count and nR are the device
- * counters when the step runs; an empty buffer at that point latches
- * LS_ERR_STATE).
+ * counters when the step runs.  A step before any ls_log_samples call is
+ * refused with LS_ERR_STATE; a step that still finds the buffer empty on the
+ * device (records logged on another stream it is not ordered after) latches
+ * LS_ERR_STATE and reads no record (its rows and targets are zero).
  * Loss = mean squared error of the predicted TTFT (seconds).  opt LS_SGD:
  * theta -= lr g; LS_ADAM: beta1 0.9, beta2 0.999, eps 1e-8, bias-corrected.
  * Updates the master weights only; routing sees them after ls_publish.
