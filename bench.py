@@ -928,9 +928,11 @@ def main():
             "cpu_baseline": cpu,
             "e2e": e2e,
             "gpu_launches": launches,
-            "launch": "each step: inputs copied into the step's buffers, then one replay of a CUDA graph "
-                      "of the step's ABI calls recorded once: snapshot + route on one branch, log + train "
-                      "on a second, joined before the publish",
+            "launch": "each step: the new instance state and records copied into the step's buffers, then "
+                      "one replay of a CUDA graph of the step's ABI calls recorded once per device copy of the "
+                      "batch (steps rotate over the copies): snapshot + route on one branch, log + train on a "
+                      "second, joined before the publish; kernels of each chain launched with programmatic "
+                      "dependent launch",
             "ms_per_step_eager": float(np.mean(eager_times)),
             "ms_per_step_instrumented": float(np.mean(traced_times)),
             "instrumented_steps": n_traced,
