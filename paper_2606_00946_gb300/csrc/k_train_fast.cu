@@ -638,7 +638,7 @@ __global__ void __launch_bounds__(256) k_tr_opt(const __grid_constant__ OptArgs 
 // every sum as the launch-per-phase path, so the same bits.
 // ---------------------------------------------------------------------------
 constexpr int kMaxPhases = 2 * (LS_MAX_LAYERS - 1);
-constexpr uint32_t kGridSpin = 1u << 21;  // barrier polls before giving up (~0.2 s)
+constexpr uint32_t kGridSpin = 1u << 21;  // barrier polls before giving up (a second or so)
 
 struct StepArgs {
   GatherArgs g;
