@@ -246,15 +246,17 @@ int ls_log_samples(ls_ctx *ctx, int32_t n, const float *feats, const float *ttft
  * 0 without one).  idx [batch] int32 on the device; NULL = indices
  * (k*batch + j) mod (nF + nR) at step k; k, count and nR are the device
  * counters when the step runs.  A step before any ls_log_samples call is
- * refused with LS_ERR_STATE; a step that still finds the buffer empty on the
+ * refused with LS_ERR_STATE.  A step that still finds the buffer empty on the
  * device (records logged on another stream it is not ordered after) latches
- * LS_ERR_STATE and reads no record (its rows and targets are zero).
+ * LS_ERR_STATE, and a step with an idx entry outside the filled buffer
+ * latches LS_ERR_ARG; such a step reads no record past the buffer and changes
+ * nothing: master weights, Adam moments and the step count stay as they
+ * were, and *loss_out receives NaN.
  * Loss = mean squared error of the predicted TTFT (seconds).  opt LS_SGD:
  * theta -= lr g; LS_ADAM: beta1 0.9, beta2 0.999, eps 1e-8, bias-corrected.
  * Updates the master weights only; routing sees them after ls_publish.
  * loss_out: device float (nullable) receives the minibatch loss before the
- * update.  An idx entry outside the filled part of the ring latches
- * LS_ERR_ARG and is read as slot 0. */
+ * update. */
 int ls_train_step(ls_ctx *ctx, int32_t batch, const int32_t *idx, int32_t opt, float lr,
                   float *loss_out, void *stream);
 

@@ -81,6 +81,9 @@ struct DevState {
   double beta_pow[2];       // beta1^step, beta2^step (fp64 running products)
   int64_t replay_count;     // records in the replay pool
   int64_t admitted;         // evicted stream positions below this were considered for the replay pool
+  int32_t train_abort;      // set by a training step's gather (empty buffer, bad slot): the step's
+                            // optimiser changes nothing and clears it
+  int32_t pad_;
 };
 
 // Row of training-buffer index u (Sec. 4.3.2: a round trains on F u R): ring

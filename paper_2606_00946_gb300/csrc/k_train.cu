@@ -115,7 +115,10 @@ __global__ void k_train_gather(int B, int d, const int32_t* __restrict__ idx, De
   const int64_t count = st->ring_count;
   const int64_t nF = count < capacity ? count : capacity;
   const int64_t valid = nF + st->replay_count;  // F u R
-  if (valid < 1 && blockIdx.x == 0 && threadIdx.x == 0) latch_error(err, LS_ERR_STATE);
+  if (valid < 1 && blockIdx.x == 0 && threadIdx.x == 0) {
+    latch_error(err, LS_ERR_STATE);
+    st->train_abort = 1;  // the optimiser of this step leaves every parameter as it is
+  }
   if (blockIdx.x == 0 && threadIdx.x == 0) set_adam_bc(st);
   const int64_t total = (int64_t)B * d;
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
@@ -125,7 +128,10 @@ __global__ void k_train_gather(int B, int d, const int32_t* __restrict__ idx, De
     if (idx) {
       slot = idx[j];
       if (slot < 0 || slot >= valid) {
-        if (k == 0) latch_error(err, LS_ERR_ARG);
+        if (k == 0) {
+          latch_error(err, LS_ERR_ARG);
+          st->train_abort = 1;
+        }
         slot = 0;
       }
     } else {
@@ -146,7 +152,8 @@ __global__ void k_train_gather(int B, int d, const int32_t* __restrict__ idx, De
 // dZ_L = 2 (yhat - y) / B and loss = mean (yhat - y)^2, one CTA (fixed order).
 __global__ void __launch_bounds__(1024) k_loss_grad(int B, const float* __restrict__ yhat,
                                                     const float* __restrict__ y,
-                                                    float* __restrict__ dz, float* loss_out) {
+                                                    float* __restrict__ dz, float* loss_out,
+                                                    const DevState* st) {
   __shared__ float part[32];
   float s = 0.0f;
   for (int j = threadIdx.x; j < B; j += blockDim.x) {
@@ -162,7 +169,7 @@ __global__ void __launch_bounds__(1024) k_loss_grad(int B, const float* __restri
     float t = threadIdx.x < (blockDim.x >> 5) ? part[threadIdx.x] : 0.0f;
 #pragma unroll
     for (int o = 16; o; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
-    if (threadIdx.x == 0 && loss_out) *loss_out = t / (float)B;
+    if (threadIdx.x == 0 && loss_out) *loss_out = st->train_abort ? __int_as_float(0x7fc00000) : t / (float)B;
   }
 }
 
@@ -261,14 +268,25 @@ __global__ void k_reduce_partials(int S, int64_t n, const float* __restrict__ pa
   }
 }
 
+// The optimiser's last block, once every block has read the step counter and
+// the abort flag: advance the step unless the gather aborted it, then clear
+// the flag for the next step.
+__device__ __forceinline__ void finish_step(DevState* st, int64_t t, bool aborted) {
+  if (!aborted) advance_step(st, t);
+  st->train_abort = 0;
+}
+
 // Optimiser updates.  Each advances the device step counter once (last block),
-// after every block has read it.
+// after every block has read it.  A step whose gather found no record or a bad
+// slot changes nothing.
 __global__ void k_sgd(int64_t n, float lr, const float* __restrict__ g, float* __restrict__ p, DevState* st) {
   const int64_t t = st->step + 1;
-  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n;
-       e += (int64_t)gridDim.x * blockDim.x)
-    p[e] = p[e] - lr * g[e];
-  if (last_block(&st->done[DONE_OPT]) && threadIdx.x == 0) advance_step(st, t);
+  const bool aborted = st->train_abort != 0;
+  if (!aborted)
+    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n;
+         e += (int64_t)gridDim.x * blockDim.x)
+      p[e] = p[e] - lr * g[e];
+  if (last_block(&st->done[DONE_OPT]) && threadIdx.x == 0) finish_step(st, t, aborted);
 }
 
 // Adam, t = steps taken + 1: bias corrections 1 - beta^t formed in fp64 by
@@ -277,7 +295,8 @@ __global__ void k_adam(int64_t n, float lr, const float* __restrict__ g, float* 
                        float* __restrict__ m, float* __restrict__ v, DevState* st) {
   const int64_t t = st->step + 1;
   const float bc1 = st->adam_bc[0], bc2 = st->adam_bc[1];
-  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n;
+  const bool aborted = st->train_abort != 0;
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; !aborted && e < n;
        e += (int64_t)gridDim.x * blockDim.x) {
     const float ge = g[e];
     const float me = 0.9f * m[e] + 0.1f * ge;
@@ -287,7 +306,7 @@ __global__ void k_adam(int64_t n, float lr, const float* __restrict__ g, float* 
     const float mh = me / bc1, vh = ve / bc2;
     p[e] = p[e] - lr * mh / (sqrtf(vh) + 1e-8f);
   }
-  if (last_block(&st->done[DONE_OPT]) && threadIdx.x == 0) advance_step(st, t);
+  if (last_block(&st->done[DONE_OPT]) && threadIdx.x == 0) finish_step(st, t, aborted);
 }
 
 template <bool TA, bool TB, int EPI>
@@ -386,7 +405,7 @@ cudaError_t run_train_step(Ctx& c, int B, const int32_t* idx, int opt, float lr,
   if (e != cudaSuccess) return e;
   e = traced(c, TR_LOSS, 1, s, [&] {
     k_loss_grad<<<1, 1024, 0, s>>>(B, c.tz + zoff[L - 1], c.ty, c.dz0,
-                                   loss_out ? loss_out : c.loss_tmp);
+                                   loss_out ? loss_out : c.loss_tmp, c.st);
     return cudaGetLastError();
   });
   if (e != cudaSuccess) return e;

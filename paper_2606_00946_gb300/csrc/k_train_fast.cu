@@ -465,7 +465,10 @@ __device__ __forceinline__ void tr_gather_items(const GatherArgs& g, int64_t fir
   const int64_t nF = count < g.capacity ? count : g.capacity;
   const int64_t valid = nF + st->replay_count;  // F u R
   const int64_t replay_base = g.replay_base;
-  if (valid < 1 && lead) latch_error(err, LS_ERR_STATE);
+  if (valid < 1 && lead) {
+    latch_error(err, LS_ERR_STATE);
+    st->train_abort = 1;  // the optimiser of this step leaves every parameter as it is
+  }
   if (lead) set_adam_bc(st);
   const int64_t total = (int64_t)rows_pad * (d_pad / 8);
   for (int64_t e = first; e < total; e += stride) {
@@ -478,7 +481,10 @@ __device__ __forceinline__ void tr_gather_items(const GatherArgs& g, int64_t fir
       if (idx) {
         slot = idx[j];
         if (slot < 0 || slot >= valid) {
-          if (c0 == 0) latch_error(err, LS_ERR_ARG);
+          if (c0 == 0) {
+            latch_error(err, LS_ERR_ARG);
+            st->train_abort = 1;
+          }
           slot = 0;
         }
       } else {
@@ -557,6 +563,9 @@ struct OptArgs {
 // optimiser update of the fp32 master, and the bf16 images of the updated
 // hidden-layer weights, for parameters [first, n) with stride `stride`.
 __device__ __forceinline__ void tr_opt_items(const OptArgs& a, int64_t first, int64_t stride) {
+  // a step whose gather found no record or a bad slot changes nothing (the
+  // images already hold the unchanged weights)
+  if (a.mode != 0 && a.st->train_abort) return;
   const float bc1 = a.st->adam_bc[0], bc2 = a.st->adam_bc[1];  // set by the gather kernel
   const MlpDesc& m = a.m;
   const int nl = m.n_layers;
@@ -617,7 +626,7 @@ __device__ __forceinline__ void tr_loss(const OptArgs& a) {
   if (a.mode != 0 && a.loss_out) {
     float s = 0.0f;
     for (int tt = 0; tt < a.T; ++tt) s += a.partLoss[tt];
-    *a.loss_out = s / (float)a.B;
+    *a.loss_out = a.st->train_abort ? __int_as_float(0x7fc00000) : s / (float)a.B;
   }
 }
 
@@ -625,9 +634,14 @@ __global__ void __launch_bounds__(256) k_tr_opt(const __grid_constant__ OptArgs 
   pdl_wait();  // gradient partials from the previous kernels of the stream
   pdl_trigger();
   const int64_t t = a.st->step + 1;
+  const bool aborted = a.mode != 0 && a.st->train_abort != 0;
   tr_opt_items(a, blockIdx.x * (int64_t)blockDim.x + threadIdx.x, (int64_t)gridDim.x * blockDim.x);
   if (blockIdx.x == 0 && threadIdx.x == 0) tr_loss(a);
-  if (a.mode != 0 && last_block(&a.st->done[DONE_OPT]) && threadIdx.x == 0) advance_step(a.st, t);
+  // the last block, once every block has read the counter and the flag
+  if (a.mode != 0 && last_block(&a.st->done[DONE_OPT]) && threadIdx.x == 0) {
+    if (!aborted) advance_step(a.st, t);
+    a.st->train_abort = 0;
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -726,7 +740,10 @@ __global__ void __launch_bounds__(kT, 1) k_tr_step(const __grid_constant__ StepA
     tr_opt_items(a.opt, first, stride);
     if (tr_grid_sync(a.bar, ++arrivals * gridDim.x, err) && blockIdx.x == 0 && tid == 0) {
       tr_loss(a.opt);
-      if (a.opt.mode != 0) advance_step(a.opt.st, a.opt.st->step + 1);
+      if (a.opt.mode != 0) {
+        if (!a.opt.st->train_abort) advance_step(a.opt.st, a.opt.st->step + 1);
+        a.opt.st->train_abort = 0;
+      }
     }
   }
   tc_fence_before();

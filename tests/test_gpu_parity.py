@@ -479,6 +479,86 @@ def test_train_on_empty_buffer_is_a_state_error(cfg_name):
     r.close()
 
 
+def _train_state(r):
+    m, v, t = r.get_opt_state()
+    return r.get_params().cpu(), m.cpu(), v.cpu(), t
+
+
+@pytest.mark.parametrize("cfg_name,train_ctas", [("tiny", 0), ("training", 0), ("training", 24)])
+def test_step_that_finds_no_record_changes_nothing(cfg_name, train_ctas):
+    # Records logged on a stream the training step is not ordered after: the
+    # log waits behind a ~0.2 s spin on its own stream, so the step runs first
+    # and finds the buffer empty on the device.  It latches LS_ERR_STATE, its
+    # loss is NaN, and parameters, Adam moments and the step count are left as
+    # they were (bit for bit); the next, ordered step then trains normally.
+    cfg = W.CONFIGS[cfg_name]
+    rng = np.random.default_rng(21)
+    x, y = W.records(rng, cfg, 512)
+    params = W.xavier_params(cfg.widths, 1)
+    mean, std = W.normaliser(np.random.default_rng(2), cfg)
+    r = H.Router(cfg.widths, cfg.d_inst, cfg.d_req, cfg.dtype, max_instances=4, max_requests=16,
+                 max_keys_per_instance=64, ring_capacity=1024, max_train_batch=4096, train_ctas=train_ctas)
+    r.set_normalizer(torch.from_numpy(mean).cuda(), torch.from_numpy(std).cuda())
+    r.set_params(torch.from_numpy(params).cuda())
+    xs, ys = torch.from_numpy(x).cuda(), torch.from_numpy(y).cuda()
+    # one Adam step on a second context's state would differ; take this one's
+    # state after a first, ordered step so that the moments are nonzero
+    r.log(xs[:256], ys[:256])
+    loss = torch.zeros(1, device="cuda")
+    r.train(256, None, opt="adam", lr=1e-3, loss_out=loss)
+    assert r.sync() == L.LS_OK
+    before = _train_state(r)
+    r2 = H.Router(cfg.widths, cfg.d_inst, cfg.d_req, cfg.dtype, max_instances=4, max_requests=16,
+                  max_keys_per_instance=64, ring_capacity=1024, max_train_batch=4096, train_ctas=train_ctas)
+    r2.set_normalizer(torch.from_numpy(mean).cuda(), torch.from_numpy(std).cuda())
+    r2.set_params(before[0].cuda())
+    r2.set_opt_state(before[1].cuda(), before[2].cuda(), before[3])
+    b2 = _train_state(r2)
+    torch.cuda.synchronize()
+    side, main = torch.cuda.Stream(), torch.cuda.Stream()
+    with torch.cuda.stream(side):
+        torch.cuda._sleep(400_000_000)          # ~0.2 s at 2 GHz, bounded
+        r2.log(xs[256:], ys[256:], stream=side)
+    r2.train(256, None, opt="adam", lr=1e-3, loss_out=loss, stream=main)
+    main.synchronize()
+    assert np.isnan(loss.item())
+    assert r2.sync() == L.LS_ERR_STATE
+    after = _train_state(r2)
+    assert torch.equal(after[0], b2[0]) and torch.equal(after[1], b2[1]) and torch.equal(after[2], b2[2])
+    assert after[3] == b2[3]
+    # ordered now: the step trains and counts
+    r2.train(256, None, opt="adam", lr=1e-3, loss_out=loss)
+    assert np.isfinite(loss.item()) and r2.sync() == L.LS_OK
+    assert _train_state(r2)[3] == b2[3] + 1 and not torch.equal(_train_state(r2)[0], b2[0])
+    r.close()
+    r2.close()
+
+
+@pytest.mark.parametrize("cfg_name", ["tiny", "training"])
+def test_step_with_bad_slot_changes_nothing(cfg_name):
+    # A minibatch slot outside the filled buffer latches LS_ERR_ARG and the
+    # step changes nothing (parameters, moments, step count; loss NaN).
+    cfg = W.CONFIGS[cfg_name]
+    x, y = W.records(np.random.default_rng(22), cfg, 300)
+    mean, std = W.normaliser(np.random.default_rng(2), cfg)
+    r = _train_router(cfg, 1024)
+    r.set_normalizer(torch.from_numpy(mean).cuda(), torch.from_numpy(std).cuda())
+    r.set_params(torch.from_numpy(W.xavier_params(cfg.widths, 3)).cuda())
+    r.log(torch.from_numpy(x).cuda(), torch.from_numpy(y).cuda())
+    loss = torch.zeros(1, device="cuda")
+    r.train(128, None, opt="adam", lr=1e-3, loss_out=loss)
+    assert r.sync() == L.LS_OK
+    before = _train_state(r)
+    idx = np.arange(128, dtype=np.int32)
+    idx[77] = 300                                   # one past the filled part
+    r.train(128, torch.from_numpy(idx).cuda(), opt="adam", lr=1e-3, loss_out=loss)
+    assert np.isnan(loss.item())
+    assert r.sync() == L.LS_ERR_ARG
+    after = _train_state(r)
+    assert all(torch.equal(a, b) for a, b in zip(after[:3], before[:3])) and after[3] == before[3]
+    r.close()
+
+
 def test_train_gradient_bf16_via_sgd():
     # SGD with lr 0.1 exposes the bf16 gradient as (w - w') / 0.1.
     cfg = W.CONFIGS["training"]
