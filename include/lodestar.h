@@ -292,7 +292,7 @@ typedef struct {
      * (Algorithm 2). */
     int32_t heuristic;
     int32_t count_col[2];  /* request count c_i = inst[i, count_col[0]] (+ inst[i, count_col[1]]
-                              when count_col[1] >= 0), fp32 */
+                              when count_col[1] >= 0), summed in fp64 */
     float theta_imbal;     /* Algorithm 1: c_max - c_min > theta_imbal -> least loaded */
     float k_overload;      /* Algorithm 1: eligible when c_i <= mean + k_overload * std */
     float tau_prefix;      /* Algorithm 2: best prefix match kept when m > tau_prefix */
@@ -356,8 +356,8 @@ int ls_get_bounds(ls_ctx *ctx, int32_t which, float *lo_out, float *hi_out, void
  *      reads;
  *   3. choice = argmin_i yhat[r,i] as in ls_route_batch, then the K-filter
  *      (when k >= 1 and the prompt has a full block): if the mean of
- *      inst_state[:, kv_col] exceeds tau_sat (decided as S > N tau_sat in
- *      fp64, S the fp32 sum in instance order) and
+ *      inst_state[:, kv_col] exceeds tau_sat (the fp64 mean: sum in instance
+ *      order, divided by N) and
  *      16 max_i h[r,i] exceeds tau_ben, the candidates are the k instances
  *      with the largest rendezvous weights mix64(g ^ mix64((i+1) G)) (ties
  *      to the lower index), g = key of the prompt's first block (the prefix
@@ -368,12 +368,12 @@ int ls_get_bounds(ls_ctx *ctx, int32_t which, float *lo_out, float *hi_out, void
  * fallback_opt (DEVICE int32 [n_req], nullable; written when a heuristic is
  * set): the heuristic's instance for every request, whatever its status.
  * With m_i = 16 h[r,i] / L (fp32) and c_i the request counts:
- *   Algorithm 1: if c_max - c_min > theta_imbal (fp32) the least-loaded
- *     instance; else, with mu and sigma the mean and population standard
- *     deviation of c (fp32, sums in instance order, two passes, each
- *     operation rounded on its own, sqrt correctly rounded), the first
- *     instance with c_i <= mu + k_overload sigma in the order (m desc, c asc,
- *     index asc); none: the least loaded.
+ *   Algorithm 1: if c_max - c_min > theta_imbal the least-loaded instance;
+ *     else, with mu and sigma the mean and population standard deviation of
+ *     c (sums in instance order, two passes, sqrt correctly rounded), the
+ *     first instance with c_i <= mu + k_overload sigma in the order (m desc,
+ *     c asc, index asc); none: the least loaded.  Counts, spread, mean,
+ *     deviation and every comparison of counts are fp64.
  *   Algorithm 2: the largest m (lowest index) if it exceeds tau_prefix, else
  *     the least loaded.
  * Least loaded = smallest c_i, lowest index among equals, NaN last.

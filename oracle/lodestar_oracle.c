@@ -381,6 +381,13 @@ static int precedes(float a, int32_t i, float b, int32_t j) {
     return i < j;
 }
 
+/* (a, i) before (b, j) in the order of or_argmin, for fp64 values. */
+static int precedes_d(double a, int32_t i, double b, int32_t j) {
+    if (isnan(a)) return isnan(b) && i < j;
+    if (isnan(b)) return 1;
+    return a < b || (a == b && i < j);
+}
+
 int or_argmin(int64_t n_req, int32_t n_inst, const float *scores, int32_t *choice, float *best) {
     for (int64_t r = 0; r < n_req; ++r) {
         int32_t c = 0;
@@ -614,9 +621,8 @@ int32_t or_hrw_candidates(uint64_t g, int32_t n_inst, int32_t K, int32_t *cand) 
  *   otherwise status 0 and choice = argmin over instances (= argmax of the
  *   reward -TTFT; order of or_argmin), then the K-filter: when K >= 1, the
  *   prompt has a full block (its group key gkey[r] is the key of block 0),
- *     mean_i inst[i, kv_col] > tau_sat   (S = fp32 sum in index order; the
- *                                         test is S > N tau_sat in fp64, the
- *                                         product exact for N < 2^29) and
+ *     mean_i inst[i, kv_col] > tau_sat   (the mean in fp64: the sum in index
+ *                                         order, divided by N) and
  *     max_i 16 h_i > tau_ben             (kappa_i |r| = 16 h_i hit tokens),
  *   status gains bit 4 and a choice outside the candidates is replaced by the
  *   argmin over the candidates.  best = scores of the final choice.
@@ -632,9 +638,10 @@ int or_guards(int64_t n_req, int32_t n_inst, const int64_t *L, const uint64_t *g
     float *x = (float *)malloc((size_t)d * sizeof(float));
     int32_t *cand = (int32_t *)malloc((size_t)(K > 0 ? K : 1) * sizeof(int32_t));
     if (!x || !cand) { free(x); free(cand); return -1; }
-    float kv_sum = 0.0f;
+    double kv_sum = 0.0;
     if (K >= 1 && kv_col >= 0 && kv_col < d_inst)
-        for (int32_t i = 0; i < n_inst; ++i) kv_sum += inst[(int64_t)i * d_inst + kv_col];
+        for (int32_t i = 0; i < n_inst; ++i) kv_sum += (double)inst[(int64_t)i * d_inst + kv_col];
+    const double kv_mean = kv_sum / (double)n_inst;
     for (int64_t r = 0; r < n_req; ++r) {
         const float *sr = scores + r * n_inst;
         const int32_t *hr = hits + r * n_inst;
@@ -662,7 +669,7 @@ int or_guards(int64_t n_req, int32_t n_inst, const int64_t *L, const uint64_t *g
         if (K >= 1 && L[r] >= OR_BLOCK && kv_col >= 0 && kv_col < d_inst) {
             int32_t hmax = 0;
             for (int32_t i = 0; i < n_inst; ++i) if (hr[i] > hmax) hmax = hr[i];
-            if ((double)kv_sum > (double)n_inst * (double)tau_sat && 16.0 * (double)hmax > (double)tau_ben) {
+            if (kv_mean > (double)tau_sat && 16.0 * (double)hmax > (double)tau_ben) {
                 int32_t m = or_hrw_candidates(gkey[r], n_inst, K, cand);
                 int in = 0;
                 for (int32_t q = 0; q < m; ++q) in |= cand[q] == c;
@@ -685,15 +692,15 @@ int or_guards(int64_t n_req, int32_t n_inst, const int64_t *L, const uint64_t *g
 /* ------------------------------------------------------------------------ */
 
 /* The heuristic choice of every request.  Inputs per instance: the request
- * count c_i = inst[i, c_col0] (+ inst[i, c_col1] when c_col1 >= 0), in fp32,
- * and per pair the prefix match ratio m_i = kappa = 16 h / L (fp32, 0 when
- * L = 0).
+ * count c_i = inst[i, c_col0] (+ inst[i, c_col1] when c_col1 >= 0), in fp64,
+ * and per pair the prefix match ratio m_i = kappa = 16 h / L (fp32 as the
+ * feature is, 0 when L = 0).
  *   mode 1, Algorithm 1 (prefix-cache and load aware):
- *     if c_max - c_min > theta_imbal (fp32): argmin_i c_i;
- *     else mu = mean c, sigma = population standard deviation (fp32: sums in
- *     index order, two passes, every operation rounded on its own, sqrt
- *     correctly rounded), and among the instances with c_i <= mu + k sigma
- *     the first in the order (m desc, c asc, index asc); none: argmin_i c_i.
+ *     if c_max - c_min > theta_imbal (fp64): argmin_i c_i;
+ *     else mu = mean c, sigma = population standard deviation (fp64: sums in
+ *     index order, two passes, sqrt correctly rounded), and among the
+ *     instances with c_i <= mu + k sigma (fp64) the first in the order
+ *     (m desc, c asc, index asc); none: argmin_i c_i.
  *   mode 2, Algorithm 2 (prefix aware, threshold tau): i* = argmax m_i
  *     (ties to the lowest index); i* if m_{i*} > tau, else argmin_i c_i.
  * argmin_i c_i takes the lowest index among equal counts, NaN after every
@@ -701,30 +708,30 @@ int or_guards(int64_t n_req, int32_t n_inst, const int64_t *L, const uint64_t *g
 int or_heuristic(int64_t n_req, int32_t n_inst, const int64_t *L, const int32_t *hits,
                  const float *inst, int d_inst, int mode, int c_col0, int c_col1,
                  float theta_imbal, float k_over, float tau, int32_t *out) {
-    float *c = (float *)malloc((size_t)n_inst * sizeof(float));
+    double *c = (double *)malloc((size_t)n_inst * sizeof(double));
     float *m = (float *)malloc((size_t)n_inst * sizeof(float));
     if (!c || !m) { free(c); free(m); return -1; }
     for (int32_t i = 0; i < n_inst; ++i) {
-        c[i] = inst[(int64_t)i * d_inst + c_col0];
-        if (c_col1 >= 0) c[i] = c[i] + inst[(int64_t)i * d_inst + c_col1];
+        c[i] = (double)inst[(int64_t)i * d_inst + c_col0];
+        if (c_col1 >= 0) c[i] = c[i] + (double)inst[(int64_t)i * d_inst + c_col1];
     }
     int32_t least = 0;
-    float cmin = INFINITY, cmax = -INFINITY;       /* NaN counts skipped here */
+    double cmin = INFINITY, cmax = -INFINITY;      /* NaN counts skipped here */
     for (int32_t i = 0; i < n_inst; ++i) {
-        if (precedes(c[i], i, c[least], least)) least = i;   /* NaN after numbers */
+        if (precedes_d(c[i], i, c[least], least)) least = i;  /* NaN after numbers */
         if (c[i] < cmin) cmin = c[i];
         if (c[i] > cmax) cmax = c[i];
     }
-    float mu = 0.0f, var = 0.0f;
+    double mu = 0.0, var = 0.0;
     for (int32_t i = 0; i < n_inst; ++i) mu += c[i];
-    mu = mu / (float)n_inst;
+    mu = mu / (double)n_inst;
     for (int32_t i = 0; i < n_inst; ++i) {
-        float dv = c[i] - mu;
+        double dv = c[i] - mu;
         var += dv * dv;
     }
-    var = var / (float)n_inst;
-    float thr = mu + k_over * sqrtf(var);
-    int imbalanced = cmax - cmin > theta_imbal;
+    var = var / (double)n_inst;
+    double thr = mu + (double)k_over * sqrt(var);
+    int imbalanced = cmax - cmin > (double)theta_imbal;
     for (int64_t r = 0; r < n_req; ++r) {
         const int32_t *hr = hits + r * n_inst;
         for (int32_t i = 0; i < n_inst; ++i) {

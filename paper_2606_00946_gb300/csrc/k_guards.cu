@@ -182,6 +182,42 @@ __device__ __forceinline__ bool in_range(float x, float lo, float hi) { return x
 
 constexpr int kHashedInst = kGuardHeurMaxInst;  // instance hashes kept in shared memory up to this count
 constexpr int kGuardThreads = 256;  // warp 0: batch-wide terms; warps 1..7: requests
+
+// Order-preserving 64-bit key of an fp64 value: keys compare as the values
+// do, -0 and +0 get one key, NaN the largest key (after every number).
+__device__ __forceinline__ uint64_t dkey(double v) {
+  if (v != v) return ~0ull;
+  const uint64_t b = (uint64_t)__double_as_longlong(__dadd_rn(v, 0.0));  // -0 + 0 = +0
+  return (b >> 63) ? ~b : (b | 0x8000000000000000ull);
+}
+__device__ __forceinline__ double dkey_value(uint64_t k) {
+  return __longlong_as_double((long long)((k >> 63) ? (k & 0x7fffffffffffffffull) : ~k));
+}
+
+constexpr float kU = 5.9604644775390625e-8f;  // 2^-24, unit roundoff of fp32
+
+// The rare exact paths, out of line so that the common path keeps its
+// registers: mu + k sigma of the counts (keys of fp64 values) and the mean of
+// a strided fp32 column, each an fp64 chain in instance order, every
+// operation rounded on its own.
+__device__ __noinline__ double threshold64(const uint64_t* ck, int N, float k) {
+  double m = 0.0;
+  for (int i = 0; i < N; ++i) m = __dadd_rn(m, dkey_value(ck[i]));
+  m = __ddiv_rn(m, (double)N);
+  double v = 0.0;
+  for (int i = 0; i < N; ++i) {
+    const double dv = __dsub_rn(dkey_value(ck[i]), m);
+    v = __dadd_rn(v, __dmul_rn(dv, dv));
+  }
+  v = __ddiv_rn(v, (double)N);
+  return __dadd_rn(m, __dmul_rn((double)k, __dsqrt_rn(v)));
+}
+
+__device__ __noinline__ double mean64(const float* col, int stride, int N) {
+  double s = 0.0;
+  for (int i = 0; i < N; ++i) s = __dadd_rn(s, (double)__ldg(col + (int64_t)i * stride));
+  return __ddiv_rn(s, (double)N);
+}
 constexpr int kBarBatch = 1, kBarInst = 2, kBarHeur = 3;
 
 // Warp 0 of a block computes the terms shared by the whole batch and hands
@@ -205,7 +241,8 @@ constexpr int kBarBatch = 1, kBarInst = 2, kBarHeur = 3;
 template <int S>
 __global__ void __launch_bounds__(kGuardThreads) k_guards(const __grid_constant__ GuardArgs a) {
   __shared__ uint64_t s_ih[kHashedInst];  // mix64((i + 1) G): the instance half of the rendezvous weight
-  __shared__ float s_c[kHashedInst];      // heuristic request counts
+  __shared__ uint64_t s_ck[kHashedInst];  // heuristic request counts (fp64) as order-preserving keys
+  __shared__ float s_c[kHashedInst];      // the counts rounded to fp32 (fast statistics)
   __shared__ uint8_t s_elig[kHashedInst]; // c_i <= mu + k sigma
   __shared__ int s_kv, s_inst_bad, s_least, s_imb;
   const int N = a.n_inst, d = kPair + a.d_inst + a.d_req;
@@ -219,31 +256,49 @@ __global__ void __launch_bounds__(kGuardThreads) k_guards(const __grid_constant_
 
   if (warp == 0) {
     if (heur) {
-      // request counts, the least-loaded instance (lowest index on ties),
-      // imbalance, and mu + k sigma: fp32 sums in instance order, two passes,
-      // every operation rounded on its own (no fused multiply-add)
-      float cmin = INFINITY, cmax = -INFINITY, cl = INFINITY;
+      // Algorithm 1's terms in fp64 (counts c_i = queued + running, their
+      // mean and population standard deviation: sums in instance order, two
+      // passes, each operation rounded on its own, sqrt correctly rounded).
+      // Order statistics (least loaded, c_min, c_max, the c ordering of the
+      // requests) are exact through order-preserving keys of the fp64 counts.
+      // The threshold mu + k sigma is first formed in fp32 with a bound on its
+      // distance from the fp64 value; only when some count lies within that
+      // bound (or a count is not a finite fp32 number) does lane 0 form the
+      // fp64 chain, so every eligibility is the fp64 decision.
+      uint64_t kmin = dkey(INFINITY), kmax = dkey(-INFINITY), kl = ~0ull;
       int least = N;
+      bool finite = true;
       for (int i = lane; i < N; i += 32) {
-        float c = __ldg(a.inst + (int64_t)i * a.d_inst + a.c_col0);
-        if (a.c_col1 >= 0) c = __fadd_rn(c, __ldg(a.inst + (int64_t)i * a.d_inst + a.c_col1));
-        s_c[i] = c;
-        cmin = fminf(cmin, c);  // NaN counts are skipped by min / max
-        cmax = fmaxf(cmax, c);
-        if (least == N || score_precedes(c, i, cl, least)) { cl = c; least = i; }  // NaN after numbers
+        double c = (double)__ldg(a.inst + (int64_t)i * a.d_inst + a.c_col0);
+        if (a.c_col1 >= 0) c = __dadd_rn(c, (double)__ldg(a.inst + (int64_t)i * a.d_inst + a.c_col1));
+        const uint64_t k = dkey(c);
+        s_ck[i] = k;
+        const float c32 = __double2float_rn(c);
+        s_c[i] = c32;
+        finite &= fabsf(c32) < 1e30f;  // NaN fails too
+        if (k != ~0ull) {               // NaN counts are skipped by min / max
+          kmin = k < kmin ? k : kmin;
+          kmax = k > kmax ? k : kmax;
+        }
+        if (least == N || k < kl || (k == kl && i < least)) { kl = k; least = i; }  // NaN after numbers
       }
 #pragma unroll
       for (int o = 16; o; o >>= 1) {
-        cmin = fminf(cmin, __shfl_xor_sync(kFull, cmin, o));
-        cmax = fmaxf(cmax, __shfl_xor_sync(kFull, cmax, o));
-        const float oc = __shfl_xor_sync(kFull, cl, o);
+        const uint64_t omin = __shfl_xor_sync(kFull, kmin, o), omax = __shfl_xor_sync(kFull, kmax, o);
+        kmin = omin < kmin ? omin : kmin;
+        kmax = omax > kmax ? omax : kmax;
+        const uint64_t ok = __shfl_xor_sync(kFull, kl, o);
         const int oi = __shfl_xor_sync(kFull, least, o);
-        if (oi < N && (least == N || score_precedes(oc, oi, cl, least))) { cl = oc; least = oi; }
+        if (oi < N && (least == N || ok < kl || (ok == kl && oi < least))) { kl = ok; least = oi; }
       }
+      finite = __all_sync(kFull, finite);
       __syncwarp();
-      float mu = 0.0f;
+      float mu = 0.0f, sa = 0.0f;
 #pragma unroll 8
-      for (int i = 0; i < N; ++i) mu = __fadd_rn(mu, s_c[i]);
+      for (int i = 0; i < N; ++i) {
+        mu = __fadd_rn(mu, s_c[i]);
+        sa = __fadd_rn(sa, fabsf(s_c[i]));
+      }
       mu = __fdiv_rn(mu, (float)N);
       float var = 0.0f;
 #pragma unroll 8
@@ -252,31 +307,67 @@ __global__ void __launch_bounds__(kGuardThreads) k_guards(const __grid_constant_
         var = __fadd_rn(var, __fmul_rn(dv, dv));
       }
       var = __fdiv_rn(var, (float)N);
-      const float thr = __fadd_rn(mu, __fmul_rn(a.k_over, __fsqrt_rn(var)));
-      for (int i = lane; i < N; i += 32) s_elig[i] = s_c[i] <= thr;
+      const float sd = __fsqrt_rn(var);
+      const float thr = __fadd_rn(mu, __fmul_rn(a.k_over, sd));
+      // |thr - thr64| <= delta: the mean's error from recursive summation,
+      // the variance's (second order in the mean's error, plus its own
+      // summation), the square root's (|sqrt x - sqrt y| <= sqrt|x - y|, or
+      // |x - y| / sqrt y), and the final roundings; doubled for margin
+      const float fn = (float)N;
+      const float dmu = 2.0f * (fn + 2.0f) * kU * (sa / fn);
+      const float dvar = dmu * dmu + 2.0f * (fn + 4.0f) * kU * (var + dmu * dmu);
+      float dsd = sqrtf(dvar);
+      if (sd > 0.0f) dsd = fminf(dsd, dvar / sd);
+      dsd += 2.0f * kU * sd;
+      const float delta = 2.0f * (dmu + fabsf(a.k_over) * dsd + 4.0f * kU * (fabsf(mu) + fabsf(a.k_over) * sd));
+      bool near = !finite || !(fabsf(thr) < 1e30f) || !(delta < 1e30f);
+      for (int i = lane; i < N && !near; i += 32) {
+        const float c = s_c[i];
+        near = c == c && fabsf(__fsub_rn(c, thr)) <= delta + 2.0f * kU * fabsf(c);
+      }
+      near = __any_sync(kFull, near);
+      if (near) {
+        double thr64 = lane == 0 ? threshold64(s_ck, N, a.k_over) : 0.0;
+        thr64 = __shfl_sync(kFull, thr64, 0);
+        for (int i = lane; i < N; i += 32) s_elig[i] = dkey_value(s_ck[i]) <= thr64;
+      } else {
+        for (int i = lane; i < N; i += 32) s_elig[i] = s_c[i] <= thr;
+      }
       if (lane == 0) {
         s_least = least;
-        s_imb = __fsub_rn(cmax, cmin) > a.theta_imbal;
+        s_imb = __dsub_rn(dkey_value(kmax), dkey_value(kmin)) > (double)a.theta_imbal;
       }
       sm100::named_bar_arrive(kBarHeur, kGuardThreads);
     }
     if (cold) return;  // no request warp waits for the rest when the batch is cold
     if (hashed)
       for (int i = lane; i < N; i += 32) s_ih[i] = bh::mix64((uint64_t)(i + 1) * kG);
-    // gpu_kv: fp32 sum in instance order (lanes load 32 values at a time, the
-    // sum takes them one by one); mean > tau_sat decided as sum > N tau_sat,
-    // the product exact in fp64
+    // gpu_kv: the fp64 mean (sum in instance order, divided by N) against
+    // tau_sat.  An fp32 sum in the same order (lanes load 32 values at a time,
+    // the sum takes them one by one) decides unless its mean lies within the
+    // recursive-summation bound of tau_sat; then lane 0 forms the fp64 sum.
     int kv = 0;
     if (a.K >= 1) {
-      float sum = 0.0f;
+      float sum = 0.0f, sa = 0.0f;
       for (int base = 0; base < N; base += 32) {
         const int i = base + lane;
         const float v = i < N ? __ldg(a.inst + (int64_t)i * a.d_inst + a.kv_col) : 0.0f;
         const int m = N - base < 32 ? N - base : 32;
 #pragma unroll 8
-        for (int q = 0; q < m; ++q) sum += __shfl_sync(kFull, v, q);
+        for (int q = 0; q < m; ++q) {
+          const float x = __shfl_sync(kFull, v, q);
+          sum = __fadd_rn(sum, x);
+          sa = __fadd_rn(sa, fabsf(x));
+        }
       }
-      kv = (double)sum > (double)N * (double)a.tau_sat;
+      const float mean = __fdiv_rn(sum, (float)N);
+      const float tol = 2.0f * ((float)(N + 2) * kU * (sa / (float)N) + 2.0f * kU * fabsf(a.tau_sat));
+      if (fabsf(mean) < 1e30f && tol < 1e30f && fabsf(__fsub_rn(mean, a.tau_sat)) > tol) {
+        kv = mean > a.tau_sat;
+      } else {
+        if (lane == 0) kv = mean64(a.inst + a.kv_col, a.d_inst, N) > (double)a.tau_sat;
+        kv = __shfl_sync(kFull, kv, 0);
+      }
     }
     if (lane == 0) s_kv = kv;
     sm100::named_bar_arrive(kBarBatch, kGuardThreads);
@@ -444,12 +535,12 @@ __global__ void __launch_bounds__(kGuardThreads) k_guards(const __grid_constant_
       // Algorithm 1: the first eligible instance in the order (m desc, c asc,
       // index asc); Algorithm 2: argmax m (lowest index), kept if m > tau
       int hh = -1, hx = -1;
-      float hc = 0.0f;
+      uint64_t hc = 0;  // count key (fp64 order)
       if (live)
         for (int i = j; i < N; i += S) {
           if (a.heur == 1 && !s_elig[i]) continue;
           const int h = __ldg(hr + i);
-          const float c = s_c[i];
+          const uint64_t c = s_ck[i];
           if (hx < 0 || h > hh || (h == hh && a.heur == 1 && (c < hc || (c == hc && i < hx))) ||
               (h == hh && a.heur == 2 && i < hx)) {
             hh = h;
@@ -460,7 +551,7 @@ __global__ void __launch_bounds__(kGuardThreads) k_guards(const __grid_constant_
 #pragma unroll
       for (int o = 1; o < S; o <<= 1) {
         const int oh = __shfl_xor_sync(kFull, hh, o), oi = __shfl_xor_sync(kFull, hx, o);
-        const float oc = __shfl_xor_sync(kFull, hc, o);
+        const uint64_t oc = __shfl_xor_sync(kFull, hc, o);
         if (oi >= 0 && (hx < 0 || oh > hh || (oh == hh && a.heur == 1 && (oc < hc || (oc == hc && oi < hx))) ||
                         (oh == hh && a.heur == 2 && oi < hx))) {
           hh = oh;

@@ -312,3 +312,57 @@ def test_fallback_heuristic_nan_counts_and_bad_arguments():
     assert L.ls_set_guards(r.h, heuristic=1, count_cols=(cfg.d_inst, -1)) == L.LS_ERR_ARG
     assert L.ls_set_guards(r.h, heuristic=1, count_cols=(0, -2)) == L.LS_ERR_ARG
     r.close()
+
+
+def test_fp64_decisions_at_their_bounds():
+    # Decisions the fp64 reading takes differently from fp32 arithmetic: the
+    # kernel's fp32 statistics find these within their error bound and take
+    # the fp64 path, so every status and fallback equals the oracle's.
+    cfg = _cfg("tiny", n_samples=0)
+    wl, dw, r = _staged(cfg, 1024)
+    N, L_ = cfg.n_inst, np.diff(wl.tok_off)
+    g = dict(n_min=0, ood=False, k=2, kv_col=KV_COL, tau_ben=-1.0)
+    base = wl.inst_state.copy()
+
+    def run(st, **hs):
+        r.snapshot(N, torch.from_numpy(st).cuda())
+        r.set_guards(**g, **hs)
+        out = r.route_guarded(dw.tok, dw.tok_off, dw.req_feats, N)
+        want = oracle.guards(L_, oracle.group_keys(wl.tok, wl.tok_off), out["hits"].cpu().numpy(), st,
+                             wl.req_feats, out["scores"].cpu().numpy(), np.full(cfg.d, -np.inf, np.float32),
+                             np.full(cfg.d, np.inf, np.float32), 0, n_min=0, ood=False, k=2, kv_col=KV_COL,
+                             tau_sat=hs["tau_sat"], tau_ben=-1.0)
+        _assert_same(out, want)
+        fb = out["fallback"].cpu().numpy()
+        if hs.get("heuristic", 0):
+            np.testing.assert_array_equal(fb, oracle.heuristic(
+                L_, out["hits"].cpu().numpy(), st, mode=hs["heuristic"], count_cols=hs["count_cols"],
+                theta_imbal=hs["theta_imbal"], k=hs["k_overload"]))
+        return out["status"].cpu().numpy(), fb
+
+    # K-filter: mean of kv = 0.5 + 2^-27 > 0.5 in fp64 (an fp32 sum gives 0.5)
+    st = base.copy()
+    st[:, KV_COL] = 0.5
+    st[1, KV_COL] = 0.5 + 2.0 ** -24
+    status, _ = run(st, tau_sat=0.5)
+    has_block = L_ >= 16
+    assert (status[has_block] == L.LS_ROUTE_KFILTER).all()
+    st[1, KV_COL] = 0.5
+    status, _ = run(st, tau_sat=0.5)
+    assert (status == 0).all()
+    # Algorithm 1: mu + k sigma = 3 exactly (k = 1) and 3 - 2^-24 (k one fp32 ulp below 1)
+    st = base.copy()
+    st[:, 0] = [1, 1, 3, 3, 1, 1, 3, 3]
+    st[:, 1] = 0
+    for k in (1.0, float(np.nextafter(np.float32(1.0), np.float32(0)))):
+        _, fb = run(st, tau_sat=2.0, heuristic=1, count_cols=(0, 1), theta_imbal=99.0, k_overload=k)
+        if k < 1.0:
+            assert np.isin(fb, [0, 1, 4, 5]).all()       # the count-3 instances are overloaded
+    # counts 2^24 + delta, distinct only in fp64; spread 3 against theta 2.5 / 3.5
+    st[:, 0] = 2.0 ** 24
+    st[:, 1] = [1, 0, 3, 2, 1, 0, 2, 3]
+    for theta, k in ((2.5, 9.0), (3.5, 9.0), (3.5, -9.0), (3.5, 0.0)):
+        run(st, tau_sat=2.0, heuristic=1, count_cols=(0, 1), theta_imbal=theta, k_overload=k)
+    _, fb = run(st, tau_sat=2.0, heuristic=1, count_cols=(0, 1), theta_imbal=2.5, k_overload=9.0)
+    assert (fb == 1).all()                               # imbalanced: the least loaded, lowest index
+    r.close()

@@ -271,6 +271,21 @@ def test_kfilter_thresholds_are_strict():
     assert (st == oracle.ROUTE_KFILTER).all()
 
 
+def test_kfilter_mean_is_taken_in_fp64():
+    # kv = [0.5, 0.5 + 2^-24, 0.5, 0.5]: the mean is 0.5 + 2^-26 > 0.5 in fp64
+    # (an fp32 running sum rounds 1 + 2^-24 to 1 and ends at exactly 2.0)
+    L, g, hits, inst, req, scores = _kv_setting(14, N=4)
+    inst[:, 4] = [0.5, 0.5 + 2.0 ** -24, 0.5, 0.5]
+    lo, hi = _wide(12)
+    _, _, st = oracle.guards(L, g, hits, inst, req, scores, lo, hi, n=1, k=1, kv_col=4,
+                             tau_sat=0.5, tau_ben=-1.0)
+    assert (st == oracle.ROUTE_KFILTER).all()
+    inst[1, 4] = 0.5
+    _, _, st = oracle.guards(L, g, hits, inst, req, scores, lo, hi, n=1, k=1, kv_col=4,
+                             tau_sat=0.5, tau_ben=-1.0)
+    assert (st == 0).all()
+
+
 def test_kfilter_reads_the_kv_column_and_needs_a_full_block():
     L, g, hits, inst, req, scores = _kv_setting(12)
     lo, hi = _wide(12)

@@ -16,11 +16,11 @@ def _m(L, h):
 
 
 def _alg1_brute(L, hits, c, theta, k):
-    c = c.astype(np.float32)
+    c = c.astype(np.float64)
     least = int(np.argmin(c))                       # first index of the smallest count
     if float(c.max()) - float(c.min()) > theta:
         return [least] * len(L)
-    thr = float(np.mean(c.astype(np.float64))) + k * float(np.std(c.astype(np.float64)))
+    thr = float(np.mean(c)) + float(np.float32(k)) * float(np.std(c))
     out = []
     for r in range(len(L)):
         m = [_m(L[r], h) for h in hits[r]]
@@ -44,7 +44,7 @@ def _setting(seed, R=50, N=12):
 def test_alg1_matches_enumeration_with_numpy_statistics():
     for seed in range(20):
         L, hits, inst = _setting(seed)
-        c = inst[:, 0] + inst[:, 1]
+        c = inst[:, 0].astype(np.float64) + inst[:, 1]
         for k in (0.0, 0.5, 1.0, 2.0):
             got = oracle.heuristic(L, hits, inst, mode=1, count_cols=(0, 1), theta_imbal=1e9, k=k)
             assert got.tolist() == _alg1_brute(L, hits, c, 1e9, k), (seed, k)
@@ -65,9 +65,27 @@ def test_alg1_overload_bound_is_inclusive():
     hits = np.array([[0, 0, 4, 1]], np.int32)        # best prefix match on instance 2 (c = 3)
     inst = np.array([[1, 0], [1, 0], [3, 0], [3, 0]], np.float32)
     assert oracle.heuristic(L, hits, inst, mode=1, count_cols=(0, -1), theta_imbal=99, k=1.0)[0] == 2
-    k_less = 1.0 - 2.0 ** -22     # 2 + k_less = 3 - ulp(3) in fp32: the bound falls just below 3
-    # just below: instances 2 and 3 are overloaded; the best of 0 and 1 (m equal, c equal) is 0
+    # k one fp32 ulp below 1: mu + k sigma = 3 - 2^-24 in fp64, just below 3 (fp32
+    # arithmetic would round it back to 3), so instances 2 and 3 are overloaded;
+    # the best of 0 and 1 (m equal, c equal) is 0
+    k_less = float(np.nextafter(np.float32(1.0), np.float32(0)))
     assert oracle.heuristic(L, hits, inst, mode=1, count_cols=(0, -1), theta_imbal=99, k=k_less)[0] == 0
+
+
+def test_alg1_counts_and_spread_are_fp64():
+    # c_i = 2^24 + {1, 0, 3, 2}: distinct in fp64 (fp32 would round 2^24 + 1 to
+    # 2^24 and 2^24 + 3 to 2^24 + 4).  No prefix match anywhere, so the order is
+    # fewest requests first: instance 1.  The spread c_max - c_min is 3.
+    L = np.array([64, 64], np.int64)
+    hits = np.zeros((2, 4), np.int32)
+    inst = np.array([[2**24, 1], [2**24, 0], [2**24, 3], [2**24, 2]], np.float32)
+    assert oracle.heuristic(L, hits, inst, mode=1, count_cols=(0, 1), theta_imbal=99, k=9.0).tolist() == [1, 1]
+    assert oracle.heuristic(L, hits, inst, mode=1, count_cols=(0, 1), theta_imbal=2.5, k=-9.0).tolist() == [1, 1]
+    # 3 > 3.5 is false: balanced; with k = -9 no instance is eligible -> least loaded (1)
+    assert oracle.heuristic(L, hits, inst, mode=1, count_cols=(0, 1), theta_imbal=3.5, k=-9.0).tolist() == [1, 1]
+    # balanced, k = 0: eligible below the mean 2^24 + 1.5, i.e. instances 0 and 1
+    hits[0] = [1, 0, 0, 0]                            # request 0 prefers instance 0 by prefix match
+    assert oracle.heuristic(L, hits, inst, mode=1, count_cols=(0, 1), theta_imbal=3.5, k=0.0).tolist() == [0, 1]
 
 
 def test_alg1_order_prefers_match_then_fewer_requests_then_index():
