@@ -67,6 +67,7 @@ def lib():
             L.or_param_count.restype = i64
             L.or_param_count.argtypes = [C.c_int, P]
             L.or_mlp_forward.argtypes = [C.c_int, C.c_int, P, P, i64, P, P]
+            L.or_mlp_forward_bounds.argtypes = [C.c_int, C.c_int, P, P, i64, P, P, P, P]
             L.or_argmin.argtypes = [i64, i32, P, P, P]
             L.or_ring_append.argtypes = [i64, C.c_int, P, P, i64, i64, P, P]
             L.or_train_step.argtypes = [C.c_int, C.c_int, P, P, P, P, i64, C.c_int, dbl,
@@ -133,14 +134,30 @@ def hash_blocks(tok, tok_off):
     return keys[: koff[-1]], koff
 
 
-def prefix_hits(req_keys, req_key_off, inst_keys, inst_key_off, by_marking: bool = False):
+def prefix_hits(req_keys, req_key_off, inst_keys, inst_key_off, by_marking: bool = False, threads: int = 1):
+    """h[r, i]; threads > 1 splits the instances over host threads (each a
+    separate call on its own instances; the result does not depend on it)."""
     rk = _c(req_keys, np.uint64) if len(req_keys) else np.zeros(1, np.uint64)
     rko = _c(req_key_off, np.int64)
     ik = _c(inst_keys, np.uint64) if len(inst_keys) else np.zeros(1, np.uint64)
     iko = _c(inst_key_off, np.int64)
     R, N = len(rko) - 1, len(iko) - 1
-    hits = np.zeros((R, N), np.int32)
     fn = lib().or_prefix_hits_by_marking if by_marking else lib().or_prefix_hits
+    if threads > 1 and N > 1:
+        import concurrent.futures as cf
+        groups = [g for g in np.array_split(np.arange(N), threads) if len(g)]
+
+        def part(g):
+            a, b = int(g[0]), int(g[-1]) + 1
+            sub_off = _c(iko[a:b + 1] - iko[a], np.int64)
+            sub = _c(ik[iko[a]:iko[b]], np.uint64) if iko[b] > iko[a] else np.zeros(1, np.uint64)
+            h = np.zeros((R, b - a), np.int32)
+            _check(fn(R, _p(rk), _p(rko), b - a, _p(sub), _p(sub_off), _p(h)), "prefix_hits")
+            return h
+
+        with cf.ThreadPoolExecutor(max_workers=len(groups)) as ex:
+            return np.concatenate(list(ex.map(part, groups)), axis=1)
+    hits = np.zeros((R, N), np.int32)
     _check(fn(R, _p(rk), _p(rko), N, _p(ik), _p(iko), _p(hits)), "prefix_hits")
     return hits
 
@@ -218,6 +235,21 @@ def mlp_forward(mode, widths, params, x) -> np.ndarray:
     return y
 
 
+def mlp_forward_bounds(mode, widths, params, x):
+    """Forward pass plus, per row, the fp32-accumulation error bound and the
+    bf16 rounding-flip sensitivity (or_mlp_forward_bounds).  Returns (y, ebound, flip)."""
+    mode = MODES.get(mode, mode)
+    w = _c(widths, np.int32)
+    p = _c(params, np.float64)
+    x = _c(x, np.float64).reshape(-1, w[0])
+    y = np.zeros(x.shape[0], np.float64)
+    eb = np.zeros(x.shape[0], np.float64)
+    fl = np.zeros(x.shape[0], np.float64)
+    _check(lib().or_mlp_forward_bounds(mode, len(w) - 1, _p(w), _p(p), x.shape[0], _p(x), _p(y), _p(eb), _p(fl)),
+           "mlp bounds")
+    return y, eb, fl
+
+
 def argmin(scores):
     s = _c(scores, np.float32)
     R, N = s.shape
@@ -227,9 +259,25 @@ def argmin(scores):
     return choice, best
 
 
-def route(wl, hits=None, inst_keys=None, params=None, mode=None, req_idx=None):
+def route(wl, hits=None, inst_keys=None, params=None, mode=None, req_idx=None, bounds=False, threads=1):
     """Full oracle route of (a subset of) a workload's requests.
-    Returns dict(hits, scores, choice, best)."""
+    Returns dict(hits, scores, choice, best); with bounds, also the per-score
+    rounding analysis of mlp_forward_bounds (ebound, flip).  threads > 1 splits
+    the requests over host threads (the C routines release the interpreter
+    lock); the result does not depend on it."""
+    if threads > 1:
+        import concurrent.futures as cf
+        R_all = len(wl.tok_off) - 1
+        idx = np.arange(R_all) if req_idx is None else np.asarray(req_idx)
+        if inst_keys is None:
+            inst_keys = instance_keys(wl)
+        parts = [p for p in np.array_split(np.arange(len(idx)), threads) if len(p)]
+        with cf.ThreadPoolExecutor(max_workers=len(parts)) as ex:
+            res = list(ex.map(lambda p: route(wl, None if hits is None else hits[p], inst_keys, params, mode,
+                                              idx[p], bounds, 1), parts))
+        out = {k: np.concatenate([r[k] for r in res]) for k in res[0]}
+        out["choice"], out["best"] = argmin(out["scores"])
+        return out
     cfg = wl.cfg
     mode = mode or cfg.dtype
     R_all = len(wl.tok_off) - 1
@@ -247,10 +295,18 @@ def route(wl, hits=None, inst_keys=None, params=None, mode=None, req_idx=None):
         hits = prefix_hits(rk, rko, ik, iko, by_marking=len(idx) * 64 < len(ik))
     L = np.diff(wl.tok_off)[idx]
     x = features(L, hits, wl.inst_state, wl.req_feats[idx], wl.mean, wl.std)
-    y = mlp_forward(mode, cfg.widths, wl.params if params is None else params, x)
+    p = wl.params if params is None else params
+    if bounds:
+        y, eb, fl = mlp_forward_bounds(mode, cfg.widths, p, x)
+    else:
+        y = mlp_forward(mode, cfg.widths, p, x)
     scores = y.astype(np.float32).reshape(len(idx), -1)
     choice, best = argmin(scores)
-    return dict(hits=hits, scores=scores, choice=choice, best=best)
+    out = dict(hits=hits, scores=scores, choice=choice, best=best)
+    if bounds:
+        out["ebound"] = eb.reshape(len(idx), -1)
+        out["flip"] = fl.reshape(len(idx), -1)
+    return out
 
 
 # --------------------------------------------------------------------------

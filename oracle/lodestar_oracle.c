@@ -368,6 +368,170 @@ int or_mlp_forward(int mode, int n_layers, const int *w, const double *params,
     return 0;
 }
 
+/* Rounding analysis of the forward pass, per row, for comparing an
+ * implementation that accumulates every dot product in fp32 (any order)
+ * with this oracle's fp64 sums.  Not part of the method: it says how far such
+ * an implementation may lie from y while computing the same definition.
+ *
+ *   ebound[r]: how far y_fp32acc may lie from y when every bf16 rounding
+ *     point takes the same value on both sides.  The rounding error of a sum
+ *     of K terms accumulated in fp32 behaves as a sum of independent errors
+ *     of at most half an ulp of each partial sum; its standard deviation is
+ *     below 2^-24 sqrt(K) sqrt(S2) / 2, S2 = sum_k (w_k a_k)^2 + b^2, and the
+ *     radius taken is eight of those, 4 2^-24 sqrt(K + 1) sqrt(S2), plus two
+ *     fp32 roundings of z (a statistical radius, not a worst-case bound: the
+ *     worst case K 2^-24 sum |w_k a_k| is a hundred times larger and is never
+ *     approached).  In F32 mode the radii carry through the layers, the
+ *     independent errors of a layer's inputs adding in quadrature
+ *     (sqrt sum_k (w_k e_k)^2; ReLU is 1-Lipschitz); in BF16 mode a
+ *     hidden activation rounded to bf16 is the same bits on both sides unless
+ *     its value lies within its radius of a bf16 rounding midpoint, so only
+ *     the output layer's own radius remains.
+ *   flip[r] (BF16): the sum over the rounding points that lie within their
+ *     radius of a midpoint (an input feature within 1 fp32 ulp, the z-score's
+ *     allowance; a hidden activation within its radius) of |y' - y|, y' the
+ *     output with that one point rounded to the other bf16 neighbour.
+ * The rows are the same as or_mlp_forward's; y is written too. */
+static double bf16_other(double v, float rounded, double *dist) {
+    /* the bf16 neighbour of fp32 value v that RNE did not choose, and the
+     * distance of v from the midpoint between the two */
+    float f = (float)v;
+    uint32_t u;
+    memcpy(&u, &f, 4);
+    uint32_t lo_u = u & 0xFFFF0000u;
+    float lo, hi;
+    memcpy(&lo, &lo_u, 4);
+    uint32_t hi_u = lo_u + 0x10000u;
+    memcpy(&hi, &hi_u, 4);
+    double mid = 0.5 * ((double)lo + (double)hi);
+    *dist = fabs(v - mid);
+    return rounded == lo ? (double)hi : (double)lo;
+}
+
+static double forward_from(int n_layers, const int *w, const double *params, int l0, const double *a_in,
+                           double *buf_a, double *buf_b) {
+    /* BF16 forward of layers l0.. from the layer-l0 input a_in (already bf16 values) */
+    double *a = buf_a, *z = buf_b;
+    for (int k = 0; k < w[l0]; ++k) a[k] = a_in[k];
+    for (int l = l0; l < n_layers; ++l) {
+        const double *W = params + param_offset(n_layers, w, l, 0);
+        const double *b = params + param_offset(n_layers, w, l, 1);
+        for (int o = 0; o < w[l + 1]; ++o) {
+            double s = 0.0;
+            for (int k = 0; k < w[l]; ++k) s += rnd_op(OR_BF16, W[(int64_t)o * w[l] + k]) * a[k];
+            z[o] = rnd(OR_BF16, s + rnd(OR_BF16, b[o]));
+        }
+        if (l + 1 < n_layers)
+            for (int o = 0; o < w[l + 1]; ++o) z[o] = rnd_op(OR_BF16, z[o] > 0.0 ? z[o] : 0.0);
+        double *t = a; a = z; z = t;
+    }
+    return a[0];
+}
+
+int or_mlp_forward_bounds(int mode, int n_layers, const int *w, const double *params, int64_t rows,
+                          const double *x, double *y, double *ebound, double *flip) {
+    int m = max_width(n_layers, w);
+    int64_t tot = 0;
+    for (int l = 0; l <= n_layers; ++l) tot += w[l];
+    double *act = (double *)malloc((size_t)tot * sizeof(double));     /* a_l per layer (as stored) */
+    double *err = (double *)malloc((size_t)tot * sizeof(double));     /* F32: bound on a_l */
+    double *alt = (double *)malloc((size_t)m * sizeof(double));
+    double *ba = (double *)malloc((size_t)m * sizeof(double));
+    double *bb = (double *)malloc((size_t)m * sizeof(double));
+    int64_t *off = (int64_t *)malloc((size_t)(n_layers + 2) * sizeof(int64_t));
+    if (!act || !err || !alt || !ba || !bb || !off) {
+        free(act); free(err); free(alt); free(ba); free(bb); free(off);
+        return -1;
+    }
+    off[0] = 0;
+    for (int l = 0; l <= n_layers; ++l) off[l + 1] = off[l] + w[l];
+    const double u = ldexp(1.0, -24);
+    for (int64_t r = 0; r < rows; ++r) {
+        const double *xr = x + r * w[0];
+        double fl = 0.0, eb = 0.0;
+        for (int k = 0; k < w[0]; ++k) {
+            act[k] = rnd_op(mode, xr[k]);
+            err[k] = 0.0;
+        }
+        int flips_n = 0;
+        /* flip candidates of the input: within 1 fp32 ulp of a bf16 midpoint */
+        double yv = 0.0;
+        for (int l = 0; l < n_layers; ++l) {
+            const double *W = params + param_offset(n_layers, w, l, 0);
+            const double *b = params + param_offset(n_layers, w, l, 1);
+            const double *a = act + off[l];
+            const double *ea = err + off[l];
+            double *an = act + off[l + 1];
+            double *en = err + off[l + 1];
+            const double gK = 4.0 * sqrt((double)w[l] + 1.0) * u;
+            for (int o = 0; o < w[l + 1]; ++o) {
+                double s = 0.0, s2 = 0.0, prop = 0.0;
+                for (int k = 0; k < w[l]; ++k) {
+                    double wk = rnd_op(mode, W[(int64_t)o * w[l] + k]);
+                    s += wk * a[k];
+                    s2 += (wk * a[k]) * (wk * a[k]);
+                    prop += (wk * ea[k]) * (wk * ea[k]);
+                }
+                double bo = rnd(mode, b[o]);
+                double z = rnd(mode, s + bo);
+                double ez = gK * sqrt(s2 + bo * bo) + 2.0 * u * fabs(z) + (mode == OR_F32 ? sqrt(prop) : 0.0);
+                if (l + 1 == n_layers) {
+                    an[o] = z;
+                    en[o] = ez + 2.0 * u * fabs(z);
+                } else {
+                    double rl = z > 0.0 ? z : 0.0;
+                    an[o] = rnd_op(mode, rl);
+                    en[o] = mode == OR_F32 ? ez : 0.0;
+                }
+            }
+        }
+        yv = act[off[n_layers]];
+        eb = err[off[n_layers]];
+        if (mode == OR_BF16) {
+            /* rounding points near a midpoint: inputs (1 fp32 ulp), hidden (their bound) */
+            for (int l = 0; l < n_layers; ++l) {
+                for (int o = 0; o < w[l]; ++o) {
+                    double pre, rad;
+                    if (l == 0) {
+                        pre = xr[o];
+                        rad = ldexp(fabs(pre), -23);
+                    } else {
+                        /* recompute the pre-rounding value and its bound */
+                        const double *W = params + param_offset(n_layers, w, l - 1, 0);
+                        const double *b = params + param_offset(n_layers, w, l - 1, 1);
+                        const double *a = act + off[l - 1];
+                        double s = 0.0, s2 = 0.0;
+                        for (int k = 0; k < w[l - 1]; ++k) {
+                            double wk = rnd_op(OR_BF16, W[(int64_t)o * w[l - 1] + k]);
+                            s += wk * a[k];
+                            s2 += (wk * a[k]) * (wk * a[k]);
+                        }
+                        double bo = rnd(OR_BF16, b[o]);
+                        double z = rnd(OR_BF16, s + bo);
+                        pre = z > 0.0 ? z : 0.0;
+                        rad = 4.0 * sqrt((double)w[l - 1] + 1.0) * u * sqrt(s2 + bo * bo) + 2.0 * u * fabs(z);
+                        if (pre == 0.0) continue;  /* relu clamps: both sides give 0 or a value within rad */
+                    }
+                    double dist;
+                    double other = bf16_other(pre, (float)act[off[l] + o], &dist);
+                    if (dist > rad) continue;
+                    for (int k = 0; k < w[l]; ++k) alt[k] = act[off[l] + k];
+                    alt[o] = other;
+                    double y2 = forward_from(n_layers, w, params, l, alt, ba, bb);
+                    fl += fabs(y2 - yv);
+                    ++flips_n;
+                }
+            }
+        }
+        (void)flips_n;
+        y[r] = yv;
+        ebound[r] = eb;
+        if (flip) flip[r] = fl;
+    }
+    free(act); free(err); free(alt); free(ba); free(bb); free(off);
+    return 0;
+}
+
 /* ------------------------------------------------------------------------ */
 /* greedy selection (Sec. 4.1; Algorithm 4 argmax of reward = -TTFT)        */
 /* ------------------------------------------------------------------------ */

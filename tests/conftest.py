@@ -24,3 +24,15 @@ def pytest_collection_modifyitems(config, items):
     for it in items:
         if "gpu" in it.keywords:
             it.add_marker(skip)
+
+
+def pytest_sessionfinish(session, exitstatus):
+    # figures of the prediction parity checks, when a report path is given
+    path = os.environ.get("LODESTAR_PARITY_REPORT")
+    if path:
+        try:
+            import parity_bars
+        except ImportError:
+            return
+        if parity_bars.STATS:
+            parity_bars.write_stats(path)

@@ -560,3 +560,47 @@ def test_linear_model_converges_to_least_squares():
     A = np.hstack([xz, np.ones((n, 1))])
     sol = np.linalg.lstsq(A, y.astype(np.float64), rcond=None)[0]
     np.testing.assert_allclose(tr.params, sol, atol=1e-8)
+
+
+# ----------------------------------------------------------------------------
+# rounding analysis of the forward pass (the parity tests' radius per row)
+# ----------------------------------------------------------------------------
+
+def test_forward_bounds_output_equals_the_forward_pass():
+    rng = np.random.default_rng(40)
+    for mode, widths in (("f32", (16, 64, 64, 1)), ("bf16", (24, 32, 32, 32, 1))):
+        params = W.xavier_params(widths, 3)
+        x = rng.standard_normal((50, widths[0])).astype(np.float32)
+        y, eb, fl = oracle.mlp_forward_bounds(mode, widths, params, x)
+        assert np.array_equal(y, oracle.mlp_forward(mode, widths, params, x))
+        assert (eb > 0).all() and (fl >= 0).all()
+        if mode == "f32":
+            assert (fl == 0).all()
+
+
+def test_forward_bounds_radius_of_a_single_dot_product():
+    # one linear layer (K = 3 inputs): radius = 4 sqrt(K + 1) 2^-24 sqrt(sum (w a)^2 + b^2)
+    # + 2 2^-24 |z| for the sum, + 2 2^-24 |z| for the output's own rounding
+    widths = (3, 1)
+    w = np.array([0.5, -0.25, 2.0], np.float32)
+    b = np.float32(0.125)
+    params = np.concatenate([w, [b]]).astype(np.float32)
+    x = np.array([[1.0, 2.0, 3.0]], np.float32)
+    y, eb, fl = oracle.mlp_forward_bounds("f32", widths, params, x)
+    z = 0.5 - 0.5 + 6.0 + 0.125
+    u = 2.0 ** -24
+    s2 = 0.25 + 0.25 + 36.0 + 0.125 ** 2
+    assert y[0] == z
+    assert np.isclose(eb[0], 4 * np.sqrt(4.0) * u * np.sqrt(s2) + 4 * u * abs(z), rtol=1e-12)
+
+
+def test_forward_bounds_flip_at_a_bf16_midpoint():
+    # hidden unit pre-activation exactly 1 + 2^-8 (the midpoint of bf16 1 and
+    # 1 + 2^-7; round-to-nearest-even keeps 1): flagged, and its flip moves the
+    # output by w2 * 2^-7 exactly; 1 + 2^-6 sits on a bf16 value: no flip
+    widths = (1, 1, 1)
+    for pre, want in ((1.0 + 2.0 ** -8, 3.0 * 2.0 ** -7), (1.0 + 2.0 ** -6, 0.0)):
+        params = np.array([1.0, pre - 1.0, 3.0, 0.0], np.float32)   # W1 = 1, b1, W2 = 3, b2 = 0
+        x = np.array([[1.0]], np.float32)
+        y, eb, fl = oracle.mlp_forward_bounds("bf16", widths, params, x)
+        assert fl[0] == want
