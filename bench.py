@@ -1,15 +1,20 @@
 """Benchmark of the Lodestar routing hot path on GB300.
 
-One step = one pass of the whole path over one batch of the homogeneous
-workload (32 instances x 4096 pending requests, prompts 64-4096 tokens with
-Zipf-shared prefixes, 64-dim features, bf16 MLP 64->256->256->1):
-  ls_snapshot_update (instance state rows)  -> ls_route_batch (hash, probe,
-  features, MLP, argmin for 131,072 pairs) -> ls_log_samples (4096 records)
+One step = one pass of the whole path over one batch of the large-cluster
+workload (256 instances x 16,384 pending requests, prompts 128-16k tokens with
+Zipf-shared prefixes over 4096 templates, 2^20 cached blocks per instance,
+128-dim features, bf16 MLP 128->512->512->1):
+  ls_snapshot_update (instance state rows) -> ls_route_batch (hash, probe,
+  features, MLP, argmin for 4,194,304 pairs) -> ls_log_samples (4096 records)
   -> ls_train_step (Adam, batch 4096) -> ls_publish.
 Metric: routing decisions per second (requests routed per second of whole
-steps).  Inputs resident in HBM and larger than L2 (consecutive timed steps
-read different device copies of the batch, 205 MB together); CUDA events on
-the launching stream; W untimed warm-up steps.
+steps).  Inputs resident in HBM and larger than L2 (541 MB of prompt tokens
+per batch); CUDA events on the launching stream; W untimed warm-up steps.
+Beside the headline, the line carries every configuration's own figures
+(tiny latency, homogeneous and heterogeneous route rates, the online-training
+configuration's samples/s, the large configuration's route rate), each with
+its roofline, and the measured ceilings (random 8-byte gathers, fp32 FMA, L2
+reads) the memory- and ALU-bound kernels are judged against.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
@@ -31,11 +36,19 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
-WORKLOAD = "homogeneous"
-WORKLOAD_DESC = (f"{WORKLOAD}: 32 instances x 4096 requests/step, prompts 64-4096 tokens with Zipf(1.1) "
-                 "prefixes over 256 templates, 16384 cached blocks/instance, bf16 MLP 64-256-256-1, "
-                 "Adam batch 4096")
-INPUT_SETS = 6   # device copies of the batch the timed steps rotate over (> L2 together)
+WORKLOAD = "large"
+DESC = {
+    "tiny": "tiny: 8 instances x 64 requests, prompts 32-512 tokens (+128-token system prompt, p 0.5), "
+            "2048 cached blocks/instance, fp32 MLP 16-64-64-1",
+    "homogeneous": "homogeneous: 32 instances x 4096 requests, prompts 64-4096 tokens with Zipf(1.1) prefixes over "
+                   "256 templates, 16384 cached blocks/instance, bf16 MLP 64-256-256-1",
+    "heterogeneous": "heterogeneous: 64 instances (3 GPU types) x 8192 requests, prompts 8k-32k tokens log-uniform, "
+                     "65536 cached blocks/instance, bf16 MLP 128-256-256-256-1",
+    "large": "large: 256 instances x 16384 requests/step, prompts 128-16384 tokens with Zipf(1.1) prefixes over 4096 "
+             "templates, 2^20 cached blocks/instance (open addressing, load 0.5), bf16 MLP 128-512-512-1, "
+             "Adam batch 4096",
+}
+INPUT_SETS_SMALL = 6   # device copies of a batch smaller than L2 that timed routes rotate over
 METRIC = "routing decisions/sec (requests routed per second of whole route+log+train+publish steps)"
 UNIT = "decisions/s"
 
@@ -43,21 +56,25 @@ UNIT = "decisions/s"
 def parse():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=2000)
-    p.add_argument("--warmup", type=int, default=10)
+    p.add_argument("--steps", type=int, default=200)
+    p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-configs", action="store_true", help="skip the other configurations' measurements")
     p.add_argument("--no-guards", action="store_true", help="skip the guarded-route measurement")
     p.add_argument("--no-replay", action="store_true", help="skip the replay-pool admission measurement")
     p.add_argument("--no-paper-point", action="store_true", help="skip the paper operating-point measurement")
     p.add_argument("--no-training-config", action="store_true",
                    help="skip the online-training throughput configuration")
+    p.add_argument("--no-probes", action="store_true", help="skip the ceiling microbenchmarks")
     p.add_argument("--paper-point-only", action="store_true", help="only the paper operating-point measurement")
     p.add_argument("--replay-only", action="store_true",
                    help="only the replay-pool admission measurement (for kernel profiling)")
     p.add_argument("--guards-only", action="store_true",
                    help="only the guarded-route measurement (--steps routes; for kernel profiling)")
+    p.add_argument("--route-only", default=None, choices=["tiny", "homogeneous", "heterogeneous", "large"],
+                   help="only --steps routes of one configuration (for kernel profiling)")
     p.add_argument("--cpu-seconds", type=float, default=12.0, help="target oracle work for cpu_baseline")
     return p.parse_args()
 
@@ -303,11 +320,29 @@ def measure_training_config(L, H, W, dev, steps=1000):
     e1.record(sb)
     e1.synchronize()
     ms = e0.elapsed_time(e1)
+    # training steps alone, issued back to back on one stream
+    alone = timed_back_to_back(lambda k: r.train(cfg.train_batch, None, opt="adam", lr=cfg.train_lr, loss_out=loss,
+                                                 stream=sb), 200, sb)
+    ms_alone = float(np.mean(alone[10:]))
     r.close()
+    # roofline of one step: its flops on the tensor cores plus its bytes
+    # (minibatch rows and targets read; Adam reads w, g, m, v and writes w, m,
+    # v and the bf16 image: 30 B per parameter) at the measured HBM rate
+    peaks = measured_peaks()[0]
+    B_ = cfg.train_batch
+    flops = train_flops(cfg.widths, B_)
+    n_params = sum(cfg.widths[l] * cfg.widths[l + 1] + cfg.widths[l + 1] for l in range(len(cfg.widths) - 1))
+    bytes_ = B_ * (cfg.d + 1) * 4 + 30 * n_params
+    t_roof = flops / (peaks["bf16_tflops"] * 1e12) + bytes_ / (peaks["hbm_gbs"] * 1e9)
+    rate_alone = B_ / (ms_alone / 1e3)
     return {"config": "training: ring 2^20 x 128 fp32, Adam lr 3e-4, batch 4096, 128-256-256-256-1 bf16",
             "train_steps": steps, "route_calls": steps // 10, "ms": ms,
             "train_samples_per_s": steps * cfg.train_batch / (ms / 1e3),
-            "routes_per_s_beside_training": (steps // 10) * cfg.n_req / (ms / 1e3)}
+            "routes_per_s_beside_training": (steps // 10) * cfg.n_req / (ms / 1e3),
+            "train_step_alone_ms": ms_alone, "train_samples_per_s_alone": rate_alone,
+            "roofline": {"step_us": 1e6 * t_roof, "samples_per_s": B_ / t_roof, "flops": flops, "bytes": bytes_,
+                         "frac_alone": rate_alone / (B_ / t_roof),
+                         "frac_beside_routes": steps * B_ / (ms / 1e3) / (B_ / t_roof)}}
 
 
 def dist_setup(n_gpus):
@@ -351,25 +386,48 @@ def mlp_flops_per_score(widths):
     return f
 
 
+def distinct_probes(hits, lens, keys, key_off):
+    """Sum over instances of the distinct block keys the prefix walk asks that
+    instance about: block b of request r is asked of instance i when blocks
+    0..b-1 are all cached there (h[r, i] >= b), the miss included.  A key
+    stands for its whole prefix (chained hash), so every request holding key k
+    at depth b gives instance i the same answer to h >= b: k counts once per
+    instance with h[r(k), i] >= b(k), r(k) any request holding it."""
+    R, N = hits.shape
+    nb = (np.asarray(lens) // 16).astype(np.int64)
+    if len(keys) == 0:
+        return 0
+    depth = np.arange(len(keys), dtype=np.int64) - np.repeat(np.asarray(key_off[:-1], np.int64), nb)
+    req = np.repeat(np.arange(R, dtype=np.int64), nb)
+    _, first = np.unique(np.asarray(keys).view(np.uint64), return_index=True)
+    r_k, b_k = req[first], depth[first]
+    big = int(max(hits.max(initial=0), nb.max(initial=0))) + 2
+    sh = np.sort((np.arange(R, dtype=np.int64)[:, None] * big + hits.astype(np.int64)).ravel())
+    cnt = (r_k + 1) * N - np.searchsorted(sh, r_k * big + b_k, side="left")
+    return int(cnt.sum())
+
+
 def route_costs(cfg, R, N, hits, lens, keys, key_off):
-    """flops of the scorer and bytes of the prefix matcher for one batch."""
+    """Algorithmic flops and bytes of one routing batch: the scorer's
+    layer-1-factorised flops (and the dense count), and the prefix matcher's
+    compulsory bytes -- every prompt token read once (4 B), 8 B per distinct
+    probed (instance, key), 8 B of outputs per request."""
     w = cfg.widths
     flops = (mlp_flops_per_score(w) * R * N + 2 * N * cfg.d_inst * w[1] + 2 * R * cfg.d_req * w[1])
-    nb = lens // 16
-    need_blocks = np.minimum(nb, hits.max(axis=1) + 1)                 # blocks that must be hashed
-    tok_bytes = 4 * int(np.sum(np.minimum(lens, 16 * need_blocks)))
-    # distinct (instance, probed key): blocks 0..h (the miss included when h < n_r)
-    pr = []
-    for i in range(N):
-        upto = np.minimum(hits[:, i] + 1, nb).astype(np.int64)
-        tot = int(upto.sum())
-        base = np.repeat(key_off[:-1], upto)
-        within = np.arange(tot) - np.repeat(np.cumsum(upto) - upto, upto)
-        pr.append(np.unique(keys[base + within]).size if tot else 0)
-    probe_bytes = 8 * int(np.sum(pr))
-    out_bytes = 4 * R * N + 8 * R
-    return dict(score_flops=float(flops), prefix_bytes=float(tok_bytes + probe_bytes + out_bytes),
-                tok_bytes=tok_bytes, probe_bytes=probe_bytes)
+    dense = sum(2 * w[l] * w[l + 1] for l in range(len(w) - 1)) * R * N
+    tok_bytes = 4 * int(np.sum(lens))
+    probe_bytes = 8 * distinct_probes(hits, lens, keys, key_off)
+    out_bytes = 8 * R
+    return dict(score_flops=float(flops), score_flops_dense=float(dense),
+                prefix_bytes=float(tok_bytes + probe_bytes + out_bytes),
+                tok_bytes=tok_bytes, probe_bytes=probe_bytes, out_bytes=out_bytes)
+
+
+def route_roofline(costs, R, N, peaks):
+    """Sum over the dependent phases of max(bytes / BW, flops / peak): the prefix
+    phase is bytes-bound, the scoring phase flops-bound."""
+    t = costs["prefix_bytes"] / (peaks["hbm_gbs"] * 1e9) + costs["score_flops"] / (peaks["bf16_tflops"] * 1e12)
+    return {"roofline_ms": 1e3 * t, "decisions_per_s": R / t, "scores_per_s": R * N / t}
 
 
 def train_flops(widths, B):
@@ -490,78 +548,97 @@ def measured_peaks():
 # CPU oracle (cpu_baseline and --impl reference)
 # ----------------------------------------------------------------------------
 
-def oracle_work(wl, inst_keys, n_req, rng):
-    """Oracle pass over a sample: route n_req requests (hash, hits, features,
-    bf16 MLP, argmin) and one training step on n_req logged records."""
+def cpu_model():
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.split(":")[0].strip() in ("Model name", "Model"):
+                v = line.split(":", 1)[1].strip()
+                if v and not v.isdigit():
+                    return v
+    except Exception:
+        pass
+    return None
+
+
+def oracle_setup(wl):
+    """The oracle's snapshot: each instance's key set hashed by the oracle and
+    sorted once (as the router's tables are built once), plus logged records
+    for its training step."""
     import oracle
+    inst_sorted = oracle.sorted_instance_keys(oracle.instance_keys(wl))
+    if wl.samples_x is not None:
+        rx, ry = wl.samples_x, wl.samples_y
+    else:
+        from paper_2606_00946_gb300 import workload as W
+        rx, ry = W.records(np.random.default_rng(wl.cfg.seed + 5000), wl.cfg, 4096)
+    return inst_sorted, rx, ry
+
+
+def oracle_work(wl, orc, n_req, rng, threads):
+    """Oracle pass over a sample: route n_req requests (hash, hits against the
+    sorted key sets, features, fp64-accumulated MLP, argmin) with the requests
+    split over `threads` host threads (the C routines release the interpreter
+    lock), then one Adam step on n_req logged records on one thread."""
+    import oracle
+    inst_sorted, rx, ry = orc
     idx = np.sort(rng.choice(len(wl.tok_off) - 1, size=n_req, replace=False))
     t0 = time.perf_counter()
-    oracle.route(wl, inst_keys=inst_keys, req_idx=idx)
+    oracle.route(wl, req_idx=idx, inst_sorted=inst_sorted, threads=threads)
     tr = oracle.Trainer(wl.cfg.widths, wl.params, wl.cfg.dtype)
-    bidx = rng.integers(0, len(wl.samples_y), size=n_req).astype(np.int32)
-    tr.step(wl.samples_x, wl.samples_y, bidx, wl.mean, wl.std, "adam", 3e-4)
+    bidx = rng.integers(0, len(ry), size=n_req).astype(np.int32)
+    tr.step(rx, ry, bidx, wl.mean, wl.std, "adam", 3e-4)
     return time.perf_counter() - t0
 
 
-def oracle_work_threads(wl, inst_keys, n_req, rng, threads):
-    """oracle_work with the requests split over `threads` host threads (the
-    oracle's C routines release the interpreter lock, so the threads run on
-    separate cores); the training step stays on one thread."""
-    import concurrent.futures as cf
-    import oracle
-    idx = np.sort(rng.choice(len(wl.tok_off) - 1, size=n_req, replace=False))
-    parts = [p for p in np.array_split(idx, threads) if len(p)]
-    t0 = time.perf_counter()
-    with cf.ThreadPoolExecutor(max_workers=threads) as ex:
-        list(ex.map(lambda p: oracle.route(wl, inst_keys=inst_keys, req_idx=p), parts))
-    tr = oracle.Trainer(wl.cfg.widths, wl.params, wl.cfg.dtype)
-    bidx = rng.integers(0, len(wl.samples_y), size=n_req).astype(np.int32)
-    tr.step(wl.samples_x, wl.samples_y, bidx, wl.mean, wl.std, "adam", 3e-4)
-    return time.perf_counter() - t0
-
-
-def cpu_baseline(wl, inst_keys, target_s):
+def cpu_baseline(wl, orc, target_s, name):
     """The oracle on the host's cores (requests over all cores), beside its
-    single-thread figure."""
+    single-thread figure.  The large configuration is sampled at 1/64 of its
+    requests; the others at about target_s of work."""
     rng = np.random.default_rng(0)
     cores = os.cpu_count() or 1
-    t_cal = oracle_work(wl, inst_keys, 16, rng)
-    n1 = int(np.clip(16 * 0.5 * target_s / max(t_cal, 1e-3), 16, len(wl.tok_off) - 1))
-    t1 = oracle_work(wl, inst_keys, n1, rng)
-    n = int(min(len(wl.tok_off) - 1, max(16, n1 * cores)))   # about the same wall time if the cores scale
-    t = oracle_work_threads(wl, inst_keys, n, rng, cores)
-    return {"value": n / t, "unit": UNIT, "cores": cores, "kind": "oracle",
+    R = len(wl.tok_off) - 1
+    t_cal = oracle_work(wl, orc, 2, rng, 1) / 2
+    n1 = int(np.clip(0.3 * target_s / max(t_cal, 1e-4), 2, R))
+    t1 = oracle_work(wl, orc, n1, rng, 1)
+    if name == "large":
+        n = R // 64
+    else:
+        n = int(min(R, max(16, n1 * cores)))
+    t = oracle_work(wl, orc, n, rng, cores)
+    return {"value": n / t, "unit": UNIT, "cores": cores, "kind": "oracle", "cpu_model": cpu_model(),
             "single_thread_value": n1 / t1,
-            "sample": f"{n} of {len(wl.tok_off) - 1} requests of the {WORKLOAD} batch routed by the C oracle "
-                      f"(hash, hits, features, fp64-accumulated bf16 MLP, argmin) over {cores} host threads, "
-                      f"plus one Adam step on {n} logged records on one thread; {t:.1f} s (one thread: "
-                      f"{n1} requests in {t1:.1f} s)"}
+            "sample": f"{n} of {R} requests of the {name} batch{' (1/64)' if name == 'large' else ''} routed by "
+                      f"the C oracle (hash, hits against each instance's sorted key set, features, "
+                      f"fp64-accumulated bf16 MLP, argmin) over {cores} host threads, plus one Adam step on {n} "
+                      f"logged records on one thread; {t:.1f} s (one thread: {n1} requests in {t1:.1f} s)"}
 
 
 def run_reference(args, world, rank):
     from paper_2606_00946_gb300 import workload as W
-    import oracle
     if rank != 0:
         return 0
     wl = W.generate(WORKLOAD)
-    inst_keys = oracle.instance_keys(wl)
+    orc = oracle_setup(wl)
     rng = np.random.default_rng(1)
     cores = os.cpu_count() or 1
-    n = 48 * max(1, cores // 4)
+    n = cores                                   # one request per host thread: about a second per step
     for _ in range(args.warmup):
-        oracle_work_threads(wl, inst_keys, n, rng, cores)
-    times = [oracle_work_threads(wl, inst_keys, n, rng, cores) for _ in range(args.steps)]
+        oracle_work(wl, orc, n, rng, cores)
+    times = [oracle_work(wl, orc, n, rng, cores) for _ in range(args.steps)]
     ms = 1e3 * float(np.mean(times))
     value = n / (ms / 1e3)
+    cfg = wl.cfg
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic (seeded generator shaped like the paper's prefix-sharing workloads)",
-            "config": {"workload": WORKLOAD_DESC, "pairs_per_step": 32 * 4096, "train_samples_per_step": 4096,
-                       "parallelism": "replicas", "sample_requests_per_step": n},
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
-                             "sample": f"{n} requests over {cores} host threads + one Adam step on {n} records "
-                                       f"per step"},
+            "config": {"workload": DESC[WORKLOAD], "pairs_per_step": cfg.n_req * cfg.n_inst,
+                       "train_samples_per_step": cfg.train_batch, "parallelism": "replicas",
+                       "sample_requests_per_step": n},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "cpu_model": cpu_model(),
+                             "sample": f"{n} requests of the {WORKLOAD} batch over {cores} host threads + one Adam "
+                                       f"step on {n} records per step"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
     return 0
@@ -570,6 +647,388 @@ def run_reference(args, world, rank):
 # ----------------------------------------------------------------------------
 # GPU arm
 # ----------------------------------------------------------------------------
+
+def timed_back_to_back(fn, n, stream):
+    """n calls issued back to back, an event on the stream between consecutive
+    ones: the host stays ahead of the GPU, so each interval is one call's
+    device time.  Returns the intervals in ms."""
+    import torch
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(n + 1)]
+    ev[0].record(stream)
+    for k in range(n):
+        fn(k)
+        ev[k + 1].record(stream)
+    ev[n].synchronize()
+    return [ev[k].elapsed_time(ev[k + 1]) for k in range(n)]
+
+
+def traced(L, r, fn, n):
+    """n calls issued one by one with every kernel launch of the context
+    bracketed by CUDA events on its launching stream (the library's tracer),
+    each call behind a ~150 us GPU spin so no interval holds host time.
+    Returns ({kernel: (launches, total_ms, timed)}, launches per call)."""
+    import torch
+    L.ls_trace_enable(r.h, True)
+    L.ls_trace_read(r.h)
+    torch.cuda.synchronize()
+    for k in range(n):
+        torch.cuda._sleep(300000)
+        fn(k)
+    torch.cuda.synchronize()
+    rc, trace = L.ls_trace_read(r.h)
+    L.ls_trace_enable(r.h, False)
+    return trace
+
+
+def kernel_rooflines(trace, n_calls, costs, cfg, R, N, Bt, peaks, peak_src):
+    """Each traced kernel's achieved rate against its bound: the prefix walk
+    (compulsory bytes, HBM), the feature image (bytes written), the scorers
+    (factorised flops, bf16 tensor), the training products (their flops)."""
+    per = {k: v[1] / max(v[2], 1) for k, v in trace.items()}
+    n_per = {k: v[0] / n_calls for k, v in trace.items()}
+    out = {}
+    for k in per:
+        d_pad = 64 * ((cfg.d + 63) // 64)
+        if k in ("prefix_index", "prefix_match"):
+            alg, peak, unit, bound = costs["prefix_bytes"] / 1e9, peaks["hbm_gbs"], "GB/s", "hbm"
+        elif k == "features":
+            alg = (R * N * (2 * d_pad + 4) + R * 8) / 1e9
+            peak, unit, bound = peaks["hbm_gbs"], "GB/s", "hbm"
+        elif k in ("score_tc", "score_simt"):
+            alg, peak, unit, bound = costs["score_flops"] / 1e12, peaks["bf16_tflops"], "TFLOP/s", "tensor"
+        elif k in ("gemm_tc_fwd", "gemm_tc_dx", "gemm_tc_dw"):
+            w = cfg.widths
+            nh = len(w) - 2
+            per_kind = {"gemm_tc_fwd": sum(2 * Bt * w[l] * w[l + 1] for l in range(nh + 1)) + 2 * Bt * w[nh],
+                        "gemm_tc_dx": sum(4 * Bt * w[l] * w[l + 1] for l in range(1, nh)),
+                        "gemm_tc_dw": 2 * Bt * w[0] * w[1]}
+            alg = per_kind[k] / max(n_per[k], 1e-9) / 1e12
+            peak, unit, bound = peaks["bf16_tflops"], "TFLOP/s", "tensor"
+        else:
+            continue
+        achieved = alg / (per[k] / 1e3)
+        out[k] = {"kernel": k, "bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
+                  "frac": achieved / peak, "traffic": profiled_traffic(k), "peak_source": f"{peak_src} (burst)",
+                  "avg_launch_ms": per[k],
+                  "timing": "CUDA events around each launch on its stream (library tracer), calls issued one by one"}
+    return out
+
+
+def setup_config(name, H, W, dev, ring=65536, **caps):
+    import torch
+    wl = W.generate(name)
+    cfg = wl.cfg
+    r = H.Router.for_config(cfg, ring_capacity=max(ring, 4 * cfg.train_batch), **caps)
+    dw = H.DeviceWorkload(wl, device=dev)
+    dw.load(r)
+    if wl.samples_x is not None:
+        rx, ry = wl.samples_x, wl.samples_y
+    else:
+        rx, ry = W.records(np.random.default_rng(cfg.seed + 5000), cfg, ring)
+    sx, sy = torch.from_numpy(rx).to(dev), torch.from_numpy(ry).to(dev)
+    r.log(sx, sy)                                      # fill the ring once
+    return wl, cfg, r, dw, sx, sy
+
+
+def input_sets(dw, small_sets):
+    """Device copies of the batch: one when it is larger than L2, else enough
+    rotating copies that consecutive calls read their prompts from HBM."""
+    bytes_ = sum(t.numel() * t.element_size() for t in (dw.tok, dw.tok_off, dw.req_feats))
+    n = 1 if bytes_ > 300e6 else small_sets
+    return [(dw.tok, dw.tok_off, dw.req_feats)] + [
+        (dw.tok.clone(), dw.tok_off.clone(), dw.req_feats.clone()) for _ in range(n - 1)], bytes_
+
+
+def batch_costs(r, wl, cfg, dw):
+    chk = r.route(dw.tok, dw.tok_off, dw.req_feats, cfg.n_inst)
+    hits = chk["hits"].cpu().numpy()
+    keys, ko = r.hash_blocks(dw.tok, dw.tok_off)
+    return route_costs(cfg, cfg.n_req, cfg.n_inst, hits, np.diff(wl.tok_off), keys.cpu().numpy(), ko.cpu().numpy())
+
+
+def measure_route(name, L, H, W, dev, stream, peaks, peak_src, steps, warmup, ctx=None):
+    """Route calls of one configuration alone (graph replays back to back):
+    decisions/s, scores/s, per-kernel rooflines and the route-level roofline."""
+    import torch
+    own = ctx is None
+    if own:
+        ctx = setup_config(name, H, W, dev)
+    wl, cfg, r, dw = ctx[:4]
+    R, N = cfg.n_req, cfg.n_inst
+    sets, set_bytes = input_sets(dw, INPUT_SETS_SMALL)
+    out = {"choice": torch.empty(R, dtype=torch.int32, device=dev),
+           "best": torch.empty(R, dtype=torch.float32, device=dev), "scores": None, "hits": None}
+
+    def call(k):
+        tok, off, req = sets[k % len(sets)]
+        r.route(tok, off, req, N, out=out)
+
+    for k in range(max(warmup, 2)):
+        call(k)
+    torch.cuda.synchronize()
+    graphs = [H.StepGraph(lambda k=k: call(k)) for k in range(len(sets))]
+    for k in range(warmup):
+        graphs[k % len(graphs)].replay()
+    torch.cuda.synchronize()
+    times = timed_back_to_back(lambda k: graphs[k % len(graphs)].replay(), steps, stream)
+    ms = float(np.mean(times))
+    n_tr = min(steps, 30)
+    trace = traced(L, r, call, n_tr)
+    costs = batch_costs(r, wl, cfg, dw)
+    rl = kernel_rooflines(trace, n_tr, costs, cfg, R, N, cfg.train_batch, peaks, peak_src)
+    per_call = {k: v[1] / max(v[2], 1) * v[0] / n_tr for k, v in trace.items()}
+    roof = route_roofline(costs, R, N, peaks)
+    dom = max(rl, key=lambda k: per_call.get(k, 0.0)) if rl else None
+    res = {"workload": DESC[name], "ms_per_route": ms, "decisions_per_s": R / (ms / 1e3),
+           "scores_per_s": R * N / (ms / 1e3), "route_roofline": roof,
+           "frac_of_route_roofline": (R / (ms / 1e3)) / roof["decisions_per_s"],
+           "dominant_kernel": dom, "roofline": rl.get(dom) if dom else None, "kernel_rooflines": rl,
+           "kernels_ms_per_route": per_call, "algorithmic": costs,
+           "l2": f"{len(sets)} device cop{'y' if len(sets) == 1 else 'ies'} of the batch "
+                 f"({len(sets) * set_bytes / 1e6:.0f} MB, L2 129 MB); no flush"}
+    if own:
+        r.close()
+    return res
+
+
+def measure_tiny(L, H, W, dev, stream, n=200):
+    """The tiny configuration is latency-bound: the device time of one route
+    call and of one replay of it captured in a graph."""
+    import torch
+    wl, cfg, r, dw = setup_config("tiny", H, W, dev)[:4]
+    out = {"choice": torch.empty(cfg.n_req, dtype=torch.int32, device=dev),
+           "best": torch.empty(cfg.n_req, device=dev), "scores": None, "hits": None}
+    call = lambda: r.route(dw.tok, dw.tok_off, dw.req_feats, cfg.n_inst, out=out)
+    for _ in range(5):
+        call()
+    torch.cuda.synchronize()
+    g = H.StepGraph(call)
+
+    def lat(fn):
+        ts = []
+        for _ in range(n):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            fn()
+            e1.record(stream)
+            e1.synchronize()
+            ts.append(1e3 * e0.elapsed_time(e1))
+        return {"p50": float(np.percentile(ts, 50)), "p99": float(np.percentile(ts, 99))}
+    res = {"workload": DESC["tiny"], "route_device_us": lat(call), "route_graph_replay_us": lat(g.replay),
+           "roofline": "n/a: latency-bound (512 scores, 5.3 MFLOP: under a microsecond at any ceiling)"}
+    r.close()
+    return res
+
+
+def measure_probes(L, dev, stream, peaks, sms):
+    """Ceilings on this GPU: random 8-byte gathers from a table in L2 (32 MB) and
+    in HBM (4 GB), fp32 FMA issue (with the SM count x 128 lanes x 2 x clock
+    figure beside it) and streaming L2 reads (64 MB buffer)."""
+    import torch
+
+    def timed(fn, reps=10):
+        fn()
+        torch.cuda.synchronize()
+        ts = []
+        for _ in range(reps):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            fn()
+            e1.record(stream)
+            e1.synchronize()
+            ts.append(e0.elapsed_time(e1))
+        return float(np.median(ts))
+
+    res = {}
+    blocks = 8 * sms
+    out = torch.empty(blocks * 256, dtype=torch.int64, device=dev)
+    for label, nbytes in (("l2", 32 << 20), ("hbm", 4 << 30)):
+        table = torch.randint(0, 2 ** 62, (nbytes // 8,), dtype=torch.int64, device=dev)
+        per = 64
+        ms = timed(lambda: L.check(L.ls_probe_gather(table, table.numel(), blocks, per, 7, out, stream)))
+        n = blocks * 256 * per
+        res[f"gather8_{label}"] = {"table_bytes": nbytes, "lookups_per_s": n / (ms / 1e3),
+                                   "GB_per_s": 8 * n / (ms / 1e6) / 1e6, "ms": ms}
+        del table
+    f = torch.empty(4 * sms * 256, dtype=torch.float32, device=dev)
+    iters = 20000
+    ms = timed(lambda: L.check(L.ls_probe_fma(4 * sms, iters, f, stream)))
+    flops = 2 * 8 * iters * 4 * sms * 256
+    res["fp32_fma"] = {"tflops": flops / (ms / 1e3) / 1e12,
+                       "theory_tflops_at_max_clock": sms * 128 * 2 * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12}
+    buf = torch.empty(64 << 20, dtype=torch.uint8, device=dev)
+    o = torch.empty(blocks * 256 * 4, dtype=torch.int32, device=dev)
+    passes = 8
+    ms = timed(lambda: L.check(L.ls_probe_read(buf, buf.numel() // 16, passes, blocks, o, stream)))
+    res["l2_read"] = {"buffer_bytes": buf.numel(), "GB_per_s": buf.numel() * passes / (ms / 1e3) / 1e9}
+    return res
+
+
+def measure_step(name, L, H, W, dev, stream, peaks, peak_src, args, ctx, clocks=None):
+    """The whole step (snapshot state + route on one graph branch, log + train
+    on a second, joined before the publish), captured once per device copy of
+    the batch and replayed back to back; then the same steps issued call by
+    call, and a traced pass for per-kernel times."""
+    import torch
+    wl, cfg, r, dw, sx, sy = ctx
+    R, N, Bt = cfg.n_req, cfg.n_inst, cfg.train_batch
+    states = [dw.inst_state, torch.from_numpy(W.instance_state(np.random.default_rng(99), cfg)).to(dev)]
+    out = {"choice": torch.empty(R, dtype=torch.int32, device=dev),
+           "best": torch.empty(R, dtype=torch.float32, device=dev), "scores": None, "hits": None}
+    loss = torch.zeros(1, device=dev)
+    stage_state = torch.empty_like(states[0])
+    stage_x = torch.empty(Bt, cfg.d, device=dev)
+    stage_y = torch.empty(Bt, device=dev)
+    sets, set_bytes = input_sets(dw, INPUT_SETS_SMALL)
+
+    def feed(k):
+        stage_state.copy_(states[k & 1], non_blocking=True)
+        a = (k * Bt) % (len(sy) - Bt + 1)
+        stage_x.copy_(sx[a:a + Bt], non_blocking=True)
+        stage_y.copy_(sy[a:a + Bt], non_blocking=True)
+
+    side = torch.cuda.Stream(dev)  # training runs beside routing (Sec. 4.3.1: off the routing path)
+
+    def body(ks=0):
+        tok, tok_off, req = sets[ks]
+        main = torch.cuda.current_stream(dev)
+        side.wait_stream(main)                      # the step's inputs are in place
+        r.snapshot(N, stage_state)
+        r.route(tok, tok_off, req, N, out=out)
+        with torch.cuda.stream(side):
+            r.log(stage_x, stage_y)
+            r.train(Bt, None, opt="adam", lr=cfg.train_lr, loss_out=loss)
+        main.wait_stream(side)                      # both branches done, then one publish
+        r.publish()
+
+    def eager_step(k):
+        feed(k)
+        body(k % len(sets))
+
+    for k in range(args.warmup):
+        eager_step(k)
+    torch.cuda.synchronize()
+    graphs = [H.StepGraph(lambda ks=ks: body(ks)) for ks in range(len(sets))]
+
+    def step(k):
+        feed(k)
+        graphs[k % len(sets)].replay()
+
+    for k in range(args.warmup):
+        step(args.warmup + k)
+    torch.cuda.synchronize()
+    if clocks is not None:
+        clocks.start()
+    cudart = torch.cuda.cudart()
+    cudart.cudaProfilerStart()                      # brackets the region for ncu --profile-from-start off
+    times = timed_back_to_back(lambda k: step(2 * args.warmup + k), args.steps, stream)
+    cudart.cudaProfilerStop()
+    torch.cuda.synchronize()
+    clk = clocks.stop() if clocks is not None else None
+    eager_times = timed_back_to_back(lambda k: eager_step(2 * args.warmup + args.steps + k),
+                                     min(args.steps, 100), stream)
+    n_traced = min(args.steps, 60)
+    trace = traced(L, r, lambda k: eager_step(k), n_traced)
+    costs = batch_costs(r, wl, cfg, dw)
+    rl = kernel_rooflines(trace, n_traced, costs, cfg, R, N, Bt, peaks, peak_src)
+    per_step = {k: v[1] / max(v[2], 1) * v[0] / n_traced for k, v in trace.items()}
+    launches = sum(v[0] for v in trace.values()) / n_traced
+    return {"times": times, "eager_times": eager_times, "clocks": clk, "costs": costs, "rooflines": rl,
+            "kernels_ms_per_step": per_step, "launches_per_step": launches, "sets": sets, "set_bytes": set_bytes,
+            "body": body, "states": states, "out": out, "loss": loss, "side": side}
+
+
+def measure_e2e(L, H, dev, stream, args, ctx, st, world):
+    """End to end through the C ABI with host buffers: every step copies its
+    inputs from pinned host memory and reads its results back.  The copies of
+    step k+1 run on a copy stream while step k computes; device input sets
+    rotate, each with its own captured graph of the step's ABI calls."""
+    import torch
+    wl, cfg, r, dw, sx, sy = ctx
+    R, N, Bt = cfg.n_req, cfg.n_inst, cfg.train_batch
+    out, loss, side = st["out"], st["loss"], st["side"]
+    h_tok = torch.from_numpy(wl.tok).pin_memory()
+    h_off = torch.from_numpy(wl.tok_off).pin_memory()
+    h_req = torch.from_numpy(wl.req_feats).pin_memory()
+    h_st = [s_.cpu().pin_memory() for s_ in st["states"]]
+    h_x = sx[:8 * Bt].cpu().pin_memory()
+    h_y = sy[:8 * Bt].cpu().pin_memory()
+    NB = 3 if h_tok.numel() * 4 > 300e6 else 4
+    sets = [{"tok": torch.empty_like(dw.tok), "off": torch.empty_like(dw.tok_off),
+             "req": torch.empty_like(dw.req_feats), "st": torch.empty_like(st["states"][0]),
+             "x": torch.empty(Bt, cfg.d, device=dev), "y": torch.empty(Bt, device=dev)} for _ in range(NB)]
+    h_choice = torch.empty(R, dtype=torch.int32).pin_memory()
+    h_best = torch.empty(R, dtype=torch.float32).pin_memory()
+    h_loss = torch.empty(1).pin_memory()
+    d0 = sets[0]
+    h2d = sum(d0[k].numel() * d0[k].element_size() for k in ("tok", "off", "req", "st", "x", "y"))
+    d2h = R * 4 + R * 4 + 4
+    cs = torch.cuda.Stream(dev)
+
+    def e2e_body(ds):
+        main = torch.cuda.current_stream(dev)
+        side.wait_stream(main)
+        r.snapshot(N, ds["st"])
+        r.route(ds["tok"], ds["off"], ds["req"], N, out=out)
+        with torch.cuda.stream(side):
+            r.log(ds["x"], ds["y"])
+            r.train(Bt, None, opt="adam", lr=cfg.train_lr, loss_out=loss)
+        main.wait_stream(side)
+        r.publish()
+
+    def copy_in(k, ds):
+        a = (k * Bt) % (7 * Bt)
+        ds["tok"].copy_(h_tok, non_blocking=True)
+        ds["off"].copy_(h_off, non_blocking=True)
+        ds["req"].copy_(h_req, non_blocking=True)
+        ds["st"].copy_(h_st[k & 1], non_blocking=True)
+        ds["x"].copy_(h_x[a:a + Bt], non_blocking=True)
+        ds["y"].copy_(h_y[a:a + Bt], non_blocking=True)
+
+    def copy_out():
+        h_choice.copy_(out["choice"], non_blocking=True)
+        h_best.copy_(out["best"], non_blocking=True)
+        h_loss.copy_(loss, non_blocking=True)
+
+    for k in range(max(args.warmup, NB)):
+        copy_in(k, sets[k % NB])
+        e2e_body(sets[k % NB])
+        copy_out()
+    torch.cuda.synchronize()
+    graphs = [H.StepGraph(lambda ds=ds: e2e_body(ds)) for ds in sets]
+    copied = [torch.cuda.Event() for _ in range(NB)]
+    free = [torch.cuda.Event() for _ in range(NB)]
+
+    def run_pipelined(k0, K):
+        main = torch.cuda.current_stream(dev)
+        for b in range(NB):
+            free[b].record(main)
+        for k in range(k0, k0 + K):
+            b = k % NB
+            cs.wait_event(free[b])            # the graph that last read this input set is done
+            with torch.cuda.stream(cs):
+                copy_in(k, sets[b])
+                copied[b].record(cs)
+            main.wait_event(copied[b])
+            graphs[b].replay()
+            free[b].record(main)
+            copy_out()
+
+    run_pipelined(0, 2 * NB)                 # warm the pipeline and the graphs
+    torch.cuda.synchronize()
+    K = min(args.steps, 100)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    cs.wait_stream(stream)
+    e0.record(stream)
+    run_pipelined(2 * NB, K)
+    e1.record(stream)
+    e1.synchronize()
+    ems = max_over_ranks(world, e0.elapsed_time(e1) / K, None)
+    return {"value": world * R / (ems / 1e3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+            "d2h_bytes_per_step": int(d2h), "ms_per_step": ems, "steps": K,
+            "pipelined": f"inputs of step k+1 copied on a copy stream while step k computes; {NB} device input sets "
+                         f"with a captured graph each; choices, best scores and loss read back every step"}
+
 
 def main():
     args = parse()
@@ -586,328 +1045,109 @@ def main():
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     B.build()
-    wl = W.generate(WORKLOAD)
-    cfg = wl.cfg
-    R, N, Bt = cfg.n_req, cfg.n_inst, cfg.train_batch
-    ring = max(cfg.n_samples, 4 * Bt)
-    r = H.Router.for_config(cfg, ring_capacity=ring)
-    dw = H.DeviceWorkload(wl, device=dev)
-    dw.load(r)
-    sx = torch.from_numpy(wl.samples_x).to(dev)
-    sy = torch.from_numpy(wl.samples_y).to(dev)
-    r.log(sx, sy)                                   # fill the ring once
-    states = [dw.inst_state, torch.from_numpy(W.instance_state(np.random.default_rng(99), cfg)).to(dev)]
-    out = {"choice": torch.empty(R, dtype=torch.int32, device=dev),
-           "best": torch.empty(R, dtype=torch.float32, device=dev), "scores": None, "hits": None}
-    loss = torch.zeros(1, device=dev)
-    flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
-    if args.paper_point_only:
-        pp = measure_paper_point(L, H, W, dev, stream)
+    peaks, peak_src = measured_peaks()
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
+
+    if args.route_only:
+        res = measure_route(args.route_only, L, H, W, dev, stream, peaks, peak_src, args.steps, args.warmup)
         if rank == 0:
-            print(json.dumps({"paper_point": pp}))
+            print(json.dumps({"route_only": args.route_only, **res}))
+        return 0
+    if args.paper_point_only or args.replay_only or args.guards_only:
+        wl, cfg, r, dw = setup_config("homogeneous", H, W, dev)[:4]
+        if args.paper_point_only:
+            res = {"paper_point": measure_paper_point(L, H, W, dev, stream)}
+        elif args.replay_only:
+            res = {"workload": "homogeneous",
+                   "replay_admission": measure_replay(L, H, W, wl, dev, flush, stream, peaks, n=max(args.steps, 4))}
+        else:
+            res = {"workload": "homogeneous", "guarded_route": measure_guards(
+                L, r, dw, cfg.n_inst, cfg.n_req, cfg.d, int(min(65536, r.info().ring_count)), cfg.d_req, flush,
+                stream, peaks, n=max(args.steps, 4))}
+        if rank == 0:
+            print(json.dumps(res))
         r.close()
         return 0
-    if args.replay_only:
-        rp = measure_replay(L, H, W, wl, dev, flush, stream, measured_peaks()[0], n=max(args.steps, 4))
-        if rank == 0:
-            print(json.dumps({"workload": WORKLOAD, "replay_admission": rp}))
-        r.close()
-        return 0
-    if args.guards_only:
-        g = measure_guards(L, r, dw, N, R, cfg.d, min(ring, int(r.info().ring_count)), cfg.d_req, flush, stream,
-                           measured_peaks()[0], n=max(args.steps, 4))
-        if rank == 0:
-            print(json.dumps({"workload": WORKLOAD, "guarded_route": g}))
-        r.close()
-        return 0
-    # the step's inputs arrive in fixed buffers (new instance state, new logged records)
-    stage_state = torch.empty_like(states[0])
-    stage_x = torch.empty(Bt, cfg.d, device=dev)
-    stage_y = torch.empty(Bt, device=dev)
 
-    def feed(k):
-        stage_state.copy_(states[k & 1], non_blocking=True)
-        a = (k * Bt) % len(wl.samples_y)
-        stage_x.copy_(sx[a:a + Bt], non_blocking=True)
-        stage_y.copy_(sy[a:a + Bt], non_blocking=True)
-
-    side = torch.cuda.Stream(dev)  # training runs beside routing (Sec. 4.3.1: off the routing path)
-    # device copies of the batch, larger than L2 together: consecutive steps
-    # read their prompts from different copies, so every step's inputs come
-    # from HBM (no L2 flush needed between steps)
-    n_sets = INPUT_SETS
-    sets = [(dw.tok, dw.tok_off, dw.req_feats)] + [
-        (dw.tok.clone(), dw.tok_off.clone(), dw.req_feats.clone()) for _ in range(n_sets - 1)]
-    set_bytes = sum(t.numel() * t.element_size() for t in sets[0])
-
-    def body(ks=0):
-        tok, tok_off, req = sets[ks]
-        main = torch.cuda.current_stream(dev)
-        side.wait_stream(main)                      # the step's inputs are in place
-        r.snapshot(N, stage_state)
-        r.route(tok, tok_off, req, N, out=out)
-        with torch.cuda.stream(side):
-            r.log(stage_x, stage_y)
-            r.train(Bt, None, opt="adam", lr=cfg.train_lr, loss_out=loss)
-        main.wait_stream(side)                      # both branches done, then one publish
-        r.publish()
-
-    def eager_step(k):
-        feed(k)
-        body(k % n_sets)
-
-    for k in range(args.warmup):
-        eager_step(k)
-    torch.cuda.synchronize()
-    graphs = [H.StepGraph(lambda ks=ks: body(ks)) for ks in range(n_sets)]  # the step's ABI calls, recorded once
-
-    def step(k):
-        feed(k)
-        graphs[k % n_sets].replay()
-
-    for k in range(args.warmup):
-        step(args.warmup + k)
-    torch.cuda.synchronize()
-    # per-pair hits of this batch (for the algorithmic byte count; not timed)
-    chk = r.route(dw.tok, dw.tok_off, dw.req_feats, N)
-    hits = chk["hits"].cpu().numpy()
-    keys, ko = r.hash_blocks(dw.tok, dw.tok_off)
-    costs = route_costs(cfg, R, N, hits, np.diff(wl.tok_off), keys.cpu().numpy(), ko.cpu().numpy())
-
+    # ---- the headline: whole steps of the large configuration -------------
+    ctx = setup_config(WORKLOAD, H, W, dev)
+    wl, cfg, r = ctx[0], ctx[1], ctx[2]
+    R, N, Bt = cfg.n_req, cfg.n_inst, cfg.train_batch
     uuid = None
     try:
         uuid = str(torch.cuda.get_device_properties(dev).uuid)
     except Exception:
         pass
-    clocks = ClockSampler(uuid)
-    cudart = torch.cuda.cudart()
-
-    def timed_pass(fn, k0, n=None):
-        # steps issued back to back, an event between consecutive steps: the
-        # host stays ahead of the GPU, so each interval is one step's device time
-        n = args.steps if n is None else n
-        ev = [torch.cuda.Event(enable_timing=True) for _ in range(n + 1)]
-        ev[0].record(stream)
-        for k in range(n):
-            fn(k0 + k)
-            ev[k + 1].record(stream)
-        ev[n].synchronize()
-        return [ev[k].elapsed_time(ev[k + 1]) for k in range(n)]
-
-    # timed region: K whole steps (graph replays), no per-kernel instrumentation
     barrier(world)
     torch.cuda.synchronize()
-    clocks.start()
-    cudart.cudaProfilerStart()                      # brackets the region for ncu --profile-from-start off
-    times = timed_pass(step, 2 * args.warmup)
-    cudart.cudaProfilerStop()
-    torch.cuda.synchronize()
-    clk = clocks.stop()
-    # the same K steps issued call by call (no graph), for comparison
-    eager_times = timed_pass(eager_step, 2 * args.warmup + args.steps)
-    # and steps issued call by call with every kernel launch bracketed by CUDA
-    # events on its launching stream: per-kernel device time for the roofline
-    L.ls_trace_enable(r.h, True)
-    L.ls_trace_read(r.h)
-    torch.cuda.synchronize()
-    n_traced = min(args.steps, 120)                 # every launch gets events from the tracer's pool
-
-    # each traced step behind a ~150 us spin on the GPU, so that the host has
-    # queued the whole step before it starts and no kernel interval includes
-    # host time; the step's interval excludes the spin
-    tev = []
-    for k in range(n_traced):
-        torch.cuda._sleep(300000)
-        e0 = torch.cuda.Event(enable_timing=True)
-        e1 = torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        eager_step(2 * args.warmup + 2 * args.steps + k)
-        e1.record(stream)
-        tev.append((e0, e1))
-    torch.cuda.synchronize()
-    traced_times = [a.elapsed_time(b) for a, b in tev]
-    torch.cuda.synchronize()
-    rc, trace = L.ls_trace_read(r.h)
-    L.ls_trace_enable(r.h, False)
+    st = measure_step(WORKLOAD, L, H, W, dev, stream, peaks, peak_src, args, ctx, clocks=ClockSampler(uuid))
     barrier(world)
-    ms = max_over_ranks(world, float(np.mean(times)), dev if world > 1 and torch.distributed.get_backend() == "nccl" else None)
+    ms = max_over_ranks(world, float(np.mean(st["times"])),
+                        dev if world > 1 and torch.distributed.get_backend() == "nccl" else None)
     value = world * R / (ms / 1e3)
+    rl = st["rooflines"]
+    route_k = [k for k in rl if k in ("prefix_index", "prefix_match", "features", "score_tc", "score_simt")]
+    dom = max(route_k, key=lambda k: st["kernels_ms_per_step"][k])
+    roofline = dict(rl[dom], branch="route (the step's critical branch)")
+    train_k = [k for k in rl if k.startswith("gemm_tc")]
+    train_roofline = (dict(rl[max(train_k, key=lambda k: st["kernels_ms_per_step"][k])], branch="train")
+                      if train_k else None)
+    roof = route_roofline(st["costs"], R, N, peaks)
+    kms = st["kernels_ms_per_step"]
+    launches_per_step = st["launches_per_step"]
+    clk = st["clocks"]
+    costs = st["costs"]
+    eager_ms = float(np.mean(st["eager_times"]))
 
-    # roofline of the dominant kernel: the largest device time per step on the
-    # step's critical branch (snapshot + route runs beside log + train, and is
-    # the longer branch); the training branch's largest kernel is reported too
-    peaks, peak_src = measured_peaks()
-    per = {k: v[1] / max(v[2], 1) for k, v in trace.items()}          # ms per timed launch
-    per_step = {k: per[k] * v[0] / n_traced for k, v in trace.items()}  # ms per step
-    n_per_step = {k: v[0] / n_traced for k, v in trace.items()}         # launches per step
-    launches = int(round(sum(v[0] for v in trace.values()) * args.steps / n_traced))
-    timing = ("kernel durations from CUDA events around each launch over steps issued call by call "
-              "(instrumented); value and ms_per_step from the K graph replays")
-
-    def kernel_roofline(k):
-        d_pad = 64 * ((cfg.d + 63) // 64)
-        if k in ("prefix_index", "prefix_match"):
-            alg, peak, unit, bound = costs["prefix_bytes"] / 1e9, peaks["hbm_gbs"], "GB/s", "hbm"
-        elif k == "features":     # feature image written + hits and offsets read
-            alg = (R * N * (2 * d_pad + 4) + R * 8) / 1e9
-            peak, unit, bound = peaks["hbm_gbs"], "GB/s", "hbm"
-        elif k in ("score_simt", "score_tc"):
-            alg, peak, unit, bound = costs["score_flops"] / 1e12, peaks["bf16_tflops"], "TFLOP/s", "tensor"
-        else:                      # training products: the kind's flops per step over its launches per step
-            # forward launches: every layer's product plus the output layer's dW
-            # (in the last hidden layer's epilogue); dW + dX launches for hidden
-            # layers l >= 1; the dW-only launch for layer 0
-            w, Bk = cfg.widths, Bt
-            nh = len(w) - 2
-            per_kind = {"gemm_tc_fwd": sum(2 * Bk * w[l] * w[l + 1] for l in range(nh + 1)) + 2 * Bk * w[nh],
-                        "gemm_tc_dx": sum(4 * Bk * w[l] * w[l + 1] for l in range(1, nh)),
-                        "gemm_tc_dw": 2 * Bk * w[0] * w[1]}
-            alg = per_kind.get(k, 0.0) / max(n_per_step[k], 1e-9) / 1e12
-            peak, unit, bound = peaks["bf16_tflops"], "TFLOP/s", "tensor"
-        achieved = alg / (per[k] / 1e3)
-        return {"kernel": k, "bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
-                "frac": achieved / peak, "traffic": profiled_traffic(k),
-                "peak_source": f"{peak_src} (burst)", "avg_launch_ms": per[k], "timing": timing}
-
-    route_kernels = [k for k in per_step if k in ("prefix_index", "prefix_match", "hash_screen", "probe_walk",
-                                                  "features", "score_tc", "score_simt", "argmin")]
-    dom = max(route_kernels, key=lambda k: per_step[k])
-    roofline = dict(kernel_roofline(dom), branch="route (the step's critical branch)")
-    route_rooflines = {k: kernel_roofline(k) for k in route_kernels}
-    train_kernels = [k for k in per_step if k in ("gemm_tc_fwd", "gemm_tc_dw", "gemm_tc_dx")]
-    train_roofline = (dict(kernel_roofline(max(train_kernels, key=lambda k: per_step[k])), branch="train")
-                      if train_kernels else None)
-
-    training_config = None
-    if not args.no_training_config:
-        training_config = measure_training_config(L, H, W, dev)
-    paper_point = None
-    if not args.no_paper_point:
-        paper_point = measure_paper_point(L, H, W, dev, stream)
-    replay = None
-    if not args.no_replay:
-        replay = measure_replay(L, H, W, wl, dev, flush, stream, peaks)
-    guards = None
-    if not args.no_guards:
-        guards = measure_guards(L, r, dw, N, R, cfg.d, min(ring, int(r.info().ring_count)), cfg.d_req, flush,
-                                stream, peaks)
-
-    # end to end through the C ABI with host buffers: every step copies its
-    # inputs from pinned host memory and reads its results back.  The copies
-    # of step k+1 run on a copy stream while step k computes (the host link,
-    # ~205 GB/s, is the limit: 35 MB of prompt tokens per step); four device
-    # input sets (140 MB, larger than L2) rotate, each with its own captured
-    # graph of the step's ABI calls.
     e2e = None
     if not args.no_e2e:
-        h_tok = torch.from_numpy(wl.tok).pin_memory()
-        h_off = torch.from_numpy(wl.tok_off).pin_memory()
-        h_req = torch.from_numpy(wl.req_feats).pin_memory()
-        h_st = [s.cpu().pin_memory() for s in states]
-        h_x = torch.from_numpy(wl.samples_x).pin_memory()
-        h_y = torch.from_numpy(wl.samples_y).pin_memory()
-        NB = 4
-        sets = [{"tok": torch.empty_like(dw.tok), "off": torch.empty_like(dw.tok_off),
-                 "req": torch.empty_like(dw.req_feats), "st": torch.empty_like(states[0]),
-                 "x": torch.empty(Bt, cfg.d, device=dev), "y": torch.empty(Bt, device=dev)} for _ in range(NB)]
-        h_choice = torch.empty(R, dtype=torch.int32).pin_memory()
-        h_best = torch.empty(R, dtype=torch.float32).pin_memory()
-        h_loss = torch.empty(1).pin_memory()
-        d0 = sets[0]
-        h2d = d0["tok"].numel() * 4 + d0["off"].numel() * 8 + d0["req"].numel() * 4 + d0["st"].numel() * 4 + \
-            d0["x"].numel() * 4 + d0["y"].numel() * 4
-        d2h = R * 4 + R * 4 + 4
-        cs = torch.cuda.Stream(dev)
-
-        def e2e_body(ds):
-            main = torch.cuda.current_stream(dev)
-            side.wait_stream(main)
-            r.snapshot(N, ds["st"])
-            r.route(ds["tok"], ds["off"], ds["req"], N, out=out)
-            with torch.cuda.stream(side):
-                r.log(ds["x"], ds["y"])
-                r.train(Bt, None, opt="adam", lr=cfg.train_lr, loss_out=loss)
-            main.wait_stream(side)
-            r.publish()
-
-        def copy_in(k, ds):
-            a = (k * Bt) % len(wl.samples_y)
-            ds["tok"].copy_(h_tok, non_blocking=True)
-            ds["off"].copy_(h_off, non_blocking=True)
-            ds["req"].copy_(h_req, non_blocking=True)
-            ds["st"].copy_(h_st[k & 1], non_blocking=True)
-            ds["x"].copy_(h_x[a:a + Bt], non_blocking=True)
-            ds["y"].copy_(h_y[a:a + Bt], non_blocking=True)
-
-        def copy_out():
-            h_choice.copy_(out["choice"], non_blocking=True)
-            h_best.copy_(out["best"], non_blocking=True)
-            h_loss.copy_(loss, non_blocking=True)
-
-        for k in range(args.warmup):
-            copy_in(k, sets[k % NB])
-            e2e_body(sets[k % NB])
-            copy_out()
-        torch.cuda.synchronize()
-        graphs = [H.StepGraph(lambda ds=ds: e2e_body(ds)) for ds in sets]
-        copied = [torch.cuda.Event() for _ in range(NB)]
-        free = [torch.cuda.Event() for _ in range(NB)]
-
-        def run_pipelined(k0, K):
-            main = torch.cuda.current_stream(dev)
-            for b in range(NB):
-                free[b].record(main)
-            for k in range(k0, k0 + K):
-                b = k % NB
-                cs.wait_event(free[b])            # the graph that last read this input set is done
-                with torch.cuda.stream(cs):
-                    copy_in(k, sets[b])
-                    copied[b].record(cs)
-                main.wait_event(copied[b])
-                graphs[b].replay()
-                free[b].record(main)
-                copy_out()
-
-        run_pipelined(0, 2 * NB)                 # warm the pipeline and the graphs
-        torch.cuda.synchronize()
-        e0 = torch.cuda.Event(enable_timing=True)
-        e1 = torch.cuda.Event(enable_timing=True)
-        cs.wait_stream(stream)
-        e0.record(stream)
-        run_pipelined(2 * NB, args.steps)
-        e1.record(stream)
-        e1.synchronize()
-        ems_pipe = e0.elapsed_time(e1) / args.steps
-        # the same steps one at a time (copy in, step, copy out; L2 flushed between)
-        et = []
-        for k in range(min(args.steps, 200)):
-            flush.fill_(k & 0xFF)
-            b = k % NB
-            e0 = torch.cuda.Event(enable_timing=True)
-            e1 = torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-            copy_in(k, sets[b])
-            graphs[b].replay()
-            copy_out()
-            e1.record(stream)
-            e1.synchronize()
-            et.append(e0.elapsed_time(e1))
-        ems = max_over_ranks(world, ems_pipe, None)
-        e2e = {"value": world * R / (ems / 1e3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
-               "d2h_bytes_per_step": int(d2h), "ms_per_step": ems,
-               "pipelined": "inputs of step k+1 copied on a copy stream while step k computes; 4 device "
-                            "input sets with a captured graph each; results read back every step",
-               "ms_per_step_one_at_a_time": float(np.mean(et))}
-
+        e2e = measure_e2e(L, H, dev, stream, args, ctx, st, world)
+    large_route = measure_route(WORKLOAD, L, H, W, dev, stream, peaks, peak_src, min(args.steps, 50),
+                                args.warmup, ctx=ctx)
     status = r.sync()
     if status != L.LS_OK:
         print(json.dumps({"error": f"device status {status}"}), file=sys.stderr)
+    del st
+    r.close()
+    torch.cuda.empty_cache()
+
+    # ---- every other configuration, each with its own roofline ------------
+    configs = {"large": {"route_only": large_route}}
+    probes = None
+    if not args.no_probes:
+        probes = measure_probes(L, dev, stream, peaks, sms)
+    if not args.no_configs:
+        configs["tiny"] = measure_tiny(L, H, W, dev, stream)
+        hctx = setup_config("homogeneous", H, W, dev)
+        hst = measure_step("homogeneous", L, H, W, dev, stream, peaks, peak_src, args, hctx)
+        configs["homogeneous"] = {
+            "route_only": measure_route("homogeneous", L, H, W, dev, stream, peaks, peak_src, args.steps,
+                                        args.warmup, ctx=hctx),
+            "step": {"ms_per_step": float(np.mean(hst["times"])),
+                     "decisions_per_s": hctx[1].n_req / (float(np.mean(hst["times"])) / 1e3),
+                     "kernels_ms_per_step": hst["kernels_ms_per_step"],
+                     "what": "snapshot + route beside log + train (Adam, batch 4096), then publish, graph replays"}}
+        del hst
+        if not args.no_guards:
+            hw, hc, hr, hd = hctx[:4]
+            configs["homogeneous"]["guarded_route"] = measure_guards(
+                L, hr, hd, hc.n_inst, hc.n_req, hc.d, int(min(65536, hr.info().ring_count)), hc.d_req, flush,
+                stream, peaks)
+        if not args.no_replay:
+            configs["homogeneous"]["replay_admission"] = measure_replay(L, H, W, hctx[0], dev, flush, stream, peaks)
+        hctx[2].close()
+        configs["heterogeneous"] = {"route_only": measure_route("heterogeneous", L, H, W, dev, stream, peaks,
+                                                                peak_src, min(args.steps, 100), args.warmup)}
+        if not args.no_training_config:
+            configs["training"] = measure_training_config(L, H, W, dev)
+        if not args.no_paper_point:
+            configs["paper_point"] = measure_paper_point(L, H, W, dev, stream)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        import oracle
-        cpu = cpu_baseline(wl, oracle.instance_keys(wl), args.cpu_seconds)
+        cpu = cpu_baseline(wl, oracle_setup(wl), args.cpu_seconds, WORKLOAD)
 
     if rank == 0:
         line = {
@@ -915,38 +1155,33 @@ def main():
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic (seeded generator shaped like the paper's prefix-sharing workloads)",
-            "config": {"workload": WORKLOAD_DESC,
-                       "pairs_per_step": R * N, "train_samples_per_step": Bt,
-                       "l2": f"inputs larger than L2: consecutive steps read {n_sets} rotating device copies of "
-                             f"the batch ({n_sets * set_bytes / 1e6:.0f} MB in all, L2 129 MB); no flush",
+            "config": {"workload": DESC[WORKLOAD], "pairs_per_step": R * N, "train_samples_per_step": Bt,
+                       "l2": "inputs larger than L2: 541 MB of prompt tokens per batch (L2 129 MB); no flush",
                        "parallelism": "replicas"},
-            "train_samples_per_s": world * Bt / (ms / 1e3),
             "scores_per_s": world * R * N / (ms / 1e3),
+            "train_samples_per_s": world * Bt / (ms / 1e3),
             "roofline": roofline,
+            "route_roofline": dict(roof, frac_of_rate=value / world / roof["decisions_per_s"],
+                                   what="sum over phases of max(bytes / measured HBM, factorised flops / measured "
+                                        "bf16): the step's decisions/s against the route's roofline rate"),
             "train_roofline": train_roofline,
-            "kernels_ms_per_step": {k: per_step[k] for k in sorted(per_step, key=lambda k: -per_step[k])},
+            "kernel_rooflines": rl,
+            "kernels_ms_per_step": {k: v for k, v in sorted(kms.items(), key=lambda kv: -kv[1])},
             "cpu_baseline": cpu,
             "e2e": e2e,
-            "gpu_launches": launches,
-            "launch": "each step: the new instance state and records copied into the step's buffers, then "
-                      "one replay of a CUDA graph of the step's ABI calls recorded once per device copy of the "
-                      "batch (steps rotate over the copies): snapshot + route on one branch, log + train on a "
-                      "second, joined before the publish; kernels of each chain launched with programmatic "
+            "gpu_launches": int(round(launches_per_step * args.steps)),
+            "gpu_launches_per_step": launches_per_step,
+            "launch": "each step: the new instance state and records copied into the step's buffers, then one "
+                      "replay of a CUDA graph of the step's ABI calls: snapshot + route on one branch, log + train "
+                      "on a second, joined before the publish; kernels of each chain launched with programmatic "
                       "dependent launch",
-            "ms_per_step_eager": float(np.mean(eager_times)),
-            "ms_per_step_instrumented": float(np.mean(traced_times)),
-            "instrumented_steps": n_traced,
-            "gpu_launches_per_step": launches / args.steps,
+            "ms_per_step_eager": eager_ms,
             "clocks": clk,
             "algorithmic": costs,
-            "guarded_route": guards,
-            "replay_admission": replay,
-            "route_rooflines": route_rooflines,
-            "paper_point": paper_point,
-            "training_config": training_config,
+            "ceilings": probes,
+            "configs": configs,
         }
         print(json.dumps(line))
-    r.close()
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()

@@ -59,6 +59,7 @@ def lib():
             L.or_hash_blocks.argtypes = [i64, P, P, P, P]
             L.or_prefix_hits.argtypes = [i64, P, P, i32, P, P, P]
             L.or_prefix_hits_by_marking.argtypes = [i64, P, P, i32, P, P, P]
+            L.or_prefix_hits_sorted.argtypes = [i64, P, P, i32, P, P, P]
             L.or_raw_features_row.argtypes = [i64, i32, P, C.c_int, P, C.c_int, P]
             L.or_raw_features_row.restype = None
             L.or_features.argtypes = [i64, i32, P, P, P, C.c_int, P, C.c_int, P, P, P]
@@ -162,6 +163,28 @@ def prefix_hits(req_keys, req_key_off, inst_keys, inst_key_off, by_marking: bool
     return hits
 
 
+def sorted_instance_keys(inst_keys):
+    """Each instance's key set sorted ascending (CSR), built once like the
+    router's snapshot tables; route() then probes it without re-sorting."""
+    ik, iko = inst_keys
+    out = np.empty_like(ik)
+    for i in range(len(iko) - 1):
+        out[iko[i]:iko[i + 1]] = np.sort(ik[iko[i]:iko[i + 1]])
+    return out, iko
+
+
+def prefix_hits_sorted(req_keys, req_key_off, sorted_keys):
+    rk = _c(req_keys, np.uint64) if len(req_keys) else np.zeros(1, np.uint64)
+    rko = _c(req_key_off, np.int64)
+    sk, sko = sorted_keys
+    sk = _c(sk, np.uint64) if len(sk) else np.zeros(1, np.uint64)
+    sko = _c(sko, np.int64)
+    R, N = len(rko) - 1, len(sko) - 1
+    hits = np.zeros((R, N), np.int32)
+    _check(lib().or_prefix_hits_sorted(R, _p(rk), _p(rko), N, _p(sk), _p(sko), _p(hits)), "prefix_hits_sorted")
+    return hits
+
+
 def instance_keys(wl, seq_keys=None, seq_key_off=None):
     """Key multiset of every instance of a workload: the oracle's own hash of
     the cached chains (first k blocks of a cached sequence) plus the
@@ -259,7 +282,8 @@ def argmin(scores):
     return choice, best
 
 
-def route(wl, hits=None, inst_keys=None, params=None, mode=None, req_idx=None, bounds=False, threads=1):
+def route(wl, hits=None, inst_keys=None, params=None, mode=None, req_idx=None, bounds=False, threads=1,
+          inst_sorted=None):
     """Full oracle route of (a subset of) a workload's requests.
     Returns dict(hits, scores, choice, best); with bounds, also the per-score
     rounding analysis of mlp_forward_bounds (ebound, flip).  threads > 1 splits
@@ -269,12 +293,12 @@ def route(wl, hits=None, inst_keys=None, params=None, mode=None, req_idx=None, b
         import concurrent.futures as cf
         R_all = len(wl.tok_off) - 1
         idx = np.arange(R_all) if req_idx is None else np.asarray(req_idx)
-        if inst_keys is None:
+        if inst_keys is None and inst_sorted is None and hits is None:
             inst_keys = instance_keys(wl)
         parts = [p for p in np.array_split(np.arange(len(idx)), threads) if len(p)]
         with cf.ThreadPoolExecutor(max_workers=len(parts)) as ex:
             res = list(ex.map(lambda p: route(wl, None if hits is None else hits[p], inst_keys, params, mode,
-                                              idx[p], bounds, 1), parts))
+                                              idx[p], bounds, 1, inst_sorted), parts))
         out = {k: np.concatenate([r[k] for r in res]) for k in res[0]}
         out["choice"], out["best"] = argmin(out["scores"])
         return out
@@ -289,10 +313,13 @@ def route(wl, hits=None, inst_keys=None, params=None, mode=None, req_idx=None, b
         sub_off[1:] = np.cumsum([len(s) for s in seqs])
         sub_tok = np.concatenate(seqs) if seqs else np.zeros(0, np.int32)
         rk, rko = hash_blocks(sub_tok, sub_off)
-        if inst_keys is None:
-            inst_keys = instance_keys(wl)
-        ik, iko = inst_keys
-        hits = prefix_hits(rk, rko, ik, iko, by_marking=len(idx) * 64 < len(ik))
+        if inst_sorted is not None:
+            hits = prefix_hits_sorted(rk, rko, inst_sorted)
+        else:
+            if inst_keys is None:
+                inst_keys = instance_keys(wl)
+            ik, iko = inst_keys
+            hits = prefix_hits(rk, rko, ik, iko, by_marking=len(idx) * 64 < len(ik))
     L = np.diff(wl.tok_off)[idx]
     x = features(L, hits, wl.inst_state, wl.req_feats[idx], wl.mean, wl.std)
     p = wl.params if params is None else params

@@ -145,6 +145,27 @@ int or_prefix_hits(int64_t n_req, const uint64_t *req_keys, const int64_t *req_k
     return 0;
 }
 
+/* The same h[r, i] against instance key sets given sorted ascending (built
+ * once, as the router's snapshot tables are, outside the routing call).
+ * Returns -2 if a set is not sorted. */
+int or_prefix_hits_sorted(int64_t n_req, const uint64_t *req_keys, const int64_t *req_key_off,
+                          int32_t n_inst, const uint64_t *sorted_keys, const int64_t *sorted_off,
+                          int32_t *hits) {
+    for (int32_t i = 0; i < n_inst; ++i) {
+        const uint64_t *set = sorted_keys + sorted_off[i];
+        int64_t n = sorted_off[i + 1] - sorted_off[i];
+        for (int64_t q = 1; q < n; ++q)
+            if (set[q - 1] > set[q]) return -2;
+        for (int64_t r = 0; r < n_req; ++r) {
+            int64_t nb = req_key_off[r + 1] - req_key_off[r];
+            int64_t b = 0;
+            while (b < nb && n > 0 && contains(set, n, req_keys[req_key_off[r] + b])) ++b;
+            hits[r * n_inst + i] = (int32_t)b;
+        }
+    }
+    return 0;
+}
+
 /* Same result, organised for few requests against huge instance sets: the
  * request keys are sorted once and every instance key is looked up among
  * them, marking (request block, instance) pairs that are cached. */

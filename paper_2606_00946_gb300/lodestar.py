@@ -88,6 +88,10 @@ _SIGS = {
     "ls_trace_enable": (C.c_int, [_P, _i32]),
     "ls_trace_read": (C.c_int, [_P, C.POINTER(ls_trace_entry), _i32, C.POINTER(_i32)]),
     "ls_prefix_hits_static": (C.c_int, [_i32, _P, _P, _i64, _P, _i64, _i32, _P, _P]),
+    # measurement kernels of include/lodestar_probe.h
+    "ls_probe_gather": (C.c_int, [_P, _i64, _i32, _i32, C.c_uint64, _P, _P]),
+    "ls_probe_fma": (C.c_int, [_i32, _i64, _P, _P]),
+    "ls_probe_read": (C.c_int, [_P, _i64, _i32, _i32, _P, _P]),
 }
 
 _lib = None
@@ -321,3 +325,16 @@ def ls_prefix_hits_static(n_req, tok, tok_off, n_tokens, tables, slots_per_insta
     return lib().ls_prefix_hits_static(int(n_req), ptr(tok), ptr(tok_off), int(n_tokens), ptr(tables),
                                        int(slots_per_instance), int(n_inst), ptr(hits_out),
                                        stream_handle(stream))
+
+
+def ls_probe_gather(table, n_slots, blocks, per_thread, seed, out, stream=None) -> int:
+    return lib().ls_probe_gather(ptr(table), int(n_slots), int(blocks), int(per_thread), int(seed), ptr(out),
+                                 stream_handle(stream))
+
+
+def ls_probe_fma(blocks, iters, out, stream=None) -> int:
+    return lib().ls_probe_fma(int(blocks), int(iters), ptr(out), stream_handle(stream))
+
+
+def ls_probe_read(buf, n16, passes, blocks, out, stream=None) -> int:
+    return lib().ls_probe_read(ptr(buf), int(n16), int(passes), int(blocks), ptr(out), stream_handle(stream))

@@ -10,11 +10,13 @@ import pytest
 from paper_2606_00946_gb300 import build as B
 from paper_2606_00946_gb300 import lodestar as L
 
-HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "lodestar.h")
+INCLUDE = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
+HEADER = os.path.join(INCLUDE, "lodestar.h")
+HEADERS = [HEADER, os.path.join(INCLUDE, "lodestar_probe.h")]
 
 
 def declared_functions():
-    src = open(HEADER).read()
+    src = "\n".join(open(h).read() for h in HEADERS)
     src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
     return sorted(set(re.findall(r"^\s*(?:const\s+)?[A-Za-z_][\w\s\*]*?\b(ls_\w+)\s*\(", src, flags=re.M)))
 

@@ -36,12 +36,8 @@ def test_route_costs_against_a_recount(bench):
     keys, key_off = oracle.hash_blocks(wl.tok, wl.tok_off)
     lens = np.diff(wl.tok_off)
     got = bench.route_costs(cfg, R, N, hits, lens, keys, key_off)
-    # tokens: each request up to the block after its longest hit (or its end)
-    tok = 0
-    for r in range(R):
-        nb = lens[r] // 16
-        need = min(nb, hits[r].max() + 1)
-        tok += 4 * min(lens[r], 16 * need)
+    # tokens: every token of every prompt once
+    assert got["tok_bytes"] == 4 * int(lens.sum())
     # probes: distinct keys each instance is asked about (the miss included)
     probes = 0
     for i in range(N):
@@ -51,11 +47,23 @@ def test_route_costs_against_a_recount(bench):
             for b in range(min(hits[r, i] + 1, nb)):
                 seen.add(int(keys[key_off[r] + b]))
         probes += 8 * len(seen)
-    assert got["tok_bytes"] == tok and got["probe_bytes"] == probes
-    assert got["prefix_bytes"] == tok + probes + 4 * R * N + 8 * R
+    assert probes > 0 and got["probe_bytes"] == probes
+    assert got["prefix_bytes"] == got["tok_bytes"] + probes + 8 * R
     w = cfg.widths
     per_pair = 2 * 6 * w[1] + sum(2 * w[l] * w[l + 1] for l in range(1, len(w) - 1))
     assert got["score_flops"] == per_pair * R * N + 2 * N * cfg.d_inst * w[1] + 2 * R * cfg.d_req * w[1]
+    assert got["score_flops_dense"] == sum(2 * w[l] * w[l + 1] for l in range(len(w) - 1)) * R * N
+
+
+def test_distinct_probes_with_shared_prefixes(bench):
+    # two requests share their first two blocks (keys 11, 12); instance 0
+    # caches both, instance 1 only block 0, instance 2 nothing
+    keys = np.array([11, 12, 13, 11, 12, 99], np.uint64)
+    key_off = np.array([0, 3, 6], np.int64)
+    lens = np.array([48, 50], np.int64)                 # 3 full blocks each
+    hits = np.array([[2, 1, 0], [2, 1, 0]], np.int32)
+    # instance 0 is asked 11, 12, 13, 99; instance 1: 11, 12; instance 2: 11
+    assert bench.distinct_probes(hits, lens, keys, key_off) == 4 + 2 + 1
 
 
 def test_code_digest_ignores_comments_only(bench, tmp_path, monkeypatch):

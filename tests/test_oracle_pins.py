@@ -604,3 +604,15 @@ def test_forward_bounds_flip_at_a_bf16_midpoint():
         x = np.array([[1.0]], np.float32)
         y, eb, fl = oracle.mlp_forward_bounds("bf16", widths, params, x)
         assert fl[0] == want
+
+
+def test_prefix_hits_on_presorted_sets_equal_the_plain_scan():
+    wl = W.generate("tiny")
+    rk, rko = oracle.hash_blocks(wl.tok, wl.tok_off)
+    ik, iko = oracle.instance_keys(wl)
+    want = oracle.prefix_hits(rk, rko, ik, iko)
+    assert np.array_equal(oracle.prefix_hits_sorted(rk, rko, oracle.sorted_instance_keys((ik, iko))), want)
+    r = oracle.route(wl, inst_sorted=oracle.sorted_instance_keys((ik, iko)))
+    assert np.array_equal(r["hits"], want)
+    with pytest.raises(Exception):                  # an unsorted set is refused
+        oracle.prefix_hits_sorted(rk, rko, (ik, iko))
