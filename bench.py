@@ -520,9 +520,11 @@ def code_digest(files):
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(kernel):
-    """DRAM bytes per launch of `kernel` from the committed ncu summaries, if the
-    summary was taken on the kernel's current source (else None)."""
+def profiled_traffic(kernel, workload):
+    """DRAM bytes per launch of `kernel` on `workload` from the committed ncu
+    summaries, if the summary was taken on the kernel's current source (else
+    None).  A capture on a smaller case of the same kernel is scaled to the
+    workload's launch when the summary says so (scale=...)."""
     import glob
     if kernel not in KERNEL_SOURCES:
         return None
@@ -531,8 +533,8 @@ def profiled_traffic(kernel):
         for line in open(path):
             if line.startswith("roofline-traffic:"):
                 kv = dict(p.split("=", 1) for p in line.split()[1:])
-                if kv.get("kernel") == kernel and kv.get("code_sha256") == sha:
-                    return float(kv["bytes_per_launch"])
+                if kv.get("kernel") == kernel and kv.get("code_sha256") == sha and kv.get("workload") == workload:
+                    return float(kv["bytes_per_launch"]) * float(kv.get("scale", "1"))
     return None
 
 
@@ -680,7 +682,7 @@ def traced(L, r, fn, n):
     return trace
 
 
-def kernel_rooflines(trace, n_calls, costs, cfg, R, N, Bt, peaks, peak_src):
+def kernel_rooflines(trace, n_calls, costs, cfg, R, N, Bt, peaks, peak_src, workload):
     """Each traced kernel's achieved rate against its bound: the prefix walk
     (compulsory bytes, HBM), the feature image (bytes written), the scorers
     (factorised flops, bf16 tensor), the training products (their flops)."""
@@ -708,7 +710,8 @@ def kernel_rooflines(trace, n_calls, costs, cfg, R, N, Bt, peaks, peak_src):
             continue
         achieved = alg / (per[k] / 1e3)
         out[k] = {"kernel": k, "bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
-                  "frac": achieved / peak, "traffic": profiled_traffic(k), "peak_source": f"{peak_src} (burst)",
+                  "frac": achieved / peak, "traffic": profiled_traffic(k, workload),
+                  "peak_source": f"{peak_src} (burst)",
                   "avg_launch_ms": per[k],
                   "timing": "CUDA events around each launch on its stream (library tracer), calls issued one by one"}
     return out
@@ -775,7 +778,7 @@ def measure_route(name, L, H, W, dev, stream, peaks, peak_src, steps, warmup, ct
     n_tr = min(steps, 30)
     trace = traced(L, r, call, n_tr)
     costs = batch_costs(r, wl, cfg, dw)
-    rl = kernel_rooflines(trace, n_tr, costs, cfg, R, N, cfg.train_batch, peaks, peak_src)
+    rl = kernel_rooflines(trace, n_tr, costs, cfg, R, N, cfg.train_batch, peaks, peak_src, name)
     per_call = {k: v[1] / max(v[2], 1) * v[0] / n_tr for k, v in trace.items()}
     roof = route_roofline(costs, R, N, peaks)
     dom = max(rl, key=lambda k: per_call.get(k, 0.0)) if rl else None
@@ -848,7 +851,7 @@ def measure_probes(L, dev, stream, peaks, sms):
         ms = timed(lambda: L.check(L.ls_probe_gather(table, table.numel(), blocks, per, 7, out, stream)))
         n = blocks * 256 * per
         res[f"gather8_{label}"] = {"table_bytes": nbytes, "lookups_per_s": n / (ms / 1e3),
-                                   "GB_per_s": 8 * n / (ms / 1e6) / 1e6, "ms": ms}
+                                   "GB_per_s": 8 * n / (ms / 1e3) / 1e9, "ms": ms}
         del table
     f = torch.empty(4 * sms * 256, dtype=torch.float32, device=dev)
     iters = 20000
@@ -930,7 +933,7 @@ def measure_step(name, L, H, W, dev, stream, peaks, peak_src, args, ctx, clocks=
     n_traced = min(args.steps, 60)
     trace = traced(L, r, lambda k: eager_step(k), n_traced)
     costs = batch_costs(r, wl, cfg, dw)
-    rl = kernel_rooflines(trace, n_traced, costs, cfg, R, N, Bt, peaks, peak_src)
+    rl = kernel_rooflines(trace, n_traced, costs, cfg, R, N, Bt, peaks, peak_src, name)
     per_step = {k: v[1] / max(v[2], 1) * v[0] / n_traced for k, v in trace.items()}
     launches = sum(v[0] for v in trace.values()) / n_traced
     return {"times": times, "eager_times": eager_times, "clocks": clk, "costs": costs, "rooflines": rl,

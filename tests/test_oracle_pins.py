@@ -5,6 +5,7 @@ brute force, exhaustive enumeration or an independent library routine, so that
 a dropped term, a wrong sign or index, or a transposed operand in the oracle
 fails at least one of them.  No GPU needed.
 """
+import dataclasses
 import os
 import shutil
 import subprocess
@@ -616,3 +617,30 @@ def test_prefix_hits_on_presorted_sets_equal_the_plain_scan():
     assert np.array_equal(r["hits"], want)
     with pytest.raises(Exception):                  # an unsorted set is refused
         oracle.prefix_hits_sorted(rk, rko, (ik, iko))
+
+
+def test_vectorised_trainer_follows_the_scalar_oracle():
+    # five bf16 Adam steps of the vectorised restatement against or_train_step:
+    # the same losses and parameters up to fp64 summation order (an fp32 or
+    # bf16 rounding point may land on the other side for a handful of values)
+    from oracle.train_np import NpTrainer, bf16
+    cfg = W.CONFIGS["training"]
+    widths = (cfg.d, 64, 64, 1)
+    rng = np.random.default_rng(50)
+    x, y = W.records(rng, dataclasses.replace(cfg, hidden=(64, 64)), 600)
+    mean, std = W.normaliser(np.random.default_rng(51), cfg)
+    params = W.xavier_params(widths, 2)
+    a = oracle.Trainer(widths, params, "bf16")
+    b = NpTrainer(widths, params)
+    for k in range(5):
+        idx = W.minibatch_indices(9, k, 600, 256)
+        la = a.step(x, y, idx, mean, std, "adam", 1e-3)
+        lb = b.step(x, y, idx, mean, std, 1e-3)
+        assert abs(la - lb) <= 1e-6 * la
+        d = np.abs(a.params - b.params)
+        assert np.mean(d <= 1e-6 * np.maximum(np.abs(a.params), 1e-3)) > 0.999
+        assert d.max() <= 3e-3                     # at most a few flipped roundings, each under lr
+    # the bf16 rounding itself against torch
+    import torch
+    v = rng.standard_normal(10000).astype(np.float32) * 3
+    assert np.array_equal(bf16(v), torch.from_numpy(v).to(torch.bfloat16).to(torch.float64).numpy())
