@@ -54,6 +54,9 @@ struct TcPlan {
   int64_t b_last_off = 0;
   int pipe = 0;                    // pipelined kernel applies (two hidden layers, resident weights)
   int pipe_smem = 0;
+  int wide = 0;                    // wide kernel applies (two hidden layers of multiples of 128, streamed weights)
+  int wide_smem = 0;
+  int wide_stages = 0;
 };
 
 // One published weight version (Sec. 4.3.1 P2: the routing side reads a

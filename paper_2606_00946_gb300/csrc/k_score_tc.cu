@@ -664,6 +664,329 @@ __global__ void __launch_bounds__(kThreadsPipe, 1) k_score_tc_pipe(const __grid_
   if (warp == 0) tmem_dealloc(tmem, 512);
 }
 
+// ---------------------------------------------------------------------------
+// Wide variant: two hidden layers whose widths are multiples of 128 (<= 512),
+// weights streamed from L2 (they do not fit in shared memory), one persistent
+// CTA per SM over 128-row tiles.  A job is one 128-column slice of a layer's
+// output: its bias product (ones x three-term bias operand, as in the
+// pipelined kernel), then its K-blocks, each a 16 KB [128 x 64] slice of the
+// published weight image.  Layer-1 jobs read the feature tile from shared
+// memory; their epilogue packs relu(z) to bf16 pairs and stores them in
+// tensor memory, where the layer-2 jobs read them as the A operand -- so the
+// 128 x H1 activation tile needs no shared memory and the layer-2 products
+// read only their weights from it.  Accumulators alternate between two
+// 128-column TMEM slots, so the epilogue of one job overlaps the next job's
+// products.
+// TMEM (512 columns): [0, 256) packed layer-1 activations, [256, 384) and
+// [384, 512) the two slots.
+// Warp roles (14 warps): 0 = MMA issuer (lane 0) and TMEM owner,
+// 1 = weight producer (lane 0, one bulk copy per 16 KB slice into a ring of
+// stages), 2..5 = feature-tile builders (template rows + pair chunk, as
+// build_tile), 6..13 = epilogue: two warps per TMEM lane quadrant, each 64
+// of a job's 128 columns.
+// ---------------------------------------------------------------------------
+constexpr int kWideBuild = 4, kWideEpi = 8;
+constexpr int kWideBuild0 = 2, kWideEpi0 = kWideBuild0 + kWideBuild;
+constexpr int kThreadsWide = (kWideEpi0 + kWideEpi) * 32;  // 448
+constexpr int kWideChunk = kTileM * 128;                    // [128 N x 64 K] bf16 = 16 KB
+constexpr uint32_t kSlot0 = 256;                             // TMEM column of accumulator slot 0
+
+// Byte offset in the published image of the [128 x 64] slice for layer l,
+// job c (output rows 128c..128c+127), K-block kb: the image stores N-chunks
+// of nc <= 256 rows x K-blocks in the 128-byte-swizzled K-major layout with
+// 8-row atoms stacked along N, so a 128-row half of a chunk is contiguous.
+__device__ __forceinline__ int64_t wide_chunk_off(const TcPlan& p, int l, int c, int kb) {
+  const int nc = p.nc[l], nk = p.in_pad[l] / 64;
+  const int nci = (128 * c) / nc, half = ((128 * c) % nc) / 128;
+  return p.img_off[l] + ((int64_t)nci * nk + kb) * nc * 128 + (int64_t)half * kWideChunk;
+}
+
+__global__ void __launch_bounds__(kThreadsWide, 1) k_score_wide(const __grid_constant__ TcArgs a) {
+  const bool pb = a.sel && *a.sel == 1;  // published buffer of this route
+  const uint8_t* __restrict__ img = pb ? a.img1 : a.img0;
+  const float* __restrict__ params = pb ? a.params1 : a.params0;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const TcPlan& p = a.p;
+  const int H1 = p.out[0], H2 = p.out[1];
+  const int J1 = H1 / 128, J2 = H2 / 128;
+  const int nk0 = p.in_pad[0] / 64, nk1 = H1 / 64;
+  const int per_tile = J1 * nk0 + J2 * nk1;
+  const int S = p.wide_stages;
+  uint8_t* X = smem;                                              // [nk0] feature-tile K-blocks
+  uint8_t* ring = X + (size_t)nk0 * kWideChunk;                   // [S] weight slices
+  uint8_t* ONE = ring + (size_t)S * kWideChunk;                   // 256 B, no swizzle
+  uint8_t* BIAS = ONE + 256;                                      // [H1 + H2 rows x 16] no swizzle
+  uint16_t* sw3 = reinterpret_cast<uint16_t*>(BIAS + (size_t)(H1 + H2) * 32);  // [H2] bf16
+  float* part = reinterpret_cast<float*>(sw3 + H2);               // [2 tiles][2 halves][128]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(part + 4 * kTileM);
+  uint64_t* full = bars;            // [S]
+  uint64_t* empty = full + S;       // [S]
+  uint64_t* x_full = empty + S;
+  uint64_t* x_empty = x_full + 1;
+  uint64_t* s_full = x_empty + 1;   // [2]
+  uint64_t* s_empty = s_full + 2;   // [2]
+  uint64_t* h1_ready = s_empty + 2;
+  uint64_t* h1_free = h1_ready + 1;
+  uint64_t* done = h1_free + 1;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(done + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int my_tiles = blockIdx.x < a.n_tiles ? (a.n_tiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
+  if (tid == 0) {
+    for (int q = 0; q < S; ++q) {
+      mbar_init(&full[q], 1);
+      mbar_init(&empty[q], 1);
+    }
+    mbar_init(x_full, kWideBuild);
+    mbar_init(x_empty, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&s_full[b], 1);
+      mbar_init(&s_empty[b], kWideEpi);
+    }
+    mbar_init(h1_ready, kWideEpi * J1);
+    mbar_init(h1_free, 1);
+    mbar_init(done, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0) {
+    tmem_alloc(tmem_holder, 512);
+    tmem_relinquish();
+  }
+  // bias operands (three exact bf16 terms of each fp32 bias), the ones
+  // operand and the bf16 output-layer weights, from the published parameters
+  for (int k = tid; k < H2; k += blockDim.x) sw3[k] = bf16_bits(__ldg(params + a.w_last_off + k));
+  for (int e = tid; e < 8 * 2; e += blockDim.x) {  // 16-byte chunks: row e / 2, K half e % 2
+    const uint4 q = (e & 1) ? make_uint4(0u, 0u, 0u, 0u) : make_uint4(0x3F803F80u, 0x3F80u, 0u, 0u);
+    *reinterpret_cast<uint4*>(ONE + nosw16_offset(e >> 1, 8 * (e & 1))) = q;
+  }
+  for (int e = tid; e < (H1 + H2) * 2; e += blockDim.x) {  // row n of [H1 | H2], K half e % 2
+    const int n = e >> 1, l = n >= H1 ? 1 : 0, o = n - (l ? H1 : 0);
+    uint4 q = make_uint4(0u, 0u, 0u, 0u);
+    if (!(e & 1)) {
+      const float b = __ldg(params + a.boff[l] + o);
+      const uint16_t hi = bf16_bits(b);
+      uint16_t mid = 0, lo = 0;
+      if (!isinf(b)) {  // b - hi and (b - hi) - mid are exact in fp32; lo holds the last 8 bits
+        const float r1 = b - __uint_as_float((uint32_t)hi << 16);
+        mid = bf16_bits(r1);
+        lo = bf16_bits(r1 - __uint_as_float((uint32_t)mid << 16));
+      }
+      q.x = (uint32_t)hi | ((uint32_t)mid << 16);
+      q.y = lo;
+    }
+    *reinterpret_cast<uint4*>(BIAS + nosw16_offset(n, 8 * (e & 1))) = q;
+  }
+  fence_async_smem();  // the bias operands are read by the tensor cores (async proxy)
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_holder;
+  const uint32_t idesc = idesc_bf16_f32(kTileM, 128);
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0 && my_tiles > 0) {
+      bool ok = true;
+      int64_t g = 0, jg = 0;  // weight slices and jobs consumed so far
+      auto job_start = [&](int64_t j, uint32_t& d) {  // wait for the slot's previous epilogue
+        const int slot = (int)(j & 1);
+        const int64_t use = j >> 1;
+        if (use >= 1 && !mbar_wait(&s_empty[slot], (uint32_t)((use - 1) & 1))) return false;
+        tc_fence_after();
+        d = tmem + kSlot0 + 128u * (uint32_t)slot;
+        return true;
+      };
+      auto next_slice = [&](uint32_t& b) {
+        const int s = (int)(g % S);
+        if (!mbar_wait(&full[s], (uint32_t)((g / S) & 1))) return false;
+        tc_fence_after();
+        b = smem_u32(ring + (size_t)s * kWideChunk);
+        return true;
+      };
+      for (int t = 0; t < my_tiles && ok; ++t) {
+        ok = mbar_wait(x_full, (uint32_t)(t & 1));
+        if (!ok) break;
+        tc_fence_after();
+        for (int c = 0; c < J1 && ok; ++c, ++jg) {
+          uint32_t d;
+          if (!(ok = job_start(jg, d))) break;
+          umma_bf16(d, sdesc_nosw(smem_u32(ONE), 128, 0),
+                    sdesc_nosw(smem_u32(BIAS + (size_t)c * 128 * 32), 128, 256), idesc, 0u);
+          for (int kb = 0; kb < nk0 && ok; ++kb, ++g) {
+            uint32_t bb;
+            if (!(ok = next_slice(bb))) break;
+            const uint32_t xa = smem_u32(X + (size_t)kb * kWideChunk);
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+              umma_bf16(d, sdesc_sw128(xa + 32u * j), sdesc_sw128(bb + 32u * j), idesc, 1u);
+            umma_commit(&empty[g % S]);
+          }
+          if (ok) umma_commit(&s_full[jg & 1]);
+        }
+        if (!ok) break;
+        umma_commit(x_empty);  // the feature tile is free once the layer-1 products are done
+        ok = mbar_wait(h1_ready, (uint32_t)(t & 1));  // every layer-1 slice packed into TMEM
+        if (!ok) break;
+        tc_fence_after();
+        for (int n = 0; n < J2 && ok; ++n, ++jg) {
+          uint32_t d;
+          if (!(ok = job_start(jg, d))) break;
+          umma_bf16(d, sdesc_nosw(smem_u32(ONE), 128, 0),
+                    sdesc_nosw(smem_u32(BIAS + (size_t)(H1 + n * 128) * 32), 128, 256), idesc, 0u);
+          for (int kb = 0; kb < nk1 && ok; ++kb, ++g) {
+            uint32_t bb;
+            if (!(ok = next_slice(bb))) break;
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+              umma_bf16_ts(d, tmem + (uint32_t)(32 * kb + 8 * j), sdesc_sw128(bb + 32u * j), idesc, 1u);
+            umma_commit(&empty[g % S]);
+          }
+          if (ok) umma_commit(&s_full[jg & 1]);
+        }
+        if (ok) umma_commit(h1_free);  // the packed activations may be overwritten
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        latch_error(a.err, LS_ERR_TIMEOUT);
+      }
+      umma_commit(done);  // every product issued has completed before TMEM is freed
+      mbar_wait(done, 0);
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ weight producer
+    if (lane == 0 && my_tiles > 0) {
+      int64_t g = 0;
+      bool ok = true;
+      for (int t = 0; t < my_tiles && ok; ++t)
+        for (int q = 0; q < per_tile; ++q, ++g) {
+          const int s = (int)(g % S);
+          const int64_t u = g / S;
+          if (u >= 1 && !(ok = mbar_wait(&empty[s], (uint32_t)((u - 1) & 1)))) break;
+          if (*abort_flag) { ok = false; break; }
+          int l, c, kb;
+          if (q < J1 * nk0) { l = 0; c = q / nk0; kb = q % nk0; }
+          else { l = 1; c = (q - J1 * nk0) / nk1; kb = (q - J1 * nk0) % nk1; }
+          mbar_arrive_expect_tx(&full[s], (uint32_t)kWideChunk);
+          bulk_g2s(ring + (size_t)s * kWideChunk, img + wide_chunk_off(p, l, c, kb), (uint32_t)kWideChunk, &full[s]);
+        }
+      if (!ok) {
+        *abort_flag = 1;
+        latch_error(a.err, LS_ERR_TIMEOUT);
+      }
+      // slices issued and never consumed (only after an abort) land in this
+      // CTA's shared memory: wait for them (bounded) before the CTA can exit
+      for (int64_t h = g - 1; h >= 0 && h >= g - S; --h) mbar_wait(&full[h % S], (uint32_t)((h / S) & 1));
+    }
+    __syncwarp();
+  } else if (warp < kWideEpi0) {
+    // ------------------------------------------------------------ feature-tile builders
+    const int bt = tid - kWideBuild0 * 32;
+    pdl_wait();  // pair chunks and template rows from the previous kernel of the stream
+    for (int t = 0; t < my_tiles; ++t) {
+      if (t >= 1 && !mbar_wait(x_empty, (uint32_t)((t - 1) & 1))) {
+        *abort_flag = 1;
+        latch_error(a.err, LS_ERR_TIMEOUT);
+        break;
+      }
+      if (*abort_flag) break;
+      const int64_t row0 = (int64_t)(blockIdx.x + (int64_t)t * gridDim.x) * kTileM;
+      build_tile<4>(a, X, row0, bt, kWideBuild * 32);
+      fence_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(x_full);
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int ew = warp - kWideEpi0;       // 0..7
+    const int q4 = warp & 3;               // TMEM lane quadrant
+    const int h = ew >> 2;                 // which 64 of a job's 128 columns
+    const int row = 32 * q4 + lane;
+    const uint32_t lane_addr = (uint32_t)(32 * q4) << 16;
+    int64_t jg = 0;
+    bool ok = true;
+    for (int t = 0; t < my_tiles; ++t) {
+      uint64_t acc = 0;  // output-layer partial, two fp32 lanes
+      for (int c = 0; c < J1; ++c, ++jg) {
+        const int slot = (int)(jg & 1);
+        bool go = ok && !*abort_flag;
+        if (go) go = mbar_wait(&s_full[slot], (uint32_t)((jg >> 1) & 1));
+        if (go && c == 0 && t >= 1) go = mbar_wait(h1_free, (uint32_t)((t - 1) & 1));
+        go = __all_sync(0xffffffffu, go);  // the tensor-memory accesses below are warp-wide
+        if (!go) {
+          ok = false;
+          *abort_flag = 1;
+        }
+        if (go) {
+          tc_fence_after();
+          const uint32_t src = tmem + lane_addr + kSlot0 + 128u * (uint32_t)slot + 64u * (uint32_t)h;
+          uint32_t v[4][16];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) tmem_ld16(src + 16u * i, v[i]);
+          tmem_wait_ld();
+          uint32_t pk[32];
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+              pk[8 * i + j] = relu_bf16x2(cvt_bf16x2(((uint64_t)v[i][2 * j + 1] << 32) | v[i][2 * j]));
+          tmem_st32(tmem + lane_addr + (uint32_t)(64 * c + 32 * h), pk);
+          tmem_wait_st();
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(&s_empty[slot]);
+          mbar_arrive(h1_ready);
+        }
+      }
+      for (int n = 0; n < J2; ++n, ++jg) {
+        const int slot = (int)(jg & 1);
+        bool go = ok && !*abort_flag;
+        if (go) go = mbar_wait(&s_full[slot], (uint32_t)((jg >> 1) & 1));
+        go = __all_sync(0xffffffffu, go);
+        if (!go) {
+          ok = false;
+          *abort_flag = 1;
+        }
+        if (go) {
+          tc_fence_after();
+          const uint32_t src = tmem + lane_addr + kSlot0 + 128u * (uint32_t)slot + 64u * (uint32_t)h;
+          const uint4* w = reinterpret_cast<const uint4*>(sw3 + 128 * n + 64 * h);
+          uint32_t va[16], vb[16];
+          tmem_ld16(src, va);
+#pragma unroll
+          for (int i = 0; i < 4; i += 2) {
+            tmem_wait_ld_regs(va);
+            tmem_ld16(src + 16u * (i + 1), vb);
+            acc = out_dot16(va, w[2 * i], w[2 * i + 1], acc);
+            tmem_wait_ld_regs(vb);
+            if (i + 2 < 4) tmem_ld16(src + 16u * (i + 2), va);
+            acc = out_dot16(vb, w[2 * i + 2], w[2 * i + 3], acc);
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&s_empty[slot]);
+      }
+      float* pt = part + (t & 1) * 2 * kTileM;
+      pt[h * kTileM + row] = __uint_as_float((uint32_t)acc) + __uint_as_float((uint32_t)(acc >> 32));
+      // the two halves of every row meet here; a stop is decided together
+      if (!named_bar_and(1, kWideEpi * 32, ok)) break;
+      if (h == 0) {
+        const int64_t g = (int64_t)(blockIdx.x + (int64_t)t * gridDim.x) * kTileM + row;
+        if (g < a.rows) a.scores[g] = (pt[row] + pt[kTileM + row]) + __ldg(params + p.b_last_off);
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tmem, 512);
+}
+
 // Per batch, before the scorer: normalised bf16 template rows (instance row i
 // holds the z-scored instance features at their feature positions 6 ..
 // 6+d_inst and zeros elsewhere; request row r likewise for the request block)
@@ -848,6 +1171,21 @@ bool plan_tc(const MlpDesc& m, TcPlan& p) {
   while ((int)p.tmem_cols < outmax) p.tmem_cols <<= 1;
   p.w_last_off = m.woff[m.n_layers - 1];
   p.b_last_off = m.boff[m.n_layers - 1];
+  // wide variant: two hidden layers, widths multiples of 128 (<= 512), the
+  // feature tile at most 128 columns, weights streamed in 16 KB slices
+  p.wide = 0;
+  if (p.n_tc == 2 && p.out[0] % 128 == 0 && p.out[1] % 128 == 0 && p.d_pad <= 128 &&
+      (p.nc[0] % 128 == 0) && (p.nc[1] % 128 == 0)) {
+    const int H1 = p.out[0], H2 = p.out[1];
+    const int64_t fixed = 1024 + (int64_t)(p.d_pad / 64) * kTileM * 128 + 256 + (int64_t)(H1 + H2) * 32 +
+                          (int64_t)H2 * 2 + 4 * kTileM * 4 + 16 * 8 + 16;
+    const int64_t stages = (kMaxSmem - fixed - 256) / (kTileM * 128 + 16);
+    if (stages >= 4) {
+      p.wide_stages = (int)std::min<int64_t>(stages, 12);
+      p.wide_smem = (int)(fixed + (int64_t)p.wide_stages * (kTileM * 128 + 16));
+      p.wide = 1;
+    }
+  }
   // pipelined variant: two hidden layers of <= 256, all weights resident
   p.pipe = 0;
   if (p.n_tc == 2 && p.out[0] <= 256 && p.out[1] <= 256 && p.nc[0] == p.out[0] && p.nc[1] == p.out[1]) {
@@ -937,6 +1275,10 @@ cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const Published* 
     cudaError_t e = cudaFuncSetAttribute(k_score_tc_pipe, cudaFuncAttributeMaxDynamicSharedMemorySize, p.pipe_smem);
     if (e != cudaSuccess) return e;
     return launch_chained(k_score_tc_pipe, dim3(grid), dim3(kThreadsPipe), (size_t)p.pipe_smem, s, 1, a);
+  } else if (p.wide && scores) {
+    cudaError_t e = cudaFuncSetAttribute(k_score_wide, cudaFuncAttributeMaxDynamicSharedMemorySize, p.wide_smem);
+    if (e != cudaSuccess) return e;
+    return launch_chained(k_score_wide, dim3(grid), dim3(kThreadsWide), (size_t)p.wide_smem, s, 1, a);
   } else {
     cudaError_t e = cudaFuncSetAttribute(k_score_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, p.smem);
     if (e != cudaSuccess) return e;

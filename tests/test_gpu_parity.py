@@ -247,6 +247,36 @@ def test_pipelined_scorer_with_tiles_across_requests(n_inst):
     r.close()
 
 
+@pytest.mark.parametrize("hidden,n_inst,wide_dims", [
+    ((512, 512), 24, False), ((512, 128), 200, False), ((128, 512), 7, False), ((256, 512), 256, True),
+    ((512, 512), 256, True)])
+def test_wide_scorer_shapes(hidden, n_inst, wide_dims):
+    # the wide tensor-core scorer (two hidden layers of multiples of 128 with
+    # weights streamed in slices; layer-1 activations packed in tensor memory)
+    # against the oracle: tiles across request boundaries, one and four
+    # layer-1 jobs, 64- and 128-column feature tiles
+    import dataclasses
+    base = W.CONFIGS["large" if wide_dims else "homogeneous"]
+    cfg = dataclasses.replace(base, hidden=hidden, n_inst=n_inst, n_req=48 if n_inst > 64 else 96,
+                              cache_blocks=1024, n_samples=0)
+    wl = W.generate(cfg)
+    r = H.Router.for_config(cfg)
+    dw = H.DeviceWorkload(wl)
+    dw.load(r)
+    assert r.info().scorer == L.LS_SCORER_TENSOR_CORES
+    out = r.route(dw.tok, dw.tok_off, dw.req_feats, n_inst)
+    ref = oracle.route(wl, bounds=True, threads=THREADS)
+    assert np.array_equal(out["hits"].cpu().numpy(), ref["hits"])
+    sg = out["scores"].cpu().numpy()
+    assert_scores_close(sg, ref, TOL["bf16"], f"wide scorer {hidden} x {n_inst}")
+    assert_choices(out["choice"].cpu().numpy(), sg, ref, TOL["bf16"])
+    # a second route of the same batch gives the same bits (no state carried between launches)
+    again = r.route(dw.tok, dw.tok_off, dw.req_feats, n_inst)
+    assert torch.equal(again["scores"], out["scores"])
+    assert r.sync() == L.LS_OK
+    r.close()
+
+
 def test_optional_outputs_do_not_change_the_result():
     wl, dw, r = staged("homogeneous")
     full = r.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)
