@@ -57,6 +57,7 @@ struct TcPlan {
   int wide = 0;                    // wide kernel applies (two hidden layers of multiples of 128, streamed weights)
   int wide_smem = 0;
   int wide_stages = 0;
+  int wide_q = 1;                  // weight slices per stage of the wide kernel
 };
 
 // One published weight version (Sec. 4.3.1 P2: the routing side reads a

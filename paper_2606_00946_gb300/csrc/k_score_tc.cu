@@ -670,7 +670,9 @@ __global__ void __launch_bounds__(kThreadsPipe, 1) k_score_tc_pipe(const __grid_
 // CTA per SM over 128-row tiles.  A job is one 128-column slice of a layer's
 // output: its bias product (ones x three-term bias operand, as in the
 // pipelined kernel), then its K-blocks, each a 16 KB [128 x 64] slice of the
-// published weight image.  Layer-1 jobs read the feature tile from shared
+// published weight image, whose 128-row N-chunks put the slices of a tile in
+// the order they are consumed; a stage of the ring is Q consecutive slices
+// brought by one bulk copy.  Layer-1 jobs read the feature tile from shared
 // memory; their epilogue packs relu(z) to bf16 pairs and stores them in
 // tensor memory, where the layer-2 jobs read them as the A operand -- so the
 // 128 x H1 activation tile needs no shared memory and the layer-2 products
@@ -691,16 +693,6 @@ constexpr int kThreadsWide = (kWideEpi0 + kWideEpi) * 32;  // 448
 constexpr int kWideChunk = kTileM * 128;                    // [128 N x 64 K] bf16 = 16 KB
 constexpr uint32_t kSlot0 = 256;                             // TMEM column of accumulator slot 0
 
-// Byte offset in the published image of the [128 x 64] slice for layer l,
-// job c (output rows 128c..128c+127), K-block kb: the image stores N-chunks
-// of nc <= 256 rows x K-blocks in the 128-byte-swizzled K-major layout with
-// 8-row atoms stacked along N, so a 128-row half of a chunk is contiguous.
-__device__ __forceinline__ int64_t wide_chunk_off(const TcPlan& p, int l, int c, int kb) {
-  const int nc = p.nc[l], nk = p.in_pad[l] / 64;
-  const int nci = (128 * c) / nc, half = ((128 * c) % nc) / 128;
-  return p.img_off[l] + ((int64_t)nci * nk + kb) * nc * 128 + (int64_t)half * kWideChunk;
-}
-
 __global__ void __launch_bounds__(kThreadsWide, 1) k_score_wide(const __grid_constant__ TcArgs a) {
   const bool pb = a.sel && *a.sel == 1;  // published buffer of this route
   const uint8_t* __restrict__ img = pb ? a.img1 : a.img0;
@@ -712,10 +704,10 @@ __global__ void __launch_bounds__(kThreadsWide, 1) k_score_wide(const __grid_con
   const int J1 = H1 / 128, J2 = H2 / 128;
   const int nk0 = p.in_pad[0] / 64, nk1 = H1 / 64;
   const int per_tile = J1 * nk0 + J2 * nk1;
-  const int S = p.wide_stages;
+  const int S = p.wide_stages, Q = p.wide_q;  // stages of Q slices each
   uint8_t* X = smem;                                              // [nk0] feature-tile K-blocks
-  uint8_t* ring = X + (size_t)nk0 * kWideChunk;                   // [S] weight slices
-  uint8_t* ONE = ring + (size_t)S * kWideChunk;                   // 256 B, no swizzle
+  uint8_t* ring = X + (size_t)nk0 * kWideChunk;                   // [S][Q] weight slices
+  uint8_t* ONE = ring + (size_t)S * Q * kWideChunk;               // 256 B, no swizzle
   uint8_t* BIAS = ONE + 256;                                      // [H1 + H2 rows x 16] no swizzle
   uint16_t* sw3 = reinterpret_cast<uint16_t*>(BIAS + (size_t)(H1 + H2) * 32);  // [H2] bf16
   float* part = reinterpret_cast<float*>(sw3 + H2);               // [2 tiles][2 halves][128]
@@ -799,12 +791,18 @@ __global__ void __launch_bounds__(kThreadsWide, 1) k_score_wide(const __grid_con
         d = tmem + kSlot0 + 128u * (uint32_t)slot;
         return true;
       };
-      auto next_slice = [&](uint32_t& b) {
-        const int s = (int)(g % S);
-        if (!mbar_wait(&full[s], (uint32_t)((g / S) & 1))) return false;
-        tc_fence_after();
-        b = smem_u32(ring + (size_t)s * kWideChunk);
+      auto next_slice = [&](uint32_t& b) {  // slice g: part g % Q of stage g / Q
+        const int64_t G = g / Q;
+        const int s = (int)(G % S);
+        if (g % Q == 0) {
+          if (!mbar_wait(&full[s], (uint32_t)((G / S) & 1))) return false;
+          tc_fence_after();
+        }
+        b = smem_u32(ring + ((size_t)s * Q + (size_t)(g % Q)) * kWideChunk);
         return true;
+      };
+      auto slice_done = [&]() {  // the stage is free once the products of its last slice complete
+        if (g % Q == Q - 1) umma_commit(&empty[(g / Q) % S]);
       };
       for (int t = 0; t < my_tiles && ok; ++t) {
         ok = mbar_wait(x_full, (uint32_t)(t & 1));
@@ -822,7 +820,7 @@ __global__ void __launch_bounds__(kThreadsWide, 1) k_score_wide(const __grid_con
 #pragma unroll
             for (int j = 0; j < 4; ++j)
               umma_bf16(d, sdesc_sw128(xa + 32u * j), sdesc_sw128(bb + 32u * j), idesc, 1u);
-            umma_commit(&empty[g % S]);
+            slice_done();
           }
           if (ok) umma_commit(&s_full[jg & 1]);
         }
@@ -842,7 +840,7 @@ __global__ void __launch_bounds__(kThreadsWide, 1) k_score_wide(const __grid_con
 #pragma unroll
             for (int j = 0; j < 4; ++j)
               umma_bf16_ts(d, tmem + (uint32_t)(32 * kb + 8 * j), sdesc_sw128(bb + 32u * j), idesc, 1u);
-            umma_commit(&empty[g % S]);
+            slice_done();
           }
           if (ok) umma_commit(&s_full[jg & 1]);
         }
@@ -858,28 +856,30 @@ __global__ void __launch_bounds__(kThreadsWide, 1) k_score_wide(const __grid_con
     __syncwarp();
   } else if (warp == 1) {
     // ------------------------------------------------------------ weight producer
+    // The image holds the per-tile stream of slices contiguously (128-row
+    // N-chunks, layer 1 then layer 2), so a stage of Q consecutive slices is
+    // one bulk copy: large copies reach several times the rate of 16 KB ones.
     if (lane == 0 && my_tiles > 0) {
-      int64_t g = 0;
+      const int64_t stages = (int64_t)my_tiles * per_tile / Q;
+      const uint32_t bytes = (uint32_t)(Q * kWideChunk);
+      int64_t G = 0;
       bool ok = true;
-      for (int t = 0; t < my_tiles && ok; ++t)
-        for (int q = 0; q < per_tile; ++q, ++g) {
-          const int s = (int)(g % S);
-          const int64_t u = g / S;
-          if (u >= 1 && !(ok = mbar_wait(&empty[s], (uint32_t)((u - 1) & 1)))) break;
-          if (*abort_flag) { ok = false; break; }
-          int l, c, kb;
-          if (q < J1 * nk0) { l = 0; c = q / nk0; kb = q % nk0; }
-          else { l = 1; c = (q - J1 * nk0) / nk1; kb = (q - J1 * nk0) % nk1; }
-          mbar_arrive_expect_tx(&full[s], (uint32_t)kWideChunk);
-          bulk_g2s(ring + (size_t)s * kWideChunk, img + wide_chunk_off(p, l, c, kb), (uint32_t)kWideChunk, &full[s]);
-        }
+      for (; G < stages; ++G) {
+        const int s = (int)(G % S);
+        const int64_t u = G / S;
+        if (u >= 1 && !(ok = mbar_wait(&empty[s], (uint32_t)((u - 1) & 1)))) break;
+        if (*abort_flag) { ok = false; break; }
+        const int q0 = (int)((G * Q) % per_tile);
+        mbar_arrive_expect_tx(&full[s], bytes);
+        bulk_g2s(ring + (size_t)s * Q * kWideChunk, img + (int64_t)q0 * kWideChunk, bytes, &full[s]);
+      }
       if (!ok) {
         *abort_flag = 1;
         latch_error(a.err, LS_ERR_TIMEOUT);
       }
-      // slices issued and never consumed (only after an abort) land in this
+      // stages issued and never consumed (only after an abort) land in this
       // CTA's shared memory: wait for them (bounded) before the CTA can exit
-      for (int64_t h = g - 1; h >= 0 && h >= g - S; --h) mbar_wait(&full[h % S], (uint32_t)((h / S) & 1));
+      for (int64_t h = G - 1; h >= 0 && h >= G - S; --h) mbar_wait(&full[h % S], (uint32_t)((h / S) & 1));
     }
     __syncwarp();
   } else if (warp < kWideEpi0) {
@@ -1171,21 +1171,6 @@ bool plan_tc(const MlpDesc& m, TcPlan& p) {
   while ((int)p.tmem_cols < outmax) p.tmem_cols <<= 1;
   p.w_last_off = m.woff[m.n_layers - 1];
   p.b_last_off = m.boff[m.n_layers - 1];
-  // wide variant: two hidden layers, widths multiples of 128 (<= 512), the
-  // feature tile at most 128 columns, weights streamed in 16 KB slices
-  p.wide = 0;
-  if (p.n_tc == 2 && p.out[0] % 128 == 0 && p.out[1] % 128 == 0 && p.d_pad <= 128 &&
-      (p.nc[0] % 128 == 0) && (p.nc[1] % 128 == 0)) {
-    const int H1 = p.out[0], H2 = p.out[1];
-    const int64_t fixed = 1024 + (int64_t)(p.d_pad / 64) * kTileM * 128 + 256 + (int64_t)(H1 + H2) * 32 +
-                          (int64_t)H2 * 2 + 4 * kTileM * 4 + 16 * 8 + 16;
-    const int64_t stages = (kMaxSmem - fixed - 256) / (kTileM * 128 + 16);
-    if (stages >= 4) {
-      p.wide_stages = (int)std::min<int64_t>(stages, 12);
-      p.wide_smem = (int)(fixed + (int64_t)p.wide_stages * (kTileM * 128 + 16));
-      p.wide = 1;
-    }
-  }
   // pipelined variant: two hidden layers of <= 256, all weights resident
   p.pipe = 0;
   if (p.n_tc == 2 && p.out[0] <= 256 && p.out[1] <= 256 && p.nc[0] == p.out[0] && p.nc[1] == p.out[1]) {
@@ -1195,6 +1180,50 @@ bool plan_tc(const MlpDesc& m, TcPlan& p) {
       p.pipe = 1;
       p.pipe_smem = (int)need;
     }
+  }
+  // wide variant (when the pipelined one does not apply): two hidden layers of
+  // multiples of 128, a feature tile of at most 128 columns.  Its image uses
+  // 128-row N-chunks, so the per-tile stream of [128 x 64] slices (layer 1
+  // jobs, then layer 2 jobs, K-blocks inner) is the image itself, contiguous;
+  // stages hold Q slices (Q in 4, 2, 1 dividing the slices per tile)
+  p.wide = 0;
+  if (!p.pipe && p.n_tc == 2 && p.out[0] % 128 == 0 && p.out[1] % 128 == 0 && p.d_pad <= 128) {
+    int64_t woff = 0;
+    q = 0;
+    for (int l = 0; l < 2; ++l) {
+      p.nc[l] = 128;
+      p.img_off[l] = woff;
+      const int nk = p.in_pad[l] / 64, nn = p.out[l] / 128;
+      for (int nci = 0; nci < nn; ++nci)
+        for (int kb = 0; kb < nk; ++kb) {
+          p.chunk_off[q] = woff + ((int64_t)nci * nk + kb) * 128 * 128;
+          p.chunk_len[q] = 128 * 128;
+          ++q;
+        }
+      woff += (int64_t)p.out[l] * p.in_pad[l] * 2;
+    }
+    p.chunks = q;
+    p.img_bytes = woff;
+    p.chunk_bytes = 128 * 128;
+    const int H1 = p.out[0], H2 = p.out[1];
+    const int per_tile = (H1 / 128) * (p.in_pad[0] / 64) + (H2 / 128) * (H1 / 64);
+    const int64_t fixed = 1024 + (int64_t)(p.d_pad / 64) * kTileM * 128 + 256 + (int64_t)(H1 + H2) * 32 +
+                          (int64_t)H2 * 2 + 4 * kTileM * 4 + 16 * 8 + 16;
+    for (int Q = 4; Q >= 1 && !p.wide; Q >>= 1) {
+      if (per_tile % Q) continue;
+      const int64_t stages = (kMaxSmem - fixed - 256) / ((int64_t)Q * kTileM * 128 + 16);
+      if (stages < 2) continue;
+      p.wide_q = Q;
+      p.wide_stages = (int)std::min<int64_t>(stages, 12);
+      p.wide_smem = (int)(fixed + (int64_t)p.wide_stages * ((int64_t)Q * kTileM * 128 + 16));
+      p.wide = 1;
+    }
+    // the generic kernel keeps working on this layout (128-row chunks)
+    const int avail = kMaxSmem - (1024 + 64) - p.a_bytes;
+    const int smax = avail / (p.chunk_bytes + 16);
+    p.resident = p.chunks <= smax ? 1 : 0;
+    p.stages = p.resident ? p.chunks : std::min(smax, 8);
+    p.smem = p.a_bytes + p.stages * p.chunk_bytes + (2 * p.stages + 1) * 8 + 16 + 1024;
   }
   return true;
 }
