@@ -268,6 +268,29 @@ int ls_train_step(ls_ctx *ctx, int32_t batch, const int32_t *idx, int32_t opt, f
  * started with (each route takes the index once, before it scores). */
 int ls_publish(ls_ctx *ctx, void *stream);
 
+/* Sequential-commit routing (Sec. 4.2 cluster snapshot manager and prefix
+ * KV-cache tracker; Sec. 4.3.1 P1: the gateway routes one request at a time):
+ * the requests are routed in order, r = 0, 1, ..., and each decision is
+ * committed before request r + 1 is scored:
+ *   - inst_state[choice[r], queue_col] += 1 (fp32; skipped for queue_col -1):
+ *     the chosen instance queues one more request;
+ *   - every full-block key of prompt r joins the chosen instance's cache (the
+ *     prefix index gains the instance's bit; distinct keys count against
+ *     max_keys_per_instance, more latch LS_ERR_TABLE_FULL).
+ * Request r is scored exactly as ls_route_batch scores it (hits, features,
+ * predictor, argmin, ties to the lowest index, NaN last) against the snapshot
+ * as the decisions for requests 0..r-1 left it.  The updates stay in the
+ * context's snapshot after the call (until the next ls_snapshot_update).
+ * scores_opt / hits_opt (DEVICE [n_req, n_inst], nullable): each request's
+ * predictions and hit lengths as seen when it was decided.  Needs the prefix
+ * index mode and n_inst x (widest layer) small enough for one CTA's shared
+ * memory (LS_ERR_ARG otherwise; the large cluster is beyond it).  One CTA walks
+ * the requests, so the call's time grows with n_req.  Other arguments, the
+ * stream rules and errors are those of ls_route_batch. */
+int ls_route_sequential(ls_ctx *ctx, int32_t n_req, const int32_t *tok, const int64_t *tok_off,
+                        const float *req_feats, int32_t queue_col, int32_t *choice, float *best, float *scores_opt,
+                        int32_t *hits_opt, uint64_t *weight_version_out, void *stream);
+
 /* ---- Algorithm 4 guards (Sec. 4.3.1 fallback; Sec. 4.1 consistent hashing) ----
  * Per-request status of a guarded route.  The low bits say whether the
  * router decided (OK) or hands the request back to the gateway's fallback

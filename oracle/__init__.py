@@ -82,6 +82,8 @@ def lib():
             L.or_replay_embed.argtypes = [C.c_int, C.c_int, P, P, i64, P, P, P, P, P]
             L.or_replay_distances.argtypes = [i64, P, i64, P, C.c_int, P, P]
             L.or_replay_select.argtypes = [i64, P, i64, P, i64, P, P]
+            L.or_route_sequential.argtypes = [C.c_int, C.c_int, P, P, i64, P, P, P, i32, P, P, P, C.c_int, P,
+                                              C.c_int, P, P, i32, P, P, P, P]
             L.or_heuristic.argtypes = [i64, i32, P, P, P, C.c_int, C.c_int, C.c_int, C.c_int, C.c_float,
                                        C.c_float, C.c_float, P]
             L.or_guards.argtypes = [i64, i32, P, P, P, P, C.c_int, P, C.c_int, P, P, P, i64, i64,
@@ -334,6 +336,34 @@ def route(wl, hits=None, inst_keys=None, params=None, mode=None, req_idx=None, b
         out["ebound"] = eb.reshape(len(idx), -1)
         out["flip"] = fl.reshape(len(idx), -1)
     return out
+
+
+def route_sequential(wl, params=None, mode=None, inst_keys=None, queue_col=0, forced=None):
+    """Sequential-commit route of all of a workload's requests
+    (or_route_sequential).  Returns dict(hits, scores, choice, inst) with inst
+    the instance rows after the last commit."""
+    cfg = wl.cfg
+    mode = MODES.get(mode or cfg.dtype, mode or cfg.dtype)
+    w = _c(cfg.widths, np.int32)
+    p = _c(wl.params if params is None else params, np.float64)
+    rk, rko = hash_blocks(wl.tok, wl.tok_off)
+    rk = _c(rk, np.uint64) if len(rk) else np.zeros(1, np.uint64)
+    ik, iko = instance_keys(wl) if inst_keys is None else inst_keys
+    ik = _c(ik, np.uint64) if len(ik) else np.zeros(1, np.uint64)
+    R, N = len(wl.tok_off) - 1, cfg.n_inst
+    L = _c(np.diff(wl.tok_off), np.int64)
+    inst = np.array(wl.inst_state, np.float32, copy=True)
+    req = _c(wl.req_feats, np.float32) if cfg.d_req else np.zeros(1, np.float32)
+    hits = np.zeros((R, N), np.int32)
+    scores = np.zeros((R, N), np.float32)
+    choice = np.zeros(R, np.int32)
+    fc = _c(forced, np.int32) if forced is not None else None
+    _check(lib().or_route_sequential(mode, len(w) - 1, _p(w), _p(p), R, _p(L), _p(rk), _p(_c(rko, np.int64)), N,
+                                     _p(ik), _p(_c(iko, np.int64)), _p(inst), cfg.d_inst, _p(req), cfg.d_req,
+                                     _p(_c(wl.mean, np.float32)), _p(_c(wl.std, np.float32)), int(queue_col),
+                                     _p(fc) if fc is not None else None, _p(hits), _p(scores), _p(choice)),
+           "route_sequential")
+    return dict(hits=hits, scores=scores, choice=choice, inst=inst)
 
 
 # --------------------------------------------------------------------------

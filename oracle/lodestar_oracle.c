@@ -1058,3 +1058,86 @@ int or_replay_select(int64_t mc, const double *dcand, int64_t nk, const double *
     free(oc); free(ok);
     return 0;
 }
+
+/* ------------------------------------------------------------------------ */
+/* sequential-commit routing (Sec. 4.2 cluster snapshot manager and prefix  */
+/* KV-cache tracker; Sec. 4.3.1 P1: requests are routed one at a time)      */
+/* ------------------------------------------------------------------------ */
+
+/* Requests r = 0, 1, ... in order.  Request r is routed as or_argmin routes
+ * it -- hit lengths against each instance's current key set, features from
+ * the current instance rows, the predictor (rounding per mode), the lowest
+ * (score, index) -- and the decision is committed before request r + 1:
+ * inst[c, q_col] += 1 (fp32; q_col < 0: no queue update) and every full-block
+ * key of prompt r joins instance c's key set.  c is the oracle's own choice,
+ * or forced[r] when forced is given (to replay another implementation's
+ * decisions and check each step).  inst is updated in place.  Outputs per
+ * request: hits [n_req, n_inst], scores [n_req, n_inst] (fp32 of the fp64
+ * forward), choice [n_req] (the oracle's own argmin). */
+typedef struct { uint64_t *k; int64_t n, cap; } or_keyset;
+
+static int keyset_has(const or_keyset *s, uint64_t key) {
+    return s->n > 0 && contains(s->k, s->n, key);
+}
+
+int or_route_sequential(int mode, int n_layers, const int *w, const double *params, int64_t n_req,
+                        const int64_t *L, const uint64_t *req_keys, const int64_t *req_key_off,
+                        int32_t n_inst, const uint64_t *inst_keys, const int64_t *inst_key_off,
+                        float *inst, int d_inst, const float *req, int d_req, const float *mean,
+                        const float *std, int32_t q_col, const int32_t *forced,
+                        int32_t *hits, float *scores, int32_t *choice) {
+    int d = 6 + d_inst + d_req, mw = max_width(n_layers, w);
+    or_keyset *base = (or_keyset *)calloc((size_t)n_inst, sizeof(or_keyset));
+    or_keyset *add = (or_keyset *)calloc((size_t)n_inst, sizeof(or_keyset));
+    float *xf = (float *)malloc((size_t)d * sizeof(float));
+    float *xz = (float *)malloc((size_t)d * sizeof(float));
+    double *xd = (double *)malloc((size_t)d * sizeof(double));
+    double *ba = (double *)malloc((size_t)mw * sizeof(double));
+    double *bb = (double *)malloc((size_t)mw * sizeof(double));
+    int rc = 0;
+    if (!base || !add || !xf || !xz || !xd || !ba || !bb) { rc = -1; goto done; }
+    for (int32_t i = 0; i < n_inst; ++i) {
+        int64_t n = inst_key_off[i + 1] - inst_key_off[i];
+        base[i].k = (uint64_t *)malloc((size_t)(n > 0 ? n : 1) * sizeof(uint64_t));
+        if (!base[i].k) { rc = -1; goto done; }
+        memcpy(base[i].k, inst_keys + inst_key_off[i], (size_t)n * sizeof(uint64_t));
+        qsort(base[i].k, (size_t)n, sizeof(uint64_t), cmp_u64);
+        base[i].n = n;
+    }
+    for (int64_t r = 0; r < n_req; ++r) {
+        const uint64_t *rk = req_keys + req_key_off[r];
+        int64_t nb = req_key_off[r + 1] - req_key_off[r];
+        int32_t c = 0;
+        for (int32_t i = 0; i < n_inst; ++i) {
+            int64_t b = 0;
+            while (b < nb && (keyset_has(&base[i], rk[b]) || keyset_has(&add[i], rk[b]))) ++b;
+            hits[r * n_inst + i] = (int32_t)b;
+            or_raw_features_row(L[r], (int32_t)b, inst + (int64_t)i * d_inst, d_inst, req + r * d_req, d_req, xf);
+            or_zscore(d, xf, mean, std, xz);
+            for (int k = 0; k < d; ++k) xd[k] = (double)xz[k];
+            float y = (float)forward_row(mode, n_layers, w, params, xd, NULL, NULL, NULL, ba, bb);
+            scores[r * n_inst + i] = y;
+            if (i > 0 && precedes(y, i, scores[r * n_inst + c], c)) c = i;
+        }
+        choice[r] = c;
+        int32_t cc = forced ? forced[r] : c;
+        if (cc < 0 || cc >= n_inst) continue;
+        if (q_col >= 0) inst[(int64_t)cc * d_inst + q_col] = inst[(int64_t)cc * d_inst + q_col] + 1.0f;
+        or_keyset *s = &add[cc];
+        if (s->n + nb > s->cap) {
+            int64_t ncap = (s->n + nb) * 2 + 16;
+            uint64_t *nk = (uint64_t *)realloc(s->k, (size_t)ncap * sizeof(uint64_t));
+            if (!nk) { rc = -1; goto done; }
+            s->k = nk;
+            s->cap = ncap;
+        }
+        memcpy(s->k + s->n, rk, (size_t)nb * sizeof(uint64_t));
+        s->n += nb;
+        qsort(s->k, (size_t)s->n, sizeof(uint64_t), cmp_u64);
+    }
+done:
+    if (base) for (int32_t i = 0; i < n_inst; ++i) free(base[i].k);
+    if (add) for (int32_t i = 0; i < n_inst; ++i) free(add[i].k);
+    free(base); free(add); free(xf); free(xz); free(xd); free(ba); free(bb);
+    return rc;
+}

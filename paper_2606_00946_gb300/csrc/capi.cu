@@ -16,7 +16,7 @@ const char* const kTraceNames[TR_COUNT] = {
     "ring_append", "publish", "train_gather", "gemm_fwd", "loss_grad", "gemm_dw", "reduce_dw",
     "colsum_db", "gemm_dx", "optimizer", "memset", "score_tc", "features", "publish_tc",
     "hash_screen", "probe_screen", "probe_walk", "gemm_tc_fwd", "gemm_tc_dw", "gemm_tc_dx", "prefix_index",
-    "index_insert", "guards", "ring_bounds", "replay_admit", "train_step"};
+    "index_insert", "guards", "ring_bounds", "replay_admit", "train_step", "route_seq"};
 }
 
 struct ls_ctx {
@@ -224,6 +224,8 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
   if (!c.use_index && cfg->prefix_mode != LS_PREFIX_FUSED) {
     A(dalloc(&c.bkeys, c.bkeys_cap));
     A(dalloc(&c.work, R * NI));
+  } else if (c.use_index) {
+    A(dalloc(&c.bkeys, c.bkeys_cap));  // block keys of a sequential-commit batch
   }
   A(dalloc(&c.work_n, 1));
   A(dalloc(&c.xin, NI * std::max(1, c.tc.d_pad)));
@@ -604,6 +606,55 @@ int ls_route_batch(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* 
                    int32_t* hits_opt, uint64_t* weight_version_out, void* stream) {
   return route_impl(h, n_req, tok, tok_off, req_feats, choice, best, nullptr, nullptr, false, scores_opt, hits_opt,
                     weight_version_out, stream);
+}
+
+int ls_route_sequential(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* tok_off,
+                        const float* req_feats, int32_t queue_col, int32_t* choice, float* best, float* scores_opt,
+                        int32_t* hits_opt, uint64_t* weight_version_out, void* stream) {
+  if (!h) return fail(LS_ERR_ARG, "ctx is NULL");
+  Ctx& c = h->c;
+  if (n_req < 0 || n_req > c.cfg.max_requests) return fail(LS_ERR_ARG, "n_req out of range");
+  if (n_req > 0 && (!tok || !tok_off || !choice || !best || (c.cfg.d_req > 0 && !req_feats)))
+    return fail(LS_ERR_ARG, "NULL argument");
+  if (queue_col < -1 || queue_col >= c.cfg.d_inst) return fail(LS_ERR_ARG, "queue_col outside [-1, d_inst)");
+  if (!c.use_index) return fail(LS_ERR_ARG, "sequential routing needs the prefix index mode");
+  if (c.n_inst < 1) return fail(LS_ERR_STATE, "no snapshot");
+  if (!c.have_norm) return fail(LS_ERR_STATE, "normaliser not set");
+  int wmax = 1;
+  for (int l = 0; l <= c.mlp.n_layers; ++l) wmax = std::max(wmax, c.mlp.w[l]);
+  if (!route_seq_smem(c.n_inst, c.cfg.d_inst, wmax, c.gW))
+    return fail(LS_ERR_ARG, "sequential routing: instances x widest layer beyond its shared-memory limit");
+  cudaStream_t s = S(stream);
+  const bool cap = capturing(s);
+  uint64_t v;
+  {
+    std::lock_guard<std::mutex> g(c.mu);
+    if (!c.have_published) return fail(LS_ERR_STATE, "no weights published");
+    v = c.version;
+    if (!cap && c.pub_recorded) LS_CK(cudaStreamWaitEvent(s, c.ev_pub, 0));
+  }
+  if (weight_version_out) *weight_version_out = v;
+  if (n_req == 0) return LS_OK;
+  LS_CK(traced(c, TR_HASH, 1, s, [&] {
+    return launch_hash_blocks(n_req, tok, tok_off, c.bkeys, nullptr, c.bkeys_cap, c.d_err, s);
+  }));
+  LS_CK(traced(c, TR_ROUTE_SEQ, 1, s, [&] {
+    return launch_route_seq(n_req, c.n_inst, c.cfg.d_inst, c.cfg.d_req, queue_col, tok_off, c.bkeys, c.bkeys_cap,
+                            req_feats, c.inst_state, c.mean, c.stdv, c.pub, c.st, c.mlp, c.gkeys, c.gmask, c.gW,
+                            (uint64_t)(c.gslots - 1), c.table_count, c.cfg.max_keys_per_instance, choice, best,
+                            scores_opt, hits_opt, c.d_err, s);
+  }));
+  if (c.use_tc && c.tc.pipe)  // instance template rows follow the updated instance rows
+    LS_CK(traced(c, TR_NORM_ROWS, 1, s, [&] {
+      return launch_inst_templates(c.n_inst, c.cfg.d_inst, c.inst_state, c.mean, c.stdv, c.tc.d_pad, c.xin, c.sms,
+                                   s);
+    }));
+  if (!cap) {
+    std::lock_guard<std::mutex> g(c.mu);
+    LS_CK(cudaEventRecord(c.ev_route, s));
+    c.route_recorded = true;
+  }
+  return LS_OK;
 }
 
 int ls_route_batch_guarded(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* tok_off,

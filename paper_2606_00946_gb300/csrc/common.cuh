@@ -119,7 +119,7 @@ enum TraceId {
   TR_GATHER, TR_GEMM_FWD, TR_LOSS, TR_GEMM_DW, TR_REDUCE, TR_COLSUM, TR_GEMM_DX, TR_OPT,
   TR_MEMSET, TR_SCORE_TC, TR_NORM_ROWS, TR_PUBLISH_TC, TR_HASH_BATCH, TR_SCREEN, TR_WALK,
   TR_GEMM_TC_FWD, TR_GEMM_TC_DW, TR_GEMM_TC_DX, TR_PREFIX_INDEX, TR_INDEX_INSERT,
-  TR_GUARDS, TR_BOUNDS, TR_REPLAY, TR_TRAIN_STEP, TR_COUNT
+  TR_GUARDS, TR_BOUNDS, TR_REPLAY, TR_TRAIN_STEP, TR_ROUTE_SEQ, TR_COUNT
 };
 extern const char* const kTraceNames[TR_COUNT];
 
@@ -446,6 +446,13 @@ cudaError_t launch_norm_rows(const int64_t* tok_off, const int32_t* hits, uint4*
                              const float* inst, int n_req, int d_req,
                              const float* req, const float* mean, const float* stdv, int d_pad,
                              uint16_t* xin, uint16_t* xrq, int sms, cudaStream_t s);
+size_t route_seq_smem(int n_inst, int d_inst, int wmax, int W);
+cudaError_t launch_route_seq(int n_req, int n_inst, int d_inst, int d_req, int q_col, const int64_t* tok_off,
+                             const uint64_t* bkeys, int64_t bcap, const float* req, float* inst, const float* mean,
+                             const float* stdv, const Published* pub, const DevState* st, const MlpDesc& m,
+                             uint64_t* gkeys, uint64_t* gmask, int W, uint64_t gslots_mask, int32_t* counts,
+                             int64_t max_keys, int32_t* choice, float* best, float* scores, int32_t* hits, int* err,
+                             cudaStream_t s);
 cudaError_t launch_inst_templates(int n_inst, int d_inst, const float* inst, const float* mean, const float* stdv,
                                   int d_pad, uint16_t* xin, int sms, cudaStream_t s);
 cudaError_t launch_feature_image(const int64_t* tok_off, const int32_t* hits, int n_inst, const uint16_t* xin,

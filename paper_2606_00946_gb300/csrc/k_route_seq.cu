@@ -1,0 +1,353 @@
+// Sequential-commit routing (Sec. 4.2 cluster snapshot manager and prefix
+// KV-cache tracker; Sec. 4.3.1 P1: the gateway routes one request at a time):
+// the requests of a batch are routed in order, and each decision is committed
+// before the next request is scored -- the chosen instance's queue count grows
+// by one and the prompt's full blocks join its cache (the prefix index gains
+// the instance's bit for each block key), so a later request with the same
+// prefix sees the hit and the longer queue.
+//
+// One persistent CTA walks the requests (the chain is inherently serial); per
+// request:
+//   1. hit lengths for every instance from the prefix index: the CTA's
+//      threads look up a chunk of the prompt's block keys at once, a block-wide
+//      prefix AND of their instance masks gives the instances matching every
+//      block so far, and each instance finds where its bit dies by bisection;
+//   2. feature rows (pair block, the instance rows as updated by earlier
+//      decisions, request extras), z-scored, bf16-rounded in bf16 mode;
+//   3. the predictor on CUDA cores: warp per output column, lanes across K,
+//      rows in turn, published weights (bf16-rounded in bf16 mode, fp32 sums);
+//   4. the argmin (lowest (score, index), NaN last);
+//   5. the commit: queue count + 1, index insertion of the prompt's keys with
+//      the chosen instance's bit (distinct keys counted against the table
+//      capacity).
+// Index reads bypass L1 (the CTA's own insertions must be visible to it).
+#include "blockhash.cuh"
+#include "common.cuh"
+
+namespace ls {
+namespace {
+using namespace bh;
+
+constexpr int kSeqThreads = 512;
+constexpr int kSeqWarps = kSeqThreads / 32;
+constexpr int kSeqMaxW = 8;  // instance-mask words (512 instances)
+
+struct SeqArgs {
+  int n_req, n_inst, d_inst, d_req, q_col;
+  const int64_t* tok_off;
+  const uint64_t* bkeys;  // block keys of the batch at (tok_off[r] - tok_off[0]) / 16 + b
+  const float* req;
+  float* inst;            // [n_inst, d_inst] instance rows (updated in place at the end)
+  const float* mean;
+  const float* stdv;
+  const float* params0;
+  const float* params1;
+  const DevState* st;
+  MlpDesc m;
+  int wmax;               // widest layer input / output
+  uint64_t* gkeys;
+  uint64_t* gmask;
+  int W;
+  uint64_t gslots_mask;
+  int32_t* counts;
+  int64_t max_keys;
+  int32_t* choice;
+  float* best;
+  float* scores;          // [n_req, n_inst] or NULL
+  int32_t* hits;          // [n_req, n_inst] or NULL
+  int* err;
+};
+
+// Index lookups through L2 (ld.global.cg), so that keys this CTA inserted are seen.
+__device__ __forceinline__ void seq_lookup(const SeqArgs& a, uint64_t key, uint64_t (&mw)[kSeqMaxW]) {
+#pragma unroll
+  for (int w = 0; w < kSeqMaxW; ++w) mw[w] = 0;
+  const uint64_t mslots = a.gslots_mask;
+  uint64_t s = key & mslots;
+  for (uint64_t n = 0; n <= mslots; ++n) {
+    const uint64_t k = a.W == 1 ? __ldcg(a.gkeys + 2 * s) : __ldcg(a.gkeys + s);
+    if (k == key) {
+      if (a.W == 1) mw[0] = __ldcg(a.gkeys + 2 * s + 1);
+      else
+        for (int w = 0; w < a.W; ++w) mw[w] = __ldcg(a.gmask + s * a.W + w);
+      return;
+    }
+    if (k == 0) return;
+    s = (s + 1) & mslots;
+  }
+}
+
+// Insertion of `key` for instance `inst` (the protocol of the snapshot's index
+// insert: CAS on an empty slot, OR of the instance's bit, a newly set bit
+// counts one distinct key of the instance).
+__device__ __forceinline__ void seq_insert(const SeqArgs& a, uint64_t key, int inst) {
+  unsigned long long* tab = reinterpret_cast<unsigned long long*>(a.gkeys);
+  const int kstride = a.W == 1 ? 2 : 1;
+  uint64_t s = key & a.gslots_mask;
+  int64_t slot = -1;
+  for (uint64_t n = 0; n <= a.gslots_mask; ++n) {
+    const unsigned long long prev = atomicCAS(tab + s * kstride, 0ull, (unsigned long long)key);
+    if (prev == 0ull || prev == key) { slot = (int64_t)s; break; }
+    s = (s + 1) & a.gslots_mask;
+  }
+  if (slot < 0) { latch_error(a.err, LS_ERR_TABLE_FULL); return; }
+  const unsigned long long bit = 1ull << (inst & 63);
+  unsigned long long* mword = a.W == 1 ? tab + 2 * slot + 1
+                                       : reinterpret_cast<unsigned long long*>(a.gmask + slot * a.W + (inst >> 6));
+  const unsigned long long old = atomicOr(mword, bit);
+  if (!(old & bit)) {
+    const int cnt = atomicAdd(a.counts + inst, 1);
+    if (cnt >= a.max_keys) latch_error(a.err, LS_ERR_TABLE_FULL);
+  }
+}
+
+__device__ __forceinline__ bool seq_precedes(float a, int i, float b, int j) {
+  const bool an = a != a, bn = b != b;
+  if (an != bn) return bn;
+  if (!an && a != b) return a < b;
+  return i < j;
+}
+
+__global__ void __launch_bounds__(kSeqThreads, 1) k_route_seq(const __grid_constant__ SeqArgs a, int64_t bcap) {
+  extern __shared__ uint8_t smem_raw[];
+  const int N = a.n_inst, DI = a.d_inst, W = a.W;
+  const MlpDesc& m = a.m;
+  const int d = m.w[0];
+  float* sinst = reinterpret_cast<float*>(smem_raw);              // [N][d_inst]
+  float* X0 = sinst + (size_t)N * (DI > 0 ? DI : 1);               // [N][wmax]
+  float* X1 = X0 + (size_t)N * a.wmax;                             // [N][wmax]
+  float* sc = X1 + (size_t)N * a.wmax;                             // [N] scores
+  int32_t* hh = reinterpret_cast<int32_t*>(sc + N);                // [N] hit lengths
+  uint64_t* PA = reinterpret_cast<uint64_t*>(hh + ((N + 1) & ~1)); // [kSeqThreads][W] prefix AND
+  uint64_t* wtot = PA + (size_t)kSeqThreads * W;                   // [kSeqWarps][W]
+  uint64_t* carry = wtot + (size_t)kSeqWarps * W;                  // [W]
+  float* rv = reinterpret_cast<float*>(carry + W);                 // [kSeqWarps] argmin values
+  int* ri = reinterpret_cast<int*>(rv + kSeqWarps);                // [kSeqWarps] argmin indices
+  __shared__ int s_buf, s_go, s_choice;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  if (tid == 0) s_buf = *reinterpret_cast<const volatile int32_t*>(&a.st->cur) == 1 ? 1 : 0;
+  for (int e = tid; e < N * DI; e += kSeqThreads) sinst[e] = a.inst[e];
+  __syncthreads();
+  const float* __restrict__ params = s_buf ? a.params1 : a.params0;
+  const int64_t base = a.tok_off[0];
+  for (int r = 0; r < a.n_req; ++r) {
+    const int64_t t0 = a.tok_off[r];
+    const int64_t L = a.tok_off[r + 1] - t0;
+    const int64_t nb = L / kBlockTok;
+    const int64_t k0 = (t0 - base) / kBlockTok;
+    // ---- 1. hit lengths
+    for (int i = tid; i < N; i += kSeqThreads) hh[i] = -1;
+    if (tid < W) {
+      const int lo = 64 * tid;
+      carry[tid] = N >= lo + 64 ? ~0ull : (N > lo ? ((1ull << (N - lo)) - 1ull) : 0ull);
+    }
+    __syncthreads();
+    for (int64_t p = 0; p < nb; p += kSeqThreads) {
+      const int64_t b = p + tid;
+      uint64_t mw[kSeqMaxW];
+      if (b < nb) {
+        const uint64_t key = k0 + b < bcap ? a.bkeys[k0 + b] : 0ull;  // past the key scratch: a miss
+        if (key) seq_lookup(a, key, mw);
+        else
+#pragma unroll
+          for (int w = 0; w < kSeqMaxW; ++w) mw[w] = 0;
+      } else {
+#pragma unroll
+        for (int w = 0; w < kSeqMaxW; ++w) mw[w] = ~0ull;  // past the prompt: changes nothing
+      }
+#pragma unroll
+      for (int w = 0; w < kSeqMaxW; ++w) {
+        if (w >= W) break;
+        uint64_t x = mw[w];
+#pragma unroll
+        for (int k = 0; k < 5; ++k) {
+          const uint64_t y = __shfl_up_sync(kFull, x, 1 << k);
+          if (lane >= (1 << k)) x &= y;
+        }
+        mw[w] = x;
+        if (lane == 31) wtot[warp * W + w] = x;
+      }
+      __syncthreads();
+#pragma unroll
+      for (int w = 0; w < kSeqMaxW; ++w) {
+        if (w >= W) break;
+        uint64_t e = carry[w];
+        for (int v = 0; v < warp; ++v) e &= wtot[v * W + w];
+        PA[tid * W + w] = e & mw[w];
+      }
+      __syncthreads();
+      const int last = (int)(nb - p < kSeqThreads ? nb - p : kSeqThreads) - 1;
+      for (int i = tid; i < N; i += kSeqThreads) {
+        if (hh[i] >= 0) continue;
+        const int wi = i >> 6;
+        const uint64_t bit = 1ull << (i & 63);
+        if (PA[last * W + wi] & bit) continue;  // still matching after this chunk
+        int lo = 0, hi = last;                   // first t whose prefix AND lost the bit
+        while (lo < hi) {
+          const int mid = (lo + hi) >> 1;
+          if (PA[mid * W + wi] & bit) lo = mid + 1; else hi = mid;
+        }
+        hh[i] = (int32_t)(p + lo);
+      }
+      __syncthreads();
+      if (tid == 0) {
+        int any = 0;
+        for (int w = 0; w < W; ++w) {
+          carry[w] = PA[last * W + w];
+          any |= carry[w] != 0;
+        }
+        s_go = any;
+      }
+      __syncthreads();
+      if (!s_go) break;
+    }
+    for (int i = tid; i < N; i += kSeqThreads)
+      if (hh[i] < 0) hh[i] = (int32_t)nb;  // matching every full block
+    __syncthreads();
+    // ---- 2. feature rows
+    for (int e = tid; e < N * d; e += kSeqThreads) {
+      const int i = e / d, k = e - i * d;
+      float raw;
+      if (k < kPair) raw = raw_feature(k, L, hh[i], nullptr, 0, nullptr);
+      else if (k < kPair + DI) raw = sinst[i * DI + (k - kPair)];
+      else raw = a.req[(int64_t)r * a.d_req + (k - kPair - DI)];
+      const float x = zscore(raw, a.mean[k], a.stdv[k]);
+      X0[i * a.wmax + k] = m.bf16 ? round_bf16(x) : x;
+    }
+    __syncthreads();
+    // ---- 3. the predictor, warp per output column
+    float* xin = X0;
+    float* xout = X1;
+    for (int l = 0; l < m.n_layers; ++l) {
+      const int in = m.w[l], out = m.w[l + 1];
+      const bool last_layer = l + 1 == m.n_layers;
+      const float* __restrict__ Wl = params + m.woff[l];
+      const float* __restrict__ bl = params + m.boff[l];
+      for (int o = warp; o < out; o += kSeqWarps) {
+        float wr[16];
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const int k = lane + 32 * j;
+          wr[j] = k < in ? __ldg(Wl + (int64_t)o * in + k) : 0.0f;
+        }
+        const float bo = __ldg(bl + o);
+        for (int i = 0; i < N; ++i) {
+          float part = 0.0f;
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const int k = lane + 32 * j;
+            if (k < in) part = fmaf(wr[j], xin[i * a.wmax + k], part);
+          }
+#pragma unroll
+          for (int s = 16; s; s >>= 1) part += __shfl_xor_sync(kFull, part, s);
+          if (lane == 0) {
+            const float z = part + bo;
+            if (last_layer) sc[i] = z;
+            else {
+              const float act = fmaxf(z, 0.0f);
+              xout[i * a.wmax + o] = m.bf16 ? round_bf16(act) : act;
+            }
+          }
+        }
+      }
+      __syncthreads();
+      float* t = xin;
+      xin = xout;
+      xout = t;
+    }
+    // ---- 4. selection
+    {
+      float bv = 0.0f;
+      int bi = -1;
+      for (int i = tid; i < N; i += kSeqThreads)
+        if (bi < 0 || seq_precedes(sc[i], i, bv, bi)) { bv = sc[i]; bi = i; }
+#pragma unroll
+      for (int s = 16; s; s >>= 1) {
+        const float ov = __shfl_xor_sync(kFull, bv, s);
+        const int oi = __shfl_xor_sync(kFull, bi, s);
+        if (oi >= 0 && (bi < 0 || seq_precedes(ov, oi, bv, bi))) { bv = ov; bi = oi; }
+      }
+      if (lane == 0) { rv[warp] = bv; ri[warp] = bi; }
+      __syncthreads();
+      if (tid == 0) {
+        float v = rv[0];
+        int c = ri[0];
+        for (int w = 1; w < kSeqWarps; ++w)
+          if (ri[w] >= 0 && (c < 0 || seq_precedes(rv[w], ri[w], v, c))) { v = rv[w]; c = ri[w]; }
+        s_choice = c;
+        a.choice[r] = c;
+        a.best[r] = v;
+        if (a.q_col >= 0 && c >= 0) sinst[c * DI + a.q_col] += 1.0f;  // ---- 5a. the queue grows
+      }
+    }
+    if (a.scores)
+      for (int i = tid; i < N; i += kSeqThreads) a.scores[(int64_t)r * N + i] = sc[i];
+    if (a.hits)
+      for (int i = tid; i < N; i += kSeqThreads) a.hits[(int64_t)r * N + i] = hh[i];
+    __syncthreads();
+    // ---- 5b. the chosen instance caches the prompt's blocks
+    const int c = s_choice;
+    if (c >= 0)
+      for (int64_t b = tid; b < nb; b += kSeqThreads)
+        if (k0 + b < bcap) seq_insert(a, a.bkeys[k0 + b], c);
+    __syncthreads();
+  }
+  for (int e = tid; e < N * DI; e += kSeqThreads) a.inst[e] = sinst[e];
+}
+
+}  // namespace
+
+// Shared memory of the sequential route, 0 if the shape does not fit.
+size_t route_seq_smem(int n_inst, int d_inst, int wmax, int W) {
+  const size_t b = (size_t)n_inst * (d_inst > 0 ? d_inst : 1) * 4 + 2 * (size_t)n_inst * wmax * 4 +
+                   (size_t)n_inst * 4 + (size_t)((n_inst + 1) & ~1) * 4 + (size_t)kSeqThreads * W * 8 +
+                   (size_t)kSeqWarps * W * 8 + (size_t)W * 8 + (size_t)kSeqWarps * 8 + 64;
+  return b <= 200 * 1024 && W <= kSeqMaxW && wmax <= 512 ? b : 0;
+}
+
+cudaError_t launch_route_seq(int n_req, int n_inst, int d_inst, int d_req, int q_col, const int64_t* tok_off,
+                             const uint64_t* bkeys, int64_t bcap, const float* req, float* inst, const float* mean,
+                             const float* stdv, const Published* pub, const DevState* st, const MlpDesc& m,
+                             uint64_t* gkeys, uint64_t* gmask, int W, uint64_t gslots_mask, int32_t* counts,
+                             int64_t max_keys, int32_t* choice, float* best, float* scores, int32_t* hits, int* err,
+                             cudaStream_t s) {
+  if (n_req <= 0) return cudaSuccess;
+  SeqArgs a{};
+  a.n_req = n_req;
+  a.n_inst = n_inst;
+  a.d_inst = d_inst;
+  a.d_req = d_req;
+  a.q_col = q_col;
+  a.tok_off = tok_off;
+  a.bkeys = bkeys;
+  a.req = req;
+  a.inst = inst;
+  a.mean = mean;
+  a.stdv = stdv;
+  a.params0 = pub[0].params;
+  a.params1 = pub[1].params;
+  a.st = st;
+  a.m = m;
+  int wmax = 1;
+  for (int l = 0; l <= m.n_layers; ++l) wmax = std::max(wmax, m.w[l]);
+  a.wmax = wmax;
+  a.gkeys = gkeys;
+  a.gmask = gmask;
+  a.W = W;
+  a.gslots_mask = gslots_mask;
+  a.counts = counts;
+  a.max_keys = max_keys;
+  a.choice = choice;
+  a.best = best;
+  a.scores = scores;
+  a.hits = hits;
+  a.err = err;
+  const size_t smem = route_seq_smem(n_inst, d_inst, wmax, W);
+  if (!smem) return cudaErrorInvalidValue;
+  cudaError_t e = cudaFuncSetAttribute(k_route_seq, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  k_route_seq<<<1, kSeqThreads, smem, s>>>(a, bcap);
+  return cudaGetLastError();
+}
+
+}  // namespace ls

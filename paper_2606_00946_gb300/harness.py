@@ -156,6 +156,19 @@ class Router:
         return dict(choice=choice, best=best, status=status, fallback=fallback, scores=scores, hits=hits,
                     version=ver)
 
+    def route_sequential(self, tok, tok_off, req_feats, n_inst, queue_col=0, stream=None):
+        """Sequential-commit route: each decision updates the chosen instance's
+        queue and cache before the next request is scored."""
+        n_req = tok_off.numel() - 1
+        choice = torch.empty(n_req, dtype=torch.int32, device="cuda")
+        best = torch.empty(n_req, dtype=torch.float32, device="cuda")
+        scores = torch.empty(n_req, n_inst, dtype=torch.float32, device="cuda")
+        hits = torch.empty(n_req, n_inst, dtype=torch.int32, device="cuda")
+        rc, ver = L.ls_route_sequential(self.h, n_req, tok, tok_off, req_feats, queue_col, choice, best, scores,
+                                        hits, stream)
+        L.check(rc)
+        return dict(choice=choice, best=best, scores=scores, hits=hits, version=ver)
+
     def replay_admit(self, diag=False, stream=None):
         """One admission round of the replay pool; with diag, returns (d, n)
         per candidate / kept slot (device tensors of the pools' capacities)."""

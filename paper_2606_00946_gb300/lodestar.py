@@ -85,6 +85,7 @@ _SIGS = {
     "ls_get_bounds": (C.c_int, [_P, _i32, _P, _P, _P]),
     "ls_route_batch_guarded": (C.c_int, [_P, _i32, _P, _P, _P, _P, _P, _P, _P, _P, _P,
                                          C.POINTER(C.c_uint64), _P]),
+    "ls_route_sequential": (C.c_int, [_P, _i32, _P, _P, _P, _i32, _P, _P, _P, _P, C.POINTER(C.c_uint64), _P]),
     "ls_trace_enable": (C.c_int, [_P, _i32]),
     "ls_trace_read": (C.c_int, [_P, C.POINTER(ls_trace_entry), _i32, C.POINTER(_i32)]),
     "ls_prefix_hits_static": (C.c_int, [_i32, _P, _P, _i64, _P, _i64, _i32, _P, _P]),
@@ -305,6 +306,15 @@ def ls_route_batch_guarded(ctx, n_req, tok, tok_off, req_feats, choice, best, st
                                       ptr(best), ptr(status), ptr(fallback_opt), ptr(scores_opt), ptr(hits_opt),
                                       C.byref(v), stream_handle(stream))
     return rc, v.value
+
+
+def ls_route_sequential(ctx, n_req, tok, tok_off, req_feats, queue_col, choice, best, scores_opt=None,
+                        hits_opt=None, stream=None):
+    ver = C.c_uint64(0)
+    rc = lib().ls_route_sequential(ctx, int(n_req), ptr(tok), ptr(tok_off), ptr(req_feats), int(queue_col),
+                                   ptr(choice), ptr(best), ptr(scores_opt), ptr(hits_opt), C.byref(ver),
+                                   stream_handle(stream))
+    return rc, ver.value
 
 
 def ls_trace_enable(ctx, on=True) -> int:
