@@ -108,21 +108,43 @@ __device__ __forceinline__ bool seq_precedes(float a, int i, float b, int j) {
   return i < j;
 }
 
+// Byte offsets of the shared-memory arrays (each 16-byte aligned).
+struct SeqSmem {
+  size_t inst, x0, x1, sc, hh, pa, wtot, carry, rv, ri, total;
+};
+__host__ __device__ __forceinline__ size_t seq_al(size_t b) { return (b + 15) & ~(size_t)15; }
+__host__ __device__ __forceinline__ SeqSmem seq_smem(int N, int DI, int wmax, int W) {
+  SeqSmem o;
+  o.inst = 0;                                                   // [N][d_inst] fp32
+  o.x0 = seq_al(o.inst + (size_t)N * (DI > 0 ? DI : 1) * 4);    // [N][wmax] fp32
+  o.x1 = seq_al(o.x0 + (size_t)N * wmax * 4);                   // [N][wmax] fp32
+  o.sc = seq_al(o.x1 + (size_t)N * wmax * 4);                   // [N] scores
+  o.hh = seq_al(o.sc + (size_t)N * 4);                          // [N] hit lengths
+  o.pa = seq_al(o.hh + (size_t)N * 4);                          // [kSeqThreads][W] prefix AND
+  o.wtot = seq_al(o.pa + (size_t)kSeqThreads * W * 8);          // [kSeqWarps][W]
+  o.carry = seq_al(o.wtot + (size_t)kSeqWarps * W * 8);         // [W]
+  o.rv = seq_al(o.carry + (size_t)W * 8);                       // [kSeqWarps] argmin values
+  o.ri = seq_al(o.rv + (size_t)kSeqWarps * 4);                  // [kSeqWarps] argmin indices
+  o.total = seq_al(o.ri + (size_t)kSeqWarps * 4);
+  return o;
+}
+
 __global__ void __launch_bounds__(kSeqThreads, 1) k_route_seq(const __grid_constant__ SeqArgs a, int64_t bcap) {
-  extern __shared__ uint8_t smem_raw[];
+  extern __shared__ __align__(16) uint8_t smem_raw[];
   const int N = a.n_inst, DI = a.d_inst, W = a.W;
   const MlpDesc& m = a.m;
   const int d = m.w[0];
-  float* sinst = reinterpret_cast<float*>(smem_raw);              // [N][d_inst]
-  float* X0 = sinst + (size_t)N * (DI > 0 ? DI : 1);               // [N][wmax]
-  float* X1 = X0 + (size_t)N * a.wmax;                             // [N][wmax]
-  float* sc = X1 + (size_t)N * a.wmax;                             // [N] scores
-  int32_t* hh = reinterpret_cast<int32_t*>(sc + N);                // [N] hit lengths
-  uint64_t* PA = reinterpret_cast<uint64_t*>(hh + ((N + 1) & ~1)); // [kSeqThreads][W] prefix AND
-  uint64_t* wtot = PA + (size_t)kSeqThreads * W;                   // [kSeqWarps][W]
-  uint64_t* carry = wtot + (size_t)kSeqWarps * W;                  // [W]
-  float* rv = reinterpret_cast<float*>(carry + W);                 // [kSeqWarps] argmin values
-  int* ri = reinterpret_cast<int*>(rv + kSeqWarps);                // [kSeqWarps] argmin indices
+  const SeqSmem o = seq_smem(N, DI, a.wmax, W);
+  float* sinst = reinterpret_cast<float*>(smem_raw + o.inst);
+  float* X0 = reinterpret_cast<float*>(smem_raw + o.x0);
+  float* X1 = reinterpret_cast<float*>(smem_raw + o.x1);
+  float* sc = reinterpret_cast<float*>(smem_raw + o.sc);
+  int32_t* hh = reinterpret_cast<int32_t*>(smem_raw + o.hh);
+  uint64_t* PA = reinterpret_cast<uint64_t*>(smem_raw + o.pa);
+  uint64_t* wtot = reinterpret_cast<uint64_t*>(smem_raw + o.wtot);
+  uint64_t* carry = reinterpret_cast<uint64_t*>(smem_raw + o.carry);
+  float* rv = reinterpret_cast<float*>(smem_raw + o.rv);
+  int* ri = reinterpret_cast<int*>(smem_raw + o.ri);
   __shared__ int s_buf, s_go, s_choice;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   if (tid == 0) s_buf = *reinterpret_cast<const volatile int32_t*>(&a.st->cur) == 1 ? 1 : 0;
@@ -299,10 +321,9 @@ __global__ void __launch_bounds__(kSeqThreads, 1) k_route_seq(const __grid_const
 
 // Shared memory of the sequential route, 0 if the shape does not fit.
 size_t route_seq_smem(int n_inst, int d_inst, int wmax, int W) {
-  const size_t b = (size_t)n_inst * (d_inst > 0 ? d_inst : 1) * 4 + 2 * (size_t)n_inst * wmax * 4 +
-                   (size_t)n_inst * 4 + (size_t)((n_inst + 1) & ~1) * 4 + (size_t)kSeqThreads * W * 8 +
-                   (size_t)kSeqWarps * W * 8 + (size_t)W * 8 + (size_t)kSeqWarps * 8 + 64;
-  return b <= 200 * 1024 && W <= kSeqMaxW && wmax <= 512 ? b : 0;
+  if (W < 1 || W > kSeqMaxW || wmax > 512 || n_inst < 1) return 0;
+  const size_t b = seq_smem(n_inst, d_inst, wmax, W).total;
+  return b <= 200 * 1024 ? b : 0;
 }
 
 cudaError_t launch_route_seq(int n_req, int n_inst, int d_inst, int d_req, int q_col, const int64_t* tok_off,
