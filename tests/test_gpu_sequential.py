@@ -62,7 +62,9 @@ CASES = [
 def test_sequential_route_steps_and_final_state(name, over):
     cfg = dataclasses.replace(W.CONFIGS[name], n_samples=0, **over)
     wl = W.generate(cfg, with_samples=False)
-    r = H.Router.for_config(cfg)
+    # room for the keys the batch's commits add (a full table latches LS_ERR_TABLE_FULL)
+    room = cfg.cache_blocks + int(np.sum(np.diff(wl.tok_off) // 16))
+    r = H.Router.for_config(cfg, max_keys_per_instance=room)
     dw = H.DeviceWorkload(wl)
     dw.load(r)
     q_col = 0
@@ -98,6 +100,17 @@ def test_sequential_route_steps_and_final_state(name, over):
     wl_f = dataclasses.replace(wl, inst_state=inst_final)
     ref_after = oracle.route(wl_f, hits=want_h, bounds=True, threads=THREADS)
     assert_scores_close(after["scores"].cpu().numpy(), ref_after, TOL[cfg.dtype], f"after sequential {name}")
+    r.close()
+
+
+def test_sequential_route_on_a_full_table_latches_table_full():
+    cfg = dataclasses.replace(W.CONFIGS["tiny"], n_samples=0)
+    wl = W.generate(cfg, with_samples=False)
+    r = H.Router.for_config(cfg)                   # caches hold exactly max_keys_per_instance blocks
+    dw = H.DeviceWorkload(wl)
+    dw.load(r)
+    r.route_sequential(dw.tok, dw.tok_off, dw.req_feats, cfg.n_inst)
+    assert r.sync() == L.LS_ERR_TABLE_FULL
     r.close()
 
 
