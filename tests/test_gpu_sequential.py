@@ -80,7 +80,7 @@ def test_sequential_route_steps_and_final_state(name, over):
     assert np.array_equal(rep["inst"], inst_final)
     assert_scores_close(gs, ref, TOL[cfg.dtype], f"sequential {name}")
     frac = assert_choices(gc, gs, ref, TOL[cfg.dtype])
-    assert frac > 0.9
+    assert frac >= (0.9 if cfg.dtype == "f32" else 0.8)   # decisions the clear-gap check pins
     assert np.array_equal(out["best"].cpu().numpy(), gs[np.arange(cfg.n_req), gc])
     # commits mattered: some later request saw a hit or a queue the batch route does not see
     batch0 = oracle.route(wl, inst_keys=(ik, iko))
