@@ -283,6 +283,36 @@ def measure_paper_point(L, H, W, dev, stream, n=400):
                     "host time here is the C-ABI call from Python until the choice is in pinned host memory"}
 
 
+def measure_sequential(L, H, W, dev, stream, name, n_req, calls=4):
+    """Sequential-commit routing (Sec. 4.2 snapshot manager; Sec. 4.3.1 P1):
+    one call routes n_req requests in order, committing each decision (queue
+    + 1, prompt blocks cached on the chosen instance) before the next request;
+    device time per call and per request (CUDA events)."""
+    import dataclasses
+    import torch
+    cfg = dataclasses.replace(W.CONFIGS[name], n_req=n_req, n_samples=0)
+    wl = W.generate(cfg, with_samples=False)
+    room = cfg.cache_blocks + (calls + 2) * int(np.sum(np.diff(wl.tok_off) // 16))
+    r = H.Router.for_config(cfg, max_keys_per_instance=room)
+    dw = H.DeviceWorkload(wl, device=dev)
+    dw.load(r)
+    r.route_sequential(dw.tok, dw.tok_off, dw.req_feats, cfg.n_inst)       # warm-up call
+    ts = []
+    for _ in range(calls):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        r.route_sequential(dw.tok, dw.tok_off, dw.req_feats, cfg.n_inst)
+        e1.record(stream)
+        e1.synchronize()
+        ts.append(e0.elapsed_time(e1))
+    status = r.sync()
+    r.close()
+    ms = float(np.median(ts))
+    return {"instances": cfg.n_inst, "predictor": "x".join(str(w) for w in cfg.widths), "requests_per_call": n_req,
+            "ms_per_call": ms, "us_per_request": 1e3 * ms / n_req, "decisions_per_s": n_req / (ms / 1e3),
+            "status": int(status)}
+
+
 def measure_training_config(L, H, W, dev, steps=1000):
     """The online-training throughput configuration: a ring of 2^20 logged
     128-dim records, Adam (lr 3e-4, batch 4096) on the 128-256-256-256-1
@@ -1147,6 +1177,9 @@ def main():
             configs["training"] = measure_training_config(L, H, W, dev)
         if not args.no_paper_point:
             configs["paper_point"] = measure_paper_point(L, H, W, dev, stream)
+            configs["sequential_commit"] = {
+                "paper": measure_sequential(L, H, W, dev, stream, "paper", 256),
+                "homogeneous": measure_sequential(L, H, W, dev, stream, "homogeneous", 512)}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
