@@ -268,6 +268,17 @@ int ls_train_step(ls_ctx *ctx, int32_t batch, const int32_t *idx, int32_t opt, f
  * started with (each route takes the index once, before it scores). */
 int ls_publish(ls_ctx *ctx, void *stream);
 
+/* The bf16 feature rows the tensor-core scorer read for the last routed batch
+ * (Sec. 4.1 Features; Algorithm 4 Normalize), rows row0 .. row0 + n_rows - 1
+ * of the batch (row r * n_inst + i), d bf16 values each (raw bit patterns),
+ * written to DEVICE out [n_rows, d].  Decoded from the buffers the scorer
+ * consumes -- the feature image's operand tiles (pipelined scorer) or the pair
+ * chunks and instance / request template rows the other tensor-core scorers
+ * combine on chip -- so this is a parity hook on the production features, not
+ * a recomputation.  Rows of the batch only (beyond it the contents are stale).
+ * LS_ERR_STATE with the CUDA-core scorer (its rows never leave registers). */
+int ls_read_features(ls_ctx *ctx, int64_t row0, int64_t n_rows, uint16_t *out, void *stream);
+
 /* Sequential-commit routing (Sec. 4.2 cluster snapshot manager and prefix
  * KV-cache tracker; Sec. 4.3.1 P1: the gateway routes one request at a time):
  * the requests are routed in order, r = 0, 1, ..., and each decision is

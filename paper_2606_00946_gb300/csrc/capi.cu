@@ -608,6 +608,17 @@ int ls_route_batch(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* 
                     weight_version_out, stream);
 }
 
+int ls_read_features(ls_ctx* h, int64_t row0, int64_t n_rows, uint16_t* out, void* stream) {
+  if (!h) return fail(LS_ERR_ARG, "ctx is NULL");
+  Ctx& c = h->c;
+  if (!c.use_tc) return fail(LS_ERR_STATE, "the CUDA-core scorer assembles feature rows in registers only");
+  if (row0 < 0 || n_rows < 0 || (n_rows > 0 && !out)) return fail(LS_ERR_ARG, "bad rows or NULL output");
+  const int64_t cap = (int64_t)c.cfg.max_requests * c.cfg.max_instances;
+  if (row0 + n_rows > cap) return fail(LS_ERR_ARG, "rows beyond the batch buffers");
+  LS_CK(launch_read_features(row0, n_rows, c.d, c.tc, c.n_inst, c.ximg, c.pairx, c.xin, c.xrq, out, S(stream)));
+  return LS_OK;
+}
+
 int ls_route_sequential(ls_ctx* h, int32_t n_req, const int32_t* tok, const int64_t* tok_off,
                         const float* req_feats, int32_t queue_col, int32_t* choice, float* best, float* scores_opt,
                         int32_t* hits_opt, uint64_t* weight_version_out, void* stream) {

@@ -447,6 +447,9 @@ cudaError_t launch_norm_rows(const int64_t* tok_off, const int32_t* hits, uint4*
                              const float* req, const float* mean, const float* stdv, int d_pad,
                              uint16_t* xin, uint16_t* xrq, int sms, cudaStream_t s);
 size_t route_seq_smem(int n_inst, int d_inst, int wmax, int W);
+cudaError_t launch_read_features(int64_t row0, int64_t n_rows, int d, const TcPlan& p, int n_inst,
+                                 const uint8_t* ximg, const uint4* pairx, const uint16_t* xin, const uint16_t* xrq,
+                                 uint16_t* out, cudaStream_t s);
 cudaError_t launch_route_seq(int n_req, int n_inst, int d_inst, int d_req, int q_col, const int64_t* tok_off,
                              const uint64_t* bkeys, int64_t bcap, const float* req, float* inst, const float* mean,
                              const float* stdv, const Published* pub, const DevState* st, const MlpDesc& m,

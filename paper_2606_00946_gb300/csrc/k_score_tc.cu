@@ -1228,6 +1228,43 @@ bool plan_tc(const MlpDesc& m, TcPlan& p) {
   return true;
 }
 
+// The bf16 feature rows the tensor-core scorers read for the last batch, row
+// r * n_inst + i of [rows, d], decoded from where they live: the feature
+// image's MMA-layout tiles (pipelined scorer), or the pair chunk OR-ed with
+// the instance and request template rows (the other tensor-core scorers,
+// exactly as their tile builders combine them).
+__global__ void k_read_features(int64_t row0, int64_t n_rows, int d, int d_pad, int n_inst, int pipe,
+                                const uint8_t* __restrict__ ximg, const uint4* __restrict__ pairx,
+                                const uint16_t* __restrict__ xin, const uint16_t* __restrict__ xrq,
+                                uint16_t* __restrict__ out) {
+  const int64_t total = n_rows * d;
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t g = row0 + e / d;
+    const int k = (int)(e % d);
+    uint16_t v;
+    if (pipe) {
+      const int64_t t = g / kTileM;
+      const int m = (int)(g - t * kTileM);
+      const int64_t xbytes = (int64_t)(d_pad / 64) * kTileM * 128;
+      v = *reinterpret_cast<const uint16_t*>(ximg + t * xbytes + sw128_offset(m, k, kTileM));
+    } else {
+      const int64_t r = g / n_inst, i = g - r * n_inst;
+      const uint16_t* pc = reinterpret_cast<const uint16_t*>(pairx + g);
+      v = (uint16_t)(xin[i * d_pad + k] | xrq[r * d_pad + k] | (k < 8 ? pc[k] : 0));
+    }
+    out[e] = v;
+  }
+}
+
+cudaError_t launch_read_features(int64_t row0, int64_t n_rows, int d, const TcPlan& p, int n_inst,
+                                 const uint8_t* ximg, const uint4* pairx, const uint16_t* xin, const uint16_t* xrq,
+                                 uint16_t* out, cudaStream_t s) {
+  if (n_rows <= 0) return cudaSuccess;
+  const int grid = (int)std::min<int64_t>((n_rows * d + 255) / 256, 4096);
+  k_read_features<<<grid, 256, 0, s>>>(row0, n_rows, d, p.d_pad, n_inst, p.pipe, ximg, pairx, xin, xrq, out);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_norm_rows(const int64_t* tok_off, const int32_t* hits, uint4* pairx, int n_inst, int d_inst,
                              const float* inst, int n_req, int d_req, const float* req, const float* mean,
                              const float* stdv, int d_pad, uint16_t* xin, uint16_t* xrq, int sms, cudaStream_t s) {

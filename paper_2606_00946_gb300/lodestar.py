@@ -85,6 +85,7 @@ _SIGS = {
     "ls_get_bounds": (C.c_int, [_P, _i32, _P, _P, _P]),
     "ls_route_batch_guarded": (C.c_int, [_P, _i32, _P, _P, _P, _P, _P, _P, _P, _P, _P,
                                          C.POINTER(C.c_uint64), _P]),
+    "ls_read_features": (C.c_int, [_P, _i64, _i64, _P, _P]),
     "ls_route_sequential": (C.c_int, [_P, _i32, _P, _P, _P, _i32, _P, _P, _P, _P, C.POINTER(C.c_uint64), _P]),
     "ls_trace_enable": (C.c_int, [_P, _i32]),
     "ls_trace_read": (C.c_int, [_P, C.POINTER(ls_trace_entry), _i32, C.POINTER(_i32)]),
@@ -306,6 +307,10 @@ def ls_route_batch_guarded(ctx, n_req, tok, tok_off, req_feats, choice, best, st
                                       ptr(best), ptr(status), ptr(fallback_opt), ptr(scores_opt), ptr(hits_opt),
                                       C.byref(v), stream_handle(stream))
     return rc, v.value
+
+
+def ls_read_features(ctx, row0, n_rows, out, stream=None) -> int:
+    return lib().ls_read_features(ctx, int(row0), int(n_rows), ptr(out), stream_handle(stream))
 
 
 def ls_route_sequential(ctx, n_req, tok, tok_off, req_feats, queue_col, choice, best, scores_opt=None,

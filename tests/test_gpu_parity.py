@@ -179,6 +179,44 @@ def test_features_parity(name):
     assert ulp.max() <= 1
 
 
+def _bf16_ordered(bits):
+    # bf16 bit patterns to integers that order as the values do (sign-magnitude -> two's complement)
+    b = bits.astype(np.int64) & 0xFFFF
+    return np.where(b & 0x8000, -(b & 0x7FFF), b)
+
+
+@pytest.mark.parametrize("case", ["homogeneous", "heterogeneous", "wide"])
+def test_production_feature_rows(case):
+    # the bf16 rows the tensor-core scorer read (feature image of the pipelined
+    # scorer; pair chunks + template rows of the others), every row of the
+    # batch, against the oracle's features rounded to bf16: at most one bf16
+    # ulp apart (the fp32 z-score may differ by one fp32 ulp under FMA
+    # contraction, which can move a bf16 rounding), almost all bit-exact
+    import dataclasses
+    own = case == "wide"
+    if own:
+        cfg = dataclasses.replace(W.CONFIGS["large"], n_req=48, cache_blocks=1024, n_samples=0)
+        wl = W.generate(cfg)
+        r = H.Router.for_config(cfg)
+        dw = H.DeviceWorkload(wl)
+        dw.load(r)
+    else:
+        wl, dw, r = staged(case)
+    cfg = wl.cfg
+    out = r.route(dw.tok, dw.tok_off, dw.req_feats, cfg.n_inst)
+    rows = cfg.n_req * cfg.n_inst
+    g = torch.empty(rows, cfg.d, dtype=torch.int16, device="cuda")
+    L.check(L.ls_read_features(r.h, 0, rows, g))
+    want = oracle.features(np.diff(wl.tok_off), out["hits"].cpu().numpy(), wl.inst_state, wl.req_feats,
+                           wl.mean, wl.std)
+    wb = torch.from_numpy(want).to(torch.bfloat16).view(torch.int16).numpy()
+    diff = np.abs(_bf16_ordered(g.cpu().numpy()) - _bf16_ordered(wb))
+    assert diff.max() <= 1, diff.max()
+    assert (diff == 0).mean() > 0.999
+    if own:
+        r.close()
+
+
 def test_route_parity_tiny_fp32():
     wl, dw, r = staged("tiny")
     out = r.route(dw.tok, dw.tok_off, dw.req_feats, wl.cfg.n_inst)

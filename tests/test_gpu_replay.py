@@ -50,7 +50,8 @@ class Pools:
     def fifo(self):
         n = len(self.y)
         nF = min(n, self.C)
-        pos = [max(p for p in range(max(0, n - self.C), n) if p % self.C == s) for s in range(nF)]
+        # slot s holds the newest stream position p < n with p % C == s
+        pos = [(n - 1) - ((n - 1 - s) % self.C) for s in range(nF)]
         return self.x[pos], self.y[pos]
 
 
@@ -108,6 +109,7 @@ def _round(cfg, wl, r, pools, rng, n_new, mode):
 
 @pytest.mark.parametrize("name,C,P,Rc,batch,mode,over", [
     ("homogeneous", 256, 256, 128, 256, "bf16", {}),                        # tensor-core distances
+    ("homogeneous", 5000, 5000, 5000, 4096, "bf16", {}),                    # the paper's pool sizes
     ("tiny", 64, 48, 24, 64, "f32", {}),                                    # CUDA-core distances
 ])
 def test_replay_rounds_parity(name, C, P, Rc, batch, mode, over):
