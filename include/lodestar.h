@@ -435,12 +435,12 @@ int ls_trace_enable(ls_ctx *ctx, int32_t on);
 int ls_trace_read(ls_ctx *ctx, ls_trace_entry *out, int32_t max_entries, int32_t *n_out);
 
 /* Prefix hit lengths without any device allocation (no counterpart in the
- * paper: the paper's router calls into a Python service and never states how
- * scratch memory is obtained).  Computes the same h[r, i] as the prefix
- * stage of ls_route_batch (Sec. 2: the first miss ends reuse; Sec. 4.1
- * Features (2)), using the two-phase kernels (hash + block-0 screen, then a
- * walk of the pairs that hit block 0), but needs no context and takes its
- * scratch from one statically sized device array compiled into the library.
+ * paper).  Computes the same h[r, i] as the prefix stage of ls_route_batch --
+ * the number of leading full blocks of prompt r whose keys are all in
+ * instance i's table -- using the two-phase kernels (hash + block-0 screen,
+ * then a walk of the pairs that hit block 0), but needs no context and takes
+ * its scratch from one statically sized device array compiled into the
+ * library.
  *
  * Who needs it: callers that must not allocate device memory while routing --
  * a routing thread that is latency-critical (cudaMalloc/cudaFree can
@@ -453,10 +453,11 @@ int ls_trace_read(ls_ctx *ctx, ls_trace_entry *out, int32_t max_entries, int32_t
  *   tok         DEVICE int32 tokens of the batch (CSR values)
  *   tok_off     DEVICE int64 [n_req + 1] CSR offsets (non-decreasing)
  *   n_tokens    HOST copy of tok_off[n_req] - tok_off[0]; the call checks the
- *               batch's block count against LS_STATIC_MAX_BLOCKS with it.  If
- *               it understates the span, blocks past the static capacity
- *               count as misses (hits come out short, nothing is written out
- *               of bounds).
+ *               batch's block count against LS_STATIC_MAX_BLOCKS with it, and
+ *               that check is only as good as this value: if it understates
+ *               the span, blocks past the static capacity count as misses
+ *               (hits come out short, nothing is written out of bounds) and
+ *               no status reports it.
  *   tables      DEVICE uint64 [n_inst * slots_per_instance]: per-instance
  *               open-addressing tables of block keys (key 0 = empty slot,
  *               linear probing from key & (slots - 1)), 16-byte aligned
@@ -473,8 +474,10 @@ int ls_trace_read(ls_ctx *ctx, ls_trace_entry *out, int32_t max_entries, int32_t
  * different host threads) race and may return wrong hit lengths: serialise
  * them on one stream or with events.
  * The first call on a device (with that device current) looks up the
- * scratch address with cudaGetSymbolAddress; make that first call outside
- * any stream capture.  Returns LS_ERR_ARG for bad arguments or a batch
+ * scratch address with cudaGetSymbolAddress and keeps it for the life of the
+ * process; make that first call outside any stream capture.  After a
+ * cudaDeviceReset (or any teardown of the device's primary context) the kept
+ * address is stale and calls on that device are undefined.  Returns LS_ERR_ARG for bad arguments or a batch
  * beyond the static limits (with a message in ls_last_error), LS_ERR_CUDA if
  * the lookup or a launch fails, else LS_OK once the work is enqueued. */
 #define LS_STATIC_MAX_BLOCKS 262144 /* full 16-token blocks per batch */
