@@ -75,6 +75,9 @@ def parse():
                    help="only the guarded-route measurement (--steps routes; for kernel profiling)")
     p.add_argument("--route-only", default=None, choices=["tiny", "homogeneous", "heterogeneous", "large"],
                    help="only --steps routes of one configuration (for kernel profiling)")
+    p.add_argument("--small", action="store_true",
+                   help="with --route-only: the configuration's shapes at 2048 requests and 4096 cached blocks per "
+                        "instance (a few hundred MB on the device, for ncu captures)")
     p.add_argument("--cpu-seconds", type=float, default=12.0, help="target oracle work for cpu_baseline")
     return p.parse_args()
 
@@ -747,9 +750,11 @@ def kernel_rooflines(trace, n_calls, costs, cfg, R, N, Bt, peaks, peak_src, work
     return out
 
 
-def setup_config(name, H, W, dev, ring=65536, **caps):
+def setup_config(name, H, W, dev, ring=65536, small=False, **caps):
+    import dataclasses
     import torch
-    wl = W.generate(name)
+    wl = W.generate(dataclasses.replace(W.CONFIGS[name], n_req=2048, cache_blocks=4096, n_samples=0)
+                    if small else name)
     cfg = wl.cfg
     r = H.Router.for_config(cfg, ring_capacity=max(ring, 4 * cfg.train_batch), **caps)
     dw = H.DeviceWorkload(wl, device=dev)
@@ -779,13 +784,13 @@ def batch_costs(r, wl, cfg, dw):
     return route_costs(cfg, cfg.n_req, cfg.n_inst, hits, np.diff(wl.tok_off), keys.cpu().numpy(), ko.cpu().numpy())
 
 
-def measure_route(name, L, H, W, dev, stream, peaks, peak_src, steps, warmup, ctx=None):
+def measure_route(name, L, H, W, dev, stream, peaks, peak_src, steps, warmup, ctx=None, small=False):
     """Route calls of one configuration alone (graph replays back to back):
     decisions/s, scores/s, per-kernel rooflines and the route-level roofline."""
     import torch
     own = ctx is None
     if own:
-        ctx = setup_config(name, H, W, dev)
+        ctx = setup_config(name, H, W, dev, small=small)
     wl, cfg, r, dw = ctx[:4]
     R, N = cfg.n_req, cfg.n_inst
     sets, set_bytes = input_sets(dw, INPUT_SETS_SMALL)
@@ -812,7 +817,8 @@ def measure_route(name, L, H, W, dev, stream, peaks, peak_src, steps, warmup, ct
     per_call = {k: v[1] / max(v[2], 1) * v[0] / n_tr for k, v in trace.items()}
     roof = route_roofline(costs, R, N, peaks)
     dom = max(rl, key=lambda k: per_call.get(k, 0.0)) if rl else None
-    res = {"workload": DESC[name], "ms_per_route": ms, "decisions_per_s": R / (ms / 1e3),
+    res = {"workload": DESC[name] + (" (reduced: 2048 requests, 4096 cached blocks per instance)" if small else ""),
+           "ms_per_route": ms, "decisions_per_s": R / (ms / 1e3),
            "scores_per_s": R * N / (ms / 1e3), "route_roofline": roof,
            "frac_of_route_roofline": (R / (ms / 1e3)) / roof["decisions_per_s"],
            "dominant_kernel": dom, "roofline": rl.get(dom) if dom else None, "kernel_rooflines": rl,
@@ -1084,7 +1090,8 @@ def main():
     flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
 
     if args.route_only:
-        res = measure_route(args.route_only, L, H, W, dev, stream, peaks, peak_src, args.steps, args.warmup)
+        res = measure_route(args.route_only, L, H, W, dev, stream, peaks, peak_src, args.steps, args.warmup,
+                            small=args.small)
         if rank == 0:
             print(json.dumps({"route_only": args.route_only, **res}))
         return 0
