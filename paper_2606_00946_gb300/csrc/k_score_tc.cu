@@ -780,69 +780,63 @@ __global__ void __launch_bounds__(kThreadsWide, 1) k_score_wide(const __grid_con
 
   if (warp == 0) {
     // ------------------------------------------------------------ MMA issuer
+    // The tensor core's instruction queue is short: products must follow one
+    // another with little scalar work between them, so this loop keeps plain
+    // counters (stage, slice within the stage, slot), a parity bit per stage
+    // and descriptors formed by addition (a shared-memory descriptor's address
+    // field is the byte address / 16).
     if (lane == 0 && my_tiles > 0) {
       bool ok = true;
-      int64_t g = 0, jg = 0;  // weight slices and jobs consumed so far
-      auto job_start = [&](int64_t j, uint32_t& d) {  // wait for the slot's previous epilogue
-        const int slot = (int)(j & 1);
-        const int64_t use = j >> 1;
-        if (use >= 1 && !mbar_wait(&s_empty[slot], (uint32_t)((use - 1) & 1))) return false;
-        tc_fence_after();
-        d = tmem + kSlot0 + 128u * (uint32_t)slot;
-        return true;
-      };
-      auto next_slice = [&](uint32_t& b) {  // slice g: part g % Q of stage g / Q
-        const int64_t G = g / Q;
-        const int s = (int)(G % S);
-        if (g % Q == 0) {
-          if (!mbar_wait(&full[s], (uint32_t)((G / S) & 1))) return false;
-          tc_fence_after();
-        }
-        b = smem_u32(ring + ((size_t)s * Q + (size_t)(g % Q)) * kWideChunk);
-        return true;
-      };
-      auto slice_done = [&]() {  // the stage is free once the products of its last slice complete
-        if (g % Q == Q - 1) umma_commit(&empty[(g / Q) % S]);
-      };
+      int st = 0, part = 0;      // ring stage and slice within it
+      uint32_t fpar = 0;         // bit s: parity of the next wait on full[s]
+      uint32_t jslot = 0;        // jobs issued so far (slot = jslot & 1)
+      const uint64_t ring_desc = sdesc_sw128(smem_u32(ring));
+      const uint64_t one_desc = sdesc_nosw(smem_u32(ONE), 128, 0);
+      const uint64_t bias_desc = sdesc_nosw(smem_u32(BIAS), 128, 256);
+      const uint64_t x_desc = sdesc_sw128(smem_u32(X));
       for (int t = 0; t < my_tiles && ok; ++t) {
         ok = mbar_wait(x_full, (uint32_t)(t & 1));
         if (!ok) break;
         tc_fence_after();
-        for (int c = 0; c < J1 && ok; ++c, ++jg) {
-          uint32_t d;
-          if (!(ok = job_start(jg, d))) break;
-          umma_bf16(d, sdesc_nosw(smem_u32(ONE), 128, 0),
-                    sdesc_nosw(smem_u32(BIAS + (size_t)c * 128 * 32), 128, 256), idesc, 0u);
-          for (int kb = 0; kb < nk0 && ok; ++kb, ++g) {
-            uint32_t bb;
-            if (!(ok = next_slice(bb))) break;
-            const uint32_t xa = smem_u32(X + (size_t)kb * kWideChunk);
-#pragma unroll
-            for (int j = 0; j < 4; ++j)
-              umma_bf16(d, sdesc_sw128(xa + 32u * j), sdesc_sw128(bb + 32u * j), idesc, 1u);
-            slice_done();
+        for (int j = 0; j < J1 + J2 && ok; ++j, ++jslot) {
+          const bool l2 = j >= J1;
+          if (j == J1) {
+            umma_commit(x_empty);  // the feature tile is free once the layer-1 products are done
+            ok = mbar_wait(h1_ready, (uint32_t)(t & 1));  // every layer-1 slice packed into TMEM
+            if (!ok) break;
+            tc_fence_after();
           }
-          if (ok) umma_commit(&s_full[jg & 1]);
-        }
-        if (!ok) break;
-        umma_commit(x_empty);  // the feature tile is free once the layer-1 products are done
-        ok = mbar_wait(h1_ready, (uint32_t)(t & 1));  // every layer-1 slice packed into TMEM
-        if (!ok) break;
-        tc_fence_after();
-        for (int n = 0; n < J2 && ok; ++n, ++jg) {
-          uint32_t d;
-          if (!(ok = job_start(jg, d))) break;
-          umma_bf16(d, sdesc_nosw(smem_u32(ONE), 128, 0),
-                    sdesc_nosw(smem_u32(BIAS + (size_t)(H1 + n * 128) * 32), 128, 256), idesc, 0u);
-          for (int kb = 0; kb < nk1 && ok; ++kb, ++g) {
-            uint32_t bb;
-            if (!(ok = next_slice(bb))) break;
+          // the slot's previous epilogue has drained it
+          const uint32_t slot = jslot & 1u;
+          if (jslot >= 2 && !(ok = mbar_wait(&s_empty[slot], ((jslot >> 1) - 1) & 1u))) break;
+          tc_fence_after();
+          const uint32_t d = tmem + kSlot0 + 128u * slot;
+          const int bias_row = l2 ? H1 + (j - J1) * 128 : j * 128;
+          umma_bf16(d, one_desc, bias_desc + (uint64_t)(bias_row * 32 / 16), idesc, 0u);
+          const int nk = l2 ? nk1 : nk0;
+          for (int kb = 0; kb < nk; ++kb) {
+            if (part == 0) {  // a new stage: wait for its copy
+              if (!(ok = mbar_wait(&full[st], (fpar >> st) & 1u))) break;
+              fpar ^= 1u << st;
+              tc_fence_after();
+            }
+            const uint64_t bd = ring_desc + (uint64_t)((st * Q + part) * (kWideChunk / 16));
+            if (l2) {
+              const uint32_t a0 = tmem + (uint32_t)(32 * kb);
 #pragma unroll
-            for (int j = 0; j < 4; ++j)
-              umma_bf16_ts(d, tmem + (uint32_t)(32 * kb + 8 * j), sdesc_sw128(bb + 32u * j), idesc, 1u);
-            slice_done();
+              for (int k = 0; k < 4; ++k) umma_bf16_ts(d, a0 + 8u * k, bd + 2u * k, idesc, 1u);
+            } else {
+              const uint64_t xd = x_desc + (uint64_t)(kb * (kWideChunk / 16));
+#pragma unroll
+              for (int k = 0; k < 4; ++k) umma_bf16(d, xd + 2u * k, bd + 2u * k, idesc, 1u);
+            }
+            if (++part == Q) {  // the stage is free once these products complete
+              umma_commit(&empty[st]);
+              part = 0;
+              st = st + 1 == S ? 0 : st + 1;
+            }
           }
-          if (ok) umma_commit(&s_full[jg & 1]);
+          if (ok) umma_commit(&s_full[slot]);
         }
         if (ok) umma_commit(h1_free);  // the packed activations may be overwritten
       }
