@@ -136,7 +136,25 @@ typedef struct {
     int32_t scorer;              /* LS_SCORER_CUDA_CORES or LS_SCORER_TENSOR_CORES in use */
     int64_t replay_count;        /* records in the replay pool */
     int64_t pending_count;       /* evicted records waiting for ls_replay_admit */
+    int32_t tc_kernel;           /* tensor-core scorer variant routes run (ls_tc_kernel) */
 } ls_info;
+
+/* Tensor-core scorer variants (all compute the same forward; which one runs is
+ * fixed by the predictor widths when the context is created):
+ *   GENERIC    any bf16 predictor with hidden widths multiples of 64, <= 512;
+ *   PIPELINED  two hidden layers <= 256 wide, weights resident in shared memory;
+ *   PAIR       otherwise two hidden layers of multiples of 128 and a feature
+ *              width <= 128: CTA pairs running 2-SM products, weights streamed;
+ *   WIDE       the same shapes on one CTA per tile, where CTA pairs cannot be
+ *              resident together, or when the environment variable LS_TC_PAIR
+ *              is "0" at context creation. */
+typedef enum {
+    LS_TC_NONE = 0,
+    LS_TC_GENERIC = 1,
+    LS_TC_PIPELINED = 2,
+    LS_TC_WIDE = 3,
+    LS_TC_PAIR = 4
+} ls_tc_kernel;
 
 /* Number of predictor parameters: sum over layers of out*in + out. */
 int64_t ls_param_count(const ls_config *cfg);

@@ -2,6 +2,7 @@
 // device memory, stream ordering of publish / route, and error reporting.
 #include <algorithm>
 #include <cmath>
+#include <cstdlib>
 #include <cstring>
 #include <string>
 #include <vector>
@@ -165,13 +166,24 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
   c.d = m.w[0];
   c.n_params = off;
   {
-    const bool can_tc = plan_tc(m, c.tc);
+    // LS_TC_PAIR=0 in the environment plans without the pair kernel (the
+    // one-CTA wide kernel takes its shapes), so that both stay exercised
+    const char* pair_env = std::getenv("LS_TC_PAIR");
+    const bool allow_pair = !(pair_env && pair_env[0] == '0');
+    const bool can_tc = plan_tc(m, c.tc, allow_pair);
     if (cfg->scorer == LS_SCORER_TENSOR_CORES && !can_tc) {
       delete h;
       return fail(LS_ERR_ARG, "tensor-core scorer needs a bf16 predictor with hidden widths that are "
                               "multiples of 64 and at most 512");
     }
     c.use_tc = can_tc && cfg->scorer != LS_SCORER_CUDA_CORES;
+    if (c.use_tc && c.tc.pair) {  // the pair kernel needs CTA pairs that fit together on the device
+      const int k = pair_max_clusters(c.tc);
+      if (k < 1)
+        plan_tc(m, c.tc, false);
+      else
+        c.tc.pair_clusters = k;
+    }
   }
   c.wt_total = wt;
   {
@@ -356,6 +368,11 @@ int ls_get_info(ls_ctx* h, ls_info* out) {
   out->train_steps = ds.step;
   out->weight_version = ds.version;
   out->scorer = c.use_tc ? LS_SCORER_TENSOR_CORES : LS_SCORER_CUDA_CORES;
+  out->tc_kernel = !c.use_tc ? LS_TC_NONE
+                   : c.tc.pipe ? LS_TC_PIPELINED
+                   : c.tc.pair ? LS_TC_PAIR
+                   : c.tc.wide ? LS_TC_WIDE
+                               : LS_TC_GENERIC;
   out->replay_count = ds.replay_count;
   out->pending_count = 0;
   if (c.cfg.replay_capacity > 0) {  // evicted positions [lo, hi) not yet considered

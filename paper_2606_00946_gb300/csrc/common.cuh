@@ -58,6 +58,12 @@ struct TcPlan {
   int wide_smem = 0;
   int wide_stages = 0;
   int wide_q = 1;                  // weight slices per stage of the wide kernel
+  int pair = 0;                    // pair kernel applies (two hidden layers of multiples of 256, 2-SM products)
+  int pair_smem = 0;
+  int pair_stages = 0;
+  int pair_q = 1;                  // 16 KB half-slices per stage of the pair kernel
+  int pair_slices = 0;             // half-slices per CTA per tile (the per-rank stream of the image)
+  int pair_clusters = 0;           // co-resident CTA pairs (0: not queried)
 };
 
 // One published weight version (Sec. 4.3.1 P2: the routing side reads a
@@ -436,7 +442,11 @@ cudaError_t launch_guards(const ls_guards& g, int n_req, int n_inst, const int32
                           cudaStream_t s);
 constexpr int kGuardHeurMaxInst = 1024;  // instances the heuristic keeps in shared memory
 
-bool plan_tc(const MlpDesc& m, TcPlan& p);
+// Plan the tensor-core scorer; `allow_pair` false leaves the pair kernel out
+// (and its image layout).
+bool plan_tc(const MlpDesc& m, TcPlan& p, bool allow_pair = true);
+// CTA pairs of the pair kernel that can be resident at once (0: none).
+int pair_max_clusters(const TcPlan& p);
 // Publish the master weights into buffer 1 - st->cur (fp32 params, the
 // transposed copy when `want_wt`, the tensor-core image when `tc`, the staged
 // feature bounds), then flip st->cur and bump the version; one launch.

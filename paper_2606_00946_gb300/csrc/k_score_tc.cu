@@ -82,7 +82,11 @@ __device__ __forceinline__ void st_shared_v4(uint8_t* p, uint32_t a, uint32_t b,
 // normalised values at their feature positions and zeros elsewhere, and the
 // pair features of each row come as one 16-byte chunk with zeros past column
 // 5 (k_norm_rows), so a 16-byte chunk of a feature row is the OR of at most
-// three loaded chunks.  `nthr` threads (index `tr`) share the tile.
+// three loaded chunks.  `nthr` threads (index `tr`) share the tile; each
+// issues the loads of its U chunks before combining any of them, so that 3 U
+// loads are in flight per thread (the loads are ordered asm, and a combine
+// between them would wait for each group in turn).  Rows past the batch are
+// zeros.
 template <int U>
 __device__ __forceinline__ void build_tile(const TcArgs& a, uint8_t* X, int64_t row0, int tr, int nthr) {
   const int cpr = a.p.d_pad / 8;  // 16-byte chunks per row
@@ -91,11 +95,11 @@ __device__ __forceinline__ void build_tile(const TcArgs& a, uint8_t* X, int64_t 
   const int64_t r0 = row0 / a.n_inst;
   const int i0 = (int)(row0 - r0 * a.n_inst);
   for (int base = 0; base < total; base += U * nthr) {
-    uint4 v[U];
+    uint4 ti[U], tq[U], tp[U];
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       const int e = base + u * nthr + tr;
-      v[u] = make_uint4(0u, 0u, 0u, 0u);
+      ti[u] = tq[u] = tp[u] = make_uint4(0u, 0u, 0u, 0u);
       if (e >= total) continue;
       const int m = csh >= 0 ? e >> csh : e / cpr, c = e - m * cpr;
       const int64_t g = row0 + m;
@@ -108,17 +112,17 @@ __device__ __forceinline__ void build_tile(const TcArgs& a, uint8_t* X, int64_t 
         r += i / a.n_inst;
         i -= (i / a.n_inst) * a.n_inst;
       }
-      const uint4 ti = ldg_stream(reinterpret_cast<const uint4*>(a.xin + (int64_t)i * a.p.d_pad) + c);
-      const uint4 tq = ldg_stream(reinterpret_cast<const uint4*>(a.xrq + r * a.p.d_pad) + c);
-      const uint4 tp = c == 0 ? ldg_stream(a.pairx + g) : make_uint4(0u, 0u, 0u, 0u);
-      v[u] = make_uint4(ti.x | tq.x | tp.x, ti.y | tq.y | tp.y, ti.z | tq.z | tp.z, ti.w | tq.w | tp.w);
+      ti[u] = ldg_stream(reinterpret_cast<const uint4*>(a.xin + (int64_t)i * a.p.d_pad) + c);
+      tq[u] = ldg_stream(reinterpret_cast<const uint4*>(a.xrq + r * a.p.d_pad) + c);
+      if (c == 0) tp[u] = ldg_stream(a.pairx + g);
     }
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       const int e = base + u * nthr + tr;
       if (e >= total) continue;
       const int m = csh >= 0 ? e >> csh : e / cpr, c = e - m * cpr;
-      st_shared_v4(X + sw128_offset(m, c * 8, kTileM), v[u].x, v[u].y, v[u].z, v[u].w);
+      st_shared_v4(X + sw128_offset(m, c * 8, kTileM), ti[u].x | tq[u].x | tp[u].x, ti[u].y | tq[u].y | tp[u].y,
+                   ti[u].z | tq[u].z | tp[u].z, ti[u].w | tq[u].w | tp[u].w);
     }
   }
 }
@@ -335,6 +339,48 @@ __device__ __forceinline__ uint64_t out_dot16(const uint32_t (&v)[16], uint4 w0,
   for (int j = 0; j < 8; ++j) {
     const uint32_t h = relu_bf16x2(cvt_bf16x2(((uint64_t)v[2 * j + 1] << 32) | v[2 * j]));
     acc = fma_f32x2(bf16x2_to_f32x2(h), bf16x2_to_f32x2(wp[j]), acc);
+  }
+  return acc;
+}
+
+// Shared-memory loads as ordered asm: they stay below the tensor-memory
+// loads and waits that precede them in the source, so the compiler does not
+// hoist a whole epilogue's weights and biases into registers at once.
+__device__ __forceinline__ float4 lds_f4(const float* p) {
+  float4 v;
+  asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(smem_u32(p)));
+  return v;
+}
+__device__ __forceinline__ float2 lds_f2(const float* p) {
+  float2 v;
+  asm volatile("ld.shared.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(smem_u32(p)));
+  return v;
+}
+__device__ __forceinline__ uint4 lds_u4(const void* p) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "r"(smem_u32(p)));
+  return v;
+}
+
+// The same with the layer's bias added first: acc += relu(bf16(v + b)) * w
+// over 16 columns, b the 16 fp32 biases and w the 16 bf16 weights of these
+// columns (both in shared memory).
+__device__ __forceinline__ uint64_t out_dot16_bias(const uint32_t (&v)[16], const float* b, const uint4* w,
+                                                   uint64_t acc) {
+  const uint4 w0 = lds_u4(w), w1 = lds_u4(w + 1);
+  const uint32_t wp[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const float4 bb = lds_f4(b + 4 * q);
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      const int j = 2 * q + u;
+      const uint64_t x = add_f32x2(((uint64_t)v[2 * j + 1] << 32) | v[2 * j], u ? f2pack(bb.z, bb.w) : f2pack(bb.x, bb.y));
+      const uint32_t h = relu_bf16x2(cvt_bf16x2(x));
+      acc = fma_f32x2(bf16x2_to_f32x2(h), bf16x2_to_f32x2(wp[j]), acc);
+    }
   }
   return acc;
 }
@@ -981,6 +1027,428 @@ __global__ void __launch_bounds__(kThreadsWide, 1) k_score_wide(const __grid_con
   if (warp == 0) tmem_dealloc(tmem, 512);
 }
 
+// 16 loaded accumulator columns -> 8 packed bf16 words relu(bf16(D + b)) at o[OFF..)
+template <int OFF>
+__device__ __forceinline__ void pack16_bias_relu(const uint32_t (&v)[16], const float* b, uint32_t (&o)[32]) {
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const float2 bb = lds_f2(b + 2 * j);
+    o[OFF + j] =
+        relu_bf16x2(cvt_bf16x2(add_f32x2(((uint64_t)v[2 * j + 1] << 32) | v[2 * j], f2pack(bb.x, bb.y))));
+  }
+}
+// 32 consecutive accumulator columns of the warp's lanes -> 16 packed words at
+// o[OFF..OFF + 16), b the 32 biases.
+template <int OFF>
+__device__ __forceinline__ void pack32_bias_relu(uint32_t taddr, const float* b, uint32_t (&o)[32]) {
+  uint32_t va[16], vb[16];
+  tmem_ld16(taddr, va);
+  tmem_ld16(taddr + 16u, vb);
+  tmem_wait_ld_regs(va);
+  pack16_bias_relu<OFF>(va, b, o);
+  tmem_wait_ld_regs(vb);
+  pack16_bias_relu<OFF + 8>(vb, b + 16, o);
+}
+// 64 columns -> 32 packed words (o[0..32)); each 16-column load overlaps the
+// packing of the one before.  Every column has been read when this returns.
+__device__ __forceinline__ void pack64_bias_relu(uint32_t taddr, const float* b, uint32_t (&o)[32]) {
+  uint32_t va[16], vb[16];
+  tmem_ld16(taddr, va);
+  tmem_wait_ld_regs(va);
+  tmem_ld16(taddr + 16u, vb);
+  pack16_bias_relu<0>(va, b, o);
+  tmem_wait_ld_regs(vb);
+  tmem_ld16(taddr + 32u, va);
+  pack16_bias_relu<8>(vb, b + 16, o);
+  tmem_wait_ld_regs(va);
+  tmem_ld16(taddr + 48u, vb);
+  pack16_bias_relu<16>(va, b + 32, o);
+  tmem_wait_ld_regs(vb);
+  pack16_bias_relu<24>(vb, b + 48, o);
+}
+
+// ---------------------------------------------------------------------------
+// Pair variant: the wide kernel's job for hidden widths that are multiples of
+// 256, on a cluster of two CTAs (one TPC) whose tensor cores run 2-SM
+// products (M = 256): CTA r builds and owns tile 2p + r of tile pair p, rows
+// 0..127 of every product are CTA 0's tile and 128..255 CTA 1's.  Jobs are
+// 256 output columns; the B operand of a job is split by rows, CTA r holding
+// rows 128 r .. 128 r + 127 (its half-slices of 16 KB, streamed from its
+// rank's part of the image).  Per SM this halves the weight bytes of the
+// one-CTA wide kernel, whose per-SM copy rate bounded it.  256-column jobs
+// keep the products long: each tcgen05 commit of a CTA pair stalls the
+// product queue for a while, so a pair kernel wants few commits per product.
+// TMEM, 512 columns in each CTA: the packed bf16 layer-1 activations H1 in
+// columns [0, H1 / 2); the accumulator D0 = columns 0..255 for layer-1 job 0,
+// compacted in place into H1 by its epilogue; D1 = columns 256..511 for
+// layer-1 job 1 and every layer-2 job, released by the epilogue as soon as it
+// has been read.  The epilogues add the biases.
+// Warp roles in each CTA: 0 = MMA issuer (CTA 0) or stage relay (CTA 1), and
+// the TMEM allocation; 1 = producer of this CTA's half-slices; 2..3 = feature
+// tile builders; 4..11 = epilogue (lane quadrant warp % 4, column half
+// (warp - 4) / 4 of a job's 256).  Barriers the issuer waits on count arrivals
+// from both CTAs and live in CTA 0 (CTA 1 arrives remotely); barriers the
+// issuer signals are committed to both CTAs.
+// ---------------------------------------------------------------------------
+constexpr int kPairBuild = 2, kPairEpi = 8;  // builder and epilogue warps of the pair kernel
+constexpr int kPairBuild0 = 2, kPairEpi0 = kPairBuild0 + kPairBuild;
+constexpr int kThreadsPair = (kPairEpi0 + kPairEpi) * 32;  // 384: up to 168 registers a thread
+constexpr int kHalfSlice = kTileM * 128;                   // [128 N x 64 K] bf16 = 16 KB
+
+// A timeout anywhere in a CTA pair stops both CTAs.
+__device__ __forceinline__ void pair_stop(volatile int* abort_flag, uint32_t rank, int* err) {
+  *abort_flag = 1;
+  st_cluster_u32((void*)abort_flag, rank ^ 1u, 1u);
+  latch_error(err, LS_ERR_TIMEOUT);
+}
+
+__global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_constant__ TcArgs a) {
+  const bool pb = a.sel && *a.sel == 1;
+  const uint8_t* __restrict__ img = pb ? a.img1 : a.img0;
+  const float* __restrict__ params = pb ? a.params1 : a.params0;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const TcPlan& p = a.p;
+  const int H1 = p.out[0], H2 = p.out[1];
+  const int J1 = H1 / 256, J2 = H2 / 256;
+  const int nk0 = p.in_pad[0] / 64, nk1 = H1 / 64;
+  const int per_tile = p.pair_slices;
+  const int S = p.pair_stages, Q = p.pair_q;
+  uint8_t* X = smem;                                                  // [nk0] feature-tile K-blocks
+  uint8_t* ring = X + (size_t)nk0 * kWideChunk;                       // [S][Q] half-slices
+  float* bias = reinterpret_cast<float*>(ring + (size_t)S * Q * kHalfSlice);  // [b1 (H1) | b2 (H2)]
+  uint16_t* sw3 = reinterpret_cast<uint16_t*>(bias + H1 + H2);        // [H2] bf16
+  float* part = reinterpret_cast<float*>(sw3 + H2);                   // [2 tiles][2 halves][128]
+  uint64_t* full = reinterpret_cast<uint64_t*>(part + 4 * kTileM);    // [S]
+  uint64_t* empty = full + S;                                         // [S]
+  uint64_t* x_full = empty + S;
+  uint64_t* x_empty = x_full + 1;
+  uint64_t* d0_full = x_empty + 1;
+  uint64_t* d1_full = d0_full + 1;
+  uint64_t* d1_empty = d1_full + 1;
+  uint64_t* h1_ready = d1_empty + 1;  // [2]: layer-1 job j's activations are in H1
+  uint64_t* done = h1_ready + 2;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(done + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+
+  const uint32_t rank = cluster_ctarank();
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int pair_id = (int)(blockIdx.x >> 1), n_pairs = (int)(gridDim.x >> 1);
+  const int tile_pairs = (a.n_tiles + 1) / 2;
+  const int my_pairs = pair_id < tile_pairs ? (tile_pairs - 1 - pair_id) / n_pairs + 1 : 0;
+  if (tid == 0) {
+    for (int q = 0; q < S; ++q) {
+      mbar_init(&full[q], rank == 0 ? 2 : 1);  // CTA 0: its own copy + the relayed arrival of CTA 1's
+      mbar_init(&empty[q], 1);
+    }
+    mbar_init(x_full, 2 * kPairBuild);
+    mbar_init(x_empty, 1);
+    mbar_init(d0_full, 1);
+    mbar_init(d1_full, 1);
+    mbar_init(d1_empty, 2 * kPairEpi);
+    mbar_init(&h1_ready[0], 2 * kPairEpi);
+    mbar_init(&h1_ready[1], 2 * kPairEpi);
+    mbar_init(done, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0) {
+    tmem_alloc_pair(tmem_holder, 512);
+    tmem_relinquish_pair();
+  }
+  for (int k = tid; k < H1 + H2; k += blockDim.x)
+    bias[k] = __ldg(params + (k < H1 ? a.boff[0] + k : a.boff[1] + k - H1));
+  for (int k = tid; k < H2; k += blockDim.x) sw3[k] = bf16_bits(__ldg(params + a.w_last_off + k));
+  tc_fence_before();
+  cluster_sync();  // barriers of both CTAs initialised before any remote arrival
+  tc_fence_after();
+  const uint32_t tmem = *tmem_holder;
+  const uint32_t idesc = idesc_bf16_f32(2 * kTileM, 256);
+  // registers: warpgroup 0 (issuer, producer, builders) needs few, the two
+  // epilogue warpgroups read a whole accumulator half per thread at once;
+  // 128 x 88 + 256 x 208 = the 384 x 168 the CTA is launched with.  Each
+  // warpgroup changes its budget at the head of its own branch.
+  if (warp < kPairEpi0) {
+    setmaxnreg_dec<88>();
+  if (warp == 0) {
+    if (rank == 0 && lane == 0) {
+      // ---------------------------------------------------------- MMA issuer
+      // As in the wide kernel: plain counters, a parity bit per stage and
+      // descriptors formed by addition keep the products back to back.
+      bool ok = true;
+      int st = 0, part_i = 0;  // ring stage and half-slice within it
+      uint32_t fpar = 0;       // bit s: parity of the next wait on full[s]
+      uint32_t u1 = 0;         // D1 uses issued so far
+      const uint64_t ring_desc = sdesc_sw128(smem_u32(ring));
+      const uint64_t x_desc = sdesc_sw128(smem_u32(X));
+      for (int t = 0; t < my_pairs && ok; ++t) {
+        if (!(ok = mbar_wait_cl(x_full, (uint32_t)(t & 1)))) break;
+        tc_fence_after();
+        for (int j = 0; j < J1 + J2 && ok; ++j) {
+          const bool l2 = j >= J1;
+          if (j == J1) umma_pair_commit_both(x_empty);  // both feature tiles free once the layer-1 products are done
+          uint32_t d = tmem;  // D0: layer-1 job 0
+          if (j > 0) {        // D1: its previous use has been read by both epilogues
+            if (u1 >= 1 && !(ok = mbar_wait_cl(d1_empty, (u1 - 1) & 1u))) break;
+            tc_fence_after();
+            d = tmem + 256u;
+          }
+          const int nk = l2 ? nk1 : nk0;
+          for (int kb = 0; kb < nk; ++kb) {
+            if (j == J1 && (kb & 3) == 0) {  // K-blocks 4 i.. read layer-1 job i's activations
+              if (!(ok = mbar_wait_cl(&h1_ready[kb >> 2], (uint32_t)(t & 1)))) break;
+              tc_fence_after();
+            }
+            if (part_i == 0) {  // a new stage: both CTAs' copies have landed
+              if (!(ok = mbar_wait_cl(&full[st], (fpar >> st) & 1u))) break;
+              fpar ^= 1u << st;
+              tc_fence_after();
+            }
+            const uint64_t bd = ring_desc + (uint64_t)((st * Q + part_i) * (kHalfSlice / 16));
+            if (l2) {
+              const uint32_t a0 = tmem + (uint32_t)(32 * kb);
+#pragma unroll
+              for (int k = 0; k < 4; ++k) umma_pair_bf16_ts(d, a0 + 8u * k, bd + 2u * k, idesc, (kb | k) ? 1u : 0u);
+            } else {
+              const uint64_t xd = x_desc + (uint64_t)(kb * (kWideChunk / 16));
+#pragma unroll
+              for (int k = 0; k < 4; ++k) umma_pair_bf16(d, xd + 2u * k, bd + 2u * k, idesc, (kb | k) ? 1u : 0u);
+            }
+            if (++part_i == Q) {  // the stage is free in both CTAs once these products complete
+              umma_pair_commit_both(&empty[st]);
+              part_i = 0;
+              st = st + 1 == S ? 0 : st + 1;
+            }
+          }
+          if (!ok) break;
+          if (j == 0) {
+            umma_pair_commit_both(d0_full);
+          } else {
+            umma_pair_commit_both(d1_full);
+            ++u1;
+          }
+        }
+      }
+      if (!ok) pair_stop(abort_flag, rank, a.err);
+      umma_pair_commit_both(done);  // every product issued has completed before TMEM is freed
+      mbar_wait(done, 0);
+    } else if (rank == 1 && lane == 0) {
+      // ---------------------------------------------------------- stage relay
+      // this CTA's half of stage G has landed -> one arrival on CTA 0's full[s]
+      const int64_t stages = (int64_t)my_pairs * per_tile / Q;
+      for (int64_t G = 0; G < stages; ++G) {
+        const int s = (int)(G % S);
+        if (!mbar_wait(&full[s], (uint32_t)((G / S) & 1))) {
+          pair_stop(abort_flag, rank, a.err);
+          break;
+        }
+        if (*abort_flag) break;
+        mbar_arrive_at(&full[s], 0);
+      }
+      mbar_wait(done, 0);  // the last commit has reached this CTA too
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0 && my_pairs > 0) {
+      const int64_t stages = (int64_t)my_pairs * per_tile / Q;
+      const uint32_t bytes = (uint32_t)(Q * kHalfSlice);
+      const uint8_t* src = img + (int64_t)rank * per_tile * kHalfSlice;
+      int64_t G = 0;
+      bool ok = true;
+      for (; G < stages; ++G) {
+        const int s = (int)(G % S);
+        const int64_t u = G / S;
+        if (u >= 1 && !(ok = mbar_wait_cl(&empty[s], (uint32_t)((u - 1) & 1)))) break;
+        if (*abort_flag) {
+          ok = false;
+          break;
+        }
+        const int q0 = (int)((G * Q) % per_tile);
+        mbar_arrive_expect_tx(&full[s], bytes);
+        bulk_g2s(ring + (size_t)s * Q * kHalfSlice, src + (int64_t)q0 * kHalfSlice, bytes, &full[s]);
+      }
+      if (!ok && !*abort_flag) pair_stop(abort_flag, rank, a.err);
+      // stages issued and never consumed (only after an abort) land in this
+      // CTA's shared memory: wait for them (bounded) before it can exit
+      if (*abort_flag)
+        for (int64_t h = G - 1; h >= 0 && h >= G - S; --h) mbar_wait(&full[h % S], (uint32_t)((h / S) & 1));
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------ feature-tile builders
+    const int bt = tid - kPairBuild0 * 32;
+    pdl_wait();  // pair chunks and template rows from the previous kernel of the stream
+    for (int t = 0; t < my_pairs; ++t) {
+      if (t >= 1 && !mbar_wait_cl(x_empty, (uint32_t)((t - 1) & 1))) {
+        pair_stop(abort_flag, rank, a.err);
+        break;
+      }
+      if (*abort_flag) break;
+      const int64_t tile = 2 * ((int64_t)pair_id + (int64_t)t * n_pairs) + rank;
+      build_tile<4>(a, X, tile * kTileM, bt, kPairBuild * 32);  // rows past the batch: zeros
+      fence_async_smem();  // the tile is read by the tensor cores (async proxy)
+      __syncwarp();
+      if (lane == 0) mbar_arrive_at(x_full, 0);
+    }
+  }
+  } else {
+    setmaxnreg_inc<208>();
+    // ------------------------------------------------------------ epilogue
+    const int ew = warp - kPairEpi0;  // 0..7
+    const int q4 = warp & 3;          // TMEM lane quadrant
+    const int h = ew >> 2;            // which 128 of a job's 256 columns
+    const int row = 32 * q4 + lane;
+    const uint32_t lane_addr = (uint32_t)(32 * q4) << 16;
+    uint32_t u1 = 0;  // D1 uses read so far
+    bool ok = true;
+    for (int t = 0; t < my_pairs; ++t) {
+      for (int j = 0; j < J1; ++j) {
+        // layer-1 job j: relu(D + b1) -> bf16 -> H1 columns [128 j + 64 h, +64)
+        bool go = ok && !*abort_flag;
+        if (go) go = j == 0 ? mbar_wait_cl(d0_full, (uint32_t)(t & 1)) : mbar_wait_cl(d1_full, u1 & 1u);
+        go = __all_sync(0xffffffffu, go);  // the tensor-memory accesses below are warp-wide
+        if (!go && ok) {
+          ok = false;
+          // the issuer, whose waits need both CTAs' epilogues, runs out too and
+          // latches the error for the pair
+          if (lane == 0) *abort_flag = 1;
+        }
+        const float* b = bias + 256 * j + 128 * h;
+        uint32_t pa[32], pb[32];
+        if (j == 0) {
+          // D0 is H1's own columns (packed column c holds features 2c, 2c + 1).
+          // Half 1 overwrites columns 64..127, which half 0 of its quadrant
+          // reads: half 0 reads them first and signals; each half then writes
+          // a block of 32 packed columns once the columns under it are consumed.
+          const uint32_t d0 = tmem + lane_addr;
+          if (h == 0) {
+            if (go) {
+              tc_fence_after();
+              pack64_bias_relu(d0 + 64u, b + 64, pb);  // features 64..127 -> columns 32..63
+            }
+            tc_fence_before();
+            named_bar_arrive(2, kPairEpi * 32);
+            if (go) {
+              pack32_bias_relu<16>(d0 + 32u, b + 32, pa);  // features 32..63 -> columns 16..31
+              tmem_st32(d0 + 32u, pb);                     // columns 32..63 are consumed now
+              pack32_bias_relu<0>(d0, b, pa);              // features 0..31 -> columns 0..15
+              tmem_st32(d0, pa);
+              tmem_wait_st();
+            }
+          } else {
+            if (go) {
+              tc_fence_after();
+              pack64_bias_relu(d0 + 128u, b, pa);  // features 128..191 -> columns 64..95
+            }
+            named_bar_sync(2, kPairEpi * 32);
+            tc_fence_after();
+            if (go) {
+              tmem_st32(d0 + 64u, pa);
+              pack64_bias_relu(d0 + 192u, b + 64, pb);  // features 192..255 -> columns 96..127
+            }
+            if (J1 > 1) {  // columns 128..255 read: layer-1 job 1 may write there
+              tc_fence_before();
+              named_bar_arrive(3, kPairEpi * 32);
+            }
+            if (go) {
+              tmem_st32(d0 + 96u, pb);
+              tmem_wait_st();
+            }
+          }
+        } else {
+          // D1 -> H1 columns [128 j + 64 h, +64), which job 0's columns 128..255
+          // held: half 0 first waits until half 1 of its quadrant has read them
+          const uint32_t src = tmem + lane_addr + 256u + 128u * (uint32_t)h;
+          const uint32_t dst = tmem + lane_addr + (uint32_t)(128 * j + 64 * h);
+          if (h == 0) {
+            tc_fence_before();
+            named_bar_sync(3, kPairEpi * 32);
+          }
+          if (go) {
+            tc_fence_after();
+            pack64_bias_relu(src, b, pa);
+            tmem_st32(dst, pa);
+            pack64_bias_relu(src + 64u, b + 64, pb);
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive_at(d1_empty, 0);  // D1 read: the next job may overwrite it
+          ++u1;
+          if (go) {
+            tmem_st32(dst + 32u, pb);
+            tmem_wait_st();
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_at(&h1_ready[j], 0);
+      }
+      uint64_t acc = 0;  // output-layer partial, two fp32 lanes
+      for (int n = 0; n < J2; ++n) {
+        // layer-2 job n: acc += relu(bf16(D + b2)) . w3 over this warp's 128
+        // columns; D1 is released once all are read
+        bool go = ok && !*abort_flag;
+        if (go) go = mbar_wait_cl(d1_full, u1 & 1u);
+        go = __all_sync(0xffffffffu, go);
+        if (!go && ok) {
+          ok = false;
+          if (lane == 0) *abort_flag = 1;
+        }
+        const uint32_t src = tmem + lane_addr + 256u + 128u * (uint32_t)h;
+        const uint4* w = reinterpret_cast<const uint4*>(sw3 + 256 * n + 128 * h);
+        const float* b = bias + H1 + 256 * n + 128 * h;
+        uint32_t va[16], vb[16], vc[16], vd[16];  // 64 columns per wait, two waits per job
+        if (go) {
+          tc_fence_after();
+          tmem_ld16(src, va);
+          tmem_ld16(src + 16u, vb);
+          tmem_ld16(src + 32u, vc);
+          tmem_ld16(src + 48u, vd);
+          tmem_wait_ld_regs(va);
+          tmem_wait_ld_regs(vb);
+          tmem_wait_ld_regs(vc);
+          tmem_wait_ld_regs(vd);
+          acc = out_dot16_bias(va, b, w, acc);
+          acc = out_dot16_bias(vb, b + 16, w + 2, acc);
+          acc = out_dot16_bias(vc, b + 32, w + 4, acc);
+          acc = out_dot16_bias(vd, b + 48, w + 6, acc);
+          tmem_ld16(src + 64u, va);
+          tmem_ld16(src + 80u, vb);
+          tmem_ld16(src + 96u, vc);
+          tmem_ld16(src + 112u, vd);
+          tmem_wait_ld_regs(va);
+          tmem_wait_ld_regs(vb);
+          tmem_wait_ld_regs(vc);
+          tmem_wait_ld_regs(vd);
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_at(d1_empty, 0);  // all of D1 read: the next job may overwrite it
+        ++u1;
+        if (go) {
+          acc = out_dot16_bias(va, b + 64, w + 8, acc);
+          acc = out_dot16_bias(vb, b + 80, w + 10, acc);
+          acc = out_dot16_bias(vc, b + 96, w + 12, acc);
+          acc = out_dot16_bias(vd, b + 112, w + 14, acc);
+        }
+      }
+      float* pt = part + (t & 1) * 2 * kTileM;
+      pt[h * kTileM + row] = __uint_as_float((uint32_t)acc) + __uint_as_float((uint32_t)(acc >> 32));
+      // the two halves of every row meet here; a stop is decided together
+      if (!named_bar_and(1, kPairEpi * 32, ok)) break;
+      if (h == 0) {
+        const int64_t g = (2 * ((int64_t)pair_id + (int64_t)t * n_pairs) + rank) * kTileM + row;
+        if (g < a.rows) a.scores[g] = (pt[row] + pt[kTileM + row]) + __ldg(params + p.b_last_off);
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // no arrival or product of either CTA is still aimed at the other
+  if (warp == 0) tmem_dealloc_pair(tmem, 512);
+}
+
 // Per batch, before the scorer: normalised bf16 template rows (instance row i
 // holds the z-scored instance features at their feature positions 6 ..
 // 6+d_inst and zeros elsewhere; request row r likewise for the request block)
@@ -1113,7 +1581,7 @@ __global__ void __launch_bounds__(256) k_feature_image(const int64_t* __restrict
 
 }  // namespace
 
-bool plan_tc(const MlpDesc& m, TcPlan& p) {
+bool plan_tc(const MlpDesc& m, TcPlan& p, bool allow_pair) {
   p = TcPlan{};
   if (!m.bf16 || m.n_layers < 2) return false;
   p.n_tc = m.n_layers - 1;
@@ -1180,6 +1648,40 @@ bool plan_tc(const MlpDesc& m, TcPlan& p) {
   // 128-row N-chunks, so the per-tile stream of [128 x 64] slices (layer 1
   // jobs, then layer 2 jobs, K-blocks inner) is the image itself, contiguous;
   // stages hold Q slices (Q in 4, 2, 1 dividing the slices per tile)
+  // pair variant (before the wide one): two hidden layers of multiples of 256
+  // (at most 512, so that the packed layer-1 activations and one 256-column
+  // accumulator fill the 512 TMEM columns), a feature tile of at most 128
+  // columns.  Each CTA of a pair streams its half of every [256 x 64] slice
+  // (16 KB: the image's per-rank streams); a stage holds Q half-slices, Q the
+  // largest divisor of the per-tile stream up to 6 that leaves two stages.
+  p.pair = 0;
+  if (allow_pair && !p.pipe && p.n_tc == 2 && p.out[0] % 256 == 0 && p.out[1] % 256 == 0 && p.d_pad <= 128) {
+    const int H1 = p.out[0], H2 = p.out[1];
+    const int nk0 = p.in_pad[0] / 64, nk1 = H1 / 64;
+    const int per_tile = (H1 / 256) * nk0 + (H2 / 256) * nk1;
+    const int64_t fixed = 1024 + (int64_t)nk0 * kTileM * 128 + (int64_t)(H1 + H2) * 4 + (int64_t)H2 * 2 +
+                          4 * kTileM * 4 + 10 * 8 + 16;
+    for (int Q = 6; Q >= 1 && !p.pair; --Q) {
+      if (per_tile % Q) continue;
+      const int64_t stages = (kMaxSmem - fixed) / ((int64_t)Q * kTileM * 128 + 16);
+      if (stages < 2) continue;
+      p.pair_q = Q;
+      p.pair_stages = (int)std::min<int64_t>(stages, 12);
+      p.pair_smem = (int)(fixed + (int64_t)p.pair_stages * ((int64_t)Q * kTileM * 128 + 16));
+      p.pair_slices = per_tile;
+      p.pair = 1;
+    }
+    if (p.pair) {
+      int64_t woff = 0;
+      for (int l = 0; l < 2; ++l) {
+        p.nc[l] = 128;
+        p.img_off[l] = woff;
+        woff += (int64_t)p.out[l] * p.in_pad[l] * 2;
+      }
+      p.img_bytes = woff;  // = 2 ranks x per_tile half-slices x 16 KB
+      return true;
+    }
+  }
   p.wide = 0;
   if (!p.pipe && p.n_tc == 2 && p.out[0] % 128 == 0 && p.out[1] % 128 == 0 && p.d_pad <= 128) {
     int64_t woff = 0;
@@ -1296,6 +1798,32 @@ cudaError_t launch_feature_image(const int64_t* tok_off, const int32_t* hits, in
                         req, mean, stdv, d_pad, rows, n_tiles, nr_max, ximg);
 }
 
+int pair_max_clusters(const TcPlan& p) {
+  if (!p.pair) return 0;
+  if (cudaFuncSetAttribute(k_score_pair, cudaFuncAttributeMaxDynamicSharedMemorySize, p.pair_smem) != cudaSuccess)
+    return 0;
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(std::max(2, sms & ~1));
+  cfg.blockDim = dim3(kThreadsPair);
+  cfg.dynamicSmemBytes = (size_t)p.pair_smem;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, k_score_pair, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return n;
+}
+
 cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const Published* pub, const int32_t* sel,
                             int n_req, int n_inst, const uint4* pairx, const uint8_t* ximg, int32_t* choice,
                             float* best,
@@ -1335,6 +1863,15 @@ cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const Published* 
     cudaError_t e = cudaFuncSetAttribute(k_score_tc_pipe, cudaFuncAttributeMaxDynamicSharedMemorySize, p.pipe_smem);
     if (e != cudaSuccess) return e;
     return launch_chained(k_score_tc_pipe, dim3(grid), dim3(kThreadsPipe), (size_t)p.pipe_smem, s, 1, a);
+  } else if (p.pair) {
+    // the image is in the pair layout, which no other scorer reads
+    if (!scores) return cudaErrorInvalidValue;
+    cudaError_t e = cudaFuncSetAttribute(k_score_pair, cudaFuncAttributeMaxDynamicSharedMemorySize, p.pair_smem);
+    if (e != cudaSuccess) return e;
+    const int tile_pairs = (a.n_tiles + 1) / 2;
+    const int fit = p.pair_clusters > 0 ? p.pair_clusters : sms / 2;
+    const int pairs = std::max(1, std::min(tile_pairs, fit));
+    return launch_chained(k_score_pair, dim3(2 * pairs), dim3(kThreadsPair), (size_t)p.pair_smem, s, 2, a);
   } else if (p.wide && scores) {
     cudaError_t e = cudaFuncSetAttribute(k_score_wide, cudaFuncAttributeMaxDynamicSharedMemorySize, p.wide_smem);
     if (e != cudaSuccess) return e;

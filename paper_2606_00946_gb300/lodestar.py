@@ -20,6 +20,7 @@ LS_F32, LS_BF16 = 0, 1
 LS_REPLACE, LS_INSERT = 0, 1
 LS_SGD, LS_ADAM = 0, 1
 LS_SCORER_AUTO, LS_SCORER_CUDA_CORES, LS_SCORER_TENSOR_CORES = 0, 1, 2
+LS_TC_NONE, LS_TC_GENERIC, LS_TC_PIPELINED, LS_TC_WIDE, LS_TC_PAIR = 0, 1, 2, 3, 4
 SCORERS = {"auto": 0, "cuda_cores": 1, "tensor_cores": 2}
 LS_STATIC_MAX_BLOCKS, LS_STATIC_MAX_PAIRS = 262144, 262144
 LS_PREFIX_AUTO, LS_PREFIX_TWO_PHASE, LS_PREFIX_FUSED, LS_PREFIX_INDEX = 0, 1, 2, 3
@@ -43,7 +44,7 @@ class ls_info(C.Structure):
     _fields_ = [("n_inst", C.c_int32), ("d", C.c_int32), ("n_params", C.c_int64),
                 ("table_slots", C.c_int64), ("ring_count", C.c_int64),
                 ("train_steps", C.c_int64), ("weight_version", C.c_uint64), ("scorer", C.c_int32),
-                ("replay_count", C.c_int64), ("pending_count", C.c_int64)]
+                ("replay_count", C.c_int64), ("pending_count", C.c_int64), ("tc_kernel", C.c_int32)]
 
 
 class ls_guards(C.Structure):

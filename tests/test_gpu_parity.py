@@ -285,23 +285,30 @@ def test_pipelined_scorer_with_tiles_across_requests(n_inst):
     r.close()
 
 
-@pytest.mark.parametrize("hidden,n_inst,wide_dims", [
-    ((512, 512), 24, False), ((512, 128), 200, False), ((128, 512), 7, False), ((256, 512), 256, True),
-    ((512, 512), 256, True)])
-def test_wide_scorer_shapes(hidden, n_inst, wide_dims):
-    # the wide tensor-core scorer (two hidden layers of multiples of 128 with
-    # weights streamed in slices; layer-1 activations packed in tensor memory)
-    # against the oracle: tiles across request boundaries, one and four
-    # layer-1 jobs, 64- and 128-column feature tiles
+@pytest.mark.parametrize("hidden,n_inst,wide_dims,n_req,kernel", [
+    ((512, 512), 24, False, 96, "pair"), ((256, 512), 256, True, 48, "pair"), ((512, 512), 256, True, 48, "pair"),
+    ((512, 512), 24, True, 100, "pair"), ((512, 256), 24, True, 5, "pair"), ((256, 256), 24, True, 100, "pair"),
+    ((512, 128), 200, False, 48, "wide"), ((128, 512), 7, False, 96, "wide"), ((256, 128), 24, True, 100, "wide"),
+    ((512, 512), 24, True, 100, "wide"), ((256, 512), 256, True, 48, "wide")])
+def test_wide_scorer_shapes(hidden, n_inst, wide_dims, n_req, kernel, monkeypatch):
+    # the streamed-weight tensor-core scorers against the oracle: the pair
+    # kernel (CTA pairs of 2-SM products, hidden widths multiples of 256) and
+    # the one-CTA wide kernel (multiples of 128; pair shapes too when planned
+    # with LS_TC_PAIR=0): tiles across request boundaries, one to four
+    # layer-1 jobs, 64- and 128-column feature tiles, an odd number of tiles
+    # (19: the last pair's second tile is past the batch) and a batch of one
+    # tile
     import dataclasses
+    if kernel == "wide":
+        monkeypatch.setenv("LS_TC_PAIR", "0")
     base = W.CONFIGS["large" if wide_dims else "homogeneous"]
-    cfg = dataclasses.replace(base, hidden=hidden, n_inst=n_inst, n_req=48 if n_inst > 64 else 96,
-                              cache_blocks=1024, n_samples=0)
+    cfg = dataclasses.replace(base, hidden=hidden, n_inst=n_inst, n_req=n_req, cache_blocks=1024, n_samples=0)
     wl = W.generate(cfg)
     r = H.Router.for_config(cfg)
     dw = H.DeviceWorkload(wl)
     dw.load(r)
     assert r.info().scorer == L.LS_SCORER_TENSOR_CORES
+    assert r.info().tc_kernel == {"wide": L.LS_TC_WIDE, "pair": L.LS_TC_PAIR}[kernel]
     out = r.route(dw.tok, dw.tok_off, dw.req_feats, n_inst)
     ref = oracle.route(wl, bounds=True, threads=THREADS)
     assert np.array_equal(out["hits"].cpu().numpy(), ref["hits"])

@@ -64,7 +64,7 @@ CALL_SAVES = {"k_guards": 16}
 
 
 def test_no_spills_on_the_path(kernels):
-    for name in ("k_score_tc_pipe", "k_feature_image", "k_prefix_index", "k_tr_gemm", "k_tr_step", "k_tr_gather",
+    for name in ("k_score_tc_pipe", "k_score_wide", "k_score_pair", "k_feature_image", "k_prefix_index", "k_tr_gemm", "k_tr_step", "k_tr_gather",
                  "k_tr_opt", "k_publish", "k_guards", "k_ring_bounds", "k_dist_rowmin"):
         for k, v in _find(kernels, name).items():
             assert v.get("spill", 0) <= 2 * CALL_SAVES.get(name, 0), (k, v)
@@ -73,6 +73,8 @@ def test_no_spills_on_the_path(kernels):
 def test_register_budgets(kernels):
     (pipe,) = _find(kernels, "k_score_tc_pipe").values()
     assert pipe["regs"] * 576 <= 65536          # 18 warps, one CTA per SM
+    (pair,) = _find(kernels, "k_score_pair").values()
+    assert pair["regs"] * 384 <= 65536          # 12 warps, one CTA per SM
     walk = [v for k, v in _find(kernels, "k_prefix_index").items() if "ILi1E" in k]
     assert walk and walk[0]["regs"] <= 72       # 7 CTAs x 128 threads per SM
     for v in _find(kernels, "k_tr_gemm").values():
