@@ -928,9 +928,16 @@ def measure_step(name, L, H, W, dev, stream, peaks, peak_src, args, ctx, clocks=
 
     side = torch.cuda.Stream(dev)  # training runs beside routing (Sec. 4.3.1: off the routing path)
 
-    def body(ks=0):
+    def body(ks=0, overlap=True):
         tok, tok_off, req = sets[ks]
         main = torch.cuda.current_stream(dev)
+        if not overlap:                             # the same calls, one after another on one stream
+            r.snapshot(N, stage_state)
+            r.route(tok, tok_off, req, N, out=out)
+            r.log(stage_x, stage_y)
+            r.train(Bt, None, opt="adam", lr=cfg.train_lr, loss_out=loss)
+            r.publish()
+            return
         side.wait_stream(main)                      # the step's inputs are in place
         r.snapshot(N, stage_state)
         r.route(tok, tok_off, req, N, out=out)
@@ -966,8 +973,16 @@ def measure_step(name, L, H, W, dev, stream, peaks, peak_src, args, ctx, clocks=
     clk = clocks.stop() if clocks is not None else None
     eager_times = timed_back_to_back(lambda k: eager_step(2 * args.warmup + args.steps + k),
                                      min(args.steps, 100), stream)
+    # per-kernel times from steps whose two branches run one after the other:
+    # a kernel of the training branch timed while the scorer holds every SM
+    # would count its wait for an SM as its own time
     n_traced = min(args.steps, 60)
-    trace = traced(L, r, lambda k: eager_step(k), n_traced)
+
+    def serial_step(k):
+        feed(k)
+        body(k % len(sets), overlap=False)
+
+    trace = traced(L, r, serial_step, n_traced)
     costs = batch_costs(r, wl, cfg, dw)
     rl = kernel_rooflines(trace, n_traced, costs, cfg, R, N, Bt, peaks, peak_src, name)
     per_step = {k: v[1] / max(v[2], 1) * v[0] / n_traced for k, v in trace.items()}
@@ -1210,6 +1225,8 @@ def main():
             "train_roofline": train_roofline,
             "kernel_rooflines": rl,
             "kernels_ms_per_step": {k: v for k, v in sorted(kms.items(), key=lambda kv: -kv[1])},
+            "kernels_timing": "CUDA events around each launch (library tracer) over steps issued call by call with "
+                              "the routing and training calls one after the other on one stream",
             "cpu_baseline": cpu,
             "e2e": e2e,
             "gpu_launches": int(round(launches_per_step * args.steps)),
