@@ -41,10 +41,10 @@
  *   - argmin ties -> lowest index, -0 == +0, NaN after every number;
  *   - guards: n = records ever appended; bounds = NaN-skipping min / max over
  *     the records the ring holds; prefix group = key of the first full block;
- *     ConsistentHash_K = top-K rendezvous hashing; gpu_kv sum in fp32 in
- *     index order; kappa_i |r| = 16 h_i; epsilon = 0, no random tiebreak;
- *   - heuristics: request count = queued + running columns, population
- *     standard deviation, sort ties to the lowest index;
+ *     ConsistentHash_K = top-K rendezvous hashing; gpu_kv mean in fp64 (sum
+ *     in index order); kappa_i |r| = 16 h_i; epsilon = 0, no random tiebreak;
+ *   - heuristics: request count = queued + running columns, mean and
+ *     population standard deviation in fp64, sort ties to the lowest index;
  *   - replay admission: one round per call, candidates ranked by distance to
  *     the nearest kept embedding, kept samples by distance to their nearest
  *     other kept sample, pairing while it raises diversity (or_replay_select).
