@@ -1084,15 +1084,15 @@ __device__ __forceinline__ void pack64_bias_relu(uint32_t taddr, const float* b,
 // layer-1 job 1 and every layer-2 job, released by the epilogue as soon as it
 // has been read.  The epilogues add the biases.
 // Warp roles in each CTA: 0 = MMA issuer (CTA 0) or stage relay (CTA 1), and
-// the TMEM allocation; 1 = producer of this CTA's half-slices; 2..3 = feature
-// tile builders; 4..11 = epilogue (lane quadrant warp % 4, column half
-// (warp - 4) / 4 of a job's 256).  Barriers the issuer waits on count arrivals
+// the TMEM allocation; 1 = producer of this CTA's half-slices; 2..7 = feature
+// tile builders; 8..15 = epilogue (lane quadrant warp % 4, column half
+// (warp - 8) / 4 of a job's 256).  Barriers the issuer waits on count arrivals
 // from both CTAs and live in CTA 0 (CTA 1 arrives remotely); barriers the
 // issuer signals are committed to both CTAs.
 // ---------------------------------------------------------------------------
-constexpr int kPairBuild = 2, kPairEpi = 8;  // builder and epilogue warps of the pair kernel
+constexpr int kPairBuild = 6, kPairEpi = 8;  // builder and epilogue warps of the pair kernel
 constexpr int kPairBuild0 = 2, kPairEpi0 = kPairBuild0 + kPairBuild;
-constexpr int kThreadsPair = (kPairEpi0 + kPairEpi) * 32;  // 384: up to 168 registers a thread
+constexpr int kThreadsPair = (kPairEpi0 + kPairEpi) * 32;  // 512: 128 registers a thread at launch
 constexpr int kHalfSlice = kTileM * 128;                   // [128 N x 64 K] bf16 = 16 KB
 
 // A timeout anywhere in a CTA pair stops both CTAs.
@@ -1164,9 +1164,9 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
   tc_fence_after();
   const uint32_t tmem = *tmem_holder;
   const uint32_t idesc = idesc_bf16_f32(2 * kTileM, 256);
-  // registers: warpgroup 0 (issuer, producer, builders) needs few, the two
-  // epilogue warpgroups read a whole accumulator half per thread at once;
-  // 128 x 88 + 256 x 208 = the 384 x 168 the CTA is launched with.  Each
+  // registers: warpgroups 0 and 1 (issuer, producer, builders) need few, the
+  // two epilogue warpgroups read 64 accumulator columns per thread at once;
+  // 256 x 88 + 256 x 168 = the 512 x 128 the CTA is launched with.  Each
   // warpgroup changes its budget at the head of its own branch.
   if (warp < kPairEpi0) {
     setmaxnreg_dec<88>();
@@ -1182,25 +1182,25 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
       const uint64_t ring_desc = sdesc_sw128(smem_u32(ring));
       const uint64_t x_desc = sdesc_sw128(smem_u32(X));
       for (int t = 0; t < my_pairs && ok; ++t) {
-        if (!(ok = mbar_wait_cl(x_full, (uint32_t)(t & 1)))) break;
+        if (!(ok = mbar_wait_cl_short(x_full, (uint32_t)(t & 1)))) break;
         tc_fence_after();
         for (int j = 0; j < J1 + J2 && ok; ++j) {
           const bool l2 = j >= J1;
           if (j == J1) umma_pair_commit_both(x_empty);  // both feature tiles free once the layer-1 products are done
           uint32_t d = tmem;  // D0: layer-1 job 0
           if (j > 0) {        // D1: its previous use has been read by both epilogues
-            if (u1 >= 1 && !(ok = mbar_wait_cl(d1_empty, (u1 - 1) & 1u))) break;
+            if (u1 >= 1 && !(ok = mbar_wait_cl_short(d1_empty, (u1 - 1) & 1u))) break;
             tc_fence_after();
             d = tmem + 256u;
           }
           const int nk = l2 ? nk1 : nk0;
           for (int kb = 0; kb < nk; ++kb) {
             if (j == J1 && (kb & 3) == 0) {  // K-blocks 4 i.. read layer-1 job i's activations
-              if (!(ok = mbar_wait_cl(&h1_ready[kb >> 2], (uint32_t)(t & 1)))) break;
+              if (!(ok = mbar_wait_cl_short(&h1_ready[kb >> 2], (uint32_t)(t & 1)))) break;
               tc_fence_after();
             }
             if (part_i == 0) {  // a new stage: both CTAs' copies have landed
-              if (!(ok = mbar_wait_cl(&full[st], (fpar >> st) & 1u))) break;
+              if (!(ok = mbar_wait_cl_short(&full[st], (fpar >> st) & 1u))) break;
               fpar ^= 1u << st;
               tc_fence_after();
             }
@@ -1293,7 +1293,7 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
     }
   }
   } else {
-    setmaxnreg_inc<208>();
+    setmaxnreg_inc<168>();
     // ------------------------------------------------------------ epilogue
     const int ew = warp - kPairEpi0;  // 0..7
     const int q4 = warp & 3;          // TMEM lane quadrant
@@ -1373,7 +1373,7 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
           }
           tc_fence_before();
           __syncwarp();
-          if (lane == 0) mbar_arrive_at(d1_empty, 0);  // D1 read: the next job may overwrite it
+          if (lane == 0) mbar_arrive_at_relaxed(d1_empty, 0);  // D1 read: the next job may overwrite it
           ++u1;
           if (go) {
             tmem_st32(dst + 32u, pb);
@@ -1382,7 +1382,7 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive_at(&h1_ready[j], 0);
+        if (lane == 0) mbar_arrive_at_relaxed(&h1_ready[j], 0);
       }
       uint64_t acc = 0;  // output-layer partial, two fp32 lanes
       for (int n = 0; n < J2; ++n) {
@@ -1398,40 +1398,29 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
         const uint32_t src = tmem + lane_addr + 256u + 128u * (uint32_t)h;
         const uint4* w = reinterpret_cast<const uint4*>(sw3 + 256 * n + 128 * h);
         const float* b = bias + H1 + 256 * n + 128 * h;
-        uint32_t va[16], vb[16], vc[16], vd[16];  // 64 columns per wait, two waits per job
+        uint32_t va[16], vb[16];
         if (go) {
           tc_fence_after();
           tmem_ld16(src, va);
-          tmem_ld16(src + 16u, vb);
-          tmem_ld16(src + 32u, vc);
-          tmem_ld16(src + 48u, vd);
+#pragma unroll
+          for (int i = 0; i < 6; i += 2) {
+            tmem_wait_ld_regs(va);
+            tmem_ld16(src + 16u * (i + 1), vb);
+            acc = out_dot16_bias(va, b + 16 * i, w + 2 * i, acc);
+            tmem_wait_ld_regs(vb);
+            tmem_ld16(src + 16u * (i + 2), va);
+            acc = out_dot16_bias(vb, b + 16 * (i + 1), w + 2 * (i + 1), acc);
+          }
           tmem_wait_ld_regs(va);
+          tmem_ld16(src + 16u * 7, vb);
+          acc = out_dot16_bias(va, b + 16 * 6, w + 12, acc);
           tmem_wait_ld_regs(vb);
-          tmem_wait_ld_regs(vc);
-          tmem_wait_ld_regs(vd);
-          acc = out_dot16_bias(va, b, w, acc);
-          acc = out_dot16_bias(vb, b + 16, w + 2, acc);
-          acc = out_dot16_bias(vc, b + 32, w + 4, acc);
-          acc = out_dot16_bias(vd, b + 48, w + 6, acc);
-          tmem_ld16(src + 64u, va);
-          tmem_ld16(src + 80u, vb);
-          tmem_ld16(src + 96u, vc);
-          tmem_ld16(src + 112u, vd);
-          tmem_wait_ld_regs(va);
-          tmem_wait_ld_regs(vb);
-          tmem_wait_ld_regs(vc);
-          tmem_wait_ld_regs(vd);
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive_at(d1_empty, 0);  // all of D1 read: the next job may overwrite it
+        if (lane == 0) mbar_arrive_at_relaxed(d1_empty, 0);  // all of D1 read: the next job may overwrite it
         ++u1;
-        if (go) {
-          acc = out_dot16_bias(va, b + 64, w + 8, acc);
-          acc = out_dot16_bias(vb, b + 80, w + 10, acc);
-          acc = out_dot16_bias(vc, b + 96, w + 12, acc);
-          acc = out_dot16_bias(vd, b + 112, w + 14, acc);
-        }
+        if (go) acc = out_dot16_bias(vb, b + 16 * 7, w + 14, acc);
       }
       float* pt = part + (t & 1) * 2 * kTileM;
       pt[h * kTileM + row] = __uint_as_float((uint32_t)acc) + __uint_as_float((uint32_t)(acc >> 32));

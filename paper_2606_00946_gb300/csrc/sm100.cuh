@@ -398,6 +398,16 @@ __device__ __forceinline__ void mbar_arrive_at(uint64_t* bar, uint32_t rank) {
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(bar)), "r"(rank));
   asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(remote) : "memory");
 }
+// Arrive without a release fence on the barrier at this offset in CTA
+// `rank`: for hand-offs whose data is not in memory the fence would order --
+// tensor-memory reads or writes the arriving thread has already completed
+// with tcgen05.wait::ld / ::st.  (A cluster-scope release costs ~1.5K cycles
+// here: it waits for every earlier memory operation of the thread.)
+__device__ __forceinline__ void mbar_arrive_at_relaxed(uint64_t* bar, uint32_t rank) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(bar)), "r"(rank));
+  asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(remote) : "memory");
+}
 // Wait with acquire at cluster scope (arrivals may come from the other CTA);
 // false after about kWaitCycles.
 __device__ __forceinline__ bool mbar_wait_cl(uint64_t* bar, uint32_t parity) {
@@ -410,6 +420,26 @@ __device__ __forceinline__ bool mbar_wait_cl(uint64_t* bar, uint32_t parity) {
         "selp.u32 %0, 1, 0, p;\n\t}\n"
         : "=r"(ok)
         : "r"(smem_u32(bar)), "r"(parity), "r"(20000u)
+        : "memory");
+    if (ok) return true;
+    if (clock64() - t0 > kWaitCycles) return false;
+  }
+}
+// The same wait with a short suspend-time hint (100 ns): for a thread on the
+// critical path.  A thread suspended with the 20 us hint was measured waking
+// ~1.7K cycles after a phase completed through arrivals from the other CTA
+// of a pair; spinning on test_wait instead took issue slots from the warps
+// beside it and was slower still.
+__device__ __forceinline__ bool mbar_wait_cl_short(uint64_t* bar, uint32_t parity) {
+  const long long t0 = clock64();
+  while (true) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}\n"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity), "r"(100u)
         : "memory");
     if (ok) return true;
     if (clock64() - t0 > kWaitCycles) return false;

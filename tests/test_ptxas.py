@@ -74,7 +74,7 @@ def test_register_budgets(kernels):
     (pipe,) = _find(kernels, "k_score_tc_pipe").values()
     assert pipe["regs"] * 576 <= 65536          # 18 warps, one CTA per SM
     (pair,) = _find(kernels, "k_score_pair").values()
-    assert pair["regs"] * 384 <= 65536          # 12 warps, one CTA per SM
+    assert pair["regs"] * 512 <= 65536          # 16 warps, one CTA per SM (budgets then moved by setmaxnreg)
     walk = [v for k, v in _find(kernels, "k_prefix_index").items() if "ILi1E" in k]
     assert walk and walk[0]["regs"] <= 72       # 7 CTAs x 128 threads per SM
     for v in _find(kernels, "k_tr_gemm").values():
