@@ -71,7 +71,7 @@ __device__ __forceinline__ uint64_t index_mask_w1(const uint64_t* __restrict__ e
 }
 
 template <int W>
-__global__ void __launch_bounds__(kNT, W <= 2 ? 7 : 1) k_prefix_index(int n_req, const int32_t* __restrict__ tok,
+__global__ void __launch_bounds__(kNT, W <= 4 ? 8 : 1) k_prefix_index(int n_req, const int32_t* __restrict__ tok,
                                                       const int64_t* __restrict__ tok_off,
                                                       const uint64_t* __restrict__ gkeys,
                                                       const uint64_t* __restrict__ gmask, uint64_t gmask_slots,
