@@ -45,6 +45,9 @@ struct SeqArgs {
   const DevState* st;
   MlpDesc m;
   int wmax;               // widest layer input / output
+  int wsm;                // 1: the weights are copied into shared memory once per call
+  int64_t wbytes;         // size of that weight region
+  int64_t woff_s[LS_MAX_LAYERS];  // byte offset of layer l's transposed weights in the weight region
   uint64_t* gkeys;
   uint64_t* gmask;
   int W;
@@ -108,25 +111,40 @@ __device__ __forceinline__ bool seq_precedes(float a, int i, float b, int j) {
   return i < j;
 }
 
-// Byte offsets of the shared-memory arrays (each 16-byte aligned).
+// Byte offsets of the shared-memory arrays (each 16-byte aligned).  Layer
+// inputs and activations take `xe` bytes each: 2 in bf16 mode (their values
+// are bf16-rounded, so bf16 holds them exactly), 4 in fp32 mode.  The weight
+// region (`wbytes`, 0 when the weights stay in global memory) holds every
+// layer's W^T [in][out] in the predictor's element type.
 struct SeqSmem {
-  size_t inst, x0, x1, sc, hh, pa, wtot, carry, rv, ri, total;
+  size_t inst, x0, x1, sc, hh, pa, wtot, carry, rv, ri, w, total;
 };
 __host__ __device__ __forceinline__ size_t seq_al(size_t b) { return (b + 15) & ~(size_t)15; }
-__host__ __device__ __forceinline__ SeqSmem seq_smem(int N, int DI, int wmax, int W) {
+__host__ __device__ __forceinline__ SeqSmem seq_smem(int N, int DI, int wmax, int W, int xe, size_t wbytes) {
   SeqSmem o;
   o.inst = 0;                                                   // [N][d_inst] fp32
-  o.x0 = seq_al(o.inst + (size_t)N * (DI > 0 ? DI : 1) * 4);    // [N][wmax] fp32
-  o.x1 = seq_al(o.x0 + (size_t)N * wmax * 4);                   // [N][wmax] fp32
-  o.sc = seq_al(o.x1 + (size_t)N * wmax * 4);                   // [N] scores
+  o.x0 = seq_al(o.inst + (size_t)N * (DI > 0 ? DI : 1) * 4);    // [N][wmax] activations
+  o.x1 = seq_al(o.x0 + (size_t)N * wmax * xe);                  // [N][wmax] activations
+  o.sc = seq_al(o.x1 + (size_t)N * wmax * xe);                  // [N] scores
   o.hh = seq_al(o.sc + (size_t)N * 4);                          // [N] hit lengths
   o.pa = seq_al(o.hh + (size_t)N * 4);                          // [kSeqThreads][W] prefix AND
   o.wtot = seq_al(o.pa + (size_t)kSeqThreads * W * 8);          // [kSeqWarps][W]
   o.carry = seq_al(o.wtot + (size_t)kSeqWarps * W * 8);         // [W]
   o.rv = seq_al(o.carry + (size_t)W * 8);                       // [kSeqWarps] argmin values
   o.ri = seq_al(o.rv + (size_t)kSeqWarps * 4);                  // [kSeqWarps] argmin indices
-  o.total = seq_al(o.ri + (size_t)kSeqWarps * 4);
+  o.w = seq_al(o.ri + (size_t)kSeqWarps * 4);                   // transposed weights (optional)
+  o.total = seq_al(o.w + wbytes);
   return o;
+}
+
+// Activation element i of an array of `xe`-byte elements, as fp32 / stored.
+__device__ __forceinline__ float seq_xget(const uint8_t* X, int64_t i, bool bf) {
+  return bf ? __uint_as_float((uint32_t)reinterpret_cast<const uint16_t*>(X)[i] << 16)
+            : reinterpret_cast<const float*>(X)[i];
+}
+__device__ __forceinline__ void seq_xset(uint8_t* X, int64_t i, float v, bool bf) {
+  if (bf) reinterpret_cast<uint16_t*>(X)[i] = (uint16_t)(__float_as_uint(round_bf16(v)) >> 16);
+  else reinterpret_cast<float*>(X)[i] = v;
 }
 
 __global__ void __launch_bounds__(kSeqThreads, 1) k_route_seq(const __grid_constant__ SeqArgs a, int64_t bcap) {
@@ -134,10 +152,12 @@ __global__ void __launch_bounds__(kSeqThreads, 1) k_route_seq(const __grid_const
   const int N = a.n_inst, DI = a.d_inst, W = a.W;
   const MlpDesc& m = a.m;
   const int d = m.w[0];
-  const SeqSmem o = seq_smem(N, DI, a.wmax, W);
+  const bool bf = m.bf16 != 0;
+  const SeqSmem o = seq_smem(N, DI, a.wmax, W, bf ? 2 : 4, a.wsm ? (size_t)a.wbytes : 0);
   float* sinst = reinterpret_cast<float*>(smem_raw + o.inst);
-  float* X0 = reinterpret_cast<float*>(smem_raw + o.x0);
-  float* X1 = reinterpret_cast<float*>(smem_raw + o.x1);
+  uint8_t* X0 = smem_raw + o.x0;
+  uint8_t* X1 = smem_raw + o.x1;
+  uint8_t* Wsm = smem_raw + o.w;
   float* sc = reinterpret_cast<float*>(smem_raw + o.sc);
   int32_t* hh = reinterpret_cast<int32_t*>(smem_raw + o.hh);
   uint64_t* PA = reinterpret_cast<uint64_t*>(smem_raw + o.pa);
@@ -151,6 +171,21 @@ __global__ void __launch_bounds__(kSeqThreads, 1) k_route_seq(const __grid_const
   for (int e = tid; e < N * DI; e += kSeqThreads) sinst[e] = a.inst[e];
   __syncthreads();
   const float* __restrict__ params = s_buf ? a.params1 : a.params0;
+  if (a.wsm) {
+    // every layer's W^T [in][out] in shared memory for the whole call (the
+    // published weights, bf16-valued in bf16 mode, so bf16 holds them exactly);
+    // read along W's rows (coalesced), written transposed
+    for (int l = 0; l < m.n_layers; ++l) {
+      const int in = m.w[l], out = m.w[l + 1];
+      const float* __restrict__ Wl = params + m.woff[l];
+      uint8_t* Wt = Wsm + a.woff_s[l];
+      for (int e = tid; e < in * out; e += kSeqThreads) {
+        const int oo = e / in, k = e - oo * in;
+        seq_xset(Wt, (int64_t)k * out + oo, __ldg(Wl + e), bf);
+      }
+    }
+    __syncthreads();
+  }
   const int64_t base = a.tok_off[0];
   for (int r = 0; r < a.n_req; ++r) {
     const int64_t t0 = a.tok_off[r];
@@ -234,46 +269,92 @@ __global__ void __launch_bounds__(kSeqThreads, 1) k_route_seq(const __grid_const
       else if (k < kPair + DI) raw = sinst[i * DI + (k - kPair)];
       else raw = a.req[(int64_t)r * a.d_req + (k - kPair - DI)];
       const float x = zscore(raw, a.mean[k], a.stdv[k]);
-      X0[i * a.wmax + k] = m.bf16 ? round_bf16(x) : x;
+      seq_xset(X0, (int64_t)i * a.wmax + k, x, bf);
     }
     __syncthreads();
-    // ---- 3. the predictor, warp per output column
-    float* xin = X0;
-    float* xout = X1;
+    // ---- 3. the predictor
+    uint8_t* xin = X0;
+    uint8_t* xout = X1;
     for (int l = 0; l < m.n_layers; ++l) {
       const int in = m.w[l], out = m.w[l + 1];
       const bool last_layer = l + 1 == m.n_layers;
-      const float* __restrict__ Wl = params + m.woff[l];
       const float* __restrict__ bl = params + m.boff[l];
-      for (int o = warp; o < out; o += kSeqWarps) {
-        float wr[16];
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          const int k = lane + 32 * j;
-          wr[j] = k < in ? __ldg(Wl + (int64_t)o * in + k) : 0.0f;
-        }
-        const float bo = __ldg(bl + o);
-        for (int i = 0; i < N; ++i) {
+      if (a.wsm && out < 32) {
+        // a narrow layer (the output layer): warp per row, lanes across K
+        const uint8_t* Wt = Wsm + a.woff_s[l];
+        for (int e = warp; e < N * out; e += kSeqWarps) {
+          const int i = e / out, oo = e - i * out;
           float part = 0.0f;
+          for (int k = lane; k < in; k += 32)
+            part = fmaf(seq_xget(Wt, (int64_t)k * out + oo, bf), seq_xget(xin, (int64_t)i * a.wmax + k, bf), part);
+#pragma unroll
+          for (int sft = 16; sft; sft >>= 1) part += __shfl_xor_sync(kFull, part, sft);
+          if (lane == 0) {
+            const float z = part + __ldg(bl + oo);
+            if (last_layer) sc[i] = z;
+            else seq_xset(xout, (int64_t)i * a.wmax + oo, fmaxf(z, 0.0f), bf);
+          }
+        }
+      } else if (a.wsm) {
+        // thread per (output, four rows): one weight and four broadcast
+        // inputs per K step, fp32 sums, the bias added after the sum
+        const uint8_t* Wt = Wsm + a.woff_s[l];
+        const int nb4 = (N + 3) >> 2;
+        const int xe = bf ? 2 : 4;
+        for (int e = tid; e < nb4 * out; e += kSeqThreads) {
+          const int oo = e % out, i0 = (e / out) * 4;
+          const uint8_t* xr[4];
+#pragma unroll
+          for (int q = 0; q < 4; ++q) xr[q] = xin + (size_t)min(i0 + q, N - 1) * a.wmax * xe;
+          const uint8_t* wp = Wt + (size_t)oo * xe;
+          const int wstep = out * xe;
+          float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll 4
+          for (int k = 0; k < in; ++k, wp += wstep) {
+            const float wv = seq_xget(wp, 0, bf);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) acc[q] = fmaf(wv, seq_xget(xr[q], k, bf), acc[q]);
+          }
+          const float bo = __ldg(bl + oo);
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            if (i0 + q >= N) break;
+            const float z = acc[q] + bo;
+            if (last_layer) sc[i0 + q] = z;
+            else seq_xset(xout, (int64_t)(i0 + q) * a.wmax + oo, fmaxf(z, 0.0f), bf);
+          }
+        }
+      } else {
+        // weights too large for shared memory: warp per output column, lanes
+        // across K, the column's weights in registers
+        const float* __restrict__ Wl = params + m.woff[l];
+        for (int oo = warp; oo < out; oo += kSeqWarps) {
+          float wr[16];
 #pragma unroll
           for (int j = 0; j < 16; ++j) {
             const int k = lane + 32 * j;
-            if (k < in) part = fmaf(wr[j], xin[i * a.wmax + k], part);
+            wr[j] = k < in ? __ldg(Wl + (int64_t)oo * in + k) : 0.0f;
           }
+          const float bo = __ldg(bl + oo);
+          for (int i = 0; i < N; ++i) {
+            float part = 0.0f;
 #pragma unroll
-          for (int s = 16; s; s >>= 1) part += __shfl_xor_sync(kFull, part, s);
-          if (lane == 0) {
-            const float z = part + bo;
-            if (last_layer) sc[i] = z;
-            else {
-              const float act = fmaxf(z, 0.0f);
-              xout[i * a.wmax + o] = m.bf16 ? round_bf16(act) : act;
+            for (int j = 0; j < 16; ++j) {
+              const int k = lane + 32 * j;
+              if (k < in) part = fmaf(wr[j], seq_xget(xin, (int64_t)i * a.wmax + k, bf), part);
+            }
+#pragma unroll
+            for (int sft = 16; sft; sft >>= 1) part += __shfl_xor_sync(kFull, part, sft);
+            if (lane == 0) {
+              const float z = part + bo;
+              if (last_layer) sc[i] = z;
+              else seq_xset(xout, (int64_t)i * a.wmax + oo, fmaxf(z, 0.0f), bf);
             }
           }
         }
       }
       __syncthreads();
-      float* t = xin;
+      uint8_t* t = xin;
       xin = xout;
       xout = t;
     }
@@ -319,10 +400,11 @@ __global__ void __launch_bounds__(kSeqThreads, 1) k_route_seq(const __grid_const
 
 }  // namespace
 
-// Shared memory of the sequential route, 0 if the shape does not fit.
+// Shared memory of the sequential route without the weight region, 0 if the
+// shape does not fit (bf16 activations: the smaller of the two layouts).
 size_t route_seq_smem(int n_inst, int d_inst, int wmax, int W) {
   if (W < 1 || W > kSeqMaxW || wmax > 512 || n_inst < 1) return 0;
-  const size_t b = seq_smem(n_inst, d_inst, wmax, W).total;
+  const size_t b = seq_smem(n_inst, d_inst, wmax, W, 4, 0).total;
   return b <= 200 * 1024 ? b : 0;
 }
 
@@ -363,8 +445,18 @@ cudaError_t launch_route_seq(int n_req, int n_inst, int d_inst, int d_req, int q
   a.scores = scores;
   a.hits = hits;
   a.err = err;
-  const size_t smem = route_seq_smem(n_inst, d_inst, wmax, W);
-  if (!smem) return cudaErrorInvalidValue;
+  if (!route_seq_smem(n_inst, d_inst, wmax, W)) return cudaErrorInvalidValue;
+  const int xe = m.bf16 ? 2 : 4;
+  int64_t wb = 0;
+  for (int l = 0; l < m.n_layers; ++l) {
+    a.woff_s[l] = wb;
+    wb += (((int64_t)m.w[l] * m.w[l + 1] * xe) + 15) & ~(int64_t)15;
+  }
+  // the weights go to shared memory when they fit beside the rest
+  const size_t with_w = seq_smem(n_inst, d_inst, wmax, W, xe, (size_t)wb).total;
+  a.wsm = with_w <= 224 * 1024 ? 1 : 0;
+  a.wbytes = a.wsm ? wb : 0;
+  const size_t smem = a.wsm ? with_w : seq_smem(n_inst, d_inst, wmax, W, xe, 0).total;
   cudaError_t e = cudaFuncSetAttribute(k_route_seq, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   k_route_seq<<<1, kSeqThreads, smem, s>>>(a, bcap);
