@@ -167,10 +167,14 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
   c.n_params = off;
   {
     // LS_TC_PAIR=0 in the environment plans without the pair kernel (the
-    // one-CTA wide kernel takes its shapes), so that both stay exercised
+    // one-CTA wide kernel takes its shapes), LS_TC_PIPE=0 without the
+    // pipelined one, so that each kernel stays exercised on shapes another
+    // one would take
     const char* pair_env = std::getenv("LS_TC_PAIR");
+    const char* pipe_env = std::getenv("LS_TC_PIPE");
     const bool allow_pair = !(pair_env && pair_env[0] == '0');
-    const bool can_tc = plan_tc(m, c.tc, allow_pair);
+    const bool allow_pipe = !(pipe_env && pipe_env[0] == '0');
+    const bool can_tc = plan_tc(m, c.tc, allow_pair, allow_pipe);
     if (cfg->scorer == LS_SCORER_TENSOR_CORES && !can_tc) {
       delete h;
       return fail(LS_ERR_ARG, "tensor-core scorer needs a bf16 predictor with hidden widths that are "
@@ -180,7 +184,7 @@ int ls_create(const ls_config* cfg, ls_ctx** out) {
     if (c.use_tc && c.tc.pair) {  // the pair kernel needs CTA pairs that fit together on the device
       const int k = pair_max_clusters(c.tc);
       if (k < 1)
-        plan_tc(m, c.tc, false);
+        plan_tc(m, c.tc, false, allow_pipe);
       else
         c.tc.pair_clusters = k;
     }

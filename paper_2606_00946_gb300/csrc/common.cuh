@@ -443,8 +443,8 @@ cudaError_t launch_guards(const ls_guards& g, int n_req, int n_inst, const int32
 constexpr int kGuardHeurMaxInst = 1024;  // instances the heuristic keeps in shared memory
 
 // Plan the tensor-core scorer; `allow_pair` false leaves the pair kernel out
-// (and its image layout).
-bool plan_tc(const MlpDesc& m, TcPlan& p, bool allow_pair = true);
+// (and its image layout), `allow_pipe` false the pipelined one.
+bool plan_tc(const MlpDesc& m, TcPlan& p, bool allow_pair = true, bool allow_pipe = true);
 // CTA pairs of the pair kernel that can be resident at once (0: none).
 int pair_max_clusters(const TcPlan& p);
 // Publish the master weights into buffer 1 - st->cur (fp32 params, the

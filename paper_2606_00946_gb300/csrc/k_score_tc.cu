@@ -1570,7 +1570,7 @@ __global__ void __launch_bounds__(256) k_feature_image(const int64_t* __restrict
 
 }  // namespace
 
-bool plan_tc(const MlpDesc& m, TcPlan& p, bool allow_pair) {
+bool plan_tc(const MlpDesc& m, TcPlan& p, bool allow_pair, bool allow_pipe) {
   p = TcPlan{};
   if (!m.bf16 || m.n_layers < 2) return false;
   p.n_tc = m.n_layers - 1;
@@ -1624,7 +1624,8 @@ bool plan_tc(const MlpDesc& m, TcPlan& p, bool allow_pair) {
   p.b_last_off = m.boff[m.n_layers - 1];
   // pipelined variant: two hidden layers of <= 256, all weights resident
   p.pipe = 0;
-  if (p.n_tc == 2 && p.out[0] <= 256 && p.out[1] <= 256 && p.nc[0] == p.out[0] && p.nc[1] == p.out[1]) {
+  if (allow_pipe && p.n_tc == 2 && p.out[0] <= 256 && p.out[1] <= 256 && p.nc[0] == p.out[0] &&
+      p.nc[1] == p.out[1]) {
     const int64_t need = 1024 + (int64_t)p.chunks * cb + kXB * (int64_t)p.d_pad * kTileM * 2 + 2 * kTileM * 128 +
                          8 * 32 + 2 * 256 * 32 + 2 * kTileM * 4 + 256 * 2 + (12 + kWBars) * 8 + 16;
     if (need <= kMaxSmem) {

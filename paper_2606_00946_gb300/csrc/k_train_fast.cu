@@ -114,25 +114,69 @@ __device__ __forceinline__ float col_reduce16(float (&v)[16]) {
   return v[0] + __shfl_xor_sync(0xffffffffu, v[0], 16);
 }
 
-// Row-major image: 16 bf16 values of row j, columns c..c+15 (c % 16 == 0).
-__device__ __forceinline__ void store_row16(uint8_t* img, int rows, int j, int c, const float (&v)[16]) {
+// Row-major image from packed bf16 pairs: w[h] holds columns c + 2h (low
+// half) and c + 2h + 1 (high half) of row j; c % 16 == 0.
+__device__ __forceinline__ void store_row16p(uint8_t* img, int rows, int j, int c, const uint32_t (&w)[8]) {
+  *reinterpret_cast<uint4*>(img + sw128_offset(j, c, rows)) = make_uint4(w[0], w[1], w[2], w[3]);
+  *reinterpret_cast<uint4*>(img + sw128_offset(j, c + 8, rows)) = make_uint4(w[4], w[5], w[6], w[7]);
+}
+
+// Transposed image [rowsT x 128] from packed bf16 pairs: element (c + u, r)
+// for u < 16, c % 16 == 0, r < 128 the tile row.  The same bytes as
+// sw128_offset(c + u, r, rowsT), with the row's swizzle phase (c + u) & 7 =
+// u & 7 folded into per-store constants.
+__device__ __forceinline__ void store_col16p(uint8_t* imgT, int rowsT, int r, int c, const uint32_t (&w)[8]) {
+  uint8_t* base = imgT + (size_t)(r >> 6) * rowsT * 128 + (size_t)c * 128 + (r & 7) * 2;
+  const uint32_t cx = (uint32_t)((r & 63) >> 3) << 4;
 #pragma unroll
-  for (int g = 0; g < 2; ++g) {
-    uint4 q;
-    q.x = pack2(v[8 * g], v[8 * g + 1]);
-    q.y = pack2(v[8 * g + 2], v[8 * g + 3]);
-    q.z = pack2(v[8 * g + 4], v[8 * g + 5]);
-    q.w = pack2(v[8 * g + 6], v[8 * g + 7]);
-    *reinterpret_cast<uint4*>(img + sw128_offset(j, c + 8 * g, rows)) = q;
+  for (int u = 0; u < 16; ++u) {
+    const uint16_t v = (u & 1) ? (uint16_t)(w[u >> 1] >> 16) : (uint16_t)(w[u >> 1] & 0xffffu);
+    *reinterpret_cast<uint16_t*>(base + u * 128 + (cx ^ ((uint32_t)(u & 7) << 4))) = v;
   }
 }
 
-// Transposed image: element (c + u, j) for u < 16; lanes hold consecutive j,
-// so each column is written as 2-byte pieces of one 64-byte run per warp.
-__device__ __forceinline__ void store_col16(uint8_t* imgT, int rowsT, int j, int c, const float (&v)[16]) {
+// Forward epilogue of one warp's columns [cbeg, cbeg + cw) of its 32 tile
+// rows (r the thread's row): Z + b, ReLU and, with `drop`, dropout of unit
+// n0 + c under the stream h1 (key rowkey + c, rowkey = (row << 20) | n0),
+// each activation rounded to bf16 once as packed pairs that both images take
+// their bytes from, and the 16-bit masks [Z > 0 and kept].
+__device__ __forceinline__ void fwd_cols(uint32_t taddr, const float* s_bias, int cbeg, int cw, uint8_t* S1,
+                                         uint8_t* S2, int NT, int r, uint16_t* mask_out, int64_t rows_pad,
+                                         bool drop, uint64_t h1, uint64_t rowkey, uint64_t drop_thr,
+                                         float drop_scale) {
+  for (int c = cbeg; c < cbeg + cw; c += 16) {
+    uint32_t v[16];
+    tmem_ld16x(taddr + (uint32_t)c, v);
+    tmem_wait_ld();
+    uint32_t w[8];
+    uint32_t bits = 0;
 #pragma unroll
-  for (int u = 0; u < 16; ++u)
-    *reinterpret_cast<uint16_t*>(imgT + sw128_offset(c + u, j, rowsT)) = bf16_bits(v[u]);
+    for (int g = 0; g < 4; ++g) {
+      const float4 q4 = reinterpret_cast<const float4*>(s_bias + c)[g];
+      const float bq[4] = {q4.x, q4.y, q4.z, q4.w};
+      float a4[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int u = 4 * g + e;
+        const float z = __uint_as_float(v[u]) + bq[e];
+        float rv = z > 0.0f ? z : 0.0f;
+        bool on = z > 0.0f;
+        if (drop) {
+          const uint64_t hu = bh::mix64(h1 ^ (rowkey + (uint64_t)(c + u)));
+          const bool keep = (hu >> 11) >= drop_thr;
+          on = on && keep;
+          rv = keep ? rv * drop_scale : 0.0f;
+        }
+        bits |= (on ? 1u : 0u) << u;
+        a4[e] = rv;
+      }
+      w[2 * g] = pack2(a4[0], a4[1]);
+      w[2 * g + 1] = pack2(a4[2], a4[3]);
+    }
+    mask_out[(int64_t)(c >> 4) * rows_pad] = (uint16_t)bits;
+    store_row16p(S1, kM, r, c, w);
+    store_col16p(S2, NT, r, c, w);
+  }
 }
 
 // Shared memory of a training-product CTA: kMaxChunks stages of one 128-row A
@@ -141,12 +185,74 @@ __device__ __forceinline__ uint8_t* tr_tail(uint8_t* smem) {
   return smem + (size_t)kMaxChunks * (kM * 128 + 256 * 128);
 }
 
+// The part of tile `bid` that reads nothing the step's earlier products
+// write: arm every chunk barrier for the tile (the chunk barriers it does not
+// use are arrived on with no bytes, so each advances one phase per tile),
+// copy the weight operand (forward and input-gradient products read the
+// weight images, which only the optimiser of the previous step writes) and
+// stage the epilogue's bias and output weights (the fp32 master).  A
+// per-launch product runs it before waiting for its predecessor.
+__device__ __forceinline__ void tr_tile_pre(const TrArgs& args, int bid, uint8_t* smem) {
+  const bool second = bid >= args.n_cta0;
+  const TrJob& J = args.job[second ? 1 : 0];
+  const int li = second ? bid - args.n_cta0 : bid;
+  const int ns = li % J.n_split, rest = li / J.n_split;
+  const int split = rest / J.m_tiles;
+  const int NT = J.NT, N = NT * J.n_split, n0 = ns * NT, nch = J.nchunks;
+  const uint32_t a_bytes = kM * 128, b_bytes = (uint32_t)NT * 128;
+  const uint32_t stage_bytes = a_bytes + b_bytes;
+  uint8_t* tail = tr_tail(smem);
+  uint64_t* full = reinterpret_cast<uint64_t*>(tail);
+  float* s_bias = reinterpret_cast<float*>(tail + 128);
+  float* s_w = s_bias + 256;
+  const int tid = threadIdx.x;
+  if (tid == 0) {
+    const bool b_static = J.epi != TE_STORE;  // the weight-gradient products read activations
+    for (int c = 0; c < nch; ++c) {
+      const int kb = split * nch + c;
+      mbar_arrive_expect_tx(&full[c], stage_bytes);
+      if (b_static) bulk_g2s(smem + (size_t)c * stage_bytes + a_bytes, J.B + (size_t)kb * N * 128 + (size_t)n0 * 128,
+                             b_bytes, &full[c]);
+    }
+    for (int c = nch; c < kMaxChunks; ++c) mbar_arrive(&full[c]);
+  }
+  for (int t = tid; t < NT; t += kT) {
+    if (J.bias) s_bias[t] = __ldg(J.bias + n0 + t);
+    if (J.epi == TE_FWD_OUT) s_w[t] = round_bf16(__ldg(J.wL + n0 + t));
+  }
+}
+
+// The operand copies of tile `bid` that tr_tile_pre left (the activation or
+// gradient operand; both operands of a weight-gradient product), by one
+// thread, onto the barriers tr_tile_pre armed.
+__device__ __forceinline__ void tr_tile_copies(const TrArgs& args, int bid, uint8_t* smem) {
+  const bool second = bid >= args.n_cta0;
+  const TrJob& J = args.job[second ? 1 : 0];
+  const int li = second ? bid - args.n_cta0 : bid;
+  const int ns = li % J.n_split, rest = li / J.n_split;
+  const int mt = rest % J.m_tiles, split = rest / J.m_tiles;
+  const int m0 = mt * kM;
+  const int NT = J.NT, N = NT * J.n_split, n0 = ns * NT, nch = J.nchunks;
+  const uint32_t a_bytes = kM * 128, b_bytes = (uint32_t)NT * 128;
+  const uint32_t stage_bytes = a_bytes + b_bytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(tr_tail(smem));
+  for (int c = 0; c < nch; ++c) {
+    const int kb = split * nch + c;
+    uint8_t* sa = smem + (size_t)c * stage_bytes;
+    bulk_g2s(sa, J.A + (size_t)kb * J.rA * 128 + (size_t)m0 * 128, a_bytes, &full[c]);
+    if (J.epi == TE_STORE) bulk_g2s(sa + a_bytes, J.B + (size_t)kb * N * 128 + (size_t)n0 * 128, b_bytes, &full[c]);
+  }
+}
+
 // One output tile (part `bid` of the products in `args`) on this CTA's shared
-// memory and TMEM accumulator.  Every mbarrier advances by one phase per tile
-// (parity `par`): chunk barriers the tile does not use are arrived on with no
-// bytes.  Returns false after a timed-out wait (error latched, copies in
-// flight waited for).
-__device__ __forceinline__ bool tr_tile(const TrArgs& args, int bid, uint8_t* smem, uint32_t tmem, uint32_t par) {
+// memory and TMEM accumulator, after tr_tile_pre of the same tile (and, when
+// `copied`, tr_tile_copies).  Every
+// mbarrier advances by one phase per tile (parity `par`).  `drain` waits for
+// the tile's image stores to reach global memory (other CTAs of the grid read
+// them); otherwise only until they have read shared memory.  Returns false
+// after a timed-out wait (error latched, copies in flight waited for).
+__device__ __forceinline__ bool tr_tile(const TrArgs& args, int bid, uint8_t* smem, uint32_t tmem, uint32_t par,
+                                        bool drain, bool copied) {
   const bool second = bid >= args.n_cta0;
   const TrJob& J = args.job[second ? 1 : 0];
   const int li = second ? bid - args.n_cta0 : bid;
@@ -171,14 +277,7 @@ __device__ __forceinline__ bool tr_tile(const TrArgs& args, int bid, uint8_t* sm
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   bool ok = true;
   if (tid == 0) {
-    for (int c = 0; c < nch; ++c) {
-      const int kb = split * nch + c;
-      uint8_t* sa = smem + (size_t)c * stage_bytes;
-      mbar_arrive_expect_tx(&full[c], stage_bytes);
-      bulk_g2s(sa, J.A + (size_t)kb * J.rA * 128 + (size_t)m0 * 128, a_bytes, &full[c]);
-      bulk_g2s(sa + a_bytes, J.B + (size_t)kb * N * 128 + (size_t)n0 * 128, b_bytes, &full[c]);
-    }
-    for (int c = nch; c < kMaxChunks; ++c) mbar_arrive(&full[c]);
+    if (!copied) tr_tile_copies(args, bid, smem);
     const uint32_t idesc = idesc_bf16_f32(kM, NT);
     for (int c = 0; c < nch; ++c) {
       if (!mbar_wait(&full[c], par)) { ok = false; break; }
@@ -189,11 +288,6 @@ __device__ __forceinline__ bool tr_tile(const TrArgs& args, int bid, uint8_t* sm
         umma_bf16(tmem, sdesc_sw128(sa + 32u * k), sdesc_sw128(sb + 32u * k), idesc, (c | k) ? 1u : 0u);
     }
     umma_commit(done);  // arrives once everything issued so far has completed
-  }
-  // side inputs of the epilogue, staged while the copies and MMAs run
-  for (int t = tid; t < NT; t += kT) {
-    if (J.bias) s_bias[t] = __ldg(J.bias + n0 + t);
-    if (J.epi == TE_FWD_OUT) s_w[t] = round_bf16(__ldg(J.wL + n0 + t));
   }
   __syncwarp();
   if (!mbar_wait(done, par)) ok = false;
@@ -241,30 +335,10 @@ __device__ __forceinline__ bool tr_tile(const TrArgs& args, int bid, uint8_t* sm
       const uint64_t t = (uint64_t)(*reinterpret_cast<const volatile int64_t*>(&args.st->step) + 1);
       h1 = bh::mix64(args.drop_seed ^ ((t << 16) | (uint64_t)J.drop_h));
     }
-    for (int c = cbeg; c < cbeg + cw; c += 16) {
-      uint32_t v[16];
-      tmem_ld16x(tmem + lane_addr + (uint32_t)c, v);
-      tmem_wait_ld();
-      float a[16];
-      uint32_t bits = 0;
-#pragma unroll
-      for (int u = 0; u < 16; ++u) {
-        const float z = __uint_as_float(v[u]) + s_bias[c + u];
-        float r = z > 0.0f ? z : 0.0f;
-        bool on = z > 0.0f;
-        if (J.drop_h > 0) {
-          const uint64_t hu = bh::mix64(h1 ^ (((uint64_t)j << 20) | (uint64_t)(n0 + c + u)));
-          const bool keep = (hu >> 11) >= args.drop_thr;
-          on = on && keep;
-          r = keep ? r * args.drop_scale : 0.0f;
-        }
-        bits |= (on ? 1u : 0u) << u;
-        a[u] = round_bf16(r);
-      }
-      J.mask_out[(int64_t)((n0 + c) >> 4) * J.rows_pad + j] = (uint16_t)bits;
-      store_row16(S1, kM, r, c, a);
-      store_col16(S2, NT, r, c, a);
-    }
+    uint16_t* mask_out = J.mask_out + j + (int64_t)(n0 >> 4) * J.rows_pad;
+    const bool drop = J.drop_h > 0;
+    fwd_cols(tmem + lane_addr, s_bias, cbeg, cw, S1, S2, NT, r, mask_out, J.rows_pad, drop, h1,
+             ((uint64_t)j << 20) | (uint64_t)n0, args.drop_thr, args.drop_scale);
   } else if (ok && J.epi == TE_DX) {
     for (int c = cbeg; c < cbeg + cw; c += 16) {
       uint32_t v[16];
@@ -275,8 +349,11 @@ __device__ __forceinline__ bool tr_tile(const TrArgs& args, int bid, uint8_t* sm
       const float sc = J.drop_h > 0 ? args.drop_scale : 1.0f;
 #pragma unroll
       for (int u = 0; u < 16; ++u) dz[u] = ((bits >> u) & 1u) ? __uint_as_float(v[u]) * sc : 0.0f;
-      if (J.out) store_row16(S1, kM, r, c, dz);
-      store_col16(S2, NT, r, c, dz);
+      uint32_t w[8];
+#pragma unroll
+      for (int h = 0; h < 8; ++h) w[h] = pack2(dz[2 * h], dz[2 * h + 1]);
+      if (J.out) store_row16p(S1, kM, r, c, w);
+      store_col16p(S2, NT, r, c, w);
       const float sb = col_reduce16(dz);
       if (lane < 16) red[q * 256 + c + lane] = sb;
     }
@@ -360,8 +437,11 @@ __device__ __forceinline__ bool tr_tile(const TrArgs& args, int bid, uint8_t* sm
           pw[u] = rd * round_bf16(pos ? z : 0.0f);
           dz[u] = pos ? rd * s_w[c + u] : 0.0f;
         }
-        if (J.out) store_row16(S1, kM, r, c, dz);
-        store_col16(S2, NT, r, c, dz);
+        uint32_t w[8];
+#pragma unroll
+        for (int h = 0; h < 8; ++h) w[h] = pack2(dz[2 * h], dz[2 * h + 1]);
+        if (J.out) store_row16p(S1, kM, r, c, w);
+        store_col16p(S2, NT, r, c, w);
         const float sw = col_reduce16(pw);
         if (lane < 16) red2[q * 256 + c + lane] = sw;
         const float sb = col_reduce16(dz);
@@ -390,7 +470,8 @@ __device__ __forceinline__ bool tr_tile(const TrArgs& args, int bid, uint8_t* sm
       for (int h = 0; h < kM / 64; ++h)
         bulk_s2g(J.outT + ((int64_t)(m0 / 64 + h) * J.rT + n0) * 128, S2 + (size_t)h * NT * 128,
                  (uint32_t)NT * 128);
-      bulk_commit_wait_all();  // before the stages are reused or the CTA exits
+      if (drain) bulk_commit_wait_all();
+      else bulk_commit_wait_read();  // before the stages are reused or the CTA exits
     }
   }
   tc_fence_before();
@@ -415,16 +496,25 @@ __global__ void __launch_bounds__(kT, 1) k_tr_gemm(const __grid_constant__ TrArg
     tmem_alloc(tmem_holder, tcols);
     tmem_relinquish();
   }
-  // operands and side inputs come from the previous kernels of the stream
+  // The next product may start now: its CTAs take SMs this grid leaves idle
+  // and run their own prologue while this one works.  Every kernel of the
+  // step after the gather starts only after the gather has passed its wait
+  // (it lets its successor in at its end), so after the previous step's
+  // optimiser has completed: the weight images and the master read before
+  // the wait below are final.
+  pdl_trigger();
+  tr_tile_pre(args, (int)blockIdx.x, smem);
+  // the activation and gradient operands come from the previous kernels of the
+  // stream: their copies start as soon as the wait returns
   pdl_wait();
+  if (threadIdx.x == 0) tr_tile_copies(args, (int)blockIdx.x, smem);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_holder;
-  tr_tile(args, (int)blockIdx.x, smem, tmem, 0);
-  // the next kernel may start once every CTA is here (a waiting CTA of it
-  // holds a whole SM, so it is not let in earlier)
-  pdl_trigger();
+  // image stores may still be in flight when the CTA exits: the grid's
+  // completion makes them visible to the next kernel
+  tr_tile(args, (int)blockIdx.x, smem, tmem, 0, false, true);
   if (threadIdx.x < 32) tmem_dealloc(tmem, tcols);
 }
 
@@ -470,9 +560,12 @@ __device__ __forceinline__ void tr_gather_items(const GatherArgs& g, int64_t fir
     st->train_abort = 1;  // the optimiser of this step leaves every parameter as it is
   }
   if (lead) set_adam_bc(st);
-  const int64_t total = (int64_t)rows_pad * (d_pad / 8);
+  const int total = rows_pad * (d_pad / 8);  // at most 2^31 / 16 rows of 128 columns
+  // rows of a multiple of four columns are read as 16-byte vectors
+  const bool vec = (d & 3) == 0;
   for (int64_t e = first; e < total; e += stride) {
-    const int j = (int)(e % rows_pad), c0 = (int)(e / rows_pad) * 8;
+    const int ei = (int)e;
+    const int j = ei % rows_pad, c0 = (ei / rows_pad) * 8;
     float v[8];
 #pragma unroll
     for (int u = 0; u < 8; ++u) v[u] = 0.0f;
@@ -492,9 +585,24 @@ __device__ __forceinline__ void tr_gather_items(const GatherArgs& g, int64_t fir
       }
       slot = union_row(slot, nF, replay_base);
       const float* row = ring_x + slot * d;
+      if (vec && c0 + 8 <= d) {
+        float x[8], mu[8], sd[8];
 #pragma unroll
-      for (int u = 0; u < 8; ++u)
-        if (c0 + u < d) v[u] = round_bf16(zscore(__ldg(row + c0 + u), __ldg(mean + c0 + u), __ldg(stdv + c0 + u)));
+        for (int h = 0; h < 2; ++h) {
+          const float4 xv = __ldg(reinterpret_cast<const float4*>(row + c0) + h);
+          const float4 mv = __ldg(reinterpret_cast<const float4*>(mean + c0) + h);
+          const float4 sv = __ldg(reinterpret_cast<const float4*>(stdv + c0) + h);
+          x[4 * h] = xv.x, x[4 * h + 1] = xv.y, x[4 * h + 2] = xv.z, x[4 * h + 3] = xv.w;
+          mu[4 * h] = mv.x, mu[4 * h + 1] = mv.y, mu[4 * h + 2] = mv.z, mu[4 * h + 3] = mv.w;
+          sd[4 * h] = sv.x, sd[4 * h + 1] = sv.y, sd[4 * h + 2] = sv.z, sd[4 * h + 3] = sv.w;
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) v[u] = round_bf16(zscore(x[u], mu[u], sd[u]));
+      } else {
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          if (c0 + u < d) v[u] = round_bf16(zscore(__ldg(row + c0 + u), __ldg(mean + c0 + u), __ldg(stdv + c0 + u)));
+      }
       if (c0 == 0) y[j] = ring_y[slot];
     } else if (j < B && c0 == 0) {
       y[j] = 0.0f;
@@ -518,16 +626,16 @@ __global__ void k_tr_gather(const __grid_constant__ GatherArgs g) {
   pdl_trigger();
 }
 
-// sum_{s < n} src[s * stride], added in order, eight loads in flight.
+// sum_{s < n} src[s * stride], added in order, sixteen loads in flight.
 __device__ __forceinline__ float ordered_sum(const float* __restrict__ src, int n, int64_t stride) {
   float g = 0.0f;
   int s = 0;
-  for (; s + 8 <= n; s += 8) {
-    float v[8];
+  for (; s + 16 <= n; s += 16) {
+    float v[16];
 #pragma unroll
-    for (int u = 0; u < 8; ++u) v[u] = __ldg(src + (int64_t)(s + u) * stride);
+    for (int u = 0; u < 16; ++u) v[u] = __ldg(src + (int64_t)(s + u) * stride);
 #pragma unroll
-    for (int u = 0; u < 8; ++u) g += v[u];
+    for (int u = 0; u < 16; ++u) g += v[u];
   }
   for (; s < n; ++s) g += __ldg(src + (int64_t)s * stride);
   return g;
@@ -557,76 +665,98 @@ struct OptArgs {
   const float* partLoss;
   int B;
   float* loss_out;
+  // one-pass launch: block b holds 256 parameters of layer l, blk0[l] <= b <
+  // blk0[l + 1], from the layer's first parameter on (opt_blocks)
+  int blk0[LS_MAX_LAYERS + 1];
 };
 
 // Gradient of every parameter as an ordered sum of its partials, the
 // optimiser update of the fp32 master, and the bf16 images of the updated
 // hidden-layer weights, for parameters [first, n) with stride `stride`.
-__device__ __forceinline__ void tr_opt_items(const OptArgs& a, int64_t first, int64_t stride) {
-  // a step whose gather found no record or a bad slot changes nothing (the
-  // images already hold the unchanged weights)
-  if (a.mode != 0 && a.st->train_abort) return;
-  const float bc1 = a.st->adam_bc[0], bc2 = a.st->adam_bc[1];  // set by the gather kernel
+// Gradient (ordered sum of its partials), optimiser update and bf16 image
+// writes of parameter e of layer l.  A step whose gather found no record or a
+// bad slot (`aborted`) changes nothing: the images already hold the unchanged
+// weights.
+__device__ __forceinline__ void tr_opt_one(const OptArgs& a, int l, int64_t e, bool aborted, float bc1, float bc2) {
   const MlpDesc& m = a.m;
-  const int nl = m.n_layers;
-  for (int64_t e = first; e < a.n; e += stride) {
-    int l = 0;
-    while (l + 1 < nl && e >= m.woff[l + 1]) ++l;
-    const int out = m.w[l + 1], in = m.w[l];
-    const OptLayer& P = a.L[l];
-    const bool is_w = e < m.boff[l];
-    int o = 0, i = 0;
-    float p = a.p[e];
-    if (a.mode != 0) {
-      float g = 0.0f;
-      if (l + 1 < nl) {
-        if (is_w) {
-          const int64_t u = e - m.woff[l];
-          o = (int)(u / in);
-          i = (int)(u - (int64_t)o * in);
-          g = ordered_sum(P.partW + (int64_t)o * P.ld + i, P.S, (int64_t)out * P.ld);
-        } else {
-          o = (int)(e - m.boff[l]);
-          g = ordered_sum(P.partB + o, a.T, out);
-        }
-      } else {
-        if (is_w) {
-          i = (int)(e - m.woff[l]);
-          g = ordered_sum(P.partW + i, a.T, P.ld);
-        } else {
-          g = ordered_sum(P.partB, a.T, 1);
-        }
-      }
-      if (a.mode == 1) {
-        p = p - a.lr * g;
-      } else {
-        const float me = 0.9f * a.mo[e] + 0.1f * g;
-        const float ve = 0.999f * a.vo[e] + 0.001f * g * g;
-        a.mo[e] = me;
-        a.vo[e] = ve;
-        const float mh = me / bc1, vh = ve / bc2;
-        p = p - a.lr * mh / (sqrtf(vh) + 1e-8f);
-      }
-      a.p[e] = p;
-    } else if (l + 1 < nl && is_w) {
-      const int64_t u = e - m.woff[l];
-      o = (int)(u / in);
-      i = (int)(u - (int64_t)o * in);
+  const int out = m.w[l + 1], in = m.w[l];
+  const OptLayer& P = a.L[l];
+  const bool hidden = l + 1 < m.n_layers, is_w = e < m.boff[l];
+  int o = 0, i = 0;
+  if (is_w) {
+    const int u = (int)(e - m.woff[l]);  // index within one layer's weights
+    if (hidden) {
+      o = u / in;
+      i = u - o * in;
+    } else {
+      i = u;
     }
-    if (l + 1 < nl && is_w) {
-      const uint16_t b = bf16_bits(p);
-      *reinterpret_cast<uint16_t*>(P.imgW + sw128_offset(o, i, out)) = b;
-      *reinterpret_cast<uint16_t*>(P.imgWT + sw128_offset(i, o, P.in_pad)) = b;
+  } else {
+    o = (int)(e - m.boff[l]);
+  }
+  float p = a.p[e];
+  if (a.mode != 0) {
+    // the moments do not depend on the gradient: their loads overlap the partials'
+    float mo = 0.0f, vo = 0.0f;
+    if (a.mode == 2) {
+      mo = a.mo[e];
+      vo = a.vo[e];
     }
+    float g;
+    if (hidden)
+      g = is_w ? ordered_sum(P.partW + (int64_t)o * P.ld + i, P.S, (int64_t)out * P.ld)
+               : ordered_sum(P.partB + o, a.T, out);
+    else
+      g = is_w ? ordered_sum(P.partW + i, a.T, P.ld) : ordered_sum(P.partB, a.T, 1);
+    if (aborted) return;
+    if (a.mode == 1) {
+      p = p - a.lr * g;
+    } else {
+      const float me = 0.9f * mo + 0.1f * g;
+      const float ve = 0.999f * vo + 0.001f * g * g;
+      a.mo[e] = me;
+      a.vo[e] = ve;
+      const float mh = me / bc1, vh = ve / bc2;
+      p = p - a.lr * mh / (sqrtf(vh) + 1e-8f);
+    }
+    a.p[e] = p;
+  }
+  if (hidden && is_w) {
+    const uint16_t b = bf16_bits(p);
+    *reinterpret_cast<uint16_t*>(P.imgW + sw128_offset(o, i, out)) = b;
+    *reinterpret_cast<uint16_t*>(P.imgWT + sw128_offset(i, o, P.in_pad)) = b;
   }
 }
 
-// The minibatch loss (sum of the tile partials in order), by one thread.
-__device__ __forceinline__ void tr_loss(const OptArgs& a) {
+// Every parameter in [first, n) with stride `stride` (the persistent step).
+__device__ __forceinline__ void tr_opt_items(const OptArgs& a, int64_t first, int64_t stride) {
+  const MlpDesc& m = a.m;
+  const int nl = m.n_layers;
+  const bool aborted = a.mode != 0 && a.st->train_abort != 0;
+  const float bc1 = a.st->adam_bc[0], bc2 = a.st->adam_bc[1];  // set by the gather kernel
+  for (int64_t e = first; e < a.n; e += stride) {
+    // the layer of parameter e: layer starts increase, so count those at or before e
+    int l = 0;
+#pragma unroll
+    for (int k = 1; k < LS_MAX_LAYERS; ++k) l += (k < nl && e >= m.woff[k]) ? 1 : 0;
+    tr_opt_one(a, l, e, aborted, bc1, bc2);
+  }
+}
+
+// The minibatch loss (sum of the tile partials in order), by one warp: the
+// lanes load 32 partials at once, every lane adds them in tile order, lane 0
+// writes the result.
+__device__ __forceinline__ void tr_loss_warp(const OptArgs& a) {
   if (a.mode != 0 && a.loss_out) {
+    const int lane = threadIdx.x & 31;
+    const bool abort = a.st->train_abort != 0;
     float s = 0.0f;
-    for (int tt = 0; tt < a.T; ++tt) s += a.partLoss[tt];
-    *a.loss_out = a.st->train_abort ? __int_as_float(0x7fc00000) : s / (float)a.B;
+    for (int t0 = 0; t0 < a.T; t0 += 32) {
+      const float v = t0 + lane < a.T ? a.partLoss[t0 + lane] : 0.0f;
+      const int n = min(32, a.T - t0);
+      for (int k = 0; k < n; ++k) s += __shfl_sync(0xffffffffu, v, k);
+    }
+    if (lane == 0) *a.loss_out = abort ? __int_as_float(0x7fc00000) : s / (float)a.B;
   }
 }
 
@@ -635,8 +765,17 @@ __global__ void __launch_bounds__(256) k_tr_opt(const __grid_constant__ OptArgs 
   pdl_trigger();
   const int64_t t = a.st->step + 1;
   const bool aborted = a.mode != 0 && a.st->train_abort != 0;
-  tr_opt_items(a, blockIdx.x * (int64_t)blockDim.x + threadIdx.x, (int64_t)gridDim.x * blockDim.x);
-  if (blockIdx.x == 0 && threadIdx.x == 0) tr_loss(a);
+  const float bc1 = a.st->adam_bc[0], bc2 = a.st->adam_bc[1];  // set by the gather kernel
+  {
+    // this block's layer and parameters (one pass: a parameter per thread)
+    const int nl = a.m.n_layers;
+    int l = 0;
+#pragma unroll
+    for (int k = 1; k < LS_MAX_LAYERS; ++k) l += (k < nl && (int)blockIdx.x >= a.blk0[k]) ? 1 : 0;
+    const int64_t e = a.m.woff[l] + (int64_t)((int)blockIdx.x - a.blk0[l]) * 256 + threadIdx.x;
+    if (e < a.m.boff[l] + a.m.w[l + 1]) tr_opt_one(a, l, e, aborted, bc1, bc2);
+  }
+  if (blockIdx.x == 0 && threadIdx.x < 32) tr_loss_warp(a);
   // the last block, once every block has read the counter and the flag
   if (a.mode != 0 && last_block(&a.st->done[DONE_OPT]) && threadIdx.x == 0) {
     if (!aborted) advance_step(a.st, t);
@@ -727,7 +866,8 @@ __global__ void __launch_bounds__(kT, 1) k_tr_step(const __grid_constant__ StepA
   for (int ph = 0; go && ph < a.n_ph; ++ph) {
     const TrArgs& P = a.ph[ph];
     for (int b = blockIdx.x; b < P.n_cta; b += gridDim.x) {
-      if (!tr_tile(P, b, smem, tmem, par)) {
+      tr_tile_pre(P, b, smem);
+      if (!tr_tile(P, b, smem, tmem, par, true, false)) {
         if (tid == 0) atomicExch(a.bar + 1, 1u);
         go = false;
         break;
@@ -738,9 +878,10 @@ __global__ void __launch_bounds__(kT, 1) k_tr_step(const __grid_constant__ StepA
   }
   if (go) {
     tr_opt_items(a.opt, first, stride);
-    if (tr_grid_sync(a.bar, ++arrivals * gridDim.x, err) && blockIdx.x == 0 && tid == 0) {
-      tr_loss(a.opt);
-      if (a.opt.mode != 0) {
+    if (tr_grid_sync(a.bar, ++arrivals * gridDim.x, err) && blockIdx.x == 0 && tid < 32) {
+      tr_loss_warp(a.opt);
+      __syncwarp();  // every lane has read the abort flag before lane 0 clears it
+      if (tid == 0 && a.opt.mode != 0) {
         if (!a.opt.st->train_abort) advance_step(a.opt.st, a.opt.st->step + 1);
         a.opt.st->train_abort = 0;
       }
@@ -872,6 +1013,19 @@ void train_fast_bind(const MlpDesc& m, TrainFast& f, uint8_t* base, float* parts
   f.partLoss = q;
 }
 
+// Blocks of the one-pass optimiser launch: 256 parameters each, within one
+// layer.  Returns the grid size.
+int opt_blocks(const MlpDesc& m, OptArgs& a) {
+  int b = 0;
+  for (int l = 0; l < m.n_layers; ++l) {
+    a.blk0[l] = b;
+    const int64_t n_l = m.boff[l] + m.w[l + 1] - m.woff[l];
+    b += (int)((n_l + 255) / 256);
+  }
+  for (int l = m.n_layers; l <= LS_MAX_LAYERS; ++l) a.blk0[l] = b;
+  return b;
+}
+
 // bf16 images of the master's hidden-layer weights (after ls_set_params).
 cudaError_t train_fast_images(Ctx& c, cudaStream_t s) {
   const MlpDesc& m = c.mlp;
@@ -887,7 +1041,7 @@ cudaError_t train_fast_images(Ctx& c, cudaStream_t s) {
   a.mode = 0;
   a.p = c.master;
   a.st = c.st;
-  const int grid = (int)std::min<int64_t>((c.n_params + 255) / 256, (int64_t)c.sms * 4);
+  const int grid = opt_blocks(m, a);
   k_tr_opt<<<grid, 256, 0, s>>>(a);
   return cudaGetLastError();
 }
@@ -1077,7 +1231,7 @@ cudaError_t run_train_fast(Ctx& c, int B, const int32_t* idx, int opt, float lr,
     });
   }
   return traced(c, TR_OPT, 1, s, [&] {
-    const int grid = (int)std::min<int64_t>((c.n_params + 255) / 256, (int64_t)c.sms * 4);
+    const int grid = opt_blocks(m, a);
     return launch_chained(k_tr_opt, dim3(grid), dim3(256), 0, s, 1, a);
   });
 }

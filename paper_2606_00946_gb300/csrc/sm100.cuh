@@ -90,6 +90,14 @@ __device__ __forceinline__ void bulk_commit_wait_all() {
   asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
 }
 
+// Waits until the committed bulk stores have read their shared-memory sources
+// (the writes to global memory may still be in flight: they are visible to
+// later kernels once this grid has completed, not to other CTAs of it).
+__device__ __forceinline__ void bulk_commit_wait_read() {
+  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+  asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
+
 __device__ __forceinline__ void fence_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
