@@ -1095,8 +1095,10 @@ cudaError_t run_train_fast(Ctx& c, int B, const int32_t* idx, int opt, float lr,
     J.epi = last ? TE_FWD_OUT : TE_FWD;
     J.m_tiles = T;
     // the persistent launch has no clusters: the output layer's row dot
-    // products stay within one CTA (all columns of the tile)
-    J.n_split = (last && one) ? 1 : n_split_for(m.w[l + 1]);
+    // products stay within one CTA (all columns of the tile).  A hidden
+    // layer of 256 columns runs as four 64-column parts (128 CTAs for a
+    // batch of 4096: half the epilogue and image stores per SM)
+    J.n_split = (last && one) ? 1 : (!last && !one && m.w[l + 1] % 256 == 0) ? 4 : n_split_for(m.w[l + 1]);
     J.splits = 1;
     J.nchunks = f.in_pad[l] / 64;
     J.NT = m.w[l + 1] / J.n_split;
