@@ -352,38 +352,6 @@ __device__ __forceinline__ float4 lds_f4(const float* p) {
                : "r"(smem_u32(p)));
   return v;
 }
-__device__ __forceinline__ float2 lds_f2(const float* p) {
-  float2 v;
-  asm volatile("ld.shared.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(smem_u32(p)));
-  return v;
-}
-__device__ __forceinline__ uint4 lds_u4(const void* p) {
-  uint4 v;
-  asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-               : "r"(smem_u32(p)));
-  return v;
-}
-
-// The same with the layer's bias added first: acc += relu(bf16(v + b)) * w
-// over 16 columns, b the 16 fp32 biases and w the 16 bf16 weights of these
-// columns (both in shared memory).
-__device__ __forceinline__ uint64_t out_dot16_bias(const uint32_t (&v)[16], const float* b, const uint4* w,
-                                                   uint64_t acc) {
-  const uint4 w0 = lds_u4(w), w1 = lds_u4(w + 1);
-  const uint32_t wp[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const float4 bb = lds_f4(b + 4 * q);
-#pragma unroll
-    for (int u = 0; u < 2; ++u) {
-      const int j = 2 * q + u;
-      const uint64_t x = add_f32x2(((uint64_t)v[2 * j + 1] << 32) | v[2 * j], u ? f2pack(bb.z, bb.w) : f2pack(bb.x, bb.y));
-      const uint32_t h = relu_bf16x2(cvt_bf16x2(x));
-      acc = fma_f32x2(bf16x2_to_f32x2(h), bf16x2_to_f32x2(wp[j]), acc);
-    }
-  }
-  return acc;
-}
 
 // Pipelined variant for predictors with two hidden layers whose weights stay
 // resident (widths <= 256), one persistent CTA per SM over 128-row tiles of
@@ -1027,44 +995,57 @@ __global__ void __launch_bounds__(kThreadsWide, 1) k_score_wide(const __grid_con
   if (warp == 0) tmem_dealloc(tmem, 512);
 }
 
-// 16 loaded accumulator columns -> 8 packed bf16 words relu(bf16(D + b)) at o[OFF..)
+// 16 loaded accumulator columns (the bias already in them) -> 8 packed bf16
+// words relu(bf16(D)) at o[OFF..)
 template <int OFF>
-__device__ __forceinline__ void pack16_bias_relu(const uint32_t (&v)[16], const float* b, uint32_t (&o)[32]) {
+__device__ __forceinline__ void pack16_relu(const uint32_t (&v)[16], uint32_t (&o)[32]) {
 #pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    const float2 bb = lds_f2(b + 2 * j);
-    o[OFF + j] =
-        relu_bf16x2(cvt_bf16x2(add_f32x2(((uint64_t)v[2 * j + 1] << 32) | v[2 * j], f2pack(bb.x, bb.y))));
-  }
+  for (int j = 0; j < 8; ++j) o[OFF + j] = cvt_relu_bf16x2(((uint64_t)v[2 * j + 1] << 32) | v[2 * j]);
 }
 // 32 consecutive accumulator columns of the warp's lanes -> 16 packed words at
-// o[OFF..OFF + 16), b the 32 biases.
+// o[OFF..OFF + 16).
 template <int OFF>
-__device__ __forceinline__ void pack32_bias_relu(uint32_t taddr, const float* b, uint32_t (&o)[32]) {
+__device__ __forceinline__ void pack32_relu(uint32_t taddr, uint32_t (&o)[32]) {
   uint32_t va[16], vb[16];
   tmem_ld16(taddr, va);
   tmem_ld16(taddr + 16u, vb);
   tmem_wait_ld_regs(va);
-  pack16_bias_relu<OFF>(va, b, o);
+  pack16_relu<OFF>(va, o);
   tmem_wait_ld_regs(vb);
-  pack16_bias_relu<OFF + 8>(vb, b + 16, o);
+  pack16_relu<OFF + 8>(vb, o);
 }
 // 64 columns -> 32 packed words (o[0..32)); each 16-column load overlaps the
 // packing of the one before.  Every column has been read when this returns.
-__device__ __forceinline__ void pack64_bias_relu(uint32_t taddr, const float* b, uint32_t (&o)[32]) {
+__device__ __forceinline__ void pack64_relu(uint32_t taddr, uint32_t (&o)[32]) {
   uint32_t va[16], vb[16];
   tmem_ld16(taddr, va);
   tmem_wait_ld_regs(va);
   tmem_ld16(taddr + 16u, vb);
-  pack16_bias_relu<0>(va, b, o);
+  pack16_relu<0>(va, o);
   tmem_wait_ld_regs(vb);
   tmem_ld16(taddr + 32u, va);
-  pack16_bias_relu<8>(vb, b + 16, o);
+  pack16_relu<8>(vb, o);
   tmem_wait_ld_regs(va);
   tmem_ld16(taddr + 48u, vb);
-  pack16_bias_relu<16>(va, b + 32, o);
+  pack16_relu<16>(va, o);
   tmem_wait_ld_regs(vb);
-  pack16_bias_relu<24>(vb, b + 48, o);
+  pack16_relu<24>(vb, o);
+}
+// Output-layer partial of 16 columns whose accumulators hold the bias: the
+// fp32 pair accumulator gains bf16(relu(z_c)) * w_c, w the 16 output weights
+// (bf16 values held as fp32 in shared memory).
+__device__ __forceinline__ uint64_t out_dot16_wf(const uint32_t (&v)[16], const float* w, uint64_t acc) {
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const float4 ww = lds_f4(w + 4 * q);
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      const int j = 2 * q + u;
+      const uint32_t hh = cvt_relu_bf16x2(((uint64_t)v[2 * j + 1] << 32) | v[2 * j]);
+      acc = fma_f32x2(bf16x2_to_f32x2(hh), u ? f2pack(ww.z, ww.w) : f2pack(ww.x, ww.y), acc);
+    }
+  }
+  return acc;
 }
 
 // ---------------------------------------------------------------------------
@@ -1116,9 +1097,15 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
   const int S = p.pair_stages, Q = p.pair_q;
   uint8_t* X = smem;                                                  // [nk0] feature-tile K-blocks
   uint8_t* ring = X + (size_t)nk0 * kWideChunk;                       // [S][Q] half-slices
-  float* bias = reinterpret_cast<float*>(ring + (size_t)S * Q * kHalfSlice);  // [b1 (H1) | b2 (H2)]
-  uint16_t* sw3 = reinterpret_cast<uint16_t*>(bias + H1 + H2);        // [H2] bf16
-  float* part = reinterpret_cast<float*>(sw3 + H2);                   // [2 tiles][2 halves][128]
+  // Each job's accumulator starts from its bias: one K = 16 product of ONE
+  // [128 x 16] (ones in columns 0..2, every row group reading the same 8
+  // rows: stride 0) and this CTA's 128 rows of the job's bias operand (the
+  // three bf16 terms hi + mid + lo of each fp32 bias, whose sum is the bias
+  // exactly), so the epilogues read no bias.
+  uint8_t* ONE = ring + (size_t)S * Q * kHalfSlice;                   // 256 B, no swizzle
+  uint8_t* BIAS = ONE + 8 * 32;                                       // [J1 + J2][128 x 16], no swizzle
+  float* w3f = reinterpret_cast<float*>(BIAS + (size_t)(J1 + J2) * kTileM * 32);  // [H2] bf16 values
+  float* part = w3f + H2;                                             // [2 tiles][2 halves][128]
   uint64_t* full = reinterpret_cast<uint64_t*>(part + 4 * kTileM);    // [S]
   uint64_t* empty = full + S;                                         // [S]
   uint64_t* x_full = empty + S;
@@ -1156,9 +1143,33 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
     tmem_alloc_pair(tmem_holder, 512);
     tmem_relinquish_pair();
   }
-  for (int k = tid; k < H1 + H2; k += blockDim.x)
-    bias[k] = __ldg(params + (k < H1 ? a.boff[0] + k : a.boff[1] + k - H1));
-  for (int k = tid; k < H2; k += blockDim.x) sw3[k] = bf16_bits(__ldg(params + a.w_last_off + k));
+  for (int k = tid; k < H2; k += blockDim.x)
+    w3f[k] = __uint_as_float((uint32_t)bf16_bits(__ldg(params + a.w_last_off + k)) << 16);
+  for (int e = tid; e < 8 * 2; e += blockDim.x) {  // 16-byte chunks: row e / 2, K half e % 2
+    const uint4 q = (e & 1) ? make_uint4(0u, 0u, 0u, 0u) : make_uint4(0x3F803F80u, 0x3F80u, 0u, 0u);
+    *reinterpret_cast<uint4*>(ONE + nosw16_offset(e >> 1, 8 * (e & 1))) = q;
+  }
+  // job jb's operand row i: output column 256 jb' + 128 rank + i of its layer
+  // (this CTA supplies those 128 columns of the job's 256)
+  for (int e = tid; e < (J1 + J2) * kTileM * 2; e += blockDim.x) {
+    const int jb = e / (2 * kTileM), i = (e >> 1) % kTileM, l = jb < J1 ? 0 : 1;
+    const int col = (jb - (l ? J1 : 0)) * 256 + (int)rank * 128 + i;
+    uint4 q = make_uint4(0u, 0u, 0u, 0u);
+    if (!(e & 1)) {
+      const float b = __ldg(params + a.boff[l] + col);
+      const uint16_t hi = bf16_bits(b);
+      uint16_t mid = 0, lo = 0;
+      if (!isinf(b)) {  // b - hi and (b - hi) - mid are exact in fp32; lo holds the last 8 bits
+        const float r1 = b - __uint_as_float((uint32_t)hi << 16);
+        mid = bf16_bits(r1);
+        lo = bf16_bits(r1 - __uint_as_float((uint32_t)mid << 16));
+      }
+      q.x = (uint32_t)hi | ((uint32_t)mid << 16);
+      q.y = lo;
+    }
+    *reinterpret_cast<uint4*>(BIAS + (size_t)jb * kTileM * 32 + nosw16_offset(i, 8 * (e & 1))) = q;
+  }
+  fence_async_smem();  // both CTAs' bias operands are read by the tensor cores (async proxy)
   tc_fence_before();
   cluster_sync();  // barriers of both CTAs initialised before any remote arrival
   tc_fence_after();
@@ -1181,6 +1192,8 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
       uint32_t u1 = 0;         // D1 uses issued so far
       const uint64_t ring_desc = sdesc_sw128(smem_u32(ring));
       const uint64_t x_desc = sdesc_sw128(smem_u32(X));
+      const uint64_t one_desc = sdesc_nosw(smem_u32(ONE), 128, 0);
+      const uint64_t bias_desc = sdesc_nosw(smem_u32(BIAS), 128, 256);
       for (int t = 0; t < my_pairs && ok; ++t) {
         if (!(ok = mbar_wait_cl_short(x_full, (uint32_t)(t & 1)))) break;
         tc_fence_after();
@@ -1194,6 +1207,7 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
             d = tmem + 256u;
           }
           const int nk = l2 ? nk1 : nk0;
+          umma_pair_bf16(d, one_desc, bias_desc + (uint64_t)(j * (kTileM * 32 / 16)), idesc, 0u);
           for (int kb = 0; kb < nk; ++kb) {
             if (j == J1 && (kb & 3) == 0) {  // K-blocks 4 i.. read layer-1 job i's activations
               if (!(ok = mbar_wait_cl_short(&h1_ready[kb >> 2], (uint32_t)(t & 1)))) break;
@@ -1208,11 +1222,11 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
             if (l2) {
               const uint32_t a0 = tmem + (uint32_t)(32 * kb);
 #pragma unroll
-              for (int k = 0; k < 4; ++k) umma_pair_bf16_ts(d, a0 + 8u * k, bd + 2u * k, idesc, (kb | k) ? 1u : 0u);
+              for (int k = 0; k < 4; ++k) umma_pair_bf16_ts(d, a0 + 8u * k, bd + 2u * k, idesc, 1u);
             } else {
               const uint64_t xd = x_desc + (uint64_t)(kb * (kWideChunk / 16));
 #pragma unroll
-              for (int k = 0; k < 4; ++k) umma_pair_bf16(d, xd + 2u * k, bd + 2u * k, idesc, (kb | k) ? 1u : 0u);
+              for (int k = 0; k < 4; ++k) umma_pair_bf16(d, xd + 2u * k, bd + 2u * k, idesc, 1u);
             }
             if (++part_i == Q) {  // the stage is free in both CTAs once these products complete
               umma_pair_commit_both(&empty[st]);
@@ -1314,7 +1328,6 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
           // latches the error for the pair
           if (lane == 0) *abort_flag = 1;
         }
-        const float* b = bias + 256 * j + 128 * h;
         uint32_t pa[32], pb[32];
         if (j == 0) {
           // D0 is H1's own columns (packed column c holds features 2c, 2c + 1).
@@ -1325,27 +1338,27 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
           if (h == 0) {
             if (go) {
               tc_fence_after();
-              pack64_bias_relu(d0 + 64u, b + 64, pb);  // features 64..127 -> columns 32..63
+              pack64_relu(d0 + 64u, pb);  // features 64..127 -> columns 32..63
             }
             tc_fence_before();
             named_bar_arrive(2, kPairEpi * 32);
             if (go) {
-              pack32_bias_relu<16>(d0 + 32u, b + 32, pa);  // features 32..63 -> columns 16..31
+              pack32_relu<16>(d0 + 32u, pa);  // features 32..63 -> columns 16..31
               tmem_st32(d0 + 32u, pb);                     // columns 32..63 are consumed now
-              pack32_bias_relu<0>(d0, b, pa);              // features 0..31 -> columns 0..15
+              pack32_relu<0>(d0, pa);         // features 0..31 -> columns 0..15
               tmem_st32(d0, pa);
               tmem_wait_st();
             }
           } else {
             if (go) {
               tc_fence_after();
-              pack64_bias_relu(d0 + 128u, b, pa);  // features 128..191 -> columns 64..95
+              pack64_relu(d0 + 128u, pa);  // features 128..191 -> columns 64..95
             }
             named_bar_sync(2, kPairEpi * 32);
             tc_fence_after();
             if (go) {
               tmem_st32(d0 + 64u, pa);
-              pack64_bias_relu(d0 + 192u, b + 64, pb);  // features 192..255 -> columns 96..127
+              pack64_relu(d0 + 192u, pb);  // features 192..255 -> columns 96..127
             }
             if (J1 > 1) {  // columns 128..255 read: layer-1 job 1 may write there
               tc_fence_before();
@@ -1367,9 +1380,9 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
           }
           if (go) {
             tc_fence_after();
-            pack64_bias_relu(src, b, pa);
+            pack64_relu(src, pa);
             tmem_st32(dst, pa);
-            pack64_bias_relu(src + 64u, b + 64, pb);
+            pack64_relu(src + 64u, pb);
           }
           tc_fence_before();
           __syncwarp();
@@ -1396,8 +1409,7 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
           if (lane == 0) *abort_flag = 1;
         }
         const uint32_t src = tmem + lane_addr + 256u + 128u * (uint32_t)h;
-        const uint4* w = reinterpret_cast<const uint4*>(sw3 + 256 * n + 128 * h);
-        const float* b = bias + H1 + 256 * n + 128 * h;
+        const float* w = w3f + 256 * n + 128 * h;
         uint32_t va[16], vb[16];
         if (go) {
           tc_fence_after();
@@ -1406,21 +1418,21 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
           for (int i = 0; i < 6; i += 2) {
             tmem_wait_ld_regs(va);
             tmem_ld16(src + 16u * (i + 1), vb);
-            acc = out_dot16_bias(va, b + 16 * i, w + 2 * i, acc);
+            acc = out_dot16_wf(va, w + 16 * i, acc);
             tmem_wait_ld_regs(vb);
             tmem_ld16(src + 16u * (i + 2), va);
-            acc = out_dot16_bias(vb, b + 16 * (i + 1), w + 2 * (i + 1), acc);
+            acc = out_dot16_wf(vb, w + 16 * (i + 1), acc);
           }
           tmem_wait_ld_regs(va);
           tmem_ld16(src + 16u * 7, vb);
-          acc = out_dot16_bias(va, b + 16 * 6, w + 12, acc);
+          acc = out_dot16_wf(va, w + 16 * 6, acc);
           tmem_wait_ld_regs(vb);
         }
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive_at_relaxed(d1_empty, 0);  // all of D1 read: the next job may overwrite it
         ++u1;
-        if (go) acc = out_dot16_bias(vb, b + 16 * 7, w + 14, acc);
+        if (go) acc = out_dot16_wf(vb, w + 16 * 7, acc);
       }
       float* pt = part + (t & 1) * 2 * kTileM;
       pt[h * kTileM + row] = __uint_as_float((uint32_t)acc) + __uint_as_float((uint32_t)(acc >> 32));
@@ -1649,8 +1661,10 @@ bool plan_tc(const MlpDesc& m, TcPlan& p, bool allow_pair, bool allow_pipe) {
     const int H1 = p.out[0], H2 = p.out[1];
     const int nk0 = p.in_pad[0] / 64, nk1 = H1 / 64;
     const int per_tile = (H1 / 256) * nk0 + (H2 / 256) * nk1;
-    const int64_t fixed = 1024 + (int64_t)nk0 * kTileM * 128 + (int64_t)(H1 + H2) * 4 + (int64_t)H2 * 2 +
-                          4 * kTileM * 4 + 10 * 8 + 16;
+    // alignment, feature tile, ONE, bias operands, fp32 output weights, row
+    // partials, barriers, TMEM holder and abort flag
+    const int64_t fixed = 1024 + (int64_t)nk0 * kTileM * 128 + 8 * 32 + (int64_t)(H1 + H2) / 256 * kTileM * 32 +
+                          (int64_t)H2 * 4 + 4 * kTileM * 4 + 10 * 8 + 16;
     for (int Q = 6; Q >= 1 && !p.pair; --Q) {
       if (per_tile % Q) continue;
       const int64_t stages = (kMaxSmem - fixed) / ((int64_t)Q * kTileM * 128 + 16);

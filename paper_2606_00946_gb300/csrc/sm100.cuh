@@ -175,6 +175,14 @@ __device__ __forceinline__ uint32_t cvt_bf16x2(uint64_t v) {
       "f"(__uint_as_float((uint32_t)v)));
   return d;
 }
+// relu(bf16(hi, lo)) of a packed fp32 pair in one conversion: .relu makes a
+// negative result 0.
+__device__ __forceinline__ uint32_t cvt_relu_bf16x2(uint64_t v) {
+  uint32_t d;
+  asm("cvt.rn.relu.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(__uint_as_float((uint32_t)(v >> 32))),
+      "f"(__uint_as_float((uint32_t)v)));
+  return d;
+}
 __device__ __forceinline__ uint32_t relu_bf16x2(uint32_t v) {
   uint32_t d;
   asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(v), "r"(0u));
