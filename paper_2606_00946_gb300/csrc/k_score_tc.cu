@@ -335,20 +335,19 @@ __global__ void __launch_bounds__(kThreadsTc, 1) k_score_tc(const __grid_constan
 // bf16(relu(z_c)) * w_c for the even and odd columns (w_c bf16, 8 per uint4).
 __device__ __forceinline__ uint64_t out_dot16(const uint32_t (&v)[16], uint4 w0, uint4 w1, uint64_t acc) {
   const uint32_t wp[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
+  float lo = __uint_as_float((uint32_t)acc), hi = __uint_as_float((uint32_t)(acc >> 32));
 #pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    const uint32_t h = relu_bf16x2(cvt_bf16x2(((uint64_t)v[2 * j + 1] << 32) | v[2 * j]));
-    acc = fma_f32x2(bf16x2_to_f32x2(h), bf16x2_to_f32x2(wp[j]), acc);
-  }
-  return acc;
+  for (int j = 0; j < 8; ++j)
+    fma2_bf16_f32(cvt_relu_bf16x2(((uint64_t)v[2 * j + 1] << 32) | v[2 * j]), wp[j], lo, hi);
+  return f2pack(lo, hi);
 }
 
 // Shared-memory loads as ordered asm: they stay below the tensor-memory
 // loads and waits that precede them in the source, so the compiler does not
 // hoist a whole epilogue's weights and biases into registers at once.
-__device__ __forceinline__ float4 lds_f4(const float* p) {
-  float4 v;
-  asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+__device__ __forceinline__ uint4 lds_u4(const void* p) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
                : "r"(smem_u32(p)));
   return v;
 }
@@ -586,7 +585,7 @@ __global__ void __launch_bounds__(kThreadsPipe, 1) k_score_tc_pipe(const __grid_
           uint32_t pk[8];
 #pragma unroll
           for (int j = 0; j < 8; ++j)
-            pk[j] = relu_bf16x2(cvt_bf16x2(((uint64_t)v[g][2 * j + 1] << 32) | v[g][2 * j]));
+            pk[j] = cvt_relu_bf16x2(((uint64_t)v[g][2 * j + 1] << 32) | v[g][2 * j]);
           const int kcol = 32 * wk + 16 * g;  // column inside the K-block
           st_shared_v4(dst + sw128_offset(row, kcol, kTileM), pk[0], pk[1], pk[2], pk[3]);
           st_shared_v4(dst + sw128_offset(row, kcol + 8, kTileM), pk[4], pk[5], pk[6], pk[7]);
@@ -940,7 +939,7 @@ __global__ void __launch_bounds__(kThreadsWide, 1) k_score_wide(const __grid_con
           for (int i = 0; i < 4; ++i)
 #pragma unroll
             for (int j = 0; j < 8; ++j)
-              pk[8 * i + j] = relu_bf16x2(cvt_bf16x2(((uint64_t)v[i][2 * j + 1] << 32) | v[i][2 * j]));
+              pk[8 * i + j] = cvt_relu_bf16x2(((uint64_t)v[i][2 * j + 1] << 32) | v[i][2 * j]);
           tmem_st32(tmem + lane_addr + (uint32_t)(64 * c + 32 * h), pk);
           tmem_wait_st();
         }
@@ -1032,20 +1031,21 @@ __device__ __forceinline__ void pack64_relu(uint32_t taddr, uint32_t (&o)[32]) {
   pack16_relu<24>(vb, o);
 }
 // Output-layer partial of 16 columns whose accumulators hold the bias: the
-// fp32 pair accumulator gains bf16(relu(z_c)) * w_c, w the 16 output weights
-// (bf16 values held as fp32 in shared memory).
-__device__ __forceinline__ uint64_t out_dot16_wf(const uint32_t (&v)[16], const float* w, uint64_t acc) {
+// fp32 pair accumulator (even columns low, odd columns high) gains
+// bf16(relu(z_c)) * w_c, w the 16 bf16 output weights in shared memory.
+__device__ __forceinline__ uint64_t out_dot16_wb(const uint32_t (&v)[16], const uint16_t* w, uint64_t acc) {
+  float lo = __uint_as_float((uint32_t)acc), hi = __uint_as_float((uint32_t)(acc >> 32));
 #pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const float4 ww = lds_f4(w + 4 * q);
+  for (int q = 0; q < 2; ++q) {
+    const uint4 ww = lds_u4(w + 8 * q);
+    const uint32_t wp[4] = {ww.x, ww.y, ww.z, ww.w};
 #pragma unroll
-    for (int u = 0; u < 2; ++u) {
-      const int j = 2 * q + u;
-      const uint32_t hh = cvt_relu_bf16x2(((uint64_t)v[2 * j + 1] << 32) | v[2 * j]);
-      acc = fma_f32x2(bf16x2_to_f32x2(hh), u ? f2pack(ww.z, ww.w) : f2pack(ww.x, ww.y), acc);
+    for (int u = 0; u < 4; ++u) {
+      const int j = 4 * q + u;
+      fma2_bf16_f32(cvt_relu_bf16x2(((uint64_t)v[2 * j + 1] << 32) | v[2 * j]), wp[u], lo, hi);
     }
   }
-  return acc;
+  return f2pack(lo, hi);
 }
 
 // ---------------------------------------------------------------------------
@@ -1104,8 +1104,8 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
   // exactly), so the epilogues read no bias.
   uint8_t* ONE = ring + (size_t)S * Q * kHalfSlice;                   // 256 B, no swizzle
   uint8_t* BIAS = ONE + 8 * 32;                                       // [J1 + J2][128 x 16], no swizzle
-  float* w3f = reinterpret_cast<float*>(BIAS + (size_t)(J1 + J2) * kTileM * 32);  // [H2] bf16 values
-  float* part = w3f + H2;                                             // [2 tiles][2 halves][128]
+  uint16_t* sw3 = reinterpret_cast<uint16_t*>(BIAS + (size_t)(J1 + J2) * kTileM * 32);  // [H2] bf16
+  float* part = reinterpret_cast<float*>(sw3 + H2);                   // [2 tiles][2 halves][128]
   uint64_t* full = reinterpret_cast<uint64_t*>(part + 4 * kTileM);    // [S]
   uint64_t* empty = full + S;                                         // [S]
   uint64_t* x_full = empty + S;
@@ -1143,8 +1143,7 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
     tmem_alloc_pair(tmem_holder, 512);
     tmem_relinquish_pair();
   }
-  for (int k = tid; k < H2; k += blockDim.x)
-    w3f[k] = __uint_as_float((uint32_t)bf16_bits(__ldg(params + a.w_last_off + k)) << 16);
+  for (int k = tid; k < H2; k += blockDim.x) sw3[k] = bf16_bits(__ldg(params + a.w_last_off + k));
   for (int e = tid; e < 8 * 2; e += blockDim.x) {  // 16-byte chunks: row e / 2, K half e % 2
     const uint4 q = (e & 1) ? make_uint4(0u, 0u, 0u, 0u) : make_uint4(0x3F803F80u, 0x3F80u, 0u, 0u);
     *reinterpret_cast<uint4*>(ONE + nosw16_offset(e >> 1, 8 * (e & 1))) = q;
@@ -1409,7 +1408,7 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
           if (lane == 0) *abort_flag = 1;
         }
         const uint32_t src = tmem + lane_addr + 256u + 128u * (uint32_t)h;
-        const float* w = w3f + 256 * n + 128 * h;
+        const uint16_t* w = sw3 + 256 * n + 128 * h;
         uint32_t va[16], vb[16];
         if (go) {
           tc_fence_after();
@@ -1418,21 +1417,21 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
           for (int i = 0; i < 6; i += 2) {
             tmem_wait_ld_regs(va);
             tmem_ld16(src + 16u * (i + 1), vb);
-            acc = out_dot16_wf(va, w + 16 * i, acc);
+            acc = out_dot16_wb(va, w + 16 * i, acc);
             tmem_wait_ld_regs(vb);
             tmem_ld16(src + 16u * (i + 2), va);
-            acc = out_dot16_wf(vb, w + 16 * (i + 1), acc);
+            acc = out_dot16_wb(vb, w + 16 * (i + 1), acc);
           }
           tmem_wait_ld_regs(va);
           tmem_ld16(src + 16u * 7, vb);
-          acc = out_dot16_wf(va, w + 16 * 6, acc);
+          acc = out_dot16_wb(va, w + 16 * 6, acc);
           tmem_wait_ld_regs(vb);
         }
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive_at_relaxed(d1_empty, 0);  // all of D1 read: the next job may overwrite it
         ++u1;
-        if (go) acc = out_dot16_wf(vb, w + 16 * 7, acc);
+        if (go) acc = out_dot16_wb(vb, w + 16 * 7, acc);
       }
       float* pt = part + (t & 1) * 2 * kTileM;
       pt[h * kTileM + row] = __uint_as_float((uint32_t)acc) + __uint_as_float((uint32_t)(acc >> 32));
@@ -1661,10 +1660,10 @@ bool plan_tc(const MlpDesc& m, TcPlan& p, bool allow_pair, bool allow_pipe) {
     const int H1 = p.out[0], H2 = p.out[1];
     const int nk0 = p.in_pad[0] / 64, nk1 = H1 / 64;
     const int per_tile = (H1 / 256) * nk0 + (H2 / 256) * nk1;
-    // alignment, feature tile, ONE, bias operands, fp32 output weights, row
+    // alignment, feature tile, ONE, bias operands, bf16 output weights, row
     // partials, barriers, TMEM holder and abort flag
     const int64_t fixed = 1024 + (int64_t)nk0 * kTileM * 128 + 8 * 32 + (int64_t)(H1 + H2) / 256 * kTileM * 32 +
-                          (int64_t)H2 * 4 + 4 * kTileM * 4 + 10 * 8 + 16;
+                          (int64_t)H2 * 2 + 4 * kTileM * 4 + 10 * 8 + 16;
     for (int Q = 6; Q >= 1 && !p.pair; --Q) {
       if (per_tile % Q) continue;
       const int64_t stages = (kMaxSmem - fixed) / ((int64_t)Q * kTileM * 128 + 16);

@@ -183,6 +183,15 @@ __device__ __forceinline__ uint32_t cvt_relu_bf16x2(uint64_t v) {
       "f"(__uint_as_float((uint32_t)v)));
   return d;
 }
+// lo += a.lo * b.lo, hi += a.hi * b.hi for packed bf16 pairs a, b: fused
+// multiply-adds of bf16 inputs into fp32 (each the fp32 fma of the exact
+// fp32 values of its inputs).
+__device__ __forceinline__ void fma2_bf16_f32(uint32_t a, uint32_t b, float& lo, float& hi) {
+  asm("{\n .reg .b16 al, ah, bl, bh;\n mov.b32 {al, ah}, %2;\n mov.b32 {bl, bh}, %3;\n"
+      " fma.rn.f32.bf16 %0, al, bl, %0;\n fma.rn.f32.bf16 %1, ah, bh, %1;\n}"
+      : "+f"(lo), "+f"(hi)
+      : "r"(a), "r"(b));
+}
 __device__ __forceinline__ uint32_t relu_bf16x2(uint32_t v) {
   uint32_t d;
   asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(v), "r"(0u));
