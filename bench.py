@@ -727,7 +727,14 @@ def kernel_rooflines(trace, n_calls, costs, cfg, R, N, Bt, peaks, peak_src, work
         if k in ("prefix_index", "prefix_match"):
             alg, peak, unit, bound = costs["prefix_bytes"] / 1e9, peaks["hbm_gbs"], "GB/s", "hbm"
         elif k == "features":
-            alg = (R * N * (2 * d_pad + 4) + R * 8) / 1e9
+            # hit lengths and prompt offsets read; written: the whole bf16
+            # feature image (pipelined scorer), else each row's 16-byte pair
+            # chunk plus the instance and request template rows
+            if costs.get("tc_kernel") == 2:
+                written = R * N * 2 * d_pad
+            else:
+                written = R * N * 16 + (R + N) * 2 * d_pad
+            alg = (R * N * 4 + R * 8 + written) / 1e9
             peak, unit, bound = peaks["hbm_gbs"], "GB/s", "hbm"
         elif k in ("score_tc", "score_simt"):
             alg, peak, unit, bound = costs["score_flops"] / 1e12, peaks["bf16_tflops"], "TFLOP/s", "tensor"
@@ -781,7 +788,9 @@ def batch_costs(r, wl, cfg, dw):
     chk = r.route(dw.tok, dw.tok_off, dw.req_feats, cfg.n_inst)
     hits = chk["hits"].cpu().numpy()
     keys, ko = r.hash_blocks(dw.tok, dw.tok_off)
-    return route_costs(cfg, cfg.n_req, cfg.n_inst, hits, np.diff(wl.tok_off), keys.cpu().numpy(), ko.cpu().numpy())
+    costs = route_costs(cfg, cfg.n_req, cfg.n_inst, hits, np.diff(wl.tok_off), keys.cpu().numpy(), ko.cpu().numpy())
+    costs["tc_kernel"] = int(r.info().tc_kernel)
+    return costs
 
 
 def measure_route(name, L, H, W, dev, stream, peaks, peak_src, steps, warmup, ctx=None, small=False):

@@ -1455,30 +1455,41 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
 // and, for every (request, instance) pair, the 16-byte first chunk of its
 // feature row holding the six z-scored pair features (Sec. 4.1 Features;
 // Algorithm 4 Normalize) with zeros in columns 6 and 7.
+template <typename I>  // index type: 32-bit when every index fits, else 64-bit
 __global__ void k_norm_rows(const int64_t* __restrict__ tok_off, const int32_t* __restrict__ hits,
                             uint4* __restrict__ pairx, int n_inst, int d_inst, const float* __restrict__ inst,
                             int n_req, int d_req, const float* __restrict__ req, const float* __restrict__ mean,
                             const float* __restrict__ stdv, int d_pad, uint16_t* __restrict__ xin,
                             uint16_t* __restrict__ xrq) {
-  const int64_t ni = (int64_t)n_inst * d_pad, nr = (int64_t)n_req * d_pad;
-  const int64_t np = (int64_t)n_req * n_inst;
-  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < ni + nr + np;
-       e += (int64_t)gridDim.x * blockDim.x) {
-    if (e < ni) {
-      const int64_t i = e / d_pad;
-      const int k = (int)(e - i * d_pad) - kPair;
-      xin[e] = (k >= 0 && k < d_inst) ? bf16_bits(zscore(inst[i * d_inst + k], mean[kPair + k], stdv[kPair + k]))
-                                      : (uint16_t)0;
-    } else if (e < ni + nr) {
-      const int64_t f = e - ni;
-      const int64_t r = f / d_pad;
-      const int k = (int)(f - r * d_pad) - kPair - d_inst;
-      xrq[f] = (k >= 0 && k < d_req)
-                   ? bf16_bits(zscore(req[r * d_req + k], mean[kPair + d_inst + k], stdv[kPair + d_inst + k]))
-                   : (uint16_t)0;
+  // items: eight template columns of an instance row, of a request row, then
+  // one (request, instance) pair
+  const I G = (I)(d_pad / 8);
+  const I ni = (I)n_inst * G, nr = (I)n_req * G, np = (I)n_req * (I)n_inst;
+  for (I e = (I)blockIdx.x * blockDim.x + threadIdx.x; e < ni + nr + np; e += (I)gridDim.x * blockDim.x) {
+    if (e < ni + nr) {
+      const bool is_inst = e < ni;
+      const I f = is_inst ? e : e - ni;
+      const I row = f / G;
+      const int c0 = (int)(f - row * G) * 8;
+      const int off = is_inst ? kPair : kPair + d_inst, dk = is_inst ? d_inst : d_req;
+      const float* src = is_inst ? inst + (int64_t)row * d_inst : req + (int64_t)row * d_req;
+      uint32_t w[4];
+#pragma unroll
+      for (int u = 0; u < 8; u += 2) {
+        uint32_t pr = 0;
+#pragma unroll
+        for (int v = 0; v < 2; ++v) {
+          const int k = c0 + u + v - off;
+          const uint16_t b = (k >= 0 && k < dk) ? bf16_bits(zscore(src[k], mean[off + k], stdv[off + k])) : (uint16_t)0;
+          pr |= (uint32_t)b << (16 * v);
+        }
+        w[u / 2] = pr;
+      }
+      uint16_t* dst = (is_inst ? xin : xrq) + (int64_t)row * d_pad + c0;
+      *reinterpret_cast<uint4*>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
     } else {
-      const int64_t g = e - ni - nr;
-      const int64_t r = g / n_inst;
+      const I g = e - ni - nr;
+      const I r = g / (I)n_inst;
       const int64_t L = __ldg(tok_off + r + 1) - __ldg(tok_off + r);
       const int h = __ldg(hits + g);
       uint16_t f[kPair];
@@ -1770,8 +1781,12 @@ cudaError_t launch_norm_rows(const int64_t* tok_off, const int32_t* hits, uint4*
   const int64_t n = (int64_t)(n_inst + n_req) * d_pad + (int64_t)n_req * n_inst;
   if (n <= 0) return cudaSuccess;
   const int grid = (int)std::min<int64_t>((n + 255) / 256, (int64_t)sms * 8);
-  k_norm_rows<<<grid, 256, 0, s>>>(tok_off, hits, pairx, n_inst, d_inst, inst, n_req, d_req, req, mean, stdv, d_pad,
-                                   xin, xrq);
+  if (n + (int64_t)grid * 256 < (1LL << 31))
+    k_norm_rows<uint32_t><<<grid, 256, 0, s>>>(tok_off, hits, pairx, n_inst, d_inst, inst, n_req, d_req, req, mean,
+                                               stdv, d_pad, xin, xrq);
+  else
+    k_norm_rows<int64_t><<<grid, 256, 0, s>>>(tok_off, hits, pairx, n_inst, d_inst, inst, n_req, d_req, req, mean,
+                                              stdv, d_pad, xin, xrq);
   return cudaGetLastError();
 }
 
