@@ -10,8 +10,8 @@
 //           swizzle, one 16-byte chunk (8 columns) per thread.  For the pair
 //           scorer a job is 256 output rows, rows 128 r .. 128 r + 127 of it
 //           (an N-chunk, [128 x 64] per K-block: a 16 KB half-slice) belong to
-//           rank r, and rank r's half-slices of a tile (layer-1 jobs, then
-//           layer-2 jobs, K-blocks inner) are contiguous;
+//           rank r, and rank r's half-slices of a tile (the jobs of layer 1,
+//           then of each later layer, K-blocks inner) are contiguous;
 //   bounds  the staged feature bounds (Algorithm 4 [l, u]), lo [d] then hi [d].
 // The last block to finish bumps the version and then flips st->cur, so a
 // route that sees the new index sees a complete buffer.
@@ -36,9 +36,9 @@ struct PubArgs {
   int in_pad[LS_MAX_LAYERS], nc[LS_MAX_LAYERS];
   int64_t img_off[LS_MAX_LAYERS];
   int64_t grp_end[LS_MAX_LAYERS];        // cumulative 8-column groups of the image, per layer
-  int pair;                              // pair-scorer layout (two layers)
+  int pair;                              // pair-scorer layout
   int pair_slices;                       // 16 KB half-slices per rank per tile
-  int pair_l1;                           // layer-1 jobs of 256 columns
+  int pair_q0[LS_MAX_LAYERS];            // first half-slice of layer l's jobs within a tile
   DevState* st;
 };
 
@@ -114,7 +114,7 @@ __global__ void __launch_bounds__(256) k_publish(const __grid_constant__ PubArgs
       int64_t off;
       if (a.pair) {  // nc == 128: N-chunk nci is rank nci % 2's half of 256-column job nci / 2
         const int j = nci >> 1, r = nci & 1, nk = a.in_pad[l] / 64;
-        const int q = (l == 0 ? j * nk : a.pair_l1 * (a.in_pad[0] / 64) + j * nk) + (k0 >> 6);
+        const int q = a.pair_q0[l] + j * nk + (k0 >> 6);
         off = ((int64_t)r * a.pair_slices + q) * (128 * 128) + sm100::sw128_offset(orow, k0 & 63, 128);
       } else {
         off = a.img_off[l] + (int64_t)nci * (a.in_pad[l] / 64) * nc * 128 + sm100::sw128_offset(orow, k0, nc);
@@ -172,7 +172,11 @@ cudaError_t launch_publish(const MlpDesc& m, const TcPlan* tc, const float* mast
   if (tc && tc->pair) {
     a.pair = 1;
     a.pair_slices = tc->pair_slices;
-    a.pair_l1 = tc->out[0] / 256;
+    int q0 = 0;
+    for (int l = 0; l < tc->n_tc; ++l) {
+      a.pair_q0[l] = q0;
+      q0 += (tc->out[l] / 256) * (tc->in_pad[l] / 64);
+    }
   }
   a.st = st;
   const int64_t total = (a.n_params + 3) / 4 + a.n_wt + groups + a.n_bounds;

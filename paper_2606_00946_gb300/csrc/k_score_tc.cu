@@ -1083,6 +1083,7 @@ __device__ __forceinline__ void pair_stop(volatile int* abort_flag, uint32_t ran
   latch_error(err, LS_ERR_TIMEOUT);
 }
 
+template <bool kThree>  // three hidden layers of 256 (else two of multiples of 256)
 __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_constant__ TcArgs a) {
   const bool pb = a.sel && *a.sel == 1;
   const uint8_t* __restrict__ img = pb ? a.img1 : a.img0;
@@ -1090,9 +1091,17 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const TcPlan& p = a.p;
-  const int H1 = p.out[0], H2 = p.out[1];
-  const int J1 = H1 / 256, J2 = H2 / 256;
-  const int nk0 = p.in_pad[0] / 64, nk1 = H1 / 64;
+  // Jobs of a tile: J1 "compaction" jobs, whose results are rounded into
+  // packed bf16 TMEM columns 0..255 (H1), then J2 output jobs.  With three
+  // hidden layers (all of 256) the second layer is compaction job 1: its A
+  // operand is H1 (columns 0..127) and its result goes to columns 128..255
+  // (H2), which the single output job (the third layer) reads.
+  constexpr bool three = kThree;
+  const int H2 = three ? 256 : p.out[1];  // the last hidden layer
+  const int J1 = three ? 2 : p.out[0] / 256, J2 = three ? 1 : H2 / 256;
+  const int nk0 = p.in_pad[0] / 64, nk1 = three ? 4 : p.in_pad[1] / 64;
+  const uint32_t out_a = three ? 128u : 0u;  // TMEM column of the output jobs' A operand
+  const int nk_c1 = three ? 4 : nk0;  // K-blocks of compaction job 1
   const int per_tile = p.pair_slices;
   const int S = p.pair_stages, Q = p.pair_q;
   uint8_t* X = smem;                                                  // [nk0] feature-tile K-blocks
@@ -1151,8 +1160,9 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
   // job jb's operand row i: output column 256 jb' + 128 rank + i of its layer
   // (this CTA supplies those 128 columns of the job's 256)
   for (int e = tid; e < (J1 + J2) * kTileM * 2; e += blockDim.x) {
-    const int jb = e / (2 * kTileM), i = (e >> 1) % kTileM, l = jb < J1 ? 0 : 1;
-    const int col = (jb - (l ? J1 : 0)) * 256 + (int)rank * 128 + i;
+    const int jb = e / (2 * kTileM), i = (e >> 1) % kTileM;
+    const int l = three ? jb : (jb < J1 ? 0 : 1);
+    const int col = (three ? 0 : (jb - (l ? J1 : 0)) * 256) + (int)rank * 128 + i;
     uint4 q = make_uint4(0u, 0u, 0u, 0u);
     if (!(e & 1)) {
       const float b = __ldg(params + a.boff[l] + col);
@@ -1198,18 +1208,27 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
         tc_fence_after();
         for (int j = 0; j < J1 + J2 && ok; ++j) {
           const bool l2 = j >= J1;
-          if (j == J1) umma_pair_commit_both(x_empty);  // both feature tiles free once the layer-1 products are done
+          // A operand in TMEM: the output jobs and, with three layers, job 1
+          const bool a_tmem = l2 || (three && j == 1);
+          // both feature tiles are free once the products reading them are done
+          if (j == (three ? 1 : J1)) umma_pair_commit_both(x_empty);
           uint32_t d = tmem;  // D0: layer-1 job 0
           if (j > 0) {        // D1: its previous use has been read by both epilogues
             if (u1 >= 1 && !(ok = mbar_wait_cl_short(d1_empty, (u1 - 1) & 1u))) break;
             tc_fence_after();
             d = tmem + 256u;
           }
-          const int nk = l2 ? nk1 : nk0;
+          const int nk = l2 ? nk1 : j == 1 ? nk_c1 : nk0;
+          const uint32_t a_base = tmem + (l2 ? out_a : 0u);
+          // the compaction job whose activations K-block 0 (three layers) or
+          // each fourth K-block (two layers) of this job waits for, if any
+          const bool wait_h = three ? j >= 1 : j == J1;
           umma_pair_bf16(d, one_desc, bias_desc + (uint64_t)(j * (kTileM * 32 / 16)), idesc, 0u);
           for (int kb = 0; kb < nk; ++kb) {
-            if (j == J1 && (kb & 3) == 0) {  // K-blocks 4 i.. read layer-1 job i's activations
-              if (!(ok = mbar_wait_cl_short(&h1_ready[kb >> 2], (uint32_t)(t & 1)))) break;
+            // K-blocks 4 i.. of the output jobs read compaction job i's activations
+            // (three layers: job 1 reads job 0's, the output job job 1's)
+            if (wait_h && (three ? kb == 0 : (kb & 3) == 0)) {
+              if (!(ok = mbar_wait_cl_short(&h1_ready[three ? j - 1 : kb >> 2], (uint32_t)(t & 1)))) break;
               tc_fence_after();
             }
             if (part_i == 0) {  // a new stage: both CTAs' copies have landed
@@ -1218,8 +1237,8 @@ __global__ void __launch_bounds__(kThreadsPair, 1) k_score_pair(const __grid_con
               tc_fence_after();
             }
             const uint64_t bd = ring_desc + (uint64_t)((st * Q + part_i) * (kHalfSlice / 16));
-            if (l2) {
-              const uint32_t a0 = tmem + (uint32_t)(32 * kb);
+            if (a_tmem) {
+              const uint32_t a0 = a_base + (uint32_t)(32 * kb);
 #pragma unroll
               for (int k = 0; k < 4; ++k) umma_pair_bf16_ts(d, a0 + 8u * k, bd + 2u * k, idesc, 1u);
             } else {
@@ -1666,15 +1685,23 @@ bool plan_tc(const MlpDesc& m, TcPlan& p, bool allow_pair, bool allow_pipe) {
   // columns.  Each CTA of a pair streams its half of every [256 x 64] slice
   // (16 KB: the image's per-rank streams); a stage holds Q half-slices, Q the
   // largest divisor of the per-tile stream up to 6 that leaves two stages.
+  // (or three hidden layers of exactly 256: the second runs as a compaction
+  // job into the TMEM columns the first left free, the third is the output job)
   p.pair = 0;
-  if (allow_pair && !p.pipe && p.n_tc == 2 && p.out[0] % 256 == 0 && p.out[1] % 256 == 0 && p.d_pad <= 128) {
-    const int H1 = p.out[0], H2 = p.out[1];
-    const int nk0 = p.in_pad[0] / 64, nk1 = H1 / 64;
-    const int per_tile = (H1 / 256) * nk0 + (H2 / 256) * nk1;
+  const bool two = p.n_tc == 2 && p.out[0] % 256 == 0 && p.out[1] % 256 == 0;
+  const bool three = p.n_tc == 3 && p.out[0] == 256 && p.out[1] == 256 && p.out[2] == 256;
+  if (allow_pair && !p.pipe && (two || three) && p.d_pad <= 128) {
+    const int HL = p.out[p.n_tc - 1];
+    const int nk0 = p.in_pad[0] / 64;
+    int per_tile = 0, jobs = 0;
+    for (int l = 0; l < p.n_tc; ++l) {
+      per_tile += (p.out[l] / 256) * (p.in_pad[l] / 64);
+      jobs += p.out[l] / 256;
+    }
     // alignment, feature tile, ONE, bias operands, bf16 output weights, row
     // partials, barriers, TMEM holder and abort flag
-    const int64_t fixed = 1024 + (int64_t)nk0 * kTileM * 128 + 8 * 32 + (int64_t)(H1 + H2) / 256 * kTileM * 32 +
-                          (int64_t)H2 * 2 + 4 * kTileM * 4 + 10 * 8 + 16;
+    const int64_t fixed = 1024 + (int64_t)nk0 * kTileM * 128 + 8 * 32 + (int64_t)jobs * kTileM * 32 +
+                          (int64_t)HL * 2 + 4 * kTileM * 4 + 10 * 8 + 16;
     for (int Q = 6; Q >= 1 && !p.pair; --Q) {
       if (per_tile % Q) continue;
       const int64_t stages = (kMaxSmem - fixed) / ((int64_t)Q * kTileM * 128 + 16);
@@ -1687,7 +1714,7 @@ bool plan_tc(const MlpDesc& m, TcPlan& p, bool allow_pair, bool allow_pipe) {
     }
     if (p.pair) {
       int64_t woff = 0;
-      for (int l = 0; l < 2; ++l) {
+      for (int l = 0; l < p.n_tc; ++l) {
         p.nc[l] = 128;
         p.img_off[l] = woff;
         woff += (int64_t)p.out[l] * p.in_pad[l] * 2;
@@ -1818,7 +1845,8 @@ cudaError_t launch_feature_image(const int64_t* tok_off, const int32_t* hits, in
 
 int pair_max_clusters(const TcPlan& p) {
   if (!p.pair) return 0;
-  if (cudaFuncSetAttribute(k_score_pair, cudaFuncAttributeMaxDynamicSharedMemorySize, p.pair_smem) != cudaSuccess)
+  auto kern = p.n_tc == 3 ? k_score_pair<true> : k_score_pair<false>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, p.pair_smem) != cudaSuccess)
     return 0;
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
@@ -1835,7 +1863,7 @@ int pair_max_clusters(const TcPlan& p) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, k_score_pair, &cfg) != cudaSuccess) {
+  if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) {
     cudaGetLastError();
     return 0;
   }
@@ -1884,12 +1912,13 @@ cudaError_t launch_score_tc(const MlpDesc& m, const TcPlan& p, const Published* 
   } else if (p.pair) {
     // the image is in the pair layout, which no other scorer reads
     if (!scores) return cudaErrorInvalidValue;
-    cudaError_t e = cudaFuncSetAttribute(k_score_pair, cudaFuncAttributeMaxDynamicSharedMemorySize, p.pair_smem);
+    auto kern = p.n_tc == 3 ? k_score_pair<true> : k_score_pair<false>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, p.pair_smem);
     if (e != cudaSuccess) return e;
     const int tile_pairs = (a.n_tiles + 1) / 2;
     const int fit = p.pair_clusters > 0 ? p.pair_clusters : sms / 2;
     const int pairs = std::max(1, std::min(tile_pairs, fit));
-    return launch_chained(k_score_pair, dim3(2 * pairs), dim3(kThreadsPair), (size_t)p.pair_smem, s, 2, a);
+    return launch_chained(kern, dim3(2 * pairs), dim3(kThreadsPair), (size_t)p.pair_smem, s, 2, a);
   } else if (p.wide && scores) {
     cudaError_t e = cudaFuncSetAttribute(k_score_wide, cudaFuncAttributeMaxDynamicSharedMemorySize, p.wide_smem);
     if (e != cudaSuccess) return e;

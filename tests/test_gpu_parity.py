@@ -289,7 +289,9 @@ def test_pipelined_scorer_with_tiles_across_requests(n_inst):
     ((512, 512), 24, False, 96, "pair"), ((256, 512), 256, True, 48, "pair"), ((512, 512), 256, True, 48, "pair"),
     ((512, 512), 24, True, 100, "pair"), ((512, 256), 24, True, 5, "pair"), ((256, 256), 24, True, 100, "pair"),
     ((512, 128), 200, False, 48, "wide"), ((128, 512), 7, False, 96, "wide"), ((256, 128), 24, True, 100, "wide"),
-    ((512, 512), 24, True, 100, "wide"), ((256, 512), 256, True, 48, "wide")])
+    ((512, 512), 24, True, 100, "wide"), ((256, 512), 256, True, 48, "wide"),
+    ((256, 256, 256), 24, True, 100, "pair"), ((256, 256, 256), 64, False, 37, "pair"),
+    ((256, 256, 256), 7, True, 5, "pair"), ((256, 256, 256), 24, True, 100, "generic")])
 def test_wide_scorer_shapes(hidden, n_inst, wide_dims, n_req, kernel, monkeypatch):
     # the streamed-weight tensor-core scorers against the oracle: the pair
     # kernel (CTA pairs of 2-SM products, hidden widths multiples of 256) and
@@ -297,9 +299,11 @@ def test_wide_scorer_shapes(hidden, n_inst, wide_dims, n_req, kernel, monkeypatc
     # with LS_TC_PAIR=0): tiles across request boundaries, one to four
     # layer-1 jobs, 64- and 128-column feature tiles, an odd number of tiles
     # (19: the last pair's second tile is past the batch) and a batch of one
-    # tile
+    # tile; three hidden layers of 256 on the pair kernel (its second layer a
+    # compaction job reading the first's activations in tensor memory) and on
+    # the generic one-tile kernel
     import dataclasses
-    if kernel == "wide":
+    if kernel in ("wide", "generic"):
         monkeypatch.setenv("LS_TC_PAIR", "0")
     base = W.CONFIGS["large" if wide_dims else "homogeneous"]
     cfg = dataclasses.replace(base, hidden=hidden, n_inst=n_inst, n_req=n_req, cache_blocks=1024, n_samples=0)
@@ -308,7 +312,7 @@ def test_wide_scorer_shapes(hidden, n_inst, wide_dims, n_req, kernel, monkeypatc
     dw = H.DeviceWorkload(wl)
     dw.load(r)
     assert r.info().scorer == L.LS_SCORER_TENSOR_CORES
-    assert r.info().tc_kernel == {"wide": L.LS_TC_WIDE, "pair": L.LS_TC_PAIR}[kernel]
+    assert r.info().tc_kernel == {"wide": L.LS_TC_WIDE, "pair": L.LS_TC_PAIR, "generic": L.LS_TC_GENERIC}[kernel]
     out = r.route(dw.tok, dw.tok_off, dw.req_feats, n_inst)
     ref = oracle.route(wl, bounds=True, threads=THREADS)
     assert np.array_equal(out["hits"].cpu().numpy(), ref["hits"])
