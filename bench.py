@@ -73,6 +73,9 @@ def parse():
                    help="only the replay-pool admission measurement (for kernel profiling)")
     p.add_argument("--guards-only", action="store_true",
                    help="only the guarded-route measurement (--steps routes; for kernel profiling)")
+    p.add_argument("--train-only", action="store_true",
+                   help="only Adam steps of the training configuration, alone (for kernel profiling: the first "
+                        "two timed steps are inside the profiler range)")
     p.add_argument("--route-only", default=None, choices=["tiny", "homogeneous", "heterogeneous", "large"],
                    help="only --steps routes of one configuration (for kernel profiling)")
     p.add_argument("--small", action="store_true",
@@ -376,6 +379,40 @@ def measure_training_config(L, H, W, dev, steps=1000):
             "roofline": {"step_us": 1e6 * t_roof, "samples_per_s": B_ / t_roof, "flops": flops, "bytes": bytes_,
                          "frac_alone": rate_alone / (B_ / t_roof),
                          "frac_beside_routes": steps * B_ / (ms / 1e3) / (B_ / t_roof)}}
+
+
+def measure_training_only(L, H, W, dev, steps, warmup):
+    """Adam steps of the training configuration alone on one stream: the
+    first two after `warmup` inside cudaProfilerStart/Stop (a target for
+    `ncu --profile-from-start off`), then `steps` back to back, timed."""
+    import torch
+    wl = W.generate("training")
+    cfg = wl.cfg
+    r = H.Router.for_config(cfg, ring_capacity=cfg.n_samples)
+    dw = H.DeviceWorkload(wl, device=dev)
+    dw.load(r)
+    r.log(torch.from_numpy(wl.samples_x).to(dev), torch.from_numpy(wl.samples_y).to(dev))
+    loss = torch.zeros(1, device=dev)
+    s = torch.cuda.current_stream(dev)
+
+    def step(k=0):
+        r.train(cfg.train_batch, None, opt="adam", lr=cfg.train_lr, loss_out=loss, stream=s)
+
+    for _ in range(max(warmup, 3)):
+        step()
+    torch.cuda.synchronize()
+    torch.cuda.cudart().cudaProfilerStart()
+    step()
+    step()
+    torch.cuda.synchronize()
+    torch.cuda.cudart().cudaProfilerStop()
+    times = timed_back_to_back(step, max(steps, 10), s)
+    ms = float(np.mean(times))
+    out = {"config": "training: ring 2^20 x 128 fp32, Adam lr 3e-4, batch 4096, 128-256-256-256-1 bf16",
+           "train_step_alone_ms": ms, "train_samples_per_s_alone": cfg.train_batch / (ms / 1e3),
+           "loss": float(loss.item()), "status": int(r.sync())}
+    r.close()
+    return out
 
 
 def dist_setup(n_gpus):
@@ -1118,6 +1155,11 @@ def main():
                             small=args.small)
         if rank == 0:
             print(json.dumps({"route_only": args.route_only, **res}))
+        return 0
+    if args.train_only:
+        res = measure_training_only(L, H, W, dev, args.steps, args.warmup)
+        if rank == 0:
+            print(json.dumps({"train_only": True, **res}))
         return 0
     if args.paper_point_only or args.replay_only or args.guards_only:
         wl, cfg, r, dw = setup_config("homogeneous", H, W, dev)[:4]
