@@ -143,11 +143,14 @@ typedef struct {
  * fixed by the predictor widths when the context is created):
  *   GENERIC    any bf16 predictor with hidden widths multiples of 64, <= 512;
  *   PIPELINED  two hidden layers <= 256 wide, weights resident in shared memory;
- *   PAIR       otherwise two hidden layers of multiples of 128 and a feature
- *              width <= 128: CTA pairs running 2-SM products, weights streamed;
- *   WIDE       the same shapes on one CTA per tile, where CTA pairs cannot be
- *              resident together, or when the environment variable LS_TC_PAIR
- *              is "0" at context creation. */
+ *   PAIR       otherwise two hidden layers of multiples of 256, or three of
+ *              exactly 256, and a feature width <= 128: CTA pairs running 2-SM
+ *              products, weights streamed;
+ *   WIDE       two hidden layers of multiples of 128 and a feature width
+ *              <= 128 on one CTA per tile, where PAIR does not apply or CTA
+ *              pairs cannot be resident together.
+ * The environment variables LS_TC_PAIR and LS_TC_PIPE set to "0" at context
+ * creation plan without the PAIR and the PIPELINED variant respectively. */
 typedef enum {
     LS_TC_NONE = 0,
     LS_TC_GENERIC = 1,
