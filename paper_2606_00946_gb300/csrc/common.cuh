@@ -93,7 +93,7 @@ struct DevState {
   int64_t admitted;         // evicted stream positions below this were considered for the replay pool
   int32_t train_abort;      // set by a training step's gather (empty buffer, bad slot): the step's
                             // optimiser changes nothing and clears it
-  int32_t pad_;
+  uint32_t walk_next;       // next request of the prefix walk in flight (0 between walks)
 };
 
 // Row of training-buffer index u (Sec. 4.3.2: a round trains on F u R): ring
@@ -116,7 +116,7 @@ __device__ __forceinline__ void advance_step(DevState* st, int64_t t) {
   st->beta_pow[1] *= 0.999;
 }
 enum { DONE_RING = 0, DONE_OPT = 1, DONE_PUB = 2, DONE_BOUNDS = 3 };
-enum { DONE_REPLAY = 4 };  // DevState::done has 6 entries
+enum { DONE_REPLAY = 4, DONE_WALK = 5 };  // DevState::done has 6 entries
 
 // Kernel-level tracing: when enabled, every launch is bracketed by CUDA events
 // recorded on the launching stream; ls_trace_read() sums the elapsed times.

@@ -16,7 +16,9 @@
 // length from one ballot; the lane that owns the instance keeps it and the
 // row is written once, coalesced, at the end.  The walk stops at the first
 // round after which no instance matches, so tokens past the longest hit plus
-// one round are never read.
+// one round are never read.  Walks differ in length by orders of magnitude,
+// so warps take requests from a shared counter (a warp that finishes a short
+// walk takes the next request) rather than a fixed share each.
 #include "blockhash.cuh"
 #include "sm100.cuh"
 
@@ -80,16 +82,19 @@ __global__ void __launch_bounds__(kNT, W <= 4 ? 8 : 1) k_prefix_index(int n_req,
   route_snapshot(st);
   const int lane = threadIdx.x & 31;
   const int64_t warps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  // G^(lane+1): the factor by which the state entering a round reaches this lane
-  uint64_t glane = 1;
-  {
-    uint64_t b = kG;
+  // G^(lane+1): the factor by which the state entering a round reaches lane
+  // `lane` (kept in shared memory: one load per round, no registers held)
+  __shared__ uint64_t s_glane[32];
+  if (threadIdx.x < 32) {
+    uint64_t g = 1, b = kG;
     for (unsigned e = (unsigned)lane + 1; e; e >>= 1) {
-      if (e & 1) glane *= b;
+      if (e & 1) g *= b;
       b *= b;
     }
+    s_glane[lane] = g;
   }
-  for (int64_t r = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; r < n_req; r += warps) {
+  __syncthreads();
+  for (int64_t r = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; r < n_req;) {
     const int64_t t0 = tok_off[r];
     const int64_t nb = (tok_off[r + 1] - t0) / kBlockTok;
     const int32_t* base = tok + t0;
@@ -121,7 +126,7 @@ __global__ void __launch_bounds__(kNT, W <= 4 ? 8 : 1) k_prefix_index(int n_req,
         const uint64_t o = __shfl_up_sync(kFull, B, off);
         if (lane >= off) B = gpow(off) * o + B;
       }
-      const uint64_t s = glane * state + B;
+      const uint64_t s = s_glane[lane] * state + B;
       const int last = (int)(nb - p < 32 ? nb - p : 32) - 1;
       state = __shfl_sync(kFull, s, last);
       uint64_t pa[W];
@@ -169,7 +174,17 @@ __global__ void __launch_bounds__(kNT, W <= 4 ? 8 : 1) k_prefix_index(int n_req,
         // instances matching every full block (or requests without a full block)
         if (i < n_inst) hrow[i] = ((alive[w] >> bit) & 1ull) ? (int32_t)nb : hreg[w][h];
       }
+    // the next request: from the counter (after each warp's first), else a fixed stride
+    if (st) {
+      uint32_t nx = 0;
+      if (lane == 0) nx = atomicAdd(&st->walk_next, 1u);
+      r = warps + (int64_t)__shfl_sync(kFull, nx, 0);
+    } else {
+      r += warps;
+    }
   }
+  // the counter starts at 0 for the next walk: reset by the last block to finish
+  if (st && last_block(&st->done[DONE_WALK]) && threadIdx.x == 0) st->walk_next = 0u;
   sm100::pdl_trigger();  // the next kernel may start once every CTA is here
 }
 
@@ -220,7 +235,6 @@ cudaError_t launch_prefix_index(int n_req, const int32_t* tok, const int64_t* to
                                 const uint64_t* gmask, int W, uint64_t gmask_slots, int n_inst, int32_t* hits,
                                 int sms, DevState* st, cudaStream_t s) {
   if (n_req <= 0) return cudaSuccess;
-  const int grid = std::max(1, std::min((n_req + kNT / 32 - 1) / (kNT / 32), sms * 16));  // one warp per request
   void (*k)(int, const int32_t*, const int64_t*, const uint64_t*, const uint64_t*, uint64_t, int, int32_t*,
             DevState*) = nullptr;
   switch (W) {
@@ -230,6 +244,19 @@ cudaError_t launch_prefix_index(int n_req, const int32_t* tok, const int64_t* to
     case 8: k = k_prefix_index<8>; break;
     default: return cudaErrorInvalidValue;
   }
+  // as many warps as are resident at once (they then take requests from the
+  // counter); with no state to keep the counter in, one warp per request
+  static int resident[9] = {};
+  if (!resident[W]) {
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k, kNT, 0) != cudaSuccess || per_sm < 1) {
+      cudaGetLastError();
+      per_sm = 1;
+    }
+    resident[W] = per_sm;
+  }
+  const int want = (n_req + kNT / 32 - 1) / (kNT / 32);
+  const int grid = std::max(1, std::min(want, st ? sms * resident[W] : sms * 16));
   return launch_chained(k, dim3(grid), dim3(kNT), 0, s, 1, n_req, tok, tok_off, gkeys, gmask, gmask_slots, n_inst,
                         hits, st);
 }
