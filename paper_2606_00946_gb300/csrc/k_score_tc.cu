@@ -1063,7 +1063,12 @@ __device__ __forceinline__ uint64_t out_dot16_wb(const uint32_t (&v)[16], const 
 // columns [0, H1 / 2); the accumulator D0 = columns 0..255 for layer-1 job 0,
 // compacted in place into H1 by its epilogue; D1 = columns 256..511 for
 // layer-1 job 1 and every layer-2 job, released by the epilogue as soon as it
-// has been read.  The epilogues add the biases.
+// has been read.  Each job's accumulator starts from its bias (one K = 16
+// product), and the epilogues convert with one ReLU-and-round instruction per
+// column pair: draining the single accumulator is the critical path.  With
+// three hidden layers of 256 (kThree) the second layer is compaction job 1,
+// its A operand H1 and its result packed into columns 128..255 (H2), which the
+// output job reads.
 // Warp roles in each CTA: 0 = MMA issuer (CTA 0) or stage relay (CTA 1), and
 // the TMEM allocation; 1 = producer of this CTA's half-slices; 2..7 = feature
 // tile builders; 8..15 = epilogue (lane quadrant warp % 4, column half
