@@ -23,6 +23,7 @@
 // Index reads bypass L1 (the CTA's own insertions must be visible to it).
 #include "blockhash.cuh"
 #include "common.cuh"
+#include "sm100.cuh"
 
 namespace ls {
 namespace {
@@ -145,6 +146,72 @@ __device__ __forceinline__ float seq_xget(const uint8_t* X, int64_t i, bool bf) 
 __device__ __forceinline__ void seq_xset(uint8_t* X, int64_t i, float v, bool bf) {
   if (bf) reinterpret_cast<uint16_t*>(X)[i] = (uint16_t)(__float_as_uint(round_bf16(v)) >> 16);
   else reinterpret_cast<float*>(X)[i] = v;
+}
+
+// One hidden or output layer of the predictor in bf16, weights W^T [in][out]
+// in shared memory: thread per (four rows, CT outputs).  Per pair of K steps
+// one weight load of CT values per step and one 4-byte load per row (x[k],
+// x[k+1]) feed 8·CT fp32 fused multiply-adds of bf16 inputs: the same
+// products, each sum in K order, as the plain fp32 loop.  ReLU and bf16
+// rounding of hidden outputs; the output layer's values go to sc.
+template <int CT>
+__device__ __forceinline__ void seq_layer_bf16(const uint8_t* Wt, const uint8_t* xin, uint8_t* xout,
+                                               const float* __restrict__ bl, int N, int in, int out, int wmax,
+                                               bool last_layer, float* sc) {
+  const int n4 = (N + 3) >> 2, oc = out / CT;
+  for (int e = threadIdx.x; e < n4 * oc; e += kSeqThreads) {
+    const int o0 = CT * (e % oc), i0 = 4 * (e / oc);
+    const uint8_t* xr[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) xr[q] = xin + (size_t)min(i0 + q, N - 1) * wmax * 2;
+    float acc[4][CT];
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+#pragma unroll
+      for (int j = 0; j < CT; ++j) acc[q][j] = 0.0f;
+    const uint8_t* wp = Wt + (size_t)o0 * 2;
+    const size_t wrow = (size_t)out * 2;
+    uint32_t w0[CT / 2], w1[CT / 2];
+    int k = 0;
+    for (; k + 2 <= in; k += 2, wp += 2 * wrow) {
+#pragma unroll
+      for (int h = 0; h < CT / 2; ++h) {
+        w0[h] = reinterpret_cast<const uint32_t*>(wp)[h];
+        w1[h] = reinterpret_cast<const uint32_t*>(wp + wrow)[h];
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const uint32_t xv = *reinterpret_cast<const uint32_t*>(xr[q] + (size_t)k * 2);
+        const uint32_t x0 = __byte_perm(xv, 0u, 0x1010), x1 = __byte_perm(xv, 0u, 0x3232);
+#pragma unroll
+        for (int h = 0; h < CT / 2; ++h) sm100::fma2_bf16_f32(x0, w0[h], acc[q][2 * h], acc[q][2 * h + 1]);
+#pragma unroll
+        for (int h = 0; h < CT / 2; ++h) sm100::fma2_bf16_f32(x1, w1[h], acc[q][2 * h], acc[q][2 * h + 1]);
+      }
+    }
+    if (k < in) {  // an odd K: the last step alone
+#pragma unroll
+      for (int h = 0; h < CT / 2; ++h) w0[h] = reinterpret_cast<const uint32_t*>(wp)[h];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const uint32_t xs = reinterpret_cast<const uint16_t*>(xr[q])[k];
+        const uint32_t x0 = xs | (xs << 16);
+#pragma unroll
+        for (int h = 0; h < CT / 2; ++h) sm100::fma2_bf16_f32(x0, w0[h], acc[q][2 * h], acc[q][2 * h + 1]);
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < CT; ++j) {
+      const float bo = __ldg(bl + o0 + j);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        if (i0 + q >= N) break;
+        const float z = acc[q][j] + bo;
+        if (last_layer) sc[i0 + q] = z;
+        else seq_xset(xout, (int64_t)(i0 + q) * wmax + o0 + j, fmaxf(z, 0.0f), true);
+      }
+    }
+  }
 }
 
 __global__ void __launch_bounds__(kSeqThreads, 1) k_route_seq(const __grid_constant__ SeqArgs a, int64_t bcap) {
@@ -295,6 +362,10 @@ __global__ void __launch_bounds__(kSeqThreads, 1) k_route_seq(const __grid_const
             else seq_xset(xout, (int64_t)i * a.wmax + oo, fmaxf(z, 0.0f), bf);
           }
         }
+      } else if (a.wsm && bf && (out & 3) == 0 && (a.wmax & 1) == 0) {
+        // bf16: thread per (four rows, four outputs) (two outputs a thread,
+        // for more threads when the rows are few, measured no faster)
+        seq_layer_bf16<4>(Wsm + a.woff_s[l], xin, xout, bl, N, in, out, a.wmax, last_layer, sc);
       } else if (a.wsm) {
         // thread per (output, four rows): one weight and four broadcast
         // inputs per K step, fp32 sums, the bias added after the sum
