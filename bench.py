@@ -1126,6 +1126,9 @@ def measure_e2e(L, H, dev, stream, args, ctx, st, world):
     ems = max_over_ranks(world, e0.elapsed_time(e1) / K, None)
     return {"value": world * R / (ems / 1e3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
             "d2h_bytes_per_step": int(d2h), "ms_per_step": ems, "steps": K,
+            # the host link's rate over the step (one GPU's copies); a pinned
+            # host-to-device copy alone moves about 210 GB/s on a GB300 host
+            "h2d_GB_per_s": h2d / (ems / 1e3) / 1e9,
             "pipelined": f"inputs of step k+1 copied on a copy stream while step k computes; {NB} device input sets "
                          f"with a captured graph each; choices, best scores and loss read back every step"}
 
