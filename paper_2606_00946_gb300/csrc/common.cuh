@@ -235,12 +235,12 @@ struct Ctx {
   int32_t* rrank = nullptr;       // rank of each candidate [P], then of each kept record [Rc]
   int64_t* rcount = nullptr;      // candidates and kept records of the round in flight [2]
   uint8_t* rimg = nullptr;        // bf16 embedding image (128-row tiles, MMA layout) for bf16 predictors
-  int64_t ring_enqueued = 0;
+  int64_t ring_enqueued = 0;     // records appended (host order); the device count is st->ring_count
   // feature bounds of the ring (Algorithm 4 [l, u]): staged by ls_refresh_bounds,
   // published by ls_publish into pub[b].bounds
   float* bounds_stage = nullptr;  // lo [d], hi [d]
   uint32_t* benc = nullptr;       // bounds being reduced, order-preserving codes [2][d]
-  ls_guards guards{};     // records appended (host order); the device count is st->ring_count
+  ls_guards guards{};             // Algorithm 4 guard parameters of guarded routes
 
   // route scratch
   int32_t* hits = nullptr;    // [max_requests, max_instances]
